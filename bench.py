@@ -1,0 +1,348 @@
+"""Benchmark: FlashRelation forward + backward on one GB300 (replicas on N GPUs).
+
+One step = relation_fwd + relation_bwd over one batch of the workload (every step of
+the operator's hot path), inputs resident in HBM.  Timed with CUDA events on the
+launching stream, per step, with the L2 flushed (a 256 MiB write) between steps, after
+W warm-up steps.  Prints ONE JSON line (rank 0).
+
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--config 10M|30M|100M|long|tiny]
+                  [--impl ours|reference] [--no-cpu-baseline]
+
+--impl reference times the fp64 CPU oracle (the reference arm of this operator: there
+is no other implementation) on the host cores over a bounded sample of the workload.
+Under torchrun (N > 1) every rank runs an independent replica of the workload on its
+own GPU (the heads are independent; nothing is exchanged) and the slowest rank's time
+is reported.
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import os
+import statistics
+import subprocess
+import sys
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+import torch  # noqa: E402
+
+from paper_2608_20172_gb300 import workloads  # noqa: E402
+
+L2_FLUSH_BYTES = 256 << 20
+
+
+def _peaks():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    try:
+        with open(path) as f:
+            p = json.load(f)
+        return {"hbm_gbs": float(p["hbm_gbs"]), "bf16_tflops": float(p["bf16_tflops"]),
+                "bf16_tflops_sustained": float(p.get("bf16_tflops_sustained", p["bf16_tflops"])),
+                "source": "measured"}
+    except (OSError, KeyError, ValueError):
+        return {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0,
+                "source": "fallback"}
+
+
+class ClockSampler:
+    """nvidia-smi clock / throttle-reason sampling while the timed region runs."""
+
+    QUERY = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+             "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+             "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, index: int):
+        self.index = index
+        self.proc = None
+
+    def __enter__(self):
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", f"--id={self.index}", f"--query-gpu={self.QUERY}",
+                 "--format=csv,noheader,nounits", "-lms", "200"],
+                stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+        except OSError:
+            self.proc = None
+        return self
+
+    def __exit__(self, *exc):
+        self.lines = []
+        if self.proc is not None:
+            self.proc.terminate()
+            try:
+                out, _ = self.proc.communicate(timeout=5)
+            except subprocess.TimeoutExpired:
+                self.proc.kill()
+                out, _ = self.proc.communicate()
+            self.lines = [ln for ln in out.splitlines() if ln.strip()]
+        return False
+
+    def summary(self):
+        sm, mx, reasons = [], None, set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for ln in getattr(self, "lines", []):
+            f = [x.strip() for x in ln.split(",")]
+            if len(f) < 9:
+                continue
+            try:
+                sm.append(float(f[1]))
+                mx = float(f[2])
+            except ValueError:
+                continue
+            for n, val in zip(names, f[5:9]):
+                if val.lower().startswith("active"):
+                    reasons.add(n)
+        if not sm:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["unsampled"], "samples": 0}
+        return {"sm_mhz": statistics.median(sm), "sm_max_mhz": mx, "reasons": sorted(reasons),
+                "samples": len(sm)}
+
+
+def _dist():
+    ws = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    if ws > 1:
+        import torch.distributed as dist
+        dist.init_process_group("nccl" if torch.cuda.is_available() else "gloo")
+        return dist, ws, rank, local
+    return None, 1, 0, local
+
+
+def _barrier(dist, dev):
+    if dist is not None:
+        dist.barrier(device_ids=[dev.index] if dev.type == "cuda" else None)
+
+
+def _max_over_ranks(dist, x: float, dev) -> float:
+    if dist is None:
+        return x
+    t = torch.tensor([x], dtype=torch.float64, device=dev)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+# ------------------------------------------------------------------------------
+# CPU oracle (baseline leg and --impl reference)
+# ------------------------------------------------------------------------------
+
+def _oracle_sample(w, n_heads):
+    """Inputs of the first n_heads (b, h) heads, fp64, [B', T, H', d] blocks."""
+    q, k, v, do = workloads.make_inputs(w)
+    heads = [(b, h) for b in range(w.B) for h in range(w.H)][:n_heads]
+    bs = sorted({b for b, _ in heads})
+    hs = sorted({h for _, h in heads})
+    sl = (slice(bs[0], bs[-1] + 1), slice(None), slice(hs[0], hs[-1] + 1))
+    return [t[sl].double().numpy() for t in (q, k, v, do)], len(bs) * len(hs)
+
+
+def _sample_heads(w):
+    # ~10-30 s of oracle work on the host: scale the sample by the per-head cost.
+    per_head = w.T * w.T * w.d
+    budget = 16 * 1024 * 1024 * 64  # 16 heads of the 10M workload
+    n = max(1, min(w.B * w.H, budget // per_head))
+    return n if n < w.H else (n // w.H) * w.H
+
+
+def cpu_oracle_run(w, n_heads=None):
+    import oracle
+    n_heads = n_heads or _sample_heads(w)
+    (q, k, v, do), used = _oracle_sample(w, n_heads)
+    threads = oracle.max_threads()
+    t0 = time.perf_counter()
+    oracle.mhr_fwd(q, k, v, workloads.LAMBDA_INIT)
+    oracle.mhr_bwd(q, k, v, do, workloads.LAMBDA_INIT)
+    dt = time.perf_counter() - t0
+    flops = 7.0 * used * w.T * w.T * w.d
+    return {"seconds": dt, "heads": used, "flops": flops, "tflops": flops / dt / 1e12,
+            "tokens_per_s": (used / w.H) * w.T / dt, "cores": threads}
+
+
+def run_reference(args, w):
+    dist, ws, rank, local = _dist()
+    if rank != 0:
+        return 0
+    n = _sample_heads(w)
+    for _ in range(args.warmup):
+        cpu_oracle_run(w, n_heads=max(1, n // 4))
+    times, res = [], None
+    for _ in range(args.steps):
+        res = cpu_oracle_run(w, n_heads=max(1, n // 4))
+        times.append(res["seconds"])
+    tot_flops = res["flops"] * args.steps
+    val = tot_flops / sum(times) / 1e12
+    sample = f"{res['heads']} of {w.B * w.H} heads per step (fwd+bwd, fp64, OpenMP over heads)"
+    line = {
+        "impl": "reference", "metric": "FlashRelation fwd+bwd TFLOP/s (7*B*H*T^2*d causal)",
+        "value": val, "unit": "TFLOP/s", "n_gpus": 0, "steps": args.steps, "warmup": args.warmup,
+        "ms_per_step": 1e3 * statistics.mean(times), "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+        "config": {"workload": w.description, "B": w.B, "H": w.H, "T": w.T, "d_h": w.d,
+                   "lambda": workloads.LAMBDA_INIT, "tau_s": workloads.TAU_S},
+        "cpu_baseline": {"value": val, "unit": "TFLOP/s", "cores": res["cores"], "kind": "oracle",
+                         "sample": sample},
+        "e2e": {"value": val, "unit": "TFLOP/s", "h2d_bytes_per_step": 0,
+                "d2h_bytes_per_step": 0},
+    }
+    print(json.dumps(line), flush=True)
+    return 0
+
+
+# ------------------------------------------------------------------------------
+# GPU arm
+# ------------------------------------------------------------------------------
+
+def run_ours(args, w):
+    from paper_2608_20172_gb300 import binding
+    dist, ws, rank, local = _dist()
+    dev = torch.device("cuda", local)
+    torch.cuda.set_device(dev)
+    binding.load()
+    lam, tau = workloads.LAMBDA_INIT, workloads.TAU_S
+    q, k, v, do = workloads.make_inputs(w, seed=0)
+    qd, kd, vd, dod = (t.to(dev) for t in (q, k, v, do))
+    y = torch.empty_like(qd)
+    logz = torch.empty((w.B, w.H, w.T), device=dev, dtype=torch.float32)
+    dq, dk, dv = torch.empty_like(qd), torch.empty_like(qd), torch.empty_like(qd)
+    dl = torch.empty(1, device=dev, dtype=torch.float32)
+    wsb = torch.empty(binding.workspace_size(qd), device=dev, dtype=torch.uint8)
+    status = torch.zeros(1, dtype=torch.int32, device=dev)
+    flush = torch.empty(L2_FLUSH_BYTES, dtype=torch.uint8, device=dev)
+    stream = torch.cuda.current_stream(dev)
+    family = args.kernel
+
+    def step():
+        binding.fwd(qd, kd, vd, lam, tau, kernel=family, out=y, logz=logz, dev_status=status,
+                    stream=stream)
+        binding.bwd(qd, kd, vd, y, dod, logz, lam, tau, kernel=family, workspace=wsb, dq=dq, dk=dk,
+                    dv=dv, dlambda=dl, dev_status=status, stream=stream)
+
+    for _ in range(args.warmup):
+        step()
+        flush.zero_()
+    torch.cuda.synchronize(dev)
+    if int(status.item()) != 0:
+        raise SystemExit(f"device status {binding.status_string(int(status.item()))}")
+
+    n = args.steps
+    ev = [[torch.cuda.Event(enable_timing=True) for _ in range(3)] for _ in range(n)]
+    _barrier(dist, dev)
+    torch.cuda.synchronize(dev)
+    with ClockSampler(dev.index) as clk:
+        for i in range(n):
+            ev[i][0].record(stream)
+            binding.fwd(qd, kd, vd, lam, tau, kernel=family, out=y, logz=logz, dev_status=status,
+                        stream=stream)
+            ev[i][1].record(stream)
+            binding.bwd(qd, kd, vd, y, dod, logz, lam, tau, kernel=family, workspace=wsb, dq=dq,
+                        dk=dk, dv=dv, dlambda=dl, dev_status=status, stream=stream)
+            ev[i][2].record(stream)
+            flush.zero_()
+        torch.cuda.synchronize(dev)
+    _barrier(dist, dev)
+    t_fwd = [ev[i][0].elapsed_time(ev[i][1]) for i in range(n)]
+    t_bwd = [ev[i][1].elapsed_time(ev[i][2]) for i in range(n)]
+    t_step = [a + b for a, b in zip(t_fwd, t_bwd)]
+    ms = _max_over_ranks(dist, statistics.mean(t_step), dev)
+    ms_fwd = _max_over_ranks(dist, statistics.mean(t_fwd), dev)
+    ms_bwd = _max_over_ranks(dist, statistics.mean(t_bwd), dev)
+    st = int(status.item())
+    if st != 0:
+        raise SystemExit(f"device status {binding.status_string(st)}")
+
+    # end to end through the public API: pinned host inputs in, results out, every step
+    hq, hk, hv, hdo = (t.pin_memory() for t in (q, k, v, do))
+    hy, hdq, hdk, hdv = (torch.empty_like(t).pin_memory() for t in (q, q, q, q))
+    hdl = torch.empty(1, dtype=torch.float32).pin_memory()
+    e2e_ev = [[torch.cuda.Event(enable_timing=True) for _ in range(2)] for _ in range(n)]
+    for i in range(n + args.warmup):
+        rec = i >= args.warmup
+        if rec:
+            e2e_ev[i - args.warmup][0].record(stream)
+        for src, dst in ((hq, qd), (hk, kd), (hv, vd), (hdo, dod)):
+            dst.copy_(src, non_blocking=True)
+        step()
+        for src, dst in ((y, hy), (dq, hdq), (dk, hdk), (dv, hdv), (dl, hdl)):
+            dst.copy_(src, non_blocking=True)
+        if rec:
+            e2e_ev[i - args.warmup][1].record(stream)
+        flush.zero_()
+    torch.cuda.synchronize(dev)
+    ms_e2e = _max_over_ranks(dist, statistics.mean(e[0].elapsed_time(e[1]) for e in e2e_ev), dev)
+    h2d = sum(t.numel() * t.element_size() for t in (hq, hk, hv, hdo))
+    d2h = sum(t.numel() * t.element_size() for t in (hy, hdq, hdk, hdv, hdl))
+
+    flops = w.flops_fwd_bwd()
+    tflops = ws * flops / (ms * 1e-3) / 1e12
+    peaks = _peaks()
+    # roofline of the dominant launch group: the backward call
+    esz = 2 if w.dtype == "bf16" else 4
+    bwd_flops = 5.0 * w.B * w.H * w.T * w.T * w.d
+    bwd_bytes = 8.0 * w.B * w.T * w.H * w.d * esz + 8.0 * w.B * w.H * w.T
+    achieved_bwd = bwd_flops / (ms_bwd * 1e-3) / 1e12
+    clocks = clk.summary() if rank == 0 else {}
+    line = {
+        "metric": "FlashRelation fwd+bwd TFLOP/s (7*B*H*T^2*d causal)",
+        "value": tflops, "unit": "TFLOP/s", "n_gpus": ws, "steps": n, "warmup": args.warmup,
+        "ms_per_step": ms, "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
+        "dtype": "bf16" if w.dtype == "bf16" else "f32", "data": "synthetic",
+        "config": {"workload": w.description, "B": w.B, "H": w.H, "T": w.T, "d_h": w.d,
+                   "lambda": workloads.LAMBDA_INIT, "tau_s": workloads.TAU_S,
+                   "kernel": family, "l2": "flushed between steps (256 MiB write)",
+                   "inputs": "Q,K,V,dO iid normal, seed 0 (workload recipe)",
+                   "parallelism": f"replicas x{ws}"},
+        "tokens_per_s": ws * w.tokens / (ms * 1e-3),
+        "pct_bf16_peak": 100.0 * tflops / (ws * peaks["bf16_tflops"]),
+        "pct_bf16_peak_sustained": 100.0 * tflops / (ws * peaks["bf16_tflops_sustained"]),
+        "ms_fwd": ms_fwd, "ms_bwd": ms_bwd,
+        "fwd_tflops": ws * w.flops_fwd() / (ms_fwd * 1e-3) / 1e12,
+        "bwd_tflops": ws * bwd_flops / (ms_bwd * 1e-3) / 1e12,
+        "roofline": {"kernel": "relation_bwd (row pre-pass + Exchange tiles + dlambda reduce)",
+                     "bound": "tensor", "achieved": achieved_bwd,
+                     "peak": peaks["bf16_tflops"], "unit": "TFLOP/s",
+                     "frac": achieved_bwd / peaks["bf16_tflops"],
+                     "peak_source": peaks["source"] + " bf16 burst",
+                     "algorithmic_bytes": bwd_bytes,
+                     "achieved_gbs": bwd_bytes / (ms_bwd * 1e-3) / 1e9, "traffic": None},
+        "e2e": {"value": ws * flops / (ms_e2e * 1e-3) / 1e12, "unit": "TFLOP/s",
+                "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h, "ms_per_step": ms_e2e},
+        "gpu_launches": n * (binding.launches_per_call(family, w.dtype, w.d, "fwd")
+                             + binding.launches_per_call(family, w.dtype, w.d, "bwd")),
+        "clocks": clocks,
+    }
+    if rank == 0 and not args.no_cpu_baseline and ws == 1:
+        cb = cpu_oracle_run(w)
+        line["cpu_baseline"] = {
+            "value": cb["tflops"], "unit": "TFLOP/s", "cores": cb["cores"], "kind": "oracle",
+            "sample": f"{cb['heads']} of {w.B * w.H} heads, fwd+bwd, fp64 C oracle, "
+                      f"{cb['seconds']:.1f} s"}
+    if rank == 0:
+        print(json.dumps(line), flush=True)
+    if dist is not None:
+        dist.destroy_process_group()
+    return 0
+
+
+def main(argv=None):
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=20)
+    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--config", default="10M", choices=sorted(workloads.WORKLOADS))
+    ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
+    ap.add_argument("--kernel", default="auto", choices=["auto", "simt", "tcgen05"])
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    args = ap.parse_args(argv)
+    args.warmup = max(args.warmup, 3)  # at least 3 untimed warm-up steps
+    w = workloads.WORKLOADS[args.config]
+    if args.impl == "reference":
+        return run_reference(args, w)
+    return run_ours(args, w)
+
+
+if __name__ == "__main__":
+    sys.exit(main())

@@ -1,0 +1,153 @@
+/*
+ * relation.h -- C ABI of the GB300 (sm_103a) FlashRelation library.
+ *
+ * The library computes the exact causal Multi-Head Relation operator of
+ * "Ask Self, Ask Others: Relation Is All You Need" (arxiv 2608.20172), forward and
+ * backward, in tiled FlashRelation form: the T x T matrices U, R and F are never
+ * written to memory.
+ *
+ * Per head, with p1 = Q (P1 after RoPE), p2 = K (P2 after RoPE) and I~ = V (the
+ * information state after head mixing), rows i = 1..T (one-based):
+ *   U_ij = p1_i . p2_j / sqrt(d_h)                           Eq. (relation-projections)
+ *   S_i  = sigmoid(U_ii / tau_S),  E_ij = SiLU(U_ij)          Eq. (causal-relation)
+ *   R_ii = S_i,  R_ij = E_ij - lambda log i (j < i),  R_ij = -inf (j > i)
+ *   F_i  = Softmax(R_i),  Y_i = sum_{j<=i} F_ij I~_j          Eq. (relation-flow)
+ * evaluated through the exact factorisation (Sec. 4.2 and Sec. 5.1):
+ *   L^E_i = LSE_{j<i} E_ij (online scan), A_i = L^E_i - lambda log i,
+ *   g_i = sigmoid(A_i - S_i), Y_i = (1 - g_i) I~_i + g_i Ibar_i, Ibar_i = sum pi^E_ij I~_j.
+ * Row 1 has no history: g_1 = 0 and Y_1 = I~_1 (App. A.1.8).  Logarithms are natural.
+ * lambda is one fp32 scalar per layer, shared by all heads (App. A.1.1); tau_S > 0
+ * (the paper fixes tau_S = 2, Sec. 3.1) and carries no gradient.
+ *
+ * Conventions shared by every entry point
+ *  - Tensors Q, K, V, O, dO, dQ, dK, dV are [B][T][H][d_h] with d_h contiguous and the
+ *    element strides sB, sT, sH of relation_shape (so [B][H][T][d_h] works too).  All
+ *    eight tensors use the same strides and dtype.  logZ is a dense fp32 [B][H][T].
+ *  - Every pointer is a device pointer (cudaMalloc / cudaMallocAsync / managed).  The
+ *    caller owns every buffer, including the backward workspace; the library allocates
+ *    no memory and keeps no per-call state.
+ *  - Calls are asynchronous on `stream` (NULL = the legacy default stream).
+ *  - Argument errors are reported synchronously by the return value and nothing is
+ *    launched.  A kernel whose pipeline wait exceeds its bound writes
+ *    RELATION_ERR_TIMEOUT into *dev_status (a device int the caller zeroes and reads
+ *    after synchronising; may be NULL) and returns without finishing its tile.
+ *  - Supported: fp32 with d_h in {32, 64, 128}; bf16 with d_h in {32, 64, 128}
+ *    (d_h 64 and 128 run on the tcgen05 tensor-core kernels).  Any T >= 1.
+ *  - Alignment: every tensor pointer 16-byte aligned and sB, sT, sH multiples of
+ *    16 bytes / element size; workspace 256-byte aligned.
+ */
+#ifndef RELATION_H
+#define RELATION_H
+
+#include <stddef.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+/* Same type as cudaStream_t / CUstream. */
+typedef struct CUstream_st* relation_stream_t;
+
+typedef enum relation_status {
+  RELATION_OK = 0,
+  RELATION_ERR_INVALID_ARG = 1, /* null pointer, bad size, non-finite lambda or tau_S   */
+  RELATION_ERR_UNSUPPORTED = 2, /* d_h / dtype combination not built                     */
+  RELATION_ERR_ALIGNMENT = 3,   /* pointer or stride alignment rule broken               */
+  RELATION_ERR_WORKSPACE = 4,   /* workspace missing or smaller than the size query      */
+  RELATION_ERR_CUDA = 5,        /* a CUDA runtime call failed (launch, attribute, ...)   */
+  RELATION_ERR_TIMEOUT = 6      /* written to *dev_status by a kernel whose wait expired */
+} relation_status;
+
+typedef enum relation_dtype { RELATION_F32 = 0, RELATION_BF16 = 1 } relation_dtype;
+
+typedef struct relation_shape {
+  int B;        /* batch                                          */
+  int T;        /* sequence length, >= 1                          */
+  int H;        /* heads (MHR, Sec. 3.2)                           */
+  int d_h;      /* head width                                     */
+  long long sB; /* element stride between batches                 */
+  long long sT; /* element stride between tokens                  */
+  long long sH; /* element stride between heads; d_h is contiguous */
+} relation_shape;
+
+/*
+ * Forward (Eqs. causal-relation, relation-flow; Sec. 5.1 and App. A.3).
+ *   q, k, v : inputs P1, P2 (after RoPE) and I~ (after Givens mixing), dtype dt.
+ *   o       : output Y, dtype dt, same layout.
+ *   logz    : output fp32 [B][H][T], logZ_i = log sum_j exp(R_ij) = logaddexp(S_i, A_i)
+ *             (logZ_1 = S_1).  This is the per-row statistic relation_bwd consumes.
+ *   lambda  : count-calibration scalar lambda_l; tau_s: Self temperature (> 0).
+ */
+relation_status relation_fwd(const void* q, const void* k, const void* v, void* o, float* logz,
+                             float lambda, float tau_s, relation_shape shp, relation_dtype dt,
+                             int* dev_status, relation_stream_t stream);
+
+/* Kernel family selection for the *_ex entry points.  AUTO takes the tcgen05
+ * tensor-core kernels where they exist (bf16, d_h 64 or 128) and the CUDA-core (SIMT)
+ * kernels otherwise; TCGEN05 returns RELATION_ERR_UNSUPPORTED where they do not exist. */
+typedef enum relation_kernel {
+  RELATION_KERNEL_AUTO = 0,
+  RELATION_KERNEL_SIMT = 1,
+  RELATION_KERNEL_TCGEN05 = 2
+} relation_kernel;
+
+/* relation_fwd with an explicit kernel family (relation_fwd == relation_fwd_ex(..., AUTO)). */
+relation_status relation_fwd_ex(const void* q, const void* k, const void* v, void* o, float* logz,
+                                float lambda, float tau_s, relation_shape shp, relation_dtype dt,
+                                relation_kernel kernel, int* dev_status, relation_stream_t stream);
+
+/* Bytes of device workspace relation_bwd needs for this shape and dtype (0 on a bad
+ * shape).  The content of the workspace need not be initialised. */
+size_t relation_bwd_workspace_size(relation_shape shp, relation_dtype dt);
+
+/*
+ * Backward (App. A.1.7), recomputing the tiles from logz.
+ *   q, k, v, o, dout, logz : the forward's inputs, its output Y, dL/dY and its logz.
+ *   dq, dk, dv             : outputs dL/dP1, dL/dP2, dL/dI~ (overwritten, not accumulated).
+ *   dlambda                : output, one device float, dL/dlambda summed over B, H and T
+ *                            (lambda is shared by the heads).  Overwritten.
+ *   workspace, ws_bytes    : device scratch of at least relation_bwd_workspace_size().
+ * The gradient follows the generic softmax form dR_ij = F_ij (H_ij - D_i) with
+ * H_ij = dO_i . I~_j and D_i = dO_i . Y_i, chained through sigma' (Self, with 1/tau_S)
+ * and SiLU' (Exchange).  dlambda = -sum_i log i sum_{j<i} dR_ij = sum_i log i dR_ii,
+ * because every row of dR sums to zero.
+ */
+relation_status relation_bwd(const void* q, const void* k, const void* v, const void* o,
+                             const void* dout, const float* logz, void* dq, void* dk, void* dv,
+                             float* dlambda, float lambda, float tau_s, relation_shape shp,
+                             relation_dtype dt, void* workspace, size_t ws_bytes,
+                             int* dev_status, relation_stream_t stream);
+
+/* relation_bwd with an explicit kernel family (relation_bwd == relation_bwd_ex(..., AUTO)). */
+relation_status relation_bwd_ex(const void* q, const void* k, const void* v, const void* o,
+                                const void* dout, const float* logz, void* dq, void* dk, void* dv,
+                                float* dlambda, float lambda, float tau_s, relation_shape shp,
+                                relation_dtype dt, void* workspace, size_t ws_bytes,
+                                relation_kernel kernel, int* dev_status, relation_stream_t stream);
+
+/* Number of kernel launches one relation_fwd_ex (backward = 0) or relation_bwd_ex
+ * (backward != 0) call makes for this dtype, head width and kernel request; 0 when the
+ * request is not supported.  Host-only query. */
+int relation_launch_count(relation_dtype dt, int d_h, relation_kernel kernel, int backward);
+
+/* Human-readable name of a status code (static string, never NULL). */
+const char* relation_status_string(relation_status s);
+
+/* Library ABI version, (major << 16) | minor. */
+int relation_version(void);
+
+/*
+ * Self-test of the bounded pipeline wait used by every tensor-core kernel: launches
+ * one tiny kernel that waits on an mbarrier nothing will ever complete, with a bound of
+ * about `timeout_us` microseconds (1..100000).  On expiry the kernel writes
+ * RELATION_ERR_TIMEOUT into *dev_status and returns; the context stays usable.
+ * The paper has no counterpart: this exists to test failure detection.
+ */
+relation_status relation_selftest_wait_timeout(int* dev_status, int timeout_us,
+                                               relation_stream_t stream);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* RELATION_H */

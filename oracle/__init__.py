@@ -94,6 +94,7 @@ class Oracle:
                                           _dp, _dp, _dp],
             "rel_oracle_fwd_scan": [i, i, _dp, _dp, _dp, d, d, i, i, _dp, _dp],
             "rel_oracle_bwd": [i, i, _dp, _dp, _dp, _dp, d, d, _dp, _dp, _dp, _dp],
+            "rel_oracle_bwd_tail": [i, i, _dp, _dp, _dp, _dp, d, d, i, _dp, _dp, _dp, _dp],
             "rel_oracle_bwd_credit": [i, i, _dp, _dp, _dp, _dp, d, d, _dp, _dp, _dp, _dp],
             "rel_oracle_mhr_fwd": [i, i, i, i, ll, ll, ll, _dp, _dp, _dp, d, d, _dp, _dp, i],
             "rel_oracle_mhr_bwd": [i, i, i, i, ll, ll, ll, _dp, _dp, _dp, _dp, d, d, _dp, _dp,
@@ -161,6 +162,19 @@ class Oracle:
                                        _p(dk), _p(dv), _p(dl)), "bwd")
         return dq, dk, dv, float(dl[0])
 
+    def bwd_tail(self, q, k, v, dy, lam: float, row_begin: int, tau_s: float = TAU_S):
+        """Backward of one head restricted to rows r >= row_begin: exact dq rows
+        >= row_begin and dk, dv rows >= row_begin (dq rows below are 0; dlambda sums
+        the processed rows).  Returns (dq, dk, dv, dlambda)."""
+        q, k, v, T, d = _head_args(q, k, v)
+        dy = _in(dy)
+        dq = np.empty((T, d)); dk = np.empty((T, d)); dv = np.empty((T, d))
+        dl = np.empty(1)
+        _check(self.lib.rel_oracle_bwd_tail(T, d, _p(q), _p(k), _p(v), _p(dy), lam, tau_s,
+                                            int(row_begin), _p(dq), _p(dk), _p(dv), _p(dl)),
+               "bwd_tail")
+        return dq, dk, dv, float(dl[0])
+
     def bwd_credit(self, q, k, v, dy, lam: float, tau_s: float = TAU_S):
         """Backward of one head via the Self-Exchange credit decomposition.
         Returns (dq, dk, dv, dlambda)."""
@@ -223,6 +237,10 @@ def fwd_scan(*a, **kw):
 
 def bwd(*a, **kw):
     return default().bwd(*a, **kw)
+
+
+def bwd_tail(*a, **kw):
+    return default().bwd_tail(*a, **kw)
 
 
 def bwd_credit(*a, **kw):

@@ -134,14 +134,16 @@ int rel_oracle_fwd_rows(int T, int d, const double* q, const double* k, const do
     double* U = (double*)malloc(sizeof(double) * (size_t)T);
     double* Rr = (double*)malloc(sizeof(double) * (size_t)T);
     double* Fr = (double*)malloc(sizeof(double) * (size_t)T);
-    if (!U || !Rr || !Fr) {
+    const int ok = U && Rr && Fr;
+    if (!ok) {
 #pragma omp atomic write
       fail = 1;
-    } else {
-#pragma omp for schedule(dynamic, 1)
-      for (int n = 0; n < nrows; ++n)
-        relation_row(rows[n], T, d, q, k, v, lambda, tau_s, U, Rr, Fr, y + (size_t)n * d, logz + n);
     }
+#pragma omp for schedule(dynamic, 1)
+    for (int n = 0; n < nrows; ++n)
+      if (ok)
+        relation_row(rows[n], T, d, q, k, v, lambda, tau_s, U, Rr, Fr, y + (size_t)n * d,
+                     logz + n);
     free(U); free(Rr); free(Fr);
   }
   return fail ? -1 : 0;
@@ -282,10 +284,16 @@ int rel_oracle_fwd_scan(int T, int d, const double* q, const double* k, const do
 /* time with the full materialised row R_i, F_i of relation_row().           */
 /* dq, dk, dv: [T][d]; dlambda: scalar.  Any of the four may be NULL.        */
 /* ------------------------------------------------------------------------ */
-int rel_oracle_bwd(int T, int d, const double* q, const double* k, const double* v,
-                   const double* dy, double lambda, double tau_s, double* dq, double* dk,
-                   double* dv, double* dlambda) {
-  if (bad_args(T, d, q, k, v) || !dy || !(tau_s > 0.0)) return -1;
+/* rel_oracle_bwd_tail: the same computation restricted to the rows r >= row_begin.
+ * Rows are independent in this form, so the outputs are exact for dq rows
+ * r >= row_begin and for dk, dv rows j >= row_begin (only rows i >= j feed key j);
+ * dq rows below row_begin are set to 0, and dlambda sums the processed rows only.
+ * rel_oracle_bwd is the case row_begin = 0. */
+int rel_oracle_bwd_tail(int T, int d, const double* q, const double* k, const double* v,
+                        const double* dy, double lambda, double tau_s, int row_begin,
+                        double* dq, double* dk, double* dv, double* dlambda) {
+  if (bad_args(T, d, q, k, v) || !dy || !(tau_s > 0.0) || row_begin < 0 || row_begin >= T)
+    return -1;
   const double inv_sqrt_d = 1.0 / sqrt((double)d);
   double* U = (double*)malloc(sizeof(double) * (size_t)T);
   double* Rr = (double*)malloc(sizeof(double) * (size_t)T);
@@ -299,7 +307,9 @@ int rel_oracle_bwd(int T, int d, const double* q, const double* k, const double*
     return -1;
   }
   double dlam = 0.0;
-  for (int r = 0; r < T; ++r) {
+  if (dq)
+    for (size_t n = 0; n < (size_t)row_begin * d; ++n) dq[n] = 0.0;
+  for (int r = row_begin; r < T; ++r) {
     double lz;
     relation_row(r, T, d, q, k, v, lambda, tau_s, U, Rr, Fr, yr, &lz);
     const double* G = dy + (size_t)r * d;
@@ -333,6 +343,12 @@ int rel_oracle_bwd(int T, int d, const double* q, const double* k, const double*
   if (dlambda) *dlambda = dlam;
   free(U); free(Rr); free(Fr); free(Hr); free(yr); free(gk); free(gv);
   return 0;
+}
+
+int rel_oracle_bwd(int T, int d, const double* q, const double* k, const double* v,
+                   const double* dy, double lambda, double tau_s, double* dq, double* dk,
+                   double* dv, double* dlambda) {
+  return rel_oracle_bwd_tail(T, d, q, k, v, dy, lambda, tau_s, 0, dq, dk, dv, dlambda);
 }
 
 /* ------------------------------------------------------------------------ */

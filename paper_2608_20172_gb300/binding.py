@@ -1,0 +1,203 @@
+"""Thin ctypes binding of librelation (include/relation.h) for torch CUDA tensors.
+
+Argument marshalling only: every step of the operator runs in the library's CUDA
+kernels.  Tensors are [B, T, H, d_h] (any strides with d_h contiguous, the same for
+all tensors of a call); logZ is a dense fp32 [B, H, T].  Calls are enqueued on the
+current torch CUDA stream unless ``stream`` is given.
+
+Loading fails loudly (``RelationLibraryMissing``) when the compiled library is absent:
+there is no CPU fallback.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+import threading
+
+import torch
+
+_HERE = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = os.path.join(_HERE, "_build", "librelation.so")
+
+# relation_status
+OK, ERR_INVALID_ARG, ERR_UNSUPPORTED, ERR_ALIGNMENT, ERR_WORKSPACE, ERR_CUDA, ERR_TIMEOUT = range(7)
+# relation_dtype
+F32, BF16 = 0, 1
+# relation_kernel
+KERNELS = {"auto": 0, "simt": 1, "tcgen05": 2}
+
+EXPORTED = ("relation_fwd", "relation_fwd_ex", "relation_bwd", "relation_bwd_ex",
+            "relation_bwd_workspace_size", "relation_status_string", "relation_version",
+            "relation_selftest_wait_timeout", "relation_launch_count")
+
+
+class RelationLibraryMissing(RuntimeError):
+    pass
+
+
+class RelationError(RuntimeError):
+    def __init__(self, code: int, where: str):
+        super().__init__(f"{where}: {status_string(code)} ({code})")
+        self.code = code
+
+
+class Shape(ctypes.Structure):
+    _fields_ = [("B", ctypes.c_int), ("T", ctypes.c_int), ("H", ctypes.c_int),
+                ("d_h", ctypes.c_int), ("sB", ctypes.c_longlong), ("sT", ctypes.c_longlong),
+                ("sH", ctypes.c_longlong)]
+
+
+_lock = threading.Lock()
+_lib = None
+
+
+def load(path: str | None = None):
+    """Load librelation.so (default: the in-tree build) and declare its signatures."""
+    global _lib
+    with _lock:
+        if _lib is not None and path is None:
+            return _lib
+        p = path or LIB_PATH
+        if not os.path.exists(p):
+            raise RelationLibraryMissing(
+                f"{p} not found: build it with paper_2608_20172_gb300.build.build()")
+        lib = ctypes.CDLL(p)
+        vp, ip = ctypes.c_void_p, ctypes.c_void_p
+        f, i, sz = ctypes.c_float, ctypes.c_int, ctypes.c_size_t
+        lib.relation_fwd.argtypes = [vp, vp, vp, vp, vp, f, f, Shape, i, ip, vp]
+        lib.relation_fwd_ex.argtypes = [vp, vp, vp, vp, vp, f, f, Shape, i, i, ip, vp]
+        lib.relation_bwd.argtypes = [vp, vp, vp, vp, vp, vp, vp, vp, vp, vp, f, f, Shape, i, vp,
+                                     sz, ip, vp]
+        lib.relation_bwd_ex.argtypes = [vp, vp, vp, vp, vp, vp, vp, vp, vp, vp, f, f, Shape, i,
+                                        vp, sz, i, ip, vp]
+        lib.relation_bwd_workspace_size.argtypes = [Shape, i]
+        lib.relation_bwd_workspace_size.restype = sz
+        lib.relation_status_string.argtypes = [i]
+        lib.relation_status_string.restype = ctypes.c_char_p
+        lib.relation_version.argtypes = []
+        lib.relation_selftest_wait_timeout.argtypes = [ip, i, vp]
+        lib.relation_launch_count.argtypes = [i, i, i, i]
+        for n in ("relation_fwd", "relation_fwd_ex", "relation_bwd", "relation_bwd_ex",
+                  "relation_version", "relation_selftest_wait_timeout", "relation_launch_count"):
+            getattr(lib, n).restype = ctypes.c_int
+        if path is None:
+            _lib = lib
+        return lib
+
+
+def status_string(code: int) -> str:
+    return load().relation_status_string(int(code)).decode()
+
+
+def _dtype_code(t: torch.Tensor) -> int:
+    if t.dtype == torch.float32:
+        return F32
+    if t.dtype == torch.bfloat16:
+        return BF16
+    raise TypeError(f"unsupported dtype {t.dtype}")
+
+
+def shape_of(t: torch.Tensor) -> Shape:
+    """relation_shape of a [B, T, H, d_h] tensor with d_h contiguous."""
+    if t.dim() != 4:
+        raise ValueError("expected a [B, T, H, d_h] tensor")
+    if t.stride(3) != 1:
+        raise ValueError("d_h must be contiguous")
+    B, T, H, d = t.shape
+    return Shape(B, T, H, d, t.stride(0), t.stride(1), t.stride(2))
+
+
+def _same_layout(ref: torch.Tensor, *others: torch.Tensor):
+    for o in others:
+        if o.shape != ref.shape or o.stride() != ref.stride() or o.dtype != ref.dtype:
+            raise ValueError("all tensors of a call need the same shape, strides and dtype")
+        if not o.is_cuda or o.device != ref.device:
+            raise ValueError("all tensors must live on the same CUDA device")
+
+
+def _stream(stream) -> int:
+    if stream is None:
+        return torch.cuda.current_stream().cuda_stream
+    return stream.cuda_stream if hasattr(stream, "cuda_stream") else int(stream)
+
+
+def _ptr(t):
+    return None if t is None else ctypes.c_void_p(t.data_ptr())
+
+
+def workspace_size(q: torch.Tensor) -> int:
+    return int(load().relation_bwd_workspace_size(shape_of(q), _dtype_code(q)))
+
+
+def fwd(q, k, v, lam: float, tau_s: float = 2.0, *, kernel: str = "auto", out=None, logz=None,
+        dev_status=None, stream=None):
+    """Forward.  Returns (Y, logZ)."""
+    _same_layout(q, k, v)
+    B, T, H, _ = q.shape
+    if out is None:
+        out = torch.empty_like(q)
+    _same_layout(q, out)
+    if logz is None:
+        logz = torch.empty((B, H, T), device=q.device, dtype=torch.float32)
+    rc = load().relation_fwd_ex(_ptr(q), _ptr(k), _ptr(v), _ptr(out), _ptr(logz), float(lam),
+                                float(tau_s), shape_of(q), _dtype_code(q), KERNELS[kernel],
+                                _ptr(dev_status), ctypes.c_void_p(_stream(stream)))
+    if rc != OK:
+        raise RelationError(rc, "relation_fwd")
+    return out, logz
+
+
+def bwd(q, k, v, o, dout, logz, lam: float, tau_s: float = 2.0, *, kernel: str = "auto",
+        workspace=None, dq=None, dk=None, dv=None, dlambda=None, dev_status=None, stream=None):
+    """Backward.  Returns (dQ, dK, dV, dlambda) with dlambda a 1-element fp32 device tensor."""
+    _same_layout(q, k, v, o, dout)
+    dq = torch.empty_like(q) if dq is None else dq
+    dk = torch.empty_like(q) if dk is None else dk
+    dv = torch.empty_like(q) if dv is None else dv
+    _same_layout(q, dq, dk, dv)
+    if dlambda is None:
+        dlambda = torch.empty(1, device=q.device, dtype=torch.float32)
+    need = workspace_size(q)
+    if workspace is None:
+        workspace = torch.empty(need, device=q.device, dtype=torch.uint8)
+    rc = load().relation_bwd_ex(_ptr(q), _ptr(k), _ptr(v), _ptr(o), _ptr(dout), _ptr(logz),
+                                _ptr(dq), _ptr(dk), _ptr(dv), _ptr(dlambda), float(lam),
+                                float(tau_s), shape_of(q), _dtype_code(q),
+                                _ptr(workspace), workspace.numel() * workspace.element_size(),
+                                KERNELS[kernel], _ptr(dev_status),
+                                ctypes.c_void_p(_stream(stream)))
+    if rc != OK:
+        raise RelationError(rc, "relation_bwd")
+    return dq, dk, dv, dlambda
+
+
+def launches_per_call(kernel: str, dtype: str, d: int, which: str) -> int:
+    """Kernel launches one fwd / bwd call makes (0 when unsupported)."""
+    dt = F32 if dtype in ("fp32", "f32", torch.float32) else BF16
+    return int(load().relation_launch_count(dt, int(d), KERNELS[kernel], int(which == "bwd")))
+
+
+def selftest_wait_timeout(dev_status: torch.Tensor, timeout_us: int = 1000, stream=None) -> int:
+    """Launch the bounded-wait self-test; returns the launch status."""
+    return int(load().relation_selftest_wait_timeout(_ptr(dev_status), int(timeout_us),
+                                                     ctypes.c_void_p(_stream(stream))))
+
+
+class RelationFunction(torch.autograd.Function):
+    """Autograd wrapper: Y = Relation(q, k, v; lambda).  lambda is a 1-element tensor
+    (its gradient is returned); tau_S is a constant."""
+
+    @staticmethod
+    def forward(ctx, q, k, v, lam, tau_s=2.0, kernel="auto"):
+        y, logz = fwd(q, k, v, float(lam), tau_s, kernel=kernel)
+        ctx.save_for_backward(q, k, v, y, logz)
+        ctx.lam, ctx.tau_s, ctx.kernel = float(lam), tau_s, kernel
+        return y
+
+    @staticmethod
+    def backward(ctx, dy):
+        q, k, v, y, logz = ctx.saved_tensors
+        if dy.stride() != q.stride() or dy.dtype != q.dtype:
+            dy = torch.empty_like(q).copy_(dy)
+        dq, dk, dv, dl = bwd(q, k, v, y, dy, logz, ctx.lam, ctx.tau_s, kernel=ctx.kernel)
+        return dq, dk, dv, dl.reshape(()).to(torch.float32), None, None

@@ -1,0 +1,156 @@
+// aux_kernels.cu -- per-row and reduction kernels shared by both backward paths, and
+// the bounded-wait self-test.
+//
+// Backward Self part (App. A.1.7), one warp per row i of one head:
+//   D_i   = dO_i . Y_i                       (sum_k F_ik H_ik, since Y_i = sum_k F_ik v_k)
+//   S_i   = sigmoid(u_ii / tau_S),  u_ii = q_i . k_i / sqrt(d)
+//   F_ii  = exp(S_i - logZ_i)
+//   dR_ii = F_ii (dO_i . v_i - D_i)
+//   dS_ii = dR_ii S_i (1 - S_i) / tau_S      (dL/du_ii)
+// and the row's share of dL/dlambda.  dL/dlambda = -sum_i log i sum_{j<i} dR_ij; each
+// row of dR sums to zero (sum_k F_ik (H_ik - D_i) = D_i - D_i), so the inner sum is
+// -dR_ii and dL/dlambda = sum_i log i dR_ii: the diagonal alone carries it.
+#include <math.h>
+
+#include "common.cuh"
+#include "kernels.h"
+
+namespace rel {
+
+size_t bwd_workspace_bytes(int B, int H, int T, int d) {
+  auto up = [](size_t x) { return (x + 255) & ~(size_t)255; };
+  const size_t rows = (size_t)B * H * T;
+  const size_t n_pre = (rows + 7) / 8;
+  return up(rows * d * sizeof(float)) + 3 * up(rows * sizeof(float)) + up(n_pre * sizeof(float));
+}
+
+BwdWorkspace carve_workspace(void* base, int B, int H, int T, int d) {
+  auto up = [](size_t x) { return (x + 255) & ~(size_t)255; };
+  const size_t rows = (size_t)B * H * T;
+  char* p = static_cast<char*>(base);
+  BwdWorkspace w;
+  w.dq_acc = reinterpret_cast<float*>(p); p += up(rows * d * sizeof(float));
+  w.D = reinterpret_cast<float*>(p); p += up(rows * sizeof(float));
+  w.F_self = reinterpret_cast<float*>(p); p += up(rows * sizeof(float));
+  w.dS_self = reinterpret_cast<float*>(p); p += up(rows * sizeof(float));
+  w.dlam_part = reinterpret_cast<float*>(p);
+  w.n_pre_blocks = (int)((rows + 7) / 8);
+  return w;
+}
+
+namespace bwd_common {
+
+constexpr int kWarps = 8;
+
+template <typename TI>
+__device__ __forceinline__ float ld(const TI* p);
+template <>
+__device__ __forceinline__ float ld<float>(const float* p) { return *p; }
+template <>
+__device__ __forceinline__ float ld<__nv_bfloat16>(const __nv_bfloat16* p) {
+  return __bfloat162float(*p);
+}
+
+template <typename TI>
+__global__ void __launch_bounds__(kWarps * 32) pre_kernel(Problem p, BwdWorkspace ws) {
+  __shared__ float part[kWarps];
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const long long gr = (long long)blockIdx.x * kWarps + warp;
+  const long long nrows = (long long)p.B * p.H * p.T;
+  float contrib = 0.f;
+  if (gr < nrows) {
+    const int bh = (int)(gr / p.T), r = (int)(gr % p.T);
+    const int b = bh / p.H, h = bh % p.H;
+    const long long off = (long long)b * p.sB + (long long)h * p.sH + (long long)r * p.sT;
+    const TI* q = reinterpret_cast<const TI*>(p.q) + off;
+    const TI* k = reinterpret_cast<const TI*>(p.k) + off;
+    const TI* v = reinterpret_cast<const TI*>(p.v) + off;
+    const TI* o = reinterpret_cast<const TI*>(p.o) + off;
+    const TI* g = reinterpret_cast<const TI*>(p.dout) + off;
+    float gy = 0.f, gv = 0.f, qk = 0.f;
+    for (int c = lane; c < p.d; c += 32) {
+      const float gc = ld<TI>(g + c);
+      gy = fmaf(gc, ld<TI>(o + c), gy);
+      gv = fmaf(gc, ld<TI>(v + c), gv);
+      qk = fmaf(ld<TI>(q + c), ld<TI>(k + c), qk);
+    }
+#pragma unroll
+    for (int s = 16; s > 0; s >>= 1) {
+      gy += __shfl_xor_sync(0xffffffffu, gy, s);
+      gv += __shfl_xor_sync(0xffffffffu, gv, s);
+      qk += __shfl_xor_sync(0xffffffffu, qk, s);
+    }
+    const float u = qk * p.inv_sqrt_d;
+    const float S = 1.0f / (1.0f + expf(-u / p.tau_s));
+    const float F = expf(S - p.logz_in[gr]);
+    const float dR = F * (gv - gy);
+    if (lane == 0) {
+      ws.D[gr] = gy;
+      ws.F_self[gr] = F;
+      ws.dS_self[gr] = dR * S * (1.0f - S) / p.tau_s;
+    }
+    contrib = logf((float)(r + 1)) * dR;
+  }
+  if (lane == 0) part[warp] = contrib;
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    float s = 0.f;
+#pragma unroll
+    for (int w = 0; w < kWarps; ++w) s += part[w];
+    ws.dlam_part[blockIdx.x] = s;
+  }
+}
+
+// One block, fixed summation order (deterministic), fp64 accumulation.
+__global__ void __launch_bounds__(1024) dlambda_kernel(BwdWorkspace ws, float* out) {
+  __shared__ double red[1024];
+  double s = 0.0;
+  for (int i = threadIdx.x; i < ws.n_pre_blocks; i += 1024) s += (double)ws.dlam_part[i];
+  red[threadIdx.x] = s;
+  __syncthreads();
+  for (int w = 512; w > 0; w >>= 1) {
+    if (threadIdx.x < w) red[threadIdx.x] += red[threadIdx.x + w];
+    __syncthreads();
+  }
+  if (threadIdx.x == 0) *out = (float)red[0];
+}
+
+cudaError_t launch_pre(const Problem& p, const BwdWorkspace& ws, cudaStream_t s) {
+  dim3 grid(ws.n_pre_blocks);
+  if (p.dtype == RELATION_F32)
+    pre_kernel<float><<<grid, kWarps * 32, 0, s>>>(p, ws);
+  else
+    pre_kernel<__nv_bfloat16><<<grid, kWarps * 32, 0, s>>>(p, ws);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_dlambda(const Problem& p, const BwdWorkspace& ws, cudaStream_t s) {
+  dlambda_kernel<<<1, 1024, 0, s>>>(ws, p.dlambda);
+  return cudaGetLastError();
+}
+
+}  // namespace bwd_common
+
+// ---------------------------------------------------------------------------
+// Bounded-wait self-test: thread 0 initialises an mbarrier expecting one arrival
+// that never comes and waits on it with the same bounded wait the pipelines use.
+// The wait expires after timeout_us, writes RELATION_ERR_TIMEOUT and returns.
+// ---------------------------------------------------------------------------
+__global__ void selftest_wait_kernel(int* dev_status, unsigned long long timeout_ns) {
+  __shared__ __align__(8) unsigned long long bar;
+  __shared__ int abort_flag;
+  if (threadIdx.x != 0) return;
+  abort_flag = 0;
+  const uint32_t b = smem_u32(&bar);
+  mbar_init(b, 1);
+  fence_mbar_init();
+  Abort ab{&abort_flag, dev_status};
+  mbar_wait(b, 0, ab, timeout_ns);
+}
+
+cudaError_t launch_selftest_wait(int* dev_status, int timeout_us, cudaStream_t s) {
+  selftest_wait_kernel<<<1, 32, 0, s>>>(dev_status, (unsigned long long)timeout_us * 1000ull);
+  return cudaGetLastError();
+}
+
+}  // namespace rel

@@ -1,0 +1,71 @@
+// kernels.h -- internal launch interface between the C ABI layer and the kernels.
+#pragma once
+
+#include <cuda_runtime.h>
+#include <stddef.h>
+
+#include "relation.h"
+
+namespace rel {
+
+// Everything a kernel launch needs; pointers are device pointers.
+struct Problem {
+  // tensors ([B][T][H][d] with element strides sB, sT, sH)
+  const void* q;
+  const void* k;
+  const void* v;
+  const void* o;     // forward output (read by the backward)
+  const void* dout;  // dL/dY
+  void* out;         // forward: Y
+  void* dq;
+  void* dk;
+  void* dv;
+  float* logz;         // forward output [B][H][T]
+  const float* logz_in;  // backward input [B][H][T]
+  float* dlambda;      // backward output (one float)
+  int* dev_status;
+  // scalars
+  float lambda;
+  float tau_s;
+  float inv_sqrt_d;
+  int B, T, H, d;
+  long long sB, sT, sH;
+  relation_dtype dtype;
+};
+
+// Backward workspace carved out of the caller's buffer (all fp32, 256-byte aligned).
+struct BwdWorkspace {
+  float* dq_acc;     // [B][H][T][d]  Exchange part of dL/dP1 before scaling (tensor-core path)
+  float* D;          // [B][H][T]     D_i = dO_i . Y_i
+  float* F_self;     // [B][H][T]     F_ii = exp(S_i - logZ_i)
+  float* dS_self;    // [B][H][T]     dL/du_ii, u = U_ii (scaled evidence)
+  float* dlam_part;  // [n_pre_blocks] per-block partial sums of log(i) dR_ii
+  int n_pre_blocks;
+};
+
+size_t bwd_workspace_bytes(int B, int H, int T, int d);
+BwdWorkspace carve_workspace(void* base, int B, int H, int T, int d);
+
+namespace simt {
+bool supports(relation_dtype dt, int d);
+cudaError_t launch_fwd(const Problem& p, cudaStream_t s);
+cudaError_t launch_bwd(const Problem& p, const BwdWorkspace& ws, cudaStream_t s);
+}  // namespace simt
+
+namespace bwd_common {
+// Per-row Self part of the backward (D_i, F_ii, dS_ii and dlambda partials).
+cudaError_t launch_pre(const Problem& p, const BwdWorkspace& ws, cudaStream_t s);
+// Deterministic dlambda reduction of the per-block partials.
+cudaError_t launch_dlambda(const Problem& p, const BwdWorkspace& ws, cudaStream_t s);
+}  // namespace bwd_common
+
+namespace tc {
+bool supports(relation_dtype dt, int d);
+cudaError_t launch_fwd(const Problem& p, cudaStream_t s);
+cudaError_t launch_bwd(const Problem& p, const BwdWorkspace& ws, cudaStream_t s);
+int bwd_launches();  // launches made by launch_bwd
+}  // namespace tc
+
+cudaError_t launch_selftest_wait(int* dev_status, int timeout_us, cudaStream_t s);
+
+}  // namespace rel

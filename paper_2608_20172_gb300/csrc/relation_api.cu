@@ -1,0 +1,175 @@
+// relation_api.cu -- the C ABI of librelation (declared in include/relation.h).
+//
+// Host code only: argument validation (nothing is launched on an error), selection of
+// the kernel family, workspace carving and launches on the caller's stream.  The
+// library allocates no device memory.
+#include <math.h>
+#include <stdint.h>
+
+#include "kernels.h"
+#include "relation.h"
+
+namespace {
+
+using rel::Problem;
+
+bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+
+size_t elem_size(relation_dtype dt) { return dt == RELATION_F32 ? 4 : 2; }
+
+relation_status check_shape(const relation_shape& s, relation_dtype dt) {
+  if (dt != RELATION_F32 && dt != RELATION_BF16) return RELATION_ERR_INVALID_ARG;
+  if (s.B < 1 || s.T < 1 || s.H < 1 || s.d_h < 1) return RELATION_ERR_INVALID_ARG;
+  if ((long long)s.B * s.H > 65535) return RELATION_ERR_UNSUPPORTED;  // grid.y limit
+  if (s.sB < 1 || s.sT < 1 || s.sH < 1) return RELATION_ERR_INVALID_ARG;
+  if (!rel::simt::supports(dt, s.d_h) && !rel::tc::supports(dt, s.d_h))
+    return RELATION_ERR_UNSUPPORTED;
+  const long long vec = 16 / (long long)elem_size(dt);
+  if (s.sB % vec || s.sT % vec || s.sH % vec) return RELATION_ERR_ALIGNMENT;
+  return RELATION_OK;
+}
+
+relation_status check_scalars(float lambda, float tau_s) {
+  if (!isfinite(lambda) || !isfinite(tau_s) || !(tau_s > 0.0f)) return RELATION_ERR_INVALID_ARG;
+  return RELATION_OK;
+}
+
+relation_status check_ptrs(std::initializer_list<const void*> ptrs) {
+  for (const void* p : ptrs)
+    if (!p) return RELATION_ERR_INVALID_ARG;
+  for (const void* p : ptrs)
+    if (!aligned16(p)) return RELATION_ERR_ALIGNMENT;
+  return RELATION_OK;
+}
+
+// Family that will run: 1 = SIMT, 2 = tcgen05; 0 when the request cannot be served.
+int pick_family(relation_kernel kernel, relation_dtype dt, int d) {
+  const bool tc = rel::tc::supports(dt, d), simt = rel::simt::supports(dt, d);
+  switch (kernel) {
+    case RELATION_KERNEL_AUTO: return tc ? 2 : (simt ? 1 : 0);
+    case RELATION_KERNEL_SIMT: return simt ? 1 : 0;
+    case RELATION_KERNEL_TCGEN05: return tc ? 2 : 0;
+  }
+  return 0;
+}
+
+Problem make_problem(relation_shape s, relation_dtype dt, float lambda, float tau_s,
+                     int* dev_status) {
+  Problem p{};
+  p.lambda = lambda;
+  p.tau_s = tau_s;
+  p.inv_sqrt_d = 1.0f / sqrtf((float)s.d_h);
+  p.B = s.B; p.T = s.T; p.H = s.H; p.d = s.d_h;
+  p.sB = s.sB; p.sT = s.sT; p.sH = s.sH;
+  p.dtype = dt;
+  p.dev_status = dev_status;
+  return p;
+}
+
+relation_status from_cuda(cudaError_t e) { return e == cudaSuccess ? RELATION_OK : RELATION_ERR_CUDA; }
+
+}  // namespace
+
+extern "C" {
+
+relation_status relation_fwd_ex(const void* q, const void* k, const void* v, void* o, float* logz,
+                                float lambda, float tau_s, relation_shape shp, relation_dtype dt,
+                                relation_kernel kernel, int* dev_status, relation_stream_t stream) {
+  relation_status st;
+  if ((st = check_shape(shp, dt)) != RELATION_OK) return st;
+  if ((st = check_scalars(lambda, tau_s)) != RELATION_OK) return st;
+  if ((st = check_ptrs({q, k, v, o, logz})) != RELATION_OK) return st;
+  if (dev_status && (reinterpret_cast<uintptr_t>(dev_status) & 3u)) return RELATION_ERR_ALIGNMENT;
+  const int fam = pick_family(kernel, dt, shp.d_h);
+  if (fam == 0) return RELATION_ERR_UNSUPPORTED;
+  Problem p = make_problem(shp, dt, lambda, tau_s, dev_status);
+  p.q = q; p.k = k; p.v = v; p.out = o; p.logz = logz;
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  return from_cuda(fam == 2 ? rel::tc::launch_fwd(p, s) : rel::simt::launch_fwd(p, s));
+}
+
+relation_status relation_fwd(const void* q, const void* k, const void* v, void* o, float* logz,
+                             float lambda, float tau_s, relation_shape shp, relation_dtype dt,
+                             int* dev_status, relation_stream_t stream) {
+  return relation_fwd_ex(q, k, v, o, logz, lambda, tau_s, shp, dt, RELATION_KERNEL_AUTO,
+                         dev_status, stream);
+}
+
+size_t relation_bwd_workspace_size(relation_shape shp, relation_dtype dt) {
+  if (check_shape(shp, dt) != RELATION_OK) return 0;
+  return rel::bwd_workspace_bytes(shp.B, shp.H, shp.T, shp.d_h);
+}
+
+relation_status relation_bwd_ex(const void* q, const void* k, const void* v, const void* o,
+                                const void* dout, const float* logz, void* dq, void* dk, void* dv,
+                                float* dlambda, float lambda, float tau_s, relation_shape shp,
+                                relation_dtype dt, void* workspace, size_t ws_bytes,
+                                relation_kernel kernel, int* dev_status, relation_stream_t stream) {
+  relation_status st;
+  if ((st = check_shape(shp, dt)) != RELATION_OK) return st;
+  if ((st = check_scalars(lambda, tau_s)) != RELATION_OK) return st;
+  if ((st = check_ptrs({q, k, v, o, dout, logz, dq, dk, dv})) != RELATION_OK) return st;
+  if (!dlambda) return RELATION_ERR_INVALID_ARG;
+  if (reinterpret_cast<uintptr_t>(dlambda) & 3u) return RELATION_ERR_ALIGNMENT;
+  if (dev_status && (reinterpret_cast<uintptr_t>(dev_status) & 3u)) return RELATION_ERR_ALIGNMENT;
+  const size_t need = rel::bwd_workspace_bytes(shp.B, shp.H, shp.T, shp.d_h);
+  if (!workspace || ws_bytes < need) return RELATION_ERR_WORKSPACE;
+  if (reinterpret_cast<uintptr_t>(workspace) & 255u) return RELATION_ERR_ALIGNMENT;
+  const int fam = pick_family(kernel, dt, shp.d_h);
+  if (fam == 0) return RELATION_ERR_UNSUPPORTED;
+
+  Problem p = make_problem(shp, dt, lambda, tau_s, dev_status);
+  p.q = q; p.k = k; p.v = v; p.o = o; p.dout = dout; p.logz_in = logz;
+  p.dq = dq; p.dk = dk; p.dv = dv; p.dlambda = dlambda;
+  rel::BwdWorkspace ws = rel::carve_workspace(workspace, shp.B, shp.H, shp.T, shp.d_h);
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  cudaError_t e = rel::bwd_common::launch_pre(p, ws, s);
+  if (e != cudaSuccess) return RELATION_ERR_CUDA;
+  e = fam == 2 ? rel::tc::launch_bwd(p, ws, s) : rel::simt::launch_bwd(p, ws, s);
+  if (e != cudaSuccess) return RELATION_ERR_CUDA;
+  return from_cuda(rel::bwd_common::launch_dlambda(p, ws, s));
+}
+
+relation_status relation_bwd(const void* q, const void* k, const void* v, const void* o,
+                             const void* dout, const float* logz, void* dq, void* dk, void* dv,
+                             float* dlambda, float lambda, float tau_s, relation_shape shp,
+                             relation_dtype dt, void* workspace, size_t ws_bytes,
+                             int* dev_status, relation_stream_t stream) {
+  return relation_bwd_ex(q, k, v, o, dout, logz, dq, dk, dv, dlambda, lambda, tau_s, shp, dt,
+                         workspace, ws_bytes, RELATION_KERNEL_AUTO, dev_status, stream);
+}
+
+const char* relation_status_string(relation_status s) {
+  switch (s) {
+    case RELATION_OK: return "RELATION_OK";
+    case RELATION_ERR_INVALID_ARG: return "RELATION_ERR_INVALID_ARG";
+    case RELATION_ERR_UNSUPPORTED: return "RELATION_ERR_UNSUPPORTED";
+    case RELATION_ERR_ALIGNMENT: return "RELATION_ERR_ALIGNMENT";
+    case RELATION_ERR_WORKSPACE: return "RELATION_ERR_WORKSPACE";
+    case RELATION_ERR_CUDA: return "RELATION_ERR_CUDA";
+    case RELATION_ERR_TIMEOUT: return "RELATION_ERR_TIMEOUT";
+  }
+  return "RELATION_ERR_UNKNOWN";
+}
+
+int relation_version(void) { return (1 << 16) | 0; }
+
+int relation_launch_count(relation_dtype dt, int d_h, relation_kernel kernel, int backward) {
+  if (dt != RELATION_F32 && dt != RELATION_BF16) return 0;
+  const int fam = pick_family(kernel, dt, d_h);
+  if (fam == 0) return 0;
+  if (!backward) return 1;
+  // row pre-pass + Exchange tiles (SIMT: dK/dV and dQ kernels; tcgen05: tile kernel and
+  // dQ finalisation) + dlambda reduction
+  return fam == 2 ? rel::tc::bwd_launches() + 2 : 4;
+}
+
+relation_status relation_selftest_wait_timeout(int* dev_status, int timeout_us,
+                                               relation_stream_t stream) {
+  if (!dev_status || timeout_us < 1 || timeout_us > 100000) return RELATION_ERR_INVALID_ARG;
+  if (reinterpret_cast<uintptr_t>(dev_status) & 3u) return RELATION_ERR_ALIGNMENT;
+  return from_cuda(
+      rel::launch_selftest_wait(dev_status, timeout_us, reinterpret_cast<cudaStream_t>(stream)));
+}
+
+}  // extern "C"

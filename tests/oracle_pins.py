@@ -342,6 +342,19 @@ def pin_mhr_bwd_sums(orc):
     assert abs(dl - tot) <= 1e-13 * max(1.0, abs(tot))
 
 
+def pin_bwd_tail_rows(orc):
+    """Rows of the softmax-gradient form are independent: restricting the backward to
+    rows r >= r0 leaves dq rows >= r0 and dk, dv rows >= r0 unchanged (only rows i >= j
+    feed key j, Eq. causal-relation)."""
+    q, k, v, g = _rand(13, 4, 32, scale=1.3)
+    full = orc.bwd(q, k, v, g, 0.5)
+    for r0 in (0, 5, 12):
+        dq, dk, dv, _ = orc.bwd_tail(q, k, v, g, 0.5, r0)
+        _close(dq[r0:], full[0][r0:], 1e-14); _close(dk[r0:], full[1][r0:], 1e-14)
+        _close(dv[r0:], full[2][r0:], 1e-14)
+        assert np.all(dq[:r0] == 0)
+
+
 ALL_PINS = [
     pin_T1_closed_form, pin_T2_hand_formula, pin_zero_evidence, pin_materialised_structure,
     pin_self_bounded_extremes, pin_factorized_equals_materialised, pin_self_exchange_split,
@@ -349,5 +362,5 @@ ALL_PINS = [
     pin_lambda_plus_limit, pin_lambda_minus_limit, pin_lambda_zero_logsumexp,
     pin_mhr_heads_independent, pin_causality, pin_rows_subset, pin_bwd_finite_differences,
     pin_bwd_two_derivations, pin_bwd_T1, pin_bwd_dv_mass, pin_bwd_lambda_plus_limit,
-    pin_mhr_bwd_sums,
+    pin_mhr_bwd_sums, pin_bwd_tail_rows,
 ]

@@ -1,0 +1,117 @@
+"""Helpers shared by the GPU parity tests: tolerances, runs through the C ABI, and
+oracle references for selected heads."""
+from __future__ import annotations
+
+import numpy as np
+import torch
+
+import oracle
+from paper_2608_20172_gb300 import binding, workloads
+
+# Tolerances (max-abs for fp32; max_elem|gpu - ref| / max_elem|ref| per tensor for bf16).
+TOL = {
+    ("fp32", "out"): 1e-4, ("fp32", "grad"): 1e-3,
+    ("bf16", "out"): 2e-2, ("bf16", "grad"): 5e-2,
+}
+
+
+def err_metric(got, ref, dtype: str) -> float:
+    got = np.asarray(got, dtype=np.float64)
+    ref = np.asarray(ref, dtype=np.float64)
+    diff = float(np.max(np.abs(got - ref))) if got.size else 0.0
+    if dtype == "fp32":
+        return diff
+    scale = float(np.max(np.abs(ref))) if ref.size else 0.0
+    return diff / max(scale, 1e-30)
+
+
+def check(name: str, got, ref, dtype: str, kind: str):
+    e = err_metric(got, ref, dtype)
+    bound = TOL[(dtype, kind)]
+    assert np.all(np.isfinite(np.asarray(got, dtype=np.float64))), f"{name}: non-finite values"
+    assert e <= bound, f"{name}: error {e:.3e} > {bound:.1e} ({dtype}, {kind})"
+    return e
+
+
+def check_logz(name: str, got, ref, dtype: str):
+    """logZ is fp32 on both paths; absolute bound 1e-4 (fp32 inputs) or 2e-2 (bf16)."""
+    got = np.asarray(got, dtype=np.float64)
+    e = float(np.max(np.abs(got - np.asarray(ref, dtype=np.float64)))) if got.size else 0.0
+    bound = 1e-4 if dtype == "fp32" else 2e-2
+    assert np.all(np.isfinite(got)), f"{name}: non-finite values"
+    assert e <= bound, f"{name}: abs error {e:.3e} > {bound:.1e}"
+    return e
+
+
+def check_dlambda(got: float, ref: float, dtype: str):
+    bound = 1e-3 if dtype == "fp32" else 5e-2
+    assert np.isfinite(got), "dlambda not finite"
+    assert abs(got - ref) <= bound * max(abs(ref), 1.0 if dtype == "fp32" else 1e-3), \
+        f"dlambda {got} vs {ref}"
+
+
+def kernel_available(kernel: str, dtype: str, d: int) -> bool:
+    """True when the C ABI serves this kernel family for (dtype, d)."""
+    dev = torch.device("cuda:0")
+    dt = torch.float32 if dtype == "fp32" else torch.bfloat16
+    x = torch.zeros((1, 1, 1, d), dtype=dt, device=dev)
+    try:
+        binding.fwd(x, x, x, 0.5, kernel=kernel)
+    except binding.RelationError as e:
+        if e.code == binding.ERR_UNSUPPORTED:
+            return False
+        raise
+    torch.cuda.synchronize()
+    return True
+
+
+def gpu_run(q, k, v, do, lam, tau=workloads.TAU_S, kernel="auto", bwd=True):
+    """Run forward (+ backward) through the C ABI on cuda:0; returns CPU tensors."""
+    dev = torch.device("cuda:0")
+    qd, kd, vd = (t.to(dev) for t in (q, k, v))
+    status = torch.zeros(1, dtype=torch.int32, device=dev)
+    y, logz = binding.fwd(qd, kd, vd, lam, tau, kernel=kernel, dev_status=status)
+    out = {"Y": y, "logZ": logz}
+    if bwd:
+        dod = do.to(dev)
+        dq, dk, dv, dl = binding.bwd(qd, kd, vd, y, dod, logz, lam, tau, kernel=kernel,
+                                     dev_status=status)
+        out.update({"dQ": dq, "dK": dk, "dV": dv, "dlambda": dl})
+    torch.cuda.synchronize()
+    st = int(status.item())
+    assert st == 0, f"device status {binding.status_string(st)}"
+    res = {n: t.float().cpu() for n, t in out.items()}
+    res["dlambda"] = float(res["dlambda"].item()) if bwd else None
+    return res
+
+
+def head(t: torch.Tensor, b: int, h: int) -> np.ndarray:
+    """[T, d] fp64 numpy view of head (b, h) of a [B, T, H, d] tensor."""
+    return t[b, :, h, :].double().numpy()
+
+
+def oracle_heads(q, k, v, do, lam, heads, tau=workloads.TAU_S, bwd=True):
+    """fp64 oracle forward (+ backward) for the listed (b, h) heads."""
+    ref = {}
+    for (b, h) in heads:
+        qh, kh, vh = head(q, b, h), head(k, b, h), head(v, b, h)
+        y, lz = oracle.fwd(qh, kh, vh, lam, tau)
+        r = {"Y": y, "logZ": lz}
+        if bwd:
+            dq, dk, dv, dl = oracle.bwd(qh, kh, vh, head(do, b, h), lam, tau)
+            r.update({"dQ": dq, "dK": dk, "dV": dv, "dlambda": dl})
+        ref[(b, h)] = r
+    return ref
+
+
+def compare_heads(res, ref, dtype, bwd=True):
+    errs = {}
+    for (b, h), r in ref.items():
+        errs[("Y", b, h)] = check(f"Y[{b},{h}]", res["Y"][b, :, h].numpy(), r["Y"], dtype, "out")
+        errs[("logZ", b, h)] = check_logz(f"logZ[{b},{h}]", res["logZ"][b, h].numpy(),
+                                          r["logZ"], dtype)
+        if bwd:
+            for n in ("dQ", "dK", "dV"):
+                errs[(n, b, h)] = check(f"{n}[{b},{h}]", res[n][b, :, h].numpy(), r[n], dtype,
+                                        "grad")
+    return errs

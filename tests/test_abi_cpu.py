@@ -1,0 +1,146 @@
+"""The C ABI library without a GPU: it loads, exports every declared symbol, and rejects
+bad arguments synchronously (before any CUDA call)."""
+import ctypes
+import os
+import re
+import subprocess
+
+import pytest
+
+from paper_2608_20172_gb300 import binding
+from paper_2608_20172_gb300 import build as libbuild
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+HEADER = os.path.join(ROOT, "include", "relation.h")
+
+
+@pytest.fixture(scope="module")
+def lib():
+    libbuild.build()
+    return binding.load()
+
+
+def declared_functions():
+    src = open(HEADER).read()
+    src = re.sub(r"/\*.*?\*/", "", src, flags=re.S)
+    return sorted(set(re.findall(r"^\s*(?:const\s+)?\w+\s*\*?\s*(relation_\w+)\s*\(", src, re.M)))
+
+
+def test_header_declares_the_boundary():
+    names = declared_functions()
+    for n in ("relation_fwd", "relation_bwd", "relation_bwd_workspace_size",
+              "relation_status_string"):
+        assert n in names
+    assert set(names) == set(binding.EXPORTED)
+
+
+def test_library_exports_every_declared_symbol(lib):
+    out = subprocess.run(["nm", "-D", "--defined-only", libbuild.LIB], capture_output=True,
+                         text=True, check=True).stdout
+    exported = set(re.findall(r"\s[TW]\s+(\w+)$", out, re.M))
+    for n in declared_functions():
+        assert n in exported, n
+        assert getattr(lib, n) is not None
+
+
+def test_status_strings(lib):
+    for code, name in enumerate(["RELATION_OK", "RELATION_ERR_INVALID_ARG",
+                                 "RELATION_ERR_UNSUPPORTED", "RELATION_ERR_ALIGNMENT",
+                                 "RELATION_ERR_WORKSPACE", "RELATION_ERR_CUDA",
+                                 "RELATION_ERR_TIMEOUT"]):
+        assert binding.status_string(code) == name
+    assert binding.status_string(99) == "RELATION_ERR_UNKNOWN"
+    assert lib.relation_version() >> 16 == 1
+
+
+def _shape(B=1, T=8, H=2, d=64, sB=None, sT=None, sH=None):
+    sH = d if sH is None else sH
+    sT = H * d if sT is None else sT
+    sB = T * H * d if sB is None else sB
+    return binding.Shape(B, T, H, d, sB, sT, sH)
+
+
+def _fwd(lib, ptrs, shape, dt=binding.BF16, lam=0.5, tau=2.0, kernel=0):
+    q, k, v, o, lz = ptrs
+    return lib.relation_fwd_ex(q, k, v, o, lz, lam, tau, shape, dt, kernel, None, None)
+
+
+GOOD = [0x10000, 0x20000, 0x30000, 0x40000, 0x50000]  # aligned, never dereferenced here
+
+
+@pytest.mark.parametrize("case,expect", [
+    ("null q", binding.ERR_INVALID_ARG),
+    ("misaligned v", binding.ERR_ALIGNMENT),
+    ("T = 0", binding.ERR_INVALID_ARG),
+    ("d = 40", binding.ERR_UNSUPPORTED),
+    ("odd stride", binding.ERR_ALIGNMENT),
+    ("tau = 0", binding.ERR_INVALID_ARG),
+    ("lambda inf", binding.ERR_INVALID_ARG),
+    ("bad dtype", binding.ERR_INVALID_ARG),
+    ("tcgen05 for fp32", binding.ERR_UNSUPPORTED),
+    ("too many heads", binding.ERR_UNSUPPORTED),
+])
+def test_fwd_rejects_bad_arguments(lib, case, expect):
+    ptrs, shape, kw = list(GOOD), _shape(), {}
+    if case == "null q":
+        ptrs[0] = None
+    elif case == "misaligned v":
+        ptrs[2] = 0x30008
+    elif case == "T = 0":
+        shape = _shape(T=0)
+    elif case == "d = 40":
+        shape = _shape(d=40)
+    elif case == "odd stride":
+        shape = _shape(sT=130)
+    elif case == "tau = 0":
+        kw["tau"] = 0.0
+    elif case == "lambda inf":
+        kw["lam"] = float("inf")
+    elif case == "bad dtype":
+        kw["dt"] = 7
+    elif case == "tcgen05 for fp32":
+        kw["dt"], kw["kernel"] = binding.F32, 2
+    elif case == "too many heads":
+        shape = _shape(B=300, H=300)
+    assert _fwd(lib, ptrs, shape, **kw) == expect
+
+
+def test_bwd_workspace_rules(lib):
+    shape = _shape(B=2, T=100, H=3, d=64)
+    need = lib.relation_bwd_workspace_size(shape, binding.BF16)
+    rows = 2 * 3 * 100
+    assert need >= rows * 64 * 4 + 3 * rows * 4
+    assert lib.relation_bwd_workspace_size(_shape(T=0), binding.BF16) == 0
+    p = [ctypes.c_void_p(0x10000 * (i + 1)) for i in range(10)]
+    args = p[:9] + [p[9]]
+    rc = lib.relation_bwd_ex(*args, 0.5, 2.0, shape, binding.BF16, ctypes.c_void_p(0x100000),
+                             need - 1, 0, None, None)
+    assert rc == binding.ERR_WORKSPACE
+    rc = lib.relation_bwd_ex(*args, 0.5, 2.0, shape, binding.BF16, None, need, 0, None, None)
+    assert rc == binding.ERR_WORKSPACE
+    rc = lib.relation_bwd_ex(*args, 0.5, 2.0, shape, binding.BF16, ctypes.c_void_p(0x100010),
+                             need, 0, None, None)
+    assert rc == binding.ERR_ALIGNMENT
+    rc = lib.relation_bwd_ex(*p[:9], None, 0.5, 2.0, shape, binding.BF16,
+                             ctypes.c_void_p(0x100000), need, 0, None, None)
+    assert rc == binding.ERR_INVALID_ARG
+
+
+def test_selftest_argument_checks(lib):
+    assert lib.relation_selftest_wait_timeout(None, 10, None) == binding.ERR_INVALID_ARG
+    assert lib.relation_selftest_wait_timeout(ctypes.c_void_p(0x1000), 0, None) == \
+        binding.ERR_INVALID_ARG
+    assert lib.relation_selftest_wait_timeout(ctypes.c_void_p(0x1002), 10, None) == \
+        binding.ERR_ALIGNMENT
+
+
+def test_binding_refuses_cpu_tensors():
+    import torch
+    x = torch.zeros(1, 4, 1, 64, dtype=torch.bfloat16)
+    with pytest.raises(ValueError):
+        binding.fwd(x, x, x, 0.5)
+
+
+def test_missing_library_fails_loudly(tmp_path):
+    with pytest.raises(binding.RelationLibraryMissing):
+        binding.load(str(tmp_path / "nope.so"))

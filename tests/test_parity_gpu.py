@@ -1,0 +1,244 @@
+"""GPU parity: the CUDA path through the C ABI against the fp64 oracle.
+
+Small shapes span several tiles and a ragged tail and are compared element by element
+on every head.  The workloads' full sizes run in the benchmark's launch configuration
+and are compared on sampled heads (every element of those heads), and on the long
+sequence on sampled rows plus two exact restrictions the causal structure allows.
+"""
+import numpy as np
+import pytest
+import torch
+
+import oracle
+from paper_2608_20172_gb300 import binding, workloads
+from tests import parity_util as pu
+
+pytestmark = pytest.mark.gpu
+
+LAM = workloads.LAMBDA_INIT
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _lib():
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    binding.load()
+
+
+def _families(dtype, d):
+    fams = ["simt"]
+    if pu.kernel_available("tcgen05", dtype, d):
+        fams.append("tcgen05")
+    return fams
+
+
+def _all_heads(w):
+    return [(b, h) for b in range(w.B) for h in range(w.H)]
+
+
+# --- fp32 -------------------------------------------------------------------
+
+def test_tiny_fp32_all_heads():
+    w = workloads.WORKLOADS["tiny"]
+    q, k, v, do = workloads.make_inputs(w)
+    res = pu.gpu_run(q, k, v, do, LAM)
+    ref = pu.oracle_heads(q, k, v, do, LAM, _all_heads(w))
+    pu.compare_heads(res, ref, "fp32")
+    pu.check_dlambda(res["dlambda"], sum(r["dlambda"] for r in ref.values()), "fp32")
+
+
+@pytest.mark.parametrize("T", [1, 2, 3, 65, 200])
+@pytest.mark.parametrize("d", [32, 64, 128])
+def test_fp32_shapes(T, d):
+    w = workloads.custom(2, 1, T, d, "fp32", qk_std=1.0 / np.sqrt(d))
+    q, k, v, do = workloads.make_inputs(w, seed=T + d)
+    res = pu.gpu_run(q, k, v, do, LAM)
+    ref = pu.oracle_heads(q, k, v, do, LAM, _all_heads(w))
+    pu.compare_heads(res, ref, "fp32")
+    pu.check_dlambda(res["dlambda"], sum(r["dlambda"] for r in ref.values()), "fp32")
+
+
+# --- bf16, small shapes, every kernel family ----------------------------------
+
+@pytest.mark.parametrize("T", [1, 2, 3, 127, 128, 129, 255, 300, 513])
+@pytest.mark.parametrize("d", [64, 128])
+def test_bf16_shapes(T, d):
+    w = workloads.custom(1, 2, T, d, "bf16")
+    q, k, v, do = workloads.make_inputs(w, seed=1000 + T + d)
+    ref = pu.oracle_heads(q, k, v, do, LAM, _all_heads(w))
+    for fam in _families("bf16", d):
+        res = pu.gpu_run(q, k, v, do, LAM, kernel=fam)
+        pu.compare_heads(res, ref, "bf16")
+        pu.check_dlambda(res["dlambda"], sum(r["dlambda"] for r in ref.values()), "bf16")
+
+
+@pytest.mark.parametrize("lam", [0.0, -1.0, 3.0])
+def test_bf16_lambda_values(lam):
+    w = workloads.custom(2, 2, 333, 64, "bf16")
+    q, k, v, do = workloads.make_inputs(w, seed=7)
+    ref = pu.oracle_heads(q, k, v, do, lam, _all_heads(w))
+    for fam in _families("bf16", 64):
+        res = pu.gpu_run(q, k, v, do, lam, kernel=fam)
+        pu.compare_heads(res, ref, "bf16")
+        pu.check_dlambda(res["dlambda"], sum(r["dlambda"] for r in ref.values()), "bf16")
+
+
+def test_bf16_32():
+    w = workloads.custom(1, 3, 150, 32, "bf16")
+    q, k, v, do = workloads.make_inputs(w, seed=3)
+    res = pu.gpu_run(q, k, v, do, LAM)
+    ref = pu.oracle_heads(q, k, v, do, LAM, _all_heads(w))
+    pu.compare_heads(res, ref, "bf16")
+
+
+def test_bhtd_layout():
+    """[B, H, T, d] storage (a permuted view) gives the same result as [B, T, H, d]."""
+    w = workloads.custom(2, 3, 200, 64, "bf16")
+    q, k, v, do = workloads.make_inputs(w, seed=11)
+    dev = torch.device("cuda:0")
+
+    def bhtd(t):
+        return t.permute(0, 2, 1, 3).contiguous().to(dev).permute(0, 2, 1, 3)
+
+    qd, kd, vd, dod = (bhtd(t) for t in (q, k, v, do))
+    y, lz = binding.fwd(qd, kd, vd, LAM)
+    dq, dk, dv, dl = binding.bwd(qd, kd, vd, y, dod, lz, LAM)
+    res = pu.gpu_run(q, k, v, do, LAM)
+    for name, t in (("Y", y), ("dQ", dq), ("dK", dk), ("dV", dv)):
+        assert torch.equal(t.float().cpu(), res[name]), name
+    assert torch.equal(lz.cpu(), res["logZ"])
+
+
+# --- full-size workloads in the benchmark's launch configuration --------------
+
+@pytest.mark.parametrize("name", ["10M", "30M", "100M"])
+def test_workload_full_size_sampled_heads(name):
+    w = workloads.WORKLOADS[name]
+    q, k, v, do = workloads.make_inputs(w)
+    res = pu.gpu_run(q, k, v, do, LAM)
+    heads = [(0, 0), (w.B - 1, w.H - 1), (w.B // 2, 1)]
+    ref = pu.oracle_heads(q, k, v, do, LAM, heads)
+    pu.compare_heads(res, ref, "bf16")
+    # every head: finite, logZ >= the Self logit's lower bound (logZ_i >= S_i > 0)
+    for n in ("Y", "dQ", "dK", "dV", "logZ"):
+        assert torch.isfinite(res[n]).all(), n
+    assert (res["logZ"] > 0).all()
+    # dlambda over all heads, from the oracle on all heads (multi-threaded)
+    _, _, _, dl_all = oracle.mhr_bwd(q.double().numpy(), k.double().numpy(), v.double().numpy(),
+                                     do.double().numpy(), LAM)
+    pu.check_dlambda(res["dlambda"], dl_all, "bf16")
+
+
+def test_long_context_full_size():
+    w = workloads.WORKLOADS["long"]
+    q, k, v, do = workloads.make_inputs(w)
+    T = w.T
+    res = pu.gpu_run(q, k, v, do, LAM)
+    for n in ("Y", "dQ", "dK", "dV", "logZ"):
+        assert torch.isfinite(res[n]).all(), n
+    # forward on sampled rows of two heads (first rows, tile edges, ragged, last rows)
+    rows = sorted({0, 1, 2, 127, 128, 129, 4095, 4096, 8191, 12345, T - 2, T - 1})
+    for (b, h) in [(0, 0), (1, 15)]:
+        qh, kh, vh = pu.head(q, b, h), pu.head(k, b, h), pu.head(v, b, h)
+        y, lz = oracle.fwd_rows(qh, kh, vh, rows, LAM)
+        pu.check(f"Y rows [{b},{h}]", res["Y"][b, rows, h].numpy(), y, "bf16", "out")
+        pu.check_logz(f"logZ rows [{b},{h}]", res["logZ"][b, h, rows].numpy(), lz, "bf16")
+    # backward, last 256 rows of one head: exact dQ rows and dK, dV keys >= T - 256
+    b, h = 1, 7
+    r0 = T - 256
+    dq, dk, dv, _ = oracle.bwd_tail(pu.head(q, b, h), pu.head(k, b, h), pu.head(v, b, h),
+                                    pu.head(do, b, h), LAM, r0)
+    pu.check("dQ tail", res["dQ"][b, r0:, h].numpy(), dq[r0:], "bf16", "grad")
+    pu.check("dK tail", res["dK"][b, r0:, h].numpy(), dk[r0:], "bf16", "grad")
+    pu.check("dV tail", res["dV"][b, r0:, h].numpy(), dv[r0:], "bf16", "grad")
+
+
+def test_long_context_prefix_gradient():
+    """dO = 0 on rows >= T' makes every gradient equal to that of the T'-prefix problem
+    (rows i >= T' then carry dR_i. = 0): the full-size launch is checked exactly on the
+    prefix, on sampled heads, including dlambda over all heads."""
+    w = workloads.WORKLOADS["long"]
+    q, k, v, do = workloads.make_inputs(w)
+    Tp = 1024
+    do = do.clone()
+    do[:, Tp:] = 0
+    res = pu.gpu_run(q, k, v, do, LAM)
+    for (b, h) in [(0, 3), (1, 12)]:
+        dq, dk, dv, _ = oracle.bwd(pu.head(q, b, h)[:Tp], pu.head(k, b, h)[:Tp],
+                                   pu.head(v, b, h)[:Tp], pu.head(do, b, h)[:Tp], LAM)
+        pu.check(f"dQ prefix [{b},{h}]", res["dQ"][b, :Tp, h].numpy(), dq, "bf16", "grad")
+        pu.check(f"dK prefix [{b},{h}]", res["dK"][b, :Tp, h].numpy(), dk, "bf16", "grad")
+        pu.check(f"dV prefix [{b},{h}]", res["dV"][b, :Tp, h].numpy(), dv, "bf16", "grad")
+    for n in ("dQ", "dK", "dV"):
+        assert torch.count_nonzero(res[n][:, Tp:]) == 0, n
+    _, _, _, dl_all = oracle.mhr_bwd(q[:, :Tp].double().numpy(), k[:, :Tp].double().numpy(),
+                                     v[:, :Tp].double().numpy(), do[:, :Tp].double().numpy(), LAM)
+    pu.check_dlambda(res["dlambda"], dl_all, "bf16")
+
+
+# --- determinism, invariants, failure detection --------------------------------
+
+def test_deterministic_repeat():
+    w = workloads.custom(2, 2, 700, 64, "bf16")
+    q, k, v, do = workloads.make_inputs(w, seed=5)
+    a = pu.gpu_run(q, k, v, do, LAM)
+    b = pu.gpu_run(q, k, v, do, LAM)
+    for n in ("Y", "logZ", "dK", "dV"):
+        assert torch.equal(a[n], b[n]), n
+    pu.check("dQ repeat", a["dQ"].numpy(), b["dQ"].numpy(), "bf16", "grad")
+
+
+def test_large_lambda_keeps_self():
+    """lambda >> 0 suppresses Exchange (-lambda log i): Y = V on rows i >= 2 up to bf16."""
+    w = workloads.custom(1, 2, 300, 64, "bf16")
+    q, k, v, do = workloads.make_inputs(w, seed=9)
+    res = pu.gpu_run(q, k, v, do, 60.0, bwd=False)
+    pu.check("Y ~ V", res["Y"].numpy(), v.float().numpy(), "bf16", "out")
+
+
+def test_wait_timeout_reports_status():
+    dev = torch.device("cuda:0")
+    st = torch.zeros(1, dtype=torch.int32, device=dev)
+    assert binding.selftest_wait_timeout(st, 2000) == binding.OK
+    torch.cuda.synchronize()
+    assert int(st.item()) == binding.ERR_TIMEOUT
+    # the context is still usable afterwards
+    w = workloads.custom(1, 1, 64, 64, "bf16")
+    q, k, v, do = workloads.make_inputs(w)
+    res = pu.gpu_run(q, k, v, do, LAM)
+    assert torch.isfinite(res["Y"]).all()
+
+
+def test_device_argument_errors():
+    dev = torch.device("cuda:0")
+    x = torch.randn(1, 64, 2, 64, device=dev).to(torch.bfloat16)
+    y, lz = binding.fwd(x, x, x, LAM)
+    with pytest.raises(binding.RelationError) as e:
+        binding.bwd(x, x, x, y, x, lz, LAM, workspace=torch.empty(16, dtype=torch.uint8, device=dev))
+    assert e.value.code == binding.ERR_WORKSPACE
+    buf = torch.empty(1 * 64 * 2 * 64 + 1, dtype=torch.bfloat16, device=dev)
+    mis = buf[1:].view(1, 64, 2, 64)
+    with pytest.raises(binding.RelationError) as e:
+        binding.fwd(mis, mis, mis, LAM)
+    assert e.value.code == binding.ERR_ALIGNMENT
+    odd = torch.zeros(1, 8, 1, 40, dtype=torch.bfloat16, device=dev)
+    with pytest.raises(binding.RelationError) as e:
+        binding.fwd(odd, odd, odd, LAM)
+    assert e.value.code == binding.ERR_UNSUPPORTED
+    with pytest.raises(binding.RelationError) as e:
+        binding.fwd(x, x, x, float("nan"))
+    assert e.value.code == binding.ERR_INVALID_ARG
+
+
+def test_autograd_wrapper_matches_binding():
+    w = workloads.custom(1, 2, 130, 64, "bf16")
+    q, k, v, do = workloads.make_inputs(w, seed=13)
+    dev = torch.device("cuda:0")
+    qd, kd, vd = (t.to(dev).requires_grad_(True) for t in (q, k, v))
+    lam = torch.tensor(LAM, device=dev, requires_grad=True)
+    y = binding.RelationFunction.apply(qd, kd, vd, lam)
+    y.backward(do.to(dev))
+    res = pu.gpu_run(q, k, v, do, LAM)
+    assert torch.equal(y.detach().float().cpu(), res["Y"])
+    assert torch.equal(kd.grad.float().cpu(), res["dK"])
+    assert abs(float(lam.grad) - res["dlambda"]) <= 1e-6 * max(1.0, abs(res["dlambda"]))
