@@ -7,9 +7,16 @@
 //   F_ii  = exp(S_i - logZ_i)
 //   dR_ii = F_ii (dO_i . v_i - D_i)
 //   dS_ii = dR_ii S_i (1 - S_i) / tau_S      (dL/du_ii)
-// and the row's share of dL/dlambda.  dL/dlambda = -sum_i log i sum_{j<i} dR_ij; each
-// row of dR sums to zero (sum_k F_ik (H_ik - D_i) = D_i - D_i), so the inner sum is
-// -dR_ii and dL/dlambda = sum_i log i dR_ii: the diagonal alone carries it.
+// and the row's Self share of dL/dlambda.
+//
+// dL/dlambda = -sum_i log i X_i with X_i = sum_{j<i} dR_ij.  Each row of dR sums to zero
+// (sum_k F_ik (H_ik - D_i) = D_i - D_i), so X_i = -dR_ii as well, and for any weight w_i
+//   -X_i = w_i dR_ii - (1 - w_i) X_i.
+// D_i is only known up to the rounding of the stored output (D_i + eps): the Self
+// estimate then errs by -F_ii eps and the Exchange sum by -g_i eps.  Taking w_i = g_i =
+// 1 - F_ii cancels eps exactly:  g_i (-F_ii eps) - F_ii (-g_i eps) = 0.  So
+//   dL/dlambda = sum_i log i g_i dR_ii  -  sum_{j<i} log i F_ii dR_ij,
+// the first sum here (per row) and the second in the Exchange tile kernel (per pair).
 #include <math.h>
 
 #include "common.cuh"
@@ -21,7 +28,9 @@ size_t bwd_workspace_bytes(int B, int H, int T, int d) {
   auto up = [](size_t x) { return (x + 255) & ~(size_t)255; };
   const size_t rows = (size_t)B * H * T;
   const size_t n_pre = (rows + 7) / 8;
-  return up(rows * d * sizeof(float)) + 3 * up(rows * sizeof(float)) + up(n_pre * sizeof(float));
+  const size_t n_main = (size_t)((T + 63) / 64) * B * H;
+  return up(rows * d * sizeof(float)) + 3 * up(rows * sizeof(float)) +
+         up((n_pre + n_main) * sizeof(float));
 }
 
 BwdWorkspace carve_workspace(void* base, int B, int H, int T, int d) {
@@ -35,6 +44,7 @@ BwdWorkspace carve_workspace(void* base, int B, int H, int T, int d) {
   w.dS_self = reinterpret_cast<float*>(p); p += up(rows * sizeof(float));
   w.dlam_part = reinterpret_cast<float*>(p);
   w.n_pre_blocks = (int)((rows + 7) / 8);
+  w.n_main_slots = ((T + 63) / 64) * B * H;
   return w;
 }
 
@@ -89,7 +99,7 @@ __global__ void __launch_bounds__(kWarps * 32) pre_kernel(Problem p, BwdWorkspac
       ws.F_self[gr] = F;
       ws.dS_self[gr] = dR * S * (1.0f - S) / p.tau_s;
     }
-    contrib = logf((float)(r + 1)) * dR;
+    contrib = logf((float)(r + 1)) * (1.0f - F) * dR;  // log i * g_i * dR_ii
   }
   if (lane == 0) part[warp] = contrib;
   __syncthreads();
@@ -102,10 +112,11 @@ __global__ void __launch_bounds__(kWarps * 32) pre_kernel(Problem p, BwdWorkspac
 }
 
 // One block, fixed summation order (deterministic), fp64 accumulation.
-__global__ void __launch_bounds__(1024) dlambda_kernel(BwdWorkspace ws, float* out) {
+__global__ void __launch_bounds__(1024) dlambda_kernel(BwdWorkspace ws, int n_main, float* out) {
   __shared__ double red[1024];
   double s = 0.0;
-  for (int i = threadIdx.x; i < ws.n_pre_blocks; i += 1024) s += (double)ws.dlam_part[i];
+  const int n = ws.n_pre_blocks + n_main;
+  for (int i = threadIdx.x; i < n; i += 1024) s += (double)ws.dlam_part[i];
   red[threadIdx.x] = s;
   __syncthreads();
   for (int w = 512; w > 0; w >>= 1) {
@@ -124,8 +135,8 @@ cudaError_t launch_pre(const Problem& p, const BwdWorkspace& ws, cudaStream_t s)
   return cudaGetLastError();
 }
 
-cudaError_t launch_dlambda(const Problem& p, const BwdWorkspace& ws, cudaStream_t s) {
-  dlambda_kernel<<<1, 1024, 0, s>>>(ws, p.dlambda);
+cudaError_t launch_dlambda(const Problem& p, const BwdWorkspace& ws, int n_main, cudaStream_t s) {
+  dlambda_kernel<<<1, 1024, 0, s>>>(ws, n_main, p.dlambda);
   return cudaGetLastError();
 }
 

@@ -39,8 +39,11 @@ struct BwdWorkspace {
   float* D;          // [B][H][T]     D_i = dO_i . Y_i
   float* F_self;     // [B][H][T]     F_ii = exp(S_i - logZ_i)
   float* dS_self;    // [B][H][T]     dL/du_ii, u = U_ii (scaled evidence)
-  float* dlam_part;  // [n_pre_blocks] per-block partial sums of log(i) dR_ii
+  // dlambda partials: [n_pre_blocks] from the row pre-pass, then [n_main_slots] from
+  // the Exchange tile kernel (one per CTA).
+  float* dlam_part;
   int n_pre_blocks;
+  int n_main_slots;  // capacity reserved for the tile kernel's CTAs
 };
 
 size_t bwd_workspace_bytes(int B, int H, int T, int d);
@@ -50,20 +53,24 @@ namespace simt {
 bool supports(relation_dtype dt, int d);
 cudaError_t launch_fwd(const Problem& p, cudaStream_t s);
 cudaError_t launch_bwd(const Problem& p, const BwdWorkspace& ws, cudaStream_t s);
+int main_ctas(const Problem& p);  // tile-kernel CTAs writing a dlambda partial
 }  // namespace simt
 
 namespace bwd_common {
 // Per-row Self part of the backward (D_i, F_ii, dS_ii and dlambda partials).
 cudaError_t launch_pre(const Problem& p, const BwdWorkspace& ws, cudaStream_t s);
-// Deterministic dlambda reduction of the per-block partials.
-cudaError_t launch_dlambda(const Problem& p, const BwdWorkspace& ws, cudaStream_t s);
+// Deterministic dlambda reduction of the pre-pass partials and the first n_main tile-kernel
+// partials.
+cudaError_t launch_dlambda(const Problem& p, const BwdWorkspace& ws, int n_main, cudaStream_t s);
 }  // namespace bwd_common
 
 namespace tc {
-bool supports(relation_dtype dt, int d);
+bool supports(relation_dtype dt, int d);      // forward
+bool supports_bwd(relation_dtype dt, int d);  // backward
 cudaError_t launch_fwd(const Problem& p, cudaStream_t s);
 cudaError_t launch_bwd(const Problem& p, const BwdWorkspace& ws, cudaStream_t s);
 int bwd_launches();  // launches made by launch_bwd
+int main_ctas(const Problem& p);
 }  // namespace tc
 
 cudaError_t launch_selftest_wait(int* dev_status, int timeout_us, cudaStream_t s);

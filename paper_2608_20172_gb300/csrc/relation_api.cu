@@ -43,8 +43,9 @@ relation_status check_ptrs(std::initializer_list<const void*> ptrs) {
 }
 
 // Family that will run: 1 = SIMT, 2 = tcgen05; 0 when the request cannot be served.
-int pick_family(relation_kernel kernel, relation_dtype dt, int d) {
-  const bool tc = rel::tc::supports(dt, d), simt = rel::simt::supports(dt, d);
+int pick_family(relation_kernel kernel, relation_dtype dt, int d, bool backward) {
+  const bool tc = backward ? rel::tc::supports_bwd(dt, d) : rel::tc::supports(dt, d);
+  const bool simt = rel::simt::supports(dt, d);
   switch (kernel) {
     case RELATION_KERNEL_AUTO: return tc ? 2 : (simt ? 1 : 0);
     case RELATION_KERNEL_SIMT: return simt ? 1 : 0;
@@ -80,7 +81,7 @@ relation_status relation_fwd_ex(const void* q, const void* k, const void* v, voi
   if ((st = check_scalars(lambda, tau_s)) != RELATION_OK) return st;
   if ((st = check_ptrs({q, k, v, o, logz})) != RELATION_OK) return st;
   if (dev_status && (reinterpret_cast<uintptr_t>(dev_status) & 3u)) return RELATION_ERR_ALIGNMENT;
-  const int fam = pick_family(kernel, dt, shp.d_h);
+  const int fam = pick_family(kernel, dt, shp.d_h, false);
   if (fam == 0) return RELATION_ERR_UNSUPPORTED;
   Problem p = make_problem(shp, dt, lambda, tau_s, dev_status);
   p.q = q; p.k = k; p.v = v; p.out = o; p.logz = logz;
@@ -115,7 +116,7 @@ relation_status relation_bwd_ex(const void* q, const void* k, const void* v, con
   const size_t need = rel::bwd_workspace_bytes(shp.B, shp.H, shp.T, shp.d_h);
   if (!workspace || ws_bytes < need) return RELATION_ERR_WORKSPACE;
   if (reinterpret_cast<uintptr_t>(workspace) & 255u) return RELATION_ERR_ALIGNMENT;
-  const int fam = pick_family(kernel, dt, shp.d_h);
+  const int fam = pick_family(kernel, dt, shp.d_h, true);
   if (fam == 0) return RELATION_ERR_UNSUPPORTED;
 
   Problem p = make_problem(shp, dt, lambda, tau_s, dev_status);
@@ -127,7 +128,8 @@ relation_status relation_bwd_ex(const void* q, const void* k, const void* v, con
   if (e != cudaSuccess) return RELATION_ERR_CUDA;
   e = fam == 2 ? rel::tc::launch_bwd(p, ws, s) : rel::simt::launch_bwd(p, ws, s);
   if (e != cudaSuccess) return RELATION_ERR_CUDA;
-  return from_cuda(rel::bwd_common::launch_dlambda(p, ws, s));
+  const int n_main = fam == 2 ? rel::tc::main_ctas(p) : rel::simt::main_ctas(p);
+  return from_cuda(rel::bwd_common::launch_dlambda(p, ws, n_main, s));
 }
 
 relation_status relation_bwd(const void* q, const void* k, const void* v, const void* o,
@@ -156,7 +158,7 @@ int relation_version(void) { return (1 << 16) | 0; }
 
 int relation_launch_count(relation_dtype dt, int d_h, relation_kernel kernel, int backward) {
   if (dt != RELATION_F32 && dt != RELATION_BF16) return 0;
-  const int fam = pick_family(kernel, dt, d_h);
+  const int fam = pick_family(kernel, dt, d_h, backward != 0);
   if (fam == 0) return 0;
   if (!backward) return 1;
   // row pre-pass + Exchange tiles (SIMT: dK/dV and dQ kernels; tcgen05: tile kernel and

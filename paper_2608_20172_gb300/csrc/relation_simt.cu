@@ -216,6 +216,8 @@ __global__ void __launch_bounds__(kThreads) bwd_dkdv_kernel(Problem p, BwdWorksp
   float* Gs = Qs + kTile * D;        // dO tile
   float* cs = Gs + kTile * D;        // -lambda log i - logZ_i
   float* Ds = cs + kTile;            // D_i
+  float* ws_l = Ds + kTile;          // log i * F_ii (Exchange weight of dlambda)
+  __shared__ float red[kThreads / 32];
   const int rl = threadIdx.x >> 2, part = threadIdx.x & 3;
   const int bh = blockIdx.y, b = bh / p.H, h = bh % p.H;
   const int k0 = blockIdx.x * kRows;
@@ -232,6 +234,7 @@ __global__ void __launch_bounds__(kThreads) bwd_dkdv_kernel(Problem p, BwdWorksp
   float kv[D / 4], vv[D / 4], dk[D / 4], dv[D / 4];
 #pragma unroll
   for (int c = 0; c < D / 4; ++c) { kv[c] = vv[c] = dk[c] = dv[c] = 0.f; }
+  float dlam = 0.f;  // -sum_i log i F_ii dR_ij over this key's Exchange pairs
   if (key_ok) {
     load_row_chunks<TI, D>(K + (long long)j * p.sT, part, kv);
     load_row_chunks<TI, D>(V + (long long)j * p.sT, part, vv);
@@ -242,8 +245,10 @@ __global__ void __launch_bounds__(kThreads) bwd_dkdv_kernel(Problem p, BwdWorksp
     stage_tile<TI, D>(Gs, G, p.sT, q0, p.T);
     for (int ii = threadIdx.x; ii < kTile; ii += kThreads) {
       const int i = q0 + ii;
-      cs[ii] = i < p.T ? -p.lambda * logf((float)(i + 1)) - logz[i] : -INFINITY;
+      const float li = logf((float)(i + 1));
+      cs[ii] = i < p.T ? -p.lambda * li - logz[i] : -INFINITY;
       Ds[ii] = i < p.T ? Drow[i] : 0.f;
+      ws_l[ii] = i < p.T ? li * ws.F_self[(long long)bh * p.T + i] : 0.f;
     }
     __syncthreads();
     for (int ii = 0; ii < kTile; ++ii) {
@@ -256,10 +261,23 @@ __global__ void __launch_bounds__(kThreads) bwd_dkdv_kernel(Problem p, BwdWorksp
         const float P = expf(E + cs[ii]);
         const float dR = P * (dP - Ds[ii]);
         const float dS = dR * (sg + E * (1.f - sg));   // SiLU'(u) = sigma + E (1 - sigma)
+        dlam = fmaf(-ws_l[ii], dR, dlam);
         axpy_part<D>(dv, P, Gs + ii * D, part);
         axpy_part<D>(dk, dS, Qs + ii * D, part);
       }
     }
+  }
+  // per-CTA dlambda partial (the 4 threads of a key hold the same value: count part 0)
+  float c = part == 0 ? dlam : 0.f;
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) c += __shfl_xor_sync(0xffffffffu, c, o);
+  if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = c;
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    float t = 0.f;
+#pragma unroll
+    for (int w = 0; w < kThreads / 32; ++w) t += red[w];
+    ws.dlam_part[ws.n_pre_blocks + blockIdx.y * gridDim.x + blockIdx.x] = t;
   }
   if (!key_ok) return;
   // Self terms of key j: dv_j += F_jj dO_j, dk_j += dS_jj q_j; then the 1/sqrt(d) of U.
@@ -373,7 +391,7 @@ static cudaError_t fwd_t(const Problem& p, cudaStream_t s) {
 
 template <typename TI, int D>
 static cudaError_t bwd_t(const Problem& p, const BwdWorkspace& ws, cudaStream_t s) {
-  const size_t smem_kv = 2u * kTile * D * sizeof(float) + 2u * kTile * sizeof(float);
+  const size_t smem_kv = 2u * kTile * D * sizeof(float) + 3u * kTile * sizeof(float);
   const size_t smem_q = 2u * kTile * D * sizeof(float);
   cudaError_t e = cudaFuncSetAttribute(bwd_dkdv_kernel<TI, D>,
                                        cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem_kv);
@@ -387,6 +405,8 @@ static cudaError_t bwd_t(const Problem& p, const BwdWorkspace& ws, cudaStream_t 
   bwd_dq_kernel<TI, D><<<grid, kThreads, smem_q, s>>>(p, ws);
   return cudaGetLastError();
 }
+
+int main_ctas(const Problem& p) { return ((p.T + kRows - 1) / kRows) * p.B * p.H; }
 
 cudaError_t launch_fwd(const Problem& p, cudaStream_t s) {
   if (p.dtype == RELATION_F32) {

@@ -1,13 +1,386 @@
-// relation_tc_fwd.cu -- placeholder until the tcgen05 forward lands.
+// relation_tc_fwd.cu -- tcgen05 / TMA / TMEM forward of FlashRelation (bf16, d_h 64 or 128).
+//
+// One CTA owns a tile of BM = 128 query rows of one head and scans the key/value tiles
+// j0 = 0, 128, ... up to and including its diagonal tile (Sec. 5.1, App. A.3).  Two CTAs
+// share an SM (each allocates 256 TMEM columns), so the tensor core of one CTA overlaps
+// the elementwise work of the other.
+//
+// Warp roles (192 threads):
+//   warps 0-3  Exchange scan + epilogue: thread t owns query row q0 + t (TMEM lane t).
+//   warp  4    TMA producer: Q tile once, then K and V tiles through a ring of stages.
+//   warp  5    TMEM allocator and MMA issuer (one elected thread).
+// Per key tile j:
+//   MMA   U_j = Q K_j^T                       -> TMEM columns [0, 128) (fp32)
+//   scan  E = SiLU(U / sqrt(d)) for keys < row (Self excluded); running maximum m (kept
+//         as an upper bound of max E, rescaling z only when it grows by > 2^8), row sum
+//         l += sum exp(E - m); P = exp(E - m) as bf16 written back into TMEM columns
+//         [0, 64) (two per 32-bit column); the diagonal tile also yields
+//         S_i = sigmoid(U_ii / (sqrt(d) tau_S)).
+//   MMA   z += P V_j  (A operand P read from TMEM)  -> TMEM columns [128, 128 + d)
+// Epilogue (App. A.3.3-A.3.5): L^E = m + log l, A = L^E - lambda log i,
+//   g = sigmoid(A - S), Y = (1 - g) v_i + g z / l, logZ = logaddexp(S, A); row 1 has an
+//   empty history: g = 0, Y = v_1, logZ = S_1 (App. A.1.8).
+// R and F never leave the SM.  Every mbarrier wait is bounded (common.cuh).
+#include <cudaTypedefs.h>
+#include <math.h>
+
+#include <mutex>
+
+#include "common.cuh"
 #include "kernels.h"
 
 namespace rel {
 namespace tc {
-bool supports(relation_dtype, int) { return false; }
-cudaError_t launch_fwd(const Problem&, cudaStream_t) { return cudaErrorNotSupported; }
+
+constexpr int BM = 128;        // query rows per CTA
+constexpr int BN = 128;        // keys per tile
+constexpr int kThreads = 192;  // 4 scan warps + TMA warp + MMA warp
+constexpr int kTmemCols = 256; // S/P tile (128) + z accumulator (<= 128)
+constexpr int kSCol = 0;
+constexpr int kOCol = 128;
+constexpr float kRescaleLog2 = 8.0f;  // rescale z only when the max grows by > 2^8
+
+template <int D>
+struct FwdCfg {
+  static constexpr int KB = D / 64;            // 64-column (128-byte) swizzle blocks along d
+  static constexpr int TILE = BN * D * 2;      // bytes of one K, V (or Q) tile
+  static constexpr int STAGES = D == 64 ? 2 : 1;
+  static constexpr int OFF_Q = 0;
+  static constexpr int OFF_K = OFF_Q + TILE;
+  static constexpr int OFF_V = OFF_K + STAGES * TILE;
+  static constexpr int OFF_BAR = OFF_V + STAGES * TILE;
+  static constexpr int SMEM = OFF_BAR + 256 + 1024;  // barriers + 1024-byte alignment slack
+};
+
+// mbarrier slots
+enum : int { B_Q = 0, B_KF = 1, B_KE = 3, B_VF = 5, B_VE = 7, B_S = 9, B_P = 10, B_O = 11 };
+
+// Bounded wait used while draining at teardown: never raises, just gives up.
+__device__ __forceinline__ void drain_wait(uint32_t bar, uint32_t parity) {
+  const unsigned long long t0 = globaltimer_ns();
+  while (!mbar_try_wait(bar, parity)) {
+    if (globaltimer_ns() - t0 > 20ull * 1000ull * 1000ull) return;  // 20 ms
+  }
+}
+
+__device__ __forceinline__ float silu_acc(float x) { return x / (1.0f + __expf(-x)); }
+
+template <int D>
+__global__ void __launch_bounds__(kThreads, 2)
+    fwd_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmK,
+                  const __grid_constant__ CUtensorMap tmV, Problem p, int n_qt) {
+  using C = FwdCfg<D>;
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>(
+      (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
+  const uint32_t sb = smem_u32(smem);
+  auto bar = [&](int i) -> uint32_t { return sb + C::OFF_BAR + 8u * (uint32_t)i; };
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(smem + C::OFF_BAR + 128);
+  volatile int* abort_flag = reinterpret_cast<volatile int*>(smem + C::OFF_BAR + 136);
+
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int BH = p.B * p.H;
+  const int qt = n_qt - 1 - (int)(blockIdx.x / BH);  // heaviest query tiles first
+  const int bh = (int)(blockIdx.x % BH);
+  const int b = bh / p.H, h = bh % p.H;
+  const int q0 = qt * BM;
+  const int n_kv = qt + 1;
+
+  if (threadIdx.x == 0) {
+    mbar_init(bar(B_Q), 1);
+    for (int s = 0; s < C::STAGES; ++s) {
+      mbar_init(bar(B_KF + s), 1);
+      mbar_init(bar(B_KE + s), 1);
+      mbar_init(bar(B_VF + s), 1);
+      mbar_init(bar(B_VE + s), 1);
+    }
+    mbar_init(bar(B_S), 1);
+    mbar_init(bar(B_P), 128);
+    mbar_init(bar(B_O), 1);
+    *abort_flag = 0;
+    fence_mbar_init();
+  }
+  if (warp == 5) tmem_alloc(smem_u32(tmem_slot), kTmemCols);
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = *tmem_slot;
+  const Abort ab{abort_flag, p.dev_status};
+
+  if (warp == 4) {
+    // ------------------------------------------------------------------ TMA producer
+    if (lane == 0) {
+      tma_prefetch_desc(&tmQ);
+      tma_prefetch_desc(&tmK);
+      tma_prefetch_desc(&tmV);
+      mbar_arrive_expect_tx(bar(B_Q), C::TILE);
+      for (int kb = 0; kb < C::KB; ++kb)
+        tma_load_4d(sb + C::OFF_Q + kb * BM * 128, &tmQ, bar(B_Q), kb * 64, q0, h, b);
+      int issued = 0;
+      for (int j = 0; j < n_kv; ++j) {
+        const int s = j % C::STAGES, u = j / C::STAGES;
+        if (u > 0 && !mbar_wait(bar(B_KE + s), (u - 1) & 1, ab)) break;
+        mbar_arrive_expect_tx(bar(B_KF + s), C::TILE);
+        for (int kb = 0; kb < C::KB; ++kb)
+          tma_load_4d(sb + C::OFF_K + s * C::TILE + kb * BN * 128, &tmK, bar(B_KF + s), kb * 64,
+                      j * BN, h, b);
+        if (u > 0 && !mbar_wait(bar(B_VE + s), (u - 1) & 1, ab)) {
+          issued = j + 1;  // K of tile j is in flight, V is not
+          break;
+        }
+        mbar_arrive_expect_tx(bar(B_VF + s), C::TILE);
+        for (int kb = 0; kb < C::KB; ++kb)
+          tma_load_4d(sb + C::OFF_V + s * C::TILE + kb * BN * 128, &tmV, bar(B_VF + s), kb * 64,
+                      j * BN, h, b);
+        issued = j + 1;
+      }
+      if (ab.raised()) {
+        // let copies already in flight land before the CTA releases its shared memory
+        drain_wait(bar(B_Q), 0);
+        for (int j = issued - C::STAGES > 0 ? issued - C::STAGES : 0; j < issued; ++j) {
+          const int s = j % C::STAGES, u = j / C::STAGES;
+          drain_wait(bar(B_KF + s), u & 1);
+          drain_wait(bar(B_VF + s), u & 1);
+        }
+      }
+    }
+  } else if (warp == 5) {
+    // ------------------------------------------------------------------ MMA issuer
+    if (lane == 0) {
+      constexpr uint32_t idesc_qk = idesc_bf16_f32(BM, BN, false, false);
+      constexpr uint32_t idesc_pv = idesc_bf16_f32(BM, D, false, true);
+      bool ok = mbar_wait(bar(B_Q), 0, ab);
+      tc_fence_after();
+      for (int j = 0; ok && j < n_kv; ++j) {
+        const int s = j % C::STAGES, u = j / C::STAGES;
+        if (!(ok = mbar_wait(bar(B_KF + s), u & 1, ab))) break;
+        tc_fence_after();
+#pragma unroll
+        for (int kk = 0; kk < D / 16; ++kk) {
+          const uint32_t koff = (kk >> 2) * (BM * 128) + (kk & 3) * 32;
+          const uint64_t a = smem_desc_sw128(sb + C::OFF_Q + koff, 16, 1024);
+          const uint64_t bd = smem_desc_sw128(sb + C::OFF_K + s * C::TILE + koff, 16, 1024);
+          mma_ss(tmem + kSCol, a, bd, idesc_qk, kk > 0 ? 1u : 0u);
+        }
+        mma_commit(bar(B_S));       // U_j ready (and every earlier z update done)
+        mma_commit(bar(B_KE + s));  // K stage free
+        if (!(ok = mbar_wait(bar(B_VF + s), u & 1, ab))) break;
+        if (!(ok = mbar_wait(bar(B_P), j & 1, ab))) break;
+        tc_fence_after();
+#pragma unroll
+        for (int kk = 0; kk < BN / 16; ++kk) {
+          const uint64_t bd =
+              smem_desc_sw128(sb + C::OFF_V + s * C::TILE + kk * 16 * 128, BN * 128, 1024);
+          mma_ts(tmem + kOCol, tmem + kSCol + kk * 8, bd, idesc_pv, (j > 0 || kk > 0) ? 1u : 0u);
+        }
+        mma_commit(bar(B_VE + s));  // V stage free
+      }
+      mma_commit(bar(B_O));  // z final (or whatever completed before an abort)
+    }
+    __syncwarp();
+  } else {
+    // ------------------------------------------------------------------ scan + epilogue
+    const int t = threadIdx.x;  // 0..127: row q0 + t, TMEM lane t
+    const int r = q0 + t;
+    const uint32_t trow = tmem + ((uint32_t)(warp * 32) << 16);
+    const float isd = p.inv_sqrt_d;
+    const float ch = 0.5f * isd;            // h = U * ch = u / 2
+    const float c2 = ch * kLog2e;           // E log2(e) = U * c2 * (1 + tanh(h))
+    float m = -INFINITY;                    // running bound of max E, log2 units
+    float l = 0.f;
+    float u_self = 0.f;
+    bool ok = true;
+    for (int j = 0; j < n_kv; ++j) {
+      ok = __all_sync(0xffffffffu, mbar_wait(bar(B_S), j & 1, ab));  // warp-uniform
+      if (!ok) break;
+      tc_fence_after();
+      uint32_t U[BN];
+      tmem_ld32(trow + kSCol + 0, U + 0);
+      tmem_ld32(trow + kSCol + 32, U + 32);
+      tmem_ld32(trow + kSCol + 64, U + 64);
+      tmem_ld32(trow + kSCol + 96, U + 96);
+      tmem_ld_wait();
+      const bool diag = (j == qt);
+      // pass 1: masked maximum of the raw evidence (keys j0 + c < row  <=>  c < t on the
+      // diagonal tile; every key of an earlier tile is history)
+      float umax = -INFINITY;
+#pragma unroll
+      for (int c = 0; c < BN; ++c) {
+        const float x = __uint_as_float(U[c]);
+        if (!diag || c < t) umax = fmaxf(umax, x);
+        if (diag && c == t) u_self = x;
+      }
+      // Upper bound of max E: SiLU is increasing on [0, inf) and negative on (-inf, 0).
+      float mt;
+      if (umax == -INFINITY) {
+        mt = -INFINITY;
+      } else if (umax >= 0.f) {
+        mt = silu_acc(umax * isd) * kLog2e;
+      } else {
+        mt = 0.f;
+      }
+      const float mn = fmaxf(m, mt);
+      const bool grow = mn > m + kRescaleLog2;  // false while both are -inf
+      const float scale = grow ? exp2f(m - mn) : 1.0f;
+      if (grow) m = mn;
+      l *= scale;
+      if (j > 0 && __any_sync(0xffffffffu, grow)) {
+        // z (TMEM) is stable: U_j's commit came after the z update of tile j-1
+#pragma unroll
+        for (int c0 = 0; c0 < D; c0 += 32) {
+          uint32_t z[32];
+          tmem_ld32(trow + kOCol + c0, z);
+          tmem_ld_wait();
+#pragma unroll
+          for (int c = 0; c < 32; ++c) z[c] = __float_as_uint(__uint_as_float(z[c]) * scale);
+          tmem_st16(trow + kOCol + c0, z);
+          tmem_st16(trow + kOCol + c0 + 16, z + 16);
+        }
+      }
+      // pass 2: P = 2^(E log2 e - m) on the history, 0 elsewhere; written back as bf16
+      const float negm = (m == -INFINITY) ? 0.f : -m;
+      float rowsum = 0.f;
+#pragma unroll
+      for (int c0 = 0; c0 < BN; c0 += 32) {
+        uint32_t pk[16];
+#pragma unroll
+        for (int c = 0; c < 32; c += 2) {
+          float pr[2];
+#pragma unroll
+          for (int e = 0; e < 2; ++e) {
+            const int cc = c0 + c + e;
+            const float x = __uint_as_float(U[cc]);
+            const float th = tanh_approx(x * ch);
+            const float w = fmaf(th, c2, c2);
+            float pv = ex2_approx(fmaf(x, w, negm));
+            if (diag && cc >= t) pv = 0.f;
+            pr[e] = pv;
+          }
+          rowsum += pr[0] + pr[1];
+          pk[c >> 1] = pack_bf16x2(pr[0], pr[1]);
+        }
+        tmem_st16(trow + kSCol + (c0 >> 1), pk);
+      }
+      l += rowsum;
+      tmem_st_wait();
+      tc_fence_before();
+      mbar_arrive(bar(B_P));
+    }
+    // ---------------------------------------------------------------- epilogue
+    if (ok) ok = __all_sync(0xffffffffu, mbar_wait(bar(B_O), 0, ab));
+    tc_fence_after();
+    if (ok) {
+      float g = 0.f, inv_l = 0.f;
+      float lz;
+      const float S = 1.0f / (1.0f + __expf(-(u_self * isd) / p.tau_s));
+      if (l > 0.f) {
+        const float A = m * kLn2 + __logf(l) - p.lambda * __logf((float)(r + 1));
+        g = 1.0f / (1.0f + __expf(S - A));
+        const float hi = fmaxf(S, A), lo = fminf(S, A);
+        lz = hi + log1pf(__expf(lo - hi));
+        inv_l = 1.0f / l;
+      } else {
+        lz = S;  // empty history (row 1)
+      }
+      const long long base = (long long)b * p.sB + (long long)h * p.sH + (long long)r * p.sT;
+      const __nv_bfloat16* vrow = reinterpret_cast<const __nv_bfloat16*>(p.v) + base;
+      __nv_bfloat16* yrow = reinterpret_cast<__nv_bfloat16*>(p.out) + base;
+#pragma unroll
+      for (int c0 = 0; c0 < D; c0 += 32) {
+        uint32_t z[32];
+        tmem_ld32(trow + kOCol + c0, z);
+        tmem_ld_wait();
+        if (r < p.T) {
+#pragma unroll
+          for (int c8 = 0; c8 < 32; c8 += 8) {
+            const uint4 vv = *reinterpret_cast<const uint4*>(vrow + c0 + c8);
+            const uint32_t vw[4] = {vv.x, vv.y, vv.z, vv.w};
+            uint32_t yw[4];
+#pragma unroll
+            for (int e = 0; e < 4; ++e) {
+              const float2 vf = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&vw[e]));
+              const float z0 = __uint_as_float(z[c8 + 2 * e]) * inv_l;
+              const float z1 = __uint_as_float(z[c8 + 2 * e + 1]) * inv_l;
+              yw[e] = pack_bf16x2(fmaf(g, z0 - vf.x, vf.x), fmaf(g, z1 - vf.y, vf.y));
+            }
+            *reinterpret_cast<uint4*>(yrow + c0 + c8) = make_uint4(yw[0], yw[1], yw[2], yw[3]);
+          }
+        }
+      }
+      if (r < p.T) p.logz[(long long)bh * p.T + r] = lz;
+    }
+  }
+
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 5) {
+    tc_fence_after();
+    tmem_dealloc(tmem, kTmemCols);
+  }
+}
+
+// ---------------------------------------------------------------------------------
+// Host side
+// ---------------------------------------------------------------------------------
+static PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
+  static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
+  static std::once_flag once;
+  std::call_once(once, [] {
+    void* ptr = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &ptr, 12000, cudaEnableDefault,
+                                         &q) == cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(ptr);
+  });
+  return fn;
+}
+
+// 4-D map over a [B][T][H][d] bf16 tensor: box = 64 columns (128 bytes) x `rows` rows of
+// one (h, b), 128-byte swizzle, zero fill outside the tensor.
+static bool make_tmap(CUtensorMap* m, const void* base, const Problem& p, int rows) {
+  auto fn = encode_fn();
+  if (!fn) return false;
+  cuuint64_t dims[4] = {(cuuint64_t)p.d, (cuuint64_t)p.T, (cuuint64_t)p.H, (cuuint64_t)p.B};
+  cuuint64_t strides[3] = {(cuuint64_t)p.sT * 2, (cuuint64_t)p.sH * 2, (cuuint64_t)p.sB * 2};
+  cuuint32_t box[4] = {64, (cuuint32_t)rows, 1, 1};
+  cuuint32_t estr[4] = {1, 1, 1, 1};
+  CUresult r = fn(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 4, const_cast<void*>(base), dims, strides,
+                  box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                  CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  return r == CUDA_SUCCESS;
+}
+
+bool supports(relation_dtype dt, int d) { return dt == RELATION_BF16 && (d == 64 || d == 128); }
+bool supports_bwd(relation_dtype, int) { return false; }
+
+template <int D>
+static cudaError_t fwd_t(const Problem& p, cudaStream_t s) {
+  CUtensorMap mq, mk, mv;
+  if (!make_tmap(&mq, p.q, p, BM) || !make_tmap(&mk, p.k, p, BN) || !make_tmap(&mv, p.v, p, BN))
+    return cudaErrorInvalidValue;
+  const int smem = FwdCfg<D>::SMEM;
+  cudaError_t e =
+      cudaFuncSetAttribute(fwd_tc_kernel<D>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+  if (e != cudaSuccess) return e;
+  const int n_qt = (p.T + BM - 1) / BM;
+  const long long grid = (long long)n_qt * p.B * p.H;
+  if (grid > 0x7fffffffLL) return cudaErrorInvalidConfiguration;
+  fwd_tc_kernel<D><<<(unsigned)grid, kThreads, smem, s>>>(mq, mk, mv, p, n_qt);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_fwd(const Problem& p, cudaStream_t s) {
+  if (p.d == 64) return fwd_t<64>(p, s);
+  if (p.d == 128) return fwd_t<128>(p, s);
+  return cudaErrorInvalidValue;
+}
+
 cudaError_t launch_bwd(const Problem&, const BwdWorkspace&, cudaStream_t) {
   return cudaErrorNotSupported;
 }
 int bwd_launches() { return 2; }
+int main_ctas(const Problem&) { return 0; }
+
 }  // namespace tc
 }  // namespace rel

@@ -50,23 +50,25 @@ def check_dlambda(got: float, ref: float, dtype: str):
         f"dlambda {got} vs {ref}"
 
 
-def kernel_available(kernel: str, dtype: str, d: int) -> bool:
-    """True when the C ABI serves this kernel family for (dtype, d)."""
-    dev = torch.device("cuda:0")
-    dt = torch.float32 if dtype == "fp32" else torch.bfloat16
-    x = torch.zeros((1, 1, 1, d), dtype=dt, device=dev)
-    try:
-        binding.fwd(x, x, x, 0.5, kernel=kernel)
-    except binding.RelationError as e:
-        if e.code == binding.ERR_UNSUPPORTED:
-            return False
-        raise
-    torch.cuda.synchronize()
-    return True
+def kernel_available(kernel: str, dtype: str, d: int, which: str = "fwd") -> bool:
+    """True when the C ABI serves this kernel family for (dtype, d) (host-side query)."""
+    return binding.launches_per_call(kernel, dtype, d, which) > 0
 
 
-def gpu_run(q, k, v, do, lam, tau=workloads.TAU_S, kernel="auto", bwd=True):
-    """Run forward (+ backward) through the C ABI on cuda:0; returns CPU tensors."""
+def kernel_combos(dtype: str, d: int):
+    """(forward family, backward family) pairs to test: the CUDA-core pair always, and
+    each tensor-core kernel the library offers for this (dtype, d)."""
+    combos = [("simt", "simt")]
+    if kernel_available("tcgen05", dtype, d, "fwd"):
+        combos.append(("tcgen05", "simt"))
+    if kernel_available("tcgen05", dtype, d, "bwd"):
+        combos.append(("tcgen05", "tcgen05"))
+    return combos
+
+
+def gpu_run(q, k, v, do, lam, tau=workloads.TAU_S, kernel="auto", bwd=True, kernel_bwd=None):
+    """Run forward (+ backward) through the C ABI on cuda:0; returns CPU tensors.
+    ``kernel`` selects the forward family, ``kernel_bwd`` (default: same) the backward."""
     dev = torch.device("cuda:0")
     qd, kd, vd = (t.to(dev) for t in (q, k, v))
     status = torch.zeros(1, dtype=torch.int32, device=dev)
@@ -74,8 +76,8 @@ def gpu_run(q, k, v, do, lam, tau=workloads.TAU_S, kernel="auto", bwd=True):
     out = {"Y": y, "logZ": logz}
     if bwd:
         dod = do.to(dev)
-        dq, dk, dv, dl = binding.bwd(qd, kd, vd, y, dod, logz, lam, tau, kernel=kernel,
-                                     dev_status=status)
+        dq, dk, dv, dl = binding.bwd(qd, kd, vd, y, dod, logz, lam, tau,
+                                     kernel=kernel_bwd or kernel, dev_status=status)
         out.update({"dQ": dq, "dK": dk, "dV": dv, "dlambda": dl})
     torch.cuda.synchronize()
     st = int(status.item())

@@ -25,11 +25,6 @@ def _lib():
     binding.load()
 
 
-def _families(dtype, d):
-    fams = ["simt"]
-    if pu.kernel_available("tcgen05", dtype, d):
-        fams.append("tcgen05")
-    return fams
 
 
 def _all_heads(w):
@@ -66,8 +61,8 @@ def test_bf16_shapes(T, d):
     w = workloads.custom(1, 2, T, d, "bf16")
     q, k, v, do = workloads.make_inputs(w, seed=1000 + T + d)
     ref = pu.oracle_heads(q, k, v, do, LAM, _all_heads(w))
-    for fam in _families("bf16", d):
-        res = pu.gpu_run(q, k, v, do, LAM, kernel=fam)
+    for kf, kb in pu.kernel_combos("bf16", d):
+        res = pu.gpu_run(q, k, v, do, LAM, kernel=kf, kernel_bwd=kb)
         pu.compare_heads(res, ref, "bf16")
         pu.check_dlambda(res["dlambda"], sum(r["dlambda"] for r in ref.values()), "bf16")
 
@@ -77,8 +72,8 @@ def test_bf16_lambda_values(lam):
     w = workloads.custom(2, 2, 333, 64, "bf16")
     q, k, v, do = workloads.make_inputs(w, seed=7)
     ref = pu.oracle_heads(q, k, v, do, lam, _all_heads(w))
-    for fam in _families("bf16", 64):
-        res = pu.gpu_run(q, k, v, do, lam, kernel=fam)
+    for kf, kb in pu.kernel_combos("bf16", 64):
+        res = pu.gpu_run(q, k, v, do, lam, kernel=kf, kernel_bwd=kb)
         pu.compare_heads(res, ref, "bf16")
         pu.check_dlambda(res["dlambda"], sum(r["dlambda"] for r in ref.values()), "bf16")
 
