@@ -27,18 +27,21 @@ namespace rel {
 size_t bwd_workspace_bytes(int B, int H, int T, int d) {
   auto up = [](size_t x) { return (x + 255) & ~(size_t)255; };
   const size_t rows = (size_t)B * H * T;
+  const size_t rows_pad = (size_t)B * H * ((T + 127) / 128 * 128);
   const size_t n_pre = (rows + 7) / 8;
   const size_t n_main = (size_t)((T + 63) / 64) * B * H;
-  return up(rows * d * sizeof(float)) + 3 * up(rows * sizeof(float)) +
+  return up(rows_pad * d * sizeof(float)) + 3 * up(rows * sizeof(float)) +
          up((n_pre + n_main) * sizeof(float));
 }
 
 BwdWorkspace carve_workspace(void* base, int B, int H, int T, int d) {
   auto up = [](size_t x) { return (x + 255) & ~(size_t)255; };
   const size_t rows = (size_t)B * H * T;
+  const int t_pad = (T + 127) / 128 * 128;
   char* p = static_cast<char*>(base);
   BwdWorkspace w;
-  w.dq_acc = reinterpret_cast<float*>(p); p += up(rows * d * sizeof(float));
+  w.t_pad = t_pad;
+  w.dq_acc = reinterpret_cast<float*>(p); p += up((size_t)B * H * t_pad * d * sizeof(float));
   w.D = reinterpret_cast<float*>(p); p += up(rows * sizeof(float));
   w.F_self = reinterpret_cast<float*>(p); p += up(rows * sizeof(float));
   w.dS_self = reinterpret_cast<float*>(p); p += up(rows * sizeof(float));
@@ -94,10 +97,15 @@ __global__ void __launch_bounds__(kWarps * 32) pre_kernel(Problem p, BwdWorkspac
     const float S = 1.0f / (1.0f + expf(-u / p.tau_s));
     const float F = expf(S - p.logz_in[gr]);
     const float dR = F * (gv - gy);
+    const float dS = dR * S * (1.0f - S) / p.tau_s;
     if (lane == 0) {
       ws.D[gr] = gy;
       ws.F_self[gr] = F;
-      ws.dS_self[gr] = dR * S * (1.0f - S) / p.tau_s;
+      ws.dS_self[gr] = dS;
+    }
+    if (p.init_dq_acc) {  // seed the fp32 dQ accumulator with the Self term, x 2 sqrt(d)
+      float* acc = ws.dq_acc + ((long long)bh * ws.t_pad + r) * p.d;
+      for (int c = lane; c < p.d; c += 32) acc[c] = 2.0f * dS * ld<TI>(k + c);
     }
     contrib = logf((float)(r + 1)) * (1.0f - F) * dR;  // log i * g_i * dR_ii
   }

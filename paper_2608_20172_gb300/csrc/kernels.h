@@ -31,11 +31,14 @@ struct Problem {
   int B, T, H, d;
   long long sB, sT, sH;
   relation_dtype dtype;
+  int init_dq_acc;  // backward: the row pre-pass seeds BwdWorkspace::dq_acc (tensor-core path)
 };
 
 // Backward workspace carved out of the caller's buffer (all fp32, 256-byte aligned).
 struct BwdWorkspace {
-  float* dq_acc;     // [B][H][T][d]  Exchange part of dL/dP1 before scaling (tensor-core path)
+  float* dq_acc;     // [B][H][T_pad][d] 2 sqrt(d) dL/dP1 in fp32, T_pad = T rounded up to 128
+                     //   (tensor-core path: seeded with the Self term, then atomically summed)
+  int t_pad;
   float* D;          // [B][H][T]     D_i = dO_i . Y_i
   float* F_self;     // [B][H][T]     F_ii = exp(S_i - logZ_i)
   float* dS_self;    // [B][H][T]     dL/du_ii, u = U_ii (scaled evidence)

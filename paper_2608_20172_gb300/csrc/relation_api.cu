@@ -122,6 +122,7 @@ relation_status relation_bwd_ex(const void* q, const void* k, const void* v, con
   Problem p = make_problem(shp, dt, lambda, tau_s, dev_status);
   p.q = q; p.k = k; p.v = v; p.o = o; p.dout = dout; p.logz_in = logz;
   p.dq = dq; p.dk = dk; p.dv = dv; p.dlambda = dlambda;
+  p.init_dq_acc = fam == 2;
   rel::BwdWorkspace ws = rel::carve_workspace(workspace, shp.B, shp.H, shp.T, shp.d_h);
   cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
   cudaError_t e = rel::bwd_common::launch_pre(p, ws, s);

@@ -338,7 +338,7 @@ static PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
 
 // 4-D map over a [B][T][H][d] bf16 tensor: box = 64 columns (128 bytes) x `rows` rows of
 // one (h, b), 128-byte swizzle, zero fill outside the tensor.
-static bool make_tmap(CUtensorMap* m, const void* base, const Problem& p, int rows) {
+bool make_tmap_bf16(CUtensorMap* m, const void* base, const Problem& p, int rows) {
   auto fn = encode_fn();
   if (!fn) return false;
   cuuint64_t dims[4] = {(cuuint64_t)p.d, (cuuint64_t)p.T, (cuuint64_t)p.H, (cuuint64_t)p.B};
@@ -352,12 +352,12 @@ static bool make_tmap(CUtensorMap* m, const void* base, const Problem& p, int ro
 }
 
 bool supports(relation_dtype dt, int d) { return dt == RELATION_BF16 && (d == 64 || d == 128); }
-bool supports_bwd(relation_dtype, int) { return false; }
 
 template <int D>
 static cudaError_t fwd_t(const Problem& p, cudaStream_t s) {
   CUtensorMap mq, mk, mv;
-  if (!make_tmap(&mq, p.q, p, BM) || !make_tmap(&mk, p.k, p, BN) || !make_tmap(&mv, p.v, p, BN))
+  if (!make_tmap_bf16(&mq, p.q, p, BM) || !make_tmap_bf16(&mk, p.k, p, BN) ||
+      !make_tmap_bf16(&mv, p.v, p, BN))
     return cudaErrorInvalidValue;
   const int smem = FwdCfg<D>::SMEM;
   cudaError_t e =
@@ -375,12 +375,6 @@ cudaError_t launch_fwd(const Problem& p, cudaStream_t s) {
   if (p.d == 128) return fwd_t<128>(p, s);
   return cudaErrorInvalidValue;
 }
-
-cudaError_t launch_bwd(const Problem&, const BwdWorkspace&, cudaStream_t) {
-  return cudaErrorNotSupported;
-}
-int bwd_launches() { return 2; }
-int main_ctas(const Problem&) { return 0; }
 
 }  // namespace tc
 }  // namespace rel
