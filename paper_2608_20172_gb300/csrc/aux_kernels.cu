@@ -30,7 +30,7 @@ size_t bwd_workspace_bytes(int B, int H, int T, int d) {
   const size_t rows_pad = (size_t)B * H * ((T + 127) / 128 * 128);
   const size_t n_pre = (rows + 7) / 8;
   const size_t n_main = (size_t)((T + 63) / 64) * B * H;
-  return up(rows_pad * d * sizeof(float)) + 3 * up(rows * sizeof(float)) +
+  return up(rows_pad * d * sizeof(float)) + 4 * up(rows * sizeof(float)) +
          up((n_pre + n_main) * sizeof(float));
 }
 
@@ -45,6 +45,7 @@ BwdWorkspace carve_workspace(void* base, int B, int H, int T, int d) {
   w.D = reinterpret_cast<float*>(p); p += up(rows * sizeof(float));
   w.F_self = reinterpret_cast<float*>(p); p += up(rows * sizeof(float));
   w.dS_self = reinterpret_cast<float*>(p); p += up(rows * sizeof(float));
+  w.wl = reinterpret_cast<float*>(p); p += up(rows * sizeof(float));
   w.dlam_part = reinterpret_cast<float*>(p);
   w.n_pre_blocks = (int)((rows + 7) / 8);
   w.n_main_slots = ((T + 63) / 64) * B * H;
@@ -102,10 +103,6 @@ __global__ void __launch_bounds__(kWarps * 32) pre_kernel(Problem p, BwdWorkspac
       ws.D[gr] = gy;
       ws.F_self[gr] = F;
       ws.dS_self[gr] = dS;
-    }
-    if (p.init_dq_acc) {  // seed the fp32 dQ accumulator with the Self term, x 2 sqrt(d)
-      float* acc = ws.dq_acc + ((long long)bh * ws.t_pad + r) * p.d;
-      for (int c = lane; c < p.d; c += 32) acc[c] = 2.0f * dS * ld<TI>(k + c);
     }
     contrib = logf((float)(r + 1)) * (1.0f - F) * dR;  // log i * g_i * dR_ii
   }

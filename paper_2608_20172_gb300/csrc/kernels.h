@@ -31,17 +31,17 @@ struct Problem {
   int B, T, H, d;
   long long sB, sT, sH;
   relation_dtype dtype;
-  int init_dq_acc;  // backward: the row pre-pass seeds BwdWorkspace::dq_acc (tensor-core path)
 };
 
 // Backward workspace carved out of the caller's buffer (all fp32, 256-byte aligned).
 struct BwdWorkspace {
   float* dq_acc;     // [B][H][T_pad][d] 2 sqrt(d) dL/dP1 in fp32, T_pad = T rounded up to 128
-                     //   (tensor-core path: seeded with the Self term, then atomically summed)
+                     //   (tensor-core path: zeroed by its row pass, then summed by TMA reduce)
   int t_pad;
   float* D;          // [B][H][T]     D_i = dO_i . Y_i
   float* F_self;     // [B][H][T]     F_ii = exp(S_i - logZ_i)
   float* dS_self;    // [B][H][T]     dL/du_ii, u = U_ii (scaled evidence)
+  float* wl;         // [B][H][T]     log i F_ii (dlambda weight of row i's Exchange pairs)
   // dlambda partials: [n_pre_blocks] from the row pre-pass, then [n_main_slots] from
   // the Exchange tile kernel (one per CTA).
   float* dlam_part;
@@ -60,7 +60,7 @@ int main_ctas(const Problem& p);  // tile-kernel CTAs writing a dlambda partial
 }  // namespace simt
 
 namespace bwd_common {
-// Per-row Self part of the backward (D_i, F_ii, dS_ii and dlambda partials).
+// Per-row Self part of the CUDA-core backward (D_i, F_ii, dS_ii and dlambda partials).
 cudaError_t launch_pre(const Problem& p, const BwdWorkspace& ws, cudaStream_t s);
 // Deterministic dlambda reduction of the pre-pass partials and the first n_main tile-kernel
 // partials.
@@ -71,7 +71,7 @@ namespace tc {
 bool supports(relation_dtype dt, int d);      // forward
 bool supports_bwd(relation_dtype dt, int d);  // backward
 cudaError_t launch_fwd(const Problem& p, cudaStream_t s);
-cudaError_t launch_bwd(const Problem& p, const BwdWorkspace& ws, cudaStream_t s);
+cudaError_t launch_bwd(const Problem& p, const BwdWorkspace& ws, cudaStream_t s);  // whole bwd
 int bwd_launches();  // launches made by launch_bwd
 int main_ctas(const Problem& p);
 }  // namespace tc

@@ -122,15 +122,14 @@ relation_status relation_bwd_ex(const void* q, const void* k, const void* v, con
   Problem p = make_problem(shp, dt, lambda, tau_s, dev_status);
   p.q = q; p.k = k; p.v = v; p.o = o; p.dout = dout; p.logz_in = logz;
   p.dq = dq; p.dk = dk; p.dv = dv; p.dlambda = dlambda;
-  p.init_dq_acc = fam == 2;
   rel::BwdWorkspace ws = rel::carve_workspace(workspace, shp.B, shp.H, shp.T, shp.d_h);
   cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  if (fam == 2) return from_cuda(rel::tc::launch_bwd(p, ws, s));  // row pass, tiles, finalise
   cudaError_t e = rel::bwd_common::launch_pre(p, ws, s);
   if (e != cudaSuccess) return RELATION_ERR_CUDA;
-  e = fam == 2 ? rel::tc::launch_bwd(p, ws, s) : rel::simt::launch_bwd(p, ws, s);
+  e = rel::simt::launch_bwd(p, ws, s);
   if (e != cudaSuccess) return RELATION_ERR_CUDA;
-  const int n_main = fam == 2 ? rel::tc::main_ctas(p) : rel::simt::main_ctas(p);
-  return from_cuda(rel::bwd_common::launch_dlambda(p, ws, n_main, s));
+  return from_cuda(rel::bwd_common::launch_dlambda(p, ws, rel::simt::main_ctas(p), s));
 }
 
 relation_status relation_bwd(const void* q, const void* k, const void* v, const void* o,
@@ -162,9 +161,9 @@ int relation_launch_count(relation_dtype dt, int d_h, relation_kernel kernel, in
   const int fam = pick_family(kernel, dt, d_h, backward != 0);
   if (fam == 0) return 0;
   if (!backward) return 1;
-  // row pre-pass + Exchange tiles (SIMT: dK/dV and dQ kernels; tcgen05: tile kernel and
-  // dQ finalisation) + dlambda reduction
-  return fam == 2 ? rel::tc::bwd_launches() + 2 : 4;
+  // SIMT: row pre-pass, dK/dV kernel, dQ kernel, dlambda reduction;
+  // tcgen05: row pass, tile kernel, finalisation (dQ conversion + dlambda reduction)
+  return fam == 2 ? rel::tc::bwd_launches() : 4;
 }
 
 relation_status relation_selftest_wait_timeout(int* dev_status, int timeout_us,

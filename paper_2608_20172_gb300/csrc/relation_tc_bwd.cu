@@ -1,23 +1,32 @@
 // relation_tc_bwd.cu -- tcgen05 / TMA / TMEM backward of FlashRelation (bf16, d_h 64/128).
 //
-// Gradient (App. A.1.7, generic softmax form) for the Exchange pairs j < i:
-//   P_ij  = exp(E_ij - lambda log i - logZ_i)        (recomputed; F_ij of the flow)
-//   dP_ij = dO_i . v_j,   dR_ij = P_ij (dP_ij - D_i)
-//   dS_ij = dR_ij SiLU'(u_ij),  SiLU'(u) = sigma(u) + u sigma(u) (1 - sigma(u))
-//   dV_j += P_ij dO_i,  dK_j += dS_ij q_i / sqrt(d),  dQ_i += dS_ij k_j / sqrt(d)
-// The Self pairs (j = i), D_i and the initial value of the fp32 dQ accumulator come from
-// the row pre-pass (aux_kernels.cu); a finalisation kernel converts dQ to bf16.
+// Gradient of the causal Relation row softmax (App. A.1.7, generic form).  For every
+// pair j <= i of one head, with F the flow and G = dL/dY:
+//   dR_ij = F_ij (dO_i . v_j - D_i),   D_i = dO_i . Y_i
+//   dS_ij = dR_ij SiLU'(u_ij)                    (Exchange, j < i)
+//   dS_ii = dR_ii S_i (1 - S_i) / tau_S          (Self, j = i; S_i = sigmoid(u_ii / tau_S))
+//   dV_j += F_ij dO_i,  dK_j += dS_ij q_i / sqrt(d),  dQ_i += dS_ij k_j / sqrt(d)
+// with F_ij = exp(E_ij - lambda log i - logZ_i) (j < i) and F_ii = exp(S_i - logZ_i).
+// The Self entry is handled inside the diagonal tile with its own role map, exactly as
+// the forward treats it.
 //
-// One CTA owns a tile of 128 keys of one head and visits the query tiles from its
-// diagonal tile to the end of the sequence.  Per query tile, with keys on TMEM lanes:
-//   MMA  U^T  = K Q^T,  dP^T = V dO^T                  (TMEM, fp32)
-//   elementwise (warps 0-3, thread = key): P and dS' = 2 dS in bf16; P into TMEM,
-//        dS' into shared memory (128-byte swizzled rows of 128 queries)
-//   MMA  dV += P^T dO (P from TMEM),  dK += dS'^T Q,  dQ_i = dS' K
-//   warps 4-7 read dQ_i (queries on lanes) and add it to the fp32 accumulator.
-// Warp 8 loads tiles with TMA and stages the per-query scalars; warp 9 issues MMAs.
-// The factor 1/2 of dS' and 1/sqrt(d) are applied in the fp32 epilogues.  dL/dlambda's
-// Exchange part  -sum log i F_ii dR_ij  is accumulated per key and reduced per CTA.
+// Three launches: a row pass (D_i, the dlambda weight log i F_ii, zeroed fp32 dQ
+// accumulator), the tile kernel, and a finalisation (dQ to bf16, dlambda reduction).
+//
+// Tile kernel: one CTA per 128 keys of one head, visiting query tiles from the diagonal
+// to the end of the sequence.  Keys sit on TMEM lanes.  Per step of W query columns:
+//   MMA  U^T = K Q^T,  dP^T = V dO^T                          (TMEM, fp32)
+//   elementwise (thread = key): P = F in bf16 back into TMEM, dS' = 2 dS in bf16 into
+//        128-byte-swizzled shared memory, and the Exchange part of dlambda
+//   MMA  dV += P^T dO (P read from TMEM),  dK += dS'^T Q
+// and once per 128-query tile  MMA dQ_t = dS' K, which warps 8-11 stage through shared
+// memory and add to the fp32 accumulator with TMA reduce-add.
+//   d_h = 64 : W = 64, two TMEM buffers; elementwise warpgroup w owns buffer w, so the
+//              MMAs of one half-tile overlap the elementwise work of the other.
+//   d_h = 128: W = 128, one buffer (TMEM is full); both warpgroups split its columns and
+//              dQ_t reuses the dP^T columns.
+// dlambda = sum_i log i g_i dR_ii - sum_{j<i} log i F_ii dR_ij (weights cancel the
+// rounding error of D_i; see aux_kernels.cu), reduced per CTA.
 #include <cudaTypedefs.h>
 #include <math.h>
 
@@ -27,34 +36,43 @@
 namespace rel {
 namespace tc {
 
+bool make_tmap_bf16(CUtensorMap* m, const void* base, const Problem& p, int rows);
+
 namespace bwd {
 
-constexpr int BK = 128;         // keys per CTA
-constexpr int BQ = 128;         // queries per step
-constexpr int kThreads = 320;   // 4 elementwise + 4 dQ + TMA + MMA warps
+constexpr int BK = 128;        // keys per CTA
+constexpr int BT = 128;        // queries per TMA tile
+constexpr int kThreads = 448;  // warps 0-7 elementwise, 8-11 dQ, 12 TMA, 13 MMA
 constexpr int kTmemCols = 512;
+constexpr int W_DQ = 8, W_TMA = 12, W_MMA = 13;
 
 template <int D>
 struct Cfg {
   static constexpr int KB = D / 64;
-  static constexpr int TILE = 128 * D * 2;           // bytes of a K, V, Q or dO tile
-  static constexpr int QS = D == 64 ? 2 : 1;         // Q / dO stages
+  static constexpr int TILE = 128 * D * 2;
+  static constexpr int NBUF = D == 64 ? 2 : 1;   // U^T / dP^T TMEM buffers
+  static constexpr int QW = D == 64 ? 64 : 128;  // query columns per step
+  static constexpr int SPT = BT / QW;            // steps per query tile
+  static constexpr int QSTG = D == 64 ? 2 : 1;   // Q / dO tile stages
+  static constexpr int DSB = D == 64 ? 2 : 1;    // dS' buffers (by tile parity)
   static constexpr int OFF_K = 0;
   static constexpr int OFF_V = OFF_K + TILE;
   static constexpr int OFF_Q = OFF_V + TILE;
-  static constexpr int OFF_DO = OFF_Q + QS * TILE;
-  static constexpr int OFF_DS = OFF_DO + QS * TILE;  // 128 keys x 128 queries bf16
-  static constexpr int OFF_STAT = OFF_DS + BK * BQ * 2;
-  static constexpr int STAT_STAGE = 3 * BQ * 4;      // c2, D, w per query
-  static constexpr int OFF_RED = OFF_STAT + QS * STAT_STAGE;
+  static constexpr int OFF_DO = OFF_Q + QSTG * TILE;
+  static constexpr int OFF_DS = OFF_DO + QSTG * TILE;
+  static constexpr int OFF_DQS = OFF_DS + DSB * 32768;     // 4 warps x 2 slots x 4 KB
+  static constexpr int OFF_STAT = OFF_DQS + 4 * 2 * 4096;  // QSTG x 4 x 128 floats
+  static constexpr int OFF_RED = OFF_STAT + QSTG * 4 * BT * 4;
   static constexpr int OFF_BAR = OFF_RED + 64;
   static constexpr int SMEM = OFF_BAR + 256 + 1024;
-  static constexpr int COL_ST = 0, COL_DPT = 128, COL_DK = 256, COL_DV = 256 + D;
-  static constexpr int COL_DQ = D == 64 ? 384 : 128;  // d=128: reuses the dP^T columns
+  static constexpr int COL_DK = 256, COL_DV = 256 + D;
+  static constexpr int COL_DQ = D == 64 ? 384 : 128;       // d = 128: dP^T columns
+  __host__ __device__ static constexpr int col_u(int b) { return b * 2 * QW; }
+  __host__ __device__ static constexpr int col_g(int b) { return b * 2 * QW + QW; }
 };
 
 enum : int {
-  B_KV = 0, B_QF = 1, B_QE = 3, B_S = 5, B_P = 6, B_DQF = 7, B_DQE = 8, B_ACC = 9
+  B_KV = 0, B_QF = 1, B_QE = 3, B_S = 5, B_P = 7, B_DQF = 9, B_DQE = 10, B_ACC = 11
 };
 
 __device__ __forceinline__ void drain_wait(uint32_t bar, uint32_t parity) {
@@ -64,11 +82,74 @@ __device__ __forceinline__ void drain_wait(uint32_t bar, uint32_t parity) {
   }
 }
 
+__device__ __forceinline__ void tma_reduce_add_2d(const CUtensorMap* m, uint32_t src, int c0,
+                                                  int c1) {
+  asm volatile(
+      "cp.reduce.async.bulk.tensor.2d.global.shared::cta.add.tile.bulk_group [%0, {%2, %3}], [%1];"
+      ::"l"(reinterpret_cast<uint64_t>(m)), "r"(src), "r"(c0), "r"(c1)
+      : "memory");
+}
+__device__ __forceinline__ void bulk_wait_read_le1() {
+  asm volatile("cp.async.bulk.wait_group.read 1;" ::: "memory");
+}
+
+// Elementwise work on 32 query columns of one key row.  Writes P (bf16x2) into pk and
+// dS' = 2 dS (bf16x2) into dk; accumulates the Exchange part of dlambda.
+template <bool DIAG>
+__device__ __forceinline__ void tile_chunk(const uint32_t (&U)[32], const uint32_t (&G)[32],
+                                           const float* st, int qloc0, int t, int key_g,
+                                           float ch, float c2k, float isd, float inv_tau,
+                                           uint32_t (&pk)[16], uint32_t (&dk)[16], float& dlam) {
+#pragma unroll
+  for (int c = 0; c < 32; c += 4) {
+    const float4 c2v = *reinterpret_cast<const float4*>(st + qloc0 + c);
+    const float4 ddv = *reinterpret_cast<const float4*>(st + BT + qloc0 + c);
+    const float4 wlv = *reinterpret_cast<const float4*>(st + 2 * BT + qloc0 + c);
+    const float c2a[4] = {c2v.x, c2v.y, c2v.z, c2v.w};
+    const float dda[4] = {ddv.x, ddv.y, ddv.z, ddv.w};
+    const float wla[4] = {wlv.x, wlv.y, wlv.z, wlv.w};
+    float pv[4], sv[4];
+#pragma unroll
+    for (int e = 0; e < 4; ++e) {
+      const float x = __uint_as_float(U[c + e]);
+      const float g = __uint_as_float(G[c + e]);
+      const float hh = x * ch;                  // u / 2
+      const float th = tanh_approx(hh);         // sigma(u) = (1 + th) / 2
+      const float w = fmaf(th, c2k, c2k);
+      float P = ex2_approx(fmaf(x, w, c2a[e]));  // exp(E - lambda log i - logZ_i)
+      float dR = P * (g - dda[e]);
+      float s2 = dR * (1.0f + th + fmaf(-hh * th, th, hh));  // 2 dR SiLU'(u)
+      float dl = -wla[e] * dR;
+      if (DIAG) {
+        const int q = qloc0 + c + e;  // tile-local query index; the key is t
+        if (q < t) {                  // not history of query q
+          P = 0.f; s2 = 0.f; dl = 0.f;
+        } else if (q == t) {          // Self entry: role map sigmoid(u / tau_S)
+          const float S = 1.0f / (1.0f + __expf(-(x * isd) * inv_tau));
+          const float lzn = st[3 * BT + q];   // -logZ_i log2 e
+          P = ex2_approx(fmaf(S, kLog2e, lzn));
+          dR = P * (g - dda[e]);
+          s2 = 2.0f * dR * S * (1.0f - S) * inv_tau;
+          dl = __logf((float)(key_g + 1)) * (1.0f - P) * dR;
+        }
+      }
+      dlam += dl;
+      pv[e] = P;
+      sv[e] = s2;
+    }
+    pk[c >> 1] = pack_bf16x2(pv[0], pv[1]);
+    pk[(c >> 1) + 1] = pack_bf16x2(pv[2], pv[3]);
+    dk[c >> 1] = pack_bf16x2(sv[0], sv[1]);
+    dk[(c >> 1) + 1] = pack_bf16x2(sv[2], sv[3]);
+  }
+}
+
 template <int D>
 __global__ void __launch_bounds__(kThreads, 1)
     bwd_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmK,
                   const __grid_constant__ CUtensorMap tmV, const __grid_constant__ CUtensorMap tmG,
-                  Problem p, BwdWorkspace ws, int n_t, int t_pad) {
+                  const __grid_constant__ CUtensorMap tmDQ, Problem p, BwdWorkspace ws, int n_t,
+                  int t_pad) {
   using C = Cfg<D>;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>(
@@ -81,27 +162,28 @@ __global__ void __launch_bounds__(kThreads, 1)
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int BH = p.B * p.H;
-  const int kt = (int)(blockIdx.x / BH);  // heaviest key tiles (most query tiles) first
+  const int kt = (int)(blockIdx.x / BH);  // key tiles with the most query tiles first
   const int bh = (int)(blockIdx.x % BH);
   const int b = bh / p.H, h = bh % p.H;
   const int k0 = kt * BK;
-  const int n_i = n_t - kt;  // query tiles kt .. n_t - 1
+  const int n_i = n_t - kt;               // query tiles kt .. n_t - 1
+  const int total = n_i * C::SPT;         // steps
 
   if (threadIdx.x == 0) {
     mbar_init(bar(B_KV), 1);
-    for (int s = 0; s < C::QS; ++s) {
+    for (int s = 0; s < 2; ++s) {
       mbar_init(bar(B_QF + s), 1);
       mbar_init(bar(B_QE + s), 1);
+      mbar_init(bar(B_S + s), 1);
+      mbar_init(bar(B_P + s), C::NBUF == 2 ? 128 : 256);
     }
-    mbar_init(bar(B_S), 1);
-    mbar_init(bar(B_P), 128);
     mbar_init(bar(B_DQF), 1);
     mbar_init(bar(B_DQE), 128);
     mbar_init(bar(B_ACC), 1);
     *abort_flag = 0;
     fence_mbar_init();
   }
-  if (warp == 9) tmem_alloc(smem_u32(tmem_slot), kTmemCols);
+  if (warp == W_MMA) tmem_alloc(smem_u32(tmem_slot), kTmemCols);
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
@@ -109,8 +191,8 @@ __global__ void __launch_bounds__(kThreads, 1)
   const Abort ab{abort_flag, p.dev_status};
   const long long rows_bh = (long long)bh * p.T;
 
-  if (warp == 8) {
-    // ---------------------------------------------------------- TMA + per-query scalars
+  if (warp == W_TMA) {
+    // ------------------------------------------------------ TMA + per-query scalars
     if (lane == 0) {
       tma_prefetch_desc(&tmQ);
       tma_prefetch_desc(&tmK);
@@ -118,269 +200,250 @@ __global__ void __launch_bounds__(kThreads, 1)
       tma_prefetch_desc(&tmG);
       mbar_arrive_expect_tx(bar(B_KV), 2 * C::TILE);
       for (int kb = 0; kb < C::KB; ++kb) {
-        tma_load_4d(sb + C::OFF_K + kb * 128 * 128, &tmK, bar(B_KV), kb * 64, k0, h, b);
-        tma_load_4d(sb + C::OFF_V + kb * 128 * 128, &tmV, bar(B_KV), kb * 64, k0, h, b);
+        tma_load_4d(sb + C::OFF_K + kb * 16384, &tmK, bar(B_KV), kb * 64, k0, h, b);
+        tma_load_4d(sb + C::OFF_V + kb * 16384, &tmV, bar(B_KV), kb * 64, k0, h, b);
       }
     }
     int issued = 0;
     for (int i = 0; i < n_i; ++i) {
-      const int s = i % C::QS, u = i / C::QS;
+      const int s = i % C::QSTG, u = i / C::QSTG;
       bool ok = true;
       if (u > 0) ok = mbar_wait(bar(B_QE + s), (u - 1) & 1, ab);
       ok = __all_sync(0xffffffffu, ok);
       if (!ok) break;
-      const int qi0 = (kt + i) * BQ;
-      float* st = reinterpret_cast<float*>(smem + C::OFF_STAT + s * C::STAT_STAGE);
-      for (int q = lane; q < BQ; q += 32) {
+      const int qi0 = (kt + i) * BT;
+      float* st = reinterpret_cast<float*>(smem + C::OFF_STAT + s * 4 * BT * 4);
+      for (int q = lane; q < BT; q += 32) {
         const int row = qi0 + q;
-        float c2 = -INFINITY, dd = 0.f, wl = 0.f;
+        float c2 = -INFINITY, dd = 0.f, wl = 0.f, lzn = -INFINITY;
         if (row < p.T) {
-          const float li = __logf((float)(row + 1));
-          c2 = (-p.lambda * li - p.logz_in[rows_bh + row]) * kLog2e;
+          const float lz = p.logz_in[rows_bh + row];
+          c2 = (-p.lambda * __logf((float)(row + 1)) - lz) * kLog2e;
           dd = ws.D[rows_bh + row];
-          wl = li * ws.F_self[rows_bh + row];
+          wl = ws.wl[rows_bh + row];
+          lzn = -lz * kLog2e;
         }
         st[q] = c2;
-        st[BQ + q] = dd;
-        st[2 * BQ + q] = wl;
+        st[BT + q] = dd;
+        st[2 * BT + q] = wl;
+        st[3 * BT + q] = lzn;
       }
       __threadfence_block();
       __syncwarp();
       if (lane == 0) {
         mbar_arrive_expect_tx(bar(B_QF + s), 2 * C::TILE);
         for (int kb = 0; kb < C::KB; ++kb) {
-          tma_load_4d(sb + C::OFF_Q + s * C::TILE + kb * 128 * 128, &tmQ, bar(B_QF + s),
-                      kb * 64, qi0, h, b);
-          tma_load_4d(sb + C::OFF_DO + s * C::TILE + kb * 128 * 128, &tmG, bar(B_QF + s),
-                      kb * 64, qi0, h, b);
+          tma_load_4d(sb + C::OFF_Q + s * C::TILE + kb * 16384, &tmQ, bar(B_QF + s), kb * 64,
+                      qi0, h, b);
+          tma_load_4d(sb + C::OFF_DO + s * C::TILE + kb * 16384, &tmG, bar(B_QF + s), kb * 64,
+                      qi0, h, b);
         }
       }
       issued = i + 1;
     }
     if (lane == 0 && ab.raised()) {
       drain_wait(bar(B_KV), 0);
-      for (int i = issued - C::QS > 0 ? issued - C::QS : 0; i < issued; ++i)
-        drain_wait(bar(B_QF + i % C::QS), (i / C::QS) & 1);
+      for (int i = issued - C::QSTG > 0 ? issued - C::QSTG : 0; i < issued; ++i)
+        drain_wait(bar(B_QF + i % C::QSTG), (i / C::QSTG) & 1);
     }
-  } else if (warp == 9) {
-    // ---------------------------------------------------------- MMA issuer
+  } else if (warp == W_MMA) {
+    // ------------------------------------------------------ MMA issuer
     if (lane == 0) {
-      constexpr uint32_t id_qk = idesc_bf16_f32(128, 128, false, false);  // U^T, dP^T
-      constexpr uint32_t id_acc = idesc_bf16_f32(128, D, false, true);    // dV, dK
-      constexpr uint32_t id_dq = idesc_bf16_f32(128, D, true, true);      // dQ
-      auto issue_scores = [&](int s) {
+      constexpr uint32_t id_s = idesc_bf16_f32(128, C::QW, false, false);  // U^T, dP^T
+      constexpr uint32_t id_acc = idesc_bf16_f32(128, D, false, true);     // dV, dK
+      constexpr uint32_t id_dq = idesc_bf16_f32(128, D, true, true);       // dQ
+      bool ok = mbar_wait(bar(B_KV), 0, ab);
+      // U^T and dP^T of step s into buffer s % NBUF
+      auto issue_sdp = [&](int s) -> bool {
+        const int t = s / C::SPT, hh = s % C::SPT, bb = s % C::NBUF, st = t % C::QSTG;
+        if (hh == 0) {
+          if (!mbar_wait(bar(B_QF + st), (t / C::QSTG) & 1, ab)) return false;
+          tc_fence_after();
+        }
+        const uint32_t qoff = hh * C::QW * 128;
 #pragma unroll
         for (int kk = 0; kk < D / 16; ++kk) {
-          const uint32_t koff = (kk >> 2) * (128 * 128) + (kk & 3) * 32;
-          mma_ss(tmem + C::COL_ST, smem_desc_sw128(sb + C::OFF_K + koff, 16, 1024),
-                 smem_desc_sw128(sb + C::OFF_Q + s * C::TILE + koff, 16, 1024), id_qk,
+          const uint32_t koff = (kk >> 2) * 16384 + (kk & 3) * 32;
+          mma_ss(tmem + C::col_u(bb), smem_desc_sw128(sb + C::OFF_K + koff, 16, 1024),
+                 smem_desc_sw128(sb + C::OFF_Q + st * C::TILE + qoff + koff, 16, 1024), id_s,
                  kk > 0 ? 1u : 0u);
         }
-      };
-      auto issue_dp = [&](int s) {
+        if (D == 128 && t > 0) {  // dP^T overwrites dQ_{t-1}: wait until it was read
+          if (!mbar_wait(bar(B_DQE), (t - 1) & 1, ab)) return false;
+          tc_fence_after();
+        }
 #pragma unroll
         for (int kk = 0; kk < D / 16; ++kk) {
-          const uint32_t koff = (kk >> 2) * (128 * 128) + (kk & 3) * 32;
-          mma_ss(tmem + C::COL_DPT, smem_desc_sw128(sb + C::OFF_V + koff, 16, 1024),
-                 smem_desc_sw128(sb + C::OFF_DO + s * C::TILE + koff, 16, 1024), id_qk,
+          const uint32_t koff = (kk >> 2) * 16384 + (kk & 3) * 32;
+          mma_ss(tmem + C::col_g(bb), smem_desc_sw128(sb + C::OFF_V + koff, 16, 1024),
+                 smem_desc_sw128(sb + C::OFF_DO + st * C::TILE + qoff + koff, 16, 1024), id_s,
                  kk > 0 ? 1u : 0u);
         }
+        mma_commit(bar(B_S + bb));
+        return true;
       };
-      bool ok = mbar_wait(bar(B_KV), 0, ab) && mbar_wait(bar(B_QF), 0, ab);
-      tc_fence_after();
-      if (ok) {
-        issue_scores(0);
-        issue_dp(0);
-        mma_commit(bar(B_S));
-      }
-      for (int i = 0; ok && i < n_i; ++i) {
-        const int s = i % C::QS;
-        if (!(ok = mbar_wait(bar(B_P), i & 1, ab))) break;
+      for (int s = 0; ok && s < C::NBUF && s < total; ++s) ok = issue_sdp(s);
+      for (int s = 0; ok && s < total; ++s) {
+        const int t = s / C::SPT, hh = s % C::SPT, bb = s % C::NBUF;
+        const int st = t % C::QSTG, dsb = t % C::DSB;
+        if (!(ok = mbar_wait(bar(B_P + bb), (s / C::NBUF) & 1, ab))) break;
         tc_fence_after();
-        const uint32_t acc0 = i > 0 ? 1u : 0u;
-        // dV += P^T dO_i   (A = P^T from TMEM; B = dO tile, N = d contiguous)
+        const uint32_t ds_base = sb + C::OFF_DS + dsb * 32768;
+        // dV += P^T dO   (P from TMEM, packed two per column)
 #pragma unroll
-        for (int kk = 0; kk < BQ / 16; ++kk)
-          mma_ts(tmem + C::COL_DV, tmem + C::COL_ST + kk * 8,
-                 smem_desc_sw128(sb + C::OFF_DO + s * C::TILE + kk * 2048, 128 * 128, 1024),
-                 id_acc, (acc0 | (kk > 0)) ? 1u : 0u);
-        // dK += dS'^T Q_i   (A = dS'^T: keys x queries, queries contiguous)
-#pragma unroll
-        for (int kk = 0; kk < BQ / 16; ++kk)
-          mma_ss(tmem + C::COL_DK,
-                 smem_desc_sw128(sb + C::OFF_DS + (kk >> 2) * 16384 + (kk & 3) * 32, 16, 1024),
-                 smem_desc_sw128(sb + C::OFF_Q + s * C::TILE + kk * 2048, 128 * 128, 1024),
-                 id_acc, (acc0 | (kk > 0)) ? 1u : 0u);
-        if (D == 64 && i > 0) {
-          if (!(ok = mbar_wait(bar(B_DQE), (i - 1) & 1, ab))) break;
-          tc_fence_after();
+        for (int kk = 0; kk < C::QW / 16; ++kk) {
+          const int q = hh * C::QW + kk * 16;
+          mma_ts(tmem + C::COL_DV, tmem + C::col_u(bb) + (kk >> 2) * 64 + (kk & 3) * 8,
+                 smem_desc_sw128(sb + C::OFF_DO + st * C::TILE + q * 128, 16384, 1024), id_acc,
+                 (s > 0 || kk > 0) ? 1u : 0u);
         }
-        // dQ_i = dS' K   (A = dS': queries x keys, queries contiguous; B = K tile)
+        // dK += dS'^T Q   (A = dS'^T, queries contiguous: K-major)
 #pragma unroll
-        for (int kk = 0; kk < BK / 16; ++kk)
-          mma_ss(tmem + C::COL_DQ, smem_desc_sw128(sb + C::OFF_DS + kk * 2048, 16384, 1024),
-                 smem_desc_sw128(sb + C::OFF_K + kk * 2048, 128 * 128, 1024), id_dq,
-                 kk > 0 ? 1u : 0u);
-        mma_commit(bar(B_DQF));
-        mma_commit(bar(B_QE + s));
-        if (i + 1 < n_i) {
-          const int s1 = (i + 1) % C::QS, u1 = (i + 1) / C::QS;
-          if (!(ok = mbar_wait(bar(B_QF + s1), u1 & 1, ab))) break;
-          tc_fence_after();
-          issue_scores(s1);
-          if (D == 128) {
-            if (!(ok = mbar_wait(bar(B_DQE), i & 1, ab))) break;
+        for (int kk = 0; kk < C::QW / 16; ++kk) {
+          const int q = hh * C::QW + kk * 16;
+          mma_ss(tmem + C::COL_DK,
+                 smem_desc_sw128(ds_base + (q >> 6) * 16384 + ((q & 63) >> 4) * 32, 16, 1024),
+                 smem_desc_sw128(sb + C::OFF_Q + st * C::TILE + q * 128, 16384, 1024), id_acc,
+                 (s > 0 || kk > 0) ? 1u : 0u);
+        }
+        if (hh == C::SPT - 1) {
+          if (D == 64 && t > 0) {
+            if (!(ok = mbar_wait(bar(B_DQE), (t - 1) & 1, ab))) break;
             tc_fence_after();
           }
-          issue_dp(s1);
-          mma_commit(bar(B_S));
+          // dQ_t = dS' K   (A = dS', queries x keys, M-major; B = K tile, N-major)
+#pragma unroll
+          for (int kk = 0; kk < BK / 16; ++kk)
+            mma_ss(tmem + C::COL_DQ, smem_desc_sw128(ds_base + kk * 2048, 16384, 1024),
+                   smem_desc_sw128(sb + C::OFF_K + kk * 2048, 16384, 1024), id_dq,
+                   kk > 0 ? 1u : 0u);
+          mma_commit(bar(B_DQF));
+          mma_commit(bar(B_QE + st));
         }
+        if (s + C::NBUF < total && !(ok = issue_sdp(s + C::NBUF))) break;
       }
       mma_commit(bar(B_ACC));
     }
     __syncwarp();
-  } else if (warp >= 4) {
-    // ---------------------------------------------------------- dQ_i -> fp32 accumulator
-    const int q = (warp - 4) * 32 + lane;
-    const uint32_t trow = tmem + ((uint32_t)((warp - 4) * 32) << 16);
+  } else if (warp >= W_DQ) {
+    // ------------------------------------------------------ dQ_t -> fp32 accumulator
+    const int quad = warp & 3;
+    const uint32_t trow = tmem + ((uint32_t)(quad * 32) << 16);
+    const uint32_t stage0 = sb + C::OFF_DQS + quad * 8192;
+    uint8_t* stage0p = smem + C::OFF_DQS + quad * 8192;
+    int chunk = 0;
     for (int i = 0; i < n_i; ++i) {
       const bool ok = __all_sync(0xffffffffu, mbar_wait(bar(B_DQF), i & 1, ab));
       if (!ok) break;
       tc_fence_after();
-      const int row = (kt + i) * BQ + q;
-      float* dst = ws.dq_acc + ((long long)bh * t_pad + row) * D;
+      const int row0 = bh * t_pad + (kt + i) * BT + quad * 32;
 #pragma unroll
-      for (int c0 = 0; c0 < D; c0 += 32) {
-        uint32_t z[32];
-        tmem_ld32(trow + C::COL_DQ + c0, z);
+      for (int c64 = 0; c64 < D; c64 += 64) {
+        uint32_t z[64];
+        tmem_ld32(trow + C::COL_DQ + c64, z);
+        tmem_ld32(trow + C::COL_DQ + c64 + 32, z + 32);
         tmem_ld_wait();
-        if (row < p.T) {
+        if (c64 + 64 == D) {
+          tc_fence_before();
+          mbar_arrive(bar(B_DQE));  // TMEM columns free for the next dQ / dP^T
+        }
 #pragma unroll
-          for (int c = 0; c < 32; c += 4)
-            atomicAdd(reinterpret_cast<float4*>(dst + c0 + c),
-                      make_float4(__uint_as_float(z[c]), __uint_as_float(z[c + 1]),
-                                  __uint_as_float(z[c + 2]), __uint_as_float(z[c + 3])));
+        for (int c0 = 0; c0 < 64; c0 += 32, ++chunk) {
+          const int slot = chunk & 1;
+          if (lane == 0) bulk_wait_read_le1();  // the slot's previous reduce has read it
+          __syncwarp();
+          uint8_t* row = stage0p + slot * 4096 + lane * 128;
+#pragma unroll
+          for (int k = 0; k < 8; ++k)
+            *reinterpret_cast<uint4*>(row + ((k ^ (lane & 7)) << 4)) =
+                make_uint4(z[c0 + 4 * k], z[c0 + 4 * k + 1], z[c0 + 4 * k + 2], z[c0 + 4 * k + 3]);
+          fence_async_smem();
+          __syncwarp();
+          if (lane == 0) {
+            tma_reduce_add_2d(&tmDQ, stage0 + slot * 4096, c64 + c0, row0);
+            tma_store_commit();
+          }
         }
       }
-      tc_fence_before();
-      mbar_arrive(bar(B_DQE));
     }
+    if (lane == 0) tma_store_wait_all();
   } else {
-    // ---------------------------------------------------------- elementwise + epilogue
-    const int t = threadIdx.x;  // key k0 + t, TMEM lane t
-    const uint32_t trow = tmem + ((uint32_t)(warp * 32) << 16);
+    // ------------------------------------------------------ elementwise + epilogue
+    const int wg = warp >> 2;                  // 0 or 1
+    const int t = (warp & 3) * 32 + lane;      // key k0 + t, TMEM lane t
+    const uint32_t trow = tmem + ((uint32_t)((warp & 3) * 32) << 16);
     const float isd = p.inv_sqrt_d;
-    const float ch = 0.5f * isd;   // h = U ch = u / 2
-    const float c2k = ch * kLog2e; // E log2 e = U c2k (1 + tanh h)
-    uint8_t* ds_row = smem + C::OFF_DS + t * 128;
-    const int sw = t & 7;
+    const float ch = 0.5f * isd;
+    const float c2k = ch * kLog2e;
+    const float inv_tau = 1.0f / p.tau_s;
+    const int key_g = k0 + t;
     float dlam = 0.f;
     bool ok = true;
+    const int bb = C::NBUF == 2 ? wg : 0;
+    const uint32_t col_u = C::col_u(bb) + (C::NBUF == 2 ? 0 : wg * 64);
+    const uint32_t col_g = C::col_g(bb) + (C::NBUF == 2 ? 0 : wg * 64);
+    const int qbase = wg * 64;                 // tile-local query columns of this warpgroup
     for (int i = 0; i < n_i; ++i) {
-      const int s = i % C::QS;
-      ok = __all_sync(0xffffffffu, mbar_wait(bar(B_S), i & 1, ab));
+      ok = __all_sync(0xffffffffu, mbar_wait(bar(B_S + bb), i & 1, ab));
       if (!ok) break;
       tc_fence_after();
-      const float* st = reinterpret_cast<const float*>(smem + C::OFF_STAT + s * C::STAT_STAGE);
-      const bool diag = (i == 0);
-#pragma unroll 1
-      for (int c0 = 0; c0 < BQ; c0 += 32) {
+      // acquire the producer's per-query scalars of this tile (already complete)
+      ok = __all_sync(0xffffffffu, mbar_wait(bar(B_QF + i % C::QSTG), (i / C::QSTG) & 1, ab));
+      if (!ok) break;
+      const float* st =
+          reinterpret_cast<const float*>(smem + C::OFF_STAT + (i % C::QSTG) * 4 * BT * 4);
+      uint8_t* ds_row = smem + C::OFF_DS + (i % C::DSB) * 32768 + wg * 16384 + t * 128;
+#pragma unroll
+      for (int c0 = 0; c0 < 64; c0 += 32) {
         uint32_t U[32], G[32];
-        tmem_ld32(trow + C::COL_ST + c0, U);
-        tmem_ld32(trow + C::COL_DPT + c0, G);
+        tmem_ld32(trow + col_u + c0, U);
+        tmem_ld32(trow + col_g + c0, G);
         tmem_ld_wait();
         uint32_t pk[16], dk[16];
+        if (i == 0)
+          tile_chunk<true>(U, G, st, qbase + c0, t, key_g, ch, c2k, isd, inv_tau, pk, dk, dlam);
+        else
+          tile_chunk<false>(U, G, st, qbase + c0, t, key_g, ch, c2k, isd, inv_tau, pk, dk, dlam);
+        tmem_st16(trow + col_u + (c0 >> 1), pk);
+        const int cb = c0 >> 3;  // first 16-byte chunk of these 32 queries in the row
 #pragma unroll
-        for (int c = 0; c < 32; c += 4) {
-          const float4 c2v = *reinterpret_cast<const float4*>(st + c0 + c);
-          const float4 ddv = *reinterpret_cast<const float4*>(st + BQ + c0 + c);
-          const float4 wlv = *reinterpret_cast<const float4*>(st + 2 * BQ + c0 + c);
-          const float c2a[4] = {c2v.x, c2v.y, c2v.z, c2v.w};
-          const float dda[4] = {ddv.x, ddv.y, ddv.z, ddv.w};
-          const float wla[4] = {wlv.x, wlv.y, wlv.z, wlv.w};
-          float pv[4], dv[4];
-#pragma unroll
-          for (int e = 0; e < 4; ++e) {
-            const int col = c0 + c + e;
-            const float x = __uint_as_float(U[c + e]);
-            const float hh = x * ch;
-            const float th = tanh_approx(hh);
-            const float w = fmaf(th, c2k, c2k);
-            float P = ex2_approx(fmaf(x, w, c2a[e]));
-            if (diag && col <= t) P = 0.f;  // history only: query > key
-            const float dR = P * (__uint_as_float(G[c + e]) - dda[e]);
-            // 2 SiLU'(u) = 1 + t + h (1 - t^2) with t = tanh(u/2), h = u/2
-            const float sp = 1.0f + th + fmaf(-hh * th, th, hh);
-            dlam = fmaf(-wla[e], dR, dlam);
-            pv[e] = P;
-            dv[e] = dR * sp;
-          }
-          pk[c >> 1] = pack_bf16x2(pv[0], pv[1]);
-          pk[(c >> 1) + 1] = pack_bf16x2(pv[2], pv[3]);
-          dk[c >> 1] = pack_bf16x2(dv[0], dv[1]);
-          dk[(c >> 1) + 1] = pack_bf16x2(dv[2], dv[3]);
-        }
-        tmem_st16(trow + C::COL_ST + (c0 >> 1), pk);
-        // dS' row t, queries c0..c0+31: 4 chunks of 16 bytes in the 128-byte swizzle
-        const int atom = c0 >> 6, cb = (c0 & 63) >> 3;
-#pragma unroll
-        for (int qd = 0; qd < 4; ++qd) {
-          const int phys = (cb + qd) ^ sw;
-          *reinterpret_cast<uint4*>(ds_row + atom * 16384 + phys * 16) =
+        for (int qd = 0; qd < 4; ++qd)
+          *reinterpret_cast<uint4*>(ds_row + (((cb + qd) ^ (t & 7)) << 4)) =
               make_uint4(dk[4 * qd], dk[4 * qd + 1], dk[4 * qd + 2], dk[4 * qd + 3]);
-        }
       }
       tmem_st_wait();
       fence_async_smem();
       tc_fence_before();
-      mbar_arrive(bar(B_P));
+      mbar_arrive(bar(B_P + bb));
     }
-    // ------------------------------------------------------------ dK, dV epilogue
+    // ---------------------------------------------------- dK (warpgroup 0) / dV (1)
     if (ok) ok = __all_sync(0xffffffffu, mbar_wait(bar(B_ACC), 0, ab));
     tc_fence_after();
     if (ok) {
-      const int j = k0 + t;
+      const int j = key_g;
       const long long off = (long long)b * p.sB + (long long)h * p.sH + (long long)j * p.sT;
-      const __nv_bfloat16* qrow = reinterpret_cast<const __nv_bfloat16*>(p.q) + off;
-      const __nv_bfloat16* grow = reinterpret_cast<const __nv_bfloat16*>(p.dout) + off;
-      __nv_bfloat16* dkrow = reinterpret_cast<__nv_bfloat16*>(p.dk) + off;
-      __nv_bfloat16* dvrow = reinterpret_cast<__nv_bfloat16*>(p.dv) + off;
       const bool valid = j < p.T;
-      const float fs = valid ? ws.F_self[rows_bh + j] : 0.f;
-      const float dss = valid ? ws.dS_self[rows_bh + j] : 0.f;
-#pragma unroll 1
+      const uint32_t col = wg == 0 ? C::COL_DK : C::COL_DV;
+      __nv_bfloat16* dst = reinterpret_cast<__nv_bfloat16*>(wg == 0 ? p.dk : p.dv) + off;
+      const float sc = wg == 0 ? 0.5f * isd : 1.0f;
+#pragma unroll
       for (int c0 = 0; c0 < D; c0 += 32) {
-        uint32_t ak[32], av[32];
-        tmem_ld32(trow + C::COL_DK + c0, ak);
-        tmem_ld32(trow + C::COL_DV + c0, av);
+        uint32_t a[32];
+        tmem_ld32(trow + col + c0, a);
         tmem_ld_wait();
         if (valid) {
 #pragma unroll
           for (int c8 = 0; c8 < 32; c8 += 8) {
-            const uint4 qv = *reinterpret_cast<const uint4*>(qrow + c0 + c8);
-            const uint4 gv = *reinterpret_cast<const uint4*>(grow + c0 + c8);
-            const uint32_t qw[4] = {qv.x, qv.y, qv.z, qv.w};
-            const uint32_t gw[4] = {gv.x, gv.y, gv.z, gv.w};
-            uint32_t ok4[4], ov4[4];
+            uint32_t o4[4];
 #pragma unroll
-            for (int e = 0; e < 4; ++e) {
-              const float2 qf = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&qw[e]));
-              const float2 gf = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&gw[e]));
-              const int c = c8 + 2 * e;
-              const float k0f = fmaf(0.5f, __uint_as_float(ak[c]), dss * qf.x) * isd;
-              const float k1f = fmaf(0.5f, __uint_as_float(ak[c + 1]), dss * qf.y) * isd;
-              const float v0f = fmaf(fs, gf.x, __uint_as_float(av[c]));
-              const float v1f = fmaf(fs, gf.y, __uint_as_float(av[c + 1]));
-              ok4[e] = pack_bf16x2(k0f, k1f);
-              ov4[e] = pack_bf16x2(v0f, v1f);
-            }
-            *reinterpret_cast<uint4*>(dkrow + c0 + c8) = make_uint4(ok4[0], ok4[1], ok4[2], ok4[3]);
-            *reinterpret_cast<uint4*>(dvrow + c0 + c8) = make_uint4(ov4[0], ov4[1], ov4[2], ov4[3]);
+            for (int e = 0; e < 4; ++e)
+              o4[e] = pack_bf16x2(__uint_as_float(a[c8 + 2 * e]) * sc,
+                                  __uint_as_float(a[c8 + 2 * e + 1]) * sc);
+            *reinterpret_cast<uint4*>(dst + c0 + c8) = make_uint4(o4[0], o4[1], o4[2], o4[3]);
           }
         }
       }
     }
-    // per-warp dlambda partial
 #pragma unroll
     for (int o = 16; o > 0; o >>= 1) dlam += __shfl_xor_sync(0xffffffffu, dlam, o);
     if (lane == 0) red[warp] = dlam;
@@ -388,27 +451,94 @@ __global__ void __launch_bounds__(kThreads, 1)
 
   tc_fence_before();
   __syncthreads();
-  if (threadIdx.x == 0)
-    ws.dlam_part[ws.n_pre_blocks + blockIdx.x] = (red[0] + red[1]) + (red[2] + red[3]);
-  if (warp == 9) {
+  if (threadIdx.x == 0) {
+    float s = 0.f;
+#pragma unroll
+    for (int w = 0; w < 8; ++w) s += red[w];
+    ws.dlam_part[ws.n_pre_blocks + blockIdx.x] = s;
+  }
+  if (warp == W_MMA) {
     tc_fence_after();
     tmem_dealloc(tmem, kTmemCols);
   }
 }
 
-// dq = bf16(dq_acc / (2 sqrt(d))) for rows < T  (dq_acc holds 2 x the unscaled sum)
+// Row pass: D_i = dO_i . Y_i, wl_i = log i F_ii with F_ii = exp(sigmoid(u_ii / tau_S) -
+// logZ_i), and a zeroed row of the fp32 dQ accumulator.  8 threads per row.
 template <int D>
-__global__ void __launch_bounds__(256) dq_finalize_kernel(Problem p, const float* dq_acc,
-                                                          int t_pad) {
-  const long long idx = (long long)blockIdx.x * blockDim.x + threadIdx.x;  // 8-wide chunk
+__global__ void __launch_bounds__(256) pre_kernel(Problem p, BwdWorkspace ws) {
+  constexpr int PER = D / 8;  // elements per thread
+  const long long gr = ((long long)blockIdx.x * 256 + threadIdx.x) >> 3;
+  const int sub = threadIdx.x & 7;
+  const long long nrows = (long long)p.B * p.H * p.T;
+  const bool live = gr < nrows;
+  const long long grc = live ? gr : 0;
+  const int bh = (int)(grc / p.T), r = (int)(grc % p.T);
+  const int b = bh / p.H, h = bh % p.H;
+  const long long off = (long long)b * p.sB + (long long)h * p.sH + (long long)r * p.sT + sub * PER;
+  float gy = 0.f, qk = 0.f;
+  if (live) {
+#pragma unroll
+    for (int c = 0; c < PER; c += 8) {
+      const uint4 gv = *reinterpret_cast<const uint4*>(reinterpret_cast<const __nv_bfloat16*>(p.dout) + off + c);
+      const uint4 ov = *reinterpret_cast<const uint4*>(reinterpret_cast<const __nv_bfloat16*>(p.o) + off + c);
+      const uint4 qv = *reinterpret_cast<const uint4*>(reinterpret_cast<const __nv_bfloat16*>(p.q) + off + c);
+      const uint4 kv = *reinterpret_cast<const uint4*>(reinterpret_cast<const __nv_bfloat16*>(p.k) + off + c);
+      const uint32_t g4[4] = {gv.x, gv.y, gv.z, gv.w}, o4[4] = {ov.x, ov.y, ov.z, ov.w};
+      const uint32_t q4[4] = {qv.x, qv.y, qv.z, qv.w}, k4[4] = {kv.x, kv.y, kv.z, kv.w};
+#pragma unroll
+      for (int e = 0; e < 4; ++e) {
+        const float2 gf = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&g4[e]));
+        const float2 of = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&o4[e]));
+        const float2 qf = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&q4[e]));
+        const float2 kf = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&k4[e]));
+        gy = fmaf(gf.x, of.x, fmaf(gf.y, of.y, gy));
+        qk = fmaf(qf.x, kf.x, fmaf(qf.y, kf.y, qk));
+      }
+    }
+  }
+#pragma unroll
+  for (int o = 4; o > 0; o >>= 1) {
+    gy += __shfl_xor_sync(0xffffffffu, gy, o);
+    qk += __shfl_xor_sync(0xffffffffu, qk, o);
+  }
+  if (!live) return;
+  if (sub == 0) {
+    const float S = 1.0f / (1.0f + expf(-(qk * p.inv_sqrt_d) / p.tau_s));
+    const float F = expf(S - p.logz_in[gr]);
+    ws.D[gr] = gy;
+    ws.wl[gr] = logf((float)(r + 1)) * F;
+  }
+  float* acc = ws.dq_acc + ((long long)bh * ws.t_pad + r) * D + sub * PER;
+#pragma unroll
+  for (int c = 0; c < PER; c += 4) *reinterpret_cast<float4*>(acc + c) = make_float4(0.f, 0.f, 0.f, 0.f);
+}
+
+// dq = bf16(dq_acc / (2 sqrt(d))) for rows < T; block 0 also reduces the tile kernel's
+// dlambda partials in a fixed order (deterministic).
+template <int D>
+__global__ void __launch_bounds__(256) finalize_kernel(Problem p, BwdWorkspace ws, int n_cta) {
+  if (blockIdx.x == 0) {
+    __shared__ double part[256];
+    double s = 0.0;
+    for (int i = threadIdx.x; i < n_cta; i += 256) s += (double)ws.dlam_part[ws.n_pre_blocks + i];
+    part[threadIdx.x] = s;
+    __syncthreads();
+    for (int w = 128; w > 0; w >>= 1) {
+      if (threadIdx.x < w) part[threadIdx.x] += part[threadIdx.x + w];
+      __syncthreads();
+    }
+    if (threadIdx.x == 0) *p.dlambda = (float)part[0];
+  }
+  const long long idx = ((long long)blockIdx.x * 256 + threadIdx.x);  // 8-wide chunk
   const long long per_row = D / 8;
   const long long n = (long long)p.B * p.H * p.T * per_row;
   if (idx >= n) return;
   const int c8 = (int)(idx % per_row) * 8;
-  const long long row = idx / per_row;  // over B*H*T
+  const long long row = idx / per_row;
   const int bh = (int)(row / p.T), r = (int)(row % p.T);
   const int b = bh / p.H, h = bh % p.H;
-  const float* src = dq_acc + ((long long)bh * t_pad + r) * D + c8;
+  const float* src = ws.dq_acc + ((long long)bh * ws.t_pad + r) * D + c8;
   const float4 a = *reinterpret_cast<const float4*>(src);
   const float4 c = *reinterpret_cast<const float4*>(src + 4);
   const float sc = 0.5f * p.inv_sqrt_d;
@@ -424,27 +554,52 @@ __global__ void __launch_bounds__(256) dq_finalize_kernel(Problem p, const float
 
 }  // namespace bwd
 
-bool make_tmap_bf16(CUtensorMap* m, const void* base, const Problem& p, int rows);
+// 2-D map over the fp32 dQ accumulator [B*H*t_pad][D]: box 32 x 32, 128-byte swizzle.
+static bool make_tmap_dq(CUtensorMap* m, float* base, int rows, int d) {
+  static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
+  if (!fn) {
+    void* ptr = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &ptr, 12000, cudaEnableDefault,
+                                         &q) != cudaSuccess ||
+        q != cudaDriverEntryPointSuccess)
+      return false;
+    fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(ptr);
+  }
+  cuuint64_t dims[2] = {(cuuint64_t)d, (cuuint64_t)rows};
+  cuuint64_t strides[1] = {(cuuint64_t)d * 4};
+  cuuint32_t box[2] = {32, 32};
+  cuuint32_t estr[2] = {1, 1};
+  return fn(m, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 2, base, dims, strides, box, estr,
+            CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+            CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
 
 template <int D>
 static cudaError_t bwd_t(const Problem& p, const BwdWorkspace& ws, cudaStream_t s) {
-  CUtensorMap mq, mk, mv, mg;
-  if (!make_tmap_bf16(&mq, p.q, p, 128) || !make_tmap_bf16(&mk, p.k, p, 128) ||
-      !make_tmap_bf16(&mv, p.v, p, 128) || !make_tmap_bf16(&mg, p.dout, p, 128))
-    return cudaErrorInvalidValue;
-  const int smem = bwd::Cfg<D>::SMEM;
-  cudaError_t e = cudaFuncSetAttribute(bwd::bwd_tc_kernel<D>,
-                                       cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
-  if (e != cudaSuccess) return e;
   const int n_t = (p.T + 127) / 128;
-  const int t_pad = n_t * 128;
+  const int t_pad = ws.t_pad;
+  CUtensorMap mq, mk, mv, mg, mdq;
+  if (!make_tmap_bf16(&mq, p.q, p, 128) || !make_tmap_bf16(&mk, p.k, p, 128) ||
+      !make_tmap_bf16(&mv, p.v, p, 128) || !make_tmap_bf16(&mg, p.dout, p, 128) ||
+      !make_tmap_dq(&mdq, ws.dq_acc, p.B * p.H * t_pad, D))
+    return cudaErrorInvalidValue;
+  const long long rows = (long long)p.B * p.H * p.T;
+  bwd::pre_kernel<D><<<(unsigned)((rows * 8 + 255) / 256), 256, 0, s>>>(p, ws);
+  cudaError_t e = cudaGetLastError();
+  if (e != cudaSuccess) return e;
+  const int smem = bwd::Cfg<D>::SMEM;
+  e = cudaFuncSetAttribute(bwd::bwd_tc_kernel<D>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                           smem);
+  if (e != cudaSuccess) return e;
   const long long grid = (long long)n_t * p.B * p.H;
   if (grid > 0x7fffffffLL) return cudaErrorInvalidConfiguration;
-  bwd::bwd_tc_kernel<D><<<(unsigned)grid, bwd::kThreads, smem, s>>>(mq, mk, mv, mg, p, ws, n_t,
-                                                                   t_pad);
+  bwd::bwd_tc_kernel<D><<<(unsigned)grid, bwd::kThreads, smem, s>>>(mq, mk, mv, mg, mdq, p, ws,
+                                                                   n_t, t_pad);
   if ((e = cudaGetLastError()) != cudaSuccess) return e;
-  const long long chunks = (long long)p.B * p.H * p.T * (D / 8);
-  bwd::dq_finalize_kernel<D><<<(unsigned)((chunks + 255) / 256), 256, 0, s>>>(p, ws.dq_acc, t_pad);
+  const long long chunks = rows * (D / 8);
+  const long long fblocks = (chunks + 255) / 256;
+  bwd::finalize_kernel<D><<<(unsigned)(fblocks > 0 ? fblocks : 1), 256, 0, s>>>(p, ws, (int)grid);
   return cudaGetLastError();
 }
 
@@ -455,7 +610,7 @@ cudaError_t launch_bwd(const Problem& p, const BwdWorkspace& ws, cudaStream_t s)
   if (p.d == 128) return bwd_t<128>(p, ws, s);
   return cudaErrorInvalidValue;
 }
-int bwd_launches() { return 2; }
+int bwd_launches() { return 3; }
 int main_ctas(const Problem& p) { return ((p.T + 127) / 128) * p.B * p.H; }
 
 }  // namespace tc
