@@ -133,6 +133,10 @@ int relation_launch_count(relation_dtype dt, int d_h, relation_kernel kernel, in
 /* Human-readable name of a status code (static string, never NULL). */
 const char* relation_status_string(relation_status s);
 
+/* When a call returned RELATION_ERR_CUDA: the CUDA error string of the failing CUDA call
+ * made by the calling thread inside the library ("no error" otherwise).  Static string. */
+const char* relation_last_cuda_error(void);
+
 /* Library ABI version, (major << 16) | minor. */
 int relation_version(void);
 

@@ -28,7 +28,7 @@ KERNELS = {"auto": 0, "simt": 1, "tcgen05": 2}
 
 EXPORTED = ("relation_fwd", "relation_fwd_ex", "relation_bwd", "relation_bwd_ex",
             "relation_bwd_workspace_size", "relation_status_string", "relation_version",
-            "relation_selftest_wait_timeout", "relation_launch_count")
+            "relation_selftest_wait_timeout", "relation_launch_count", "relation_last_cuda_error")
 
 
 class RelationLibraryMissing(RuntimeError):
@@ -37,7 +37,10 @@ class RelationLibraryMissing(RuntimeError):
 
 class RelationError(RuntimeError):
     def __init__(self, code: int, where: str):
-        super().__init__(f"{where}: {status_string(code)} ({code})")
+        msg = f"{where}: {status_string(code)} ({code})"
+        if code == ERR_CUDA:
+            msg += f": {load().relation_last_cuda_error().decode()}"
+        super().__init__(msg)
         self.code = code
 
 
@@ -77,6 +80,8 @@ def load(path: str | None = None):
         lib.relation_version.argtypes = []
         lib.relation_selftest_wait_timeout.argtypes = [ip, i, vp]
         lib.relation_launch_count.argtypes = [i, i, i, i]
+        lib.relation_last_cuda_error.argtypes = []
+        lib.relation_last_cuda_error.restype = ctypes.c_char_p
         for n in ("relation_fwd", "relation_fwd_ex", "relation_bwd", "relation_bwd_ex",
                   "relation_version", "relation_selftest_wait_timeout", "relation_launch_count"):
             getattr(lib, n).restype = ctypes.c_int

@@ -78,4 +78,8 @@ int main_ctas(const Problem& p);
 
 cudaError_t launch_selftest_wait(int* dev_status, int timeout_us, cudaStream_t s);
 
+// Where the last failing CUDA step of this thread happened (reported by
+// relation_last_cuda_error); launchers set it before returning an error.
+void note_failure(const char* where);
+
 }  // namespace rel

@@ -5,6 +5,7 @@
 // library allocates no device memory.
 #include <math.h>
 #include <stdint.h>
+#include <stdio.h>
 
 #include "kernels.h"
 #include "relation.h"
@@ -67,9 +68,22 @@ Problem make_problem(relation_shape s, relation_dtype dt, float lambda, float ta
   return p;
 }
 
-relation_status from_cuda(cudaError_t e) { return e == cudaSuccess ? RELATION_OK : RELATION_ERR_CUDA; }
+thread_local cudaError_t g_last_cuda_error = cudaSuccess;
+thread_local const char* g_last_where = "";
+thread_local char g_last_message[256];
+
+relation_status from_cuda(cudaError_t e) {
+  if (e == cudaSuccess) return RELATION_OK;
+  if (e == cudaErrorInvalidValue && !g_last_where[0]) g_last_where = "launch";
+  g_last_cuda_error = e;
+  return RELATION_ERR_CUDA;
+}
 
 }  // namespace
+
+namespace rel {
+void note_failure(const char* where) { g_last_where = where; }
+}  // namespace rel
 
 extern "C" {
 
@@ -126,9 +140,9 @@ relation_status relation_bwd_ex(const void* q, const void* k, const void* v, con
   cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
   if (fam == 2) return from_cuda(rel::tc::launch_bwd(p, ws, s));  // row pass, tiles, finalise
   cudaError_t e = rel::bwd_common::launch_pre(p, ws, s);
-  if (e != cudaSuccess) return RELATION_ERR_CUDA;
+  if (e != cudaSuccess) return from_cuda(e);
   e = rel::simt::launch_bwd(p, ws, s);
-  if (e != cudaSuccess) return RELATION_ERR_CUDA;
+  if (e != cudaSuccess) return from_cuda(e);
   return from_cuda(rel::bwd_common::launch_dlambda(p, ws, rel::simt::main_ctas(p), s));
 }
 
@@ -152,6 +166,12 @@ const char* relation_status_string(relation_status s) {
     case RELATION_ERR_TIMEOUT: return "RELATION_ERR_TIMEOUT";
   }
   return "RELATION_ERR_UNKNOWN";
+}
+
+const char* relation_last_cuda_error(void) {
+  snprintf(g_last_message, sizeof(g_last_message), "%s%s%s", g_last_where,
+           g_last_where[0] ? ": " : "", cudaGetErrorString(g_last_cuda_error));
+  return g_last_message;
 }
 
 int relation_version(void) { return (1 << 16) | 0; }

@@ -355,19 +355,24 @@ bool supports(relation_dtype dt, int d) { return dt == RELATION_BF16 && (d == 64
 
 template <int D>
 static cudaError_t fwd_t(const Problem& p, cudaStream_t s) {
-  CUtensorMap mq, mk, mv;
-  if (!make_tmap_bf16(&mq, p.q, p, BM) || !make_tmap_bf16(&mk, p.k, p, BN) ||
-      !make_tmap_bf16(&mv, p.v, p, BN))
-    return cudaErrorInvalidValue;
+  // A runtime call first: it makes the primary context current on this thread, which the
+  // driver's tensor-map encoder needs.
   const int smem = FwdCfg<D>::SMEM;
   cudaError_t e =
       cudaFuncSetAttribute(fwd_tc_kernel<D>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
-  if (e != cudaSuccess) return e;
+  if (e != cudaSuccess) { note_failure("forward: shared memory attribute"); return e; }
+  CUtensorMap mq, mk, mv;
+  if (!make_tmap_bf16(&mq, p.q, p, BM) || !make_tmap_bf16(&mk, p.k, p, BN) ||
+      !make_tmap_bf16(&mv, p.v, p, BN)) {
+    note_failure("forward: TMA descriptor of Q/K/V");
+    return cudaErrorInvalidValue;
+  }
   const int n_qt = (p.T + BM - 1) / BM;
   const long long grid = (long long)n_qt * p.B * p.H;
   if (grid > 0x7fffffffLL) return cudaErrorInvalidConfiguration;
   fwd_tc_kernel<D><<<(unsigned)grid, kThreads, smem, s>>>(mq, mk, mv, p, n_qt);
-  return cudaGetLastError();
+  if ((e = cudaGetLastError()) != cudaSuccess) note_failure("forward: kernel launch");
+  return e;
 }
 
 cudaError_t launch_fwd(const Problem& p, cudaStream_t s) {
