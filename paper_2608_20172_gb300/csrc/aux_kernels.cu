@@ -31,7 +31,7 @@ size_t bwd_workspace_bytes(int B, int H, int T, int d) {
   const size_t n_pre = (rows + 7) / 8;
   const size_t n_main = (size_t)((T + 63) / 64) * B * H;
   return up(rows_pad * d * sizeof(float)) + 4 * up(rows * sizeof(float)) +
-         up((n_pre + n_main) * sizeof(float));
+         up(rows_pad * 4 * sizeof(float)) + up((n_pre + n_main) * sizeof(float));
 }
 
 BwdWorkspace carve_workspace(void* base, int B, int H, int T, int d) {
@@ -46,6 +46,7 @@ BwdWorkspace carve_workspace(void* base, int B, int H, int T, int d) {
   w.F_self = reinterpret_cast<float*>(p); p += up(rows * sizeof(float));
   w.dS_self = reinterpret_cast<float*>(p); p += up(rows * sizeof(float));
   w.wl = reinterpret_cast<float*>(p); p += up(rows * sizeof(float));
+  w.stats = reinterpret_cast<float*>(p); p += up((size_t)B * H * t_pad * 4 * sizeof(float));
   w.dlam_part = reinterpret_cast<float*>(p);
   w.n_pre_blocks = (int)((rows + 7) / 8);
   w.n_main_slots = ((T + 63) / 64) * B * H;

@@ -89,58 +89,96 @@ __device__ __forceinline__ void tma_reduce_add_2d(const CUtensorMap* m, uint32_t
       ::"l"(reinterpret_cast<uint64_t>(m)), "r"(src), "r"(c0), "r"(c1)
       : "memory");
 }
+// 1-D bulk copy global -> shared completing on an mbarrier (16-byte aligned, size % 16 == 0)
+__device__ __forceinline__ void bulk_load(uint32_t dst, const void* src, uint32_t bytes,
+                                          uint32_t bar) {
+  asm volatile(
+      "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];"
+      ::"r"(dst), "l"(reinterpret_cast<uint64_t>(src)), "r"(bytes), "r"(bar)
+      : "memory");
+}
 __device__ __forceinline__ void bulk_wait_read_le1() {
   asm volatile("cp.async.bulk.wait_group.read 1;" ::: "memory");
 }
 
-// Elementwise work on 32 query columns of one key row.  Writes P (bf16x2) into pk and
-// dS' = 2 dS (bf16x2) into dk; accumulates the Exchange part of dlambda.
+// Per-thread constants of the elementwise step.
+struct EwConst {
+  float ch;       // u / 2 = U ch       (U = raw q . k, u = U / sqrt(d))
+  float c2k;      // E log2 e = U c2k (1 + tanh(u / 2))
+  float ch_self;  // u / (2 tau_S) = U ch_self
+  float inv2tau;  // 1 / (2 tau_S)
+  float li;       // log(i) of this thread's own row (the Self entry on the diagonal)
+};
+
+// Elementwise work on 32 query columns of one key row (this thread's key).  st holds the
+// tile's per-query scalars, structure of arrays: [0,128) c2 = (-lambda log i - logZ_i)
+// log2 e, [128,256) -D_i, [256,384) -log i F_ii, [384,512) -logZ_i log2 e.
+// Produces P = F_ij and dS' = 2 dS_ij as bf16 pairs and accumulates the dlambda terms.
+//   Exchange:  P = 2^(U c2k (1 + t) + c2),  t = tanh(u/2),
+//              2 SiLU'(u) = a (1 + h (1 - t)) with a = 1 + t, h = u / 2.
+//   Self (DIAG, query == key):  S = (1 + tanh(u / (2 tau_S))) / 2 = a / 2,
+//              P = 2^(S log2 e - logZ log2 e),  2 dS/du = a (1 - t) / (2 tau_S).
 template <bool DIAG>
-__device__ __forceinline__ void tile_chunk(const uint32_t (&U)[32], const uint32_t (&G)[32],
-                                           const float* st, int qloc0, int t, int key_g,
-                                           float ch, float c2k, float isd, float inv_tau,
-                                           uint32_t (&pk)[16], uint32_t (&dk)[16], float& dlam) {
+__device__ __forceinline__ void ew_chunk(const uint32_t (&U)[32], const uint32_t (&G)[32],
+                                         const float* st, int qloc0, int t, const EwConst& k,
+                                         uint32_t (&pk)[16], uint32_t (&dk)[16], float2& dl2) {
+  if (!DIAG) {
+    const float2 ch2 = make_float2(k.ch, k.ch), c2k2 = make_float2(k.c2k, k.c2k);
+    const float2 one2 = make_float2(1.f, 1.f);
 #pragma unroll
-  for (int c = 0; c < 32; c += 4) {
-    const float4 c2v = *reinterpret_cast<const float4*>(st + qloc0 + c);
-    const float4 ddv = *reinterpret_cast<const float4*>(st + BT + qloc0 + c);
-    const float4 wlv = *reinterpret_cast<const float4*>(st + 2 * BT + qloc0 + c);
-    const float c2a[4] = {c2v.x, c2v.y, c2v.z, c2v.w};
-    const float dda[4] = {ddv.x, ddv.y, ddv.z, ddv.w};
-    const float wla[4] = {wlv.x, wlv.y, wlv.z, wlv.w};
-    float pv[4], sv[4];
+    for (int c = 0; c < 32; c += 4) {
+      const float4 c2v = *reinterpret_cast<const float4*>(st + qloc0 + c);
+      const float4 ndv = *reinterpret_cast<const float4*>(st + BT + qloc0 + c);
+      const float4 nwv = *reinterpret_cast<const float4*>(st + 2 * BT + qloc0 + c);
 #pragma unroll
-    for (int e = 0; e < 4; ++e) {
-      const float x = __uint_as_float(U[c + e]);
-      const float g = __uint_as_float(G[c + e]);
-      const float hh = x * ch;                  // u / 2
-      const float th = tanh_approx(hh);         // sigma(u) = (1 + th) / 2
-      const float w = fmaf(th, c2k, c2k);
-      float P = ex2_approx(fmaf(x, w, c2a[e]));  // exp(E - lambda log i - logZ_i)
-      float dR = P * (g - dda[e]);
-      float s2 = dR * (1.0f + th + fmaf(-hh * th, th, hh));  // 2 dR SiLU'(u)
-      float dl = -wla[e] * dR;
-      if (DIAG) {
-        const int q = qloc0 + c + e;  // tile-local query index; the key is t
-        if (q < t) {                  // not history of query q
-          P = 0.f; s2 = 0.f; dl = 0.f;
-        } else if (q == t) {          // Self entry: role map sigmoid(u / tau_S)
-          const float S = 1.0f / (1.0f + __expf(-(x * isd) * inv_tau));
-          const float lzn = st[3 * BT + q];   // -logZ_i log2 e
-          P = ex2_approx(fmaf(S, kLog2e, lzn));
-          dR = P * (g - dda[e]);
-          s2 = 2.0f * dR * S * (1.0f - S) * inv_tau;
-          dl = __logf((float)(key_g + 1)) * (1.0f - P) * dR;
-        }
+      for (int e = 0; e < 4; e += 2) {
+        const float2 x = make_float2(__uint_as_float(U[c + e]), __uint_as_float(U[c + e + 1]));
+        const float2 g = make_float2(__uint_as_float(G[c + e]), __uint_as_float(G[c + e + 1]));
+        const float2 c2 = e == 0 ? make_float2(c2v.x, c2v.y) : make_float2(c2v.z, c2v.w);
+        const float2 nd = e == 0 ? make_float2(ndv.x, ndv.y) : make_float2(ndv.z, ndv.w);
+        const float2 nw = e == 0 ? make_float2(nwv.x, nwv.y) : make_float2(nwv.z, nwv.w);
+        const float2 h = __fmul2_rn(x, ch2);
+        const float2 th = make_float2(tanh_approx(h.x), tanh_approx(h.y));
+        const float2 a = __fadd2_rn(th, one2);
+        const float2 w = __fmul2_rn(a, c2k2);
+        const float2 ex = __ffma2_rn(x, w, c2);
+        const float2 P = make_float2(ex2_approx(ex.x), ex2_approx(ex.y));
+        const float2 dR = __fmul2_rn(P, __fadd2_rn(g, nd));
+        const float2 b = __ffma2_rn(make_float2(-h.x, -h.y), th, h);  // h (1 - t)
+        const float2 sp = __ffma2_rn(a, b, a);                        // 2 SiLU'(u)
+        const float2 dS = __fmul2_rn(dR, sp);
+        dl2 = __ffma2_rn(nw, dR, dl2);
+        pk[(c + e) >> 1] = pack_bf16x2(P.x, P.y);
+        dk[(c + e) >> 1] = pack_bf16x2(dS.x, dS.y);
       }
-      dlam += dl;
-      pv[e] = P;
-      sv[e] = s2;
     }
-    pk[c >> 1] = pack_bf16x2(pv[0], pv[1]);
-    pk[(c >> 1) + 1] = pack_bf16x2(pv[2], pv[3]);
-    dk[c >> 1] = pack_bf16x2(sv[0], sv[1]);
-    dk[(c >> 1) + 1] = pack_bf16x2(sv[2], sv[3]);
+  } else {
+    const float half_log2e = 0.5f * kLog2e;
+#pragma unroll
+    for (int c = 0; c < 32; c += 2) {
+      float pv[2], sv[2];
+#pragma unroll
+      for (int e = 0; e < 2; ++e) {
+        const int q = qloc0 + c + e;  // tile-local query index; this thread's key is t
+        const bool self = (q == t), keep = (q >= t);
+        const float x = __uint_as_float(U[c + e]);
+        const float g = __uint_as_float(G[c + e]);
+        const float h = x * (self ? k.ch_self : k.ch);
+        const float th = tanh_approx(h);
+        const float a = 1.0f + th;
+        const float w = a * (self ? half_log2e : k.c2k);
+        float P = ex2_approx(fmaf(self ? 1.0f : x, w, self ? st[3 * BT + q] : st[q]));
+        P = keep ? P : 0.f;
+        const float dR = P * (g + st[BT + q]);
+        const float m = fmaf(self ? k.inv2tau : h, 1.0f - th, self ? 0.f : 1.f);
+        sv[e] = dR * a * m;
+        pv[e] = P;
+        const float wgt = self ? k.li * (1.0f - P) : st[2 * BT + q];
+        dl2.x = fmaf(wgt, dR, dl2.x);
+      }
+      pk[c >> 1] = pack_bf16x2(pv[0], pv[1]);
+      dk[c >> 1] = pack_bf16x2(sv[0], sv[1]);
+    }
   }
 }
 
@@ -189,7 +227,6 @@ __global__ void __launch_bounds__(kThreads, 1)
   tc_fence_after();
   const uint32_t tmem = *tmem_slot;
   const Abort ab{abort_flag, p.dev_status};
-  const long long rows_bh = (long long)bh * p.T;
 
   if (warp == W_TMA) {
     // ------------------------------------------------------ TMA + per-query scalars
@@ -205,41 +242,22 @@ __global__ void __launch_bounds__(kThreads, 1)
       }
     }
     int issued = 0;
-    for (int i = 0; i < n_i; ++i) {
-      const int s = i % C::QSTG, u = i / C::QSTG;
-      bool ok = true;
-      if (u > 0) ok = mbar_wait(bar(B_QE + s), (u - 1) & 1, ab);
-      ok = __all_sync(0xffffffffu, ok);
-      if (!ok) break;
-      const int qi0 = (kt + i) * BT;
-      float* st = reinterpret_cast<float*>(smem + C::OFF_STAT + s * 4 * BT * 4);
-      for (int q = lane; q < BT; q += 32) {
-        const int row = qi0 + q;
-        float c2 = -INFINITY, dd = 0.f, wl = 0.f, lzn = -INFINITY;
-        if (row < p.T) {
-          const float lz = p.logz_in[rows_bh + row];
-          c2 = (-p.lambda * __logf((float)(row + 1)) - lz) * kLog2e;
-          dd = ws.D[rows_bh + row];
-          wl = ws.wl[rows_bh + row];
-          lzn = -lz * kLog2e;
-        }
-        st[q] = c2;
-        st[BT + q] = dd;
-        st[2 * BT + q] = wl;
-        st[3 * BT + q] = lzn;
-      }
-      __threadfence_block();
-      __syncwarp();
-      if (lane == 0) {
-        mbar_arrive_expect_tx(bar(B_QF + s), 2 * C::TILE);
+    if (lane == 0) {
+      for (int i = 0; i < n_i; ++i) {
+        const int s = i % C::QSTG, u = i / C::QSTG;
+        if (u > 0 && !mbar_wait(bar(B_QE + s), (u - 1) & 1, ab)) break;
+        const int qi0 = (kt + i) * BT;
+        mbar_arrive_expect_tx(bar(B_QF + s), 2 * C::TILE + 4 * BT * 4);
         for (int kb = 0; kb < C::KB; ++kb) {
           tma_load_4d(sb + C::OFF_Q + s * C::TILE + kb * 16384, &tmQ, bar(B_QF + s), kb * 64,
                       qi0, h, b);
           tma_load_4d(sb + C::OFF_DO + s * C::TILE + kb * 16384, &tmG, bar(B_QF + s), kb * 64,
                       qi0, h, b);
         }
+        bulk_load(sb + C::OFF_STAT + s * 4 * BT * 4,
+                  ws.stats + ((long long)bh * n_t + kt + i) * 4 * BT, 4 * BT * 4, bar(B_QF + s));
+        issued = i + 1;
       }
-      issued = i + 1;
     }
     if (lane == 0 && ab.raised()) {
       drain_wait(bar(B_KV), 0);
@@ -373,11 +391,14 @@ __global__ void __launch_bounds__(kThreads, 1)
     const int t = (warp & 3) * 32 + lane;      // key k0 + t, TMEM lane t
     const uint32_t trow = tmem + ((uint32_t)((warp & 3) * 32) << 16);
     const float isd = p.inv_sqrt_d;
-    const float ch = 0.5f * isd;
-    const float c2k = ch * kLog2e;
-    const float inv_tau = 1.0f / p.tau_s;
+    EwConst kc;
+    kc.ch = 0.5f * isd;
+    kc.c2k = kc.ch * kLog2e;
+    kc.ch_self = kc.ch / p.tau_s;
+    kc.inv2tau = 0.5f / p.tau_s;
     const int key_g = k0 + t;
-    float dlam = 0.f;
+    kc.li = __logf((float)(key_g + 1));
+    float2 dl2 = make_float2(0.f, 0.f);
     bool ok = true;
     const int bb = C::NBUF == 2 ? wg : 0;
     const uint32_t col_u = C::col_u(bb) + (C::NBUF == 2 ? 0 : wg * 64);
@@ -393,7 +414,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       const float* st =
           reinterpret_cast<const float*>(smem + C::OFF_STAT + (i % C::QSTG) * 4 * BT * 4);
       uint8_t* ds_row = smem + C::OFF_DS + (i % C::DSB) * 32768 + wg * 16384 + t * 128;
-#pragma unroll
+#pragma unroll 1
       for (int c0 = 0; c0 < 64; c0 += 32) {
         uint32_t U[32], G[32];
         tmem_ld32(trow + col_u + c0, U);
@@ -401,9 +422,9 @@ __global__ void __launch_bounds__(kThreads, 1)
         tmem_ld_wait();
         uint32_t pk[16], dk[16];
         if (i == 0)
-          tile_chunk<true>(U, G, st, qbase + c0, t, key_g, ch, c2k, isd, inv_tau, pk, dk, dlam);
+          ew_chunk<true>(U, G, st, qbase + c0, t, kc, pk, dk, dl2);
         else
-          tile_chunk<false>(U, G, st, qbase + c0, t, key_g, ch, c2k, isd, inv_tau, pk, dk, dlam);
+          ew_chunk<false>(U, G, st, qbase + c0, t, kc, pk, dk, dl2);
         tmem_st16(trow + col_u + (c0 >> 1), pk);
         const int cb = c0 >> 3;  // first 16-byte chunk of these 32 queries in the row
 #pragma unroll
@@ -416,6 +437,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       tc_fence_before();
       mbar_arrive(bar(B_P + bb));
     }
+    float dlam = dl2.x + dl2.y;
     // ---------------------------------------------------- dK (warpgroup 0) / dV (1)
     if (ok) ok = __all_sync(0xffffffffu, mbar_wait(bar(B_ACC), 0, ab));
     tc_fence_after();
@@ -463,21 +485,25 @@ __global__ void __launch_bounds__(kThreads, 1)
   }
 }
 
-// Row pass: D_i = dO_i . Y_i, wl_i = log i F_ii with F_ii = exp(sigmoid(u_ii / tau_S) -
-// logZ_i), and a zeroed row of the fp32 dQ accumulator.  8 threads per row.
+// Row pass over the padded rows r < t_pad of every head, 8 threads per row:
+//   D_i = dO_i . Y_i,  F_ii = exp(sigmoid(u_ii / tau_S) - logZ_i),
+// written as the per-query scalars of the tile kernel (structure of arrays per 128-row
+// tile: c2 = (-lambda log i - logZ_i) log2 e, -D_i, -log i F_ii, -logZ_i log2 e), and a
+// zeroed row of the fp32 dQ accumulator.  Padding rows get neutral scalars (P = 0).
 template <int D>
-__global__ void __launch_bounds__(256) pre_kernel(Problem p, BwdWorkspace ws) {
+__global__ void __launch_bounds__(256) pre_kernel(Problem p, BwdWorkspace ws, int n_t) {
   constexpr int PER = D / 8;  // elements per thread
   const long long gr = ((long long)blockIdx.x * 256 + threadIdx.x) >> 3;
   const int sub = threadIdx.x & 7;
-  const long long nrows = (long long)p.B * p.H * p.T;
+  const long long nrows = (long long)p.B * p.H * ws.t_pad;
   const bool live = gr < nrows;
   const long long grc = live ? gr : 0;
-  const int bh = (int)(grc / p.T), r = (int)(grc % p.T);
+  const int bh = (int)(grc / ws.t_pad), r = (int)(grc % ws.t_pad);
+  const bool real = live && r < p.T;
   const int b = bh / p.H, h = bh % p.H;
   const long long off = (long long)b * p.sB + (long long)h * p.sH + (long long)r * p.sT + sub * PER;
   float gy = 0.f, qk = 0.f;
-  if (live) {
+  if (real) {
 #pragma unroll
     for (int c = 0; c < PER; c += 8) {
       const uint4 gv = *reinterpret_cast<const uint4*>(reinterpret_cast<const __nv_bfloat16*>(p.dout) + off + c);
@@ -504,10 +530,21 @@ __global__ void __launch_bounds__(256) pre_kernel(Problem p, BwdWorkspace ws) {
   }
   if (!live) return;
   if (sub == 0) {
-    const float S = 1.0f / (1.0f + expf(-(qk * p.inv_sqrt_d) / p.tau_s));
-    const float F = expf(S - p.logz_in[gr]);
-    ws.D[gr] = gy;
-    ws.wl[gr] = logf((float)(r + 1)) * F;
+    float c2 = -INFINITY, nd = 0.f, nw = 0.f, lzn = -INFINITY;
+    if (real) {
+      const float lz = p.logz_in[(long long)bh * p.T + r];
+      const float li = logf((float)(r + 1));
+      const float S = 1.0f / (1.0f + expf(-(qk * p.inv_sqrt_d) / p.tau_s));
+      c2 = (-p.lambda * li - lz) * kLog2e;
+      nd = -gy;
+      nw = -li * expf(S - lz);
+      lzn = -lz * kLog2e;
+    }
+    float* st = ws.stats + ((long long)bh * n_t + (r >> 7)) * 4 * BT + (r & 127);
+    st[0] = c2;
+    st[BT] = nd;
+    st[2 * BT] = nw;
+    st[3 * BT] = lzn;
   }
   float* acc = ws.dq_acc + ((long long)bh * ws.t_pad + r) * D + sub * PER;
 #pragma unroll
@@ -596,7 +633,8 @@ static cudaError_t bwd_t(const Problem& p, const BwdWorkspace& ws, cudaStream_t 
     return cudaErrorInvalidValue;
   }
   const long long rows = (long long)p.B * p.H * p.T;
-  bwd::pre_kernel<D><<<(unsigned)((rows * 8 + 255) / 256), 256, 0, s>>>(p, ws);
+  const long long rows_pad = (long long)p.B * p.H * t_pad;
+  bwd::pre_kernel<D><<<(unsigned)((rows_pad * 8 + 255) / 256), 256, 0, s>>>(p, ws, n_t);
   if ((e = cudaGetLastError()) != cudaSuccess) { note_failure("backward: row pass launch"); return e; }
   const long long grid = (long long)n_t * p.B * p.H;
   if (grid > 0x7fffffffLL) return cudaErrorInvalidConfiguration;
