@@ -21,10 +21,12 @@
 //   MMA  dV += P^T dO (P read from TMEM),  dK += dS'^T Q
 // and once per 128-query tile  MMA dQ_t = dS' K, which warps 8-11 stage through shared
 // memory and add to the fp32 accumulator with TMA reduce-add.
-//   d_h = 64 : W = 64, two TMEM buffers; elementwise warpgroup w owns buffer w, so the
-//              MMAs of one half-tile overlap the elementwise work of the other.
-//   d_h = 128: W = 128, one buffer (TMEM is full); both warpgroups split its columns and
-//              dQ_t reuses the dP^T columns.
+//   d_h = 64 : W = 64 on two TMEM buffers: the MMAs of one buffer (dV, dK of the last
+//              step, U^T / dP^T of the next) overlap the elementwise work on the other.
+//   d_h = 128: W = 128 on one buffer (TMEM is full); dQ_t reuses the dP^T columns.
+// Both elementwise warpgroups split every step's columns.  A tcgen05.mma costs at least
+// ~46 cycles whatever its N (measured on GB300: N = 32, 64, 128 run at 35%, 66%, 99% of
+// the per-SM peak), so the steps keep N >= 64.
 // dlambda = sum_i log i g_i dR_ii - sum_{j<i} log i F_ii dR_ij (weights cancel the
 // rounding error of D_i; see aux_kernels.cu), reduced per CTA.
 #include <cudaTypedefs.h>
@@ -51,7 +53,8 @@ struct Cfg {
   static constexpr int KB = D / 64;
   static constexpr int TILE = 128 * D * 2;
   static constexpr int NBUF = D == 64 ? 2 : 1;   // U^T / dP^T TMEM buffers
-  static constexpr int QW = D == 64 ? 64 : 128;  // query columns per step
+  static constexpr int QW = D == 64 ? 64 : 128;  // query columns per step (both warpgroups
+                                                 // split them: QW / 2 each)
   static constexpr int SPT = BT / QW;            // steps per query tile
   static constexpr int QSTG = D == 64 ? 2 : 1;   // Q / dO tile stages
   static constexpr int DSB = D == 64 ? 2 : 1;    // dS' buffers (by tile parity)
@@ -65,8 +68,9 @@ struct Cfg {
   static constexpr int OFF_RED = OFF_STAT + QSTG * 4 * BT * 4;
   static constexpr int OFF_BAR = OFF_RED + 64;
   static constexpr int SMEM = OFF_BAR + 256 + 1024;
-  static constexpr int COL_DK = 256, COL_DV = 256 + D;
-  static constexpr int COL_DQ = D == 64 ? 384 : 128;       // d = 128: dP^T columns
+  static constexpr int COL_DK = NBUF * 2 * QW;              // 256 / 256
+  static constexpr int COL_DV = COL_DK + D;                  // 320 / 384
+  static constexpr int COL_DQ = D == 64 ? 384 : QW;          // d = 128: the dP^T columns
   __host__ __device__ static constexpr int col_u(int b) { return b * 2 * QW; }
   __host__ __device__ static constexpr int col_g(int b) { return b * 2 * QW + QW; }
 };
@@ -194,8 +198,8 @@ __global__ void __launch_bounds__(kThreads, 1)
       (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
   const uint32_t sb = smem_u32(smem);
   auto bar = [&](int i) -> uint32_t { return sb + C::OFF_BAR + 8u * (uint32_t)i; };
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(smem + C::OFF_BAR + 128);
-  volatile int* abort_flag = reinterpret_cast<volatile int*>(smem + C::OFF_BAR + 136);
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(smem + C::OFF_BAR + 192);
+  volatile int* abort_flag = reinterpret_cast<volatile int*>(smem + C::OFF_BAR + 200);
   float* red = reinterpret_cast<float*>(smem + C::OFF_RED);
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -212,8 +216,10 @@ __global__ void __launch_bounds__(kThreads, 1)
     for (int s = 0; s < 2; ++s) {
       mbar_init(bar(B_QF + s), 1);
       mbar_init(bar(B_QE + s), 1);
+    }
+    for (int s = 0; s < C::NBUF; ++s) {
       mbar_init(bar(B_S + s), 1);
-      mbar_init(bar(B_P + s), C::NBUF == 2 ? 128 : 256);
+      mbar_init(bar(B_P + s), 256);  // both elementwise warpgroups
     }
     mbar_init(bar(B_DQF), 1);
     mbar_init(bar(B_DQE), 128);
@@ -278,7 +284,7 @@ __global__ void __launch_bounds__(kThreads, 1)
           if (!mbar_wait(bar(B_QF + st), (t / C::QSTG) & 1, ab)) return false;
           tc_fence_after();
         }
-        const uint32_t qoff = hh * C::QW * 128;
+        const uint32_t qoff = hh * C::QW * 128;  // rows of the query tile (32-row aligned)
 #pragma unroll
         for (int kk = 0; kk < D / 16; ++kk) {
           const uint32_t koff = (kk >> 2) * 16384 + (kk & 3) * 32;
@@ -300,32 +306,38 @@ __global__ void __launch_bounds__(kThreads, 1)
         mma_commit(bar(B_S + bb));
         return true;
       };
-      for (int s = 0; ok && s < C::NBUF && s < total; ++s) ok = issue_sdp(s);
+      // U^T / dP^T of step sn may be issued once its buffer is free (step sn - NBUF done)
+      // and once the GEMM that releases the Q/dO stage of its tile (dQ of tile
+      // tn - QSTG) has been issued: waiting for that tile's load earlier would deadlock.
+      int sn = 0, tiles_done = 0;
+      while (ok && sn < total && sn < C::NBUF) ok = issue_sdp(sn++);
       for (int s = 0; ok && s < total; ++s) {
         const int t = s / C::SPT, hh = s % C::SPT, bb = s % C::NBUF;
         const int st = t % C::QSTG, dsb = t % C::DSB;
         if (!(ok = mbar_wait(bar(B_P + bb), (s / C::NBUF) & 1, ab))) break;
         tc_fence_after();
         const uint32_t ds_base = sb + C::OFF_DS + dsb * 32768;
-        // dV += P^T dO   (P from TMEM, packed two per column)
+        // dV += P^T dO and dK += dS'^T Q with the A operands in TMEM: every 32-query chunk
+        // keeps its 16 packed columns of P (dS') at the start of its own U^T (dP^T) columns.
+        const uint32_t pcol = C::col_u(bb), dcol = C::col_g(bb);
 #pragma unroll
         for (int kk = 0; kk < C::QW / 16; ++kk) {
           const int q = hh * C::QW + kk * 16;
-          mma_ts(tmem + C::COL_DV, tmem + C::col_u(bb) + (kk >> 2) * 64 + (kk & 3) * 8,
+          const uint32_t acol = (kk >> 1) * 32 + (kk & 1) * 8;
+          mma_ts(tmem + C::COL_DV, tmem + pcol + acol,
                  smem_desc_sw128(sb + C::OFF_DO + st * C::TILE + q * 128, 16384, 1024), id_acc,
                  (s > 0 || kk > 0) ? 1u : 0u);
         }
-        // dK += dS'^T Q   (A = dS'^T, queries contiguous: K-major)
 #pragma unroll
         for (int kk = 0; kk < C::QW / 16; ++kk) {
           const int q = hh * C::QW + kk * 16;
-          mma_ss(tmem + C::COL_DK,
-                 smem_desc_sw128(ds_base + (q >> 6) * 16384 + ((q & 63) >> 4) * 32, 16, 1024),
+          const uint32_t acol = (kk >> 1) * 32 + (kk & 1) * 8;
+          mma_ts(tmem + C::COL_DK, tmem + dcol + acol,
                  smem_desc_sw128(sb + C::OFF_Q + st * C::TILE + q * 128, 16384, 1024), id_acc,
                  (s > 0 || kk > 0) ? 1u : 0u);
         }
         if (hh == C::SPT - 1) {
-          if (D == 64 && t > 0) {
+          if (t > 0) {  // dQ_{t-1} has been read out of TMEM
             if (!(ok = mbar_wait(bar(B_DQE), (t - 1) & 1, ab))) break;
             tc_fence_after();
           }
@@ -337,8 +349,10 @@ __global__ void __launch_bounds__(kThreads, 1)
                    kk > 0 ? 1u : 0u);
           mma_commit(bar(B_DQF));
           mma_commit(bar(B_QE + st));
+          ++tiles_done;
         }
-        if (s + C::NBUF < total && !(ok = issue_sdp(s + C::NBUF))) break;
+        while (ok && sn < total && sn <= s + C::NBUF && sn / C::SPT - C::QSTG < tiles_done)
+          ok = issue_sdp(sn++);
       }
       mma_commit(bar(B_ACC));
     }
@@ -400,12 +414,9 @@ __global__ void __launch_bounds__(kThreads, 1)
     kc.li = __logf((float)(key_g + 1));
     float2 dl2 = make_float2(0.f, 0.f);
     bool ok = true;
-    const int bb = C::NBUF == 2 ? wg : 0;
-    const uint32_t col_u = C::col_u(bb) + (C::NBUF == 2 ? 0 : wg * 64);
-    const uint32_t col_g = C::col_g(bb) + (C::NBUF == 2 ? 0 : wg * 64);
-    const int qbase = wg * 64;                 // tile-local query columns of this warpgroup
-    for (int i = 0; i < n_i; ++i) {
-      ok = __all_sync(0xffffffffu, mbar_wait(bar(B_S + bb), i & 1, ab));
+    for (int s = 0; s < total; ++s) {
+      const int bb = s % C::NBUF, i = s / C::SPT, qs = (s % C::SPT) * C::QW;
+      ok = __all_sync(0xffffffffu, mbar_wait(bar(B_S + bb), (s / C::NBUF) & 1, ab));
       if (!ok) break;
       tc_fence_after();
       // acquire the producer's per-query scalars of this tile (already complete)
@@ -413,20 +424,24 @@ __global__ void __launch_bounds__(kThreads, 1)
       if (!ok) break;
       const float* st =
           reinterpret_cast<const float*>(smem + C::OFF_STAT + (i % C::QSTG) * 4 * BT * 4);
-      uint8_t* ds_row = smem + C::OFF_DS + (i % C::DSB) * 32768 + wg * 16384 + t * 128;
 #pragma unroll 1
-      for (int c0 = 0; c0 < 64; c0 += 32) {
+      for (int ck = 0; ck < C::QW / 64; ++ck) {
+        const int cl = wg * (C::QW / 2) + ck * 32;  // chunk's first column within the step
+        const int q0 = qs + cl;                       // tile-local query index
         uint32_t U[32], G[32];
-        tmem_ld32(trow + col_u + c0, U);
-        tmem_ld32(trow + col_g + c0, G);
+        tmem_ld32(trow + C::col_u(bb) + cl, U);
+        tmem_ld32(trow + C::col_g(bb) + cl, G);
         tmem_ld_wait();
         uint32_t pk[16], dk[16];
         if (i == 0)
-          ew_chunk<true>(U, G, st, qbase + c0, t, kc, pk, dk, dl2);
+          ew_chunk<true>(U, G, st, q0, t, kc, pk, dk, dl2);
         else
-          ew_chunk<false>(U, G, st, qbase + c0, t, kc, pk, dk, dl2);
-        tmem_st16(trow + col_u + (c0 >> 1), pk);
-        const int cb = c0 >> 3;  // first 16-byte chunk of these 32 queries in the row
+          ew_chunk<false>(U, G, st, q0, t, kc, pk, dk, dl2);
+        tmem_st16(trow + C::col_u(bb) + cl, pk);  // P   (A operand of dV += P^T dO)
+        tmem_st16(trow + C::col_g(bb) + cl, dk);  // dS' (A operand of dK += dS'^T Q)
+        // dS' row t, queries q0 .. q0+31 for dQ = dS' K: 4 chunks of the 128-byte swizzle
+        uint8_t* ds_row = smem + C::OFF_DS + (i % C::DSB) * 32768 + (q0 >> 6) * 16384 + t * 128;
+        const int cb = (q0 & 63) >> 3;
 #pragma unroll
         for (int qd = 0; qd < 4; ++qd)
           *reinterpret_cast<uint4*>(ds_row + (((cb + qd) ^ (t & 7)) << 4)) =
