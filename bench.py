@@ -62,8 +62,8 @@ class ClockSampler:
     def __enter__(self):
         try:
             self.proc = subprocess.Popen(
-                ["nvidia-smi", f"--id={self.index}", f"--query-gpu={self.QUERY}",
-                 "--format=csv,noheader,nounits", "-lms", "200"],
+                ["nvidia-smi", f"--id={self.index}", f"--query-gpu=timestamp,{self.QUERY}",
+                 "--format=csv,noheader,nounits", "-lms", "50"],
                 stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
         except OSError:
             self.proc = None
@@ -81,13 +81,24 @@ class ClockSampler:
             self.lines = [ln for ln in out.splitlines() if ln.strip()]
         return False
 
-    def summary(self):
+    def summary(self, t_begin=None, t_end=None):
+        """Median SM clock and active throttle reasons over the samples taken between the
+        host times t_begin and t_end (all samples when no window is given)."""
+        import datetime
         sm, mx, reasons = [], None, set()
         names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
         for ln in getattr(self, "lines", []):
             f = [x.strip() for x in ln.split(",")]
-            if len(f) < 9:
+            if len(f) < 10:
                 continue
+            if t_begin is not None:
+                try:
+                    ts = datetime.datetime.strptime(f[0], "%Y/%m/%d %H:%M:%S.%f").timestamp()
+                except ValueError:
+                    ts = None
+                if ts is not None and not (t_begin - 0.06 <= ts <= t_end + 0.06):
+                    continue
+            f = f[1:]
             try:
                 sm.append(float(f[1]))
                 mx = float(f[2])
@@ -100,6 +111,24 @@ class ClockSampler:
             return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["unsampled"], "samples": 0}
         return {"sm_mhz": statistics.median(sm), "sm_max_mhz": mx, "reasons": sorted(reasons),
                 "samples": len(sm)}
+
+
+def _profiled_traffic(w, kernel):
+    """DRAM bytes per launch of `kernel` from the committed ncu summary for this workload,
+    scaled to it, or None when there is none or the kernel source changed since."""
+    import hashlib
+    path = os.path.join(ROOT, "profiles", f"{kernel}_traffic.json")
+    try:
+        with open(path) as f:
+            rec = json.load(f)
+        src = os.path.join(ROOT, rec["source"])
+        with open(src, "rb") as f:
+            if hashlib.sha256(f.read()).hexdigest() != rec["source_sha256"]:
+                return None
+        units = w.B * w.H * w.T * w.T  # traffic scales with the causal tile count
+        return rec["dram_bytes_per_launch"] * units / rec["units"]
+    except (OSError, KeyError, ValueError):
+        return None
 
 
 def _dist():
@@ -141,25 +170,32 @@ def _oracle_sample(w, n_heads):
 
 
 def _sample_heads(w):
-    # ~10-30 s of oracle work on the host: scale the sample by the per-head cost.
+    # a bounded sample: at most the cost of 128 heads of T=1024, d=64 (about 1 s of
+    # OpenMP oracle work on 16 cores), whole batches of heads where possible
     per_head = w.T * w.T * w.d
-    budget = 16 * 1024 * 1024 * 64  # 16 heads of the 10M workload
+    budget = 128 * 1024 * 1024 * 64
     n = max(1, min(w.B * w.H, budget // per_head))
     return n if n < w.H else (n // w.H) * w.H
 
 
-def cpu_oracle_run(w, n_heads=None):
+def cpu_oracle_run(w, n_heads=None, min_seconds=0.0, max_reps=20):
+    """Time the fp64 oracle (forward + backward) on the first n_heads heads of the workload,
+    repeating the sample until min_seconds of CPU work have run."""
     import oracle
     n_heads = n_heads or _sample_heads(w)
     (q, k, v, do), used = _oracle_sample(w, n_heads)
     threads = oracle.max_threads()
-    t0 = time.perf_counter()
-    oracle.mhr_fwd(q, k, v, workloads.LAMBDA_INIT)
-    oracle.mhr_bwd(q, k, v, do, workloads.LAMBDA_INIT)
-    dt = time.perf_counter() - t0
-    flops = 7.0 * used * w.T * w.T * w.d
-    return {"seconds": dt, "heads": used, "flops": flops, "tflops": flops / dt / 1e12,
-            "tokens_per_s": (used / w.H) * w.T / dt, "cores": threads}
+    reps, dt = 0, 0.0
+    while reps < max_reps and (reps == 0 or dt < min_seconds):
+        t0 = time.perf_counter()
+        oracle.mhr_fwd(q, k, v, workloads.LAMBDA_INIT)
+        oracle.mhr_bwd(q, k, v, do, workloads.LAMBDA_INIT)
+        dt += time.perf_counter() - t0
+        reps += 1
+    flops = 7.0 * used * w.T * w.T * w.d * reps
+    return {"seconds": dt, "heads": used, "reps": reps, "flops": flops,
+            "tflops": flops / dt / 1e12, "tokens_per_s": reps * (used / w.H) * w.T / dt,
+            "cores": threads}
 
 
 def run_reference(args, w):
@@ -229,27 +265,41 @@ def run_ours(args, w):
         raise SystemExit(f"device status {binding.status_string(int(status.item()))}")
 
     n = args.steps
-    ev = [[torch.cuda.Event(enable_timing=True) for _ in range(3)] for _ in range(n)]
+    # per step: forward | backward row pass | backward tiles | backward finalisation
+    ev = [[torch.cuda.Event(enable_timing=True) for _ in range(5)] for _ in range(n)]
     _barrier(dist, dev)
     torch.cuda.synchronize(dev)
     with ClockSampler(dev.index) as clk:
+        time.sleep(0.3)  # let the sampler start before the timed region
+        t_begin = time.time()
         for i in range(n):
             ev[i][0].record(stream)
             binding.fwd(qd, kd, vd, lam, tau, kernel=family, out=y, logz=logz, dev_status=status,
                         stream=stream)
             ev[i][1].record(stream)
-            binding.bwd(qd, kd, vd, y, dod, logz, lam, tau, kernel=family, workspace=wsb, dq=dq,
-                        dk=dk, dv=dv, dlambda=dl, dev_status=status, stream=stream)
-            ev[i][2].record(stream)
+            for j, stage in enumerate((binding.BWD_PREPARE, binding.BWD_TILES,
+                                       binding.BWD_FINALIZE)):
+                binding.bwd(qd, kd, vd, y, dod, logz, lam, tau, kernel=family, workspace=wsb,
+                            dq=dq, dk=dk, dv=dv, dlambda=dl, dev_status=status, stream=stream,
+                            stages=stage)
+                ev[i][2 + j].record(stream)
             flush.zero_()
         torch.cuda.synchronize(dev)
+        t_end = time.time()
+        time.sleep(0.1)
     _barrier(dist, dev)
     t_fwd = [ev[i][0].elapsed_time(ev[i][1]) for i in range(n)]
-    t_bwd = [ev[i][1].elapsed_time(ev[i][2]) for i in range(n)]
+    t_pre = [ev[i][1].elapsed_time(ev[i][2]) for i in range(n)]
+    t_til = [ev[i][2].elapsed_time(ev[i][3]) for i in range(n)]
+    t_fin = [ev[i][3].elapsed_time(ev[i][4]) for i in range(n)]
+    t_bwd = [a + b + c for a, b, c in zip(t_pre, t_til, t_fin)]
     t_step = [a + b for a, b in zip(t_fwd, t_bwd)]
     ms = _max_over_ranks(dist, statistics.mean(t_step), dev)
     ms_fwd = _max_over_ranks(dist, statistics.mean(t_fwd), dev)
     ms_bwd = _max_over_ranks(dist, statistics.mean(t_bwd), dev)
+    ms_tiles = _max_over_ranks(dist, statistics.mean(t_til), dev)
+    ms_pre = _max_over_ranks(dist, statistics.mean(t_pre), dev)
+    ms_fin = _max_over_ranks(dist, statistics.mean(t_fin), dev)
     st = int(status.item())
     if st != 0:
         raise SystemExit(f"device status {binding.status_string(st)}")
@@ -279,12 +329,13 @@ def run_ours(args, w):
     flops = w.flops_fwd_bwd()
     tflops = ws * flops / (ms * 1e-3) / 1e12
     peaks = _peaks()
-    # roofline of the dominant launch group: the backward call
     esz = 2 if w.dtype == "bf16" else 4
-    bwd_flops = 5.0 * w.B * w.H * w.T * w.T * w.d
-    bwd_bytes = 8.0 * w.B * w.T * w.H * w.d * esz + 8.0 * w.B * w.H * w.T
-    achieved_bwd = bwd_flops / (ms_bwd * 1e-3) / 1e12
-    clocks = clk.summary() if rank == 0 else {}
+    bwd_flops = 5.0 * w.B * w.H * w.T * w.T * w.d  # causal bwd incl. the U recompute
+    tiles_tflops = bwd_flops / (ms_tiles * 1e-3) / 1e12
+    fwd_tflops = w.flops_fwd() / (ms_fwd * 1e-3) / 1e12
+    kname = "bwd_tc_kernel" if family != "simt" and w.dtype == "bf16" else "bwd_dkdv+dq (simt)"
+    traffic = _profiled_traffic(w, "bwd_tc_kernel") if kname == "bwd_tc_kernel" else None
+    clocks = clk.summary(t_begin, t_end) if rank == 0 else {}
     line = {
         "metric": "FlashRelation fwd+bwd TFLOP/s (7*B*H*T^2*d causal)",
         "value": tflops, "unit": "TFLOP/s", "n_gpus": ws, "steps": n, "warmup": args.warmup,
@@ -299,15 +350,18 @@ def run_ours(args, w):
         "pct_bf16_peak": 100.0 * tflops / (ws * peaks["bf16_tflops"]),
         "pct_bf16_peak_sustained": 100.0 * tflops / (ws * peaks["bf16_tflops_sustained"]),
         "ms_fwd": ms_fwd, "ms_bwd": ms_bwd,
-        "fwd_tflops": ws * w.flops_fwd() / (ms_fwd * 1e-3) / 1e12,
+        "ms_bwd_stages": {"prepare": ms_pre, "tiles": ms_tiles, "finalize": ms_fin},
+        "fwd_tflops": ws * fwd_tflops,
         "bwd_tflops": ws * bwd_flops / (ms_bwd * 1e-3) / 1e12,
-        "roofline": {"kernel": "relation_bwd (row pre-pass + Exchange tiles + dlambda reduce)",
-                     "bound": "tensor", "achieved": achieved_bwd,
+        "roofline": {"kernel": kname, "bound": "tensor", "achieved": tiles_tflops,
                      "peak": peaks["bf16_tflops"], "unit": "TFLOP/s",
-                     "frac": achieved_bwd / peaks["bf16_tflops"],
-                     "peak_source": peaks["source"] + " bf16 burst",
-                     "algorithmic_bytes": bwd_bytes,
-                     "achieved_gbs": bwd_bytes / (ms_bwd * 1e-3) / 1e9, "traffic": None},
+                     "frac": tiles_tflops / peaks["bf16_tflops"],
+                     "peak_source": f"{peaks['source']} dense bf16 (burst, cuBLAS)",
+                     "algorithmic_flops_per_launch": bwd_flops,
+                     "traffic": traffic,
+                     "algorithmic_bytes_per_launch": 8.0 * w.B * w.T * w.H * w.d * esz,
+                     "fwd_kernel": {"achieved": fwd_tflops,
+                                    "frac": fwd_tflops / peaks["bf16_tflops"]}},
         "e2e": {"value": ws * flops / (ms_e2e * 1e-3) / 1e12, "unit": "TFLOP/s",
                 "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h, "ms_per_step": ms_e2e},
         "gpu_launches": n * (binding.launches_per_call(family, w.dtype, w.d, "fwd")
@@ -315,11 +369,11 @@ def run_ours(args, w):
         "clocks": clocks,
     }
     if rank == 0 and not args.no_cpu_baseline and ws == 1:
-        cb = cpu_oracle_run(w)
+        cb = cpu_oracle_run(w, min_seconds=10.0)
         line["cpu_baseline"] = {
             "value": cb["tflops"], "unit": "TFLOP/s", "cores": cb["cores"], "kind": "oracle",
-            "sample": f"{cb['heads']} of {w.B * w.H} heads, fwd+bwd, fp64 C oracle, "
-                      f"{cb['seconds']:.1f} s"}
+            "sample": f"{cb['heads']} of {w.B * w.H} heads x {cb['reps']}, fwd+bwd, fp64 C "
+                      f"oracle (OpenMP over heads), {cb['seconds']:.1f} s"}
     if rank == 0:
         print(json.dumps(line), flush=True)
     if dist is not None:
@@ -330,7 +384,7 @@ def run_ours(args, w):
 def main(argv=None):
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
-    ap.add_argument("--steps", type=int, default=20)
+    ap.add_argument("--steps", type=int, default=400)
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--config", default="10M", choices=sorted(workloads.WORKLOADS))
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])

@@ -130,6 +130,23 @@ relation_status relation_bwd_ex(const void* q, const void* k, const void* v, con
  * request is not supported.  Host-only query. */
 int relation_launch_count(relation_dtype dt, int d_h, relation_kernel kernel, int backward);
 
+/* The backward as three stages, each launched only when its bit is set in `stages`:
+ *   RELATION_BWD_PREPARE  per-row pass: D_i = dO_i . Y_i, the Self quantities and the
+ *                         per-query scalars the tile stage reads (into the workspace)
+ *   RELATION_BWD_TILES    the causal tile loop producing dK, dV and the dQ accumulator
+ *   RELATION_BWD_FINALIZE dQ in the output dtype and the dlambda reduction
+ * Running the three in order on one stream (stages = RELATION_BWD_ALL) is relation_bwd_ex.
+ * The stages communicate through the workspace only; a stage assumes the earlier ones ran
+ * on the same arguments and workspace. */
+enum { RELATION_BWD_PREPARE = 1, RELATION_BWD_TILES = 2, RELATION_BWD_FINALIZE = 4,
+       RELATION_BWD_ALL = 7 };
+relation_status relation_bwd_stages(const void* q, const void* k, const void* v, const void* o,
+                                    const void* dout, const float* logz, void* dq, void* dk,
+                                    void* dv, float* dlambda, float lambda, float tau_s,
+                                    relation_shape shp, relation_dtype dt, void* workspace,
+                                    size_t ws_bytes, relation_kernel kernel, unsigned stages,
+                                    int* dev_status, relation_stream_t stream);
+
 /* Human-readable name of a status code (static string, never NULL). */
 const char* relation_status_string(relation_status s);
 

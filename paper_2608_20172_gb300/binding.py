@@ -28,7 +28,8 @@ KERNELS = {"auto": 0, "simt": 1, "tcgen05": 2}
 
 EXPORTED = ("relation_fwd", "relation_fwd_ex", "relation_bwd", "relation_bwd_ex",
             "relation_bwd_workspace_size", "relation_status_string", "relation_version",
-            "relation_selftest_wait_timeout", "relation_launch_count", "relation_last_cuda_error")
+            "relation_selftest_wait_timeout", "relation_launch_count", "relation_last_cuda_error",
+            "relation_bwd_stages")
 
 
 class RelationLibraryMissing(RuntimeError):
@@ -73,6 +74,9 @@ def load(path: str | None = None):
                                      sz, ip, vp]
         lib.relation_bwd_ex.argtypes = [vp, vp, vp, vp, vp, vp, vp, vp, vp, vp, f, f, Shape, i,
                                         vp, sz, i, ip, vp]
+        lib.relation_bwd_stages.argtypes = [vp, vp, vp, vp, vp, vp, vp, vp, vp, vp, f, f, Shape,
+                                            i, vp, sz, i, ctypes.c_uint, ip, vp]
+        lib.relation_bwd_stages.restype = ctypes.c_int
         lib.relation_bwd_workspace_size.argtypes = [Shape, i]
         lib.relation_bwd_workspace_size.restype = sz
         lib.relation_status_string.argtypes = [i]
@@ -152,9 +156,14 @@ def fwd(q, k, v, lam: float, tau_s: float = 2.0, *, kernel: str = "auto", out=No
     return out, logz
 
 
+BWD_PREPARE, BWD_TILES, BWD_FINALIZE, BWD_ALL = 1, 2, 4, 7
+
+
 def bwd(q, k, v, o, dout, logz, lam: float, tau_s: float = 2.0, *, kernel: str = "auto",
-        workspace=None, dq=None, dk=None, dv=None, dlambda=None, dev_status=None, stream=None):
-    """Backward.  Returns (dQ, dK, dV, dlambda) with dlambda a 1-element fp32 device tensor."""
+        workspace=None, dq=None, dk=None, dv=None, dlambda=None, dev_status=None, stream=None,
+        stages: int = BWD_ALL):
+    """Backward.  Returns (dQ, dK, dV, dlambda) with dlambda a 1-element fp32 device tensor.
+    ``stages`` selects a subset of the three backward stages (see relation_bwd_stages)."""
     _same_layout(q, k, v, o, dout)
     dq = torch.empty_like(q) if dq is None else dq
     dk = torch.empty_like(q) if dk is None else dk
@@ -165,12 +174,12 @@ def bwd(q, k, v, o, dout, logz, lam: float, tau_s: float = 2.0, *, kernel: str =
     need = workspace_size(q)
     if workspace is None:
         workspace = torch.empty(need, device=q.device, dtype=torch.uint8)
-    rc = load().relation_bwd_ex(_ptr(q), _ptr(k), _ptr(v), _ptr(o), _ptr(dout), _ptr(logz),
-                                _ptr(dq), _ptr(dk), _ptr(dv), _ptr(dlambda), float(lam),
-                                float(tau_s), shape_of(q), _dtype_code(q),
-                                _ptr(workspace), workspace.numel() * workspace.element_size(),
-                                KERNELS[kernel], _ptr(dev_status),
-                                ctypes.c_void_p(_stream(stream)))
+    rc = load().relation_bwd_stages(_ptr(q), _ptr(k), _ptr(v), _ptr(o), _ptr(dout), _ptr(logz),
+                                    _ptr(dq), _ptr(dk), _ptr(dv), _ptr(dlambda), float(lam),
+                                    float(tau_s), shape_of(q), _dtype_code(q),
+                                    _ptr(workspace), workspace.numel() * workspace.element_size(),
+                                    KERNELS[kernel], int(stages), _ptr(dev_status),
+                                    ctypes.c_void_p(_stream(stream)))
     if rc != OK:
         raise RelationError(rc, "relation_bwd")
     return dq, dk, dv, dlambda

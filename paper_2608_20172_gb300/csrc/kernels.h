@@ -72,8 +72,9 @@ namespace tc {
 bool supports(relation_dtype dt, int d);      // forward
 bool supports_bwd(relation_dtype dt, int d);  // backward
 cudaError_t launch_fwd(const Problem& p, cudaStream_t s);
-cudaError_t launch_bwd(const Problem& p, const BwdWorkspace& ws, cudaStream_t s);  // whole bwd
-int bwd_launches();  // launches made by launch_bwd
+// Backward stages (bit 1: row pass, 2: tile kernel, 4: finalisation).
+cudaError_t launch_bwd(const Problem& p, const BwdWorkspace& ws, unsigned stages, cudaStream_t s);
+int bwd_launches();  // launches made by launch_bwd with every stage
 int main_ctas(const Problem& p);
 }  // namespace tc
 

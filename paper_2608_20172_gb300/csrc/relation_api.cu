@@ -115,12 +115,14 @@ size_t relation_bwd_workspace_size(relation_shape shp, relation_dtype dt) {
   return rel::bwd_workspace_bytes(shp.B, shp.H, shp.T, shp.d_h);
 }
 
-relation_status relation_bwd_ex(const void* q, const void* k, const void* v, const void* o,
-                                const void* dout, const float* logz, void* dq, void* dk, void* dv,
-                                float* dlambda, float lambda, float tau_s, relation_shape shp,
-                                relation_dtype dt, void* workspace, size_t ws_bytes,
-                                relation_kernel kernel, int* dev_status, relation_stream_t stream) {
+relation_status relation_bwd_stages(const void* q, const void* k, const void* v, const void* o,
+                                    const void* dout, const float* logz, void* dq, void* dk,
+                                    void* dv, float* dlambda, float lambda, float tau_s,
+                                    relation_shape shp, relation_dtype dt, void* workspace,
+                                    size_t ws_bytes, relation_kernel kernel, unsigned stages,
+                                    int* dev_status, relation_stream_t stream) {
   relation_status st;
+  if (stages == 0 || (stages & ~7u)) return RELATION_ERR_INVALID_ARG;
   if ((st = check_shape(shp, dt)) != RELATION_OK) return st;
   if ((st = check_scalars(lambda, tau_s)) != RELATION_OK) return st;
   if ((st = check_ptrs({q, k, v, o, dout, logz, dq, dk, dv})) != RELATION_OK) return st;
@@ -138,12 +140,21 @@ relation_status relation_bwd_ex(const void* q, const void* k, const void* v, con
   p.dq = dq; p.dk = dk; p.dv = dv; p.dlambda = dlambda;
   rel::BwdWorkspace ws = rel::carve_workspace(workspace, shp.B, shp.H, shp.T, shp.d_h);
   cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
-  if (fam == 2) return from_cuda(rel::tc::launch_bwd(p, ws, s));  // row pass, tiles, finalise
-  cudaError_t e = rel::bwd_common::launch_pre(p, ws, s);
-  if (e != cudaSuccess) return from_cuda(e);
-  e = rel::simt::launch_bwd(p, ws, s);
-  if (e != cudaSuccess) return from_cuda(e);
-  return from_cuda(rel::bwd_common::launch_dlambda(p, ws, rel::simt::main_ctas(p), s));
+  if (fam == 2) return from_cuda(rel::tc::launch_bwd(p, ws, stages, s));
+  cudaError_t e = cudaSuccess;
+  if ((stages & 1) && (e = rel::bwd_common::launch_pre(p, ws, s)) != cudaSuccess) return from_cuda(e);
+  if ((stages & 2) && (e = rel::simt::launch_bwd(p, ws, s)) != cudaSuccess) return from_cuda(e);
+  if (stages & 4) e = rel::bwd_common::launch_dlambda(p, ws, rel::simt::main_ctas(p), s);
+  return from_cuda(e);
+}
+
+relation_status relation_bwd_ex(const void* q, const void* k, const void* v, const void* o,
+                                const void* dout, const float* logz, void* dq, void* dk, void* dv,
+                                float* dlambda, float lambda, float tau_s, relation_shape shp,
+                                relation_dtype dt, void* workspace, size_t ws_bytes,
+                                relation_kernel kernel, int* dev_status, relation_stream_t stream) {
+  return relation_bwd_stages(q, k, v, o, dout, logz, dq, dk, dv, dlambda, lambda, tau_s, shp, dt,
+                             workspace, ws_bytes, kernel, RELATION_BWD_ALL, dev_status, stream);
 }
 
 relation_status relation_bwd(const void* q, const void* k, const void* v, const void* o,

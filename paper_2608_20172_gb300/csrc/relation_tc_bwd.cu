@@ -628,46 +628,55 @@ static bool make_tmap_dq(CUtensorMap* m, float* base, int rows, int d) {
 }
 
 template <int D>
-static cudaError_t bwd_t(const Problem& p, const BwdWorkspace& ws, cudaStream_t s) {
+static cudaError_t bwd_t(const Problem& p, const BwdWorkspace& ws, unsigned stages,
+                         cudaStream_t s) {
   const int n_t = (p.T + 127) / 128;
   const int t_pad = ws.t_pad;
-  // A runtime call first: it makes the device's primary context current on this thread,
-  // which the driver's tensor-map encoder needs (e.g. on a fresh autograd worker thread).
-  const int smem = bwd::Cfg<D>::SMEM;
-  cudaError_t e = cudaFuncSetAttribute(bwd::bwd_tc_kernel<D>,
-                                       cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
-  if (e != cudaSuccess) { note_failure("backward: shared memory attribute"); return e; }
-  CUtensorMap mq, mk, mv, mg, mdq;
-  if (!make_tmap_bf16(&mq, p.q, p, 128) || !make_tmap_bf16(&mk, p.k, p, 128) ||
-      !make_tmap_bf16(&mv, p.v, p, 128) || !make_tmap_bf16(&mg, p.dout, p, 128)) {
-    note_failure("backward: TMA descriptor of Q/K/V/dO");
-    return cudaErrorInvalidValue;
-  }
-  if (!make_tmap_dq(&mdq, ws.dq_acc, p.B * p.H * t_pad, D)) {
-    note_failure("backward: TMA descriptor of the dQ accumulator");
-    return cudaErrorInvalidValue;
-  }
   const long long rows = (long long)p.B * p.H * p.T;
-  const long long rows_pad = (long long)p.B * p.H * t_pad;
-  bwd::pre_kernel<D><<<(unsigned)((rows_pad * 8 + 255) / 256), 256, 0, s>>>(p, ws, n_t);
-  if ((e = cudaGetLastError()) != cudaSuccess) { note_failure("backward: row pass launch"); return e; }
   const long long grid = (long long)n_t * p.B * p.H;
   if (grid > 0x7fffffffLL) return cudaErrorInvalidConfiguration;
-  bwd::bwd_tc_kernel<D><<<(unsigned)grid, bwd::kThreads, smem, s>>>(mq, mk, mv, mg, mdq, p, ws,
-                                                                   n_t, t_pad);
-  if ((e = cudaGetLastError()) != cudaSuccess) { note_failure("backward: tile kernel launch"); return e; }
-  const long long chunks = rows * (D / 8);
-  const long long fblocks = (chunks + 255) / 256;
-  bwd::finalize_kernel<D><<<(unsigned)(fblocks > 0 ? fblocks : 1), 256, 0, s>>>(p, ws, (int)grid);
-  if ((e = cudaGetLastError()) != cudaSuccess) note_failure("backward: finalisation launch");
+  cudaError_t e = cudaSuccess;
+  if (stages & 1) {
+    const long long rows_pad = (long long)p.B * p.H * t_pad;
+    bwd::pre_kernel<D><<<(unsigned)((rows_pad * 8 + 255) / 256), 256, 0, s>>>(p, ws, n_t);
+    if ((e = cudaGetLastError()) != cudaSuccess) { note_failure("backward: row pass launch"); return e; }
+  }
+  if (stages & 2) {
+    // A runtime call first: it makes the device's primary context current on this thread,
+    // which the driver's tensor-map encoder needs (e.g. on a fresh autograd worker thread).
+    const int smem = bwd::Cfg<D>::SMEM;
+    e = cudaFuncSetAttribute(bwd::bwd_tc_kernel<D>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                             smem);
+    if (e != cudaSuccess) { note_failure("backward: shared memory attribute"); return e; }
+    CUtensorMap mq, mk, mv, mg, mdq;
+    if (!make_tmap_bf16(&mq, p.q, p, 128) || !make_tmap_bf16(&mk, p.k, p, 128) ||
+        !make_tmap_bf16(&mv, p.v, p, 128) || !make_tmap_bf16(&mg, p.dout, p, 128)) {
+      note_failure("backward: TMA descriptor of Q/K/V/dO");
+      return cudaErrorInvalidValue;
+    }
+    if (!make_tmap_dq(&mdq, ws.dq_acc, p.B * p.H * t_pad, D)) {
+      note_failure("backward: TMA descriptor of the dQ accumulator");
+      return cudaErrorInvalidValue;
+    }
+    bwd::bwd_tc_kernel<D><<<(unsigned)grid, bwd::kThreads, smem, s>>>(mq, mk, mv, mg, mdq, p, ws,
+                                                                     n_t, t_pad);
+    if ((e = cudaGetLastError()) != cudaSuccess) { note_failure("backward: tile kernel launch"); return e; }
+  }
+  if (stages & 4) {
+    const long long chunks = rows * (D / 8);
+    const long long fblocks = (chunks + 255) / 256;
+    bwd::finalize_kernel<D><<<(unsigned)(fblocks > 0 ? fblocks : 1), 256, 0, s>>>(p, ws, (int)grid);
+    if ((e = cudaGetLastError()) != cudaSuccess) note_failure("backward: finalisation launch");
+  }
   return e;
 }
 
 bool supports_bwd(relation_dtype dt, int d) { return dt == RELATION_BF16 && (d == 64 || d == 128); }
 
-cudaError_t launch_bwd(const Problem& p, const BwdWorkspace& ws, cudaStream_t s) {
-  if (p.d == 64) return bwd_t<64>(p, ws, s);
-  if (p.d == 128) return bwd_t<128>(p, ws, s);
+cudaError_t launch_bwd(const Problem& p, const BwdWorkspace& ws, unsigned stages,
+                       cudaStream_t s) {
+  if (p.d == 64) return bwd_t<64>(p, ws, stages, s);
+  if (p.d == 128) return bwd_t<128>(p, ws, stages, s);
   return cudaErrorInvalidValue;
 }
 int bwd_launches() { return 3; }
