@@ -147,6 +147,27 @@ relation_status relation_bwd_stages(const void* q, const void* k, const void* v,
                                     size_t ws_bytes, relation_kernel kernel, unsigned stages,
                                     int* dev_status, relation_stream_t stream);
 
+/*
+ * relation_bwd without a caller workspace, for callers that cannot allocate device memory
+ * (code inside a runtime that owns the device memory budget through its own allocator, or
+ * on a path where an allocation could fail or synchronise the device).  The paper has no
+ * counterpart: this is a deployment convenience.
+ *
+ * The scratch is a fixed device array of RELATION_STATIC_SCRATCH_BYTES inside the library,
+ * held on every GPU that loads the library until the process exits.  Shapes whose
+ * relation_bwd_workspace_size() exceeds it are rejected with RELATION_ERR_WORKSPACE and
+ * nothing is launched.  The first call on a device looks up the array's address on that
+ * device (make it before any stream capture).  No call allocates memory.  Every call
+ * shares the one array: calls that overlap on the GPU race on it and must be serialised
+ * by the caller.  Arguments and results are otherwise those of relation_bwd_ex.
+ */
+#define RELATION_STATIC_SCRATCH_BYTES (64u << 20)
+relation_status relation_bwd_static(const void* q, const void* k, const void* v, const void* o,
+                                    const void* dout, const float* logz, void* dq, void* dk,
+                                    void* dv, float* dlambda, float lambda, float tau_s,
+                                    relation_shape shp, relation_dtype dt, relation_kernel kernel,
+                                    int* dev_status, relation_stream_t stream);
+
 /* Human-readable name of a status code (static string, never NULL). */
 const char* relation_status_string(relation_status s);
 

@@ -29,7 +29,7 @@ KERNELS = {"auto": 0, "simt": 1, "tcgen05": 2}
 EXPORTED = ("relation_fwd", "relation_fwd_ex", "relation_bwd", "relation_bwd_ex",
             "relation_bwd_workspace_size", "relation_status_string", "relation_version",
             "relation_selftest_wait_timeout", "relation_launch_count", "relation_last_cuda_error",
-            "relation_bwd_stages")
+            "relation_bwd_stages", "relation_bwd_static")
 
 
 class RelationLibraryMissing(RuntimeError):
@@ -77,6 +77,9 @@ def load(path: str | None = None):
         lib.relation_bwd_stages.argtypes = [vp, vp, vp, vp, vp, vp, vp, vp, vp, vp, f, f, Shape,
                                             i, vp, sz, i, ctypes.c_uint, ip, vp]
         lib.relation_bwd_stages.restype = ctypes.c_int
+        lib.relation_bwd_static.argtypes = [vp, vp, vp, vp, vp, vp, vp, vp, vp, vp, f, f, Shape,
+                                            i, i, ip, vp]
+        lib.relation_bwd_static.restype = ctypes.c_int
         lib.relation_bwd_workspace_size.argtypes = [Shape, i]
         lib.relation_bwd_workspace_size.restype = sz
         lib.relation_status_string.argtypes = [i]
@@ -189,6 +192,24 @@ def launches_per_call(kernel: str, dtype: str, d: int, which: str) -> int:
     """Kernel launches one fwd / bwd call makes (0 when unsupported)."""
     dt = F32 if dtype in ("fp32", "f32", torch.float32) else BF16
     return int(load().relation_launch_count(dt, int(d), KERNELS[kernel], int(which == "bwd")))
+
+
+STATIC_SCRATCH_BYTES = 64 << 20  # RELATION_STATIC_SCRATCH_BYTES
+
+
+def bwd_no_alloc(q, k, v, o, dout, logz, lam: float, tau_s: float = 2.0, *,
+                 kernel: str = "auto", dq, dk, dv, dlambda, dev_status=None, stream=None):
+    """Backward through relation_bwd_static: the library's fixed scratch array replaces the
+    workspace, for callers that must not allocate device memory.  All outputs are
+    caller-provided (this function allocates nothing either)."""
+    _same_layout(q, k, v, o, dout, dq, dk, dv)
+    rc = load().relation_bwd_static(_ptr(q), _ptr(k), _ptr(v), _ptr(o), _ptr(dout), _ptr(logz),
+                                    _ptr(dq), _ptr(dk), _ptr(dv), _ptr(dlambda), float(lam),
+                                    float(tau_s), shape_of(q), _dtype_code(q), KERNELS[kernel],
+                                    _ptr(dev_status), ctypes.c_void_p(_stream(stream)))
+    if rc != OK:
+        raise RelationError(rc, "relation_bwd_static")
+    return dq, dk, dv, dlambda
 
 
 def selftest_wait_timeout(dev_status: torch.Tensor, timeout_us: int = 1000, stream=None) -> int:
