@@ -65,6 +65,69 @@ __device__ __forceinline__ void drain_wait(uint32_t bar, uint32_t parity) {
 
 __device__ __forceinline__ float silu_acc(float x) { return x / (1.0f + __expf(-x)); }
 
+__device__ __forceinline__ float fmax3(float a, float b, float c) {
+  float d;
+  asm("max.f32 %0, %1, %2, %3;" : "=f"(d) : "f"(a), "f"(b), "f"(c));
+  return d;
+}
+
+// Maximum of the raw evidence U over the row's history; on the diagonal tile only the
+// columns c < t count and U[t] (the Self evidence U_ii) is returned in u_self.
+template <bool DIAG>
+__device__ __forceinline__ float row_max(const uint32_t (&U)[BN], int t, float& u_self) {
+  if (!DIAG) {
+    float m0 = __uint_as_float(U[0]), m1 = __uint_as_float(U[1]);
+    float m2 = __uint_as_float(U[2]), m3 = __uint_as_float(U[3]);
+#pragma unroll
+    for (int c = 4; c < BN; c += 8) {
+      m0 = fmax3(m0, __uint_as_float(U[c]), __uint_as_float(U[c + 1]));
+      m1 = fmax3(m1, __uint_as_float(U[c + 2]), __uint_as_float(U[c + 3]));
+      m2 = fmax3(m2, __uint_as_float(U[c + 4]), __uint_as_float(U[c + 5]));
+      m3 = fmax3(m3, __uint_as_float(U[c + 6]), __uint_as_float(U[c + 7]));
+    }
+    return fmaxf(fmax3(m0, m1, m2), m3);
+  }
+  float m = -INFINITY;
+#pragma unroll
+  for (int c = 0; c < BN; ++c) {
+    const float x = __uint_as_float(U[c]);
+    m = c < t ? fmaxf(m, x) : m;
+    u_self = c == t ? x : u_self;
+  }
+  return m;
+}
+
+// P = 2^(U c2k (1 + tanh(U ch)) - m) for the 128 keys of the tile (0 off the history on
+// the diagonal tile), written to TMEM as bf16 pairs; returns the row sum as two halves.
+template <bool DIAG>
+__device__ __forceinline__ float2 scan_p(const uint32_t (&U)[BN], int t, uint32_t trow, float ch,
+                                         float c2k, float negm) {
+  const float2 ch2 = make_float2(ch, ch), c2k2 = make_float2(c2k, c2k);
+  const float2 nm2 = make_float2(negm, negm);
+  float2 sum = make_float2(0.f, 0.f);
+#pragma unroll
+  for (int c0 = 0; c0 < BN; c0 += 32) {
+    uint32_t pk[16];
+#pragma unroll
+    for (int c = 0; c < 32; c += 2) {
+      const float2 x = make_float2(__uint_as_float(U[c0 + c]), __uint_as_float(U[c0 + c + 1]));
+      const float2 h = __fmul2_rn(x, ch2);
+      const float2 th = make_float2(tanh_approx(h.x), tanh_approx(h.y));
+      const float2 w = __ffma2_rn(th, c2k2, c2k2);  // log2(e) sigma(u) / sqrt(d), times 2
+      const float2 e = __ffma2_rn(x, w, nm2);
+      float2 pv = make_float2(ex2_approx(e.x), ex2_approx(e.y));
+      if (DIAG) {
+        pv.x = (c0 + c < t) ? pv.x : 0.f;
+        pv.y = (c0 + c + 1 < t) ? pv.y : 0.f;
+      }
+      sum = __fadd2_rn(sum, pv);
+      pk[c >> 1] = pack_bf16x2(pv.x, pv.y);
+    }
+    tmem_st16(trow + kSCol + (c0 >> 1), pk);
+  }
+  return sum;
+}
+
 template <int D>
 __global__ void __launch_bounds__(kThreads, 2)
     fwd_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmK,
@@ -185,7 +248,7 @@ __global__ void __launch_bounds__(kThreads, 2)
     const uint32_t trow = tmem + ((uint32_t)(warp * 32) << 16);
     const float isd = p.inv_sqrt_d;
     const float ch = 0.5f * isd;            // h = U * ch = u / 2
-    const float c2 = ch * kLog2e;           // E log2(e) = U * c2 * (1 + tanh(h))
+    const float c2k = ch * kLog2e;          // E log2(e) = U * c2k * (1 + tanh(h))
     float m = -INFINITY;                    // running bound of max E, log2 units
     float l = 0.f;
     float u_self = 0.f;
@@ -201,15 +264,9 @@ __global__ void __launch_bounds__(kThreads, 2)
       tmem_ld32(trow + kSCol + 96, U + 96);
       tmem_ld_wait();
       const bool diag = (j == qt);
-      // pass 1: masked maximum of the raw evidence (keys j0 + c < row  <=>  c < t on the
-      // diagonal tile; every key of an earlier tile is history)
-      float umax = -INFINITY;
-#pragma unroll
-      for (int c = 0; c < BN; ++c) {
-        const float x = __uint_as_float(U[c]);
-        if (!diag || c < t) umax = fmaxf(umax, x);
-        if (diag && c == t) u_self = x;
-      }
+      // Pass 1: maximum of the raw evidence over the row's history (keys j0 + c < row,
+      // i.e. c < t on the diagonal tile; every key of an earlier tile), and U_ii.
+      const float umax = diag ? row_max<true>(U, t, u_self) : row_max<false>(U, t, u_self);
       // Upper bound of max E: SiLU is increasing on [0, inf) and negative on (-inf, 0).
       float mt;
       if (umax == -INFINITY) {
@@ -237,30 +294,11 @@ __global__ void __launch_bounds__(kThreads, 2)
           tmem_st16(trow + kOCol + c0 + 16, z + 16);
         }
       }
-      // pass 2: P = 2^(E log2 e - m) on the history, 0 elsewhere; written back as bf16
+      // Pass 2: P = 2^(E log2 e - m) on the history, 0 elsewhere; written back as bf16.
       const float negm = (m == -INFINITY) ? 0.f : -m;
-      float rowsum = 0.f;
-#pragma unroll
-      for (int c0 = 0; c0 < BN; c0 += 32) {
-        uint32_t pk[16];
-#pragma unroll
-        for (int c = 0; c < 32; c += 2) {
-          float pr[2];
-#pragma unroll
-          for (int e = 0; e < 2; ++e) {
-            const int cc = c0 + c + e;
-            const float x = __uint_as_float(U[cc]);
-            const float th = tanh_approx(x * ch);
-            const float w = fmaf(th, c2, c2);
-            float pv = ex2_approx(fmaf(x, w, negm));
-            if (diag && cc >= t) pv = 0.f;
-            pr[e] = pv;
-          }
-          rowsum += pr[0] + pr[1];
-          pk[c >> 1] = pack_bf16x2(pr[0], pr[1]);
-        }
-        tmem_st16(trow + kSCol + (c0 >> 1), pk);
-      }
+      const float2 rs = diag ? scan_p<true>(U, t, trow, ch, c2k, negm)
+                             : scan_p<false>(U, t, trow, ch, c2k, negm);
+      const float rowsum = rs.x + rs.y;
       l += rowsum;
       tmem_st_wait();
       tc_fence_before();
