@@ -10,13 +10,15 @@
 //   warp  4    TMA producer: Q tile once, then K and V tiles through a ring of stages.
 //   warp  5    TMEM allocator and MMA issuer (one elected thread).
 // Per key tile j:
-//   MMA   U_j = Q K_j^T                       -> TMEM columns [0, 128) (fp32)
+// The scan advances 64 keys per step through two TMEM buffers, so the MMAs of one step
+// (U of step s + 2, z += P V of step s) overlap the elementwise work of the next.  Step s:
+//   MMA   U = Q K^T over 64 keys                 -> TMEM columns [64 b, 64 b + 64), b = s & 1
 //   scan  E = SiLU(U / sqrt(d)) for keys < row (Self excluded); running maximum m (kept
 //         as an upper bound of max E, rescaling z only when it grows by > 2^8), row sum
-//         l += sum exp(E - m); P = exp(E - m) as bf16 written back into TMEM columns
-//         [0, 64) (two per 32-bit column); the diagonal tile also yields
+//         l += sum exp(E - m); P = exp(E - m) as bf16 written back into the buffer's
+//         first 32 columns (two per 32-bit column); the diagonal tile also yields
 //         S_i = sigmoid(U_ii / (sqrt(d) tau_S)).
-//   MMA   z += P V_j  (A operand P read from TMEM)  -> TMEM columns [128, 128 + d)
+//   MMA   z += P V  (A operand P read from TMEM)  -> TMEM columns [128, 128 + d)
 // Epilogue (App. A.3.3-A.3.5): L^E = m + log l, A = L^E - lambda log i,
 //   g = sigmoid(A - S), Y = (1 - g) v_i + g z / l, logZ = logaddexp(S, A); row 1 has an
 //   empty history: g = 0, Y = v_1, logZ = S_1 (App. A.1.8).
@@ -33,10 +35,11 @@ namespace rel {
 namespace tc {
 
 constexpr int BM = 128;        // query rows per CTA
-constexpr int BN = 128;        // keys per tile
+constexpr int BN = 128;        // keys per K/V tile (TMA granularity)
+constexpr int HN = 64;         // keys per scan step: two steps per K/V tile
 constexpr int kThreads = 192;  // 4 scan warps + TMA warp + MMA warp
-constexpr int kTmemCols = 256; // S/P tile (128) + z accumulator (<= 128)
-constexpr int kSCol = 0;
+constexpr int kTmemCols = 256; // two U/P buffers of 64 columns + z accumulator (<= 128)
+constexpr int kSCol = 0;       // buffer b at kSCol + 64 b
 constexpr int kOCol = 128;
 constexpr float kRescaleLog2 = 8.0f;  // rescale z only when the max grows by > 2^8
 
@@ -53,7 +56,9 @@ struct FwdCfg {
 };
 
 // mbarrier slots
-enum : int { B_Q = 0, B_KF = 1, B_KE = 3, B_VF = 5, B_VE = 7, B_S = 9, B_P = 10, B_O = 11 };
+enum : int {
+  B_Q = 0, B_KF = 1, B_KE = 3, B_VF = 5, B_VE = 7, B_S = 9, B_P = 11, B_O = 13, B_OD = 14
+};
 
 // Bounded wait used while draining at teardown: never raises, just gives up.
 __device__ __forceinline__ void drain_wait(uint32_t bar, uint32_t parity) {
@@ -74,12 +79,12 @@ __device__ __forceinline__ float fmax3(float a, float b, float c) {
 // Maximum of the raw evidence U over the row's history; on the diagonal tile only the
 // columns c < t count and U[t] (the Self evidence U_ii) is returned in u_self.
 template <bool DIAG>
-__device__ __forceinline__ float row_max(const uint32_t (&U)[BN], int t, float& u_self) {
+__device__ __forceinline__ float row_max(const uint32_t (&U)[HN], int t, float& u_self) {
   if (!DIAG) {
     float m0 = __uint_as_float(U[0]), m1 = __uint_as_float(U[1]);
     float m2 = __uint_as_float(U[2]), m3 = __uint_as_float(U[3]);
 #pragma unroll
-    for (int c = 4; c < BN; c += 8) {
+    for (int c = 4; c < HN; c += 8) {
       m0 = fmax3(m0, __uint_as_float(U[c]), __uint_as_float(U[c + 1]));
       m1 = fmax3(m1, __uint_as_float(U[c + 2]), __uint_as_float(U[c + 3]));
       m2 = fmax3(m2, __uint_as_float(U[c + 4]), __uint_as_float(U[c + 5]));
@@ -89,7 +94,7 @@ __device__ __forceinline__ float row_max(const uint32_t (&U)[BN], int t, float& 
   }
   float m = -INFINITY;
 #pragma unroll
-  for (int c = 0; c < BN; ++c) {
+  for (int c = 0; c < HN; ++c) {
     const float x = __uint_as_float(U[c]);
     m = c < t ? fmaxf(m, x) : m;
     u_self = c == t ? x : u_self;
@@ -97,16 +102,17 @@ __device__ __forceinline__ float row_max(const uint32_t (&U)[BN], int t, float& 
   return m;
 }
 
-// P = 2^(U c2k (1 + tanh(U ch)) - m) for the 128 keys of the tile (0 off the history on
-// the diagonal tile), written to TMEM as bf16 pairs; returns the row sum as two halves.
+// P = 2^(U c2k (1 + tanh(U ch)) - m) for the 64 keys of a step (0 off the history on
+// the diagonal tile), written to TMEM columns pcol.. as bf16 pairs; returns the row sum
+// as two halves.
 template <bool DIAG>
-__device__ __forceinline__ float2 scan_p(const uint32_t (&U)[BN], int t, uint32_t trow, float ch,
+__device__ __forceinline__ float2 scan_p(const uint32_t (&U)[HN], int t, uint32_t pcol, float ch,
                                          float c2k, float negm) {
   const float2 ch2 = make_float2(ch, ch), c2k2 = make_float2(c2k, c2k);
   const float2 nm2 = make_float2(negm, negm);
   float2 sum = make_float2(0.f, 0.f);
 #pragma unroll
-  for (int c0 = 0; c0 < BN; c0 += 32) {
+  for (int c0 = 0; c0 < HN; c0 += 32) {
     uint32_t pk[16];
 #pragma unroll
     for (int c = 0; c < 32; c += 2) {
@@ -123,7 +129,7 @@ __device__ __forceinline__ float2 scan_p(const uint32_t (&U)[BN], int t, uint32_
       sum = __fadd2_rn(sum, pv);
       pk[c >> 1] = pack_bf16x2(pv.x, pv.y);
     }
-    tmem_st16(trow + kSCol + (c0 >> 1), pk);
+    tmem_st16(pcol + (c0 >> 1), pk);
   }
   return sum;
 }
@@ -131,7 +137,8 @@ __device__ __forceinline__ float2 scan_p(const uint32_t (&U)[BN], int t, uint32_
 template <int D>
 __global__ void __launch_bounds__(kThreads, 2)
     fwd_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmK,
-                  const __grid_constant__ CUtensorMap tmV, Problem p, int n_qt) {
+                  const __grid_constant__ CUtensorMap tmV, const __grid_constant__ CUtensorMap tmO,
+                  Problem p, int n_qt) {
   using C = FwdCfg<D>;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>(
@@ -157,9 +164,12 @@ __global__ void __launch_bounds__(kThreads, 2)
       mbar_init(bar(B_VF + s), 1);
       mbar_init(bar(B_VE + s), 1);
     }
-    mbar_init(bar(B_S), 1);
-    mbar_init(bar(B_P), 128);
+    for (int bb = 0; bb < 2; ++bb) {
+      mbar_init(bar(B_S + bb), 1);
+      mbar_init(bar(B_P + bb), 128);
+    }
     mbar_init(bar(B_O), 1);
+    mbar_init(bar(B_OD), 1);
     *abort_flag = 0;
     fence_mbar_init();
   }
@@ -210,33 +220,48 @@ __global__ void __launch_bounds__(kThreads, 2)
   } else if (warp == 5) {
     // ------------------------------------------------------------------ MMA issuer
     if (lane == 0) {
-      constexpr uint32_t idesc_qk = idesc_bf16_f32(BM, BN, false, false);
+      constexpr uint32_t idesc_qk = idesc_bf16_f32(BM, HN, false, false);
       constexpr uint32_t idesc_pv = idesc_bf16_f32(BM, D, false, true);
-      bool ok = mbar_wait(bar(B_Q), 0, ab);
-      tc_fence_after();
-      for (int j = 0; ok && j < n_kv; ++j) {
-        const int s = j % C::STAGES, u = j / C::STAGES;
-        if (!(ok = mbar_wait(bar(B_KF + s), u & 1, ab))) break;
-        tc_fence_after();
+      const int total = 2 * n_kv;  // scan steps: two 64-key halves per K/V tile
+      // U of step s = Q K^T over keys [64 (s & 1), +64) of tile s / 2, into buffer s & 1
+      auto issue_u = [&](int s) -> bool {
+        const int j = s >> 1, hh = s & 1, st = j % C::STAGES;
+        if (hh == 0) {
+          if (!mbar_wait(bar(B_KF + st), (j / C::STAGES) & 1, ab)) return false;
+          tc_fence_after();
+        }
 #pragma unroll
         for (int kk = 0; kk < D / 16; ++kk) {
-          const uint32_t koff = (kk >> 2) * (BM * 128) + (kk & 3) * 32;
+          const uint32_t koff = (kk >> 2) * (BN * 128) + (kk & 3) * 32;
           const uint64_t a = smem_desc_sw128(sb + C::OFF_Q + koff, 16, 1024);
-          const uint64_t bd = smem_desc_sw128(sb + C::OFF_K + s * C::TILE + koff, 16, 1024);
-          mma_ss(tmem + kSCol, a, bd, idesc_qk, kk > 0 ? 1u : 0u);
-        }
-        mma_commit(bar(B_S));       // U_j ready (and every earlier z update done)
-        mma_commit(bar(B_KE + s));  // K stage free
-        if (!(ok = mbar_wait(bar(B_VF + s), u & 1, ab))) break;
-        if (!(ok = mbar_wait(bar(B_P), j & 1, ab))) break;
-        tc_fence_after();
-#pragma unroll
-        for (int kk = 0; kk < BN / 16; ++kk) {
           const uint64_t bd =
-              smem_desc_sw128(sb + C::OFF_V + s * C::TILE + kk * 16 * 128, BN * 128, 1024);
-          mma_ts(tmem + kOCol, tmem + kSCol + kk * 8, bd, idesc_pv, (j > 0 || kk > 0) ? 1u : 0u);
+              smem_desc_sw128(sb + C::OFF_K + st * C::TILE + hh * HN * 128 + koff, 16, 1024);
+          mma_ss(tmem + kSCol + hh * HN, a, bd, idesc_qk, kk > 0 ? 1u : 0u);
         }
-        mma_commit(bar(B_VE + s));  // V stage free
+        mma_commit(bar(B_S + hh));  // U ready (and every earlier z update done)
+        if (hh == 1) mma_commit(bar(B_KE + st));  // K stage free
+        return true;
+      };
+      bool ok = mbar_wait(bar(B_Q), 0, ab);
+      tc_fence_after();
+      if (ok) ok = issue_u(0);
+      if (ok && total > 1) ok = issue_u(1);
+      for (int s = 0; ok && s < total; ++s) {
+        const int j = s >> 1, hh = s & 1, st = j % C::STAGES;
+        if (hh == 0 && !(ok = mbar_wait(bar(B_VF + st), (j / C::STAGES) & 1, ab))) break;
+        if (!(ok = mbar_wait(bar(B_P + hh), (s >> 1) & 1, ab))) break;
+        tc_fence_after();
+        // z += P V over the step's 64 keys (A = P from TMEM; B = V rows, N = d contiguous)
+#pragma unroll
+        for (int kk = 0; kk < HN / 16; ++kk) {
+          const uint64_t bd = smem_desc_sw128(
+              sb + C::OFF_V + st * C::TILE + (hh * HN + kk * 16) * 128, BN * 128, 1024);
+          mma_ts(tmem + kOCol, tmem + kSCol + hh * HN + kk * 8, bd, idesc_pv,
+                 (s > 0 || kk > 0) ? 1u : 0u);
+        }
+        mma_commit(bar(B_OD));  // z update of step s done
+        if (hh == 1) mma_commit(bar(B_VE + st));  // V stage free
+        if (s + 2 < total && !(ok = issue_u(s + 2))) break;  // buffer hh: P read above
       }
       mma_commit(bar(B_O));  // z final (or whatever completed before an abort)
     }
@@ -253,20 +278,21 @@ __global__ void __launch_bounds__(kThreads, 2)
     float l = 0.f;
     float u_self = 0.f;
     bool ok = true;
-    for (int j = 0; j < n_kv; ++j) {
-      ok = __all_sync(0xffffffffu, mbar_wait(bar(B_S), j & 1, ab));  // warp-uniform
+    for (int s = 0; s < 2 * n_kv; ++s) {
+      const int j = s >> 1, hh = s & 1;
+      ok = __all_sync(0xffffffffu, mbar_wait(bar(B_S + hh), (s >> 1) & 1, ab));  // warp-uniform
       if (!ok) break;
       tc_fence_after();
-      uint32_t U[BN];
-      tmem_ld32(trow + kSCol + 0, U + 0);
-      tmem_ld32(trow + kSCol + 32, U + 32);
-      tmem_ld32(trow + kSCol + 64, U + 64);
-      tmem_ld32(trow + kSCol + 96, U + 96);
+      const uint32_t ucol = trow + kSCol + hh * HN;
+      uint32_t U[HN];
+      tmem_ld32(ucol, U);
+      tmem_ld32(ucol + 32, U + 32);
       tmem_ld_wait();
       const bool diag = (j == qt);
-      // Pass 1: maximum of the raw evidence over the row's history (keys j0 + c < row,
-      // i.e. c < t on the diagonal tile; every key of an earlier tile), and U_ii.
-      const float umax = diag ? row_max<true>(U, t, u_self) : row_max<false>(U, t, u_self);
+      const int tl = t - hh * HN;  // this row's index relative to the step's first key
+      // Pass 1: maximum of the raw evidence over the row's history (on the diagonal tile
+      // only the keys before the row, c < tl; every key of an earlier tile), and U_ii.
+      const float umax = diag ? row_max<true>(U, tl, u_self) : row_max<false>(U, tl, u_self);
       // Upper bound of max E: SiLU is increasing on [0, inf) and negative on (-inf, 0).
       float mt;
       if (umax == -INFINITY) {
@@ -281,8 +307,12 @@ __global__ void __launch_bounds__(kThreads, 2)
       const float scale = grow ? exp2f(m - mn) : 1.0f;
       if (grow) m = mn;
       l *= scale;
-      if (j > 0 && __any_sync(0xffffffffu, grow)) {
-        // z (TMEM) is stable: U_j's commit came after the z update of tile j-1
+      if (s > 0 && __any_sync(0xffffffffu, grow)) {
+        // rescale z once the z update of step s-1 has landed (the one of step s waits
+        // for this step's P)
+        ok = __all_sync(0xffffffffu, mbar_wait(bar(B_OD), (s - 1) & 1, ab));
+        if (!ok) break;
+        tc_fence_after();
 #pragma unroll
         for (int c0 = 0; c0 < D; c0 += 32) {
           uint32_t z[32];
@@ -296,13 +326,12 @@ __global__ void __launch_bounds__(kThreads, 2)
       }
       // Pass 2: P = 2^(E log2 e - m) on the history, 0 elsewhere; written back as bf16.
       const float negm = (m == -INFINITY) ? 0.f : -m;
-      const float2 rs = diag ? scan_p<true>(U, t, trow, ch, c2k, negm)
-                             : scan_p<false>(U, t, trow, ch, c2k, negm);
-      const float rowsum = rs.x + rs.y;
-      l += rowsum;
+      const float2 rs = diag ? scan_p<true>(U, tl, ucol, ch, c2k, negm)
+                             : scan_p<false>(U, tl, ucol, ch, c2k, negm);
+      l += rs.x + rs.y;
       tmem_st_wait();
       tc_fence_before();
-      mbar_arrive(bar(B_P));
+      mbar_arrive(bar(B_P + hh));
     }
     // ---------------------------------------------------------------- epilogue
     if (ok) ok = __all_sync(0xffffffffu, mbar_wait(bar(B_O), 0, ab));
@@ -320,31 +349,45 @@ __global__ void __launch_bounds__(kThreads, 2)
       } else {
         lz = S;  // empty history (row 1)
       }
-      const long long base = (long long)b * p.sB + (long long)h * p.sH + (long long)r * p.sT;
-      const __nv_bfloat16* vrow = reinterpret_cast<const __nv_bfloat16*>(p.v) + base;
-      __nv_bfloat16* yrow = reinterpret_cast<__nv_bfloat16*>(p.out) + base;
+      // v_i from the diagonal tile's V rows, still in shared memory (row t of the stage,
+      // 128-byte swizzle); Y staged in the Q tile's space (free: every MMA has completed)
+      // and written by one TMA store of 32 rows per warp (rows >= T are clipped).
+      const uint8_t* vrow = smem + C::OFF_V + (qt % C::STAGES) * C::TILE + t * 128;
+      uint8_t* ystage = smem + C::OFF_Q + warp * (32 * D * 2) + lane * 128;
 #pragma unroll
       for (int c0 = 0; c0 < D; c0 += 32) {
         uint32_t z[32];
         tmem_ld32(trow + kOCol + c0, z);
         tmem_ld_wait();
-        if (r < p.T) {
+        const int kb = c0 >> 6;  // 64-column block of the tile
 #pragma unroll
-          for (int c8 = 0; c8 < 32; c8 += 8) {
-            const uint4 vv = *reinterpret_cast<const uint4*>(vrow + c0 + c8);
-            const uint32_t vw[4] = {vv.x, vv.y, vv.z, vv.w};
-            uint32_t yw[4];
+        for (int c8 = 0; c8 < 32; c8 += 8) {
+          const int chunk = ((c0 & 63) + c8) >> 3;  // 16-byte chunk within the 128-byte row
+          const uint4 vv = *reinterpret_cast<const uint4*>(vrow + kb * BN * 128 +
+                                                           ((chunk ^ (t & 7)) << 4));
+          const uint32_t vw[4] = {vv.x, vv.y, vv.z, vv.w};
+          uint32_t yw[4];
 #pragma unroll
-            for (int e = 0; e < 4; ++e) {
-              const float2 vf = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&vw[e]));
-              const float z0 = __uint_as_float(z[c8 + 2 * e]) * inv_l;
-              const float z1 = __uint_as_float(z[c8 + 2 * e + 1]) * inv_l;
-              yw[e] = pack_bf16x2(fmaf(g, z0 - vf.x, vf.x), fmaf(g, z1 - vf.y, vf.y));
-            }
-            *reinterpret_cast<uint4*>(yrow + c0 + c8) = make_uint4(yw[0], yw[1], yw[2], yw[3]);
+          for (int e = 0; e < 4; ++e) {
+            const float2 vf = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&vw[e]));
+            const float z0 = __uint_as_float(z[c8 + 2 * e]) * inv_l;
+            const float z1 = __uint_as_float(z[c8 + 2 * e + 1]) * inv_l;
+            yw[e] = pack_bf16x2(fmaf(g, z0 - vf.x, vf.x), fmaf(g, z1 - vf.y, vf.y));
           }
+          *reinterpret_cast<uint4*>(ystage + kb * (32 * 128) + ((chunk ^ (lane & 7)) << 4)) =
+              make_uint4(yw[0], yw[1], yw[2], yw[3]);
         }
       }
+      fence_async_smem();
+      __syncwarp();
+      if (lane == 0) {
+        for (int kb = 0; kb < C::KB; ++kb)
+          tma_store_4d(&tmO, sb + C::OFF_Q + warp * (32 * D * 2) + kb * (32 * 128), kb * 64,
+                       q0 + warp * 32, h, b);
+        tma_store_commit();
+        tma_store_wait_all();  // the staging buffer must outlive the store
+      }
+      __syncwarp();
       if (r < p.T) p.logz[(long long)bh * p.T + r] = lz;
     }
   }
@@ -399,16 +442,16 @@ static cudaError_t fwd_t(const Problem& p, cudaStream_t s) {
   cudaError_t e =
       cudaFuncSetAttribute(fwd_tc_kernel<D>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
   if (e != cudaSuccess) { note_failure("forward: shared memory attribute"); return e; }
-  CUtensorMap mq, mk, mv;
+  CUtensorMap mq, mk, mv, mo;
   if (!make_tmap_bf16(&mq, p.q, p, BM) || !make_tmap_bf16(&mk, p.k, p, BN) ||
-      !make_tmap_bf16(&mv, p.v, p, BN)) {
-    note_failure("forward: TMA descriptor of Q/K/V");
+      !make_tmap_bf16(&mv, p.v, p, BN) || !make_tmap_bf16(&mo, p.out, p, 32)) {
+    note_failure("forward: TMA descriptor of Q/K/V/Y");
     return cudaErrorInvalidValue;
   }
   const int n_qt = (p.T + BM - 1) / BM;
   const long long grid = (long long)n_qt * p.B * p.H;
   if (grid > 0x7fffffffLL) return cudaErrorInvalidConfiguration;
-  fwd_tc_kernel<D><<<(unsigned)grid, kThreads, smem, s>>>(mq, mk, mv, p, n_qt);
+  fwd_tc_kernel<D><<<(unsigned)grid, kThreads, smem, s>>>(mq, mk, mv, mo, p, n_qt);
   if ((e = cudaGetLastError()) != cudaSuccess) note_failure("forward: kernel launch");
   return e;
 }
