@@ -14,19 +14,21 @@
 // accumulator), the tile kernel, and a finalisation (dQ to bf16, dlambda reduction).
 //
 // Tile kernel: one CTA per 128 keys of one head, visiting query tiles from the diagonal
-// to the end of the sequence.  Keys sit on TMEM lanes.  Per step of W query columns:
+// to the end of the sequence.  Keys sit on TMEM lanes.  Per step of 64 query columns:
 //   MMA  U^T = K Q^T,  dP^T = V dO^T                          (TMEM, fp32)
 //   elementwise (thread = key): P = F in bf16 back into TMEM, dS' = 2 dS in bf16 into
 //        128-byte-swizzled shared memory, and the Exchange part of dlambda
 //   MMA  dV += P^T dO (P read from TMEM),  dK += dS'^T Q
-// and once per 128-query tile  MMA dQ_t = dS' K, which warps 8-11 stage through shared
-// memory and add to the fp32 accumulator with TMA reduce-add.
-//   d_h = 64 : W = 64 on two TMEM buffers: the MMAs of one buffer (dV, dK of the last
-//              step, U^T / dP^T of the next) overlap the elementwise work on the other.
-//   d_h = 128: W = 128 on one buffer (TMEM is full); dQ_t reuses the dP^T columns.
-// Both elementwise warpgroups split every step's columns.  A tcgen05.mma costs at least
-// ~46 cycles whatever its N (measured on GB300: N = 32, 64, 128 run at 35%, 66%, 99% of
-// the per-SM peak), so the steps keep N >= 64.
+// Two TMEM buffers of U^T / dP^T: the MMAs of one buffer (dV, dK of the last step, U^T /
+// dP^T of the next) overlap the elementwise work on the other; both elementwise
+// warpgroups work on every step.  dQ goes to an fp32 accumulator through TMA reduce-add,
+// staged by warps 8-11:
+//   d_h = 64 : dQ_t = dS' K once per 128-query tile, in TMEM columns of its own.
+//   d_h = 128: dQ^T = K^T dS'^T once per step (d on TMEM lanes), written into the step's
+//              dP^T columns after dK has read dS' (TMEM is full otherwise); the next U^T
+//              of the buffer is issued after it, the next dP^T after its read-out.
+// A tcgen05.mma costs at least ~46 cycles whatever its N (measured on GB300: N = 32, 64,
+// 128 run at 35%, 66%, 99% of the per-SM peak), so the steps keep N >= 64.
 // dlambda = sum_i log i g_i dR_ii - sum_{j<i} log i F_ii dR_ij (weights cancel the
 // rounding error of D_i; see aux_kernels.cu), reduced per CTA.
 #include <cudaTypedefs.h>
@@ -51,32 +53,46 @@ constexpr int W_DQ = 8, W_TMA = 12, W_MMA = 13;
 template <int D>
 struct Cfg {
   static constexpr int KB = D / 64;
-  static constexpr int TILE = 128 * D * 2;
-  static constexpr int NBUF = D == 64 ? 2 : 1;   // U^T / dP^T TMEM buffers
-  static constexpr int QW = D == 64 ? 64 : 128;  // query columns per step (both warpgroups
-                                                 // split them: QW / 2 each)
-  static constexpr int SPT = BT / QW;            // steps per query tile
-  static constexpr int QSTG = D == 64 ? 2 : 1;   // Q / dO tile stages
-  static constexpr int DSB = D == 64 ? 2 : 1;    // dS' buffers (by tile parity)
+  static constexpr int KVT = 128 * D * 2;  // one K or V tile
+  // Q / dO staging and the dQ product:
+  //   d_h = 64 : per 128-query tile (two stages); dQ_t = dS' K once per tile into its own
+  //              TMEM columns.
+  //   d_h = 128: per 64-query step (three stages); dQ^T = K^T dS'^T once per step into the
+  //              step's own dP^T columns, after dK has read dS' out of them.
+  static constexpr bool HALF = D == 128;
+  static constexpr int NBUF = 2;               // U^T / dP^T TMEM buffers
+  static constexpr int QW = 64;                // query columns per step
+  static constexpr int SPT = BT / QW;          // steps per query tile
+  static constexpr int QROWS = HALF ? QW : BT; // query rows per Q / dO stage
+  static constexpr int QSZ = QROWS * D * 2;    // bytes of one Q (or dO) stage (16 KB)
+  static constexpr int KBQ = QROWS * 128;      // stride of the 64-column blocks of a stage
+  static constexpr int NQS = HALF ? 3 : 2;     // Q / dO stages
+  static constexpr int SW = QROWS;             // per-query scalars of a stage: array stride
+  static constexpr int STB = 4 * SW * 4;       // bytes of one stage's scalars
+  static constexpr int DSZ = HALF ? 16384 : 32768;  // one dS' buffer (per step / per tile)
+  static constexpr int DQSLOTS = HALF ? 1 : 2;      // 4 KB staging slots per dQ warp
   static constexpr int OFF_K = 0;
-  static constexpr int OFF_V = OFF_K + TILE;
-  static constexpr int OFF_Q = OFF_V + TILE;
-  static constexpr int OFF_DO = OFF_Q + QSTG * TILE;
-  static constexpr int OFF_DS = OFF_DO + QSTG * TILE;
-  static constexpr int OFF_DQS = OFF_DS + DSB * 32768;     // 4 warps x 2 slots x 4 KB
-  static constexpr int OFF_STAT = OFF_DQS + 4 * 2 * 4096;  // QSTG x 4 x 128 floats
-  static constexpr int OFF_RED = OFF_STAT + QSTG * 4 * BT * 4;
+  static constexpr int OFF_V = OFF_K + KVT;
+  static constexpr int OFF_Q = OFF_V + KVT;
+  static constexpr int OFF_DO = OFF_Q + NQS * QSZ;
+  static constexpr int OFF_DS = OFF_DO + NQS * QSZ;
+  static constexpr int OFF_DQS = OFF_DS + 2 * DSZ;
+  static constexpr int OFF_STAT = OFF_DQS + 4 * DQSLOTS * 4096;
+  static constexpr int OFF_RED = OFF_STAT + NQS * STB;
   static constexpr int OFF_BAR = OFF_RED + 64;
   static constexpr int SMEM = OFF_BAR + 256 + 1024;
-  static constexpr int COL_DK = NBUF * 2 * QW;              // 256 / 256
-  static constexpr int COL_DV = COL_DK + D;                  // 320 / 384
-  static constexpr int COL_DQ = D == 64 ? 384 : QW;          // d = 128: the dP^T columns
+  static constexpr int COL_DK = NBUF * 2 * QW;  // 256
+  static constexpr int COL_DV = COL_DK + D;     // 320 / 384
+  static constexpr int COL_DQ = 384;            // d_h = 64 only
   __host__ __device__ static constexpr int col_u(int b) { return b * 2 * QW; }
   __host__ __device__ static constexpr int col_g(int b) { return b * 2 * QW + QW; }
+  // Q / dO stage unit of a step: the step itself (d_h = 128) or its query tile
+  __host__ __device__ static constexpr int unit_of(int s) { return HALF ? s : s / SPT; }
 };
+static_assert(Cfg<64>::SMEM <= 232448 && Cfg<128>::SMEM <= 232448, "shared memory");
 
 enum : int {
-  B_KV = 0, B_QF = 1, B_QE = 3, B_S = 5, B_P = 7, B_DQF = 9, B_DQE = 10, B_ACC = 11
+  B_KV = 0, B_QF = 1, B_QE = 4, B_S = 7, B_P = 9, B_DQF = 11, B_DQE = 13, B_ACC = 15
 };
 
 __device__ __forceinline__ void drain_wait(uint32_t bar, uint32_t parity) {
@@ -104,6 +120,9 @@ __device__ __forceinline__ void bulk_load(uint32_t dst, const void* src, uint32_
 __device__ __forceinline__ void bulk_wait_read_le1() {
   asm volatile("cp.async.bulk.wait_group.read 1;" ::: "memory");
 }
+__device__ __forceinline__ void bulk_wait_read_0() {
+  asm volatile("cp.async.bulk.wait_group.read 0;" ::: "memory");
+}
 
 // Per-thread constants of the elementwise step.
 struct EwConst {
@@ -114,26 +133,27 @@ struct EwConst {
   float li;       // log(i) of this thread's own row (the Self entry on the diagonal)
 };
 
-// Elementwise work on 32 query columns of one key row (this thread's key).  st holds the
-// tile's per-query scalars, structure of arrays: [0,128) c2 = (-lambda log i - logZ_i)
-// log2 e, [128,256) -D_i, [256,384) -log i F_ii, [384,512) -logZ_i log2 e.
+// Elementwise work on 32 query columns of one key row (this thread's key t).  st points at
+// the chunk's first query in the stage's per-query scalars, four arrays of stride SW:
+// [0] c2 = (-lambda log i - logZ_i) log2 e, [SW] -D_i, [2 SW] -log i F_ii,
+// [3 SW] -logZ_i log2 e.  qt0 is the tile-local index of the chunk's first query.
 // Produces P = F_ij and dS' = 2 dS_ij as bf16 pairs and accumulates the dlambda terms.
 //   Exchange:  P = 2^(U c2k (1 + t) + c2),  t = tanh(u/2),
 //              2 SiLU'(u) = a (1 + h (1 - t)) with a = 1 + t, h = u / 2.
 //   Self (DIAG, query == key):  S = (1 + tanh(u / (2 tau_S))) / 2 = a / 2,
 //              P = 2^(S log2 e - logZ log2 e),  2 dS/du = a (1 - t) / (2 tau_S).
-template <bool DIAG>
+template <bool DIAG, int SW>
 __device__ __forceinline__ void ew_chunk(const uint32_t (&U)[32], const uint32_t (&G)[32],
-                                         const float* st, int qloc0, int t, const EwConst& k,
+                                         const float* st, int qt0, int t, const EwConst& k,
                                          uint32_t (&pk)[16], uint32_t (&dk)[16], float2& dl2) {
   if (!DIAG) {
     const float2 ch2 = make_float2(k.ch, k.ch), c2k2 = make_float2(k.c2k, k.c2k);
     const float2 one2 = make_float2(1.f, 1.f);
 #pragma unroll
     for (int c = 0; c < 32; c += 4) {
-      const float4 c2v = *reinterpret_cast<const float4*>(st + qloc0 + c);
-      const float4 ndv = *reinterpret_cast<const float4*>(st + BT + qloc0 + c);
-      const float4 nwv = *reinterpret_cast<const float4*>(st + 2 * BT + qloc0 + c);
+      const float4 c2v = *reinterpret_cast<const float4*>(st + c);
+      const float4 ndv = *reinterpret_cast<const float4*>(st + SW + c);
+      const float4 nwv = *reinterpret_cast<const float4*>(st + 2 * SW + c);
 #pragma unroll
       for (int e = 0; e < 4; e += 2) {
         const float2 x = make_float2(__uint_as_float(U[c + e]), __uint_as_float(U[c + e + 1]));
@@ -163,21 +183,21 @@ __device__ __forceinline__ void ew_chunk(const uint32_t (&U)[32], const uint32_t
       float pv[2], sv[2];
 #pragma unroll
       for (int e = 0; e < 2; ++e) {
-        const int q = qloc0 + c + e;  // tile-local query index; this thread's key is t
+        const int j = c + e, q = qt0 + j;  // tile-local query index; this thread's key is t
         const bool self = (q == t), keep = (q >= t);
-        const float x = __uint_as_float(U[c + e]);
-        const float g = __uint_as_float(G[c + e]);
+        const float x = __uint_as_float(U[j]);
+        const float g = __uint_as_float(G[j]);
         const float h = x * (self ? k.ch_self : k.ch);
         const float th = tanh_approx(h);
         const float a = 1.0f + th;
         const float w = a * (self ? half_log2e : k.c2k);
-        float P = ex2_approx(fmaf(self ? 1.0f : x, w, self ? st[3 * BT + q] : st[q]));
+        float P = ex2_approx(fmaf(self ? 1.0f : x, w, self ? st[3 * SW + j] : st[j]));
         P = keep ? P : 0.f;
-        const float dR = P * (g + st[BT + q]);
+        const float dR = P * (g + st[SW + j]);
         const float m = fmaf(self ? k.inv2tau : h, 1.0f - th, self ? 0.f : 1.f);
         sv[e] = dR * a * m;
         pv[e] = P;
-        const float wgt = self ? k.li * (1.0f - P) : st[2 * BT + q];
+        const float wgt = self ? k.li * (1.0f - P) : st[2 * SW + j];
         dl2.x = fmaf(wgt, dR, dl2.x);
       }
       pk[c >> 1] = pack_bf16x2(pv[0], pv[1]);
@@ -208,21 +228,22 @@ __global__ void __launch_bounds__(kThreads, 1)
   const int bh = (int)(blockIdx.x % BH);
   const int b = bh / p.H, h = bh % p.H;
   const int k0 = kt * BK;
-  const int n_i = n_t - kt;               // query tiles kt .. n_t - 1
-  const int total = n_i * C::SPT;         // steps
+  const int n_i = n_t - kt;                   // query tiles kt .. n_t - 1
+  const int total = n_i * C::SPT;             // steps
+  const int n_units = C::HALF ? total : n_i;  // Q / dO stage loads
 
   if (threadIdx.x == 0) {
     mbar_init(bar(B_KV), 1);
-    for (int s = 0; s < 2; ++s) {
+    for (int s = 0; s < C::NQS; ++s) {
       mbar_init(bar(B_QF + s), 1);
       mbar_init(bar(B_QE + s), 1);
     }
     for (int s = 0; s < C::NBUF; ++s) {
       mbar_init(bar(B_S + s), 1);
       mbar_init(bar(B_P + s), 256);  // both elementwise warpgroups
+      mbar_init(bar(B_DQF + s), 1);
+      mbar_init(bar(B_DQE + s), 128);
     }
-    mbar_init(bar(B_DQF), 1);
-    mbar_init(bar(B_DQE), 128);
     mbar_init(bar(B_ACC), 1);
     *abort_flag = 0;
     fence_mbar_init();
@@ -241,7 +262,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       tma_prefetch_desc(&tmK);
       tma_prefetch_desc(&tmV);
       tma_prefetch_desc(&tmG);
-      mbar_arrive_expect_tx(bar(B_KV), 2 * C::TILE);
+      mbar_arrive_expect_tx(bar(B_KV), 2 * C::KVT);
       for (int kb = 0; kb < C::KB; ++kb) {
         tma_load_4d(sb + C::OFF_K + kb * 16384, &tmK, bar(B_KV), kb * 64, k0, h, b);
         tma_load_4d(sb + C::OFF_V + kb * 16384, &tmV, bar(B_KV), kb * 64, k0, h, b);
@@ -249,92 +270,127 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
     int issued = 0;
     if (lane == 0) {
-      for (int i = 0; i < n_i; ++i) {
-        const int s = i % C::QSTG, u = i / C::QSTG;
-        if (u > 0 && !mbar_wait(bar(B_QE + s), (u - 1) & 1, ab)) break;
-        const int qi0 = (kt + i) * BT;
-        mbar_arrive_expect_tx(bar(B_QF + s), 2 * C::TILE + 4 * BT * 4);
+      for (int u = 0; u < n_units; ++u) {
+        const int s = u % C::NQS, r = u / C::NQS;
+        if (r > 0 && !mbar_wait(bar(B_QE + s), (r - 1) & 1, ab)) break;
+        const int tile = C::HALF ? u / C::SPT : u;
+        const int qoff = C::HALF ? (u % C::SPT) * C::QW : 0;
+        const int qi0 = (kt + tile) * BT + qoff;
+        mbar_arrive_expect_tx(bar(B_QF + s), 2 * C::QSZ + C::STB);
         for (int kb = 0; kb < C::KB; ++kb) {
-          tma_load_4d(sb + C::OFF_Q + s * C::TILE + kb * 16384, &tmQ, bar(B_QF + s), kb * 64,
+          tma_load_4d(sb + C::OFF_Q + s * C::QSZ + kb * C::KBQ, &tmQ, bar(B_QF + s), kb * 64,
                       qi0, h, b);
-          tma_load_4d(sb + C::OFF_DO + s * C::TILE + kb * 16384, &tmG, bar(B_QF + s), kb * 64,
+          tma_load_4d(sb + C::OFF_DO + s * C::QSZ + kb * C::KBQ, &tmG, bar(B_QF + s), kb * 64,
                       qi0, h, b);
         }
-        bulk_load(sb + C::OFF_STAT + s * 4 * BT * 4,
-                  ws.stats + ((long long)bh * n_t + kt + i) * 4 * BT, 4 * BT * 4, bar(B_QF + s));
-        issued = i + 1;
+        const float* src = ws.stats + ((long long)bh * n_t + kt + tile) * 4 * BT + qoff;
+        if (C::HALF) {
+          for (int a = 0; a < 4; ++a)
+            bulk_load(sb + C::OFF_STAT + s * C::STB + a * C::SW * 4, src + a * BT, C::SW * 4,
+                      bar(B_QF + s));
+        } else {
+          bulk_load(sb + C::OFF_STAT + s * C::STB, src, C::STB, bar(B_QF + s));
+        }
+        issued = u + 1;
       }
     }
     if (lane == 0 && ab.raised()) {
       drain_wait(bar(B_KV), 0);
-      for (int i = issued - C::QSTG > 0 ? issued - C::QSTG : 0; i < issued; ++i)
-        drain_wait(bar(B_QF + i % C::QSTG), (i / C::QSTG) & 1);
+      for (int i = issued - C::NQS > 0 ? issued - C::NQS : 0; i < issued; ++i)
+        drain_wait(bar(B_QF + i % C::NQS), (i / C::NQS) & 1);
     }
   } else if (warp == W_MMA) {
     // ------------------------------------------------------ MMA issuer
     if (lane == 0) {
       constexpr uint32_t id_s = idesc_bf16_f32(128, C::QW, false, false);  // U^T, dP^T
       constexpr uint32_t id_acc = idesc_bf16_f32(128, D, false, true);     // dV, dK
-      constexpr uint32_t id_dq = idesc_bf16_f32(128, D, true, true);       // dQ
+      constexpr uint32_t id_dq = C::HALF ? idesc_bf16_f32(128, C::QW, true, true)  // dQ^T
+                                         : idesc_bf16_f32(128, D, true, true);     // dQ
       bool ok = mbar_wait(bar(B_KV), 0, ab);
-      // U^T and dP^T of step s into buffer s % NBUF
-      auto issue_sdp = [&](int s) -> bool {
-        const int t = s / C::SPT, hh = s % C::SPT, bb = s % C::NBUF, st = t % C::QSTG;
-        if (hh == 0) {
-          if (!mbar_wait(bar(B_QF + st), (t / C::QSTG) & 1, ab)) return false;
+      // U^T of step s into buffer s % NBUF (waits for its Q / dO stage)
+      auto issue_u = [&](int s) -> bool {
+        const int u = C::unit_of(s), st = u % C::NQS, bb = s % C::NBUF, hh = s % C::SPT;
+        if (C::HALF || hh == 0) {
+          if (!mbar_wait(bar(B_QF + st), (u / C::NQS) & 1, ab)) return false;
           tc_fence_after();
         }
-        const uint32_t qoff = hh * C::QW * 128;  // rows of the query tile (32-row aligned)
+        const uint32_t rows = C::HALF ? 0u : (uint32_t)(hh * C::QW * 128);  // the step's rows
 #pragma unroll
         for (int kk = 0; kk < D / 16; ++kk) {
-          const uint32_t koff = (kk >> 2) * 16384 + (kk & 3) * 32;
-          mma_ss(tmem + C::col_u(bb), smem_desc_sw128(sb + C::OFF_K + koff, 16, 1024),
-                 smem_desc_sw128(sb + C::OFF_Q + st * C::TILE + qoff + koff, 16, 1024), id_s,
+          const uint32_t kof = (kk >> 2) * 16384 + (kk & 3) * 32;
+          const uint32_t qof = (kk >> 2) * C::KBQ + (kk & 3) * 32;
+          mma_ss(tmem + C::col_u(bb), smem_desc_sw128(sb + C::OFF_K + kof, 16, 1024),
+                 smem_desc_sw128(sb + C::OFF_Q + st * C::QSZ + rows + qof, 16, 1024), id_s,
                  kk > 0 ? 1u : 0u);
         }
-        if (D == 128 && t > 0) {  // dP^T overwrites dQ_{t-1}: wait until it was read
-          if (!mbar_wait(bar(B_DQE), (t - 1) & 1, ab)) return false;
-          tc_fence_after();
-        }
+        return true;
+      };
+      // dP^T of step s (after issue_u(s)), then the step's S barrier
+      auto issue_dp = [&](int s) {
+        const int st = C::unit_of(s) % C::NQS, bb = s % C::NBUF, hh = s % C::SPT;
+        const uint32_t rows = C::HALF ? 0u : (uint32_t)(hh * C::QW * 128);
 #pragma unroll
         for (int kk = 0; kk < D / 16; ++kk) {
-          const uint32_t koff = (kk >> 2) * 16384 + (kk & 3) * 32;
-          mma_ss(tmem + C::col_g(bb), smem_desc_sw128(sb + C::OFF_V + koff, 16, 1024),
-                 smem_desc_sw128(sb + C::OFF_DO + st * C::TILE + qoff + koff, 16, 1024), id_s,
+          const uint32_t kof = (kk >> 2) * 16384 + (kk & 3) * 32;
+          const uint32_t qof = (kk >> 2) * C::KBQ + (kk & 3) * 32;
+          mma_ss(tmem + C::col_g(bb), smem_desc_sw128(sb + C::OFF_V + kof, 16, 1024),
+                 smem_desc_sw128(sb + C::OFF_DO + st * C::QSZ + rows + qof, 16, 1024), id_s,
                  kk > 0 ? 1u : 0u);
         }
         mma_commit(bar(B_S + bb));
-        return true;
       };
-      // U^T / dP^T of step sn may be issued once its buffer is free (step sn - NBUF done)
-      // and once the GEMM that releases the Q/dO stage of its tile (dQ of tile
-      // tn - QSTG) has been issued: waiting for that tile's load earlier would deadlock.
-      int sn = 0, tiles_done = 0;
-      while (ok && sn < total && sn < C::NBUF) ok = issue_sdp(sn++);
+      // d_h = 64: U^T / dP^T of step sn may be issued once its buffer is free (step
+      // sn - NBUF done) and once the GEMM that releases the Q/dO stage it loads into has
+      // been issued: waiting for that stage's load earlier would deadlock.
+      int sn = 0, units_done = 0;
+      while (ok && sn < total && sn < C::NBUF) {
+        ok = issue_u(sn);
+        if (ok) issue_dp(sn);
+        ++sn;
+      }
       for (int s = 0; ok && s < total; ++s) {
         const int t = s / C::SPT, hh = s % C::SPT, bb = s % C::NBUF;
-        const int st = t % C::QSTG, dsb = t % C::DSB;
+        const int st = C::unit_of(s) % C::NQS;
         if (!(ok = mbar_wait(bar(B_P + bb), (s / C::NBUF) & 1, ab))) break;
         tc_fence_after();
-        const uint32_t ds_base = sb + C::OFF_DS + dsb * 32768;
         // dV += P^T dO and dK += dS'^T Q with the A operands in TMEM: every 32-query chunk
         // keeps its 16 packed columns of P (dS') at the start of its own U^T (dP^T) columns.
         const uint32_t pcol = C::col_u(bb), dcol = C::col_g(bb);
+        const uint32_t rows = C::HALF ? 0u : (uint32_t)(hh * C::QW * 128);
 #pragma unroll
         for (int kk = 0; kk < C::QW / 16; ++kk) {
-          const int q = hh * C::QW + kk * 16;
           const uint32_t acol = (kk >> 1) * 32 + (kk & 1) * 8;
           mma_ts(tmem + C::COL_DV, tmem + pcol + acol,
-                 smem_desc_sw128(sb + C::OFF_DO + st * C::TILE + q * 128, 16384, 1024), id_acc,
-                 (s > 0 || kk > 0) ? 1u : 0u);
+                 smem_desc_sw128(sb + C::OFF_DO + st * C::QSZ + rows + kk * 2048, C::KBQ, 1024),
+                 id_acc, (s > 0 || kk > 0) ? 1u : 0u);
         }
 #pragma unroll
         for (int kk = 0; kk < C::QW / 16; ++kk) {
-          const int q = hh * C::QW + kk * 16;
           const uint32_t acol = (kk >> 1) * 32 + (kk & 1) * 8;
           mma_ts(tmem + C::COL_DK, tmem + dcol + acol,
-                 smem_desc_sw128(sb + C::OFF_Q + st * C::TILE + q * 128, 16384, 1024), id_acc,
-                 (s > 0 || kk > 0) ? 1u : 0u);
+                 smem_desc_sw128(sb + C::OFF_Q + st * C::QSZ + rows + kk * 2048, C::KBQ, 1024),
+                 id_acc, (s > 0 || kk > 0) ? 1u : 0u);
+        }
+        if (C::HALF) {
+          mma_commit(bar(B_QE + st));  // the step's Q / dO rows are no longer needed
+          // Buffer bb next holds step s + 2.  Issue order (executed in order): dQ^T of step
+          // s over dS' in the dP^T columns, which dK has read; U^T of step s + 2 over P,
+          // which dV has read; dP^T of step s + 2 once dQ^T has been read out.
+          // dQ^T = K^T dS'^T (A = K tile, d-major; B = the step's dS', query-major)
+          const uint32_t dsb = sb + C::OFF_DS + (s & 1) * C::DSZ;
+#pragma unroll
+          for (int kk = 0; kk < BK / 16; ++kk)
+            mma_ss(tmem + C::col_g(bb), smem_desc_sw128(sb + C::OFF_K + kk * 2048, 16384, 1024),
+                   smem_desc_sw128(dsb + kk * 2048, 16384, 1024), id_dq, kk > 0 ? 1u : 0u);
+          mma_commit(bar(B_DQF + bb));
+          const int s2 = s + C::NBUF;
+          if (s2 < total && !(ok = issue_u(s2))) break;
+          if (s2 < total) {
+            if (!(ok = mbar_wait(bar(B_DQE + bb), (s / C::NBUF) & 1, ab))) break;
+            tc_fence_after();
+            issue_dp(s2);
+          }
+          continue;
         }
         if (hh == C::SPT - 1) {
           if (t > 0) {  // dQ_{t-1} has been read out of TMEM
@@ -342,6 +398,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             tc_fence_after();
           }
           // dQ_t = dS' K   (A = dS', queries x keys, M-major; B = K tile, N-major)
+          const uint32_t ds_base = sb + C::OFF_DS + (t & 1) * C::DSZ;
 #pragma unroll
           for (int kk = 0; kk < BK / 16; ++kk)
             mma_ss(tmem + C::COL_DQ, smem_desc_sw128(ds_base + kk * 2048, 16384, 1024),
@@ -349,51 +406,88 @@ __global__ void __launch_bounds__(kThreads, 1)
                    kk > 0 ? 1u : 0u);
           mma_commit(bar(B_DQF));
           mma_commit(bar(B_QE + st));
-          ++tiles_done;
+          ++units_done;
         }
-        while (ok && sn < total && sn <= s + C::NBUF && sn / C::SPT - C::QSTG < tiles_done)
-          ok = issue_sdp(sn++);
+        while (ok && sn < total && sn <= s + C::NBUF && C::unit_of(sn) - C::NQS < units_done) {
+          ok = issue_u(sn);
+          if (ok) issue_dp(sn);
+          ++sn;
+        }
       }
       mma_commit(bar(B_ACC));
     }
     __syncwarp();
   } else if (warp >= W_DQ) {
-    // ------------------------------------------------------ dQ_t -> fp32 accumulator
+    // ------------------------------------------------------ dQ -> fp32 accumulator
     const int quad = warp & 3;
     const uint32_t trow = tmem + ((uint32_t)(quad * 32) << 16);
-    const uint32_t stage0 = sb + C::OFF_DQS + quad * 8192;
-    uint8_t* stage0p = smem + C::OFF_DQS + quad * 8192;
-    int chunk = 0;
-    for (int i = 0; i < n_i; ++i) {
-      const bool ok = __all_sync(0xffffffffu, mbar_wait(bar(B_DQF), i & 1, ab));
-      if (!ok) break;
-      tc_fence_after();
-      const int row0 = bh * t_pad + (kt + i) * BT + quad * 32;
-#pragma unroll
-      for (int c64 = 0; c64 < D; c64 += 64) {
+    const uint32_t stage0 = sb + C::OFF_DQS + quad * C::DQSLOTS * 4096;
+    uint8_t* stage0p = smem + C::OFF_DQS + quad * C::DQSLOTS * 4096;
+    if (C::HALF) {
+      // TMEM lanes are d indices here: this warp holds d = 32 quad .. 32 quad + 31 of the
+      // step's 64 queries and writes them as 32-query x 32-d boxes, transposed.
+      for (int s = 0; s < total; ++s) {
+        const int bb = s % C::NBUF;
+        const bool ok = __all_sync(0xffffffffu, mbar_wait(bar(B_DQF + bb), (s / C::NBUF) & 1, ab));
+        if (!ok) break;
+        tc_fence_after();
         uint32_t z[64];
-        tmem_ld32(trow + C::COL_DQ + c64, z);
-        tmem_ld32(trow + C::COL_DQ + c64 + 32, z + 32);
+        tmem_ld32(trow + C::col_g(bb), z);
+        tmem_ld32(trow + C::col_g(bb) + 32, z + 32);
         tmem_ld_wait();
-        if (c64 + 64 == D) {
-          tc_fence_before();
-          mbar_arrive(bar(B_DQE));  // TMEM columns free for the next dQ / dP^T
-        }
+        tc_fence_before();
+        mbar_arrive(bar(B_DQE + bb));  // the buffer may take the next dP^T
+        const int row0 = bh * t_pad + (kt + s / C::SPT) * BT + (s % C::SPT) * C::QW;
+        const uint32_t sw = (uint32_t)(lane & 3) << 2;
 #pragma unroll
-        for (int c0 = 0; c0 < 64; c0 += 32, ++chunk) {
-          const int slot = chunk & 1;
-          if (lane == 0) bulk_wait_read_le1();  // the slot's previous reduce has read it
+        for (int c = 0; c < 2; ++c) {
+          if (lane == 0) bulk_wait_read_0();  // the slot's previous reduce has read it
           __syncwarp();
-          uint8_t* row = stage0p + slot * 4096 + lane * 128;
 #pragma unroll
-          for (int k = 0; k < 8; ++k)
-            *reinterpret_cast<uint4*>(row + ((k ^ (lane & 7)) << 4)) =
-                make_uint4(z[c0 + 4 * k], z[c0 + 4 * k + 1], z[c0 + 4 * k + 2], z[c0 + 4 * k + 3]);
+          for (int q = 0; q < 32; ++q)
+            *reinterpret_cast<uint32_t*>(stage0p + q * 128 + (((lane >> 2) ^ (q & 7)) << 4) +
+                                         sw) = z[c * 32 + q];
           fence_async_smem();
           __syncwarp();
           if (lane == 0) {
-            tma_reduce_add_2d(&tmDQ, stage0 + slot * 4096, c64 + c0, row0);
+            tma_reduce_add_2d(&tmDQ, stage0, quad * 32, row0 + c * 32);
             tma_store_commit();
+          }
+        }
+      }
+    } else {
+      int chunk = 0;
+      for (int i = 0; i < n_i; ++i) {
+        const bool ok = __all_sync(0xffffffffu, mbar_wait(bar(B_DQF), i & 1, ab));
+        if (!ok) break;
+        tc_fence_after();
+        const int row0 = bh * t_pad + (kt + i) * BT + quad * 32;
+#pragma unroll
+        for (int c64 = 0; c64 < D; c64 += 64) {
+          uint32_t z[64];
+          tmem_ld32(trow + C::COL_DQ + c64, z);
+          tmem_ld32(trow + C::COL_DQ + c64 + 32, z + 32);
+          tmem_ld_wait();
+          if (c64 + 64 == D) {
+            tc_fence_before();
+            mbar_arrive(bar(B_DQE));  // TMEM columns free for the next dQ
+          }
+#pragma unroll
+          for (int c0 = 0; c0 < 64; c0 += 32, ++chunk) {
+            const int slot = chunk & 1;
+            if (lane == 0) bulk_wait_read_le1();  // the slot's previous reduce has read it
+            __syncwarp();
+            uint8_t* row = stage0p + slot * 4096 + lane * 128;
+#pragma unroll
+            for (int k = 0; k < 8; ++k)
+              *reinterpret_cast<uint4*>(row + ((k ^ (lane & 7)) << 4)) =
+                  make_uint4(z[c0 + 4 * k], z[c0 + 4 * k + 1], z[c0 + 4 * k + 2], z[c0 + 4 * k + 3]);
+            fence_async_smem();
+            __syncwarp();
+            if (lane == 0) {
+              tma_reduce_add_2d(&tmDQ, stage0 + slot * 4096, c64 + c0, row0);
+              tma_store_commit();
+            }
           }
         }
       }
@@ -401,6 +495,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     if (lane == 0) tma_store_wait_all();
   } else {
     // ------------------------------------------------------ elementwise + epilogue
+    // Both warpgroups work on every step: warpgroup wg takes its 32 query columns.
     const int wg = warp >> 2;                  // 0 or 1
     const int t = (warp & 3) * 32 + lane;      // key k0 + t, TMEM lane t
     const uint32_t trow = tmem + ((uint32_t)((warp & 3) * 32) << 16);
@@ -415,38 +510,39 @@ __global__ void __launch_bounds__(kThreads, 1)
     float2 dl2 = make_float2(0.f, 0.f);
     bool ok = true;
     for (int s = 0; s < total; ++s) {
-      const int bb = s % C::NBUF, i = s / C::SPT, qs = (s % C::SPT) * C::QW;
+      const int bb = s % C::NBUF, i = s / C::SPT, hh = s % C::SPT;
+      const int u = C::unit_of(s), st = u % C::NQS;
       ok = __all_sync(0xffffffffu, mbar_wait(bar(B_S + bb), (s / C::NBUF) & 1, ab));
       if (!ok) break;
       tc_fence_after();
-      // acquire the producer's per-query scalars of this tile (already complete)
-      ok = __all_sync(0xffffffffu, mbar_wait(bar(B_QF + i % C::QSTG), (i / C::QSTG) & 1, ab));
+      // acquire the producer's per-query scalars of this stage (already complete)
+      ok = __all_sync(0xffffffffu, mbar_wait(bar(B_QF + st), (u / C::NQS) & 1, ab));
       if (!ok) break;
-      const float* st =
-          reinterpret_cast<const float*>(smem + C::OFF_STAT + (i % C::QSTG) * 4 * BT * 4);
-#pragma unroll 1
-      for (int ck = 0; ck < C::QW / 64; ++ck) {
-        const int cl = wg * (C::QW / 2) + ck * 32;  // chunk's first column within the step
-        const int q0 = qs + cl;                       // tile-local query index
-        uint32_t U[32], G[32];
-        tmem_ld32(trow + C::col_u(bb) + cl, U);
-        tmem_ld32(trow + C::col_g(bb) + cl, G);
-        tmem_ld_wait();
-        uint32_t pk[16], dk[16];
-        if (i == 0)
-          ew_chunk<true>(U, G, st, q0, t, kc, pk, dk, dl2);
-        else
-          ew_chunk<false>(U, G, st, q0, t, kc, pk, dk, dl2);
-        tmem_st16(trow + C::col_u(bb) + cl, pk);  // P   (A operand of dV += P^T dO)
-        tmem_st16(trow + C::col_g(bb) + cl, dk);  // dS' (A operand of dK += dS'^T Q)
-        // dS' row t, queries q0 .. q0+31 for dQ = dS' K: 4 chunks of the 128-byte swizzle
-        uint8_t* ds_row = smem + C::OFF_DS + (i % C::DSB) * 32768 + (q0 >> 6) * 16384 + t * 128;
-        const int cb = (q0 & 63) >> 3;
+      const float* sts = reinterpret_cast<const float*>(smem + C::OFF_STAT + st * C::STB);
+      const int cl = wg * 32;             // the chunk's first column within the step
+      const int qt0 = hh * C::QW + cl;    // tile-local query index
+      uint32_t U[32], G[32];
+      tmem_ld32(trow + C::col_u(bb) + cl, U);
+      tmem_ld32(trow + C::col_g(bb) + cl, G);
+      tmem_ld_wait();
+      uint32_t pk[16], dk[16];
+      const float* stc = sts + (C::HALF ? cl : qt0);
+      if (i == 0)
+        ew_chunk<true, C::SW>(U, G, stc, qt0, t, kc, pk, dk, dl2);
+      else
+        ew_chunk<false, C::SW>(U, G, stc, qt0, t, kc, pk, dk, dl2);
+      tmem_st16(trow + C::col_u(bb) + cl, pk);  // P   (A operand of dV += P^T dO)
+      tmem_st16(trow + C::col_g(bb) + cl, dk);  // dS' (A operand of dK += dS'^T Q)
+      // dS' row t (key), 32 queries, into the 128-byte-swizzled query-major layout the dQ
+      // product reads: 64-query blocks of 128 key rows
+      uint8_t* ds_row = C::HALF ? smem + C::OFF_DS + (s & 1) * C::DSZ + t * 128
+                                : smem + C::OFF_DS + (i & 1) * C::DSZ + (qt0 >> 6) * 16384 +
+                                      t * 128;
+      const int cb = (qt0 & 63) >> 3;
 #pragma unroll
-        for (int qd = 0; qd < 4; ++qd)
-          *reinterpret_cast<uint4*>(ds_row + (((cb + qd) ^ (t & 7)) << 4)) =
-              make_uint4(dk[4 * qd], dk[4 * qd + 1], dk[4 * qd + 2], dk[4 * qd + 3]);
-      }
+      for (int qd = 0; qd < 4; ++qd)
+        *reinterpret_cast<uint4*>(ds_row + (((cb + qd) ^ (t & 7)) << 4)) =
+            make_uint4(dk[4 * qd], dk[4 * qd + 1], dk[4 * qd + 2], dk[4 * qd + 3]);
       tmem_st_wait();
       fence_async_smem();
       tc_fence_before();
@@ -649,8 +745,9 @@ static cudaError_t bwd_t(const Problem& p, const BwdWorkspace& ws, unsigned stag
                              smem);
     if (e != cudaSuccess) { note_failure("backward: shared memory attribute"); return e; }
     CUtensorMap mq, mk, mv, mg, mdq;
-    if (!make_tmap_bf16(&mq, p.q, p, 128) || !make_tmap_bf16(&mk, p.k, p, 128) ||
-        !make_tmap_bf16(&mv, p.v, p, 128) || !make_tmap_bf16(&mg, p.dout, p, 128)) {
+    constexpr int qrows = bwd::Cfg<D>::QROWS;
+    if (!make_tmap_bf16(&mq, p.q, p, qrows) || !make_tmap_bf16(&mk, p.k, p, 128) ||
+        !make_tmap_bf16(&mv, p.v, p, 128) || !make_tmap_bf16(&mg, p.dout, p, qrows)) {
       note_failure("backward: TMA descriptor of Q/K/V/dO");
       return cudaErrorInvalidValue;
     }
