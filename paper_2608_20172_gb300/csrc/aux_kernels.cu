@@ -24,11 +24,20 @@
 
 namespace rel {
 
+// dlambda partial slots of the row pass: one per block of either row pass (8 rows per
+// block in the SIMT pass, 32 padded rows per block in the tensor-core pass).
+static size_t pre_slots(int B, int H, int T) {
+  const size_t rows = (size_t)B * H * T;
+  const size_t rows_pad = (size_t)B * H * ((T + 127) / 128 * 128);
+  const size_t a = (rows + 7) / 8, b = rows_pad / 32;
+  return a > b ? a : b;
+}
+
 size_t bwd_workspace_bytes(int B, int H, int T, int d) {
   auto up = [](size_t x) { return (x + 255) & ~(size_t)255; };
   const size_t rows = (size_t)B * H * T;
   const size_t rows_pad = (size_t)B * H * ((T + 127) / 128 * 128);
-  const size_t n_pre = (rows + 7) / 8;
+  const size_t n_pre = pre_slots(B, H, T);
   const size_t n_main = (size_t)((T + 63) / 64) * B * H;
   return up(rows_pad * d * sizeof(float)) + 4 * up(rows * sizeof(float)) +
          up(rows_pad * 4 * sizeof(float)) + up((n_pre + n_main) * sizeof(float));
@@ -48,7 +57,7 @@ BwdWorkspace carve_workspace(void* base, int B, int H, int T, int d) {
   w.wl = reinterpret_cast<float*>(p); p += up(rows * sizeof(float));
   w.stats = reinterpret_cast<float*>(p); p += up((size_t)B * H * t_pad * 4 * sizeof(float));
   w.dlam_part = reinterpret_cast<float*>(p);
-  w.n_pre_blocks = (int)((rows + 7) / 8);
+  w.n_pre_blocks = (int)pre_slots(B, H, T);
   w.n_main_slots = ((T + 63) / 64) * B * H;
   return w;
 }

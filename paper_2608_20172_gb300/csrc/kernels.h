@@ -42,9 +42,10 @@ struct BwdWorkspace {
   float* F_self;     // [B][H][T]     F_ii = exp(S_i - logZ_i)
   float* dS_self;    // [B][H][T]     dL/du_ii, u = U_ii (scaled evidence)
   float* wl;         // [B][H][T]     log i F_ii (dlambda weight of row i's Exchange pairs)
-  float* stats;      // [B][H][T_pad/128][4][128] per-query scalars of the tensor-core backward
-  // dlambda partials: [n_pre_blocks] from the row pre-pass, then [n_main_slots] from
-  // the Exchange tile kernel (one per CTA).
+  float* stats;      // [B][H][T_pad/128][3][128] per-query scalars of the tensor-core backward
+  // dlambda partials: [n_pre_blocks] from the row pre-pass (the Self terms; the SIMT pass
+  // fills the first ceil(rows / 8), the tensor-core pass the first T_pad B H / 32), then
+  // [n_main_slots] from the Exchange tile kernel (one per CTA).
   float* dlam_part;
   int n_pre_blocks;
   int n_main_slots;  // capacity reserved for the tile kernel's CTAs

@@ -7,11 +7,13 @@
 //   dS_ii = dR_ii S_i (1 - S_i) / tau_S          (Self, j = i; S_i = sigmoid(u_ii / tau_S))
 //   dV_j += F_ij dO_i,  dK_j += dS_ij q_i / sqrt(d),  dQ_i += dS_ij k_j / sqrt(d)
 // with F_ij = exp(E_ij - lambda log i - logZ_i) (j < i) and F_ii = exp(S_i - logZ_i).
-// The Self entry is handled inside the diagonal tile with its own role map, exactly as
-// the forward treats it.
+// The Self entries (j = i) are computed per row in fp32 by the row pass and added by the
+// dK / dV epilogue and the dQ finalisation; the tile kernel handles the Exchange pairs
+// (j < i) only.
 //
-// Three launches: a row pass (D_i, the dlambda weight log i F_ii, zeroed fp32 dQ
-// accumulator), the tile kernel, and a finalisation (dQ to bf16, dlambda reduction).
+// Three launches: a row pass (D_i, the Self entries and their dlambda terms, the tile
+// kernel's per-query scalars, zeroed fp32 dQ accumulator), the tile kernel, and a
+// finalisation (dQ to bf16 plus the Self term, dlambda reduction).
 //
 // Tile kernel: one CTA per 128 keys of one head, visiting query tiles from the diagonal
 // to the end of the sequence.  Keys sit on TMEM lanes.  Per step of 64 query columns:
@@ -29,8 +31,10 @@
 //              of the buffer is issued after it, the next dP^T after its read-out.
 // A tcgen05.mma costs at least ~46 cycles whatever its N (measured on GB300: N = 32, 64,
 // 128 run at 35%, 66%, 99% of the per-SM peak), so the steps keep N >= 64.
-// dlambda = sum_i log i g_i dR_ii - sum_{j<i} log i F_ii dR_ij (weights cancel the
-// rounding error of D_i; see aux_kernels.cu), reduced per CTA.
+// dlambda = sum_i log i (1 - F_ii) dR_ii - sum_{j<i} log i F_ii dR_ij: the row pass sums
+// the first part per block, the tile kernel the second per CTA.  In exact arithmetic it
+// equals sum_i log i dR_ii; this weighting cancels the rounding error of D_i (see
+// aux_kernels.cu).
 #include <cudaTypedefs.h>
 #include <math.h>
 
@@ -68,7 +72,7 @@ struct Cfg {
   static constexpr int KBQ = QROWS * 128;      // stride of the 64-column blocks of a stage
   static constexpr int NQS = HALF ? 3 : 2;     // Q / dO stages
   static constexpr int SW = QROWS;             // per-query scalars of a stage: array stride
-  static constexpr int STB = 4 * SW * 4;       // bytes of one stage's scalars
+  static constexpr int STB = 3 * SW * 4;       // bytes of one stage's scalars
   static constexpr int DSZ = HALF ? 16384 : 32768;  // one dS' buffer (per step / per tile)
   static constexpr int DQSLOTS = HALF ? 1 : 2;      // 4 KB staging slots per dQ warp
   static constexpr int OFF_K = 0;
@@ -126,82 +130,58 @@ __device__ __forceinline__ void bulk_wait_read_0() {
 
 // Per-thread constants of the elementwise step.
 struct EwConst {
-  float ch;       // u / 2 = U ch       (U = raw q . k, u = U / sqrt(d))
-  float c2k;      // E log2 e = U c2k (1 + tanh(u / 2))
-  float ch_self;  // u / (2 tau_S) = U ch_self
-  float inv2tau;  // 1 / (2 tau_S)
-  float li;       // log(i) of this thread's own row (the Self entry on the diagonal)
+  float ch;   // u / 2 = U ch       (U = raw q . k, u = U / sqrt(d))
+  float c2k;  // E log2 e = U c2k (1 + tanh(u / 2))
 };
 
-// Elementwise work on 32 query columns of one key row (this thread's key t).  st points at
-// the chunk's first query in the stage's per-query scalars, four arrays of stride SW:
-// [0] c2 = (-lambda log i - logZ_i) log2 e, [SW] -D_i, [2 SW] -log i F_ii,
-// [3 SW] -logZ_i log2 e.  qt0 is the tile-local index of the chunk's first query.
-// Produces P = F_ij and dS' = 2 dS_ij as bf16 pairs and accumulates the dlambda terms.
-//   Exchange:  P = 2^(U c2k (1 + t) + c2),  t = tanh(u/2),
-//              2 SiLU'(u) = a (1 + h (1 - t)) with a = 1 + t, h = u / 2.
-//   Self (DIAG, query == key):  S = (1 + tanh(u / (2 tau_S))) / 2 = a / 2,
-//              P = 2^(S log2 e - logZ log2 e),  2 dS/du = a (1 - t) / (2 tau_S).
+// Elementwise work on 32 query columns of one key row (this thread's key t), Exchange
+// entries only.  st points at the chunk's first query in the stage's per-query scalars,
+// three arrays of stride SW: [0] c2 = (-lambda log i - logZ_i) log2 e, [SW] -D_i,
+// [2 SW] -log i F_ii.  qt0 is the tile-local index of the chunk's first query.
+// Produces P = F_ij and dS' = 2 dS_ij as bf16 pairs and accumulates the dlambda terms:
+//   P = 2^(U c2k (1 + t) + c2),  t = tanh(u/2),
+//   2 SiLU'(u) = a (1 + h (1 - t)) with a = 1 + t, h = u / 2.
+// On the diagonal tile (DIAG) the entries with query <= key get c2 = -inf, so P, dS' and
+// their dlambda terms are exactly zero: the Self entry (query == key) is not part of
+// the tile; the row pass and the epilogues add it.
 template <bool DIAG, int SW>
 __device__ __forceinline__ void ew_chunk(const uint32_t (&U)[32], const uint32_t (&G)[32],
                                          const float* st, int qt0, int t, const EwConst& k,
                                          uint32_t (&pk)[16], uint32_t (&dk)[16], float2& dl2) {
-  if (!DIAG) {
-    const float2 ch2 = make_float2(k.ch, k.ch), c2k2 = make_float2(k.c2k, k.c2k);
-    const float2 one2 = make_float2(1.f, 1.f);
+  const float2 ch2 = make_float2(k.ch, k.ch), c2k2 = make_float2(k.c2k, k.c2k);
+  const float2 one2 = make_float2(1.f, 1.f);
 #pragma unroll
-    for (int c = 0; c < 32; c += 4) {
-      const float4 c2v = *reinterpret_cast<const float4*>(st + c);
-      const float4 ndv = *reinterpret_cast<const float4*>(st + SW + c);
-      const float4 nwv = *reinterpret_cast<const float4*>(st + 2 * SW + c);
-#pragma unroll
-      for (int e = 0; e < 4; e += 2) {
-        const float2 x = make_float2(__uint_as_float(U[c + e]), __uint_as_float(U[c + e + 1]));
-        const float2 g = make_float2(__uint_as_float(G[c + e]), __uint_as_float(G[c + e + 1]));
-        const float2 c2 = e == 0 ? make_float2(c2v.x, c2v.y) : make_float2(c2v.z, c2v.w);
-        const float2 nd = e == 0 ? make_float2(ndv.x, ndv.y) : make_float2(ndv.z, ndv.w);
-        const float2 nw = e == 0 ? make_float2(nwv.x, nwv.y) : make_float2(nwv.z, nwv.w);
-        const float2 h = __fmul2_rn(x, ch2);
-        const float2 th = make_float2(tanh_approx(h.x), tanh_approx(h.y));
-        const float2 a = __fadd2_rn(th, one2);
-        const float2 w = __fmul2_rn(a, c2k2);
-        const float2 ex = __ffma2_rn(x, w, c2);
-        const float2 P = make_float2(ex2_approx(ex.x), ex2_approx(ex.y));
-        const float2 dR = __fmul2_rn(P, __fadd2_rn(g, nd));
-        const float2 b = __ffma2_rn(make_float2(-h.x, -h.y), th, h);  // h (1 - t)
-        const float2 sp = __ffma2_rn(a, b, a);                        // 2 SiLU'(u)
-        const float2 dS = __fmul2_rn(dR, sp);
-        dl2 = __ffma2_rn(nw, dR, dl2);
-        pk[(c + e) >> 1] = pack_bf16x2(P.x, P.y);
-        dk[(c + e) >> 1] = pack_bf16x2(dS.x, dS.y);
-      }
+  for (int c = 0; c < 32; c += 4) {
+    float4 c2v = *reinterpret_cast<const float4*>(st + c);
+    const float4 ndv = *reinterpret_cast<const float4*>(st + SW + c);
+    const float4 nwv = *reinterpret_cast<const float4*>(st + 2 * SW + c);
+    if (DIAG) {  // keep query > key
+      const int q = qt0 + c;
+      c2v.x = q > t ? c2v.x : -INFINITY;
+      c2v.y = q + 1 > t ? c2v.y : -INFINITY;
+      c2v.z = q + 2 > t ? c2v.z : -INFINITY;
+      c2v.w = q + 3 > t ? c2v.w : -INFINITY;
     }
-  } else {
-    const float half_log2e = 0.5f * kLog2e;
 #pragma unroll
-    for (int c = 0; c < 32; c += 2) {
-      float pv[2], sv[2];
-#pragma unroll
-      for (int e = 0; e < 2; ++e) {
-        const int j = c + e, q = qt0 + j;  // tile-local query index; this thread's key is t
-        const bool self = (q == t), keep = (q >= t);
-        const float x = __uint_as_float(U[j]);
-        const float g = __uint_as_float(G[j]);
-        const float h = x * (self ? k.ch_self : k.ch);
-        const float th = tanh_approx(h);
-        const float a = 1.0f + th;
-        const float w = a * (self ? half_log2e : k.c2k);
-        float P = ex2_approx(fmaf(self ? 1.0f : x, w, self ? st[3 * SW + j] : st[j]));
-        P = keep ? P : 0.f;
-        const float dR = P * (g + st[SW + j]);
-        const float m = fmaf(self ? k.inv2tau : h, 1.0f - th, self ? 0.f : 1.f);
-        sv[e] = dR * a * m;
-        pv[e] = P;
-        const float wgt = self ? k.li * (1.0f - P) : st[2 * SW + j];
-        dl2.x = fmaf(wgt, dR, dl2.x);
-      }
-      pk[c >> 1] = pack_bf16x2(pv[0], pv[1]);
-      dk[c >> 1] = pack_bf16x2(sv[0], sv[1]);
+    for (int e = 0; e < 4; e += 2) {
+      const float2 x = make_float2(__uint_as_float(U[c + e]), __uint_as_float(U[c + e + 1]));
+      const float2 g = make_float2(__uint_as_float(G[c + e]), __uint_as_float(G[c + e + 1]));
+      const float2 c2 = e == 0 ? make_float2(c2v.x, c2v.y) : make_float2(c2v.z, c2v.w);
+      const float2 nd = e == 0 ? make_float2(ndv.x, ndv.y) : make_float2(ndv.z, ndv.w);
+      const float2 nw = e == 0 ? make_float2(nwv.x, nwv.y) : make_float2(nwv.z, nwv.w);
+      const float2 h = __fmul2_rn(x, ch2);
+      const float2 th = make_float2(tanh_approx(h.x), tanh_approx(h.y));
+      const float2 a = __fadd2_rn(th, one2);
+      const float2 w = __fmul2_rn(a, c2k2);
+      const float2 ex = __ffma2_rn(x, w, c2);
+      const float2 P = make_float2(ex2_approx(ex.x), ex2_approx(ex.y));
+      const float2 dR = __fmul2_rn(P, __fadd2_rn(g, nd));
+      const float2 b = __ffma2_rn(make_float2(-h.x, -h.y), th, h);  // h (1 - t)
+      const float2 sp = __ffma2_rn(a, b, a);                        // 2 SiLU'(u)
+      const float2 dS = __fmul2_rn(dR, sp);
+      dl2 = __ffma2_rn(nw, dR, dl2);
+      pk[(c + e) >> 1] = pack_bf16x2(P.x, P.y);
+      dk[(c + e) >> 1] = pack_bf16x2(dS.x, dS.y);
     }
   }
 }
@@ -283,9 +263,9 @@ __global__ void __launch_bounds__(kThreads, 1)
           tma_load_4d(sb + C::OFF_DO + s * C::QSZ + kb * C::KBQ, &tmG, bar(B_QF + s), kb * 64,
                       qi0, h, b);
         }
-        const float* src = ws.stats + ((long long)bh * n_t + kt + tile) * 4 * BT + qoff;
+        const float* src = ws.stats + ((long long)bh * n_t + kt + tile) * 3 * BT + qoff;
         if (C::HALF) {
-          for (int a = 0; a < 4; ++a)
+          for (int a = 0; a < 3; ++a)
             bulk_load(sb + C::OFF_STAT + s * C::STB + a * C::SW * 4, src + a * BT, C::SW * 4,
                       bar(B_QF + s));
         } else {
@@ -503,10 +483,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     EwConst kc;
     kc.ch = 0.5f * isd;
     kc.c2k = kc.ch * kLog2e;
-    kc.ch_self = kc.ch / p.tau_s;
-    kc.inv2tau = 0.5f / p.tau_s;
     const int key_g = k0 + t;
-    kc.li = __logf((float)(key_g + 1));
     float2 dl2 = make_float2(0.f, 0.f);
     bool ok = true;
     for (int s = 0; s < total; ++s) {
@@ -550,12 +527,26 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
     float dlam = dl2.x + dl2.y;
     // ---------------------------------------------------- dK (warpgroup 0) / dV (1)
+    // Exchange sums from TMEM plus the Self entry of key j (from the row pass):
+    //   dK_j = (sum dS'_ij q_i) / (2 sqrt d) + dS_jj q_j / sqrt d
+    //   dV_j =  sum P_ij dO_i               + F_jj dO_j
+    // The Self operands (q_j or dO_j, and the scalar) are fetched while the last MMAs run.
+    const int j = key_g;
+    const long long off = (long long)b * p.sB + (long long)h * p.sH + (long long)j * p.sT;
+    const bool valid = j < p.T;
+    uint4 rowv[D / 8];
+    float self = 0.f;
+    if (valid) {
+      const __nv_bfloat16* row =
+          reinterpret_cast<const __nv_bfloat16*>(wg == 0 ? p.q : p.dout) + off;
+#pragma unroll
+      for (int c = 0; c < D / 8; ++c) rowv[c] = *reinterpret_cast<const uint4*>(row + 8 * c);
+      const long long srow = (long long)bh * p.T + j;
+      self = wg == 0 ? ws.dS_self[srow] * isd : ws.F_self[srow];
+    }
     if (ok) ok = __all_sync(0xffffffffu, mbar_wait(bar(B_ACC), 0, ab));
     tc_fence_after();
     if (ok) {
-      const int j = key_g;
-      const long long off = (long long)b * p.sB + (long long)h * p.sH + (long long)j * p.sT;
-      const bool valid = j < p.T;
       const uint32_t col = wg == 0 ? C::COL_DK : C::COL_DV;
       __nv_bfloat16* dst = reinterpret_cast<__nv_bfloat16*>(wg == 0 ? p.dk : p.dv) + off;
       const float sc = wg == 0 ? 0.5f * isd : 1.0f;
@@ -567,11 +558,15 @@ __global__ void __launch_bounds__(kThreads, 1)
         if (valid) {
 #pragma unroll
           for (int c8 = 0; c8 < 32; c8 += 8) {
+            const uint4 rv = rowv[(c0 + c8) / 8];
+            const uint32_t r4[4] = {rv.x, rv.y, rv.z, rv.w};
             uint32_t o4[4];
 #pragma unroll
-            for (int e = 0; e < 4; ++e)
-              o4[e] = pack_bf16x2(__uint_as_float(a[c8 + 2 * e]) * sc,
-                                  __uint_as_float(a[c8 + 2 * e + 1]) * sc);
+            for (int e = 0; e < 4; ++e) {
+              const float2 rf = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&r4[e]));
+              o4[e] = pack_bf16x2(fmaf(__uint_as_float(a[c8 + 2 * e]), sc, self * rf.x),
+                                  fmaf(__uint_as_float(a[c8 + 2 * e + 1]), sc, self * rf.y));
+            }
             *reinterpret_cast<uint4*>(dst + c0 + c8) = make_uint4(o4[0], o4[1], o4[2], o4[3]);
           }
         }
@@ -597,12 +592,17 @@ __global__ void __launch_bounds__(kThreads, 1)
 }
 
 // Row pass over the padded rows r < t_pad of every head, 8 threads per row:
-//   D_i = dO_i . Y_i,  F_ii = exp(sigmoid(u_ii / tau_S) - logZ_i),
-// written as the per-query scalars of the tile kernel (structure of arrays per 128-row
-// tile: c2 = (-lambda log i - logZ_i) log2 e, -D_i, -log i F_ii, -logZ_i log2 e), and a
-// zeroed row of the fp32 dQ accumulator.  Padding rows get neutral scalars (P = 0).
+//   D_i = dO_i . Y_i,  g_ii = dO_i . v_i,  S_i = sigmoid(u_ii / tau_S),
+//   F_ii = exp(S_i - logZ_i) (the Self flow),
+//   Self entry: dR_ii = F_ii (g_ii - D_i),  dS_ii = dR_ii S_i (1 - S_i) / tau_S
+//   (F_self, dS_self for the epilogues) and its dlambda term log i (1 - F_ii) dR_ii
+//   (one partial per block);
+// the per-query scalars of the tile kernel (three arrays per 128-row tile:
+// c2 = (-lambda log i - logZ_i) log2 e, -D_i, -log i F_ii) and a zeroed row of the fp32 dQ
+// accumulator.  Padding rows get neutral scalars (P = 0).
 template <int D>
 __global__ void __launch_bounds__(256) pre_kernel(Problem p, BwdWorkspace ws, int n_t) {
+  __shared__ float part[8];
   constexpr int PER = D / 8;  // elements per thread
   const long long gr = ((long long)blockIdx.x * 256 + threadIdx.x) >> 3;
   const int sub = threadIdx.x & 7;
@@ -613,23 +613,27 @@ __global__ void __launch_bounds__(256) pre_kernel(Problem p, BwdWorkspace ws, in
   const bool real = live && r < p.T;
   const int b = bh / p.H, h = bh % p.H;
   const long long off = (long long)b * p.sB + (long long)h * p.sH + (long long)r * p.sT + sub * PER;
-  float gy = 0.f, qk = 0.f;
+  float gy = 0.f, gv = 0.f, qk = 0.f;
   if (real) {
+    auto bf = [](const void* base, long long o) {
+      return *reinterpret_cast<const uint4*>(reinterpret_cast<const __nv_bfloat16*>(base) + o);
+    };
 #pragma unroll
     for (int c = 0; c < PER; c += 8) {
-      const uint4 gv = *reinterpret_cast<const uint4*>(reinterpret_cast<const __nv_bfloat16*>(p.dout) + off + c);
-      const uint4 ov = *reinterpret_cast<const uint4*>(reinterpret_cast<const __nv_bfloat16*>(p.o) + off + c);
-      const uint4 qv = *reinterpret_cast<const uint4*>(reinterpret_cast<const __nv_bfloat16*>(p.q) + off + c);
-      const uint4 kv = *reinterpret_cast<const uint4*>(reinterpret_cast<const __nv_bfloat16*>(p.k) + off + c);
-      const uint32_t g4[4] = {gv.x, gv.y, gv.z, gv.w}, o4[4] = {ov.x, ov.y, ov.z, ov.w};
+      const uint4 gv4 = bf(p.dout, off + c), ov = bf(p.o, off + c), vv = bf(p.v, off + c);
+      const uint4 qv = bf(p.q, off + c), kv = bf(p.k, off + c);
+      const uint32_t g4[4] = {gv4.x, gv4.y, gv4.z, gv4.w}, o4[4] = {ov.x, ov.y, ov.z, ov.w};
+      const uint32_t v4[4] = {vv.x, vv.y, vv.z, vv.w};
       const uint32_t q4[4] = {qv.x, qv.y, qv.z, qv.w}, k4[4] = {kv.x, kv.y, kv.z, kv.w};
 #pragma unroll
       for (int e = 0; e < 4; ++e) {
         const float2 gf = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&g4[e]));
         const float2 of = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&o4[e]));
+        const float2 vf = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&v4[e]));
         const float2 qf = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&q4[e]));
         const float2 kf = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&k4[e]));
         gy = fmaf(gf.x, of.x, fmaf(gf.y, of.y, gy));
+        gv = fmaf(gf.x, vf.x, fmaf(gf.y, vf.y, gv));
         qk = fmaf(qf.x, kf.x, fmaf(qf.y, kf.y, qk));
       }
     }
@@ -637,38 +641,59 @@ __global__ void __launch_bounds__(256) pre_kernel(Problem p, BwdWorkspace ws, in
 #pragma unroll
   for (int o = 4; o > 0; o >>= 1) {
     gy += __shfl_xor_sync(0xffffffffu, gy, o);
+    gv += __shfl_xor_sync(0xffffffffu, gv, o);
     qk += __shfl_xor_sync(0xffffffffu, qk, o);
   }
-  if (!live) return;
-  if (sub == 0) {
-    float c2 = -INFINITY, nd = 0.f, nw = 0.f, lzn = -INFINITY;
+  float contrib = 0.f;
+  if (live && sub == 0) {
+    float c2 = -INFINITY, nd = 0.f, nw = 0.f;
     if (real) {
-      const float lz = p.logz_in[(long long)bh * p.T + r];
+      const long long srow = (long long)bh * p.T + r;
+      const float lz = p.logz_in[srow];
       const float li = logf((float)(r + 1));
       const float S = 1.0f / (1.0f + expf(-(qk * p.inv_sqrt_d) / p.tau_s));
+      const float F = expf(S - lz);
+      const float dR = F * (gv - gy);
+      ws.F_self[srow] = F;
+      ws.dS_self[srow] = dR * S * (1.0f - S) / p.tau_s;
+      contrib = li * (1.0f - F) * dR;
       c2 = (-p.lambda * li - lz) * kLog2e;
       nd = -gy;
-      nw = -li * expf(S - lz);
-      lzn = -lz * kLog2e;
+      nw = -li * F;
     }
-    float* st = ws.stats + ((long long)bh * n_t + (r >> 7)) * 4 * BT + (r & 127);
+    float* st = ws.stats + ((long long)bh * n_t + (r >> 7)) * 3 * BT + (r & 127);
     st[0] = c2;
     st[BT] = nd;
     st[2 * BT] = nw;
-    st[3 * BT] = lzn;
   }
-  float* acc = ws.dq_acc + ((long long)bh * ws.t_pad + r) * D + sub * PER;
 #pragma unroll
-  for (int c = 0; c < PER; c += 4) *reinterpret_cast<float4*>(acc + c) = make_float4(0.f, 0.f, 0.f, 0.f);
+  for (int o = 16; o > 0; o >>= 1) contrib += __shfl_xor_sync(0xffffffffu, contrib, o);
+  if ((threadIdx.x & 31) == 0) part[threadIdx.x >> 5] = contrib;
+  if (live) {
+    float* acc = ws.dq_acc + ((long long)bh * ws.t_pad + r) * D + sub * PER;
+#pragma unroll
+    for (int c = 0; c < PER; c += 4)
+      *reinterpret_cast<float4*>(acc + c) = make_float4(0.f, 0.f, 0.f, 0.f);
+  }
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    float t = 0.f;
+#pragma unroll
+    for (int w = 0; w < 8; ++w) t += part[w];
+    ws.dlam_part[blockIdx.x] = t;
+  }
 }
 
-// dq = bf16(dq_acc / (2 sqrt(d))) for rows < T; block 0 also reduces the tile kernel's
-// dlambda partials in a fixed order (deterministic).
+// dq = bf16(dq_acc / (2 sqrt(d)) + dS_ii k_i / sqrt(d)) for rows < T (the Exchange sums
+// plus the Self entry); block 0 also reduces the dlambda partials of the row pass
+// (n_pre) and of the tile kernel (n_cta) in a fixed order (deterministic).
 template <int D>
-__global__ void __launch_bounds__(256) finalize_kernel(Problem p, BwdWorkspace ws, int n_cta) {
+__global__ void __launch_bounds__(256) finalize_kernel(Problem p, BwdWorkspace ws, int n_pre,
+                                                       int n_cta) {
   if (blockIdx.x == 0) {
     __shared__ double part[256];
     double s = 0.0;
+    for (int i = threadIdx.x; i < n_pre; i += 256) s += (double)ws.dlam_part[i];
     for (int i = threadIdx.x; i < n_cta; i += 256) s += (double)ws.dlam_part[ws.n_pre_blocks + i];
     part[threadIdx.x] = s;
     __syncthreads();
@@ -689,15 +714,20 @@ __global__ void __launch_bounds__(256) finalize_kernel(Problem p, BwdWorkspace w
   const float* src = ws.dq_acc + ((long long)bh * ws.t_pad + r) * D + c8;
   const float4 a = *reinterpret_cast<const float4*>(src);
   const float4 c = *reinterpret_cast<const float4*>(src + 4);
+  const long long off = (long long)b * p.sB + (long long)h * p.sH + (long long)r * p.sT + c8;
+  const uint4 kv = *reinterpret_cast<const uint4*>(reinterpret_cast<const __nv_bfloat16*>(p.k) + off);
   const float sc = 0.5f * p.inv_sqrt_d;
+  const float self = ws.dS_self[row] * p.inv_sqrt_d;
+  const float2 k0 = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&kv.x));
+  const float2 k1 = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&kv.y));
+  const float2 k2 = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&kv.z));
+  const float2 k3 = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&kv.w));
   uint4 o;
-  o.x = pack_bf16x2(a.x * sc, a.y * sc);
-  o.y = pack_bf16x2(a.z * sc, a.w * sc);
-  o.z = pack_bf16x2(c.x * sc, c.y * sc);
-  o.w = pack_bf16x2(c.z * sc, c.w * sc);
-  __nv_bfloat16* dst = reinterpret_cast<__nv_bfloat16*>(p.dq) + (long long)b * p.sB +
-                       (long long)h * p.sH + (long long)r * p.sT + c8;
-  *reinterpret_cast<uint4*>(dst) = o;
+  o.x = pack_bf16x2(fmaf(a.x, sc, self * k0.x), fmaf(a.y, sc, self * k0.y));
+  o.y = pack_bf16x2(fmaf(a.z, sc, self * k1.x), fmaf(a.w, sc, self * k1.y));
+  o.z = pack_bf16x2(fmaf(c.x, sc, self * k2.x), fmaf(c.y, sc, self * k2.y));
+  o.w = pack_bf16x2(fmaf(c.z, sc, self * k3.x), fmaf(c.w, sc, self * k3.y));
+  *reinterpret_cast<uint4*>(reinterpret_cast<__nv_bfloat16*>(p.dq) + off) = o;
 }
 
 }  // namespace bwd
@@ -762,7 +792,9 @@ static cudaError_t bwd_t(const Problem& p, const BwdWorkspace& ws, unsigned stag
   if (stages & 4) {
     const long long chunks = rows * (D / 8);
     const long long fblocks = (chunks + 255) / 256;
-    bwd::finalize_kernel<D><<<(unsigned)(fblocks > 0 ? fblocks : 1), 256, 0, s>>>(p, ws, (int)grid);
+    const int n_pre = (int)((long long)p.B * p.H * t_pad / 32);  // row-pass blocks
+    bwd::finalize_kernel<D><<<(unsigned)(fblocks > 0 ? fblocks : 1), 256, 0, s>>>(p, ws, n_pre,
+                                                                                (int)grid);
     if ((e = cudaGetLastError()) != cudaSuccess) note_failure("backward: finalisation launch");
   }
   return e;
