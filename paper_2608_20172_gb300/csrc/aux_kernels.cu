@@ -39,7 +39,8 @@ size_t bwd_workspace_bytes(int B, int H, int T, int d) {
   const size_t rows_pad = (size_t)B * H * ((T + 127) / 128 * 128);
   const size_t n_pre = pre_slots(B, H, T);
   const size_t n_main = (size_t)((T + 63) / 64) * B * H;
-  return up(rows_pad * d * sizeof(float)) + 4 * up(rows * sizeof(float)) +
+  const size_t dpad = (size_t)(d + 63) / 64 * 64;  // the tensor-core path pads d_h to 64 / 128
+  return up(rows_pad * dpad * sizeof(float)) + 4 * up(rows * sizeof(float)) +
          up(rows_pad * 4 * sizeof(float)) + up((n_pre + n_main) * sizeof(float));
 }
 
@@ -50,7 +51,8 @@ BwdWorkspace carve_workspace(void* base, int B, int H, int T, int d) {
   char* p = static_cast<char*>(base);
   BwdWorkspace w;
   w.t_pad = t_pad;
-  w.dq_acc = reinterpret_cast<float*>(p); p += up((size_t)B * H * t_pad * d * sizeof(float));
+  const size_t dpad = (size_t)(d + 63) / 64 * 64;
+  w.dq_acc = reinterpret_cast<float*>(p); p += up((size_t)B * H * t_pad * dpad * sizeof(float));
   w.D = reinterpret_cast<float*>(p); p += up(rows * sizeof(float));
   w.F_self = reinterpret_cast<float*>(p); p += up(rows * sizeof(float));
   w.dS_self = reinterpret_cast<float*>(p); p += up(rows * sizeof(float));

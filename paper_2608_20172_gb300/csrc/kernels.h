@@ -35,7 +35,8 @@ struct Problem {
 
 // Backward workspace carved out of the caller's buffer (all fp32, 256-byte aligned).
 struct BwdWorkspace {
-  float* dq_acc;     // [B][H][T_pad][d] 2 sqrt(d) dL/dP1 in fp32, T_pad = T rounded up to 128
+  float* dq_acc;     // [B][H][T_pad][d_pad] 2 sqrt(d) dL/dP1 in fp32, T_pad = T rounded up to
+                     //   128, d_pad = d rounded up to 64
                      //   (tensor-core path: zeroed by its row pass, then summed by TMA reduce)
   int t_pad;
   float* D;          // [B][H][T]     D_i = dO_i . Y_i

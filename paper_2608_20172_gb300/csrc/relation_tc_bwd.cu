@@ -540,7 +540,8 @@ __global__ void __launch_bounds__(kThreads, 1)
       const __nv_bfloat16* row =
           reinterpret_cast<const __nv_bfloat16*>(wg == 0 ? p.q : p.dout) + off;
 #pragma unroll
-      for (int c = 0; c < D / 8; ++c) rowv[c] = *reinterpret_cast<const uint4*>(row + 8 * c);
+      for (int c = 0; c < D / 8; ++c)
+        rowv[c] = 8 * c < p.d ? *reinterpret_cast<const uint4*>(row + 8 * c) : make_uint4(0, 0, 0, 0);
       const long long srow = (long long)bh * p.T + j;
       self = wg == 0 ? ws.dS_self[srow] * isd : ws.F_self[srow];
     }
@@ -567,7 +568,8 @@ __global__ void __launch_bounds__(kThreads, 1)
               o4[e] = pack_bf16x2(fmaf(__uint_as_float(a[c8 + 2 * e]), sc, self * rf.x),
                                   fmaf(__uint_as_float(a[c8 + 2 * e + 1]), sc, self * rf.y));
             }
-            *reinterpret_cast<uint4*>(dst + c0 + c8) = make_uint4(o4[0], o4[1], o4[2], o4[3]);
+            if (c0 + c8 < p.d)  // padding columns (d_h < D) are not stored
+              *reinterpret_cast<uint4*>(dst + c0 + c8) = make_uint4(o4[0], o4[1], o4[2], o4[3]);
           }
         }
       }
@@ -620,6 +622,7 @@ __global__ void __launch_bounds__(256) pre_kernel(Problem p, BwdWorkspace ws, in
     };
 #pragma unroll
     for (int c = 0; c < PER; c += 8) {
+      if (sub * PER + c >= p.d) break;  // padding columns (d_h < D)
       const uint4 gv4 = bf(p.dout, off + c), ov = bf(p.o, off + c), vv = bf(p.v, off + c);
       const uint4 qv = bf(p.q, off + c), kv = bf(p.k, off + c);
       const uint32_t g4[4] = {gv4.x, gv4.y, gv4.z, gv4.w}, o4[4] = {ov.x, ov.y, ov.z, ov.w};
@@ -704,7 +707,7 @@ __global__ void __launch_bounds__(256) finalize_kernel(Problem p, BwdWorkspace w
     if (threadIdx.x == 0) *p.dlambda = (float)part[0];
   }
   const long long idx = ((long long)blockIdx.x * 256 + threadIdx.x);  // 8-wide chunk
-  const long long per_row = D / 8;
+  const long long per_row = p.d / 8;  // 8-column chunks of the real columns
   const long long n = (long long)p.B * p.H * p.T * per_row;
   if (idx >= n) return;
   const int c8 = (int)(idx % per_row) * 8;
@@ -790,7 +793,7 @@ static cudaError_t bwd_t(const Problem& p, const BwdWorkspace& ws, unsigned stag
     if ((e = cudaGetLastError()) != cudaSuccess) { note_failure("backward: tile kernel launch"); return e; }
   }
   if (stages & 4) {
-    const long long chunks = rows * (D / 8);
+    const long long chunks = rows * (p.d / 8);
     const long long fblocks = (chunks + 255) / 256;
     const int n_pre = (int)((long long)p.B * p.H * t_pad / 32);  // row-pass blocks
     bwd::finalize_kernel<D><<<(unsigned)(fblocks > 0 ? fblocks : 1), 256, 0, s>>>(p, ws, n_pre,
@@ -800,13 +803,12 @@ static cudaError_t bwd_t(const Problem& p, const BwdWorkspace& ws, unsigned stag
   return e;
 }
 
-bool supports_bwd(relation_dtype dt, int d) { return dt == RELATION_BF16 && (d == 64 || d == 128); }
+bool supports_bwd(relation_dtype dt, int d) { return supports(dt, d); }
 
 cudaError_t launch_bwd(const Problem& p, const BwdWorkspace& ws, unsigned stages,
                        cudaStream_t s) {
-  if (p.d == 64) return bwd_t<64>(p, ws, stages, s);
-  if (p.d == 128) return bwd_t<128>(p, ws, stages, s);
-  return cudaErrorInvalidValue;
+  if (!supports_bwd(p.dtype, p.d)) return cudaErrorInvalidValue;
+  return p.d <= 64 ? bwd_t<64>(p, ws, stages, s) : bwd_t<128>(p, ws, stages, s);
 }
 int bwd_launches() { return 3; }
 int main_ctas(const Problem& p) { return ((p.T + 127) / 128) * p.B * p.H; }

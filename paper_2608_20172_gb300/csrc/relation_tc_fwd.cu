@@ -432,7 +432,12 @@ bool make_tmap_bf16(CUtensorMap* m, const void* base, const Problem& p, int rows
   return r == CUDA_SUCCESS;
 }
 
-bool supports(relation_dtype dt, int d) { return dt == RELATION_BF16 && (d == 64 || d == 128); }
+// bf16 with d_h a multiple of 8 up to 128: the kernels run at d_pad = 64 or 128, the TMA
+// loads filling columns d_h .. d_pad - 1 with zeros (they add nothing to U, z or the
+// gradients) and the TMA stores clipping them.
+bool supports(relation_dtype dt, int d) {
+  return dt == RELATION_BF16 && d >= 8 && d <= 128 && d % 8 == 0;
+}
 
 template <int D>
 static cudaError_t fwd_t(const Problem& p, cudaStream_t s) {
@@ -457,9 +462,8 @@ static cudaError_t fwd_t(const Problem& p, cudaStream_t s) {
 }
 
 cudaError_t launch_fwd(const Problem& p, cudaStream_t s) {
-  if (p.d == 64) return fwd_t<64>(p, s);
-  if (p.d == 128) return fwd_t<128>(p, s);
-  return cudaErrorInvalidValue;
+  if (!supports(p.dtype, p.d)) return cudaErrorInvalidValue;
+  return p.d <= 64 ? fwd_t<64>(p, s) : fwd_t<128>(p, s);
 }
 
 }  // namespace tc

@@ -64,8 +64,8 @@ def kernel_available(kernel: str, dtype: str, d: int, which: str = "fwd") -> boo
 def kernel_combos(dtype: str, d: int):
     """(forward family, backward family) pairs to test: the CUDA-core pair always, and
     each tensor-core kernel the library offers for this (dtype, d)."""
-    combos = [("simt", "simt")]
-    if kernel_available("tcgen05", dtype, d, "fwd"):
+    combos = [("simt", "simt")] if kernel_available("simt", dtype, d, "fwd") else []
+    if kernel_available("tcgen05", dtype, d, "fwd") and combos:
         combos.append(("tcgen05", "simt"))
     if kernel_available("tcgen05", dtype, d, "bwd"):
         combos.append(("tcgen05", "tcgen05"))

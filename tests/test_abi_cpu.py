@@ -72,7 +72,8 @@ GOOD = [0x10000, 0x20000, 0x30000, 0x40000, 0x50000]  # aligned, never dereferen
     ("null q", binding.ERR_INVALID_ARG),
     ("misaligned v", binding.ERR_ALIGNMENT),
     ("T = 0", binding.ERR_INVALID_ARG),
-    ("d = 40", binding.ERR_UNSUPPORTED),
+    ("d = 36", binding.ERR_UNSUPPORTED),
+    ("d = 136", binding.ERR_UNSUPPORTED),
     ("odd stride", binding.ERR_ALIGNMENT),
     ("tau = 0", binding.ERR_INVALID_ARG),
     ("lambda inf", binding.ERR_INVALID_ARG),
@@ -88,8 +89,10 @@ def test_fwd_rejects_bad_arguments(lib, case, expect):
         ptrs[2] = 0x30008
     elif case == "T = 0":
         shape = _shape(T=0)
-    elif case == "d = 40":
-        shape = _shape(d=40)
+    elif case == "d = 36":
+        shape = _shape(d=36)
+    elif case == "d = 136":
+        shape = _shape(d=136)
     elif case == "odd stride":
         shape = _shape(sT=130)
     elif case == "tau = 0":

@@ -81,9 +81,25 @@ def test_bf16_lambda_values(lam):
 def test_bf16_32():
     w = workloads.custom(1, 3, 150, 32, "bf16")
     q, k, v, do = workloads.make_inputs(w, seed=3)
-    res = pu.gpu_run(q, k, v, do, LAM)
     ref = pu.oracle_heads(q, k, v, do, LAM, _all_heads(w))
+    for kf, kb in pu.kernel_combos("bf16", 32):
+        res = pu.gpu_run(q, k, v, do, LAM, kernel=kf, kernel_bwd=kb)
+        pu.compare_heads(res, ref, "bf16")
+
+
+@pytest.mark.parametrize("T", [1, 129, 300])
+@pytest.mark.parametrize("d", [16, 48, 80, 96])
+def test_bf16_padded_head_sizes(T, d):
+    """Head sizes other than 64 and 128 (the paper's layer geometry uses d_h = 48 and 80)
+    run the tensor-core kernels on tiles zero-padded to 64 or 128 columns."""
+    assert pu.kernel_available("tcgen05", "bf16", d, "fwd")
+    assert pu.kernel_available("tcgen05", "bf16", d, "bwd")
+    w = workloads.custom(1, 2, T, d, "bf16")
+    q, k, v, do = workloads.make_inputs(w, seed=2000 + T + d)
+    ref = pu.oracle_heads(q, k, v, do, LAM, _all_heads(w))
+    res = pu.gpu_run(q, k, v, do, LAM, kernel="tcgen05")
     pu.compare_heads(res, ref, "bf16")
+    pu.check_dlambda(res["dlambda"], sum(r["dlambda"] for r in ref.values()), "bf16")
 
 
 def test_bhtd_layout():
@@ -216,7 +232,7 @@ def test_device_argument_errors():
     with pytest.raises(binding.RelationError) as e:
         binding.fwd(mis, mis, mis, LAM)
     assert e.value.code == binding.ERR_ALIGNMENT
-    odd = torch.zeros(1, 8, 1, 40, dtype=torch.bfloat16, device=dev)
+    odd = torch.zeros(1, 8, 1, 136, dtype=torch.bfloat16, device=dev)
     with pytest.raises(binding.RelationError) as e:
         binding.fwd(odd, odd, odd, LAM)
     assert e.value.code == binding.ERR_UNSUPPORTED
