@@ -96,6 +96,21 @@ relation_status relation_fwd_ex(const void* q, const void* k, const void* v, voi
                                 float lambda, float tau_s, relation_shape shp, relation_dtype dt,
                                 relation_kernel kernel, int* dev_status, relation_stream_t stream);
 
+/*
+ * relation_fwd_ex with one more output, the Self flow of every row:
+ *   self_flow [B][H][T] fp32 : F_ii = exp(R_ii - logZ_i) = sigmoid(S_i - A_i) = 1 - g_i,
+ * the share of row i's normalised flow F that stays on the Self relation (Sec. 4.2, the
+ * Self-Exchange factorisation; its complement g_i is the Exchange share).  This is the
+ * per-row quantity behind the paper's "Self flow" and "Self / Exchange" structural
+ * diagnostics (App. B.4, B.5); averaging it is left to the caller.  Row 1 has no history: F_11 = 1.  self_flow may be null (then this is
+ * relation_fwd_ex); otherwise it must be 16-byte aligned.  Y and logz are identical to
+ * relation_fwd_ex's.
+ */
+relation_status relation_fwd_flow(const void* q, const void* k, const void* v, void* o,
+                                  float* logz, float* self_flow, float lambda, float tau_s,
+                                  relation_shape shp, relation_dtype dt, relation_kernel kernel,
+                                  int* dev_status, relation_stream_t stream);
+
 /* Bytes of device workspace relation_bwd needs for this shape and dtype (0 on a bad
  * shape).  The content of the workspace need not be initialised. */
 size_t relation_bwd_workspace_size(relation_shape shp, relation_dtype dt);

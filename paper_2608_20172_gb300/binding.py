@@ -29,7 +29,7 @@ KERNELS = {"auto": 0, "simt": 1, "tcgen05": 2}
 EXPORTED = ("relation_fwd", "relation_fwd_ex", "relation_bwd", "relation_bwd_ex",
             "relation_bwd_workspace_size", "relation_status_string", "relation_version",
             "relation_selftest_wait_timeout", "relation_launch_count", "relation_last_cuda_error",
-            "relation_bwd_stages", "relation_bwd_static")
+            "relation_bwd_stages", "relation_bwd_static", "relation_fwd_flow")
 
 
 class RelationLibraryMissing(RuntimeError):
@@ -70,6 +70,7 @@ def load(path: str | None = None):
         f, i, sz = ctypes.c_float, ctypes.c_int, ctypes.c_size_t
         lib.relation_fwd.argtypes = [vp, vp, vp, vp, vp, f, f, Shape, i, ip, vp]
         lib.relation_fwd_ex.argtypes = [vp, vp, vp, vp, vp, f, f, Shape, i, i, ip, vp]
+        lib.relation_fwd_flow.argtypes = [vp, vp, vp, vp, vp, vp, f, f, Shape, i, i, ip, vp]
         lib.relation_bwd.argtypes = [vp, vp, vp, vp, vp, vp, vp, vp, vp, vp, f, f, Shape, i, vp,
                                      sz, ip, vp]
         lib.relation_bwd_ex.argtypes = [vp, vp, vp, vp, vp, vp, vp, vp, vp, vp, f, f, Shape, i,
@@ -157,6 +158,28 @@ def fwd(q, k, v, lam: float, tau_s: float = 2.0, *, kernel: str = "auto", out=No
     if rc != OK:
         raise RelationError(rc, "relation_fwd")
     return out, logz
+
+
+def fwd_flow(q, k, v, lam: float, tau_s: float = 2.0, *, kernel: str = "auto", out=None,
+             logz=None, self_flow=None, dev_status=None, stream=None):
+    """Forward with the Self flow F_ii = 1 - g_i of every row as a side output.
+    Returns (Y, logZ, F_self) with F_self [B, H, T] fp32."""
+    _same_layout(q, k, v)
+    B, T, H, _ = q.shape
+    if out is None:
+        out = torch.empty_like(q)
+    _same_layout(q, out)
+    if logz is None:
+        logz = torch.empty((B, H, T), device=q.device, dtype=torch.float32)
+    if self_flow is None:
+        self_flow = torch.empty((B, H, T), device=q.device, dtype=torch.float32)
+    rc = load().relation_fwd_flow(_ptr(q), _ptr(k), _ptr(v), _ptr(out), _ptr(logz),
+                                  _ptr(self_flow), float(lam), float(tau_s), shape_of(q),
+                                  _dtype_code(q), KERNELS[kernel], _ptr(dev_status),
+                                  ctypes.c_void_p(_stream(stream)))
+    if rc != OK:
+        raise RelationError(rc, "relation_fwd_flow")
+    return out, logz, self_flow
 
 
 BWD_PREPARE, BWD_TILES, BWD_FINALIZE, BWD_ALL = 1, 2, 4, 7

@@ -21,6 +21,7 @@ struct Problem {
   void* dk;
   void* dv;
   float* logz;         // forward output [B][H][T]
+  float* fself;        // optional forward output [B][H][T]: the Self flow F_ii (may be null)
   const float* logz_in;  // backward input [B][H][T]
   float* dlambda;      // backward output (one float)
   int* dev_status;

@@ -87,20 +87,29 @@ void note_failure(const char* where) { g_last_where = where; }
 
 extern "C" {
 
-relation_status relation_fwd_ex(const void* q, const void* k, const void* v, void* o, float* logz,
-                                float lambda, float tau_s, relation_shape shp, relation_dtype dt,
-                                relation_kernel kernel, int* dev_status, relation_stream_t stream) {
+relation_status relation_fwd_flow(const void* q, const void* k, const void* v, void* o,
+                                  float* logz, float* self_flow, float lambda, float tau_s,
+                                  relation_shape shp, relation_dtype dt, relation_kernel kernel,
+                                  int* dev_status, relation_stream_t stream) {
   relation_status st;
   if ((st = check_shape(shp, dt)) != RELATION_OK) return st;
   if ((st = check_scalars(lambda, tau_s)) != RELATION_OK) return st;
   if ((st = check_ptrs({q, k, v, o, logz})) != RELATION_OK) return st;
+  if (self_flow && (st = check_ptrs({self_flow})) != RELATION_OK) return st;
   if (dev_status && (reinterpret_cast<uintptr_t>(dev_status) & 3u)) return RELATION_ERR_ALIGNMENT;
   const int fam = pick_family(kernel, dt, shp.d_h, false);
   if (fam == 0) return RELATION_ERR_UNSUPPORTED;
   Problem p = make_problem(shp, dt, lambda, tau_s, dev_status);
-  p.q = q; p.k = k; p.v = v; p.out = o; p.logz = logz;
+  p.q = q; p.k = k; p.v = v; p.out = o; p.logz = logz; p.fself = self_flow;
   cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
   return from_cuda(fam == 2 ? rel::tc::launch_fwd(p, s) : rel::simt::launch_fwd(p, s));
+}
+
+relation_status relation_fwd_ex(const void* q, const void* k, const void* v, void* o, float* logz,
+                                float lambda, float tau_s, relation_shape shp, relation_dtype dt,
+                                relation_kernel kernel, int* dev_status, relation_stream_t stream) {
+  return relation_fwd_flow(q, k, v, o, logz, nullptr, lambda, tau_s, shp, dt, kernel, dev_status,
+                           stream);
 }
 
 relation_status relation_fwd(const void* q, const void* k, const void* v, void* o, float* logz,

@@ -183,10 +183,11 @@ __global__ void __launch_bounds__(kThreads) fwd_kernel(Problem p) {
   if (!row_ok) return;
 
   float g = 0.f, lz = s_self;
-  float inv_l = 0.f;
+  float inv_l = 0.f, fself = 1.0f;  // F_ii = 1 - g: the Self flow
   if (r > 0 && l > 0.f) {
     const float A = m + logf(l) - p.lambda * logf((float)(r + 1));
     g = 1.0f / (1.0f + expf(s_self - A));
+    fself = 1.0f / (1.0f + expf(A - s_self));
     const float hi = fmaxf(s_self, A), lo = fminf(s_self, A);
     lz = hi + log1pf(expf(lo - hi));
     inv_l = 1.0f / l;
@@ -203,7 +204,10 @@ __global__ void __launch_bounds__(kThreads) fwd_kernel(Problem p) {
     y.w = (1.f - g) * vi[4 * c + 3] + g * (z[4 * c + 3] * inv_l);
     IO<TI>::store4(Y + Chunks<D>::col(part, c), y);
   }
-  if (part == 0) p.logz[(long long)bh * p.T + r] = lz;
+  if (part == 0) {
+    p.logz[(long long)bh * p.T + r] = lz;
+    if (p.fself) p.fself[(long long)bh * p.T + r] = fself;
+  }
 }
 
 // ---------------------------------------------------------------------------

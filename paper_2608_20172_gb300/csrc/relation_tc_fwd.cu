@@ -337,12 +337,13 @@ __global__ void __launch_bounds__(kThreads, 2)
     if (ok) ok = __all_sync(0xffffffffu, mbar_wait(bar(B_O), 0, ab));
     tc_fence_after();
     if (ok) {
-      float g = 0.f, inv_l = 0.f;
+      float g = 0.f, inv_l = 0.f, fself = 1.0f;  // F_ii = 1 - g: the Self flow
       float lz;
       const float S = 1.0f / (1.0f + __expf(-(u_self * isd) / p.tau_s));
       if (l > 0.f) {
         const float A = m * kLn2 + __logf(l) - p.lambda * __logf((float)(r + 1));
         g = 1.0f / (1.0f + __expf(S - A));
+        fself = 1.0f / (1.0f + __expf(A - S));
         const float hi = fmaxf(S, A), lo = fminf(S, A);
         lz = hi + log1pf(__expf(lo - hi));
         inv_l = 1.0f / l;
@@ -388,7 +389,10 @@ __global__ void __launch_bounds__(kThreads, 2)
         tma_store_wait_all();  // the staging buffer must outlive the store
       }
       __syncwarp();
-      if (r < p.T) p.logz[(long long)bh * p.T + r] = lz;
+      if (r < p.T) {
+        p.logz[(long long)bh * p.T + r] = lz;
+        if (p.fself) p.fself[(long long)bh * p.T + r] = fself;
+      }
     }
   }
 

@@ -253,3 +253,32 @@ def test_autograd_wrapper_matches_binding():
     assert torch.equal(y.detach().float().cpu(), res["Y"])
     assert torch.equal(kd.grad.float().cpu(), res["dK"])
     assert abs(float(lam.grad) - res["dlambda"]) <= 1e-6 * max(1.0, abs(res["dlambda"]))
+
+
+# --- Self-flow side output ------------------------------------------------------
+
+@pytest.mark.parametrize("dtype,d,T", [("fp32", 64, 200), ("bf16", 64, 300), ("bf16", 128, 257),
+                                       ("bf16", 48, 130)])
+def test_self_flow_side_output(dtype, d, T):
+    """relation_fwd_flow returns F_ii = 1 - g_i per row (the Self share of the flow) next to
+    the same Y and logZ as relation_fwd, for every kernel family that serves the shape."""
+    w = workloads.custom(2, 2, T, d, dtype, qk_std=(1.0 / np.sqrt(d)) if dtype == "fp32" else 1.0)
+    q, k, v, _ = workloads.make_inputs(w, seed=5000 + T + d)
+    dev = torch.device("cuda:0")
+    qd, kd, vd = (t.to(dev) for t in (q, k, v))
+    tol = 1e-5 if dtype == "fp32" else 2e-3
+    fams = [f for f in ("simt", "tcgen05") if pu.kernel_available(f, dtype, d, "fwd")]
+    assert fams
+    for fam in fams:
+        y0, lz0 = binding.fwd(qd, kd, vd, LAM, kernel=fam)
+        y, lz, fs = binding.fwd_flow(qd, kd, vd, LAM, kernel=fam)
+        torch.cuda.synchronize()
+        assert torch.equal(y, y0) and torch.equal(lz, lz0), fam
+        fs = fs.cpu().numpy()
+        for b in range(w.B):
+            for h in range(w.H):
+                ref = oracle.fwd_factorized(q[b, :, h].double().numpy(), k[b, :, h].double().numpy(),
+                                            v[b, :, h].double().numpy(), LAM)
+                err = np.abs(fs[b, h] - ref["Fii"]).max()
+                assert err <= tol, f"{fam} head ({b},{h}): max |F_ii - ref| = {err:.3g} > {tol}"
+                assert fs[b, h, 0] == 1.0
