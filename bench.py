@@ -232,6 +232,49 @@ def run_reference(args, w):
 # GPU arm
 # ------------------------------------------------------------------------------
 
+DECODE_CFG = {"B": 32, "H": 16, "T": 8192, "d_h": 128}  # bf16 cache of 2.1 GB (K + V)
+
+
+def decode_measure(binding, dev, peaks, steps=20, warmup=3):
+    """relation_decode on a bf16 cache larger than L2 (every sequence at full length):
+    algorithmic bytes = the K and V rows read + q, Y, logZ; HBM roofline."""
+    c = DECODE_CFG
+    B, H, T, d = c["B"], c["H"], c["T"], c["d_h"]
+    g = torch.Generator(device="cpu").manual_seed(0)
+    kc = torch.randn((B, T, H, d), generator=g).to(torch.bfloat16).to(dev)
+    vc = torch.randn((B, T, H, d), generator=g).to(torch.bfloat16).to(dev)
+    qn = torch.randn((B, H, d), generator=g).to(torch.bfloat16).to(dev)
+    lens = torch.full((B,), T, dtype=torch.int32, device=dev)
+    out = torch.empty_like(qn)
+    logz = torch.empty((B, H), dtype=torch.float32, device=dev)
+    wsb = torch.empty(binding.decode_workspace_size(kc), dtype=torch.uint8, device=dev)
+    status = torch.zeros(1, dtype=torch.int32, device=dev)
+    stream = torch.cuda.current_stream(dev)
+    call = lambda: binding.decode(qn, kc, vc, lens, workloads.LAMBDA_INIT, out=out, logz=logz,
+                                  workspace=wsb, dev_status=status, stream=stream)
+    for _ in range(warmup):
+        call()
+    ev = [torch.cuda.Event(enable_timing=True) for _ in range(steps + 1)]
+    torch.cuda.synchronize(dev)
+    ev[0].record(stream)
+    for i in range(steps):
+        call()
+        ev[i + 1].record(stream)
+    torch.cuda.synchronize(dev)
+    if int(status.item()) != 0:
+        raise SystemExit(f"decode device status {binding.status_string(int(status.item()))}")
+    ms = statistics.mean(ev[i].elapsed_time(ev[i + 1]) for i in range(steps))
+    nbytes = 2.0 * B * T * H * d * 2 + 2.0 * B * H * d * 2 + B * H * 4
+    gbs = nbytes / (ms * 1e-3) / 1e9
+    return {"config": {**c, "dtype": "bf16", "lengths": "all T",
+                       "l2": "cache 2.1 GB > L2, no flush"},
+            "ms_per_call": ms, "tokens_per_s": B / (ms * 1e-3),
+            "roofline": {"bound": "hbm", "achieved": gbs, "peak": peaks["hbm_gbs"],
+                         "unit": "GB/s", "frac": gbs / peaks["hbm_gbs"],
+                         "algorithmic_bytes_per_call": nbytes},
+            "gpu_launches_per_call": 2}
+
+
 def run_ours(args, w):
     from paper_2608_20172_gb300 import binding
     dist, ws, rank, local = _dist()
@@ -368,6 +411,8 @@ def run_ours(args, w):
                              + binding.launches_per_call(family, w.dtype, w.d, "bwd")),
         "clocks": clocks,
     }
+    if rank == 0 and ws == 1:
+        line["decode"] = decode_measure(binding, dev, peaks)
     if rank == 0 and not args.no_cpu_baseline and ws == 1:
         cb = cpu_oracle_run(w, min_seconds=10.0)
         line["cpu_baseline"] = {

@@ -111,6 +111,29 @@ relation_status relation_fwd_flow(const void* q, const void* k, const void* v, v
                                   relation_shape shp, relation_dtype dt, relation_kernel kernel,
                                   int* dev_status, relation_stream_t stream);
 
+/*
+ * Decoding: the forward row of one new token per sequence, against a key/value cache.
+ *   q        [B][H][d_h] queries of the new tokens, element strides q_sB, q_sH (d_h
+ *            contiguous); o (output Y) has the same layout.
+ *   k_cache, v_cache : [B][T][H][d_h] with the strides of `cache` (T = cache capacity).
+ *   lengths  device int[B]: rows of sequence b in the cache, 1 <= len_b <= T; row
+ *            len_b - 1 holds the new token's key and value, and len_b is its one-based
+ *            position i in ln(i).
+ *   logz     [B][H] fp32 output: log of the new row's normaliser.
+ *   workspace, ws_bytes : device scratch of relation_decode_workspace_size(cache, dt).
+ * Y and logz equal row len_b - 1 of relation_fwd over the first len_b cache rows (the
+ * Self-Exchange row of Sec. 3.1 in the factorised form of Sec. 4.2): Exchange over the
+ * len_b - 1 history rows, Self with the token's own key.  bf16 or fp32 with any 1 <= d_h <= 128.
+ * A length outside [1, T] is not read: the heads of that sequence are skipped and
+ * dev_status (if given) receives RELATION_ERR_INVALID_ARG.  Asynchronous on `stream`.
+ */
+size_t relation_decode_workspace_size(relation_shape cache, relation_dtype dt);
+relation_status relation_decode(const void* q, const void* k_cache, const void* v_cache,
+                                const int* lengths, void* o, float* logz, float lambda,
+                                float tau_s, relation_shape cache, long long q_sB, long long q_sH,
+                                relation_dtype dt, void* workspace, size_t ws_bytes,
+                                int* dev_status, relation_stream_t stream);
+
 /* Bytes of device workspace relation_bwd needs for this shape and dtype (0 on a bad
  * shape).  The content of the workspace need not be initialised. */
 size_t relation_bwd_workspace_size(relation_shape shp, relation_dtype dt);

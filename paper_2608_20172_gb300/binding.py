@@ -29,7 +29,8 @@ KERNELS = {"auto": 0, "simt": 1, "tcgen05": 2}
 EXPORTED = ("relation_fwd", "relation_fwd_ex", "relation_bwd", "relation_bwd_ex",
             "relation_bwd_workspace_size", "relation_status_string", "relation_version",
             "relation_selftest_wait_timeout", "relation_launch_count", "relation_last_cuda_error",
-            "relation_bwd_stages", "relation_bwd_static", "relation_fwd_flow")
+            "relation_bwd_stages", "relation_bwd_static", "relation_fwd_flow",
+            "relation_decode", "relation_decode_workspace_size")
 
 
 class RelationLibraryMissing(RuntimeError):
@@ -71,6 +72,11 @@ def load(path: str | None = None):
         lib.relation_fwd.argtypes = [vp, vp, vp, vp, vp, f, f, Shape, i, ip, vp]
         lib.relation_fwd_ex.argtypes = [vp, vp, vp, vp, vp, f, f, Shape, i, i, ip, vp]
         lib.relation_fwd_flow.argtypes = [vp, vp, vp, vp, vp, vp, f, f, Shape, i, i, ip, vp]
+        ll = ctypes.c_longlong
+        lib.relation_decode.argtypes = [vp, vp, vp, vp, vp, vp, f, f, Shape, ll, ll, i, vp,
+                                        ctypes.c_size_t, ip, vp]
+        lib.relation_decode_workspace_size.argtypes = [Shape, i]
+        lib.relation_decode_workspace_size.restype = ctypes.c_size_t
         lib.relation_bwd.argtypes = [vp, vp, vp, vp, vp, vp, vp, vp, vp, vp, f, f, Shape, i, vp,
                                      sz, ip, vp]
         lib.relation_bwd_ex.argtypes = [vp, vp, vp, vp, vp, vp, vp, vp, vp, vp, f, f, Shape, i,
@@ -180,6 +186,40 @@ def fwd_flow(q, k, v, lam: float, tau_s: float = 2.0, *, kernel: str = "auto", o
     if rc != OK:
         raise RelationError(rc, "relation_fwd_flow")
     return out, logz, self_flow
+
+
+def decode_workspace_size(k_cache) -> int:
+    """Device bytes relation_decode needs for a [B, T, H, d] cache of this dtype."""
+    return int(load().relation_decode_workspace_size(shape_of(k_cache), _dtype_code(k_cache)))
+
+
+def decode(q, k_cache, v_cache, lengths, lam: float, tau_s: float = 2.0, *, out=None, logz=None,
+           workspace=None, dev_status=None, stream=None):
+    """One new token per sequence against a [B, T, H, d] key/value cache whose row
+    lengths[b] - 1 is that token.  q is [B, H, d]; lengths is a device int32 [B].
+    Returns (Y [B, H, d], logZ [B, H])."""
+    _same_layout(k_cache, v_cache)
+    B, T, H, d = k_cache.shape
+    if tuple(q.shape) != (B, H, d) or q.stride(2) != 1 or q.dtype != k_cache.dtype:
+        raise ValueError("q must be [B, H, d] with d contiguous, of the cache's dtype")
+    if lengths.dtype != torch.int32 or lengths.numel() != B or not lengths.is_contiguous():
+        raise ValueError("lengths must be a contiguous int32 tensor of B entries")
+    out = torch.empty_like(q) if out is None else out
+    if tuple(out.stride()) != tuple(q.stride()):
+        raise ValueError("out must have q's layout")
+    if logz is None:
+        logz = torch.empty((B, H), device=q.device, dtype=torch.float32)
+    need = decode_workspace_size(k_cache)
+    if workspace is None:
+        workspace = torch.empty(need, device=q.device, dtype=torch.uint8)
+    rc = load().relation_decode(_ptr(q), _ptr(k_cache), _ptr(v_cache), _ptr(lengths), _ptr(out),
+                                _ptr(logz), float(lam), float(tau_s), shape_of(k_cache),
+                                q.stride(0), q.stride(1), _dtype_code(q), _ptr(workspace),
+                                workspace.numel() * workspace.element_size(), _ptr(dev_status),
+                                ctypes.c_void_p(_stream(stream)))
+    if rc != OK:
+        raise RelationError(rc, "relation_decode")
+    return out, logz
 
 
 BWD_PREPARE, BWD_TILES, BWD_FINALIZE, BWD_ALL = 1, 2, 4, 7

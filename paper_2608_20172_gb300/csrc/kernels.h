@@ -81,6 +81,24 @@ int bwd_launches();  // launches made by launch_bwd with every stage
 int main_ctas(const Problem& p);
 }  // namespace tc
 
+// Decoding: one new token per sequence against a key/value cache (relation_decode.cu).
+struct DecodeProblem {
+  const void* q;        // [B][H][d] queries of the new tokens (element strides qsB, qsH)
+  const void* k;        // caches [B][T][H][d] (element strides sB, sT, sH); row len_b - 1 of
+  const void* v;        //   sequence b is the new token
+  const int* lengths;   // device [B]: cached rows per sequence, 1 <= len_b <= T
+  void* out;            // [B][H][d] like q
+  float* logz;          // [B][H]
+  int* dev_status;      // nullable: RELATION_ERR_INVALID_ARG for a length outside [1, T]
+  float lambda, tau_s, inv_sqrt_d;
+  int B, T, H, d;
+  long long sB, sT, sH, qsB, qsH;
+  relation_dtype dtype;
+};
+int decode_chunks(int t_max);
+size_t decode_workspace_bytes(int B, int H, int t_max);
+cudaError_t launch_decode(const DecodeProblem& p, void* workspace, cudaStream_t s);
+
 cudaError_t launch_selftest_wait(int* dev_status, int timeout_us, cudaStream_t s);
 
 // Where the last failing CUDA step of this thread happened (reported by

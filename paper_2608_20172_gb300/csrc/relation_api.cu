@@ -119,6 +119,41 @@ relation_status relation_fwd(const void* q, const void* k, const void* v, void* 
                          dev_status, stream);
 }
 
+size_t relation_decode_workspace_size(relation_shape cache, relation_dtype dt) {
+  if (dt != RELATION_F32 && dt != RELATION_BF16) return 0;
+  if (cache.B < 1 || cache.T < 1 || cache.H < 1 || cache.d_h < 1 || cache.d_h > 128) return 0;
+  return rel::decode_workspace_bytes(cache.B, cache.H, cache.T);
+}
+
+relation_status relation_decode(const void* q, const void* k_cache, const void* v_cache,
+                                const int* lengths, void* o, float* logz, float lambda,
+                                float tau_s, relation_shape cache, long long q_sB, long long q_sH,
+                                relation_dtype dt, void* workspace, size_t ws_bytes,
+                                int* dev_status, relation_stream_t stream) {
+  relation_status st;
+  if (dt != RELATION_F32 && dt != RELATION_BF16) return RELATION_ERR_INVALID_ARG;
+  if (cache.B < 1 || cache.T < 1 || cache.H < 1 || cache.d_h < 1) return RELATION_ERR_INVALID_ARG;
+  if (cache.d_h > 128) return RELATION_ERR_UNSUPPORTED;
+  if ((long long)cache.B * cache.H > 0x7fffffffLL) return RELATION_ERR_UNSUPPORTED;
+  if (cache.sB < 1 || cache.sT < 1 || cache.sH < 1 || q_sB < 1 || q_sH < 1)
+    return RELATION_ERR_INVALID_ARG;
+  if ((st = check_scalars(lambda, tau_s)) != RELATION_OK) return st;
+  if ((st = check_ptrs({q, k_cache, v_cache, lengths, o, logz, workspace})) != RELATION_OK)
+    return st;
+  if (dev_status && (reinterpret_cast<uintptr_t>(dev_status) & 3u)) return RELATION_ERR_ALIGNMENT;
+  if (ws_bytes < rel::decode_workspace_bytes(cache.B, cache.H, cache.T))
+    return RELATION_ERR_WORKSPACE;
+  rel::DecodeProblem p{};
+  p.q = q; p.k = k_cache; p.v = v_cache; p.lengths = lengths; p.out = o; p.logz = logz;
+  p.dev_status = dev_status;
+  p.lambda = lambda; p.tau_s = tau_s; p.inv_sqrt_d = 1.0f / sqrtf((float)cache.d_h);
+  p.B = cache.B; p.T = cache.T; p.H = cache.H; p.d = cache.d_h;
+  p.sB = cache.sB; p.sT = cache.sT; p.sH = cache.sH; p.qsB = q_sB; p.qsH = q_sH;
+  p.dtype = dt;
+  if (rel::decode_chunks(cache.T) > 65535) return RELATION_ERR_UNSUPPORTED;  // grid.y limit
+  return from_cuda(rel::launch_decode(p, workspace, reinterpret_cast<cudaStream_t>(stream)));
+}
+
 size_t relation_bwd_workspace_size(relation_shape shp, relation_dtype dt) {
   if (check_shape(shp, dt) != RELATION_OK) return 0;
   return rel::bwd_workspace_bytes(shp.B, shp.H, shp.T, shp.d_h);
