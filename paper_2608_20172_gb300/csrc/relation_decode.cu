@@ -13,8 +13,8 @@
 // rows.  Memory-bound: every cached key and value is read once.
 //
 // Two launches.  The partial pass splits each history into chunks of kChunk rows, one CTA
-// per (head, chunk): 8 warps take the chunk's rows in turn, the lanes of a warp spanning
-// d, and the CTA leaves (m, l, z) = (max E, sum e^{E - m}, sum e^{E - m} v) in the
+// per (head, chunk): 8 warps take the chunk's rows in turn (scores with four lanes per
+// key, P V with the lanes spanning d), and the CTA leaves (m, l, z) = (max E, sum e^{E - m}, sum e^{E - m} v) in the
 // workspace.  The combine pass (one CTA per head, one thread per column) merges the
 // chunks with the associative (m, l, z) rule of the tiled scan (App. A.3) and applies the
 // Self-Exchange epilogue.
@@ -39,8 +39,57 @@ __device__ __forceinline__ float ldf<__nv_bfloat16>(const __nv_bfloat16* p) {
   return __bfloat162float(*p);
 }
 
+// Loads of n consecutive elements as fp32 (n * sizeof(TI) is 4, 8 or 16 bytes, aligned).
+template <typename TI, int N>
+__device__ __forceinline__ void ld_vec(const TI* p, float* out) {
+  if constexpr (sizeof(TI) == 4) {
+    static_assert(N % 4 == 0 || N <= 2, "fp32 vector width");
+    if constexpr (N == 1) {
+      out[0] = __ldg(reinterpret_cast<const float*>(p));
+    } else if constexpr (N == 2) {
+      const float2 v = __ldg(reinterpret_cast<const float2*>(p));
+      out[0] = v.x; out[1] = v.y;
+    } else {
+#pragma unroll
+      for (int i = 0; i < N; i += 4) {
+        const float4 v = __ldg(reinterpret_cast<const float4*>(p + i));
+        out[i] = v.x; out[i + 1] = v.y; out[i + 2] = v.z; out[i + 3] = v.w;
+      }
+    }
+  } else {
+    if constexpr (N == 2) {
+      const uint32_t w = __ldg(reinterpret_cast<const unsigned int*>(p));
+      const float2 f = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&w));
+      out[0] = f.x; out[1] = f.y;
+    } else if constexpr (N == 4) {
+      const uint2 w = __ldg(reinterpret_cast<const uint2*>(p));
+      const uint32_t ww[2] = {w.x, w.y};
+#pragma unroll
+      for (int e = 0; e < 2; ++e) {
+        const float2 f = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&ww[e]));
+        out[2 * e] = f.x; out[2 * e + 1] = f.y;
+      }
+    } else {
+      static_assert(N % 8 == 0, "bf16 vector width");
+#pragma unroll
+      for (int i = 0; i < N; i += 8) {
+        const uint4 w = __ldg(reinterpret_cast<const uint4*>(p + i));
+        const uint32_t ww[4] = {w.x, w.y, w.z, w.w};
+#pragma unroll
+        for (int e = 0; e < 4; ++e) {
+          const float2 f = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&ww[e]));
+          out[i + 2 * e] = f.x; out[i + 2 * e + 1] = f.y;
+        }
+      }
+    }
+  }
+}
+
 // Partial (m, l, z) of history rows [c0, min(c0 + kChunk, len - 1)) of head (b, h).
-template <typename TI>
+// D = 64 or 128: vector loads (scores: four lanes per key, each a quarter of the row;
+// P V: each lane D / 32 consecutive columns).  D = 0: any d_h <= 128, one element per
+// lane per load.
+template <typename TI, int D>
 __global__ void __launch_bounds__(kWarps * 32) partial_kernel(DecodeProblem p, float* part) {
   __shared__ float e_s[kChunk];
   __shared__ float red[kWarps];
@@ -58,31 +107,61 @@ __global__ void __launch_bounds__(kWarps * 32) partial_kernel(DecodeProblem p, f
   const int c0 = chunk * kChunk;
   const int n = max(0, min(kChunk, hist - c0));
   const TI* qv = reinterpret_cast<const TI*>(p.q) + (long long)b * p.qsB + (long long)h * p.qsH;
-  const TI* kc = reinterpret_cast<const TI*>(p.k) + (long long)b * p.sB + (long long)h * p.sH;
-  const TI* vc = reinterpret_cast<const TI*>(p.v) + (long long)b * p.sB + (long long)h * p.sH;
-  constexpr int PL = kMaxD / 32;  // columns per lane (at most)
-  float qr[PL];
-#pragma unroll
-  for (int e = 0; e < PL; ++e) {
-    const int c = lane + 32 * e;
-    qr[e] = c < p.d ? ldf<TI>(qv + c) : 0.f;
-  }
-  // E_j for the chunk's rows, and the running maximum
+  const TI* kc = reinterpret_cast<const TI*>(p.k) + (long long)b * p.sB + (long long)h * p.sH +
+                 (long long)c0 * p.sT;
+  const TI* vc = reinterpret_cast<const TI*>(p.v) + (long long)b * p.sB + (long long)h * p.sH +
+                 (long long)c0 * p.sT;
+  constexpr int PL = D > 0 ? D / 32 : kMaxD / 32;  // columns per lane in the P V pass
   float mx = -INFINITY;
-  for (int jj = warp; jj < n; jj += kWarps) {
-    const TI* kr = kc + (long long)(c0 + jj) * p.sT;
-    float s = 0.f;
+  if constexpr (D > 0) {
+    // scores: lane = 4 key + quarter; keys jj = 8 (warp + kWarps it) + lane / 4
+    constexpr int QD = D / 4;
+    const int sub = lane & 3, slot = lane >> 2;
+    float qr[QD];
+    ld_vec<TI, QD>(qv + sub * QD, qr);
+    for (int base = warp * 8; base < n; base += 8 * kWarps) {
+      const int jj = base + slot;
+      float kr[QD];
+      if (jj < n) ld_vec<TI, QD>(kc + (long long)jj * p.sT + sub * QD, kr);
+      else
+#pragma unroll
+        for (int e = 0; e < QD; ++e) kr[e] = 0.f;
+      float s = 0.f;
+#pragma unroll
+      for (int e = 0; e < QD; ++e) s = fmaf(qr[e], kr[e], s);
+      s += __shfl_xor_sync(0xffffffffu, s, 1);
+      s += __shfl_xor_sync(0xffffffffu, s, 2);
+      if (jj < n) {
+        const float u = s * p.inv_sqrt_d;
+        const float E = u / (1.0f + expf(-u));  // SiLU(u)
+        if (sub == 0) e_s[jj] = E;
+        mx = fmaxf(mx, E);
+      }
+    }
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, o));
+  } else {
+    float qr[PL];
 #pragma unroll
     for (int e = 0; e < PL; ++e) {
       const int c = lane + 32 * e;
-      if (c < p.d) s = fmaf(qr[e], ldf<TI>(kr + c), s);
+      qr[e] = c < p.d ? ldf<TI>(qv + c) : 0.f;
     }
+    for (int jj = warp; jj < n; jj += kWarps) {
+      const TI* kr = kc + (long long)jj * p.sT;
+      float s = 0.f;
 #pragma unroll
-    for (int o = 16; o > 0; o >>= 1) s += __shfl_xor_sync(0xffffffffu, s, o);
-    const float u = s * p.inv_sqrt_d;
-    const float E = u / (1.0f + expf(-u));  // SiLU(u)
-    if (lane == 0) e_s[jj] = E;
-    mx = fmaxf(mx, E);
+      for (int e = 0; e < PL; ++e) {
+        const int c = lane + 32 * e;
+        if (c < p.d) s = fmaf(qr[e], ldf<TI>(kr + c), s);
+      }
+#pragma unroll
+      for (int o = 16; o > 0; o >>= 1) s += __shfl_xor_sync(0xffffffffu, s, o);
+      const float u = s * p.inv_sqrt_d;
+      const float E = u / (1.0f + expf(-u));  // SiLU(u)
+      if (lane == 0) e_s[jj] = E;
+      mx = fmaxf(mx, E);
+    }
   }
   if (lane == 0) red[warp] = mx;
   __syncthreads();
@@ -94,20 +173,32 @@ __global__ void __launch_bounds__(kWarps * 32) partial_kernel(DecodeProblem p, f
   float l = 0.f, z[PL];
 #pragma unroll
   for (int e = 0; e < PL; ++e) z[e] = 0.f;
-  for (int jj = warp; jj < n; jj += kWarps) {
-    const float P = expf(e_s[jj] - m);
-    l += P;
-    const TI* vr = vc + (long long)(c0 + jj) * p.sT;
+  if constexpr (D > 0) {
+    const int col = lane * PL;
+#pragma unroll 4
+    for (int jj = warp; jj < n; jj += kWarps) {
+      const float P = expf(e_s[jj] - m);
+      l += P;
+      float vr[PL];
+      ld_vec<TI, PL>(vc + (long long)jj * p.sT + col, vr);
 #pragma unroll
-    for (int e = 0; e < PL; ++e) {
-      const int c = lane + 32 * e;
-      if (c < p.d) z[e] = fmaf(P, ldf<TI>(vr + c), z[e]);
+      for (int e = 0; e < PL; ++e) z[e] = fmaf(P, vr[e], z[e]);
     }
-  }
 #pragma unroll
-  for (int e = 0; e < PL; ++e) {
-    const int c = lane + 32 * e;
-    if (c < kMaxD) zs[warp][c] = z[e];
+    for (int e = 0; e < PL; ++e) zs[warp][col + e] = z[e];
+  } else {
+    for (int jj = warp; jj < n; jj += kWarps) {
+      const float P = expf(e_s[jj] - m);
+      l += P;
+      const TI* vr = vc + (long long)jj * p.sT;
+#pragma unroll
+      for (int e = 0; e < PL; ++e) {
+        const int c = lane + 32 * e;
+        if (c < p.d) z[e] = fmaf(P, ldf<TI>(vr + c), z[e]);
+      }
+    }
+#pragma unroll
+    for (int e = 0; e < PL; ++e) zs[warp][lane + 32 * e] = z[e];
   }
   if (lane == 0) red[warp] = l;
   __syncthreads();
@@ -186,7 +277,20 @@ __global__ void __launch_bounds__(kMaxD) combine_kernel(DecodeProblem p, const f
 
 template <typename TI>
 cudaError_t launch_t(const DecodeProblem& p, float* part, int n_chunks, cudaStream_t s) {
-  partial_kernel<TI><<<dim3((unsigned)(p.B * p.H), (unsigned)n_chunks), kWarps * 32, 0, s>>>(p, part);
+  const dim3 grid((unsigned)(p.B * p.H), (unsigned)n_chunks);
+  // vector loads need 16-byte aligned rows (strides are multiples of 16 bytes) and q
+  const bool qal = (reinterpret_cast<uintptr_t>(p.q) & 15u) == 0 &&
+                   (p.qsB * (long long)sizeof(TI)) % 16 == 0 &&
+                   (p.qsH * (long long)sizeof(TI)) % 16 == 0;
+  const bool kal = (p.sB * (long long)sizeof(TI)) % 16 == 0 &&
+                   (p.sT * (long long)sizeof(TI)) % 16 == 0 &&
+                   (p.sH * (long long)sizeof(TI)) % 16 == 0;
+  if (qal && kal && p.d == 128)
+    partial_kernel<TI, 128><<<grid, kWarps * 32, 0, s>>>(p, part);
+  else if (qal && kal && p.d == 64)
+    partial_kernel<TI, 64><<<grid, kWarps * 32, 0, s>>>(p, part);
+  else
+    partial_kernel<TI, 0><<<grid, kWarps * 32, 0, s>>>(p, part);
   cudaError_t e = cudaGetLastError();
   if (e != cudaSuccess) { note_failure("decode: partial pass launch"); return e; }
   combine_kernel<TI><<<(unsigned)(p.B * p.H), kMaxD, 0, s>>>(p, part, n_chunks);
