@@ -7,8 +7,10 @@ it, and it uses nothing from the CUDA library: the two share no code.
 The arithmetic lives in ``relation_oracle.c`` (plain C, fp64), which follows the
 paper's definitions: Eq. (causal-relation) and Eq. (relation-flow) for the
 materialised forward, App. A.1.2-A.1.8 for the factorised form, App. A.3 for the
-tiled Exchange scan and App. A.1.7 for the two backward derivations.  This module
-only marshals numpy arrays.
+tiled Exchange scan and App. A.1.7 for the two backward derivations.
+``linear_oracle.c`` (plain C, fp64) holds Linear Relation (Sec. 5.2, App. A.4): the
+recurrent step, its unrolled form and the reverse-mode backward of the recurrence.
+This module only marshals numpy arrays.
 
 ``Oracle(path)`` binds one compiled copy of the C file; the module-level functions
 use the default copy built from ``relation_oracle.c`` by :func:`build`.
@@ -26,6 +28,9 @@ _HERE = os.path.dirname(os.path.abspath(__file__))
 SOURCE = os.path.join(_HERE, "relation_oracle.c")
 _BUILD = os.path.join(_HERE, "_build")
 _LIB_PATH = os.path.join(_BUILD, "liboracle.so")
+LINEAR_SOURCE = os.path.join(_HERE, "linear_oracle.c")
+_LINEAR_LIB_PATH = os.path.join(_BUILD, "liblinear_oracle.so")
+_linear = None
 _lock = threading.Lock()
 _default = None
 
@@ -45,11 +50,13 @@ def compile_source(src: str, out: str) -> str:
 
 
 def build(force: bool = False) -> str:
-    """Compile relation_oracle.c into oracle/_build/liboracle.so (gcc, -fopenmp)."""
-    if (not force and os.path.exists(_LIB_PATH)
-            and os.path.getmtime(_LIB_PATH) >= os.path.getmtime(SOURCE)):
-        return _LIB_PATH
-    return compile_source(SOURCE, _LIB_PATH)
+    """Compile relation_oracle.c into oracle/_build/liboracle.so and linear_oracle.c into
+    oracle/_build/liblinear_oracle.so (gcc, -fopenmp); returns the first."""
+    for src, out in ((SOURCE, _LIB_PATH), (LINEAR_SOURCE, _LINEAR_LIB_PATH)):
+        if (force or not os.path.exists(out)
+                or os.path.getmtime(out) < os.path.getmtime(src)):
+            compile_source(src, out)
+    return _LIB_PATH
 
 
 def _in(a) -> np.ndarray:
@@ -257,3 +264,82 @@ def mhr_bwd(*a, **kw):
 
 def max_threads() -> int:
     return default().max_threads()
+
+
+# --- Linear Relation (linear_oracle.c) ---------------------------------------------
+
+class LinearOracle:
+    """One loaded copy of the compiled Linear Relation oracle (one head per call,
+    [T, d] arrays: p1, p2 after RoPE, information v, retention alpha in (0, 1])."""
+
+    def __init__(self, path: str):
+        lib = ctypes.CDLL(path)
+        i, d = ctypes.c_int, ctypes.c_double
+        sig = {
+            "rel_linear_fwd": [i, i, _dp, _dp, _dp, _dp, d, _dp, _dp, _dp],
+            "rel_linear_fwd_unrolled": [i, i, _dp, _dp, _dp, _dp, d, _dp],
+            "rel_linear_bwd": [i, i, _dp, _dp, _dp, _dp, _dp, d, _dp, _dp, _dp, _dp],
+        }
+        for name, args in sig.items():
+            fn = getattr(lib, name)
+            fn.argtypes = args
+            fn.restype = ctypes.c_int
+        self.lib = lib
+
+    @staticmethod
+    def _args(p1, p2, v, alpha):
+        p1, p2, v, alpha = _in(p1), _in(p2), _in(v), _in(alpha)
+        if p1.ndim != 2 or not (p1.shape == p2.shape == v.shape == alpha.shape):
+            raise ValueError("one head: p1, p2, v, alpha must all be [T, d]")
+        return p1, p2, v, alpha, p1.shape[0], p1.shape[1]
+
+    def fwd(self, p1, p2, v, alpha, tau_s: float = TAU_S, want_states: bool = False):
+        """Recurrent forward (App. A.4.2).  Returns (Y [T, d], S [T]) or, with
+        ``want_states``, (Y, S, C [T + 1, d, d]) with C[0] = 0."""
+        p1, p2, v, alpha, T, d = self._args(p1, p2, v, alpha)
+        y = np.empty((T, d)); S = np.empty(T)
+        C = np.empty((T + 1, d, d)) if want_states else None
+        _check(self.lib.rel_linear_fwd(T, d, _p(p1), _p(p2), _p(v), _p(alpha), tau_s, _p(y),
+                                       _p(S), _p(C)), "linear_fwd")
+        return (y, S, C) if want_states else (y, S)
+
+    def fwd_unrolled(self, p1, p2, v, alpha, tau_s: float = TAU_S):
+        """Unrolled forward (App. A.4.4-A.4.5), for tiny T.  Returns Y [T, d]."""
+        p1, p2, v, alpha, T, d = self._args(p1, p2, v, alpha)
+        y = np.empty((T, d))
+        _check(self.lib.rel_linear_fwd_unrolled(T, d, _p(p1), _p(p2), _p(v), _p(alpha), tau_s,
+                                                _p(y)), "linear_fwd_unrolled")
+        return y
+
+    def bwd(self, p1, p2, v, alpha, dy, tau_s: float = TAU_S):
+        """Reverse-mode backward of the recurrence.  Returns (dp1, dp2, dv, dalpha)."""
+        p1, p2, v, alpha, T, d = self._args(p1, p2, v, alpha)
+        dy = _in(dy)
+        if dy.shape != (T, d):
+            raise ValueError("dy must be [T, d]")
+        out = [np.empty((T, d)) for _ in range(4)]
+        _check(self.lib.rel_linear_bwd(T, d, _p(p1), _p(p2), _p(v), _p(alpha), _p(dy), tau_s,
+                                       *(_p(o) for o in out)), "linear_bwd")
+        return tuple(out)
+
+
+def linear() -> LinearOracle:
+    """The Linear Relation oracle compiled from linear_oracle.c (built on first use)."""
+    global _linear
+    with _lock:
+        if _linear is None:
+            build()
+            _linear = LinearOracle(_LINEAR_LIB_PATH)
+        return _linear
+
+
+def linear_fwd(*a, **kw):
+    return linear().fwd(*a, **kw)
+
+
+def linear_fwd_unrolled(*a, **kw):
+    return linear().fwd_unrolled(*a, **kw)
+
+
+def linear_bwd(*a, **kw):
+    return linear().bwd(*a, **kw)
