@@ -112,6 +112,25 @@ relation_status relation_fwd_flow(const void* q, const void* k, const void* v, v
                                   int* dev_status, relation_stream_t stream);
 
 /*
+ * Linear Relation forward (Sec. 5.2, Eq. (decayed-relation-state); App. A.4): the
+ * recurrent Exchange form, per head with the d_h x d_h state C_0 = 0,
+ *   S_t = sigmoid(p1_t . p2_t / (tau_S sqrt d_h)),  ^p = p / |p|
+ *   C^- = Diag(alpha_t) C_{t-1},  E_t = S_t (C^-)^T ^p1_t,  Y_t = I~_t + E_t,
+ *   C_t = C^- + S_t ^p2_t I~_t^T.
+ *   p1, p2, v : [B][T][H][d_h] relation coordinates (after RoPE) and information, in dt.
+ *   alpha     : [B][T][H][d_h] fp32 channel-wise retention in (0, 1] (the KDA-style
+ *               parameterisation of Eq. (retention-vector) is upstream), with the same
+ *               element strides as p1.
+ *   y         : [B][T][H][d_h] output in dt, same strides.
+ * fp32 or bf16 with d_h in {32, 64} (other widths: RELATION_ERR_UNSUPPORTED); the state is
+ * kept in fp32.  A zero p1 or p2 row is outside the operator's domain.  Asynchronous on
+ * `stream`; nothing is allocated.
+ */
+relation_status relation_linear_fwd(const void* p1, const void* p2, const void* v,
+                                   const float* alpha, void* y, float tau_s, relation_shape shp,
+                                   relation_dtype dt, int* dev_status, relation_stream_t stream);
+
+/*
  * Decoding: the forward row of one new token per sequence, against a key/value cache.
  *   q        [B][H][d_h] queries of the new tokens, element strides q_sB, q_sH (d_h
  *            contiguous); o (output Y) has the same layout.

@@ -95,6 +95,28 @@ struct DecodeProblem {
   long long sB, sT, sH, qsB, qsH;
   relation_dtype dtype;
 };
+// Linear Relation (relation_linear.cu).
+struct LinearProblem {
+  const void* p1;       // [B][T][H][d] relation coordinates after RoPE (strides sB, sT, sH)
+  const void* p2;
+  const void* v;        // information I~
+  const float* alpha;   // retention in (0, 1], fp32, same shape and element strides
+  void* y;              // forward output
+  const void* dy;       // backward input dL/dY
+  void* dp1;            // backward outputs (input dtype), dalpha fp32
+  void* dp2;
+  void* dv;
+  float* dalpha;
+  void* workspace;      // backward scratch
+  int* dev_status;
+  float tau_s;
+  int B, T, H, d;
+  long long sB, sT, sH;
+  relation_dtype dtype;
+};
+bool linear_supports(relation_dtype dt, int d);
+cudaError_t launch_linear_fwd(const LinearProblem& p, cudaStream_t s);
+
 int decode_chunks(int t_max);
 size_t decode_workspace_bytes(int B, int H, int t_max);
 cudaError_t launch_decode(const DecodeProblem& p, void* workspace, cudaStream_t s);

@@ -119,6 +119,25 @@ relation_status relation_fwd(const void* q, const void* k, const void* v, void* 
                          dev_status, stream);
 }
 
+relation_status relation_linear_fwd(const void* p1, const void* p2, const void* v,
+                                   const float* alpha, void* y, float tau_s, relation_shape shp,
+                                   relation_dtype dt, int* dev_status, relation_stream_t stream) {
+  relation_status st;
+  if (dt != RELATION_F32 && dt != RELATION_BF16) return RELATION_ERR_INVALID_ARG;
+  if (shp.B < 1 || shp.T < 1 || shp.H < 1 || shp.d_h < 1) return RELATION_ERR_INVALID_ARG;
+  if (shp.sB < 1 || shp.sT < 1 || shp.sH < 1) return RELATION_ERR_INVALID_ARG;
+  if (!rel::linear_supports(dt, shp.d_h)) return RELATION_ERR_UNSUPPORTED;
+  if ((long long)shp.B * shp.H > 0x7fffffffLL) return RELATION_ERR_UNSUPPORTED;
+  if (!isfinite(tau_s) || !(tau_s > 0.0f)) return RELATION_ERR_INVALID_ARG;
+  if ((st = check_ptrs({p1, p2, v, alpha, y})) != RELATION_OK) return st;
+  if (dev_status && (reinterpret_cast<uintptr_t>(dev_status) & 3u)) return RELATION_ERR_ALIGNMENT;
+  rel::LinearProblem p{};
+  p.p1 = p1; p.p2 = p2; p.v = v; p.alpha = alpha; p.y = y; p.dev_status = dev_status;
+  p.tau_s = tau_s; p.B = shp.B; p.T = shp.T; p.H = shp.H; p.d = shp.d_h;
+  p.sB = shp.sB; p.sT = shp.sT; p.sH = shp.sH; p.dtype = dt;
+  return from_cuda(rel::launch_linear_fwd(p, reinterpret_cast<cudaStream_t>(stream)));
+}
+
 size_t relation_decode_workspace_size(relation_shape cache, relation_dtype dt) {
   if (dt != RELATION_F32 && dt != RELATION_BF16) return 0;
   if (cache.B < 1 || cache.T < 1 || cache.H < 1 || cache.d_h < 1 || cache.d_h > 128) return 0;

@@ -83,6 +83,25 @@ def custom(B: int, H: int, T: int, d: int, dtype: str = "bf16", qk_std: float = 
     return Workload(f"custom_{B}x{H}x{T}x{d}_{dtype}", B, H, T, d, dtype, qk_std, v_std)
 
 
+def make_linear_inputs(w: Workload, seed: int = 0):
+    """Linear Relation inputs on the CPU: p1, p2, v [B, T, H, d] of the workload's dtype
+    (p1, p2 ~ N(0, qk_std^2), v ~ N(0, v_std^2)), the retention alpha [B, T, H, d] fp32 and
+    dY ~ N(0, 1).  alpha follows a KDA-style draw, alpha = exp(-A softplus(z - 4)) with a
+    per-(head, channel) rate A ~ U(1, 16) and z ~ N(0, 1) per token, which puts most
+    channels between 0.75 and 0.99."""
+    g = torch.Generator().manual_seed(seed + 7919)
+    shape = (w.B, w.T, w.H, w.d)
+    dt = torch.float32 if w.dtype == "fp32" else torch.bfloat16
+    p1 = (torch.randn(shape, generator=g) * w.qk_std).to(dt)
+    p2 = (torch.randn(shape, generator=g) * w.qk_std).to(dt)
+    v = (torch.randn(shape, generator=g) * w.v_std).to(dt)
+    A = torch.rand((1, 1, w.H, w.d), generator=g) * 15.0 + 1.0
+    z = torch.randn(shape, generator=g)
+    alpha = torch.exp(-A * torch.nn.functional.softplus(z - 4.0)).float()
+    dy = torch.randn(shape, generator=g).to(dt)
+    return p1, p2, v, alpha, dy
+
+
 def make_inputs(w: Workload, seed: int = 0, with_grad_out: bool = True):
     """Draw (q, k, v, dout) on the CPU as [B, T, H, d] tensors of the workload's dtype.
 

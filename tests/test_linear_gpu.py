@@ -1,0 +1,55 @@
+"""GPU parity of Linear Relation (Sec. 5.2, App. A.4) against the fp64 oracle, every head
+element by element, at sizes that span several staged chunks and a ragged tail."""
+import numpy as np
+import pytest
+import torch
+
+import oracle
+from paper_2608_20172_gb300 import binding, workloads
+from tests import parity_util as pu
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _lib():
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    binding.load()
+
+
+def _heads(x, b, h):
+    return x[b, :, h].double().numpy()
+
+
+@pytest.mark.parametrize("dtype", ["fp32", "bf16"])
+@pytest.mark.parametrize("d", [32, 64])
+@pytest.mark.parametrize("T", [1, 17, 200])
+def test_linear_forward(dtype, d, T):
+    w = workloads.custom(2, 2, T, d, dtype)
+    p1, p2, v, alpha, _ = workloads.make_linear_inputs(w, seed=T + d)
+    dev = torch.device("cuda:0")
+    status = torch.zeros(1, dtype=torch.int32, device=dev)
+    y = binding.linear_fwd(p1.to(dev), p2.to(dev), v.to(dev), alpha.to(dev), dev_status=status)
+    torch.cuda.synchronize()
+    assert int(status.item()) == 0
+    y = y.float().cpu().numpy()
+    for b in range(w.B):
+        for h in range(w.H):
+            ref, _ = oracle.linear_fwd(_heads(p1, b, h), _heads(p2, b, h), _heads(v, b, h),
+                                       _heads(alpha, b, h))
+            pu.check(f"linear Y ({b},{h})", y[b, :, h], ref, dtype, "out")
+
+
+def test_linear_bhtd_layout():
+    """[B, H, T, d] storage (a permuted view) gives the same output as [B, T, H, d]."""
+    w = workloads.custom(2, 3, 70, 64, "bf16")
+    p1, p2, v, alpha, _ = workloads.make_linear_inputs(w, seed=1)
+    dev = torch.device("cuda:0")
+
+    def bhtd(t):
+        return t.permute(0, 2, 1, 3).contiguous().to(dev).permute(0, 2, 1, 3)
+
+    y0 = binding.linear_fwd(*(t.to(dev) for t in (p1, p2, v, alpha)))
+    y1 = binding.linear_fwd(*(bhtd(t) for t in (p1, p2, v, alpha)))
+    assert torch.equal(y0.cpu(), y1.cpu())
