@@ -131,6 +131,22 @@ relation_status relation_linear_fwd(const void* p1, const void* p2, const void* 
                                    relation_dtype dt, int* dev_status, relation_stream_t stream);
 
 /*
+ * Linear Relation backward: the reverse-mode derivative of the recurrence above (the paper
+ * writes out the forward only), given dy = dL/dY:
+ *   dp1, dp2, dv : [B][T][H][d_h] in dt, with the inputs' strides (overwritten);
+ *   dalpha       : [B][T][H][d_h] fp32 with alpha's strides (overwritten);
+ *   workspace    : device scratch of relation_linear_bwd_workspace_size(shp, dt) bytes
+ *                  (state checkpoints every 8 tokens plus two fp32 [B][H][T][d_h] arrays).
+ * Same dtypes and widths as relation_linear_fwd; asynchronous on `stream`.
+ */
+size_t relation_linear_bwd_workspace_size(relation_shape shp, relation_dtype dt);
+relation_status relation_linear_bwd(const void* p1, const void* p2, const void* v,
+                                   const float* alpha, const void* dy, void* dp1, void* dp2,
+                                   void* dv, float* dalpha, float tau_s, relation_shape shp,
+                                   relation_dtype dt, void* workspace, size_t ws_bytes,
+                                   int* dev_status, relation_stream_t stream);
+
+/*
  * Decoding: the forward row of one new token per sequence, against a key/value cache.
  *   q        [B][H][d_h] queries of the new tokens, element strides q_sB, q_sH (d_h
  *            contiguous); o (output Y) has the same layout.

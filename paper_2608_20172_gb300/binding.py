@@ -30,7 +30,8 @@ EXPORTED = ("relation_fwd", "relation_fwd_ex", "relation_bwd", "relation_bwd_ex"
             "relation_bwd_workspace_size", "relation_status_string", "relation_version",
             "relation_selftest_wait_timeout", "relation_launch_count", "relation_last_cuda_error",
             "relation_bwd_stages", "relation_bwd_static", "relation_fwd_flow",
-            "relation_decode", "relation_decode_workspace_size", "relation_linear_fwd")
+            "relation_decode", "relation_decode_workspace_size", "relation_linear_fwd",
+            "relation_linear_bwd", "relation_linear_bwd_workspace_size")
 
 
 class RelationLibraryMissing(RuntimeError):
@@ -77,6 +78,10 @@ def load(path: str | None = None):
                                         ctypes.c_size_t, ip, vp]
         lib.relation_decode_workspace_size.argtypes = [Shape, i]
         lib.relation_linear_fwd.argtypes = [vp, vp, vp, vp, vp, f, Shape, i, ip, vp]
+        lib.relation_linear_bwd.argtypes = [vp, vp, vp, vp, vp, vp, vp, vp, vp, f, Shape, i, vp,
+                                            ctypes.c_size_t, ip, vp]
+        lib.relation_linear_bwd_workspace_size.argtypes = [Shape, i]
+        lib.relation_linear_bwd_workspace_size.restype = ctypes.c_size_t
         lib.relation_decode_workspace_size.restype = ctypes.c_size_t
         lib.relation_bwd.argtypes = [vp, vp, vp, vp, vp, vp, vp, vp, vp, vp, f, f, Shape, i, vp,
                                      sz, ip, vp]
@@ -204,6 +209,28 @@ def linear_fwd(p1, p2, v, alpha, tau_s: float = 2.0, *, out=None, dev_status=Non
     if rc != OK:
         raise RelationError(rc, "relation_linear_fwd")
     return out
+
+
+def linear_bwd(p1, p2, v, alpha, dy, tau_s: float = 2.0, *, workspace=None, dev_status=None,
+               stream=None):
+    """Linear Relation backward.  Returns (dp1, dp2, dv, dalpha) with dalpha fp32."""
+    _same_layout(p1, p2, v, dy)
+    if alpha.dtype != torch.float32 or tuple(alpha.shape) != tuple(p1.shape) or \
+            tuple(alpha.stride()) != tuple(p1.stride()):
+        raise ValueError("alpha must be fp32 with p1's shape and strides")
+    dp1, dp2, dv = torch.empty_like(p1), torch.empty_like(p1), torch.empty_like(p1)
+    dalpha = torch.empty_like(alpha)
+    need = int(load().relation_linear_bwd_workspace_size(shape_of(p1), _dtype_code(p1)))
+    if workspace is None:
+        workspace = torch.empty(max(need, 16), device=p1.device, dtype=torch.uint8)
+    rc = load().relation_linear_bwd(_ptr(p1), _ptr(p2), _ptr(v), _ptr(alpha), _ptr(dy),
+                                    _ptr(dp1), _ptr(dp2), _ptr(dv), _ptr(dalpha), float(tau_s),
+                                    shape_of(p1), _dtype_code(p1), _ptr(workspace),
+                                    workspace.numel() * workspace.element_size(),
+                                    _ptr(dev_status), ctypes.c_void_p(_stream(stream)))
+    if rc != OK:
+        raise RelationError(rc, "relation_linear_bwd")
+    return dp1, dp2, dv, dalpha
 
 
 def decode_workspace_size(k_cache) -> int:

@@ -116,6 +116,8 @@ struct LinearProblem {
 };
 bool linear_supports(relation_dtype dt, int d);
 cudaError_t launch_linear_fwd(const LinearProblem& p, cudaStream_t s);
+size_t linear_bwd_workspace_bytes(int B, int H, int T, int d);
+cudaError_t launch_linear_bwd(const LinearProblem& p, cudaStream_t s);
 
 int decode_chunks(int t_max);
 size_t decode_workspace_bytes(int B, int H, int t_max);

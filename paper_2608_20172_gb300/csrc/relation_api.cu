@@ -138,6 +138,38 @@ relation_status relation_linear_fwd(const void* p1, const void* p2, const void* 
   return from_cuda(rel::launch_linear_fwd(p, reinterpret_cast<cudaStream_t>(stream)));
 }
 
+size_t relation_linear_bwd_workspace_size(relation_shape shp, relation_dtype dt) {
+  if (dt != RELATION_F32 && dt != RELATION_BF16) return 0;
+  if (shp.B < 1 || shp.T < 1 || shp.H < 1 || !rel::linear_supports(dt, shp.d_h)) return 0;
+  return rel::linear_bwd_workspace_bytes(shp.B, shp.H, shp.T, shp.d_h);
+}
+
+relation_status relation_linear_bwd(const void* p1, const void* p2, const void* v,
+                                   const float* alpha, const void* dy, void* dp1, void* dp2,
+                                   void* dv, float* dalpha, float tau_s, relation_shape shp,
+                                   relation_dtype dt, void* workspace, size_t ws_bytes,
+                                   int* dev_status, relation_stream_t stream) {
+  relation_status st;
+  if (dt != RELATION_F32 && dt != RELATION_BF16) return RELATION_ERR_INVALID_ARG;
+  if (shp.B < 1 || shp.T < 1 || shp.H < 1 || shp.d_h < 1) return RELATION_ERR_INVALID_ARG;
+  if (shp.sB < 1 || shp.sT < 1 || shp.sH < 1) return RELATION_ERR_INVALID_ARG;
+  if (!rel::linear_supports(dt, shp.d_h)) return RELATION_ERR_UNSUPPORTED;
+  if ((long long)shp.B * shp.H > 0x7fffffffLL) return RELATION_ERR_UNSUPPORTED;
+  if (!isfinite(tau_s) || !(tau_s > 0.0f)) return RELATION_ERR_INVALID_ARG;
+  if ((st = check_ptrs({p1, p2, v, alpha, dy, dp1, dp2, dv, dalpha, workspace})) != RELATION_OK)
+    return st;
+  if (dev_status && (reinterpret_cast<uintptr_t>(dev_status) & 3u)) return RELATION_ERR_ALIGNMENT;
+  if (ws_bytes < rel::linear_bwd_workspace_bytes(shp.B, shp.H, shp.T, shp.d_h))
+    return RELATION_ERR_WORKSPACE;
+  rel::LinearProblem p{};
+  p.p1 = p1; p.p2 = p2; p.v = v; p.alpha = alpha; p.dy = dy;
+  p.dp1 = dp1; p.dp2 = dp2; p.dv = dv; p.dalpha = dalpha; p.workspace = workspace;
+  p.dev_status = dev_status; p.tau_s = tau_s;
+  p.B = shp.B; p.T = shp.T; p.H = shp.H; p.d = shp.d_h;
+  p.sB = shp.sB; p.sT = shp.sT; p.sH = shp.sH; p.dtype = dt;
+  return from_cuda(rel::launch_linear_bwd(p, reinterpret_cast<cudaStream_t>(stream)));
+}
+
 size_t relation_decode_workspace_size(relation_shape cache, relation_dtype dt) {
   if (dt != RELATION_F32 && dt != RELATION_BF16) return 0;
   if (cache.B < 1 || cache.T < 1 || cache.H < 1 || cache.d_h < 1 || cache.d_h > 128) return 0;

@@ -16,6 +16,8 @@
 // order; tokens are staged through shared memory in chunks of kChunkT, double-buffered,
 // with S_t, 1/|p1_t|, 1/|p2_t| computed per chunk (S is folded into the coordinates:
 // q'_t = S_t ^p1_t, k'_t = S_t ^p2_t).
+// The backward (below) walks the tokens in reverse with the adjoint state, recomputing
+// the states of each chunk of kChunkB tokens from checkpoints the kernel stores first.
 #include <math.h>
 
 #include "common.cuh"
@@ -43,25 +45,26 @@ __device__ __forceinline__ void stx<__nv_bfloat16>(__nv_bfloat16* p, float v) {
   *p = __float2bfloat16_rn(v);
 }
 
-// Shared staging of one chunk: per token the four vectors alpha, q', k', I~ (fp32).
-template <int D>
+// Shared staging of one chunk of NTOK tokens: per token the four vectors alpha, q', k',
+// I~ (fp32).
+template <int D, int NTOK = kChunkT>
 struct Chunk {
-  float vec[kChunkT][4][D];  // [0] alpha, [1] p1 -> q', [2] p2 -> k', [3] I~
-  float scal[kChunkT][4];    // S, 1/|p1|, 1/|p2|
+  float vec[NTOK][4][D];  // [0] alpha, [1] p1 -> q', [2] p2 -> k', [3] I~
+  float scal[NTOK][4];    // S, 1/|p1|, 1/|p2|
 };
 
 // Raw loads of chunk `ch` (tokens ch * kChunkT ...) into registers: element e of the
 // chunk's 4 * kChunkT * D values goes to thread e % NT, slot e / NT.
-template <typename TI, int D, int NT>
+template <typename TI, int D, int NT, int NTOK = kChunkT>
 struct Loader {
-  static constexpr int N = 4 * kChunkT * D / NT;  // values per thread
+  static constexpr int N = 4 * NTOK * D / NT;  // values per thread
   float r[N];
   __device__ __forceinline__ void load(const LinearProblem& p, int b, int h, int ch) {
 #pragma unroll
     for (int n = 0; n < N; ++n) {
       const int e = n * NT + (int)threadIdx.x;
       const int c = e % D, a = (e / D) % 4, tt = e / (4 * D);
-      const int t = ch * kChunkT + tt;
+      const int t = ch * NTOK + tt;
       float x = 0.f;
       if (t < p.T) {
         const long long off = (long long)b * p.sB + (long long)t * p.sT + (long long)h * p.sH + c;
@@ -73,7 +76,7 @@ struct Loader {
       r[n] = x;
     }
   }
-  __device__ __forceinline__ void store(Chunk<D>& s) const {
+  __device__ __forceinline__ void store(Chunk<D, NTOK>& s) const {
 #pragma unroll
     for (int n = 0; n < N; ++n) {
       const int e = n * NT + (int)threadIdx.x;
@@ -84,11 +87,11 @@ struct Loader {
 
 // Ask Self for the chunk's tokens (one warp per token), then fold S into the unit
 // coordinates.  Two block barriers; the caller has made the raw values visible.
-template <int D, int NT>
-__device__ __forceinline__ void ask_self_chunk(Chunk<D>& s, float tau_s) {
+template <int D, int NT, int NTOK = kChunkT>
+__device__ __forceinline__ void ask_self_chunk(Chunk<D, NTOK>& s, float tau_s) {
   constexpr int NW = NT / 32;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  for (int tt = warp; tt < kChunkT; tt += NW) {
+  for (int tt = warp; tt < NTOK; tt += NW) {
     float s12 = 0.f, s11 = 0.f, s22 = 0.f;
     for (int c = lane; c < D; c += 32) {
       const float a = s.vec[tt][1][c], b = s.vec[tt][2][c];
@@ -109,7 +112,7 @@ __device__ __forceinline__ void ask_self_chunk(Chunk<D>& s, float tau_s) {
     }
   }
   __syncthreads();
-  for (int e = threadIdx.x; e < kChunkT * 2 * D; e += NT) {
+  for (int e = threadIdx.x; e < NTOK * 2 * D; e += NT) {
     const int c = e % D, a = 1 + (e / D) % 2, tt = e / (2 * D);
     s.vec[tt][a][c] *= s.scal[tt][0] * s.scal[tt][a];
   }
@@ -184,7 +187,246 @@ cudaError_t fwd_t(const LinearProblem& p, cudaStream_t s) {
   return e;
 }
 
+// ---------------------------------------------------------------------------------
+// Backward.  Reverse-mode derivative of the recurrent step, in reverse token order, with
+// the adjoint dC of the state (S folded into q' = S ^p1 and k' = S ^p2):
+//   dI~_t = dY_t + dC_t^T k'_t,   dk'_t = dC_t I~_t,   dq'_t = C^- dY_t,
+//   dC^- = dC_t + q'_t dY_t^T,   dalpha_t = rowsum(dC^- * C_{t-1}),   dC_{t-1} = Diag(alpha_t) dC^-
+// (C^- = Diag(alpha_t) C_{t-1}); a per-token pass then turns dq', dk' into dp1, dp2
+// through the normalisation and S.  Thread (c, half) owns row c of the state for half of
+// the columns, so the row sums (dk', dq', dalpha) are a pair shuffle and the column sum
+// (dI~) is reduced across rows by a shuffle reduce-scatter within each warp and shared
+// memory across warps.
+//   1. checkpoint pass: forward over the tokens, storing the state before every chunk of
+//      kChunkB tokens in the workspace;
+//   2. reverse sweep: per chunk (last first), the states before each of its tokens are
+//      recomputed from the checkpoint into shared memory, then the tokens are walked
+//      backwards;
+//   3. per-token pass: dp1, dp2.
+constexpr int kChunkB = 8;
+
+template <int D>
+struct BwdSmem {
+  Chunk<D, kChunkB> tok;                // alpha, q', k', I~ of the chunk
+  float g[kChunkB][D];                  // dY of the chunk
+  float red[kChunkB][2 * D / 32][D];    // per-warp column sums of dC^T k'
+  float st[kChunkB][D][D];              // C_{t-1} of each token of the chunk
+};
+
+template <int D>
+__host__ __device__ constexpr long long ckpt_floats(int T) {
+  return (long long)((T + kChunkB - 1) / kChunkB) * D * D;
+}
+
+template <typename TI, int D>
+__global__ void __launch_bounds__(2 * D) bwd_kernel(LinearProblem p) {
+  constexpr int NT = 2 * D, R = D / 2, NW = NT / 32;
+  extern __shared__ __align__(16) uint8_t smem_raw[];
+  BwdSmem<D>& sm = *reinterpret_cast<BwdSmem<D>*>(smem_raw);
+  const int bh = blockIdx.x, b = bh / p.H, h = bh % p.H;
+  const int c = threadIdx.x >> 1, hc = threadIdx.x & 1, j0 = hc * R;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int n_ch = (p.T + kChunkB - 1) / kChunkB;
+  float* ckpt = reinterpret_cast<float*>(p.workspace) + (long long)bh * ckpt_floats<D>(p.T);
+  float* dqk = reinterpret_cast<float*>(p.workspace) + (long long)p.B * p.H * ckpt_floats<D>(p.T) +
+               (long long)bh * p.T * 2 * D;  // [T][2][D]: dq', dk'
+  const long long hb = (long long)b * p.sB + (long long)h * p.sH;
+  Loader<TI, D, NT, kChunkB> ld;
+  auto stage = [&](int ch) {  // token data of chunk ch into sm.tok (and dY into sm.g)
+    __syncthreads();          // the previous chunk's data is no longer read
+    ld.load(p, b, h, ch);
+    ld.store(sm.tok);
+    for (int e = threadIdx.x; e < kChunkB * D; e += NT) {
+      const int tt = e / D, cc = e % D, t = ch * kChunkB + tt;
+      sm.g[tt][cc] = t < p.T ? ldx<TI>(reinterpret_cast<const TI*>(p.dy) + hb +
+                                       (long long)t * p.sT + cc)
+                             : 0.f;
+    }
+    __syncthreads();
+    ask_self_chunk<D, NT, kChunkB>(sm.tok, p.tau_s);
+  };
+  // 1. checkpoint pass: only the row update C <- Diag(alpha) C + k' I~^T is needed
+  float C[R];
+#pragma unroll
+  for (int i = 0; i < R; ++i) C[i] = 0.f;
+  for (int ch = 0; ch < n_ch; ++ch) {
+    float* ck = ckpt + (long long)ch * D * D + c * D + j0;
+#pragma unroll
+    for (int i = 0; i < R; i += 4)
+      *reinterpret_cast<float4*>(ck + i) = make_float4(C[i], C[i + 1], C[i + 2], C[i + 3]);
+    if (ch + 1 == n_ch) break;  // the last chunk's end state is not needed
+    stage(ch);
+    for (int tt = 0; tt < kChunkB; ++tt) {
+      const float a = sm.tok.vec[tt][0][c], kp = sm.tok.vec[tt][2][c];
+      const float* I = &sm.tok.vec[tt][3][j0];
+#pragma unroll
+      for (int i = 0; i < R; ++i) C[i] = fmaf(kp, I[i], a * C[i]);
+    }
+  }
+  // 2. reverse sweep
+  float dC[R];
+#pragma unroll
+  for (int i = 0; i < R; ++i) dC[i] = 0.f;
+  for (int ch = n_ch - 1; ch >= 0; --ch) {
+    stage(ch);
+    const int nt = min(kChunkB, p.T - ch * kChunkB);
+    const float* ck = ckpt + (long long)ch * D * D + c * D + j0;
+#pragma unroll
+    for (int i = 0; i < R; i += 4) {
+      const float4 x = *reinterpret_cast<const float4*>(ck + i);
+      C[i] = x.x; C[i + 1] = x.y; C[i + 2] = x.z; C[i + 3] = x.w;
+    }
+    for (int tt = 0; tt < nt; ++tt) {  // C_{t-1} of each token into shared memory
+      float* dst = &sm.st[tt][c][j0];
+#pragma unroll
+      for (int i = 0; i < R; i += 4)
+        *reinterpret_cast<float4*>(dst + i) = make_float4(C[i], C[i + 1], C[i + 2], C[i + 3]);
+      const float a = sm.tok.vec[tt][0][c], kp = sm.tok.vec[tt][2][c];
+      const float* I = &sm.tok.vec[tt][3][j0];
+#pragma unroll
+      for (int i = 0; i < R; ++i) C[i] = fmaf(kp, I[i], a * C[i]);
+    }
+    for (int tt = nt - 1; tt >= 0; --tt) {
+      const int t = ch * kChunkB + tt;
+      const float a = sm.tok.vec[tt][0][c], qp = sm.tok.vec[tt][1][c];
+      const float kp = sm.tok.vec[tt][2][c];
+      const float* I = &sm.tok.vec[tt][3][j0];
+      const float* G = &sm.g[tt][j0];
+      const float* Cp = &sm.st[tt][c][j0];
+      float dk = 0.f, dq = 0.f, da = 0.f, col[R];
+#pragma unroll
+      for (int i = 0; i < R; ++i) {
+        const float cp = Cp[i], g = G[i];
+        col[i] = dC[i] * kp;              // this row's share of dC^T k'
+        dk = fmaf(dC[i], I[i], dk);
+        dq = fmaf(a * cp, g, dq);
+        const float dcm = fmaf(qp, g, dC[i]);
+        da = fmaf(dcm, cp, da);
+        dC[i] = a * dcm;                   // dL/dC_{t-1}
+      }
+      dk += __shfl_xor_sync(0xffffffffu, dk, 1);
+      dq += __shfl_xor_sync(0xffffffffu, dq, 1);
+      da += __shfl_xor_sync(0xffffffffu, da, 1);
+      if (hc == 0) {
+        p.dalpha[hb + (long long)t * p.sT + c] = da;
+        dqk[(long long)t * 2 * D + c] = dq;
+        dqk[(long long)t * 2 * D + D + c] = dk;
+      }
+      // column sums over the warp's 16 rows: reduce-scatter over lane bits 1..4
+      int off = 0, n = R;
+#pragma unroll
+      for (int m = 16; m >= 2; m >>= 1) {
+        n >>= 1;
+        const bool up = (lane & m) != 0;
+#pragma unroll
+        for (int i = 0; i < R / 2; ++i) {
+          if (i < n) {
+            const float send = up ? col[i] : col[i + n];
+            const float keep = up ? col[i + n] : col[i];
+            col[i] = keep + __shfl_xor_sync(0xffffffffu, send, m);
+          }
+        }
+        off += up ? n : 0;
+      }
+#pragma unroll
+      for (int i = 0; i < R / 16; ++i) sm.red[tt][warp][j0 + off + i] = col[i];
+    }
+    __syncthreads();
+    for (int e = threadIdx.x; e < nt * D; e += NT) {  // dI~_t = dY_t + dC_t^T k'_t
+      const int tt = e / D, jj = e % D, t = ch * kChunkB + tt;
+      float s = sm.g[tt][jj];
+#pragma unroll
+      for (int w = 0; w < NW; ++w) s += sm.red[tt][w][jj];
+      stx<TI>(reinterpret_cast<TI*>(p.dv) + hb + (long long)t * p.sT + jj, s);
+    }
+  }
+}
+
+// dp1, dp2 of every token (one warp per token) from dq', dk' through q' = S p1 / |p1|,
+// k' = S p2 / |p2| and S = sigmoid(p1 . p2 / (tau_S sqrt d)).
+template <typename TI, int D>
+__global__ void __launch_bounds__(256) post_kernel(LinearProblem p) {
+  constexpr int PL = D / 32;
+  const long long tok = ((long long)blockIdx.x * 256 + threadIdx.x) >> 5;
+  const int lane = threadIdx.x & 31;
+  if (tok >= (long long)p.B * p.H * p.T) return;
+  const int bh = (int)(tok / p.T), t = (int)(tok % p.T), b = bh / p.H, h = bh % p.H;
+  const long long off = (long long)b * p.sB + (long long)h * p.sH + (long long)t * p.sT;
+  const float* dqk = reinterpret_cast<const float*>(p.workspace) +
+                     (long long)p.B * p.H * ckpt_floats<D>(p.T) + ((long long)bh * p.T + t) * 2 * D;
+  float x1[PL], x2[PL], g1[PL], g2[PL];
+  float s12 = 0.f, s11 = 0.f, s22 = 0.f;
+#pragma unroll
+  for (int e = 0; e < PL; ++e) {
+    const int cc = lane + 32 * e;
+    x1[e] = ldx<TI>(reinterpret_cast<const TI*>(p.p1) + off + cc);
+    x2[e] = ldx<TI>(reinterpret_cast<const TI*>(p.p2) + off + cc);
+    g1[e] = dqk[cc];
+    g2[e] = dqk[D + cc];
+    s12 = fmaf(x1[e], x2[e], s12);
+    s11 = fmaf(x1[e], x1[e], s11);
+    s22 = fmaf(x2[e], x2[e], s22);
+  }
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) {
+    s12 += __shfl_xor_sync(0xffffffffu, s12, o);
+    s11 += __shfl_xor_sync(0xffffffffu, s11, o);
+    s22 += __shfl_xor_sync(0xffffffffu, s22, o);
+  }
+  const float rsd = rsqrtf((float)D);
+  const float S = 1.0f / (1.0f + expf(-s12 * rsd / p.tau_s));
+  const float in1 = rsqrtf(s11), in2 = rsqrtf(s22);
+  // q' = S q^, k' = S k^:  dS = dq' . q^ + dk' . k^,  dq^ = S dq',  dk^ = S dk'
+  float a1 = 0.f, a2 = 0.f;  // q^ . dq', k^ . dk'
+#pragma unroll
+  for (int e = 0; e < PL; ++e) {
+    a1 = fmaf(x1[e] * in1, g1[e], a1);
+    a2 = fmaf(x2[e] * in2, g2[e], a2);
+  }
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) {
+    a1 += __shfl_xor_sync(0xffffffffu, a1, o);
+    a2 += __shfl_xor_sync(0xffffffffu, a2, o);
+  }
+  const float dS = a1 + a2;
+  const float du = dS * S * (1.0f - S) / p.tau_s * rsd;
+#pragma unroll
+  for (int e = 0; e < PL; ++e) {
+    const int cc = lane + 32 * e;
+    // d/dp of p / |p| applied to S dq':  S (dq' - q^ (q^ . dq')) / |p|
+    const float d1 = S * (g1[e] - x1[e] * in1 * a1) * in1 + du * x2[e];
+    const float d2 = S * (g2[e] - x2[e] * in2 * a2) * in2 + du * x1[e];
+    stx<TI>(reinterpret_cast<TI*>(p.dp1) + off + cc, d1);
+    stx<TI>(reinterpret_cast<TI*>(p.dp2) + off + cc, d2);
+  }
+}
+
+template <typename TI, int D>
+cudaError_t bwd_t(const LinearProblem& p, cudaStream_t s) {
+  const int smem = (int)sizeof(BwdSmem<D>);
+  cudaError_t e = cudaFuncSetAttribute(bwd_kernel<TI, D>,
+                                       cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+  if (e != cudaSuccess) { note_failure("linear backward: shared memory attribute"); return e; }
+  bwd_kernel<TI, D><<<(unsigned)(p.B * p.H), 2 * D, smem, s>>>(p);
+  if ((e = cudaGetLastError()) != cudaSuccess) { note_failure("linear backward: launch"); return e; }
+  const long long toks = (long long)p.B * p.H * p.T;
+  post_kernel<TI, D><<<(unsigned)((toks * 32 + 255) / 256), 256, 0, s>>>(p);
+  if ((e = cudaGetLastError()) != cudaSuccess) note_failure("linear backward: per-token pass");
+  return e;
+}
+
 }  // namespace lin
+
+size_t linear_bwd_workspace_bytes(int B, int H, int T, int d) {
+  const long long per = d == 32 ? lin::ckpt_floats<32>(T) : lin::ckpt_floats<64>(T);
+  return (size_t)((long long)B * H * per + (long long)B * H * T * 2 * d) * sizeof(float);
+}
+
+cudaError_t launch_linear_bwd(const LinearProblem& p, cudaStream_t s) {
+  if (p.dtype == RELATION_F32)
+    return p.d == 32 ? lin::bwd_t<float, 32>(p, s) : lin::bwd_t<float, 64>(p, s);
+  return p.d == 32 ? lin::bwd_t<__nv_bfloat16, 32>(p, s) : lin::bwd_t<__nv_bfloat16, 64>(p, s);
+}
 
 bool linear_supports(relation_dtype dt, int d) {
   return (dt == RELATION_F32 || dt == RELATION_BF16) && (d == 32 || d == 64);

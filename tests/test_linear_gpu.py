@@ -41,6 +41,29 @@ def test_linear_forward(dtype, d, T):
             pu.check(f"linear Y ({b},{h})", y[b, :, h], ref, dtype, "out")
 
 
+@pytest.mark.parametrize("dtype", ["fp32", "bf16"])
+@pytest.mark.parametrize("d", [32, 64])
+@pytest.mark.parametrize("T", [1, 8, 9, 100])
+def test_linear_backward(dtype, d, T):
+    """Gradients of every input, including the retention, against the oracle's reverse-
+    mode backward on every head (T spans whole 8-token chunks and ragged tails)."""
+    w = workloads.custom(2, 2, T, d, dtype)
+    p1, p2, v, alpha, dy = workloads.make_linear_inputs(w, seed=100 + T + d)
+    dev = torch.device("cuda:0")
+    status = torch.zeros(1, dtype=torch.int32, device=dev)
+    g = binding.linear_bwd(*(t.to(dev) for t in (p1, p2, v, alpha, dy)), dev_status=status)
+    torch.cuda.synchronize()
+    assert int(status.item()) == 0
+    g = [t.float().cpu().numpy() for t in g]
+    for b in range(w.B):
+        for h in range(w.H):
+            ref = oracle.linear_bwd(_heads(p1, b, h), _heads(p2, b, h), _heads(v, b, h),
+                                    _heads(alpha, b, h), _heads(dy, b, h))
+            for name, got, r in zip(("dp1", "dp2", "dv", "dalpha"), g, ref):
+                pu.check(f"linear {name} ({b},{h}) T={T}", got[b, :, h], r,
+                         "fp32" if name == "dalpha" and dtype == "fp32" else dtype, "grad")
+
+
 def test_linear_bhtd_layout():
     """[B, H, T, d] storage (a permuted view) gives the same output as [B, T, H, d]."""
     w = workloads.custom(2, 3, 70, 64, "bf16")
