@@ -275,6 +275,50 @@ def decode_measure(binding, dev, peaks, steps=20, warmup=3):
             "gpu_launches_per_call": 2}
 
 
+LINEAR_CFG = {"B": 8, "H": 12, "T": 2048, "d_h": 64}  # the 100M layer geometry, bf16
+FP32_FMA_TFLOPS = 152 * 128 * 2 * 2.07e9 / 1e12  # 152 SMs x 128 FFMA lanes x 2 flops x 2.07 GHz
+
+
+def linear_measure(binding, dev, steps=20, warmup=3):
+    """Linear Relation forward and backward on the 100M geometry (bf16, one CTA per head).
+    Arithmetic per token and head: forward 5 d^2 (decay, read, write); backward 16 d^2
+    (checkpoint pass 3, chunk recompute 3, reverse step 10).  ALU roofline against the
+    fp32 FMA peak of the SMs."""
+    c = LINEAR_CFG
+    w = workloads.custom(c["B"], c["H"], c["T"], c["d_h"], "bf16")
+    p1, p2, v, alpha, dy = (t.to(dev) for t in workloads.make_linear_inputs(w, seed=0))
+    out = torch.empty_like(p1)
+    status = torch.zeros(1, dtype=torch.int32, device=dev)
+    stream = torch.cuda.current_stream(dev)
+    need = int(binding.load().relation_linear_bwd_workspace_size(binding.shape_of(p1),
+                                                                  binding.BF16))
+    wsb = torch.empty(need, dtype=torch.uint8, device=dev)
+    fwd = lambda: binding.linear_fwd(p1, p2, v, alpha, out=out, dev_status=status, stream=stream)
+    bwd = lambda: binding.linear_bwd(p1, p2, v, alpha, dy, workspace=wsb, dev_status=status,
+                                     stream=stream)
+    for _ in range(warmup):
+        fwd(); bwd()
+    ev = [[torch.cuda.Event(enable_timing=True) for _ in range(3)] for _ in range(steps)]
+    torch.cuda.synchronize(dev)
+    for e in ev:
+        e[0].record(stream); fwd(); e[1].record(stream); bwd(); e[2].record(stream)
+    torch.cuda.synchronize(dev)
+    if int(status.item()) != 0:
+        raise SystemExit(f"linear device status {binding.status_string(int(status.item()))}")
+    ms_f = statistics.mean(e[0].elapsed_time(e[1]) for e in ev)
+    ms_b = statistics.mean(e[1].elapsed_time(e[2]) for e in ev)
+    tok_h = w.B * w.T * w.H
+    fl_f, fl_b = 5.0 * tok_h * w.d * w.d, 16.0 * tok_h * w.d * w.d
+    ach = fl_f / (ms_f * 1e-3) / 1e12
+    return {"config": {**c, "dtype": "bf16", "alpha": "KDA-style draw (workloads)"},
+            "ms_fwd": ms_f, "ms_bwd": ms_b, "tokens_per_s": w.B * w.T / ((ms_f + ms_b) * 1e-3),
+            "roofline": {"bound": "alu", "kernel": "linear fwd_kernel", "achieved": ach,
+                         "peak": FP32_FMA_TFLOPS, "unit": "TFLOP/s (fp32 FMA)",
+                         "frac": ach / FP32_FMA_TFLOPS,
+                         "bwd_achieved": fl_b / (ms_b * 1e-3) / 1e12},
+            "gpu_launches_per_step": 3}
+
+
 def run_ours(args, w):
     from paper_2608_20172_gb300 import binding
     dist, ws, rank, local = _dist()
@@ -413,6 +457,7 @@ def run_ours(args, w):
     }
     if rank == 0 and ws == 1:
         line["decode"] = decode_measure(binding, dev, peaks)
+        line["linear"] = linear_measure(binding, dev)
     if rank == 0 and not args.no_cpu_baseline and ws == 1:
         cb = cpu_oracle_run(w, min_seconds=10.0)
         line["cpu_baseline"] = {

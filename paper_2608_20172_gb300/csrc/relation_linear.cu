@@ -10,12 +10,12 @@
 // of Eq. (retention-vector) is upstream), p1, p2 are taken after RoPE (upstream).
 //
 // The recurrence never mixes information columns: column j of C evolves on its own.  The
-// forward therefore gives thread (j, half) column j for half of the rows, with that part
-// of the state in registers; a token costs d/2 multiply-adds three times per thread and
-// one pair shuffle (the two halves of the read).  One CTA per (b, h) walks the tokens in
-// order; tokens are staged through shared memory in chunks of kChunkT, double-buffered,
-// with S_t, 1/|p1_t|, 1/|p2_t| computed per chunk (S is folded into the coordinates:
-// q'_t = S_t ^p1_t, k'_t = S_t ^p2_t).
+// forward therefore gives each column to kRG threads, each keeping d / kRG rows of it in
+// registers; a token costs 3 d / kRG multiply-adds per thread (the read is summed over
+// the column's threads once per chunk).  One CTA per (b, h) walks the tokens in
+// order; tokens are staged through shared memory in double-buffered chunks, with S_t,
+// 1/|p1_t|, 1/|p2_t| computed per chunk (S is folded into the coordinates:
+// q'_t = S_t ^p1_t, k'_t = S_t ^p2_t).  Loads are 4-element vectors without conditions.
 // The backward (below) walks the tokens in reverse with the adjoint state, recomputing
 // the states of each chunk of kChunkB tokens from checkpoints the kernel stores first.
 #include <math.h>
@@ -53,34 +53,54 @@ struct Chunk {
   float scal[NTOK][4];    // S, 1/|p1|, 1/|p2|
 };
 
-// Raw loads of chunk `ch` (tokens ch * kChunkT ...) into registers: element e of the
-// chunk's 4 * kChunkT * D values goes to thread e % NT, slot e / NT.
+// Four consecutive elements as fp32 (8- or 16-byte aligned vector load).
+template <typename TI>
+__device__ __forceinline__ float4 ld4(const TI* p);
+template <>
+__device__ __forceinline__ float4 ld4<float>(const float* p) {
+  return *reinterpret_cast<const float4*>(p);
+}
+template <>
+__device__ __forceinline__ float4 ld4<__nv_bfloat16>(const __nv_bfloat16* p) {
+  const uint2 w = *reinterpret_cast<const uint2*>(p);
+  const float2 lo = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&w.x));
+  const float2 hi = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&w.y));
+  return make_float4(lo.x, lo.y, hi.x, hi.y);
+}
+
+// Loads of chunk `ch` (tokens ch * NTOK ...) into registers as 4-element vectors: vector
+// v of an array (token v / (D/4), columns 4 (v % (D/4)) ..) goes to thread v % NT.  The
+// loads carry no condition (rows past T are clamped to T - 1 and zeroed after the load),
+// so a thread's loads are all in flight together.
 template <typename TI, int D, int NT, int NTOK = kChunkT>
 struct Loader {
-  static constexpr int N = 4 * NTOK * D / NT;  // values per thread
-  float r[N];
+  static constexpr int NV = NTOK * D / 4 / NT;  // vectors per thread and array
+  static_assert(NV >= 1 && NV * NT * 4 == NTOK * D, "chunk / thread split");
+  float4 r[4][NV];
   __device__ __forceinline__ void load(const LinearProblem& p, int b, int h, int ch) {
 #pragma unroll
-    for (int n = 0; n < N; ++n) {
-      const int e = n * NT + (int)threadIdx.x;
-      const int c = e % D, a = (e / D) % 4, tt = e / (4 * D);
-      const int t = ch * NTOK + tt;
-      float x = 0.f;
-      if (t < p.T) {
-        const long long off = (long long)b * p.sB + (long long)t * p.sT + (long long)h * p.sH + c;
-        if (a == 0) x = p.alpha[off];
-        else if (a == 1) x = ldx<TI>(reinterpret_cast<const TI*>(p.p1) + off);
-        else if (a == 2) x = ldx<TI>(reinterpret_cast<const TI*>(p.p2) + off);
-        else x = ldx<TI>(reinterpret_cast<const TI*>(p.v) + off);
-      }
-      r[n] = x;
+    for (int n = 0; n < NV; ++n) {
+      const int v = n * NT + (int)threadIdx.x;
+      const int tt = v / (D / 4), c4 = (v % (D / 4)) * 4;
+      const int t = ch * NTOK + tt, tc = min(t, p.T - 1);
+      const long long off =
+          (long long)b * p.sB + (long long)tc * p.sT + (long long)h * p.sH + c4;
+      float4 x[4];
+      x[0] = ld4<float>(p.alpha + off);
+      x[1] = ld4<TI>(reinterpret_cast<const TI*>(p.p1) + off);
+      x[2] = ld4<TI>(reinterpret_cast<const TI*>(p.p2) + off);
+      x[3] = ld4<TI>(reinterpret_cast<const TI*>(p.v) + off);
+#pragma unroll
+      for (int a = 0; a < 4; ++a) r[a][n] = t < p.T ? x[a] : make_float4(0.f, 0.f, 0.f, 0.f);
     }
   }
   __device__ __forceinline__ void store(Chunk<D, NTOK>& s) const {
 #pragma unroll
-    for (int n = 0; n < N; ++n) {
-      const int e = n * NT + (int)threadIdx.x;
-      (&s.vec[0][0][0])[e] = r[n];
+    for (int n = 0; n < NV; ++n) {
+      const int v = n * NT + (int)threadIdx.x;
+      const int tt = v / (D / 4), c4 = (v % (D / 4)) * 4;
+#pragma unroll
+      for (int a = 0; a < 4; ++a) *reinterpret_cast<float4*>(&s.vec[tt][a][c4]) = r[a][n];
     }
   }
 };
@@ -119,29 +139,42 @@ __device__ __forceinline__ void ask_self_chunk(Chunk<D, NTOK>& s, float tau_s) {
   __syncthreads();
 }
 
-// Forward: one CTA per head, thread (j, half) = column j, rows half * D/2 .. + D/2.
+// Forward: one CTA per head, kRG threads per column.  Thread (j, rg) = tid % D, tid / D
+// keeps rows rg * D/kRG .. + D/kRG of column j in registers.  A warp shares one row group,
+// so the per-token alpha, q', k' reads are one shared-memory broadcast per vector, and
+// each thread's partial read goes to shared memory: Y_t = I~_t + sum_rg e_rg is formed per
+// chunk (the output does not feed back into the recurrence), with no per-token shuffle.
+constexpr int kRG = 4;
+constexpr int kChunkF = 32;  // tokens per staged chunk (forward)
+
+template <int D>
+struct FwdSmem {
+  Chunk<D, kChunkF> buf[2];
+  float epart[kChunkF][kRG][D];  // partial reads of the chunk's tokens
+};
+
 template <typename TI, int D>
-__global__ void __launch_bounds__(2 * D) fwd_kernel(LinearProblem p) {
-  constexpr int NT = 2 * D, R = D / 2;
+__global__ void __launch_bounds__(kRG * D) fwd_kernel(LinearProblem p) {
+  constexpr int NT = kRG * D, R = D / kRG;
   extern __shared__ __align__(16) uint8_t smem_raw[];
-  Chunk<D>* buf = reinterpret_cast<Chunk<D>*>(smem_raw);
+  FwdSmem<D>& sm = *reinterpret_cast<FwdSmem<D>*>(smem_raw);
   const int bh = blockIdx.x, b = bh / p.H, h = bh % p.H;
-  const int j = threadIdx.x >> 1, half = threadIdx.x & 1, r0 = half * R;
-  const int n_ch = (p.T + kChunkT - 1) / kChunkT;
+  const int j = threadIdx.x % D, rg = threadIdx.x / D, r0 = rg * R;
+  const int n_ch = (p.T + kChunkF - 1) / kChunkF;
   float C[R];
 #pragma unroll
   for (int r = 0; r < R; ++r) C[r] = 0.f;
-  Loader<TI, D, NT> ld;
+  Loader<TI, D, NT, kChunkF> ld;
   ld.load(p, b, h, 0);
-  ld.store(buf[0]);
+  ld.store(sm.buf[0]);
   __syncthreads();
-  ask_self_chunk<D, NT>(buf[0], p.tau_s);
-  TI* Y = reinterpret_cast<TI*>(p.y) + (long long)b * p.sB + (long long)h * p.sH + j;
+  ask_self_chunk<D, NT, kChunkF>(sm.buf[0], p.tau_s);
+  TI* Y = reinterpret_cast<TI*>(p.y) + (long long)b * p.sB + (long long)h * p.sH;
   for (int ch = 0; ch < n_ch; ++ch) {
-    Chunk<D>& cur = buf[ch & 1];
+    Chunk<D, kChunkF>& cur = sm.buf[ch & 1];
     const bool more = ch + 1 < n_ch;
     if (more) ld.load(p, b, h, ch + 1);  // in flight while this chunk is computed
-    const int nt = min(kChunkT, p.T - ch * kChunkT);
+    const int nt = min(kChunkF, p.T - ch * kChunkF);
     for (int tt = 0; tt < nt; ++tt) {
       const float* al = &cur.vec[tt][0][r0];
       const float* qp = &cur.vec[tt][1][r0];
@@ -162,27 +195,33 @@ __global__ void __launch_bounds__(2 * D) fwd_kernel(LinearProblem p) {
           C[r + u] = fmaf(kv[u], I, cm);       // Become Others: write S k^ I~
         }
       }
-      e += __shfl_xor_sync(0xffffffffu, e, 1);  // the other half of the rows
-      if (half == 0) stx<TI>(Y + (long long)(ch * kChunkT + tt) * p.sT, I + e);  // Answer
+      sm.epart[tt][rg][j] = e;
+    }
+    __syncthreads();  // the chunk's partial reads are complete
+    for (int e = threadIdx.x; e < nt * D; e += NT) {  // Answer: Y_t = I~_t + E_t
+      const int tt = e / D, jj = e % D;
+      float y = cur.vec[tt][3][jj];
+#pragma unroll
+      for (int g = 0; g < kRG; ++g) y += sm.epart[tt][g][jj];
+      stx<TI>(Y + (long long)(ch * kChunkF + tt) * p.sT + jj, y);
     }
     if (more) {
-      // nxt held chunk ch - 1, which every thread finished before the barriers that ended
-      // the previous iteration
-      Chunk<D>& nxt = buf[(ch + 1) & 1];
+      // nxt held chunk ch - 1, which every thread finished before the barrier above
+      Chunk<D, kChunkF>& nxt = sm.buf[(ch + 1) & 1];
       ld.store(nxt);
-      __syncthreads();
-      ask_self_chunk<D, NT>(nxt, p.tau_s);
+      __syncthreads();  // also: epart is read above before the next chunk overwrites it
+      ask_self_chunk<D, NT, kChunkF>(nxt, p.tau_s);
     }
   }
 }
 
 template <typename TI, int D>
 cudaError_t fwd_t(const LinearProblem& p, cudaStream_t s) {
-  const int smem = 2 * (int)sizeof(Chunk<D>);
+  const int smem = (int)sizeof(FwdSmem<D>);
   cudaError_t e = cudaFuncSetAttribute(fwd_kernel<TI, D>,
                                        cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
   if (e != cudaSuccess) { note_failure("linear forward: shared memory attribute"); return e; }
-  fwd_kernel<TI, D><<<(unsigned)(p.B * p.H), 2 * D, smem, s>>>(p);
+  fwd_kernel<TI, D><<<(unsigned)(p.B * p.H), kRG * D, smem, s>>>(p);
   if ((e = cudaGetLastError()) != cudaSuccess) note_failure("linear forward: launch");
   return e;
 }
@@ -236,11 +275,11 @@ __global__ void __launch_bounds__(2 * D) bwd_kernel(LinearProblem p) {
     __syncthreads();          // the previous chunk's data is no longer read
     ld.load(p, b, h, ch);
     ld.store(sm.tok);
-    for (int e = threadIdx.x; e < kChunkB * D; e += NT) {
-      const int tt = e / D, cc = e % D, t = ch * kChunkB + tt;
-      sm.g[tt][cc] = t < p.T ? ldx<TI>(reinterpret_cast<const TI*>(p.dy) + hb +
-                                       (long long)t * p.sT + cc)
-                             : 0.f;
+    for (int v4 = threadIdx.x; v4 < kChunkB * D / 4; v4 += NT) {
+      const int tt = v4 / (D / 4), c4 = (v4 % (D / 4)) * 4, t = ch * kChunkB + tt;
+      const float4 g = ld4<TI>(reinterpret_cast<const TI*>(p.dy) + hb +
+                               (long long)min(t, p.T - 1) * p.sT + c4);
+      *reinterpret_cast<float4*>(&sm.g[tt][c4]) = t < p.T ? g : make_float4(0.f, 0.f, 0.f, 0.f);
     }
     __syncthreads();
     ask_self_chunk<D, NT, kChunkB>(sm.tok, p.tau_s);
