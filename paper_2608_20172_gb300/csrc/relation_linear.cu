@@ -232,24 +232,29 @@ cudaError_t fwd_t(const LinearProblem& p, cudaStream_t s) {
 //   dI~_t = dY_t + dC_t^T k'_t,   dk'_t = dC_t I~_t,   dq'_t = C^- dY_t,
 //   dC^- = dC_t + q'_t dY_t^T,   dalpha_t = rowsum(dC^- * C_{t-1}),   dC_{t-1} = Diag(alpha_t) dC^-
 // (C^- = Diag(alpha_t) C_{t-1}); a per-token pass then turns dq', dk' into dp1, dp2
-// through the normalisation and S.  Thread (c, half) owns row c of the state for half of
-// the columns, so the row sums (dk', dq', dalpha) are a pair shuffle and the column sum
+// through the normalisation and S.  kQ threads own row c of the state, a quarter of the
+// columns each, so the row sums (dk', dq', dalpha) are two shuffles and the column sum
 // (dI~) is reduced across rows by a shuffle reduce-scatter within each warp and shared
 // memory across warps.
-//   1. checkpoint pass: forward over the tokens, storing the state before every chunk of
-//      kChunkB tokens in the workspace;
-//   2. reverse sweep: per chunk (last first), the states before each of its tokens are
-//      recomputed from the checkpoint into shared memory, then the tokens are walked
-//      backwards;
+//   1. checkpoint pass: forward over the tokens, storing the state before every kChunkB
+//      tokens in the workspace;
+//   2. reverse sweep: tokens staged kStageB at a time; per sub-chunk of kChunkB (last
+//      first), the states before each of its tokens are recomputed from the checkpoint into
+//      shared memory, then the tokens are walked backwards;
 //   3. per-token pass: dp1, dp2.
-constexpr int kChunkB = 8;
+constexpr int kChunkB = 8;   // tokens per checkpoint / recomputed sub-chunk
+constexpr int kStageB = 16;  // tokens per staged chunk (two sub-chunks)
+constexpr int kQ = 4;        // threads per state row (each a quarter of the columns)
 
 template <int D>
 struct BwdSmem {
-  Chunk<D, kChunkB> tok;                // alpha, q', k', I~ of the chunk
-  float g[kChunkB][D];                  // dY of the chunk
-  float red[kChunkB][2 * D / 32][D];    // per-warp column sums of dC^T k'
-  float st[kChunkB][D][D];              // C_{t-1} of each token of the chunk
+  Chunk<D, kStageB> tok;                  // alpha, q', k', I~ of the staged chunk
+  float g[kStageB][D];                    // dY of the staged chunk
+  float red[kStageB][kQ * D / 32][D];     // per-warp column sums of dC^T k'
+  // C_{t-1} of each token of a sub-chunk, each thread's slice as float4s indexed
+  // [token][k][thread]: a thread only reads its own slice back, and consecutive lanes
+  // touch consecutive 16-byte words (no bank conflicts)
+  float4 st[kChunkB][D / (4 * kQ)][kQ * D];
 };
 
 template <int D>
@@ -258,125 +263,147 @@ __host__ __device__ constexpr long long ckpt_floats(int T) {
 }
 
 template <typename TI, int D>
-__global__ void __launch_bounds__(2 * D) bwd_kernel(LinearProblem p) {
-  constexpr int NT = 2 * D, R = D / 2, NW = NT / 32;
+__global__ void __launch_bounds__(kQ * D) bwd_kernel(LinearProblem p) {
+  constexpr int NT = kQ * D, R = D / kQ, NW = NT / 32;
   extern __shared__ __align__(16) uint8_t smem_raw[];
   BwdSmem<D>& sm = *reinterpret_cast<BwdSmem<D>*>(smem_raw);
   const int bh = blockIdx.x, b = bh / p.H, h = bh % p.H;
-  const int c = threadIdx.x >> 1, hc = threadIdx.x & 1, j0 = hc * R;
+  const int c = threadIdx.x / kQ, j0 = (threadIdx.x % kQ) * R;
+  const bool lead = threadIdx.x % kQ == 0;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int n_ch = (p.T + kChunkB - 1) / kChunkB;
+  const int n_st = (p.T + kStageB - 1) / kStageB;
   float* ckpt = reinterpret_cast<float*>(p.workspace) + (long long)bh * ckpt_floats<D>(p.T);
   float* dqk = reinterpret_cast<float*>(p.workspace) + (long long)p.B * p.H * ckpt_floats<D>(p.T) +
                (long long)bh * p.T * 2 * D;  // [T][2][D]: dq', dk'
   const long long hb = (long long)b * p.sB + (long long)h * p.sH;
-  Loader<TI, D, NT, kChunkB> ld;
-  auto stage = [&](int ch) {  // token data of chunk ch into sm.tok (and dY into sm.g)
-    __syncthreads();          // the previous chunk's data is no longer read
-    ld.load(p, b, h, ch);
+  Loader<TI, D, NT, kStageB> ld;
+  auto stage = [&](int sc, bool with_dy) {  // token data of staged chunk sc
+    __syncthreads();                         // the previous chunk's data is no longer read
+    ld.load(p, b, h, sc);
     ld.store(sm.tok);
-    for (int v4 = threadIdx.x; v4 < kChunkB * D / 4; v4 += NT) {
-      const int tt = v4 / (D / 4), c4 = (v4 % (D / 4)) * 4, t = ch * kChunkB + tt;
-      const float4 g = ld4<TI>(reinterpret_cast<const TI*>(p.dy) + hb +
-                               (long long)min(t, p.T - 1) * p.sT + c4);
-      *reinterpret_cast<float4*>(&sm.g[tt][c4]) = t < p.T ? g : make_float4(0.f, 0.f, 0.f, 0.f);
+    if (with_dy) {
+      for (int v4 = threadIdx.x; v4 < kStageB * D / 4; v4 += NT) {
+        const int tt = v4 / (D / 4), c4 = (v4 % (D / 4)) * 4, t = sc * kStageB + tt;
+        const float4 g = ld4<TI>(reinterpret_cast<const TI*>(p.dy) + hb +
+                                 (long long)min(t, p.T - 1) * p.sT + c4);
+        *reinterpret_cast<float4*>(&sm.g[tt][c4]) = t < p.T ? g : make_float4(0.f, 0.f, 0.f, 0.f);
+      }
     }
     __syncthreads();
-    ask_self_chunk<D, NT, kChunkB>(sm.tok, p.tau_s);
+    ask_self_chunk<D, NT, kStageB>(sm.tok, p.tau_s);
   };
-  // 1. checkpoint pass: only the row update C <- Diag(alpha) C + k' I~^T is needed
+  auto row_step = [&](float (&Cs)[R], int tt) {  // C <- Diag(alpha) C + k' I~^T, own row
+    const float a = sm.tok.vec[tt][0][c], kp = sm.tok.vec[tt][2][c];
+    const float* I = &sm.tok.vec[tt][3][j0];
+#pragma unroll
+    for (int i = 0; i < R; i += 4) {
+      const float4 i4 = *reinterpret_cast<const float4*>(I + i);
+      Cs[i] = fmaf(kp, i4.x, a * Cs[i]);
+      Cs[i + 1] = fmaf(kp, i4.y, a * Cs[i + 1]);
+      Cs[i + 2] = fmaf(kp, i4.z, a * Cs[i + 2]);
+      Cs[i + 3] = fmaf(kp, i4.w, a * Cs[i + 3]);
+    }
+  };
+  // 1. checkpoint pass: the state before every kChunkB tokens
   float C[R];
 #pragma unroll
   for (int i = 0; i < R; ++i) C[i] = 0.f;
-  for (int ch = 0; ch < n_ch; ++ch) {
-    float* ck = ckpt + (long long)ch * D * D + c * D + j0;
+  for (int sc = 0; sc < n_st; ++sc) {
+    const int nt = min(kStageB, p.T - sc * kStageB);
+    stage(sc, false);
+    for (int tt = 0; tt < nt; ++tt) {
+      if (tt % kChunkB == 0) {
+        float* ck = ckpt + (long long)((sc * kStageB + tt) / kChunkB) * D * D + c * D + j0;
 #pragma unroll
-    for (int i = 0; i < R; i += 4)
-      *reinterpret_cast<float4*>(ck + i) = make_float4(C[i], C[i + 1], C[i + 2], C[i + 3]);
-    if (ch + 1 == n_ch) break;  // the last chunk's end state is not needed
-    stage(ch);
-    for (int tt = 0; tt < kChunkB; ++tt) {
-      const float a = sm.tok.vec[tt][0][c], kp = sm.tok.vec[tt][2][c];
-      const float* I = &sm.tok.vec[tt][3][j0];
-#pragma unroll
-      for (int i = 0; i < R; ++i) C[i] = fmaf(kp, I[i], a * C[i]);
+        for (int i = 0; i < R; i += 4)
+          *reinterpret_cast<float4*>(ck + i) = make_float4(C[i], C[i + 1], C[i + 2], C[i + 3]);
+      }
+      row_step(C, tt);
     }
   }
   // 2. reverse sweep
   float dC[R];
 #pragma unroll
   for (int i = 0; i < R; ++i) dC[i] = 0.f;
-  for (int ch = n_ch - 1; ch >= 0; --ch) {
-    stage(ch);
-    const int nt = min(kChunkB, p.T - ch * kChunkB);
-    const float* ck = ckpt + (long long)ch * D * D + c * D + j0;
+  for (int sc = n_st - 1; sc >= 0; --sc) {
+    stage(sc, true);
+    const int nt = min(kStageB, p.T - sc * kStageB);
+    for (int sub = (nt - 1) / kChunkB; sub >= 0; --sub) {
+      const int tb = sub * kChunkB, ns = min(kChunkB, nt - tb);
+      const float* ck = ckpt + (long long)((sc * kStageB + tb) / kChunkB) * D * D + c * D + j0;
 #pragma unroll
-    for (int i = 0; i < R; i += 4) {
-      const float4 x = *reinterpret_cast<const float4*>(ck + i);
-      C[i] = x.x; C[i + 1] = x.y; C[i + 2] = x.z; C[i + 3] = x.w;
-    }
-    for (int tt = 0; tt < nt; ++tt) {  // C_{t-1} of each token into shared memory
-      float* dst = &sm.st[tt][c][j0];
-#pragma unroll
-      for (int i = 0; i < R; i += 4)
-        *reinterpret_cast<float4*>(dst + i) = make_float4(C[i], C[i + 1], C[i + 2], C[i + 3]);
-      const float a = sm.tok.vec[tt][0][c], kp = sm.tok.vec[tt][2][c];
-      const float* I = &sm.tok.vec[tt][3][j0];
-#pragma unroll
-      for (int i = 0; i < R; ++i) C[i] = fmaf(kp, I[i], a * C[i]);
-    }
-    for (int tt = nt - 1; tt >= 0; --tt) {
-      const int t = ch * kChunkB + tt;
-      const float a = sm.tok.vec[tt][0][c], qp = sm.tok.vec[tt][1][c];
-      const float kp = sm.tok.vec[tt][2][c];
-      const float* I = &sm.tok.vec[tt][3][j0];
-      const float* G = &sm.g[tt][j0];
-      const float* Cp = &sm.st[tt][c][j0];
-      float dk = 0.f, dq = 0.f, da = 0.f, col[R];
-#pragma unroll
-      for (int i = 0; i < R; ++i) {
-        const float cp = Cp[i], g = G[i];
-        col[i] = dC[i] * kp;              // this row's share of dC^T k'
-        dk = fmaf(dC[i], I[i], dk);
-        dq = fmaf(a * cp, g, dq);
-        const float dcm = fmaf(qp, g, dC[i]);
-        da = fmaf(dcm, cp, da);
-        dC[i] = a * dcm;                   // dL/dC_{t-1}
+      for (int i = 0; i < R; i += 4) {
+        const float4 x = *reinterpret_cast<const float4*>(ck + i);
+        C[i] = x.x; C[i + 1] = x.y; C[i + 2] = x.z; C[i + 3] = x.w;
       }
-      dk += __shfl_xor_sync(0xffffffffu, dk, 1);
-      dq += __shfl_xor_sync(0xffffffffu, dq, 1);
-      da += __shfl_xor_sync(0xffffffffu, da, 1);
-      if (hc == 0) {
-        p.dalpha[hb + (long long)t * p.sT + c] = da;
-        dqk[(long long)t * 2 * D + c] = dq;
-        dqk[(long long)t * 2 * D + D + c] = dk;
+      for (int u = 0; u < ns; ++u) {  // C_{t-1} of each token of the sub-chunk
+#pragma unroll
+        for (int i = 0; i < R; i += 4)
+          sm.st[u][i / 4][threadIdx.x] = make_float4(C[i], C[i + 1], C[i + 2], C[i + 3]);
+        if (u + 1 < ns) row_step(C, tb + u);
       }
-      // column sums over the warp's 16 rows: reduce-scatter over lane bits 1..4
-      int off = 0, n = R;
+      for (int u = ns - 1; u >= 0; --u) {
+        const int tt = tb + u, t = sc * kStageB + tt;
+        const float a = sm.tok.vec[tt][0][c], qp = sm.tok.vec[tt][1][c];
+        const float kp = sm.tok.vec[tt][2][c];
+        const float* I = &sm.tok.vec[tt][3][j0];
+        const float* G = &sm.g[tt][j0];
+        float Cp[R];
 #pragma unroll
-      for (int m = 16; m >= 2; m >>= 1) {
-        n >>= 1;
-        const bool up = (lane & m) != 0;
-#pragma unroll
-        for (int i = 0; i < R / 2; ++i) {
-          if (i < n) {
-            const float send = up ? col[i] : col[i + n];
-            const float keep = up ? col[i + n] : col[i];
-            col[i] = keep + __shfl_xor_sync(0xffffffffu, send, m);
-          }
+        for (int i = 0; i < R; i += 4) {
+          const float4 x = sm.st[u][i / 4][threadIdx.x];
+          Cp[i] = x.x; Cp[i + 1] = x.y; Cp[i + 2] = x.z; Cp[i + 3] = x.w;
         }
-        off += up ? n : 0;
-      }
+        float dk = 0.f, dq = 0.f, da = 0.f, col[R];
 #pragma unroll
-      for (int i = 0; i < R / 16; ++i) sm.red[tt][warp][j0 + off + i] = col[i];
+        for (int i = 0; i < R; ++i) {
+          const float cp = Cp[i], g = G[i];
+          col[i] = dC[i] * kp;              // this row's share of dC^T k'
+          dk = fmaf(dC[i], I[i], dk);
+          dq = fmaf(a * cp, g, dq);
+          const float dcm = fmaf(qp, g, dC[i]);
+          da = fmaf(dcm, cp, da);
+          dC[i] = a * dcm;                   // dL/dC_{t-1}
+        }
+#pragma unroll
+        for (int o = 1; o < kQ; o <<= 1) {  // the row's kQ threads
+          dk += __shfl_xor_sync(0xffffffffu, dk, o);
+          dq += __shfl_xor_sync(0xffffffffu, dq, o);
+          da += __shfl_xor_sync(0xffffffffu, da, o);
+        }
+        if (lead) {
+          p.dalpha[hb + (long long)t * p.sT + c] = da;
+          dqk[(long long)t * 2 * D + c] = dq;
+          dqk[(long long)t * 2 * D + D + c] = dk;
+        }
+        // column sums over the warp's 32 / kQ rows: reduce-scatter over the lane bits above
+        // the kQ column threads
+        int off = 0, n = R;
+#pragma unroll
+        for (int m = 16; m >= kQ; m >>= 1) {
+          n >>= 1;
+          const bool up = (lane & m) != 0;
+#pragma unroll
+          for (int i = 0; i < R / 2; ++i) {
+            if (i < n) {
+              const float send = up ? col[i] : col[i + n];
+              const float keep = up ? col[i + n] : col[i];
+              col[i] = keep + __shfl_xor_sync(0xffffffffu, send, m);
+            }
+          }
+          off += up ? n : 0;
+        }
+#pragma unroll
+        for (int i = 0; i < R / (32 / kQ); ++i) sm.red[tt][warp][j0 + off + i] = col[i];
+      }
     }
     __syncthreads();
     for (int e = threadIdx.x; e < nt * D; e += NT) {  // dI~_t = dY_t + dC_t^T k'_t
-      const int tt = e / D, jj = e % D, t = ch * kChunkB + tt;
-      float s = sm.g[tt][jj];
+      const int tt = e / D, jj = e % D, t = sc * kStageB + tt;
+      float s2 = sm.g[tt][jj];
 #pragma unroll
-      for (int w = 0; w < NW; ++w) s += sm.red[tt][w][jj];
-      stx<TI>(reinterpret_cast<TI*>(p.dv) + hb + (long long)t * p.sT + jj, s);
+      for (int w = 0; w < NW; ++w) s2 += sm.red[tt][w][jj];
+      stx<TI>(reinterpret_cast<TI*>(p.dv) + hb + (long long)t * p.sT + jj, s2);
     }
   }
 }
@@ -446,7 +473,7 @@ cudaError_t bwd_t(const LinearProblem& p, cudaStream_t s) {
   cudaError_t e = cudaFuncSetAttribute(bwd_kernel<TI, D>,
                                        cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
   if (e != cudaSuccess) { note_failure("linear backward: shared memory attribute"); return e; }
-  bwd_kernel<TI, D><<<(unsigned)(p.B * p.H), 2 * D, smem, s>>>(p);
+  bwd_kernel<TI, D><<<(unsigned)(p.B * p.H), kQ * D, smem, s>>>(p);
   if ((e = cudaGetLastError()) != cudaSuccess) { note_failure("linear backward: launch"); return e; }
   const long long toks = (long long)p.B * p.H * p.T;
   post_kernel<TI, D><<<(unsigned)((toks * 32 + 255) / 256), 256, 0, s>>>(p);
