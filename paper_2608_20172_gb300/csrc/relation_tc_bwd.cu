@@ -472,7 +472,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
       }
     }
-    if (lane == 0) tma_store_wait_all();
+    if (lane == 0) tma_store_wait_read_all();  // the staging reads; the adds finish with the kernel
   } else {
     // ------------------------------------------------------ elementwise + epilogue
     // Both warpgroups work on every step: warpgroup wg takes its 32 query columns.

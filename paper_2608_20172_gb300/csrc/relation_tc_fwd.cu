@@ -386,7 +386,7 @@ __global__ void __launch_bounds__(kThreads, 2)
           tma_store_4d(&tmO, sb + C::OFF_Q + warp * (32 * D * 2) + kb * (32 * 128), kb * 64,
                        q0 + warp * 32, h, b);
         tma_store_commit();
-        tma_store_wait_all();  // the staging buffer must outlive the store
+        tma_store_wait_read_all();  // the staging buffer must outlive the store's reads
       }
       __syncwarp();
       if (r < p.T) {
