@@ -190,7 +190,8 @@ template <int D>
 __global__ void __launch_bounds__(kThreads, 1)
     bwd_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmK,
                   const __grid_constant__ CUtensorMap tmV, const __grid_constant__ CUtensorMap tmG,
-                  const __grid_constant__ CUtensorMap tmDQ, Problem p, BwdWorkspace ws, int n_t,
+                  const __grid_constant__ CUtensorMap tmDQ, const __grid_constant__ CUtensorMap tmDK,
+                  const __grid_constant__ CUtensorMap tmDV, Problem p, BwdWorkspace ws, int n_t,
                   int t_pad) {
   using C = Cfg<D>;
   extern __shared__ uint8_t smem_raw[];
@@ -242,6 +243,8 @@ __global__ void __launch_bounds__(kThreads, 1)
       tma_prefetch_desc(&tmK);
       tma_prefetch_desc(&tmV);
       tma_prefetch_desc(&tmG);
+      tma_prefetch_desc(&tmDK);
+      tma_prefetch_desc(&tmDV);
       mbar_arrive_expect_tx(bar(B_KV), 2 * C::KVT);
       for (int kb = 0; kb < C::KB; ++kb) {
         tma_load_4d(sb + C::OFF_K + kb * 16384, &tmK, bar(B_KV), kb * 64, k0, h, b);
@@ -323,6 +326,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       // sn - NBUF done) and once the GEMM that releases the Q/dO stage it loads into has
       // been issued: waiting for that stage's load earlier would deadlock.
       int sn = 0, units_done = 0;
+      bool acc_done = false;  // B_ACC committed
       while (ok && sn < total && sn < C::NBUF) {
         ok = issue_u(sn);
         if (ok) issue_dp(sn);
@@ -350,6 +354,10 @@ __global__ void __launch_bounds__(kThreads, 1)
           mma_ts(tmem + C::COL_DK, tmem + dcol + acol,
                  smem_desc_sw128(sb + C::OFF_Q + st * C::QSZ + rows + kk * 2048, C::KBQ, 1024),
                  id_acc, (s > 0 || kk > 0) ? 1u : 0u);
+        }
+        if (s == total - 1) {  // dK and dV are final: the epilogue need not wait for dQ
+          mma_commit(bar(B_ACC));
+          acc_done = true;
         }
         if (C::HALF) {
           mma_commit(bar(B_QE + st));  // the step's Q / dO rows are no longer needed
@@ -394,7 +402,7 @@ __global__ void __launch_bounds__(kThreads, 1)
           ++sn;
         }
       }
-      mma_commit(bar(B_ACC));
+      if (!acc_done) mma_commit(bar(B_ACC));  // after an abort: whatever completed
     }
     __syncwarp();
   } else if (warp >= W_DQ) {
@@ -530,49 +538,64 @@ __global__ void __launch_bounds__(kThreads, 1)
     // Exchange sums from TMEM plus the Self entry of key j (from the row pass):
     //   dK_j = (sum dS'_ij q_i) / (2 sqrt d) + dS_jj q_j / sqrt d
     //   dV_j =  sum P_ij dO_i               + F_jj dO_j
-    // The Self operands (q_j or dO_j, and the scalar) are fetched while the last MMAs run.
-    const int j = key_g;
-    const long long off = (long long)b * p.sB + (long long)h * p.sH + (long long)j * p.sT;
-    const bool valid = j < p.T;
+    // The Self operands (q_j or dO_j, and the scalar) are loaded before the wait for the
+    // last MMAs and first used after it: the loads carry no condition (rows past T and
+    // padding columns read a clamped address; their results are never stored).
+    const int jr = min(key_g, p.T - 1);
+    const __nv_bfloat16* srow_ptr =
+        reinterpret_cast<const __nv_bfloat16*>(wg == 0 ? p.q : p.dout) + (long long)b * p.sB +
+        (long long)h * p.sH + (long long)jr * p.sT;
     uint4 rowv[D / 8];
-    float self = 0.f;
-    if (valid) {
-      const __nv_bfloat16* row =
-          reinterpret_cast<const __nv_bfloat16*>(wg == 0 ? p.q : p.dout) + off;
 #pragma unroll
-      for (int c = 0; c < D / 8; ++c)
-        rowv[c] = 8 * c < p.d ? *reinterpret_cast<const uint4*>(row + 8 * c) : make_uint4(0, 0, 0, 0);
-      const long long srow = (long long)bh * p.T + j;
-      self = wg == 0 ? ws.dS_self[srow] * isd : ws.F_self[srow];
-    }
+    for (int c = 0; c < D / 8; ++c)
+      rowv[c] = *reinterpret_cast<const uint4*>(srow_ptr + min(8 * c, p.d - 8));
+    const float self_raw = wg == 0 ? ws.dS_self[(long long)bh * p.T + jr]
+                                   : ws.F_self[(long long)bh * p.T + jr];
     if (ok) ok = __all_sync(0xffffffffu, mbar_wait(bar(B_ACC), 0, ab));
     tc_fence_after();
     if (ok) {
       const uint32_t col = wg == 0 ? C::COL_DK : C::COL_DV;
-      __nv_bfloat16* dst = reinterpret_cast<__nv_bfloat16*>(wg == 0 ? p.dk : p.dv) + off;
       const float sc = wg == 0 ? 0.5f * isd : 1.0f;
+      const float self = wg == 0 ? self_raw * isd : self_raw;
+      // Staged as 32 rows x D per warp (128-byte swizzle) in the Q (dK) or dO (dV) stages,
+      // which no MMA reads any more (B_ACC follows the last one that did), and written by
+      // TMA stores that clip rows past T and padding columns.
+      const int wq = warp & 3;
+      const uint32_t stg_off = (wg == 0 ? C::OFF_Q : C::OFF_DO) + wq * (32 * D * 2);
+      uint8_t* stg = smem + stg_off + lane * 128;
 #pragma unroll
       for (int c0 = 0; c0 < D; c0 += 32) {
         uint32_t a[32];
         tmem_ld32(trow + col + c0, a);
         tmem_ld_wait();
-        if (valid) {
+        const int kb = c0 >> 6;  // 64-column block
 #pragma unroll
-          for (int c8 = 0; c8 < 32; c8 += 8) {
-            const uint4 rv = rowv[(c0 + c8) / 8];
-            const uint32_t r4[4] = {rv.x, rv.y, rv.z, rv.w};
-            uint32_t o4[4];
+        for (int c8 = 0; c8 < 32; c8 += 8) {
+          const uint4 rv = rowv[(c0 + c8) / 8];
+          const uint32_t r4[4] = {rv.x, rv.y, rv.z, rv.w};
+          uint32_t o4[4];
 #pragma unroll
-            for (int e = 0; e < 4; ++e) {
-              const float2 rf = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&r4[e]));
-              o4[e] = pack_bf16x2(fmaf(__uint_as_float(a[c8 + 2 * e]), sc, self * rf.x),
-                                  fmaf(__uint_as_float(a[c8 + 2 * e + 1]), sc, self * rf.y));
-            }
-            if (c0 + c8 < p.d)  // padding columns (d_h < D) are not stored
-              *reinterpret_cast<uint4*>(dst + c0 + c8) = make_uint4(o4[0], o4[1], o4[2], o4[3]);
+          for (int e = 0; e < 4; ++e) {
+            const float2 rf = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&r4[e]));
+            o4[e] = pack_bf16x2(fmaf(__uint_as_float(a[c8 + 2 * e]), sc, self * rf.x),
+                                fmaf(__uint_as_float(a[c8 + 2 * e + 1]), sc, self * rf.y));
           }
+          const int chunk = ((c0 & 63) + c8) >> 3;  // 16-byte chunk within the 128-byte row
+          *reinterpret_cast<uint4*>(stg + kb * (32 * 128) + ((chunk ^ (lane & 7)) << 4)) =
+              make_uint4(o4[0], o4[1], o4[2], o4[3]);
         }
       }
+      fence_async_smem();
+      __syncwarp();
+      if (lane == 0) {
+        const CUtensorMap* tm = wg == 0 ? &tmDK : &tmDV;
+#pragma unroll
+        for (int kb = 0; kb < C::KB; ++kb)
+          tma_store_4d(tm, sb + stg_off + kb * (32 * 128), kb * 64, k0 + wq * 32, h, b);
+        tma_store_commit();
+        tma_store_wait_read_all();  // the staging must outlive the store's reads
+      }
+      __syncwarp();
     }
 #pragma unroll
     for (int o = 16; o > 0; o >>= 1) dlam += __shfl_xor_sync(0xffffffffu, dlam, o);
@@ -777,19 +800,20 @@ static cudaError_t bwd_t(const Problem& p, const BwdWorkspace& ws, unsigned stag
     e = cudaFuncSetAttribute(bwd::bwd_tc_kernel<D>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                              smem);
     if (e != cudaSuccess) { note_failure("backward: shared memory attribute"); return e; }
-    CUtensorMap mq, mk, mv, mg, mdq;
+    CUtensorMap mq, mk, mv, mg, mdq, mdk, mdv;
     constexpr int qrows = bwd::Cfg<D>::QROWS;
     if (!make_tmap_bf16(&mq, p.q, p, qrows) || !make_tmap_bf16(&mk, p.k, p, 128) ||
-        !make_tmap_bf16(&mv, p.v, p, 128) || !make_tmap_bf16(&mg, p.dout, p, qrows)) {
-      note_failure("backward: TMA descriptor of Q/K/V/dO");
+        !make_tmap_bf16(&mv, p.v, p, 128) || !make_tmap_bf16(&mg, p.dout, p, qrows) ||
+        !make_tmap_bf16(&mdk, p.dk, p, 32) || !make_tmap_bf16(&mdv, p.dv, p, 32)) {
+      note_failure("backward: TMA descriptor of Q/K/V/dO/dK/dV");
       return cudaErrorInvalidValue;
     }
     if (!make_tmap_dq(&mdq, ws.dq_acc, p.B * p.H * t_pad, D)) {
       note_failure("backward: TMA descriptor of the dQ accumulator");
       return cudaErrorInvalidValue;
     }
-    bwd::bwd_tc_kernel<D><<<(unsigned)grid, bwd::kThreads, smem, s>>>(mq, mk, mv, mg, mdq, p, ws,
-                                                                     n_t, t_pad);
+    bwd::bwd_tc_kernel<D><<<(unsigned)grid, bwd::kThreads, smem, s>>>(mq, mk, mv, mg, mdq, mdk,
+                                                                     mdv, p, ws, n_t, t_pad);
     if ((e = cudaGetLastError()) != cudaSuccess) { note_failure("backward: tile kernel launch"); return e; }
   }
   if (stages & 4) {
