@@ -7,13 +7,13 @@
 //   dS_ii = dR_ii S_i (1 - S_i) / tau_S          (Self, j = i; S_i = sigmoid(u_ii / tau_S))
 //   dV_j += F_ij dO_i,  dK_j += dS_ij q_i / sqrt(d),  dQ_i += dS_ij k_j / sqrt(d)
 // with F_ij = exp(E_ij - lambda log i - logZ_i) (j < i) and F_ii = exp(S_i - logZ_i).
-// The Self entries (j = i) are computed per row in fp32 by the row pass and added by the
-// dK / dV epilogue and the dQ finalisation; the tile kernel handles the Exchange pairs
-// (j < i) only.
+// The Self entries (j = i) are computed per row in fp32 by the row pass; the tile kernel
+// computes the Exchange pairs (j < i) and places the Self values on the diagonal of its
+// diagonal tile, so that its dV, dK and dQ products include them.
 //
 // Three launches: a row pass (D_i, the Self entries and their dlambda terms, the tile
 // kernel's per-query scalars, zeroed fp32 dQ accumulator), the tile kernel, and a
-// finalisation (dQ to bf16 plus the Self term, dlambda reduction).
+// finalisation (dQ to bf16, dlambda reduction).
 //
 // Tile kernel: one CTA per 128 keys of one head, visiting query tiles from the diagonal
 // to the end of the sequence.  Keys sit on TMEM lanes.  Per step of 64 query columns:
@@ -74,10 +74,12 @@ struct Cfg {
   static constexpr int SW = QROWS;             // per-query scalars of a stage: array stride
   static constexpr int STB = 3 * SW * 4;       // bytes of one stage's scalars
   static constexpr int DSZ = HALF ? 16384 : 32768;  // one dS' buffer (per step / per tile)
-  static constexpr int DQSLOTS = HALF ? 1 : 2;      // 4 KB staging slots per dQ warp
-  static constexpr int OFF_K = 0;
-  static constexpr int OFF_V = OFF_K + KVT;
-  static constexpr int OFF_Q = OFF_V + KVT;
+  static constexpr int DQSLOTS = 1;                 // 4 KB staging slot per dQ warp
+  // K / V buffers: d_h = 64 runs persistent CTAs and loads the next unit's K and V while
+  // the current unit runs; d_h = 128 takes one unit per CTA.
+  static constexpr int NKV = HALF ? 1 : 2;
+  static constexpr int OFF_KV = 0;                  // buffer k: K at + 2 KVT k, V after it
+  static constexpr int OFF_Q = OFF_KV + NKV * 2 * KVT;
   static constexpr int OFF_DO = OFF_Q + NQS * QSZ;
   static constexpr int OFF_DS = OFF_DO + NQS * QSZ;
   static constexpr int OFF_DQS = OFF_DS + 2 * DSZ;
@@ -96,8 +98,10 @@ struct Cfg {
 static_assert(Cfg<64>::SMEM <= 232448 && Cfg<128>::SMEM <= 232448, "shared memory");
 
 enum : int {
-  B_KV = 0, B_QF = 1, B_QE = 4, B_S = 7, B_P = 9, B_DQF = 11, B_DQE = 13, B_ACC = 15
+  B_KV = 0, B_QF = 1, B_QE = 4, B_S = 7, B_P = 9, B_DQF = 11, B_DQE = 13, B_ACC = 15,
+  B_KVE = 16, B_STG = 18, B_KV1 = 19  // B_KVE + k: K / V buffer k free; B_KV1: buffer 1 full
 };
+__device__ __forceinline__ int kv_full(int k) { return k == 0 ? B_KV : B_KV1; }
 
 __device__ __forceinline__ void drain_wait(uint32_t bar, uint32_t parity) {
   const unsigned long long t0 = globaltimer_ns();
@@ -142,12 +146,14 @@ struct EwConst {
 //   P = 2^(U c2k (1 + t) + c2),  t = tanh(u/2),
 //   2 SiLU'(u) = a (1 + h (1 - t)) with a = 1 + t, h = u / 2.
 // On the diagonal tile (DIAG) the entries with query <= key get c2 = -inf, so P, dS' and
-// their dlambda terms are exactly zero: the Self entry (query == key) is not part of
-// the tile; the row pass and the epilogues add it.
+// their dlambda terms are exactly zero; the Self entry (query == key) then takes the
+// row pass's values, P = F_tt and dS' = 2 dS_tt (self2 = {F_tt, dS_tt}), so that the
+// dV, dK and dQ products include it (its dlambda term is the row pass's).
 template <bool DIAG, int SW>
 __device__ __forceinline__ void ew_chunk(const uint32_t (&U)[32], const uint32_t (&G)[32],
                                          const float* st, int qt0, int t, const EwConst& k,
-                                         uint32_t (&pk)[16], uint32_t (&dk)[16], float2& dl2) {
+                                         float2 self2, uint32_t (&pk)[16], uint32_t (&dk)[16],
+                                         float2& dl2) {
   const float2 ch2 = make_float2(k.ch, k.ch), c2k2 = make_float2(k.c2k, k.c2k);
   const float2 one2 = make_float2(1.f, 1.f);
 #pragma unroll
@@ -178,9 +184,15 @@ __device__ __forceinline__ void ew_chunk(const uint32_t (&U)[32], const uint32_t
       const float2 dR = __fmul2_rn(P, __fadd2_rn(g, nd));
       const float2 b = __ffma2_rn(make_float2(-h.x, -h.y), th, h);  // h (1 - t)
       const float2 sp = __ffma2_rn(a, b, a);                        // 2 SiLU'(u)
-      const float2 dS = __fmul2_rn(dR, sp);
+      float2 dS = __fmul2_rn(dR, sp);
       dl2 = __ffma2_rn(nw, dR, dl2);
-      pk[(c + e) >> 1] = pack_bf16x2(P.x, P.y);
+      float2 Pv = P;
+      if (DIAG) {
+        const int q = qt0 + c + e;
+        if (q == t) { Pv.x = self2.x; dS.x = 2.0f * self2.y; }
+        if (q + 1 == t) { Pv.y = self2.x; dS.y = 2.0f * self2.y; }
+      }
+      pk[(c + e) >> 1] = pack_bf16x2(Pv.x, Pv.y);
       dk[(c + e) >> 1] = pack_bf16x2(dS.x, dS.y);
     }
   }
@@ -205,16 +217,37 @@ __global__ void __launch_bounds__(kThreads, 1)
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int BH = p.B * p.H;
-  const int kt = (int)(blockIdx.x / BH);  // key tiles with the most query tiles first
-  const int bh = (int)(blockIdx.x % BH);
-  const int b = bh / p.H, h = bh % p.H;
-  const int k0 = kt * BK;
-  const int n_i = n_t - kt;                   // query tiles kt .. n_t - 1
-  const int total = n_i * C::SPT;             // steps
-  const int n_units = C::HALF ? total : n_i;  // Q / dO stage loads
+  const int n_work = n_t * BH;  // work units (key tile, head), most query tiles first
+  // A unit: keys kt * 128 .. of head bh, query tiles kt .. n_t - 1.  Round r of the grid
+  // takes units r G .. r G + G - 1 (G = gridDim.x), CTA c the unit r G + c in even rounds
+  // and r G + G - 1 - c in odd ones: the units come heaviest first, so the zigzag evens
+  // out the CTAs' work.  Every role walks the same sequence and keeps running counts
+  // (units, steps, Q / dO stage loads, query tiles) from which the barrier phases follow.
+  auto unit_at = [&](int r) -> int {
+    const int c = (r & 1) ? (int)(gridDim.x - 1 - blockIdx.x) : (int)blockIdx.x;
+    return r * (int)gridDim.x + c;
+  };
+  struct Unit {
+    int kt, bh, b, h, k0, n_i, total, n_units;
+  };
+  auto unit = [&](int w) {
+    Unit u;
+    u.kt = w / BH;
+    u.bh = w % BH;
+    u.b = u.bh / p.H;
+    u.h = u.bh % p.H;
+    u.k0 = u.kt * BK;
+    u.n_i = n_t - u.kt;
+    u.total = u.n_i * C::SPT;
+    u.n_units = C::HALF ? u.total : u.n_i;
+    return u;
+  };
 
   if (threadIdx.x == 0) {
-    mbar_init(bar(B_KV), 1);
+    for (int k = 0; k < C::NKV; ++k) {
+      mbar_init(bar(kv_full(k)), 1);
+      mbar_init(bar(B_KVE + k), 1);
+    }
     for (int s = 0; s < C::NQS; ++s) {
       mbar_init(bar(B_QF + s), 1);
       mbar_init(bar(B_QE + s), 1);
@@ -226,6 +259,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       mbar_init(bar(B_DQE + s), 128);
     }
     mbar_init(bar(B_ACC), 1);
+    mbar_init(bar(B_STG), 256);
     *abort_flag = 0;
     fence_mbar_init();
   }
@@ -245,28 +279,23 @@ __global__ void __launch_bounds__(kThreads, 1)
       tma_prefetch_desc(&tmG);
       tma_prefetch_desc(&tmDK);
       tma_prefetch_desc(&tmDV);
-      mbar_arrive_expect_tx(bar(B_KV), 2 * C::KVT);
-      for (int kb = 0; kb < C::KB; ++kb) {
-        tma_load_4d(sb + C::OFF_K + kb * 16384, &tmK, bar(B_KV), kb * 64, k0, h, b);
-        tma_load_4d(sb + C::OFF_V + kb * 16384, &tmV, bar(B_KV), kb * 64, k0, h, b);
-      }
-    }
-    int issued = 0;
-    if (lane == 0) {
-      for (int u = 0; u < n_units; ++u) {
-        const int s = u % C::NQS, r = u / C::NQS;
-        if (r > 0 && !mbar_wait(bar(B_QE + s), (r - 1) & 1, ab)) break;
+      bool ok = true;
+      int ul = 0, gq0 = 0, kv_issued = 0, q_issued = 0;
+      // Q / dO stage load g (global count) for local unit u of U
+      auto load_q = [&](const Unit& U, int u) -> bool {
+        const int g = gq0 + u, s = g % C::NQS, r = g / C::NQS;
+        if (r > 0 && !mbar_wait(bar(B_QE + s), (r - 1) & 1, ab)) return false;
         const int tile = C::HALF ? u / C::SPT : u;
         const int qoff = C::HALF ? (u % C::SPT) * C::QW : 0;
-        const int qi0 = (kt + tile) * BT + qoff;
+        const int qi0 = (U.kt + tile) * BT + qoff;
         mbar_arrive_expect_tx(bar(B_QF + s), 2 * C::QSZ + C::STB);
         for (int kb = 0; kb < C::KB; ++kb) {
           tma_load_4d(sb + C::OFF_Q + s * C::QSZ + kb * C::KBQ, &tmQ, bar(B_QF + s), kb * 64,
-                      qi0, h, b);
+                      qi0, U.h, U.b);
           tma_load_4d(sb + C::OFF_DO + s * C::QSZ + kb * C::KBQ, &tmG, bar(B_QF + s), kb * 64,
-                      qi0, h, b);
+                      qi0, U.h, U.b);
         }
-        const float* src = ws.stats + ((long long)bh * n_t + kt + tile) * 3 * BT + qoff;
+        const float* src = ws.stats + ((long long)U.bh * n_t + U.kt + tile) * 3 * BT + qoff;
         if (C::HALF) {
           for (int a = 0; a < 3; ++a)
             bulk_load(sb + C::OFF_STAT + s * C::STB + a * C::SW * 4, src + a * BT, C::SW * 4,
@@ -274,13 +303,34 @@ __global__ void __launch_bounds__(kThreads, 1)
         } else {
           bulk_load(sb + C::OFF_STAT + s * C::STB, src, C::STB, bar(B_QF + s));
         }
-        issued = u + 1;
+        q_issued = g + 1;
+        return true;
+      };
+      for (int w; ok && (w = unit_at(ul)) < n_work; ++ul) {
+        const Unit U = unit(w);
+        // K / V into buffer ul % NKV once the last MMA of the unit that used it before
+        // (unit ul - NKV) has completed; with two buffers this load overlaps the previous
+        // unit's work
+        const int kvb = ul % C::NKV;
+        const uint32_t kvs = sb + C::OFF_KV + kvb * 2 * C::KVT;
+        if (ul >= C::NKV && !(ok = mbar_wait(bar(B_KVE + kvb), ((ul - C::NKV) / C::NKV) & 1, ab)))
+          break;
+        mbar_arrive_expect_tx(bar(kv_full(kvb)), 2 * C::KVT);
+        for (int kb = 0; kb < C::KB; ++kb) {
+          tma_load_4d(kvs + kb * 16384, &tmK, bar(kv_full(kvb)), kb * 64, U.k0, U.h, U.b);
+          tma_load_4d(kvs + C::KVT + kb * 16384, &tmV, bar(kv_full(kvb)), kb * 64, U.k0, U.h, U.b);
+        }
+        ++kv_issued;
+        for (int u = 0; ok && u < U.n_units; ++u) ok = load_q(U, u);
+        gq0 += U.n_units;
       }
-    }
-    if (lane == 0 && ab.raised()) {
-      drain_wait(bar(B_KV), 0);
-      for (int i = issued - C::NQS > 0 ? issued - C::NQS : 0; i < issued; ++i)
-        drain_wait(bar(B_QF + i % C::NQS), (i / C::NQS) & 1);
+      if (ab.raised()) {
+        // let copies already in flight land before the CTA releases its shared memory
+        for (int k = kv_issued - C::NKV > 0 ? kv_issued - C::NKV : 0; k < kv_issued; ++k)
+          drain_wait(bar(kv_full(k % C::NKV)), (k / C::NKV) & 1);
+        for (int g = q_issued - C::NQS > 0 ? q_issued - C::NQS : 0; g < q_issued; ++g)
+          drain_wait(bar(B_QF + g % C::NQS), (g / C::NQS) & 1);
+      }
     }
   } else if (warp == W_MMA) {
     // ------------------------------------------------------ MMA issuer
@@ -289,12 +339,23 @@ __global__ void __launch_bounds__(kThreads, 1)
       constexpr uint32_t id_acc = idesc_bf16_f32(128, D, false, true);     // dV, dK
       constexpr uint32_t id_dq = C::HALF ? idesc_bf16_f32(128, C::QW, true, true)  // dQ^T
                                          : idesc_bf16_f32(128, D, true, true);     // dQ
-      bool ok = mbar_wait(bar(B_KV), 0, ab);
-      // U^T of step s into buffer s % NBUF (waits for its Q / dO stage)
-      auto issue_u = [&](int s) -> bool {
-        const int u = C::unit_of(s), st = u % C::NQS, bb = s % C::NBUF, hh = s % C::SPT;
+      bool ok = true;
+      bool acc_done = false;  // B_ACC of the current unit committed
+      // A unit's running offsets (steps, Q / dO stage loads) and its K / V tiles
+      struct Ctx {
+        int gs0, gq0;
+        uint32_t ks, vs;
+      };
+      auto ctx_of = [&](int ul_, int gs0_, int gq0_) {
+        const uint32_t k = sb + C::OFF_KV + (ul_ % C::NKV) * 2 * C::KVT;
+        return Ctx{gs0_, gq0_, k, k + C::KVT};
+      };
+      // U^T of step s into buffer (gs0 + s) % NBUF (waits for its Q / dO stage)
+      auto issue_u = [&](const Ctx& x, int s) -> bool {
+        const int g = x.gq0 + C::unit_of(s), st = g % C::NQS, bb = (x.gs0 + s) % C::NBUF;
+        const int hh = s % C::SPT;
         if (C::HALF || hh == 0) {
-          if (!mbar_wait(bar(B_QF + st), (u / C::NQS) & 1, ab)) return false;
+          if (!mbar_wait(bar(B_QF + st), (g / C::NQS) & 1, ab)) return false;
           tc_fence_after();
         }
         const uint32_t rows = C::HALF ? 0u : (uint32_t)(hh * C::QW * 128);  // the step's rows
@@ -302,105 +363,141 @@ __global__ void __launch_bounds__(kThreads, 1)
         for (int kk = 0; kk < D / 16; ++kk) {
           const uint32_t kof = (kk >> 2) * 16384 + (kk & 3) * 32;
           const uint32_t qof = (kk >> 2) * C::KBQ + (kk & 3) * 32;
-          mma_ss(tmem + C::col_u(bb), smem_desc_sw128(sb + C::OFF_K + kof, 16, 1024),
+          mma_ss(tmem + C::col_u(bb), smem_desc_sw128(x.ks + kof, 16, 1024),
                  smem_desc_sw128(sb + C::OFF_Q + st * C::QSZ + rows + qof, 16, 1024), id_s,
                  kk > 0 ? 1u : 0u);
         }
         return true;
       };
       // dP^T of step s (after issue_u(s)), then the step's S barrier
-      auto issue_dp = [&](int s) {
-        const int st = C::unit_of(s) % C::NQS, bb = s % C::NBUF, hh = s % C::SPT;
+      auto issue_dp = [&](const Ctx& x, int s) {
+        const int st = (x.gq0 + C::unit_of(s)) % C::NQS, bb = (x.gs0 + s) % C::NBUF;
+        const int hh = s % C::SPT;
         const uint32_t rows = C::HALF ? 0u : (uint32_t)(hh * C::QW * 128);
 #pragma unroll
         for (int kk = 0; kk < D / 16; ++kk) {
           const uint32_t kof = (kk >> 2) * 16384 + (kk & 3) * 32;
           const uint32_t qof = (kk >> 2) * C::KBQ + (kk & 3) * 32;
-          mma_ss(tmem + C::col_g(bb), smem_desc_sw128(sb + C::OFF_V + kof, 16, 1024),
+          mma_ss(tmem + C::col_g(bb), smem_desc_sw128(x.vs + kof, 16, 1024),
                  smem_desc_sw128(sb + C::OFF_DO + st * C::QSZ + rows + qof, 16, 1024), id_s,
                  kk > 0 ? 1u : 0u);
         }
         mma_commit(bar(B_S + bb));
       };
-      // d_h = 64: U^T / dP^T of step sn may be issued once its buffer is free (step
-      // sn - NBUF done) and once the GEMM that releases the Q/dO stage it loads into has
-      // been issued: waiting for that stage's load earlier would deadlock.
-      int sn = 0, units_done = 0;
-      bool acc_done = false;  // B_ACC committed
-      while (ok && sn < total && sn < C::NBUF) {
-        ok = issue_u(sn);
-        if (ok) issue_dp(sn);
-        ++sn;
-      }
-      for (int s = 0; ok && s < total; ++s) {
-        const int t = s / C::SPT, hh = s % C::SPT, bb = s % C::NBUF;
-        const int st = C::unit_of(s) % C::NQS;
-        if (!(ok = mbar_wait(bar(B_P + bb), (s / C::NBUF) & 1, ab))) break;
-        tc_fence_after();
-        // dV += P^T dO and dK += dS'^T Q with the A operands in TMEM: every 32-query chunk
-        // keeps its 16 packed columns of P (dS') at the start of its own U^T (dP^T) columns.
-        const uint32_t pcol = C::col_u(bb), dcol = C::col_g(bb);
-        const uint32_t rows = C::HALF ? 0u : (uint32_t)(hh * C::QW * 128);
-#pragma unroll
-        for (int kk = 0; kk < C::QW / 16; ++kk) {
-          const uint32_t acol = (kk >> 1) * 32 + (kk & 1) * 8;
-          mma_ts(tmem + C::COL_DV, tmem + pcol + acol,
-                 smem_desc_sw128(sb + C::OFF_DO + st * C::QSZ + rows + kk * 2048, C::KBQ, 1024),
-                 id_acc, (s > 0 || kk > 0) ? 1u : 0u);
-        }
-#pragma unroll
-        for (int kk = 0; kk < C::QW / 16; ++kk) {
-          const uint32_t acol = (kk >> 1) * 32 + (kk & 1) * 8;
-          mma_ts(tmem + C::COL_DK, tmem + dcol + acol,
-                 smem_desc_sw128(sb + C::OFF_Q + st * C::QSZ + rows + kk * 2048, C::KBQ, 1024),
-                 id_acc, (s > 0 || kk > 0) ? 1u : 0u);
-        }
-        if (s == total - 1) {  // dK and dV are final: the epilogue need not wait for dQ
-          mma_commit(bar(B_ACC));
-          acc_done = true;
-        }
-        if (C::HALF) {
-          mma_commit(bar(B_QE + st));  // the step's Q / dO rows are no longer needed
-          // Buffer bb next holds step s + 2.  Issue order (executed in order): dQ^T of step
-          // s over dS' in the dP^T columns, which dK has read; U^T of step s + 2 over P,
-          // which dV has read; dP^T of step s + 2 once dQ^T has been read out.
-          // dQ^T = K^T dS'^T (A = K tile, d-major; B = the step's dS', query-major)
-          const uint32_t dsb = sb + C::OFF_DS + (s & 1) * C::DSZ;
-#pragma unroll
-          for (int kk = 0; kk < BK / 16; ++kk)
-            mma_ss(tmem + C::col_g(bb), smem_desc_sw128(sb + C::OFF_K + kk * 2048, 16384, 1024),
-                   smem_desc_sw128(dsb + kk * 2048, 16384, 1024), id_dq, kk > 0 ? 1u : 0u);
-          mma_commit(bar(B_DQF + bb));
-          const int s2 = s + C::NBUF;
-          if (s2 < total && !(ok = issue_u(s2))) break;
-          if (s2 < total) {
-            if (!(ok = mbar_wait(bar(B_DQE + bb), (s / C::NBUF) & 1, ab))) break;
-            tc_fence_after();
-            issue_dp(s2);
-          }
-          continue;
-        }
-        if (hh == C::SPT - 1) {
-          if (t > 0) {  // dQ_{t-1} has been read out of TMEM
-            if (!(ok = mbar_wait(bar(B_DQE), (t - 1) & 1, ab))) break;
-            tc_fence_after();
-          }
-          // dQ_t = dS' K   (A = dS', queries x keys, M-major; B = K tile, N-major)
-          const uint32_t ds_base = sb + C::OFF_DS + (t & 1) * C::DSZ;
-#pragma unroll
-          for (int kk = 0; kk < BK / 16; ++kk)
-            mma_ss(tmem + C::COL_DQ, smem_desc_sw128(ds_base + kk * 2048, 16384, 1024),
-                   smem_desc_sw128(sb + C::OFF_K + kk * 2048, 16384, 1024), id_dq,
-                   kk > 0 ? 1u : 0u);
-          mma_commit(bar(B_DQF));
-          mma_commit(bar(B_QE + st));
-          ++units_done;
-        }
-        while (ok && sn < total && sn <= s + C::NBUF && C::unit_of(sn) - C::NQS < units_done) {
-          ok = issue_u(sn);
-          if (ok) issue_dp(sn);
+      int ul = 0, gs0 = 0, gq0 = 0, gt0 = 0;
+      int pre = 0;  // steps of the current unit issued ahead by the previous unit
+      for (int w; ok && (w = unit_at(ul)) < n_work; ++ul) {
+        const Unit U = unit(w);
+        const int total = U.total;
+        acc_done = false;
+        const int kvb = ul % C::NKV;
+        const Ctx x = ctx_of(ul, gs0, gq0);
+        const uint32_t ks = x.ks;
+        if (pre == 0 && !(ok = mbar_wait(bar(kv_full(kvb)), (ul / C::NKV) & 1, ab))) break;
+        // d_h = 64: U^T / dP^T of step sn may be issued once its buffer is free (step
+        // sn - NBUF done) and once the GEMM that releases the Q/dO stage it loads into has
+        // been issued: waiting for that stage's load earlier would deadlock.
+        int sn = pre, units_done = 0;
+        pre = 0;
+        while (ok && sn < total && sn < C::NBUF) {
+          ok = issue_u(x, sn);
+          if (ok) issue_dp(x, sn);
           ++sn;
         }
+        for (int s = 0; ok && s < total; ++s) {
+          const int t = s / C::SPT, hh = s % C::SPT, g = gs0 + s, bb = g % C::NBUF;
+          const int st = (gq0 + C::unit_of(s)) % C::NQS;
+          if (!(ok = mbar_wait(bar(B_P + bb), (g / C::NBUF) & 1, ab))) break;
+          tc_fence_after();
+          // dV += P^T dO and dK += dS'^T Q with the A operands in TMEM: every 32-query chunk
+          // keeps its 16 packed columns of P (dS') at the start of its own U^T (dP^T)
+          // columns.  The first step of a unit starts the sums afresh; the epilogue has
+          // read the previous unit's sums before its warps finished this step (B_P).
+          const uint32_t pcol = C::col_u(bb), dcol = C::col_g(bb);
+          const uint32_t rows = C::HALF ? 0u : (uint32_t)(hh * C::QW * 128);
+#pragma unroll
+          for (int kk = 0; kk < C::QW / 16; ++kk) {
+            const uint32_t acol = (kk >> 1) * 32 + (kk & 1) * 8;
+            mma_ts(tmem + C::COL_DV, tmem + pcol + acol,
+                   smem_desc_sw128(sb + C::OFF_DO + st * C::QSZ + rows + kk * 2048, C::KBQ, 1024),
+                   id_acc, (s > 0 || kk > 0) ? 1u : 0u);
+          }
+#pragma unroll
+          for (int kk = 0; kk < C::QW / 16; ++kk) {
+            const uint32_t acol = (kk >> 1) * 32 + (kk & 1) * 8;
+            mma_ts(tmem + C::COL_DK, tmem + dcol + acol,
+                   smem_desc_sw128(sb + C::OFF_Q + st * C::QSZ + rows + kk * 2048, C::KBQ, 1024),
+                   id_acc, (s > 0 || kk > 0) ? 1u : 0u);
+          }
+          if (s == total - 1) {  // dK and dV are final: the epilogue need not wait for dQ
+            mma_commit(bar(B_ACC));
+            acc_done = true;
+            // d_h = 64: the next unit's first steps go ahead of this unit's last dQ (their
+            // buffers were read by the dV / dK just issued; its K / V came in beforehand)
+            const int wn = C::HALF ? n_work : unit_at(ul + 1);
+            if (wn < n_work) {
+              const Unit N = unit(wn);
+              if (!(ok = mbar_wait(bar(kv_full((ul + 1) % C::NKV)), ((ul + 1) / C::NKV) & 1, ab)))
+                break;
+              const Ctx xn = ctx_of(ul + 1, gs0 + total, gq0 + U.n_units);
+              while (ok && pre < N.total && pre < C::NBUF) {
+                ok = issue_u(xn, pre);
+                if (ok) issue_dp(xn, pre);
+                ++pre;
+              }
+              if (!ok) break;
+            }
+          }
+          if (C::HALF) {
+            mma_commit(bar(B_QE + st));  // the step's Q / dO rows are no longer needed
+            // Buffer bb next holds step s + 2.  Issue order (executed in order): dQ^T of
+            // step s over dS' in the dP^T columns, which dK has read; U^T of step s + 2
+            // over P, which dV has read; dP^T of step s + 2 once dQ^T has been read out.
+            // dQ^T = K^T dS'^T (A = K tile, d-major; B = the step's dS', query-major)
+            const uint32_t dsb = sb + C::OFF_DS + (g & 1) * C::DSZ;
+#pragma unroll
+            for (int kk = 0; kk < BK / 16; ++kk)
+              mma_ss(tmem + C::col_g(bb), smem_desc_sw128(ks + kk * 2048, 16384, 1024),
+                     smem_desc_sw128(dsb + kk * 2048, 16384, 1024), id_dq, kk > 0 ? 1u : 0u);
+            mma_commit(bar(B_DQF + bb));
+            const int s2 = s + C::NBUF;
+            if (s2 < total && !(ok = issue_u(x, s2))) break;
+            if (s2 < total) {
+              if (!(ok = mbar_wait(bar(B_DQE + bb), (g / C::NBUF) & 1, ab))) break;
+              tc_fence_after();
+              issue_dp(x, s2);
+            }
+            continue;
+          }
+          if (hh == C::SPT - 1) {
+            const int gt = gt0 + t;
+            if (gt > 0) {  // dQ of the previous query tile has been read out of TMEM
+              if (!(ok = mbar_wait(bar(B_DQE), (gt - 1) & 1, ab))) break;
+              tc_fence_after();
+            }
+            // dQ_t = dS' K   (A = dS', queries x keys, M-major; B = K tile, N-major)
+            const uint32_t ds_base = sb + C::OFF_DS + (gt & 1) * C::DSZ;
+#pragma unroll
+            for (int kk = 0; kk < BK / 16; ++kk)
+              mma_ss(tmem + C::COL_DQ, smem_desc_sw128(ds_base + kk * 2048, 16384, 1024),
+                     smem_desc_sw128(ks + kk * 2048, 16384, 1024), id_dq,
+                     kk > 0 ? 1u : 0u);
+            mma_commit(bar(B_DQF));
+            mma_commit(bar(B_QE + st));
+            ++units_done;
+          }
+          while (ok && sn < total && sn <= s + C::NBUF &&
+                 C::unit_of(sn) - C::NQS < units_done) {
+            ok = issue_u(x, sn);
+            if (ok) issue_dp(x, sn);
+            ++sn;
+          }
+        }
+        if (!ok) break;
+        mma_commit(bar(B_KVE + kvb));  // every MMA of the unit (K / V buffer free) done
+        gs0 += total;
+        gq0 += U.n_units;
+        gt0 += U.n_i;
       }
       if (!acc_done) mma_commit(bar(B_ACC));  // after an abort: whatever completed
     }
@@ -411,74 +508,81 @@ __global__ void __launch_bounds__(kThreads, 1)
     const uint32_t trow = tmem + ((uint32_t)(quad * 32) << 16);
     const uint32_t stage0 = sb + C::OFF_DQS + quad * C::DQSLOTS * 4096;
     uint8_t* stage0p = smem + C::OFF_DQS + quad * C::DQSLOTS * 4096;
-    if (C::HALF) {
-      // TMEM lanes are d indices here: this warp holds d = 32 quad .. 32 quad + 31 of the
-      // step's 64 queries and writes them as 32-query x 32-d boxes, transposed.
-      for (int s = 0; s < total; ++s) {
-        const int bb = s % C::NBUF;
-        const bool ok = __all_sync(0xffffffffu, mbar_wait(bar(B_DQF + bb), (s / C::NBUF) & 1, ab));
-        if (!ok) break;
-        tc_fence_after();
-        uint32_t z[64];
-        tmem_ld32(trow + C::col_g(bb), z);
-        tmem_ld32(trow + C::col_g(bb) + 32, z + 32);
-        tmem_ld_wait();
-        tc_fence_before();
-        mbar_arrive(bar(B_DQE + bb));  // the buffer may take the next dP^T
-        const int row0 = bh * t_pad + (kt + s / C::SPT) * BT + (s % C::SPT) * C::QW;
-        const uint32_t sw = (uint32_t)(lane & 3) << 2;
-#pragma unroll
-        for (int c = 0; c < 2; ++c) {
-          if (lane == 0) bulk_wait_read_0();  // the slot's previous reduce has read it
-          __syncwarp();
-#pragma unroll
-          for (int q = 0; q < 32; ++q)
-            *reinterpret_cast<uint32_t*>(stage0p + q * 128 + (((lane >> 2) ^ (q & 7)) << 4) +
-                                         sw) = z[c * 32 + q];
-          fence_async_smem();
-          __syncwarp();
-          if (lane == 0) {
-            tma_reduce_add_2d(&tmDQ, stage0, quad * 32, row0 + c * 32);
-            tma_store_commit();
-          }
-        }
-      }
-    } else {
-      int chunk = 0;
-      for (int i = 0; i < n_i; ++i) {
-        const bool ok = __all_sync(0xffffffffu, mbar_wait(bar(B_DQF), i & 1, ab));
-        if (!ok) break;
-        tc_fence_after();
-        const int row0 = bh * t_pad + (kt + i) * BT + quad * 32;
-#pragma unroll
-        for (int c64 = 0; c64 < D; c64 += 64) {
+    bool ok = true;
+    int gs0 = 0, gt0 = 0, chunk = 0;
+    for (int r = 0, w; ok && (w = unit_at(r)) < n_work; ++r) {
+      const Unit U = unit(w);
+      if (C::HALF) {
+        // TMEM lanes are d indices here: this warp holds d = 32 quad .. 32 quad + 31 of the
+        // step's 64 queries and writes them as 32-query x 32-d boxes, transposed.
+        for (int s = 0; s < U.total; ++s) {
+          const int g = gs0 + s, bb = g % C::NBUF;
+          ok = __all_sync(0xffffffffu, mbar_wait(bar(B_DQF + bb), (g / C::NBUF) & 1, ab));
+          if (!ok) break;
+          tc_fence_after();
           uint32_t z[64];
-          tmem_ld32(trow + C::COL_DQ + c64, z);
-          tmem_ld32(trow + C::COL_DQ + c64 + 32, z + 32);
+          tmem_ld32(trow + C::col_g(bb), z);
+          tmem_ld32(trow + C::col_g(bb) + 32, z + 32);
           tmem_ld_wait();
-          if (c64 + 64 == D) {
-            tc_fence_before();
-            mbar_arrive(bar(B_DQE));  // TMEM columns free for the next dQ
-          }
+          tc_fence_before();
+          mbar_arrive(bar(B_DQE + bb));  // the buffer may take the next dP^T
+          const int row0 = U.bh * t_pad + (U.kt + s / C::SPT) * BT + (s % C::SPT) * C::QW;
+          const uint32_t sw = (uint32_t)(lane & 3) << 2;
 #pragma unroll
-          for (int c0 = 0; c0 < 64; c0 += 32, ++chunk) {
-            const int slot = chunk & 1;
-            if (lane == 0) bulk_wait_read_le1();  // the slot's previous reduce has read it
+          for (int c = 0; c < 2; ++c) {
+            if (lane == 0) bulk_wait_read_0();  // the slot's previous reduce has read it
             __syncwarp();
-            uint8_t* row = stage0p + slot * 4096 + lane * 128;
 #pragma unroll
-            for (int k = 0; k < 8; ++k)
-              *reinterpret_cast<uint4*>(row + ((k ^ (lane & 7)) << 4)) =
-                  make_uint4(z[c0 + 4 * k], z[c0 + 4 * k + 1], z[c0 + 4 * k + 2], z[c0 + 4 * k + 3]);
+            for (int q = 0; q < 32; ++q)
+              *reinterpret_cast<uint32_t*>(stage0p + q * 128 + (((lane >> 2) ^ (q & 7)) << 4) +
+                                           sw) = z[c * 32 + q];
             fence_async_smem();
             __syncwarp();
             if (lane == 0) {
-              tma_reduce_add_2d(&tmDQ, stage0 + slot * 4096, c64 + c0, row0);
+              tma_reduce_add_2d(&tmDQ, stage0, quad * 32, row0 + c * 32);
               tma_store_commit();
             }
           }
         }
+      } else {
+        for (int i = 0; i < U.n_i; ++i) {
+          const int gt = gt0 + i;
+          ok = __all_sync(0xffffffffu, mbar_wait(bar(B_DQF), gt & 1, ab));
+          if (!ok) break;
+          tc_fence_after();
+          const int row0 = U.bh * t_pad + (U.kt + i) * BT + quad * 32;
+#pragma unroll
+          for (int c64 = 0; c64 < D; c64 += 64) {
+            uint32_t z[64];
+            tmem_ld32(trow + C::COL_DQ + c64, z);
+            tmem_ld32(trow + C::COL_DQ + c64 + 32, z + 32);
+            tmem_ld_wait();
+            if (c64 + 64 == D) {
+              tc_fence_before();
+              mbar_arrive(bar(B_DQE));  // TMEM columns free for the next dQ
+            }
+#pragma unroll
+            for (int c0 = 0; c0 < 64; c0 += 32, ++chunk) {
+              const int slot = chunk % C::DQSLOTS;
+              if (lane == 0) bulk_wait_read_0();  // the slot's previous reduce has read it
+              __syncwarp();
+              uint8_t* row = stage0p + slot * 4096 + lane * 128;
+#pragma unroll
+              for (int k = 0; k < 8; ++k)
+                *reinterpret_cast<uint4*>(row + ((k ^ (lane & 7)) << 4)) =
+                    make_uint4(z[c0 + 4 * k], z[c0 + 4 * k + 1], z[c0 + 4 * k + 2], z[c0 + 4 * k + 3]);
+              fence_async_smem();
+              __syncwarp();
+              if (lane == 0) {
+                tma_reduce_add_2d(&tmDQ, stage0 + slot * 4096, c64 + c0, row0);
+                tma_store_commit();
+              }
+            }
+          }
+        }
       }
+      gs0 += U.total;
+      gt0 += U.n_i;
     }
     if (lane == 0) tma_store_wait_read_all();  // the staging reads; the adds finish with the kernel
   } else {
@@ -486,82 +590,86 @@ __global__ void __launch_bounds__(kThreads, 1)
     // Both warpgroups work on every step: warpgroup wg takes its 32 query columns.
     const int wg = warp >> 2;                  // 0 or 1
     const int t = (warp & 3) * 32 + lane;      // key k0 + t, TMEM lane t
-    const uint32_t trow = tmem + ((uint32_t)((warp & 3) * 32) << 16);
+    const int wq = warp & 3;
+    const uint32_t trow = tmem + ((uint32_t)(wq * 32) << 16);
     const float isd = p.inv_sqrt_d;
     EwConst kc;
     kc.ch = 0.5f * isd;
     kc.c2k = kc.ch * kLog2e;
-    const int key_g = k0 + t;
     float2 dl2 = make_float2(0.f, 0.f);
     bool ok = true;
-    for (int s = 0; s < total; ++s) {
-      const int bb = s % C::NBUF, i = s / C::SPT, hh = s % C::SPT;
-      const int u = C::unit_of(s), st = u % C::NQS;
-      ok = __all_sync(0xffffffffu, mbar_wait(bar(B_S + bb), (s / C::NBUF) & 1, ab));
+    int ul = 0, gs0 = 0, gq0 = 0, gt0 = 0;
+    for (int w; ok && (w = unit_at(ul)) < n_work; ++ul) {
+      const Unit U = unit(w);
+      // The Self entry of this thread's key (row pass), placed on the diagonal tile's
+      // diagonal; keys past T read a clamped row (their products are never stored).
+      const long long self_row = (long long)U.bh * p.T + min(U.k0 + t, p.T - 1);
+      const float2 self2 = make_float2(ws.F_self[self_row], ws.dS_self[self_row]);
+      for (int s = 0; s < U.total; ++s) {
+        const int g = gs0 + s, bb = g % C::NBUF, i = s / C::SPT, hh = s % C::SPT;
+        const int gu = gq0 + C::unit_of(s), st = gu % C::NQS;
+        ok = __all_sync(0xffffffffu, mbar_wait(bar(B_S + bb), (g / C::NBUF) & 1, ab));
+        if (!ok) break;
+        tc_fence_after();
+        // acquire the producer's per-query scalars of this stage (already complete)
+        ok = __all_sync(0xffffffffu, mbar_wait(bar(B_QF + st), (gu / C::NQS) & 1, ab));
+        if (!ok) break;
+        const float* sts = reinterpret_cast<const float*>(smem + C::OFF_STAT + st * C::STB);
+        const int cl = wg * 32;             // the chunk's first column within the step
+        const int qt0 = hh * C::QW + cl;    // tile-local query index
+        uint32_t U_[32], G[32];
+        tmem_ld32(trow + C::col_u(bb) + cl, U_);
+        tmem_ld32(trow + C::col_g(bb) + cl, G);
+        tmem_ld_wait();
+        uint32_t pk[16], dk[16];
+        const float* stc = sts + (C::HALF ? cl : qt0);
+        if (i == 0)
+          ew_chunk<true, C::SW>(U_, G, stc, qt0, t, kc, self2, pk, dk, dl2);
+        else
+          ew_chunk<false, C::SW>(U_, G, stc, qt0, t, kc, self2, pk, dk, dl2);
+        tmem_st16(trow + C::col_u(bb) + cl, pk);  // P   (A operand of dV += P^T dO)
+        tmem_st16(trow + C::col_g(bb) + cl, dk);  // dS' (A operand of dK += dS'^T Q)
+        if (s == 0 && ul > 0) {
+          // the previous unit's dK / dV staging, in the dS' buffer written next, has been
+          // read by the stores of all eight warps
+          if (lane == 0) tma_store_wait_read_all();
+          __syncwarp();
+          mbar_arrive(bar(B_STG));
+          ok = __all_sync(0xffffffffu, mbar_wait(bar(B_STG), (ul - 1) & 1, ab));
+          if (!ok) break;
+        }
+        // dS' row t (key), 32 queries, into the 128-byte-swizzled query-major layout the
+        // dQ product reads: 64-query blocks of 128 key rows
+        uint8_t* ds_row = C::HALF ? smem + C::OFF_DS + (g & 1) * C::DSZ + t * 128
+                                  : smem + C::OFF_DS + ((gt0 + i) & 1) * C::DSZ +
+                                        (qt0 >> 6) * 16384 + t * 128;
+        const int cb = (qt0 & 63) >> 3;
+#pragma unroll
+        for (int qd = 0; qd < 4; ++qd)
+          *reinterpret_cast<uint4*>(ds_row + (((cb + qd) ^ (t & 7)) << 4)) =
+              make_uint4(dk[4 * qd], dk[4 * qd + 1], dk[4 * qd + 2], dk[4 * qd + 3]);
+        tmem_st_wait();
+        fence_async_smem();
+        tc_fence_before();
+        mbar_arrive(bar(B_P + bb));
+      }
       if (!ok) break;
+      // -------------------------------------------------- dK (warpgroup 0) / dV (1)
+      // The sums over the unit's queries, Self entry included (diagonal of P and dS'):
+      //   dK_j = (sum_i dS'_ij q_i) / (2 sqrt d),   dV_j = sum_i P_ij dO_i
+      if (!(ok = __all_sync(0xffffffffu, mbar_wait(bar(B_ACC), ul & 1, ab)))) break;
       tc_fence_after();
-      // acquire the producer's per-query scalars of this stage (already complete)
-      ok = __all_sync(0xffffffffu, mbar_wait(bar(B_QF + st), (u / C::NQS) & 1, ab));
-      if (!ok) break;
-      const float* sts = reinterpret_cast<const float*>(smem + C::OFF_STAT + st * C::STB);
-      const int cl = wg * 32;             // the chunk's first column within the step
-      const int qt0 = hh * C::QW + cl;    // tile-local query index
-      uint32_t U[32], G[32];
-      tmem_ld32(trow + C::col_u(bb) + cl, U);
-      tmem_ld32(trow + C::col_g(bb) + cl, G);
-      tmem_ld_wait();
-      uint32_t pk[16], dk[16];
-      const float* stc = sts + (C::HALF ? cl : qt0);
-      if (i == 0)
-        ew_chunk<true, C::SW>(U, G, stc, qt0, t, kc, pk, dk, dl2);
-      else
-        ew_chunk<false, C::SW>(U, G, stc, qt0, t, kc, pk, dk, dl2);
-      tmem_st16(trow + C::col_u(bb) + cl, pk);  // P   (A operand of dV += P^T dO)
-      tmem_st16(trow + C::col_g(bb) + cl, dk);  // dS' (A operand of dK += dS'^T Q)
-      // dS' row t (key), 32 queries, into the 128-byte-swizzled query-major layout the dQ
-      // product reads: 64-query blocks of 128 key rows
-      uint8_t* ds_row = C::HALF ? smem + C::OFF_DS + (s & 1) * C::DSZ + t * 128
-                                : smem + C::OFF_DS + (i & 1) * C::DSZ + (qt0 >> 6) * 16384 +
-                                      t * 128;
-      const int cb = (qt0 & 63) >> 3;
-#pragma unroll
-      for (int qd = 0; qd < 4; ++qd)
-        *reinterpret_cast<uint4*>(ds_row + (((cb + qd) ^ (t & 7)) << 4)) =
-            make_uint4(dk[4 * qd], dk[4 * qd + 1], dk[4 * qd + 2], dk[4 * qd + 3]);
-      tmem_st_wait();
-      fence_async_smem();
-      tc_fence_before();
-      mbar_arrive(bar(B_P + bb));
-    }
-    float dlam = dl2.x + dl2.y;
-    // ---------------------------------------------------- dK (warpgroup 0) / dV (1)
-    // Exchange sums from TMEM plus the Self entry of key j (from the row pass):
-    //   dK_j = (sum dS'_ij q_i) / (2 sqrt d) + dS_jj q_j / sqrt d
-    //   dV_j =  sum P_ij dO_i               + F_jj dO_j
-    // The Self operands (q_j or dO_j, and the scalar) are loaded before the wait for the
-    // last MMAs and first used after it: the loads carry no condition (rows past T and
-    // padding columns read a clamped address; their results are never stored).
-    const int jr = min(key_g, p.T - 1);
-    const __nv_bfloat16* srow_ptr =
-        reinterpret_cast<const __nv_bfloat16*>(wg == 0 ? p.q : p.dout) + (long long)b * p.sB +
-        (long long)h * p.sH + (long long)jr * p.sT;
-    uint4 rowv[D / 8];
-#pragma unroll
-    for (int c = 0; c < D / 8; ++c)
-      rowv[c] = *reinterpret_cast<const uint4*>(srow_ptr + min(8 * c, p.d - 8));
-    const float self_raw = wg == 0 ? ws.dS_self[(long long)bh * p.T + jr]
-                                   : ws.F_self[(long long)bh * p.T + jr];
-    if (ok) ok = __all_sync(0xffffffffu, mbar_wait(bar(B_ACC), 0, ab));
-    tc_fence_after();
-    if (ok) {
       const uint32_t col = wg == 0 ? C::COL_DK : C::COL_DV;
       const float sc = wg == 0 ? 0.5f * isd : 1.0f;
-      const float self = wg == 0 ? self_raw * isd : self_raw;
-      // Staged as 32 rows x D per warp (128-byte swizzle) in the Q (dK) or dO (dV) stages,
-      // which no MMA reads any more (B_ACC follows the last one that did), and written by
-      // TMA stores that clip rows past T and padding columns.
-      const int wq = warp & 3;
-      const uint32_t stg_off = (wg == 0 ? C::OFF_Q : C::OFF_DO) + wq * (32 * D * 2);
+      // Staged as 32 rows x D per warp (128-byte swizzle) and written by TMA stores that
+      // clip rows past T and padding columns.  d_h = 64: in the dS' buffer the next unit
+      // writes first (its last reader, the dQ of the tile before last, precedes B_ACC);
+      // d_h = 128 (one unit per CTA): in the Q (dK) and dO (dV) stages, which no MMA
+      // reads any more.
+      const uint32_t stg_off =
+          (C::HALF ? (wg == 0 ? C::OFF_Q : C::OFF_DO)
+                   : C::OFF_DS + ((gt0 + U.n_i) & 1) * C::DSZ + wg * (4 * 32 * D * 2)) +
+          wq * (32 * D * 2);
       uint8_t* stg = smem + stg_off + lane * 128;
 #pragma unroll
       for (int c0 = 0; c0 < D; c0 += 32) {
@@ -571,15 +679,11 @@ __global__ void __launch_bounds__(kThreads, 1)
         const int kb = c0 >> 6;  // 64-column block
 #pragma unroll
         for (int c8 = 0; c8 < 32; c8 += 8) {
-          const uint4 rv = rowv[(c0 + c8) / 8];
-          const uint32_t r4[4] = {rv.x, rv.y, rv.z, rv.w};
           uint32_t o4[4];
 #pragma unroll
-          for (int e = 0; e < 4; ++e) {
-            const float2 rf = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&r4[e]));
-            o4[e] = pack_bf16x2(fmaf(__uint_as_float(a[c8 + 2 * e]), sc, self * rf.x),
-                                fmaf(__uint_as_float(a[c8 + 2 * e + 1]), sc, self * rf.y));
-          }
+          for (int e = 0; e < 4; ++e)
+            o4[e] = pack_bf16x2(__uint_as_float(a[c8 + 2 * e]) * sc,
+                                __uint_as_float(a[c8 + 2 * e + 1]) * sc);
           const int chunk = ((c0 & 63) + c8) >> 3;  // 16-byte chunk within the 128-byte row
           *reinterpret_cast<uint4*>(stg + kb * (32 * 128) + ((chunk ^ (lane & 7)) << 4)) =
               make_uint4(o4[0], o4[1], o4[2], o4[3]);
@@ -591,12 +695,16 @@ __global__ void __launch_bounds__(kThreads, 1)
         const CUtensorMap* tm = wg == 0 ? &tmDK : &tmDV;
 #pragma unroll
         for (int kb = 0; kb < C::KB; ++kb)
-          tma_store_4d(tm, sb + stg_off + kb * (32 * 128), kb * 64, k0 + wq * 32, h, b);
-        tma_store_commit();
-        tma_store_wait_read_all();  // the staging must outlive the store's reads
+          tma_store_4d(tm, sb + stg_off + kb * (32 * 128), kb * 64, U.k0 + wq * 32, U.h, U.b);
+        tma_store_commit();  // its reads are awaited before the staging is written again
       }
       __syncwarp();
+      gs0 += U.total;
+      gq0 += U.n_units;
+      gt0 += U.n_i;
     }
+    if (lane == 0) tma_store_wait_read_all();  // the staging must outlive the store's reads
+    float dlam = dl2.x + dl2.y;
 #pragma unroll
     for (int o = 16; o > 0; o >>= 1) dlam += __shfl_xor_sync(0xffffffffu, dlam, o);
     if (lane == 0) red[warp] = dlam;
@@ -620,7 +728,7 @@ __global__ void __launch_bounds__(kThreads, 1)
 //   D_i = dO_i . Y_i,  g_ii = dO_i . v_i,  S_i = sigmoid(u_ii / tau_S),
 //   F_ii = exp(S_i - logZ_i) (the Self flow),
 //   Self entry: dR_ii = F_ii (g_ii - D_i),  dS_ii = dR_ii S_i (1 - S_i) / tau_S
-//   (F_self, dS_self for the epilogues) and its dlambda term log i (1 - F_ii) dR_ii
+//   (F_self, dS_self for the tile kernel's diagonal) and its dlambda term log i (1 - F_ii) dR_ii
 //   (one partial per block);
 // the per-query scalars of the tile kernel (three arrays per 128-row tile:
 // c2 = (-lambda log i - logZ_i) log2 e, -D_i, -log i F_ii) and a zeroed row of the fp32 dQ
@@ -710,9 +818,10 @@ __global__ void __launch_bounds__(256) pre_kernel(Problem p, BwdWorkspace ws, in
   }
 }
 
-// dq = bf16(dq_acc / (2 sqrt(d)) + dS_ii k_i / sqrt(d)) for rows < T (the Exchange sums
-// plus the Self entry); block 0 also reduces the dlambda partials of the row pass
-// (n_pre) and of the tile kernel (n_cta) in a fixed order (deterministic).
+// dq = bf16(dq_acc / (2 sqrt(d))) for rows < T (the accumulator holds the Exchange sums
+// and the Self entry, which the diagonal tile carries); block 0 also reduces the dlambda
+// partials of the row pass (n_pre) and of the tile kernel (n_cta) in a fixed order
+// (deterministic).
 template <int D>
 __global__ void __launch_bounds__(256) finalize_kernel(Problem p, BwdWorkspace ws, int n_pre,
                                                        int n_cta) {
@@ -741,18 +850,12 @@ __global__ void __launch_bounds__(256) finalize_kernel(Problem p, BwdWorkspace w
   const float4 a = *reinterpret_cast<const float4*>(src);
   const float4 c = *reinterpret_cast<const float4*>(src + 4);
   const long long off = (long long)b * p.sB + (long long)h * p.sH + (long long)r * p.sT + c8;
-  const uint4 kv = *reinterpret_cast<const uint4*>(reinterpret_cast<const __nv_bfloat16*>(p.k) + off);
   const float sc = 0.5f * p.inv_sqrt_d;
-  const float self = ws.dS_self[row] * p.inv_sqrt_d;
-  const float2 k0 = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&kv.x));
-  const float2 k1 = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&kv.y));
-  const float2 k2 = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&kv.z));
-  const float2 k3 = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&kv.w));
   uint4 o;
-  o.x = pack_bf16x2(fmaf(a.x, sc, self * k0.x), fmaf(a.y, sc, self * k0.y));
-  o.y = pack_bf16x2(fmaf(a.z, sc, self * k1.x), fmaf(a.w, sc, self * k1.y));
-  o.z = pack_bf16x2(fmaf(c.x, sc, self * k2.x), fmaf(c.y, sc, self * k2.y));
-  o.w = pack_bf16x2(fmaf(c.z, sc, self * k3.x), fmaf(c.w, sc, self * k3.y));
+  o.x = pack_bf16x2(a.x * sc, a.y * sc);
+  o.y = pack_bf16x2(a.z * sc, a.w * sc);
+  o.z = pack_bf16x2(c.x * sc, c.y * sc);
+  o.w = pack_bf16x2(c.z * sc, c.w * sc);
   *reinterpret_cast<uint4*>(reinterpret_cast<__nv_bfloat16*>(p.dq) + off) = o;
 }
 
@@ -779,14 +882,26 @@ static bool make_tmap_dq(CUtensorMap* m, float* base, int rows, int d) {
             CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
+// Tile-kernel CTAs.  d_h <= 64: persistent, one CTA per SM over the (key tile, head)
+// units; d_h = 128 stages dK / dV in its Q / dO stages and takes one unit per CTA.
+static long long tile_grid(const Problem& p) {
+  const long long units = (long long)((p.T + 127) / 128) * p.B * p.H;
+  if (p.d > 64) return units;
+  int dev = 0, nsm = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess ||
+      cudaDeviceGetAttribute(&nsm, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || nsm < 1)
+    return units;
+  return units < nsm ? units : nsm;
+}
+
 template <int D>
 static cudaError_t bwd_t(const Problem& p, const BwdWorkspace& ws, unsigned stages,
                          cudaStream_t s) {
   const int n_t = (p.T + 127) / 128;
   const int t_pad = ws.t_pad;
   const long long rows = (long long)p.B * p.H * p.T;
-  const long long grid = (long long)n_t * p.B * p.H;
-  if (grid > 0x7fffffffLL) return cudaErrorInvalidConfiguration;
+  if ((long long)n_t * p.B * p.H > 0x7fffffffLL) return cudaErrorInvalidConfiguration;
+  const long long grid = tile_grid(p);
   cudaError_t e = cudaSuccess;
   if (stages & 1) {
     const long long rows_pad = (long long)p.B * p.H * t_pad;
