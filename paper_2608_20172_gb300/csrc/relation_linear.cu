@@ -10,12 +10,14 @@
 // of Eq. (retention-vector) is upstream), p1, p2 are taken after RoPE (upstream).
 //
 // The recurrence never mixes information columns: column j of C evolves on its own.  The
-// forward therefore gives each column to kRG threads, each keeping d / kRG rows of it in
-// registers; a token costs 3 d / kRG multiply-adds per thread (the read is summed over
-// the column's threads once per chunk).  One CTA per (b, h) walks the tokens in
-// order; tokens are staged through shared memory in double-buffered chunks, with S_t,
-// 1/|p1_t|, 1/|p2_t| computed per chunk (S is folded into the coordinates:
-// q'_t = S_t ^p1_t, k'_t = S_t ^p2_t).  Loads are 4-element vectors without conditions.
+// kernels therefore split a head's columns across several CTAs (no exchange between them;
+// each runs Ask Self for the whole token).  In the forward a column belongs to RG threads,
+// each keeping R = d / RG of its rows in registers; a token costs 3 R multiply-adds per
+// thread (the read is summed over the column's threads once per chunk).  A CTA walks the
+// tokens in order; tokens are staged through shared memory in double-buffered chunks, Ask
+// Self (S_t, 1/|p1_t|, 1/|p2_t|) being taken on the way in, by shuffles among the threads
+// that load a token, and folded into the coordinates (q'_t = S_t ^p1_t, k'_t = S_t ^p2_t).
+// Loads are 4-element vectors without conditions.
 // The backward (below) walks the tokens in reverse with the adjoint state, recomputing
 // the states of each chunk of kChunkB tokens from checkpoints the kernel stores first.
 #include <math.h>
@@ -49,8 +51,7 @@ __device__ __forceinline__ void stx<__nv_bfloat16>(__nv_bfloat16* p, float v) {
 // I~ (fp32).
 template <int D, int NTOK = kChunkT>
 struct Chunk {
-  float vec[NTOK][4][D];  // [0] alpha, [1] p1 -> q', [2] p2 -> k', [3] I~
-  float scal[NTOK][4];    // S, 1/|p1|, 1/|p2|
+  float vec[NTOK][4][D];  // [0] alpha, [1] q' = S ^p1, [2] k' = S ^p2, [3] I~
 };
 
 // Four consecutive elements as fp32 (8- or 16-byte aligned vector load).
@@ -94,86 +95,85 @@ struct Loader {
       for (int a = 0; a < 4; ++a) r[a][n] = t < p.T ? x[a] : make_float4(0.f, 0.f, 0.f, 0.f);
     }
   }
-  __device__ __forceinline__ void store(Chunk<D, NTOK>& s) const {
+  // Ask Self on the way to shared memory: the D / 4 consecutive threads holding a token's
+  // vectors reduce p1 . p2, |p1|^2, |p2|^2 by shuffles, and each scales its pieces into
+  // q' = S_t p1 / |p1|, k' = S_t p2 / |p2| with S_t = sigmoid(p1 . p2 / (tau_S sqrt d)).
+  __device__ __forceinline__ void store(Chunk<D, NTOK>& s, float tau_s) const {
+    const float inv_t = 1.0f / (tau_s * sqrtf((float)D));
 #pragma unroll
     for (int n = 0; n < NV; ++n) {
       const int v = n * NT + (int)threadIdx.x;
       const int tt = v / (D / 4), c4 = (v % (D / 4)) * 4;
+      const float4 a = r[1][n], k = r[2][n];
+      float s12 = a.x * k.x + a.y * k.y + a.z * k.z + a.w * k.w;
+      float s11 = a.x * a.x + a.y * a.y + a.z * a.z + a.w * a.w;
+      float s22 = k.x * k.x + k.y * k.y + k.z * k.z + k.w * k.w;
 #pragma unroll
-      for (int a = 0; a < 4; ++a) *reinterpret_cast<float4*>(&s.vec[tt][a][c4]) = r[a][n];
+      for (int o = 1; o < D / 4; o <<= 1) {
+        s12 += __shfl_xor_sync(0xffffffffu, s12, o);
+        s11 += __shfl_xor_sync(0xffffffffu, s11, o);
+        s22 += __shfl_xor_sync(0xffffffffu, s22, o);
+      }
+      const float S = 1.0f / (1.0f + expf(-s12 * inv_t));
+      const float f1 = s11 > 0.f ? S * rsqrtf(s11) : 0.f;
+      const float f2 = s22 > 0.f ? S * rsqrtf(s22) : 0.f;
+      *reinterpret_cast<float4*>(&s.vec[tt][0][c4]) = r[0][n];
+      *reinterpret_cast<float4*>(&s.vec[tt][1][c4]) = make_float4(a.x * f1, a.y * f1, a.z * f1, a.w * f1);
+      *reinterpret_cast<float4*>(&s.vec[tt][2][c4]) = make_float4(k.x * f2, k.y * f2, k.z * f2, k.w * f2);
+      *reinterpret_cast<float4*>(&s.vec[tt][3][c4]) = r[3][n];
     }
   }
 };
 
-// Ask Self for the chunk's tokens (one warp per token), then fold S into the unit
-// coordinates.  Two block barriers; the caller has made the raw values visible.
-template <int D, int NT, int NTOK = kChunkT>
-__device__ __forceinline__ void ask_self_chunk(Chunk<D, NTOK>& s, float tau_s) {
-  constexpr int NW = NT / 32;
-  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  for (int tt = warp; tt < NTOK; tt += NW) {
-    float s12 = 0.f, s11 = 0.f, s22 = 0.f;
-    for (int c = lane; c < D; c += 32) {
-      const float a = s.vec[tt][1][c], b = s.vec[tt][2][c];
-      s12 = fmaf(a, b, s12);
-      s11 = fmaf(a, a, s11);
-      s22 = fmaf(b, b, s22);
-    }
-#pragma unroll
-    for (int o = 16; o > 0; o >>= 1) {
-      s12 += __shfl_xor_sync(0xffffffffu, s12, o);
-      s11 += __shfl_xor_sync(0xffffffffu, s11, o);
-      s22 += __shfl_xor_sync(0xffffffffu, s22, o);
-    }
-    if (lane == 0) {
-      s.scal[tt][0] = 1.0f / (1.0f + expf(-s12 / (tau_s * sqrtf((float)D))));
-      s.scal[tt][1] = s11 > 0.f ? rsqrtf(s11) : 0.f;
-      s.scal[tt][2] = s22 > 0.f ? rsqrtf(s22) : 0.f;
-    }
-  }
-  __syncthreads();
-  for (int e = threadIdx.x; e < NTOK * 2 * D; e += NT) {
-    const int c = e % D, a = 1 + (e / D) % 2, tt = e / (2 * D);
-    s.vec[tt][a][c] *= s.scal[tt][0] * s.scal[tt][a];
-  }
-  __syncthreads();
-}
+// Forward: NS CTAs per head, each owning NC = D / NS information columns (the columns
+// evolve independently, so the split needs no exchange; every CTA runs Ask Self for the
+// whole token).  RG threads per column: thread (j, rg) = tid % NC, tid / NC keeps rows
+// rg * R .. + R of column j in registers.  Threads of a warp share at most two row groups,
+// so the per-token alpha, q', k' reads are shared-memory broadcasts, and each thread's
+// partial read goes to shared memory: Y_t = I~_t + sum_rg e_rg is formed per chunk (the
+// output does not feed back into the recurrence), with no per-token shuffle.
+constexpr int kChunkF = 16;  // tokens per staged chunk (forward)
 
-// Forward: one CTA per head, kRG threads per column.  Thread (j, rg) = tid % D, tid / D
-// keeps rows rg * D/kRG .. + D/kRG of column j in registers.  A warp shares one row group,
-// so the per-token alpha, q', k' reads are one shared-memory broadcast per vector, and
-// each thread's partial read goes to shared memory: Y_t = I~_t + sum_rg e_rg is formed per
-// chunk (the output does not feed back into the recurrence), with no per-token shuffle.
-constexpr int kRG = 4;
-constexpr int kChunkF = 32;  // tokens per staged chunk (forward)
+template <int D, int NS>
+struct FwdCfg {
+  static constexpr int NT = D == 64 ? 256 : 128;  // threads
+  static constexpr int NC = D / NS;               // columns per CTA
+  static constexpr int RG = NT / NC;              // row groups
+  static constexpr int R = D / RG;                // rows per thread
+  static_assert(R % 4 == 0 && RG * R == D, "row split");
+};
 
-template <int D>
+template <int D, int NS>
 struct FwdSmem {
   Chunk<D, kChunkF> buf[2];
-  float epart[kChunkF][kRG][D];  // partial reads of the chunk's tokens
+  float epart[kChunkF][FwdCfg<D, NS>::RG][FwdCfg<D, NS>::NC];  // partial reads
 };
 
-template <typename TI, int D>
-__global__ void __launch_bounds__(kRG * D) fwd_kernel(LinearProblem p) {
-  constexpr int NT = kRG * D, R = D / kRG;
+template <typename TI, int D, int NS>
+__global__ void __launch_bounds__(FwdCfg<D, NS>::NT) fwd_kernel(LinearProblem p) {
+  using F = FwdCfg<D, NS>;
+  constexpr int NT = F::NT, NC = F::NC, RG = F::RG, R = F::R;
   extern __shared__ __align__(16) uint8_t smem_raw[];
-  FwdSmem<D>& sm = *reinterpret_cast<FwdSmem<D>*>(smem_raw);
-  const int bh = blockIdx.x, b = bh / p.H, h = bh % p.H;
-  const int j = threadIdx.x % D, rg = threadIdx.x / D, r0 = rg * R;
+  FwdSmem<D, NS>& sm = *reinterpret_cast<FwdSmem<D, NS>*>(smem_raw);
+  const int bh = blockIdx.x / NS, js = blockIdx.x % NS, b = bh / p.H, h = bh % p.H;
+  const int jl = threadIdx.x % NC, rg = threadIdx.x / NC, r0 = rg * R;
+  const int j = js * NC + jl;  // this thread's column of C
   const int n_ch = (p.T + kChunkF - 1) / kChunkF;
   float C[R];
 #pragma unroll
   for (int r = 0; r < R; ++r) C[r] = 0.f;
-  Loader<TI, D, NT, kChunkF> ld;
-  ld.load(p, b, h, 0);
-  ld.store(sm.buf[0]);
+  // Chunk c is loaded into registers two chunks ahead, by loader c % 2, while chunk c - 2
+  // is computed, and stored to shared memory once chunk c - 1 is done.
+  Loader<TI, D, NT, kChunkF> ld0, ld1;
+  ld0.load(p, b, h, 0);
+  if (n_ch > 1) ld1.load(p, b, h, 1);
+  ld0.store(sm.buf[0], p.tau_s);
   __syncthreads();
-  ask_self_chunk<D, NT, kChunkF>(sm.buf[0], p.tau_s);
   TI* Y = reinterpret_cast<TI*>(p.y) + (long long)b * p.sB + (long long)h * p.sH;
-  for (int ch = 0; ch < n_ch; ++ch) {
+  // chunk ch; `nxt` holds chunk ch + 1, `fre` takes chunk ch + 2
+  auto chunk = [&](int ch, Loader<TI, D, NT, kChunkF>& nxt, Loader<TI, D, NT, kChunkF>& fre) {
     Chunk<D, kChunkF>& cur = sm.buf[ch & 1];
-    const bool more = ch + 1 < n_ch;
-    if (more) ld.load(p, b, h, ch + 1);  // in flight while this chunk is computed
+    if (ch + 2 < n_ch) fre.load(p, b, h, ch + 2);  // in flight for two chunks
     const int nt = min(kChunkF, p.T - ch * kChunkF);
     for (int tt = 0; tt < nt; ++tt) {
       const float* al = &cur.vec[tt][0][r0];
@@ -195,33 +195,41 @@ __global__ void __launch_bounds__(kRG * D) fwd_kernel(LinearProblem p) {
           C[r + u] = fmaf(kv[u], I, cm);       // Become Others: write S k^ I~
         }
       }
-      sm.epart[tt][rg][j] = e;
+      sm.epart[tt][rg][jl] = e;
     }
     __syncthreads();  // the chunk's partial reads are complete
-    for (int e = threadIdx.x; e < nt * D; e += NT) {  // Answer: Y_t = I~_t + E_t
-      const int tt = e / D, jj = e % D;
-      float y = cur.vec[tt][3][jj];
+    for (int e = threadIdx.x; e < nt * NC; e += NT) {  // Answer: Y_t = I~_t + E_t
+      const int tt = e / NC, cl = e % NC;
+      float y = cur.vec[tt][3][js * NC + cl];
 #pragma unroll
-      for (int g = 0; g < kRG; ++g) y += sm.epart[tt][g][jj];
-      stx<TI>(Y + (long long)(ch * kChunkF + tt) * p.sT + jj, y);
+      for (int g = 0; g < RG; ++g) y += sm.epart[tt][g][cl];
+      stx<TI>(Y + (long long)(ch * kChunkF + tt) * p.sT + js * NC + cl, y);
     }
-    if (more) {
-      // nxt held chunk ch - 1, which every thread finished before the barrier above
-      Chunk<D, kChunkF>& nxt = sm.buf[(ch + 1) & 1];
-      ld.store(nxt);
+    if (ch + 1 < n_ch) {
+      // buffer (ch + 1) & 1 held chunk ch - 1, which every thread finished before the
+      // barrier above
+      nxt.store(sm.buf[(ch + 1) & 1], p.tau_s);
       __syncthreads();  // also: epart is read above before the next chunk overwrites it
-      ask_self_chunk<D, NT, kChunkF>(nxt, p.tau_s);
     }
+  };
+  for (int ch = 0; ch < n_ch; ch += 2) {
+    chunk(ch, ld1, ld0);
+    if (ch + 1 < n_ch) chunk(ch + 1, ld0, ld1);
   }
 }
 
+// column splits: the forward at d_h = 64 runs 4 CTAs per head, at d_h = 32 two
+template <int D>
+constexpr int fwd_splits() { return D == 64 ? 4 : 2; }
+
 template <typename TI, int D>
 cudaError_t fwd_t(const LinearProblem& p, cudaStream_t s) {
-  const int smem = (int)sizeof(FwdSmem<D>);
-  cudaError_t e = cudaFuncSetAttribute(fwd_kernel<TI, D>,
+  constexpr int NS = fwd_splits<D>();
+  const int smem = (int)sizeof(FwdSmem<D, NS>);
+  cudaError_t e = cudaFuncSetAttribute(fwd_kernel<TI, D, NS>,
                                        cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
   if (e != cudaSuccess) { note_failure("linear forward: shared memory attribute"); return e; }
-  fwd_kernel<TI, D><<<(unsigned)(p.B * p.H), kRG * D, smem, s>>>(p);
+  fwd_kernel<TI, D, NS><<<(unsigned)(p.B * p.H * NS), FwdCfg<D, NS>::NT, smem, s>>>(p);
   if ((e = cudaGetLastError()) != cudaSuccess) note_failure("linear forward: launch");
   return e;
 }
@@ -232,31 +240,40 @@ cudaError_t fwd_t(const LinearProblem& p, cudaStream_t s) {
 //   dI~_t = dY_t + dC_t^T k'_t,   dk'_t = dC_t I~_t,   dq'_t = C^- dY_t,
 //   dC^- = dC_t + q'_t dY_t^T,   dalpha_t = rowsum(dC^- * C_{t-1}),   dC_{t-1} = Diag(alpha_t) dC^-
 // (C^- = Diag(alpha_t) C_{t-1}); a per-token pass then turns dq', dk' into dp1, dp2
-// through the normalisation and S.  kQ threads own row c of the state, a quarter of the
-// columns each, so the row sums (dk', dq', dalpha) are two shuffles and the column sum
-// (dI~) is reduced across rows by a shuffle reduce-scatter within each warp and shared
-// memory across warps.
+// through the normalisation and S.  NS CTAs per head each own NC = D / NS columns of the
+// state (and of dC): the column sum (dI~) stays within a CTA, the row sums (dk', dq',
+// dalpha) are partial sums over the CTA's columns, added up by the per-token pass.  kQ
+// threads own row c of the CTA's columns, a quarter each, so a row sum is two shuffles
+// and the column sum is reduced across rows by a shuffle reduce-scatter within each warp
+// and shared memory across warps.
 //   1. checkpoint pass: forward over the tokens, storing the state before every kChunkB
 //      tokens in the workspace;
 //   2. reverse sweep: tokens staged kStageB at a time; per sub-chunk of kChunkB (last
 //      first), the states before each of its tokens are recomputed from the checkpoint into
 //      shared memory, then the tokens are walked backwards;
-//   3. per-token pass: dp1, dp2.
+//   3. per-token pass: dalpha and, through the normalisation and S, dp1, dp2.
 constexpr int kChunkB = 8;   // tokens per checkpoint / recomputed sub-chunk
 constexpr int kStageB = 16;  // tokens per staged chunk (two sub-chunks)
 constexpr int kQ = 4;        // threads per state row (each a quarter of the columns)
 
+// column splits of the backward: two CTAs per head at d_h = 64, one at d_h = 32 (the
+// reduce-scatter below needs R = NC / kQ >= 32 / kQ)
+template <int D>
+constexpr int bwd_splits() { return D == 64 ? 2 : 1; }
+
 template <int D>
 struct BwdSmem {
+  static constexpr int NC = D / bwd_splits<D>();
   Chunk<D, kStageB> tok;                  // alpha, q', k', I~ of the staged chunk
   float g[kStageB][D];                    // dY of the staged chunk
-  float red[kStageB][kQ * D / 32][D];     // per-warp column sums of dC^T k'
+  float red[kStageB][kQ * D / 32][NC];    // per-warp column sums of dC^T k'
   // C_{t-1} of each token of a sub-chunk, each thread's slice as float4s indexed
   // [token][k][thread]: a thread only reads its own slice back, and consecutive lanes
   // touch consecutive 16-byte words (no bank conflicts)
-  float4 st[kChunkB][D / (4 * kQ)][kQ * D];
+  float4 st[kChunkB][NC / (4 * kQ)][kQ * D];
 };
 
+// checkpointed state of one head (all column splits together)
 template <int D>
 __host__ __device__ constexpr long long ckpt_floats(int T) {
   return (long long)((T + kChunkB - 1) / kChunkB) * D * D;
@@ -264,33 +281,44 @@ __host__ __device__ constexpr long long ckpt_floats(int T) {
 
 template <typename TI, int D>
 __global__ void __launch_bounds__(kQ * D) bwd_kernel(LinearProblem p) {
-  constexpr int NT = kQ * D, R = D / kQ, NW = NT / 32;
+  constexpr int NS = bwd_splits<D>(), NC = D / NS;
+  constexpr int NT = kQ * D, R = NC / kQ, NW = NT / 32;
+  static_assert(R >= 32 / kQ && R % 4 == 0, "reduce-scatter over the warp's rows");
   extern __shared__ __align__(16) uint8_t smem_raw[];
   BwdSmem<D>& sm = *reinterpret_cast<BwdSmem<D>*>(smem_raw);
-  const int bh = blockIdx.x, b = bh / p.H, h = bh % p.H;
-  const int c = threadIdx.x / kQ, j0 = (threadIdx.x % kQ) * R;
+  const int bh = blockIdx.x / NS, js = blockIdx.x % NS, b = bh / p.H, h = bh % p.H;
+  const int c = threadIdx.x / kQ, jl0 = (threadIdx.x % kQ) * R;  // row; first local column
+  const int j0 = js * NC + jl0;                                  // first column of C
   const bool lead = threadIdx.x % kQ == 0;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int n_st = (p.T + kStageB - 1) / kStageB;
-  float* ckpt = reinterpret_cast<float*>(p.workspace) + (long long)bh * ckpt_floats<D>(p.T);
+  // checkpoints of this CTA's columns: [n_ck][D rows][NC]
+  float* ckpt = reinterpret_cast<float*>(p.workspace) + (long long)bh * ckpt_floats<D>(p.T) +
+                (long long)js * (ckpt_floats<D>(p.T) / NS);
+  // partial row sums over this CTA's columns, [T][3][D]: dq', dk', dalpha
   float* dqk = reinterpret_cast<float*>(p.workspace) + (long long)p.B * p.H * ckpt_floats<D>(p.T) +
-               (long long)bh * p.T * 2 * D;  // [T][2][D]: dq', dk'
+               ((long long)bh * NS + js) * p.T * 3 * D;
   const long long hb = (long long)b * p.sB + (long long)h * p.sH;
+  // The token data of the next staged chunk is loaded into registers (fetch) while the
+  // current one is processed, and stored to shared memory when it is due (stage).
+  static_assert(kStageB * D / 4 == NT, "one dY vector per thread and chunk");
   Loader<TI, D, NT, kStageB> ld;
-  auto stage = [&](int sc, bool with_dy) {  // token data of staged chunk sc
-    __syncthreads();                         // the previous chunk's data is no longer read
+  float4 gpre = make_float4(0.f, 0.f, 0.f, 0.f);  // this thread's dY vector
+  auto fetch = [&](int sc, bool with_dy) {
     ld.load(p, b, h, sc);
-    ld.store(sm.tok);
     if (with_dy) {
-      for (int v4 = threadIdx.x; v4 < kStageB * D / 4; v4 += NT) {
-        const int tt = v4 / (D / 4), c4 = (v4 % (D / 4)) * 4, t = sc * kStageB + tt;
-        const float4 g = ld4<TI>(reinterpret_cast<const TI*>(p.dy) + hb +
-                                 (long long)min(t, p.T - 1) * p.sT + c4);
-        *reinterpret_cast<float4*>(&sm.g[tt][c4]) = t < p.T ? g : make_float4(0.f, 0.f, 0.f, 0.f);
-      }
+      const int tt = threadIdx.x / (D / 4), c4 = (threadIdx.x % (D / 4)) * 4, t = sc * kStageB + tt;
+      const float4 g = ld4<TI>(reinterpret_cast<const TI*>(p.dy) + hb +
+                               (long long)min(t, p.T - 1) * p.sT + c4);
+      gpre = t < p.T ? g : make_float4(0.f, 0.f, 0.f, 0.f);
     }
+  };
+  auto stage = [&](bool with_dy) {  // the fetched chunk into shared memory
+    __syncthreads();                 // the previous chunk's data is no longer read
+    ld.store(sm.tok, p.tau_s);
+    if (with_dy)
+      *reinterpret_cast<float4*>(&sm.g[threadIdx.x / (D / 4)][(threadIdx.x % (D / 4)) * 4]) = gpre;
     __syncthreads();
-    ask_self_chunk<D, NT, kStageB>(sm.tok, p.tau_s);
   };
   auto row_step = [&](float (&Cs)[R], int tt) {  // C <- Diag(alpha) C + k' I~^T, own row
     const float a = sm.tok.vec[tt][0][c], kp = sm.tok.vec[tt][2][c];
@@ -308,12 +336,15 @@ __global__ void __launch_bounds__(kQ * D) bwd_kernel(LinearProblem p) {
   float C[R];
 #pragma unroll
   for (int i = 0; i < R; ++i) C[i] = 0.f;
+  fetch(0, false);
   for (int sc = 0; sc < n_st; ++sc) {
     const int nt = min(kStageB, p.T - sc * kStageB);
-    stage(sc, false);
+    stage(false);
+    if (sc + 1 < n_st) fetch(sc + 1, false);
+    else fetch(n_st - 1, true);  // the reverse sweep's first chunk
     for (int tt = 0; tt < nt; ++tt) {
       if (tt % kChunkB == 0) {
-        float* ck = ckpt + (long long)((sc * kStageB + tt) / kChunkB) * D * D + c * D + j0;
+        float* ck = ckpt + (long long)((sc * kStageB + tt) / kChunkB) * D * NC + c * NC + jl0;
 #pragma unroll
         for (int i = 0; i < R; i += 4)
           *reinterpret_cast<float4*>(ck + i) = make_float4(C[i], C[i + 1], C[i + 2], C[i + 3]);
@@ -326,11 +357,12 @@ __global__ void __launch_bounds__(kQ * D) bwd_kernel(LinearProblem p) {
 #pragma unroll
   for (int i = 0; i < R; ++i) dC[i] = 0.f;
   for (int sc = n_st - 1; sc >= 0; --sc) {
-    stage(sc, true);
+    stage(true);
+    if (sc > 0) fetch(sc - 1, true);
     const int nt = min(kStageB, p.T - sc * kStageB);
     for (int sub = (nt - 1) / kChunkB; sub >= 0; --sub) {
       const int tb = sub * kChunkB, ns = min(kChunkB, nt - tb);
-      const float* ck = ckpt + (long long)((sc * kStageB + tb) / kChunkB) * D * D + c * D + j0;
+      const float* ck = ckpt + (long long)((sc * kStageB + tb) / kChunkB) * D * NC + c * NC + jl0;
 #pragma unroll
       for (int i = 0; i < R; i += 4) {
         const float4 x = *reinterpret_cast<const float4*>(ck + i);
@@ -372,9 +404,9 @@ __global__ void __launch_bounds__(kQ * D) bwd_kernel(LinearProblem p) {
           da += __shfl_xor_sync(0xffffffffu, da, o);
         }
         if (lead) {
-          p.dalpha[hb + (long long)t * p.sT + c] = da;
-          dqk[(long long)t * 2 * D + c] = dq;
-          dqk[(long long)t * 2 * D + D + c] = dk;
+          dqk[(long long)t * 3 * D + c] = dq;
+          dqk[(long long)t * 3 * D + D + c] = dk;
+          dqk[(long long)t * 3 * D + 2 * D + c] = da;
         }
         // column sums over the warp's 32 / kQ rows: reduce-scatter over the lane bits above
         // the kQ column threads
@@ -394,21 +426,22 @@ __global__ void __launch_bounds__(kQ * D) bwd_kernel(LinearProblem p) {
           off += up ? n : 0;
         }
 #pragma unroll
-        for (int i = 0; i < R / (32 / kQ); ++i) sm.red[tt][warp][j0 + off + i] = col[i];
+        for (int i = 0; i < R / (32 / kQ); ++i) sm.red[tt][warp][jl0 + off + i] = col[i];
       }
     }
     __syncthreads();
-    for (int e = threadIdx.x; e < nt * D; e += NT) {  // dI~_t = dY_t + dC_t^T k'_t
-      const int tt = e / D, jj = e % D, t = sc * kStageB + tt;
-      float s2 = sm.g[tt][jj];
+    for (int e = threadIdx.x; e < nt * NC; e += NT) {  // dI~_t = dY_t + dC_t^T k'_t
+      const int tt = e / NC, cl = e % NC, t = sc * kStageB + tt;
+      float s2 = sm.g[tt][js * NC + cl];
 #pragma unroll
-      for (int w = 0; w < NW; ++w) s2 += sm.red[tt][w][jj];
-      stx<TI>(reinterpret_cast<TI*>(p.dv) + hb + (long long)t * p.sT + jj, s2);
+      for (int w = 0; w < NW; ++w) s2 += sm.red[tt][w][cl];
+      stx<TI>(reinterpret_cast<TI*>(p.dv) + hb + (long long)t * p.sT + js * NC + cl, s2);
     }
   }
 }
 
-// dp1, dp2 of every token (one warp per token) from dq', dk' through q' = S p1 / |p1|,
+// dalpha, dp1, dp2 of every token (one warp per token): the column splits' partial sums of
+// dalpha, dq', dk' added up, then dq', dk' taken through q' = S p1 / |p1|,
 // k' = S p2 / |p2| and S = sigmoid(p1 . p2 / (tau_S sqrt d)).
 template <typename TI, int D>
 __global__ void __launch_bounds__(256) post_kernel(LinearProblem p) {
@@ -418,8 +451,9 @@ __global__ void __launch_bounds__(256) post_kernel(LinearProblem p) {
   if (tok >= (long long)p.B * p.H * p.T) return;
   const int bh = (int)(tok / p.T), t = (int)(tok % p.T), b = bh / p.H, h = bh % p.H;
   const long long off = (long long)b * p.sB + (long long)h * p.sH + (long long)t * p.sT;
+  constexpr int NS = bwd_splits<D>();
   const float* dqk = reinterpret_cast<const float*>(p.workspace) +
-                     (long long)p.B * p.H * ckpt_floats<D>(p.T) + ((long long)bh * p.T + t) * 2 * D;
+                     (long long)p.B * p.H * ckpt_floats<D>(p.T) + ((long long)bh * NS * p.T + t) * 3 * D;
   float x1[PL], x2[PL], g1[PL], g2[PL];
   float s12 = 0.f, s11 = 0.f, s22 = 0.f;
 #pragma unroll
@@ -427,8 +461,17 @@ __global__ void __launch_bounds__(256) post_kernel(LinearProblem p) {
     const int cc = lane + 32 * e;
     x1[e] = ldx<TI>(reinterpret_cast<const TI*>(p.p1) + off + cc);
     x2[e] = ldx<TI>(reinterpret_cast<const TI*>(p.p2) + off + cc);
-    g1[e] = dqk[cc];
-    g2[e] = dqk[D + cc];
+    g1[e] = 0.f;
+    g2[e] = 0.f;
+    float da = 0.f;
+#pragma unroll
+    for (int js = 0; js < NS; ++js) {
+      const float* part = dqk + (long long)js * p.T * 3 * D;
+      g1[e] += part[cc];
+      g2[e] += part[D + cc];
+      da += part[2 * D + cc];
+    }
+    p.dalpha[off + cc] = da;
     s12 = fmaf(x1[e], x2[e], s12);
     s11 = fmaf(x1[e], x1[e], s11);
     s22 = fmaf(x2[e], x2[e], s22);
@@ -473,7 +516,7 @@ cudaError_t bwd_t(const LinearProblem& p, cudaStream_t s) {
   cudaError_t e = cudaFuncSetAttribute(bwd_kernel<TI, D>,
                                        cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
   if (e != cudaSuccess) { note_failure("linear backward: shared memory attribute"); return e; }
-  bwd_kernel<TI, D><<<(unsigned)(p.B * p.H), kQ * D, smem, s>>>(p);
+  bwd_kernel<TI, D><<<(unsigned)(p.B * p.H * bwd_splits<D>()), kQ * D, smem, s>>>(p);
   if ((e = cudaGetLastError()) != cudaSuccess) { note_failure("linear backward: launch"); return e; }
   const long long toks = (long long)p.B * p.H * p.T;
   post_kernel<TI, D><<<(unsigned)((toks * 32 + 255) / 256), 256, 0, s>>>(p);
@@ -485,7 +528,8 @@ cudaError_t bwd_t(const LinearProblem& p, cudaStream_t s) {
 
 size_t linear_bwd_workspace_bytes(int B, int H, int T, int d) {
   const long long per = d == 32 ? lin::ckpt_floats<32>(T) : lin::ckpt_floats<64>(T);
-  return (size_t)((long long)B * H * per + (long long)B * H * T * 2 * d) * sizeof(float);
+  const int ns = d == 32 ? lin::bwd_splits<32>() : lin::bwd_splits<64>();
+  return (size_t)((long long)B * H * per + (long long)B * H * ns * T * 3 * d) * sizeof(float);
 }
 
 cudaError_t launch_linear_bwd(const LinearProblem& p, cudaStream_t s) {
