@@ -223,7 +223,10 @@ __global__ void __launch_bounds__(kThreads, 1)
   // and r G + G - 1 - c in odd ones: the units come heaviest first, so the zigzag evens
   // out the CTAs' work.  Every role walks the same sequence and keeps running counts
   // (units, steps, Q / dO stage loads, query tiles) from which the barrier phases follow.
+  // d_h = 128 takes one unit per CTA (the launch gives one CTA per unit): its loops over
+  // units end after the first at compile time.
   auto unit_at = [&](int r) -> int {
+    if (C::HALF) return r == 0 ? (int)blockIdx.x : n_work;
     const int c = (r & 1) ? (int)(gridDim.x - 1 - blockIdx.x) : (int)blockIdx.x;
     return r * (int)gridDim.x + c;
   };
