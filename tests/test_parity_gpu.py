@@ -282,3 +282,30 @@ def test_self_flow_side_output(dtype, d, T):
                 err = np.abs(fs[b, h] - ref["Fii"]).max()
                 assert err <= tol, f"{fam} head ({b},{h}): max |F_ii - ref| = {err:.3g} > {tol}"
                 assert fs[b, h, 0] == 1.0
+
+
+# --- the persistent backward: many (key tile, head) units per CTA ---------------
+
+@pytest.mark.parametrize("B,H,T,d", [(4, 80, 300, 64), (2, 100, 200, 48), (1, 400, 129, 64)])
+def test_persistent_backward_many_units(B, H, T, d):
+    """More units than SMs, of mixed sizes (ragged last key tile): every CTA walks several
+    units, so the cross-unit K/V double buffer, the staging reuse and the zigzag order
+    are all exercised.  Sampled heads against the oracle element by element, every head
+    against the CUDA-core backward (an independent GPU implementation), and dlambda
+    over all heads against the oracle."""
+    w = workloads.custom(B, H, T, d, "bf16")
+    q, k, v, do = workloads.make_inputs(w)
+    res = pu.gpu_run(q, k, v, do, LAM)
+    heads = [(0, 0), (B - 1, H - 1), (B // 2, H // 2), (0, H - 1), (B - 1, 1)]
+    ref = pu.oracle_heads(q, k, v, do, LAM, heads)
+    pu.compare_heads(res, ref, "bf16")
+    if pu.kernel_available("simt", "bf16", d, "bwd"):
+        alt = pu.gpu_run(q, k, v, do, LAM, kernel_bwd="simt")
+        for n in ("dQ", "dK", "dV"):
+            for b in range(B):
+                for h in range(H):
+                    e = pu.err_metric(res[n][b, :, h].numpy(), alt[n][b, :, h].numpy(), "bf16")
+                    assert e <= 2 * pu.TOL[("bf16", "grad")], f"{n}[{b},{h}] vs CUDA-core: {e:.3e}"
+    _, _, _, dl_all = oracle.mhr_bwd(q.double().numpy(), k.double().numpy(), v.double().numpy(),
+                                     do.double().numpy(), LAM)
+    pu.check_dlambda(res["dlambda"], dl_all, "bf16")
