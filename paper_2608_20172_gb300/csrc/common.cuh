@@ -218,6 +218,13 @@ __device__ __forceinline__ void tmem_st16(uint32_t taddr, const uint32_t* r) {
       : "memory");
 }
 
+__device__ __forceinline__ void tmem_st8(uint32_t taddr, const uint32_t* r) {
+  asm volatile(
+      "tcgen05.st.sync.aligned.32x32b.x8.b32 [%0], {%1, %2, %3, %4, %5, %6, %7, %8};" ::"r"(taddr),
+      "r"(r[0]), "r"(r[1]), "r"(r[2]), "r"(r[3]), "r"(r[4]), "r"(r[5]), "r"(r[6]), "r"(r[7])
+      : "memory");
+}
+
 // Shared-memory matrix descriptor (tcgen05 "version 1" format):
 //   bits  0-13 start address >> 4, 16-29 leading byte offset >> 4,
 //   bits 32-45 stride byte offset >> 4, 46-47 version = 1, 49-51 base offset = 0,

@@ -149,15 +149,15 @@ struct EwConst {
 // their dlambda terms are exactly zero; the Self entry (query == key) then takes the
 // row pass's values, P = F_tt and dS' = 2 dS_tt (self2 = {F_tt, dS_tt}), so that the
 // dV, dK and dQ products include it (its dlambda term is the row pass's).
-template <bool DIAG, int SW>
-__device__ __forceinline__ void ew_chunk(const uint32_t (&U)[32], const uint32_t (&G)[32],
+template <bool DIAG, int SW, int N>
+__device__ __forceinline__ void ew_chunk(const uint32_t (&U)[N], const uint32_t (&G)[N],
                                          const float* st, int qt0, int t, const EwConst& k,
-                                         float2 self2, uint32_t (&pk)[16], uint32_t (&dk)[16],
-                                         float2& dl2) {
+                                         float2 self2, uint32_t (&pk)[N / 2],
+                                         uint32_t (&dk)[N / 2], float2& dl2) {
   const float2 ch2 = make_float2(k.ch, k.ch), c2k2 = make_float2(k.c2k, k.c2k);
   const float2 one2 = make_float2(1.f, 1.f);
 #pragma unroll
-  for (int c = 0; c < 32; c += 4) {
+  for (int c = 0; c < N; c += 4) {
     float4 c2v = *reinterpret_cast<const float4*>(st + c);
     const float4 ndv = *reinterpret_cast<const float4*>(st + SW + c);
     const float4 nwv = *reinterpret_cast<const float4*>(st + 2 * SW + c);
@@ -620,18 +620,38 @@ __global__ void __launch_bounds__(kThreads, 1)
         const float* sts = reinterpret_cast<const float*>(smem + C::OFF_STAT + st * C::STB);
         const int cl = wg * 32;             // the chunk's first column within the step
         const int qt0 = hh * C::QW + cl;    // tile-local query index
-        uint32_t U_[32], G[32];
-        tmem_ld32(trow + C::col_u(bb) + cl, U_);
-        tmem_ld32(trow + C::col_g(bb) + cl, G);
+        // Two halves of 16 queries: the second half's TMEM load is in flight while the
+        // first is computed.  P (dS') of queries cl + 16 h .. go packed to columns
+        // cl + 8 h .. of the U^T (dP^T) columns, which the first half has already read.
+        uint32_t U0[16], G0[16], U1[16], G1[16];
+        tmem_ld16(trow + C::col_u(bb) + cl, U0);
+        tmem_ld16(trow + C::col_g(bb) + cl, G0);
         tmem_ld_wait();
+        tmem_ld16(trow + C::col_u(bb) + cl + 16, U1);
+        tmem_ld16(trow + C::col_g(bb) + cl + 16, G1);
         uint32_t pk[16], dk[16];
         const float* stc = sts + (C::HALF ? cl : qt0);
-        if (i == 0)
-          ew_chunk<true, C::SW>(U_, G, stc, qt0, t, kc, self2, pk, dk, dl2);
-        else
-          ew_chunk<false, C::SW>(U_, G, stc, qt0, t, kc, self2, pk, dk, dl2);
-        tmem_st16(trow + C::col_u(bb) + cl, pk);  // P   (A operand of dV += P^T dO)
-        tmem_st16(trow + C::col_g(bb) + cl, dk);  // dS' (A operand of dK += dS'^T Q)
+        {
+          uint32_t (&p0)[8] = *reinterpret_cast<uint32_t(*)[8]>(pk);
+          uint32_t (&d0)[8] = *reinterpret_cast<uint32_t(*)[8]>(dk);
+          if (i == 0)
+            ew_chunk<true, C::SW, 16>(U0, G0, stc, qt0, t, kc, self2, p0, d0, dl2);
+          else
+            ew_chunk<false, C::SW, 16>(U0, G0, stc, qt0, t, kc, self2, p0, d0, dl2);
+          tmem_st8(trow + C::col_u(bb) + cl, p0);  // P   (A operand of dV += P^T dO)
+          tmem_st8(trow + C::col_g(bb) + cl, d0);  // dS' (A operand of dK += dS'^T Q)
+        }
+        tmem_ld_wait();
+        {
+          uint32_t (&p1)[8] = *reinterpret_cast<uint32_t(*)[8]>(pk + 8);
+          uint32_t (&d1)[8] = *reinterpret_cast<uint32_t(*)[8]>(dk + 8);
+          if (i == 0)
+            ew_chunk<true, C::SW, 16>(U1, G1, stc + 16, qt0 + 16, t, kc, self2, p1, d1, dl2);
+          else
+            ew_chunk<false, C::SW, 16>(U1, G1, stc + 16, qt0 + 16, t, kc, self2, p1, d1, dl2);
+          tmem_st8(trow + C::col_u(bb) + cl + 8, p1);
+          tmem_st8(trow + C::col_g(bb) + cl + 8, d1);
+        }
         if (s == 0 && ul > 0) {
           // the previous unit's dK / dV staging, in the dS' buffer written next, has been
           // read by the stores of all eight warps
