@@ -275,12 +275,56 @@ def decode_measure(binding, dev, peaks, steps=20, warmup=3):
             "gpu_launches_per_call": 2}
 
 
+LAYER_CFG = {"B": 2, "H": 16, "T": 16384, "d_h": 128}  # the long geometry, bf16 (> L2)
+
+
+def layer_measure(binding, dev, peaks, steps=10, warmup=3):
+    """The layer's transforms around the operator (RoPE of P1, P2 and the Givens mixing of
+    I; their gradient) on the long geometry: algorithmic bytes = prep reads P1, P2, I and
+    writes Q, K, V; grad reads dQ, dK, dV, I and writes dP1, dP2, dI; HBM roofline."""
+    c = LAYER_CFG
+    B, H, T, d = c["B"], c["H"], c["T"], c["d_h"]
+    g = torch.Generator(device="cpu").manual_seed(0)
+    xs = [torch.randn((B, T, H, d), generator=g).to(torch.bfloat16).to(dev) for _ in range(4)]
+    theta = (torch.rand(H // 2, generator=g) * 2.0 - 1.0).float().to(dev)
+    outs = tuple(torch.empty_like(xs[0]) for _ in range(3))
+    ws = torch.empty(max(binding.layer_grad_workspace_size(xs[0]), 16), dtype=torch.uint8,
+                     device=dev)
+    stream = torch.cuda.current_stream(dev)
+
+    def timed(call):
+        for _ in range(warmup):
+            call()
+        ev = [torch.cuda.Event(enable_timing=True) for _ in range(steps + 1)]
+        torch.cuda.synchronize(dev)
+        ev[0].record(stream)
+        for i in range(steps):
+            call()
+            ev[i + 1].record(stream)
+        torch.cuda.synchronize(dev)
+        return statistics.mean(ev[i].elapsed_time(ev[i + 1]) for i in range(steps))
+
+    ms_p = timed(lambda: binding.layer_prep(xs[0], xs[1], xs[2], theta, 1, out=outs,
+                                            stream=stream))
+    ms_g = timed(lambda: binding.layer_grad(xs[0], xs[1], xs[2], xs[3], theta, 1, workspace=ws,
+                                            stream=stream))
+    one = B * T * H * d * 2.0
+    gb_p, gb_g = 6 * one / (ms_p * 1e-3) / 1e9, 7 * one / (ms_g * 1e-3) / 1e9
+    return {"config": {**c, "dtype": "bf16", "pairing": "B", "l2": "arrays 134 MB each > L2"},
+            "ms_prep": ms_p, "ms_grad": ms_g,
+            "roofline": {"bound": "hbm", "kernel": "layer prep_kernel", "achieved": gb_p,
+                         "peak": peaks["hbm_gbs"], "unit": "GB/s", "frac": gb_p / peaks["hbm_gbs"],
+                         "grad_achieved": gb_g, "grad_frac": gb_g / peaks["hbm_gbs"],
+                         "algorithmic_bytes_prep": 6 * one, "algorithmic_bytes_grad": 7 * one},
+            "gpu_launches_per_call": {"prep": 1, "grad": 2}}
+
+
 LINEAR_CFG = {"B": 8, "H": 12, "T": 2048, "d_h": 64}  # the 100M layer geometry, bf16
 FP32_FMA_TFLOPS = 152 * 128 * 2 * 2.07e9 / 1e12  # 152 SMs x 128 FFMA lanes x 2 flops x 2.07 GHz
 
 
 def linear_measure(binding, dev, steps=20, warmup=3):
-    """Linear Relation forward and backward on the 100M geometry (bf16, one CTA per head).
+    """Linear Relation forward and backward on the 100M geometry (bf16, column splits).
     Arithmetic per token and head: forward 5 d^2 (decay, read, write); backward 16 d^2
     (checkpoint pass 3, chunk recompute 3, reverse step 10).  ALU roofline against the
     fp32 FMA peak of the SMs."""
@@ -458,6 +502,7 @@ def run_ours(args, w):
     if rank == 0 and ws == 1:
         line["decode"] = decode_measure(binding, dev, peaks)
         line["linear"] = linear_measure(binding, dev)
+        line["layer"] = layer_measure(binding, dev, peaks)
     if rank == 0 and not args.no_cpu_baseline and ws == 1:
         cb = cpu_oracle_run(w, min_seconds=10.0)
         line["cpu_baseline"] = {

@@ -136,7 +136,8 @@ relation_status relation_linear_fwd(const void* p1, const void* p2, const void* 
  *   dp1, dp2, dv : [B][T][H][d_h] in dt, with the inputs' strides (overwritten);
  *   dalpha       : [B][T][H][d_h] fp32 with alpha's strides (overwritten);
  *   workspace    : device scratch of relation_linear_bwd_workspace_size(shp, dt) bytes
- *                  (state checkpoints every 8 tokens plus two fp32 [B][H][T][d_h] arrays).
+ *                  (state checkpoints every 8 tokens plus fp32 partial row sums of the
+ *                  state's column splits, [B][H][splits][T][3][d_h]).
  * Same dtypes and widths as relation_linear_fwd; asynchronous on `stream`.
  */
 size_t relation_linear_bwd_workspace_size(relation_shape shp, relation_dtype dt);
@@ -168,6 +169,45 @@ relation_status relation_decode(const void* q, const void* k_cache, const void* 
                                 float tau_s, relation_shape cache, long long q_sB, long long q_sH,
                                 relation_dtype dt, void* workspace, size_t ws_bytes,
                                 int* dev_status, relation_stream_t stream);
+
+/*
+ * The paper layer's transforms around the operator (Sec. 3.1-3.2, Eq. (givens-rotation),
+ * App. A.2.2, App. B.3), producing the operator's inputs from the projected states:
+ *   q = RoPE(p1), k = RoPE(p2): full-head rotary embedding, channel pairs (2c, 2c+1)
+ *       of the row at position m (zero-based, restarting at every sequence) turned by
+ *       m * rope_base^(-2c/d_h) (the paper's base is 1e4);
+ *   v = Givens(info): head pairs (a, b) mixed on every channel with angle theta[k],
+ *       v_a = cos info_a - sin info_b,  v_b = sin info_a + cos info_b;
+ *       pairing 0: (0,1), (2,3), ..., (H-2,H-1); pairing 1: (1,2), ..., (H-1,0) (the
+ *       paper's alternating sets M_A and M_B, zero-based).
+ *   p1, p2, info, q, k, v : [B][T][H][d_h] in dt with the strides of `shp`; each output
+ *       may alias its input (q = p1, k = p2, v = info).
+ *   theta : device float[H/2], fp32.
+ * H even, d_h a multiple of 8 up to 256, H/2 <= 128; fp32 or bf16 (rotations in fp32; the
+ * RoPE angles are reduced modulo 2 pi in fp64).  Other shapes: RELATION_ERR_UNSUPPORTED.
+ * Asynchronous on `stream`; nothing is allocated.
+ */
+relation_status relation_layer_prep(const void* p1, const void* p2, const void* info,
+                                    const float* theta, int pairing, float rope_base, void* q,
+                                    void* k, void* v, relation_shape shp, relation_dtype dt,
+                                    relation_stream_t stream);
+
+/*
+ * Gradient of relation_layer_prep: from the operator's dq, dk, dv (as relation_bwd
+ * returns them) and the forward's info and theta,
+ *   dp1 = RoPE^T(dq), dp2 = RoPE^T(dk), dinfo = Givens^T(dv) (each may alias its input),
+ *   dtheta : device float[H/2], dtheta_k = sum over b, t, channels of
+ *            dv_a (-sin info_a - cos info_b) + dv_b (cos info_a - sin info_b)
+ *            (overwritten; summed in a fixed order, deterministic);
+ *   workspace : device scratch of relation_layer_grad_workspace_size(shp, dt) bytes.
+ * Same shapes and dtypes as relation_layer_prep; asynchronous on `stream`.
+ */
+size_t relation_layer_grad_workspace_size(relation_shape shp, relation_dtype dt);
+relation_status relation_layer_grad(const void* dq, const void* dk, const void* dv,
+                                    const void* info, const float* theta, int pairing,
+                                    float rope_base, void* dp1, void* dp2, void* dinfo,
+                                    float* dtheta, relation_shape shp, relation_dtype dt,
+                                    void* workspace, size_t ws_bytes, relation_stream_t stream);
 
 /* Bytes of device workspace relation_bwd needs for this shape and dtype (0 on a bad
  * shape).  The content of the workspace need not be initialised. */

@@ -31,7 +31,8 @@ EXPORTED = ("relation_fwd", "relation_fwd_ex", "relation_bwd", "relation_bwd_ex"
             "relation_selftest_wait_timeout", "relation_launch_count", "relation_last_cuda_error",
             "relation_bwd_stages", "relation_bwd_static", "relation_fwd_flow",
             "relation_decode", "relation_decode_workspace_size", "relation_linear_fwd",
-            "relation_linear_bwd", "relation_linear_bwd_workspace_size")
+            "relation_linear_bwd", "relation_linear_bwd_workspace_size", "relation_layer_prep",
+            "relation_layer_grad", "relation_layer_grad_workspace_size")
 
 
 class RelationLibraryMissing(RuntimeError):
@@ -81,6 +82,11 @@ def load(path: str | None = None):
         lib.relation_linear_bwd.argtypes = [vp, vp, vp, vp, vp, vp, vp, vp, vp, f, Shape, i, vp,
                                             ctypes.c_size_t, ip, vp]
         lib.relation_linear_bwd_workspace_size.argtypes = [Shape, i]
+        lib.relation_layer_prep.argtypes = [vp, vp, vp, vp, i, f, vp, vp, vp, Shape, i, vp]
+        lib.relation_layer_grad.argtypes = [vp, vp, vp, vp, vp, i, f, vp, vp, vp, vp, Shape, i,
+                                            vp, sz, vp]
+        lib.relation_layer_grad_workspace_size.argtypes = [Shape, i]
+        lib.relation_layer_grad_workspace_size.restype = sz
         lib.relation_linear_bwd_workspace_size.restype = ctypes.c_size_t
         lib.relation_decode_workspace_size.restype = ctypes.c_size_t
         lib.relation_bwd.argtypes = [vp, vp, vp, vp, vp, vp, vp, vp, vp, vp, f, f, Shape, i, vp,
@@ -231,6 +237,56 @@ def linear_bwd(p1, p2, v, alpha, dy, tau_s: float = 2.0, *, workspace=None, dev_
     if rc != OK:
         raise RelationError(rc, "relation_linear_bwd")
     return dp1, dp2, dv, dalpha
+
+
+def _layer_args(theta, pairing, rope_base, x):
+    if theta.dtype != torch.float32 or theta.device != x.device or theta.numel() != x.shape[2] // 2:
+        raise ValueError("theta must be fp32 [H/2] on the inputs' device")
+    if pairing not in (0, 1):
+        raise ValueError("pairing must be 0 (pairs (0,1), (2,3), ...) or 1 ((1,2), ..., (H-1,0))")
+    return theta.contiguous(), int(pairing), float(rope_base)
+
+
+def layer_prep(p1, p2, info, theta, pairing: int = 0, rope_base: float = 1.0e4, *, out=None,
+               stream=None):
+    """The layer's transforms before the operator: returns (q, k, v) = (RoPE(p1),
+    RoPE(p2), Givens(info)) for [B, T, H, d] inputs of one layout, theta fp32 [H/2]."""
+    _same_layout(p1, p2, info)
+    theta, pairing, rope_base = _layer_args(theta, pairing, rope_base, p1)
+    q, k, v = out if out is not None else (torch.empty_like(p1), torch.empty_like(p1),
+                                           torch.empty_like(p1))
+    _same_layout(p1, q, k, v)
+    rc = load().relation_layer_prep(_ptr(p1), _ptr(p2), _ptr(info), _ptr(theta), pairing,
+                                    rope_base, _ptr(q), _ptr(k), _ptr(v), shape_of(p1),
+                                    _dtype_code(p1), ctypes.c_void_p(_stream(stream)))
+    if rc != OK:
+        raise RelationError(rc, "relation_layer_prep")
+    return q, k, v
+
+
+def layer_grad_workspace_size(x) -> int:
+    """Device bytes relation_layer_grad needs for a [B, T, H, d] tensor of this dtype."""
+    return int(load().relation_layer_grad_workspace_size(shape_of(x), _dtype_code(x)))
+
+
+def layer_grad(dq, dk, dv, info, theta, pairing: int = 0, rope_base: float = 1.0e4, *,
+               workspace=None, stream=None):
+    """Gradient of layer_prep: returns (dp1, dp2, dinfo, dtheta)."""
+    _same_layout(dq, dk, dv, info)
+    theta, pairing, rope_base = _layer_args(theta, pairing, rope_base, dq)
+    dp1, dp2, dinfo = torch.empty_like(dq), torch.empty_like(dq), torch.empty_like(dq)
+    dtheta = torch.empty_like(theta)
+    need = layer_grad_workspace_size(dq)
+    if workspace is None:
+        workspace = torch.empty(max(need, 16), device=dq.device, dtype=torch.uint8)
+    rc = load().relation_layer_grad(_ptr(dq), _ptr(dk), _ptr(dv), _ptr(info), _ptr(theta),
+                                    pairing, rope_base, _ptr(dp1), _ptr(dp2), _ptr(dinfo),
+                                    _ptr(dtheta), shape_of(dq), _dtype_code(dq), _ptr(workspace),
+                                    workspace.numel() * workspace.element_size(),
+                                    ctypes.c_void_p(_stream(stream)))
+    if rc != OK:
+        raise RelationError(rc, "relation_layer_grad")
+    return dp1, dp2, dinfo, dtheta
 
 
 def decode_workspace_size(k_cache) -> int:

@@ -119,6 +119,32 @@ cudaError_t launch_linear_fwd(const LinearProblem& p, cudaStream_t s);
 size_t linear_bwd_workspace_bytes(int B, int H, int T, int d);
 cudaError_t launch_linear_bwd(const LinearProblem& p, cudaStream_t s);
 
+// The layer's transforms around the operator (RoPE of P1, P2; Givens mixing of the
+// information states) and their gradients.  prep: in1, in2, in3 = P1, P2, I and out1,
+// out2, out3 = Q, K, V.  grad: in1, in2, in3 = dQ, dK, dV, in4 = I and out1, out2, out3 =
+// dP1, dP2, dI, with dtheta [H/2] (fp32) and dtheta_part the per-CTA partials.
+struct LayerProblem {
+  const void* in1;
+  const void* in2;
+  const void* in3;
+  const void* in4;
+  void* out1;
+  void* out2;
+  void* out3;
+  const float* theta;   // [H/2] Givens angles, fp32, device
+  float* dtheta;        // [H/2], grad only
+  float* dtheta_part;   // grad only: caller workspace
+  int pairing;          // 0: (0,1), (2,3), ...; 1: (1,2), ..., (H-1,0)
+  float rope_base;
+  int B, T, H, d;
+  long long sB, sT, sH;
+  relation_dtype dtype;
+};
+bool layer_supports(relation_dtype dt, int d, int H);
+size_t layer_grad_workspace_bytes(int B, int T, int H);
+cudaError_t launch_layer_prep(const LayerProblem& p, cudaStream_t s);
+cudaError_t launch_layer_grad(const LayerProblem& p, cudaStream_t s);
+
 int decode_chunks(int t_max);
 size_t decode_workspace_bytes(int B, int H, int t_max);
 cudaError_t launch_decode(const DecodeProblem& p, void* workspace, cudaStream_t s);

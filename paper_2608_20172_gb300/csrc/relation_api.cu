@@ -170,6 +170,69 @@ relation_status relation_linear_bwd(const void* p1, const void* p2, const void* 
   return from_cuda(rel::launch_linear_bwd(p, reinterpret_cast<cudaStream_t>(stream)));
 }
 
+namespace {
+
+relation_status check_layer(const relation_shape& shp, relation_dtype dt, int pairing,
+                            float rope_base) {
+  if (dt != RELATION_F32 && dt != RELATION_BF16) return RELATION_ERR_INVALID_ARG;
+  if (shp.B < 1 || shp.T < 1 || shp.H < 1 || shp.d_h < 1) return RELATION_ERR_INVALID_ARG;
+  if (shp.sB < 1 || shp.sT < 1 || shp.sH < 1) return RELATION_ERR_INVALID_ARG;
+  if (pairing != 0 && pairing != 1) return RELATION_ERR_INVALID_ARG;
+  if (!isfinite(rope_base) || !(rope_base > 0.0f)) return RELATION_ERR_INVALID_ARG;
+  if (!rel::layer_supports(dt, shp.d_h, shp.H)) return RELATION_ERR_UNSUPPORTED;
+  if ((long long)shp.B * ((shp.T + 15) / 16) > 0x7fffffffLL) return RELATION_ERR_UNSUPPORTED;
+  const long long vec = 16 / (long long)elem_size(dt);
+  if (shp.sB % vec || shp.sT % vec || shp.sH % vec) return RELATION_ERR_ALIGNMENT;
+  return RELATION_OK;
+}
+
+rel::LayerProblem layer_problem(const relation_shape& shp, relation_dtype dt, int pairing,
+                                float rope_base, const float* theta) {
+  rel::LayerProblem p{};
+  p.theta = theta; p.pairing = pairing; p.rope_base = rope_base;
+  p.B = shp.B; p.T = shp.T; p.H = shp.H; p.d = shp.d_h;
+  p.sB = shp.sB; p.sT = shp.sT; p.sH = shp.sH; p.dtype = dt;
+  return p;
+}
+
+}  // namespace
+
+relation_status relation_layer_prep(const void* p1, const void* p2, const void* info,
+                                    const float* theta, int pairing, float rope_base, void* q,
+                                    void* k, void* v, relation_shape shp, relation_dtype dt,
+                                    relation_stream_t stream) {
+  relation_status st;
+  if ((st = check_layer(shp, dt, pairing, rope_base)) != RELATION_OK) return st;
+  if ((st = check_ptrs({p1, p2, info, q, k, v})) != RELATION_OK) return st;
+  if (!theta || (reinterpret_cast<uintptr_t>(theta) & 3u)) return RELATION_ERR_INVALID_ARG;
+  rel::LayerProblem p = layer_problem(shp, dt, pairing, rope_base, theta);
+  p.in1 = p1; p.in2 = p2; p.in3 = info; p.out1 = q; p.out2 = k; p.out3 = v;
+  return from_cuda(rel::launch_layer_prep(p, reinterpret_cast<cudaStream_t>(stream)));
+}
+
+size_t relation_layer_grad_workspace_size(relation_shape shp, relation_dtype dt) {
+  if (check_layer(shp, dt, 0, 1.0f) != RELATION_OK) return 0;
+  return rel::layer_grad_workspace_bytes(shp.B, shp.T, shp.H);
+}
+
+relation_status relation_layer_grad(const void* dq, const void* dk, const void* dv,
+                                    const void* info, const float* theta, int pairing,
+                                    float rope_base, void* dp1, void* dp2, void* dinfo,
+                                    float* dtheta, relation_shape shp, relation_dtype dt,
+                                    void* workspace, size_t ws_bytes, relation_stream_t stream) {
+  relation_status st;
+  if ((st = check_layer(shp, dt, pairing, rope_base)) != RELATION_OK) return st;
+  if ((st = check_ptrs({dq, dk, dv, info, dp1, dp2, dinfo, workspace})) != RELATION_OK) return st;
+  if (!theta || (reinterpret_cast<uintptr_t>(theta) & 3u)) return RELATION_ERR_INVALID_ARG;
+  if (!dtheta || (reinterpret_cast<uintptr_t>(dtheta) & 3u)) return RELATION_ERR_INVALID_ARG;
+  if (ws_bytes < rel::layer_grad_workspace_bytes(shp.B, shp.T, shp.H)) return RELATION_ERR_WORKSPACE;
+  rel::LayerProblem p = layer_problem(shp, dt, pairing, rope_base, theta);
+  p.in1 = dq; p.in2 = dk; p.in3 = dv; p.in4 = info;
+  p.out1 = dp1; p.out2 = dp2; p.out3 = dinfo;
+  p.dtheta = dtheta; p.dtheta_part = reinterpret_cast<float*>(workspace);
+  return from_cuda(rel::launch_layer_grad(p, reinterpret_cast<cudaStream_t>(stream)));
+}
+
 size_t relation_decode_workspace_size(relation_shape cache, relation_dtype dt) {
   if (dt != RELATION_F32 && dt != RELATION_BF16) return 0;
   if (cache.B < 1 || cache.T < 1 || cache.H < 1 || cache.d_h < 1 || cache.d_h > 128) return 0;

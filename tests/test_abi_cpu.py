@@ -147,3 +147,53 @@ def test_binding_refuses_cpu_tensors():
 def test_missing_library_fails_loudly(tmp_path):
     with pytest.raises(binding.RelationLibraryMissing):
         binding.load(str(tmp_path / "nope.so"))
+
+
+@pytest.mark.parametrize("case,expect", [
+    ("odd H", binding.ERR_UNSUPPORTED),
+    ("d = 36", binding.ERR_UNSUPPORTED),
+    ("d = 264", binding.ERR_UNSUPPORTED),
+    ("pairing 2", binding.ERR_INVALID_ARG),
+    ("base 0", binding.ERR_INVALID_ARG),
+    ("null theta", binding.ERR_INVALID_ARG),
+    ("misaligned k", binding.ERR_ALIGNMENT),
+    ("odd stride", binding.ERR_ALIGNMENT),
+])
+def test_layer_prep_rejects_bad_arguments(lib, case, expect):
+    p = [ctypes.c_void_p(0x10000 * (i + 1)) for i in range(6)]
+    theta = ctypes.c_void_p(0x90000)
+    shape, pairing, base = _shape(H=4), 0, 1.0e4
+    if case == "odd H":
+        shape = _shape(H=3)
+    elif case == "d = 36":
+        shape = _shape(H=4, d=36)
+    elif case == "d = 264":
+        shape = _shape(H=4, d=264)
+    elif case == "pairing 2":
+        pairing = 2
+    elif case == "base 0":
+        base = 0.0
+    elif case == "null theta":
+        theta = None
+    elif case == "misaligned k":
+        p[4] = ctypes.c_void_p(0x50008)
+    elif case == "odd stride":
+        shape = _shape(H=4, sT=260)
+    rc = lib.relation_layer_prep(p[0], p[1], p[2], theta, pairing, base, p[3], p[4], p[5], shape,
+                                 binding.BF16, None)
+    assert rc == expect
+
+
+def test_layer_grad_workspace_rules(lib):
+    shape = _shape(B=2, T=100, H=4, d=64)
+    need = lib.relation_layer_grad_workspace_size(shape, binding.BF16)
+    assert need == 2 * ((100 + 15) // 16) * 2 * 4  # one fp32 partial per CTA and head pair
+    assert lib.relation_layer_grad_workspace_size(_shape(H=3), binding.BF16) == 0
+    p = [ctypes.c_void_p(0x10000 * (i + 1)) for i in range(7)]
+    theta, dtheta = ctypes.c_void_p(0x90000), ctypes.c_void_p(0xA0000)
+    rc = lib.relation_layer_grad(p[0], p[1], p[2], p[3], theta, 0, 1.0e4, p[4], p[5], p[6], dtheta,
+                                 shape, binding.BF16, ctypes.c_void_p(0x100000), need - 1, None)
+    assert rc == binding.ERR_WORKSPACE
+    rc = lib.relation_layer_grad(p[0], p[1], p[2], p[3], theta, 0, 1.0e4, p[4], p[5], p[6], None,
+                                 shape, binding.BF16, ctypes.c_void_p(0x100000), need, None)
+    assert rc == binding.ERR_INVALID_ARG
