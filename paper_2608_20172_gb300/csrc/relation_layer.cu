@@ -18,8 +18,8 @@
 // once in shared memory and reused by every head: m * base^(-2c/d) is formed and reduced
 // modulo 2 pi in fp64 (positions reach 16k, where an fp32 angle would be off by ~1e-3
 // rad), then its cosine and sine are taken in fp32.  dtheta is summed per CTA in a fixed
-// order and the partials are added up in fp64 by a second, single-block kernel
-// (deterministic).
+// order and the partials are added up in fp64 by a second kernel, one block per head
+// pair (deterministic).
 #include <math.h>
 
 #include "common.cuh"
@@ -265,22 +265,19 @@ __global__ void __launch_bounds__(kThreads) grad_kernel(LayerProblem p) {
   }
 }
 
-// dtheta_k = sum over CTAs of the partials, in fp64 and a fixed order
+// dtheta_k = sum over CTAs of the partials, in fp64 and a fixed order; one block per pair
 __global__ void __launch_bounds__(256) dtheta_kernel(LayerProblem p, int n_cta) {
   __shared__ double red[256];
-  const int np = p.H / 2;
-  for (int k = 0; k < np; ++k) {
-    double s = 0.0;
-    for (int c = threadIdx.x; c < n_cta; c += 256) s += (double)p.dtheta_part[(long long)c * np + k];
-    red[threadIdx.x] = s;
-    __syncthreads();
-    for (int w = 128; w > 0; w >>= 1) {
-      if (threadIdx.x < w) red[threadIdx.x] += red[threadIdx.x + w];
-      __syncthreads();
-    }
-    if (threadIdx.x == 0) p.dtheta[k] = (float)red[0];
+  const int np = p.H / 2, k = blockIdx.x;
+  double s = 0.0;
+  for (int c = threadIdx.x; c < n_cta; c += 256) s += (double)p.dtheta_part[(long long)c * np + k];
+  red[threadIdx.x] = s;
+  __syncthreads();
+  for (int w = 128; w > 0; w >>= 1) {
+    if (threadIdx.x < w) red[threadIdx.x] += red[threadIdx.x + w];
     __syncthreads();
   }
+  if (threadIdx.x == 0) p.dtheta[k] = (float)red[0];
 }
 
 int ctas(const LayerProblem& p) { return p.B * ((p.T + kTok - 1) / kTok); }
@@ -315,7 +312,7 @@ cudaError_t launch_layer_grad(const LayerProblem& p, cudaStream_t s) {
     layer::grad_kernel<__nv_bfloat16><<<grid, layer::kThreads, 0, s>>>(p);
   cudaError_t e = cudaGetLastError();
   if (e != cudaSuccess) { note_failure("layer grad: launch"); return e; }
-  layer::dtheta_kernel<<<1, 256, 0, s>>>(p, grid);
+  layer::dtheta_kernel<<<p.H / 2, 256, 0, s>>>(p, grid);
   if ((e = cudaGetLastError()) != cudaSuccess) note_failure("layer grad: dtheta launch");
   return e;
 }
