@@ -15,8 +15,10 @@
 // kernel's per-query scalars, zeroed fp32 dQ accumulator), the tile kernel, and a
 // finalisation (dQ to bf16, dlambda reduction).
 //
-// Tile kernel: one CTA per 128 keys of one head, visiting query tiles from the diagonal
-// to the end of the sequence.  Keys sit on TMEM lanes.  Per step of 64 query columns:
+// Tile kernel: a unit is 128 keys of one head, visiting query tiles from the diagonal to
+// the end of the sequence; d_h = 64 runs one persistent CTA per SM over the units (K/V
+// double-buffered, the next unit's first steps issued before the current unit's last dQ),
+// d_h = 128 one CTA per unit.  Keys sit on TMEM lanes.  Per step of 64 query columns:
 //   MMA  U^T = K Q^T,  dP^T = V dO^T                          (TMEM, fp32)
 //   elementwise (thread = key): P = F in bf16 back into TMEM, dS' = 2 dS in bf16 into
 //        128-byte-swizzled shared memory, and the Exchange part of dlambda
