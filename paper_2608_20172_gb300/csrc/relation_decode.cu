@@ -114,27 +114,38 @@ __global__ void __launch_bounds__(kWarps * 32) partial_kernel(DecodeProblem p, f
   constexpr int PL = D > 0 ? D / 32 : kMaxD / 32;  // columns per lane in the P V pass
   float mx = -INFINITY;
   if constexpr (D > 0) {
-    // scores: lane = 4 key + quarter; keys jj = 8 (warp + kWarps it) + lane / 4
+    // scores: lane = 4 key + quarter; per iteration two groups of 8 keys,
+    // jj = base + lane / 4 and jj + 8 kWarps, loaded together (rows past the chunk read a
+    // clamped row and are dropped)
     constexpr int QD = D / 4;
     const int sub = lane & 3, slot = lane >> 2;
     float qr[QD];
     ld_vec<TI, QD>(qv + sub * QD, qr);
-    for (int base = warp * 8; base < n; base += 8 * kWarps) {
-      const int jj = base + slot;
-      float kr[QD];
-      if (jj < n) ld_vec<TI, QD>(kc + (long long)jj * p.sT + sub * QD, kr);
-      else
+    for (int base = warp * 8; base < n; base += 16 * kWarps) {
+      const int j0 = base + slot, j1 = j0 + 8 * kWarps;
+      float k0[QD], k1[QD];
+      ld_vec<TI, QD>(kc + (long long)min(j0, n - 1) * p.sT + sub * QD, k0);
+      ld_vec<TI, QD>(kc + (long long)min(j1, n - 1) * p.sT + sub * QD, k1);
+      float s0 = 0.f, s1 = 0.f;
 #pragma unroll
-        for (int e = 0; e < QD; ++e) kr[e] = 0.f;
-      float s = 0.f;
-#pragma unroll
-      for (int e = 0; e < QD; ++e) s = fmaf(qr[e], kr[e], s);
-      s += __shfl_xor_sync(0xffffffffu, s, 1);
-      s += __shfl_xor_sync(0xffffffffu, s, 2);
-      if (jj < n) {
-        const float u = s * p.inv_sqrt_d;
+      for (int e = 0; e < QD; ++e) {
+        s0 = fmaf(qr[e], k0[e], s0);
+        s1 = fmaf(qr[e], k1[e], s1);
+      }
+      s0 += __shfl_xor_sync(0xffffffffu, s0, 1);
+      s1 += __shfl_xor_sync(0xffffffffu, s1, 1);
+      s0 += __shfl_xor_sync(0xffffffffu, s0, 2);
+      s1 += __shfl_xor_sync(0xffffffffu, s1, 2);
+      if (j0 < n) {
+        const float u = s0 * p.inv_sqrt_d;
         const float E = u / (1.0f + expf(-u));  // SiLU(u)
-        if (sub == 0) e_s[jj] = E;
+        if (sub == 0) e_s[j0] = E;
+        mx = fmaxf(mx, E);
+      }
+      if (j1 < n) {
+        const float u = s1 * p.inv_sqrt_d;
+        const float E = u / (1.0f + expf(-u));
+        if (sub == 0) e_s[j1] = E;
         mx = fmaxf(mx, E);
       }
     }
@@ -175,7 +186,7 @@ __global__ void __launch_bounds__(kWarps * 32) partial_kernel(DecodeProblem p, f
   for (int e = 0; e < PL; ++e) z[e] = 0.f;
   if constexpr (D > 0) {
     const int col = lane * PL;
-#pragma unroll 4
+#pragma unroll 8
     for (int jj = warp; jj < n; jj += kWarps) {
       const float P = expf(e_s[jj] - m);
       l += P;
