@@ -119,9 +119,6 @@ __device__ __forceinline__ void tma_store_4d(const CUtensorMap* m, uint32_t src,
 __device__ __forceinline__ void tma_store_commit() {
   asm volatile("cp.async.bulk.commit_group;" ::: "memory");
 }
-__device__ __forceinline__ void tma_store_wait_all() {
-  asm volatile("cp.async.bulk.wait_group 0;" ::: "memory");
-}
 // Wait until every committed bulk store / reduce has finished reading shared memory (its
 // global writes may still be in flight; they complete before the kernel does).  Enough
 // before a CTA releases or reuses the staging buffers.
