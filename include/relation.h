@@ -31,8 +31,9 @@
  *    launched.  A kernel whose pipeline wait exceeds its bound writes
  *    RELATION_ERR_TIMEOUT into *dev_status (a device int the caller zeroes and reads
  *    after synchronising; may be NULL) and returns without finishing its tile.
- *  - Supported: fp32 with d_h in {32, 64, 128}; bf16 with d_h in {32, 64, 128}
- *    (d_h 64 and 128 run on the tcgen05 tensor-core kernels).  Any T >= 1.
+ *  - Supported: fp32 with d_h in {32, 64, 128} (CUDA-core kernels); bf16 with any d_h
+ *    that is a multiple of 8 up to 128 (tcgen05 tensor-core kernels, zero-padded to 64
+ *    or 128 inside; d_h 32, 64 and 128 also on the CUDA-core kernels).  Any T >= 1.
  *  - Alignment: every tensor pointer 16-byte aligned and sB, sT, sH multiples of
  *    16 bytes / element size; workspace 256-byte aligned.
  */
@@ -83,8 +84,9 @@ relation_status relation_fwd(const void* q, const void* k, const void* v, void* 
                              int* dev_status, relation_stream_t stream);
 
 /* Kernel family selection for the *_ex entry points.  AUTO takes the tcgen05
- * tensor-core kernels where they exist (bf16, d_h 64 or 128) and the CUDA-core (SIMT)
- * kernels otherwise; TCGEN05 returns RELATION_ERR_UNSUPPORTED where they do not exist. */
+ * tensor-core kernels where they exist (bf16, d_h a multiple of 8 up to 128) and the
+ * CUDA-core (SIMT) kernels otherwise; TCGEN05 returns RELATION_ERR_UNSUPPORTED where they
+ * do not exist. */
 typedef enum relation_kernel {
   RELATION_KERNEL_AUTO = 0,
   RELATION_KERNEL_SIMT = 1,
