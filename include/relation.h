@@ -124,7 +124,7 @@ relation_status relation_fwd_flow(const void* q, const void* k, const void* v, v
  *               parameterisation of Eq. (retention-vector) is upstream), with the same
  *               element strides as p1.
  *   y         : [B][T][H][d_h] output in dt, same strides.
- * fp32 or bf16 with d_h in {32, 64} (other widths: RELATION_ERR_UNSUPPORTED); the state is
+ * fp32 or bf16 with d_h in {32, 64, 128} (other widths: RELATION_ERR_UNSUPPORTED); the state is
  * kept in fp32.  A zero p1 or p2 row is outside the operator's domain.  Asynchronous on
  * `stream`; nothing is allocated.
  */

@@ -136,7 +136,7 @@ constexpr int kChunkF = 16;  // tokens per staged chunk (forward)
 
 template <int D, int NS>
 struct FwdCfg {
-  static constexpr int NT = D == 64 ? 256 : 128;  // threads
+  static constexpr int NT = D == 32 ? 128 : 256;  // threads
   static constexpr int NC = D / NS;               // columns per CTA
   static constexpr int RG = NT / NC;              // row groups
   static constexpr int R = D / RG;                // rows per thread
@@ -218,9 +218,10 @@ __global__ void __launch_bounds__(FwdCfg<D, NS>::NT) fwd_kernel(LinearProblem p)
   }
 }
 
-// column splits: the forward at d_h = 64 runs 4 CTAs per head, at d_h = 32 two
+// column splits of the forward: 16 columns per CTA (d_h = 32: 2 CTAs per head, 64: 4,
+// 128: 8)
 template <int D>
-constexpr int fwd_splits() { return D == 64 ? 4 : 2; }
+constexpr int fwd_splits() { return D / 16; }
 
 template <typename TI, int D>
 cudaError_t fwd_t(const LinearProblem& p, cudaStream_t s) {
@@ -256,10 +257,10 @@ constexpr int kChunkB = 8;   // tokens per checkpoint / recomputed sub-chunk
 constexpr int kStageB = 16;  // tokens per staged chunk (two sub-chunks)
 constexpr int kQ = 4;        // threads per state row (each a quarter of the columns)
 
-// column splits of the backward: two CTAs per head at d_h = 64, one at d_h = 32 (the
-// reduce-scatter below needs R = NC / kQ >= 32 / kQ)
+// column splits of the backward: 32 columns per CTA (d_h = 32: one CTA per head, 64: 2,
+// 128: 4; the reduce-scatter below needs R = NC / kQ >= 32 / kQ)
 template <int D>
-constexpr int bwd_splits() { return D == 64 ? 2 : 1; }
+constexpr int bwd_splits() { return D / 32; }
 
 template <int D>
 struct BwdSmem {
@@ -527,25 +528,31 @@ cudaError_t bwd_t(const LinearProblem& p, cudaStream_t s) {
 }  // namespace lin
 
 size_t linear_bwd_workspace_bytes(int B, int H, int T, int d) {
-  const long long per = d == 32 ? lin::ckpt_floats<32>(T) : lin::ckpt_floats<64>(T);
-  const int ns = d == 32 ? lin::bwd_splits<32>() : lin::bwd_splits<64>();
+  const long long per = (long long)((T + lin::kChunkB - 1) / lin::kChunkB) * d * d;
+  const int ns = d / 32;  // bwd_splits
   return (size_t)((long long)B * H * per + (long long)B * H * ns * T * 3 * d) * sizeof(float);
 }
 
 cudaError_t launch_linear_bwd(const LinearProblem& p, cudaStream_t s) {
   if (p.dtype == RELATION_F32)
-    return p.d == 32 ? lin::bwd_t<float, 32>(p, s) : lin::bwd_t<float, 64>(p, s);
-  return p.d == 32 ? lin::bwd_t<__nv_bfloat16, 32>(p, s) : lin::bwd_t<__nv_bfloat16, 64>(p, s);
+    return p.d == 32 ? lin::bwd_t<float, 32>(p, s)
+                     : p.d == 64 ? lin::bwd_t<float, 64>(p, s) : lin::bwd_t<float, 128>(p, s);
+  return p.d == 32 ? lin::bwd_t<__nv_bfloat16, 32>(p, s)
+                   : p.d == 64 ? lin::bwd_t<__nv_bfloat16, 64>(p, s)
+                               : lin::bwd_t<__nv_bfloat16, 128>(p, s);
 }
 
 bool linear_supports(relation_dtype dt, int d) {
-  return (dt == RELATION_F32 || dt == RELATION_BF16) && (d == 32 || d == 64);
+  return (dt == RELATION_F32 || dt == RELATION_BF16) && (d == 32 || d == 64 || d == 128);
 }
 
 cudaError_t launch_linear_fwd(const LinearProblem& p, cudaStream_t s) {
   if (p.dtype == RELATION_F32)
-    return p.d == 32 ? lin::fwd_t<float, 32>(p, s) : lin::fwd_t<float, 64>(p, s);
-  return p.d == 32 ? lin::fwd_t<__nv_bfloat16, 32>(p, s) : lin::fwd_t<__nv_bfloat16, 64>(p, s);
+    return p.d == 32 ? lin::fwd_t<float, 32>(p, s)
+                     : p.d == 64 ? lin::fwd_t<float, 64>(p, s) : lin::fwd_t<float, 128>(p, s);
+  return p.d == 32 ? lin::fwd_t<__nv_bfloat16, 32>(p, s)
+                   : p.d == 64 ? lin::fwd_t<__nv_bfloat16, 64>(p, s)
+                               : lin::fwd_t<__nv_bfloat16, 128>(p, s);
 }
 
 }  // namespace rel

@@ -23,7 +23,7 @@ def _heads(x, b, h):
 
 
 @pytest.mark.parametrize("dtype", ["fp32", "bf16"])
-@pytest.mark.parametrize("d", [32, 64])
+@pytest.mark.parametrize("d", [32, 64, 128])
 @pytest.mark.parametrize("T", [1, 17, 200])
 def test_linear_forward(dtype, d, T):
     w = workloads.custom(2, 2, T, d, dtype)
@@ -42,7 +42,7 @@ def test_linear_forward(dtype, d, T):
 
 
 @pytest.mark.parametrize("dtype", ["fp32", "bf16"])
-@pytest.mark.parametrize("d", [32, 64])
+@pytest.mark.parametrize("d", [32, 64, 128])
 @pytest.mark.parametrize("T", [1, 8, 9, 100])
 def test_linear_backward(dtype, d, T):
     """Gradients of every input, including the retention, against the oracle's reverse-
