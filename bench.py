@@ -506,6 +506,8 @@ def run_ours(args, w):
         "tokens_per_s": ws * w.tokens / (ms * 1e-3),
         "pct_bf16_peak": 100.0 * tflops / (ws * peaks["bf16_tflops"]),
         "pct_bf16_peak_sustained": 100.0 * tflops / (ws * peaks["bf16_tflops_sustained"]),
+        # the same time under the algorithmic minimum without the U recompute, 6 B H T^2 d
+        "tflops_6bht2d": tflops * 6.0 / 7.0,
         "ms_fwd": ms_fwd, "ms_bwd": ms_bwd,
         "ms_bwd_stages": {"prepare": ms_pre, "tiles": ms_tiles, "finalize": ms_fin},
         "fwd_tflops": ws * fwd_tflops,
