@@ -125,8 +125,9 @@ relation_status relation_fwd_flow(const void* q, const void* k, const void* v, v
  *               element strides as p1.
  *   y         : [B][T][H][d_h] output in dt, same strides.
  * fp32 or bf16 with d_h in {32, 64, 128} (other widths: RELATION_ERR_UNSUPPORTED); the state is
- * kept in fp32.  A zero p1 or p2 row is outside the operator's domain.  Asynchronous on
- * `stream`; nothing is allocated.
+ * kept in fp32.  Element strides sB, sT, sH must be multiples of 4 and every pointer
+ * 16-byte aligned (else RELATION_ERR_ALIGNMENT).  A zero p1 or p2 row is outside the
+ * operator's domain.  Asynchronous on `stream`; nothing is allocated.
  */
 relation_status relation_linear_fwd(const void* p1, const void* p2, const void* v,
                                    const float* alpha, void* y, float tau_s, relation_shape shp,

@@ -197,3 +197,67 @@ def test_layer_grad_workspace_rules(lib):
     rc = lib.relation_layer_grad(p[0], p[1], p[2], p[3], theta, 0, 1.0e4, p[4], p[5], p[6], None,
                                  shape, binding.BF16, ctypes.c_void_p(0x100000), need, None)
     assert rc == binding.ERR_INVALID_ARG
+
+
+@pytest.mark.parametrize("case,expect", [
+    ("d = 48", binding.ERR_UNSUPPORTED),
+    ("stride not a multiple of 4", binding.ERR_ALIGNMENT),
+    ("null alpha", binding.ERR_INVALID_ARG),
+    ("tau = 0", binding.ERR_INVALID_ARG),
+    ("misaligned y", binding.ERR_ALIGNMENT),
+])
+def test_linear_rejects_bad_arguments(lib, case, expect):
+    p = [ctypes.c_void_p(0x10000 * (i + 1)) for i in range(5)]
+    shape, tau = _shape(d=64), 2.0
+    if case == "d = 48":
+        shape = _shape(d=48)
+    elif case == "stride not a multiple of 4":
+        shape = _shape(d=64, sH=66, sT=2 * 66, sB=8 * 2 * 66)
+    elif case == "null alpha":
+        p[3] = None
+    elif case == "tau = 0":
+        tau = 0.0
+    elif case == "misaligned y":
+        p[4] = ctypes.c_void_p(0x50004)
+    rc = lib.relation_linear_fwd(p[0], p[1], p[2], p[3], p[4], tau, shape, binding.BF16, None,
+                                 None)
+    assert rc == expect
+
+
+def test_linear_bwd_workspace_rules(lib):
+    shape = _shape(B=2, T=20, H=3, d=64)
+    need = lib.relation_linear_bwd_workspace_size(shape, binding.BF16)
+    # checkpoints every 8 tokens (3 of 64 x 64) plus the column splits' partial row sums
+    assert need == (2 * 3 * 3 * 64 * 64 + 2 * 3 * 2 * 20 * 3 * 64) * 4
+    assert lib.relation_linear_bwd_workspace_size(_shape(d=48), binding.BF16) == 0
+    p = [ctypes.c_void_p(0x10000 * (i + 1)) for i in range(9)]
+    rc = lib.relation_linear_bwd(*p, 2.0, shape, binding.BF16, ctypes.c_void_p(0x100000), need - 1,
+                                 None, None)
+    assert rc == binding.ERR_WORKSPACE
+
+
+@pytest.mark.parametrize("case,expect", [
+    ("d = 136", binding.ERR_UNSUPPORTED),
+    ("null lengths", binding.ERR_INVALID_ARG),
+    ("lambda nan", binding.ERR_INVALID_ARG),
+    ("small workspace", binding.ERR_WORKSPACE),
+    ("q stride 0", binding.ERR_INVALID_ARG),
+])
+def test_decode_rejects_bad_arguments(lib, case, expect):
+    p = [ctypes.c_void_p(0x10000 * (i + 1)) for i in range(6)]
+    cache, lam, qsB, qsH = _shape(B=2, T=64, H=2, d=64), 0.5, 128, 64
+    need = lib.relation_decode_workspace_size(cache, binding.BF16)
+    ws = need
+    if case == "d = 136":
+        cache = _shape(B=2, T=64, H=2, d=136)
+    elif case == "null lengths":
+        p[3] = None
+    elif case == "lambda nan":
+        lam = float("nan")
+    elif case == "small workspace":
+        ws = need - 1
+    elif case == "q stride 0":
+        qsB = 0
+    rc = lib.relation_decode(p[0], p[1], p[2], p[3], p[4], p[5], lam, 2.0, cache, qsB, qsH,
+                             binding.BF16, ctypes.c_void_p(0x100000), ws, None, None)
+    assert rc == expect
