@@ -127,7 +127,8 @@ relation_status relation_linear_fwd(const void* p1, const void* p2, const void* 
   if (shp.B < 1 || shp.T < 1 || shp.H < 1 || shp.d_h < 1) return RELATION_ERR_INVALID_ARG;
   if (shp.sB < 1 || shp.sT < 1 || shp.sH < 1) return RELATION_ERR_INVALID_ARG;
   if (!rel::linear_supports(dt, shp.d_h)) return RELATION_ERR_UNSUPPORTED;
-  if ((long long)shp.B * shp.H > 0x7fffffffLL) return RELATION_ERR_UNSUPPORTED;
+  // grid: up to 8 column splits per head
+  if ((long long)shp.B * shp.H * 8 > 0x7fffffffLL) return RELATION_ERR_UNSUPPORTED;
   // 4-element vector loads of every token row (alpha is fp32 with the same strides)
   if (shp.sB % 4 || shp.sT % 4 || shp.sH % 4) return RELATION_ERR_ALIGNMENT;
   if (!isfinite(tau_s) || !(tau_s > 0.0f)) return RELATION_ERR_INVALID_ARG;
@@ -156,7 +157,8 @@ relation_status relation_linear_bwd(const void* p1, const void* p2, const void* 
   if (shp.B < 1 || shp.T < 1 || shp.H < 1 || shp.d_h < 1) return RELATION_ERR_INVALID_ARG;
   if (shp.sB < 1 || shp.sT < 1 || shp.sH < 1) return RELATION_ERR_INVALID_ARG;
   if (!rel::linear_supports(dt, shp.d_h)) return RELATION_ERR_UNSUPPORTED;
-  if ((long long)shp.B * shp.H > 0x7fffffffLL) return RELATION_ERR_UNSUPPORTED;
+  // grid: up to 8 column splits per head
+  if ((long long)shp.B * shp.H * 8 > 0x7fffffffLL) return RELATION_ERR_UNSUPPORTED;
   // 4-element vector loads of every token row (alpha is fp32 with the same strides)
   if (shp.sB % 4 || shp.sT % 4 || shp.sH % 4) return RELATION_ERR_ALIGNMENT;
   if (!isfinite(tau_s) || !(tau_s > 0.0f)) return RELATION_ERR_INVALID_ARG;
