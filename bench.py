@@ -319,6 +319,48 @@ def layer_measure(binding, dev, peaks, steps=10, warmup=3):
             "gpu_launches_per_call": {"prep": 1, "grad": 2}}
 
 
+def sdpa_context(w, dev, steps=20, warmup=3):
+    """Context only, not this library: PyTorch's causal scaled-dot-product attention
+    (softmax attention, the paper's comparison operator) forward + backward on the same
+    B, H, T, d_h and dtype, counted with the same 7 B H T^2 d convention.  GPU: CUDA
+    events with the L2 flushed between steps; CPU (tests): wall clock."""
+    g = torch.Generator(device="cpu").manual_seed(0)
+    shape = (w.B, w.H, w.T, w.d)
+    dt = w.torch_dtype
+    q, k, v, do = (torch.randn(shape, generator=g).to(dt).to(dev) for _ in range(4))
+    q.requires_grad_(True)
+    k.requires_grad_(True)
+    v.requires_grad_(True)
+    cuda = dev.type == "cuda"
+    flush = torch.empty(L2_FLUSH_BYTES if cuda else 16, dtype=torch.uint8, device=dev)
+
+    def step():
+        out = torch.nn.functional.scaled_dot_product_attention(q, k, v, is_causal=True)
+        out.backward(do)
+        q.grad = k.grad = v.grad = None
+
+    for _ in range(warmup):
+        step()
+    times = []
+    for _ in range(steps):
+        flush.zero_()
+        if cuda:
+            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            e0.record()
+            step()
+            e1.record()
+            torch.cuda.synchronize(dev)
+            times.append(e0.elapsed_time(e1))
+        else:
+            t0 = time.perf_counter()
+            step()
+            times.append((time.perf_counter() - t0) * 1e3)
+    ms = statistics.mean(times)
+    return {"operator": "torch scaled_dot_product_attention, causal (softmax attention)",
+            "ms_per_step": ms, "tflops": w.flops_fwd_bwd() / (ms * 1e-3) / 1e12,
+            "note": "context only: a different operator through PyTorch's kernels"}
+
+
 LINEAR_CFG = {"B": 8, "H": 12, "T": 2048, "d_h": 64}  # the 100M layer geometry, bf16
 FP32_FMA_TFLOPS = 152 * 128 * 2 * 2.07e9 / 1e12  # 152 SMs x 128 FFMA lanes x 2 flops x 2.07 GHz
 
@@ -533,6 +575,10 @@ def run_ours(args, w):
         line["decode"] = decode_measure(binding, dev, peaks)
         line["linear"] = linear_measure(binding, dev)
         line["layer"] = layer_measure(binding, dev, peaks)
+        try:
+            line["context_sdpa"] = sdpa_context(w, dev)
+        except Exception as exc:  # context only: never at the expense of the line
+            line["context_sdpa"] = {"not_measured": f"{type(exc).__name__}: {exc}"[:200]}
     if rank == 0 and not args.no_cpu_baseline and ws == 1:
         cb = cpu_oracle_run(w, min_seconds=10.0)
         line["cpu_baseline"] = {

@@ -80,3 +80,12 @@ def test_max_over_ranks_gloo(tmp_path):
 
 def test_max_over_ranks_single_process_is_identity():
     assert bench._max_over_ranks(None, 2.25, torch.device("cpu")) == 2.25
+
+
+def test_sdpa_context_runs_on_cpu():
+    """The context measurement's code path (PyTorch SDPA fwd+bwd, same flop convention)."""
+    from paper_2608_20172_gb300 import workloads
+    w = workloads.custom(1, 2, 64, 16, "fp32")
+    r = bench.sdpa_context(w, torch.device("cpu"), steps=2, warmup=1)
+    assert r["ms_per_step"] > 0 and r["tflops"] > 0
+    assert "context only" in r["note"]
