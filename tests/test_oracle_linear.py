@@ -174,3 +174,52 @@ def test_linear_mutant_is_caught(mutant):
             except (AssertionError, ValueError, FloatingPointError):
                 caught.append(pin.__name__)
         assert caught, f"no pin catches the planted mistake '{name}'"
+
+
+# --- the chunked (block-parallel) evaluation, pinned to the recurrence -------------
+
+def pin_chunked_equals_recurrent(ch, lo=None):
+    """oracle/linear_chunked.py regroups the recurrence into blocks of L tokens; for every
+    block size its Y equals the recurrent oracle's (which covers the state handed from
+    block to block whenever T > L)."""
+    lo = lo or oracle.linear()
+    for T, d, seed in [(1, 3, 40), (7, 4, 41), (20, 6, 42)]:
+        p1, p2, v, a = _inputs(T, d, seed, 0.3, 1.0)
+        y, _ = lo.fwd(p1, p2, v, a)
+        for L in sorted({1, 2, 3, 5, 8, T}):
+            yc, _ = ch.linear_fwd_chunked(p1, p2, v, a, L)
+            assert np.abs(yc - y).max() <= 1e-12 * max(1.0, np.abs(y).max()), (T, d, L)
+
+
+def test_chunked_oracle_pin():
+    from oracle import linear_chunked
+    pin_chunked_equals_recurrent(linear_chunked)
+
+
+CHUNKED_MUTANTS = [
+    ("current token in its own read", "A = np.tril(Qb @ Kb.T, -1)", "A = np.tril(Qb @ Kb.T, 0)"),
+    ("inter-block term dropped", "Y[sl] = v[sl] + Qb @ C + A @ v[sl]",
+     "Y[sl] = v[sl] + A @ v[sl]"),
+    ("state not decayed across the block", "C = a[-1][:, None] * C + (a[-1] * Kb).T @ v[sl]",
+     "C = C + (a[-1] * Kb).T @ v[sl]"),
+    ("exclusive cumulative retention", "a = np.cumprod(alpha[sl], axis=0)",
+     "a = np.cumprod(alpha[sl], axis=0) / alpha[sl]"),
+]
+
+
+@pytest.mark.parametrize("mutant", CHUNKED_MUTANTS, ids=[m[0] for m in CHUNKED_MUTANTS])
+def test_chunked_mutant_is_caught(mutant):
+    import importlib.util
+    from oracle import linear_chunked
+    name, old, new = mutant
+    src = open(linear_chunked.__file__).read()
+    assert src.count(old) == 1, f"mutation site for '{name}' not unique/not found"
+    with tempfile.TemporaryDirectory() as tmp:
+        path = os.path.join(tmp, "chunked_mutant.py")
+        with open(path, "w") as f:
+            f.write(src.replace(old, new))
+        spec = importlib.util.spec_from_file_location("chunked_mutant", path)
+        mod = importlib.util.module_from_spec(spec)
+        spec.loader.exec_module(mod)
+        with pytest.raises(AssertionError):
+            pin_chunked_equals_recurrent(mod)
