@@ -10,8 +10,9 @@ materialised forward, App. A.1.2-A.1.8 for the factorised form, App. A.3 for the
 tiled Exchange scan and App. A.1.7 for the two backward derivations.
 ``linear_oracle.c`` (plain C, fp64) holds Linear Relation (Sec. 5.2, App. A.4): the
 recurrent step, its unrolled form and the reverse-mode backward of the recurrence.
-``linear_chunked.py`` (plain numpy, fp64) evaluates the same Linear Relation forward block
-by block (the form a block-parallel kernel computes), pinned to the recurrence.
+``linear_chunked.py`` (plain numpy, fp64) evaluates the same Linear Relation forward and
+backward block by block (the form a block-parallel kernel computes), pinned to the
+recurrence.
 ``layer.py`` (plain numpy, fp64) holds the layer's transforms around the operator: RoPE
 on P1, P2 and the Givens mixing of the information states, with their gradients.
 This module only marshals numpy arrays.

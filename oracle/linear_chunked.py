@@ -47,5 +47,62 @@ def linear_fwd_chunked(p1, p2, v, alpha, L: int, tau_s: float = 2.0):
         Kb = k[sl] / a
         A = np.tril(Qb @ Kb.T, -1)                 # strictly earlier tokens of the block
         Y[sl] = v[sl] + Qb @ C + A @ v[sl]         # Answer: I~ + inter + intra
-        C = a[-1][:, None] * C + (a[-1] * Kb).T @ v[sl]
+        C = a[-1][:, None] * C + (a[-1] * Kb).T @ v[sl]  # the state handed on
     return Y, C
+
+
+def linear_bwd_chunked(p1, p2, v, alpha, dy, L: int, tau_s: float = 2.0):
+    """(dp1, dp2, dv, dalpha) of L = sum(dy * Y) for the forward above, by reverse mode
+    through the block form, last block first, with dC the adjoint of the state a block
+    hands on.  Per block (C_0 the entering state, A = tril(Qb Kb^T, -1), Ka = a_L * Kb):
+        dI~  = dY + A^T dY + Ka dC
+        dA   = tril(dY I~^T, -1)
+        dQb  = dA Kb + dY C_0^T,      dKb = dA^T Qb + a_L * (I~ dC^T)
+        dC_0 = Qb^T dY + Diag(a_L) dC
+        da_t = dQb_t * q'_t - dKb_t * k'_t / a_t^2   (+ for t = L the state's a_L terms)
+        dalpha_u = sum_{t >= u} da_t * a_t / alpha_u
+    then dq' = a * dQb, dk' = dKb / a, and (dp1, dp2) through S and the normalisation."""
+    p1, p2, v, alpha, dy = (np.asarray(x, dtype=np.float64) for x in (p1, p2, v, alpha, dy))
+    T, d = p1.shape
+    S, q, k = _self_coords(p1, p2, tau_s)
+    # forward: the state entering every block
+    C = np.zeros((d, d))
+    starts = list(range(0, T, L))
+    C_in = []
+    for t0 in starts:
+        sl = slice(t0, min(T, t0 + L))
+        a = np.cumprod(alpha[sl], axis=0)
+        Kb = k[sl] / a
+        C_in.append(C)
+        C = a[-1][:, None] * C + (a[-1] * Kb).T @ v[sl]
+    dq, dk, dv, dal = (np.zeros((T, d)) for _ in range(4))
+    dC = np.zeros((d, d))
+    for t0, C0 in zip(reversed(starts), reversed(C_in)):
+        sl = slice(t0, min(T, t0 + L))
+        a = np.cumprod(alpha[sl], axis=0)
+        qs, ks, I, g = q[sl], k[sl], v[sl], dy[sl]
+        Qb, Kb = a * qs, ks / a
+        A = np.tril(Qb @ Kb.T, -1)
+        aL = a[-1]
+        Ka = aL * Kb
+        dv[sl] = g + A.T @ g + Ka @ dC
+        dA = np.tril(g @ I.T, -1)
+        dQb = dA @ Kb + g @ C0.T
+        dKb = dA.T @ Qb + aL * (I @ dC.T)
+        da = dQb * qs - dKb * ks / (a * a)
+        # C_L[c, :] = a_L[c] (C_0[c, :] + sum_t Kb_t[c] I~_t): the a_L factor
+        da[-1] += np.sum(dC * (C0 + Kb.T @ I), axis=1)
+        dal[sl] = np.cumsum((da * a)[::-1], axis=0)[::-1] / alpha[sl]
+        dq[sl] = a * dQb
+        dk[sl] = dKb / a
+        dC = Qb.T @ g + aL[:, None] * dC
+    # q' = S ^p1, k' = S ^p2, S = sigmoid(p1 . p2 / (tau_S sqrt d))
+    n1 = np.linalg.norm(p1, axis=1, keepdims=True)
+    n2 = np.linalg.norm(p2, axis=1, keepdims=True)
+    h1, h2 = p1 / n1, p2 / n2
+    dS = np.sum(dq * h1, axis=1) + np.sum(dk * h2, axis=1)
+    du = (dS * S * (1.0 - S) / (tau_s * np.sqrt(d)))[:, None]
+    g1, g2 = S[:, None] * dq, S[:, None] * dk
+    dp1 = (g1 - h1 * np.sum(h1 * g1, axis=1, keepdims=True)) / n1 + du * p2
+    dp2 = (g2 - h2 * np.sum(h2 * g2, axis=1, keepdims=True)) / n2 + du * p1
+    return dp1, dp2, dv, dal

@@ -197,13 +197,15 @@ def test_chunked_oracle_pin():
 
 
 CHUNKED_MUTANTS = [
-    ("current token in its own read", "A = np.tril(Qb @ Kb.T, -1)", "A = np.tril(Qb @ Kb.T, 0)"),
+    ("current token in its own read", "A = np.tril(Qb @ Kb.T, -1)                 # strictly",
+     "A = np.tril(Qb @ Kb.T, 0)                 # strictly"),
     ("inter-block term dropped", "Y[sl] = v[sl] + Qb @ C + A @ v[sl]",
      "Y[sl] = v[sl] + A @ v[sl]"),
-    ("state not decayed across the block", "C = a[-1][:, None] * C + (a[-1] * Kb).T @ v[sl]",
-     "C = C + (a[-1] * Kb).T @ v[sl]"),
-    ("exclusive cumulative retention", "a = np.cumprod(alpha[sl], axis=0)",
-     "a = np.cumprod(alpha[sl], axis=0) / alpha[sl]"),
+    ("state not decayed across the block",
+     "C = a[-1][:, None] * C + (a[-1] * Kb).T @ v[sl]  # the state handed on",
+     "C = C + (a[-1] * Kb).T @ v[sl]  # the state handed on"),
+    ("exclusive cumulative retention", "a = np.cumprod(alpha[sl], axis=0)          # a_t",
+     "a = np.cumprod(alpha[sl], axis=0) / alpha[sl]  # a_t"),
 ]
 
 
@@ -223,3 +225,53 @@ def test_chunked_mutant_is_caught(mutant):
         spec.loader.exec_module(mod)
         with pytest.raises(AssertionError):
             pin_chunked_equals_recurrent(mod)
+
+
+def pin_chunked_backward_equals_recurrent(ch, lo=None):
+    """The block-form backward equals the recurrent oracle's reverse mode for every block
+    size (all four gradients)."""
+    lo = lo or oracle.linear()
+    rng = np.random.default_rng(43)
+    for T, d in [(1, 3), (7, 4), (20, 6)]:
+        p1, p2, v, dy = (rng.standard_normal((T, d)) for _ in range(4))
+        a = rng.uniform(0.3, 1.0, (T, d))
+        ref = lo.bwd(p1, p2, v, a, dy)
+        for L in sorted({1, 2, 3, 5, 8, T}):
+            got = ch.linear_bwd_chunked(p1, p2, v, a, dy, L)
+            for name, x, y in zip(("dp1", "dp2", "dv", "dalpha"), got, ref):
+                assert np.abs(x - y).max() <= 1e-11 * max(1.0, np.abs(y).max()), (T, d, L, name)
+
+
+def test_chunked_backward_pin():
+    from oracle import linear_chunked
+    pin_chunked_backward_equals_recurrent(linear_chunked)
+
+
+CHUNKED_BWD_MUTANTS = [
+    ("dI~ misses the state's adjoint", "dv[sl] = g + A.T @ g + Ka @ dC", "dv[sl] = g + A.T @ g"),
+    ("dC_0 not decayed", "dC = Qb.T @ g + aL[:, None] * dC", "dC = Qb.T @ g + dC"),
+    ("a_L factor of the handed-on state dropped",
+     "da[-1] += np.sum(dC * (C0 + Kb.T @ I), axis=1)", "da[-1] += np.sum(dC * C0, axis=1)"),
+    ("retention gradient not accumulated over later tokens",
+     "dal[sl] = np.cumsum((da * a)[::-1], axis=0)[::-1] / alpha[sl]",
+     "dal[sl] = da * a / alpha[sl]"),
+    ("inter-block read missing from dQb", "dQb = dA @ Kb + g @ C0.T", "dQb = dA @ Kb"),
+]
+
+
+@pytest.mark.parametrize("mutant", CHUNKED_BWD_MUTANTS, ids=[m[0] for m in CHUNKED_BWD_MUTANTS])
+def test_chunked_backward_mutant_is_caught(mutant):
+    import importlib.util
+    from oracle import linear_chunked
+    name, old, new = mutant
+    src = open(linear_chunked.__file__).read()
+    assert src.count(old) == 1, f"mutation site for '{name}' not unique/not found"
+    with tempfile.TemporaryDirectory() as tmp:
+        path = os.path.join(tmp, "chunked_bwd_mutant.py")
+        with open(path, "w") as f:
+            f.write(src.replace(old, new))
+        spec = importlib.util.spec_from_file_location("chunked_bwd_mutant", path)
+        mod = importlib.util.module_from_spec(spec)
+        spec.loader.exec_module(mod)
+        with pytest.raises(AssertionError):
+            pin_chunked_backward_equals_recurrent(mod)
