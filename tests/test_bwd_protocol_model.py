@@ -1,5 +1,6 @@
-"""A host-side model of the persistent d_h = 64 backward tile kernel's barrier protocol
-(relation_tc_bwd.cu): the TMA, MMA, elementwise and dQ roles as sequences of mbarrier
+"""A host-side model of the backward tile kernel's barrier protocol (relation_tc_bwd.cu;
+the persistent d_h = 64 form and the one-unit d_h = 128 form with its per-step dQ^T): the
+TMA, MMA, elementwise and dQ roles as sequences of mbarrier
 waits and arrivals with the phase arithmetic the kernel uses, run under many random
 interleavings and unit sequences.  Checks that every role finishes (no deadlock) and that
 no wait polls a barrier that has already run two phases past the one it waits for (an
@@ -195,3 +196,80 @@ def test_model_detects_a_broken_protocol():
             run([3, 2], 0)
     finally:
         mma = saved
+
+
+# --- d_h = 128: one unit per CTA, Q/dO staged per 64-query step (three stages), and
+# --- dQ^T per step into the step's dP^T columns, read out before the next dP^T
+
+NQS_H = 3
+
+
+def tma_half(n_i):
+    yield ("arrive", "KV0")
+    for g in range(n_i * SPT):
+        s, r = g % NQS_H, g // NQS_H
+        if r > 0:
+            yield ("wait", f"QE{s}", r - 1)
+        yield ("arrive", f"QF{s}")
+
+
+def mma_half(n_i):
+    total = n_i * SPT
+
+    def issue_u(s):
+        yield ("wait", f"QF{s % NQS_H}", s // NQS_H)
+
+    yield ("wait", "KV0", 0)
+    for sn in range(min(total, NBUF)):
+        yield from issue_u(sn)
+        yield ("arrive", f"S{sn % NBUF}")
+    for s in range(total):
+        bb = s % NBUF
+        yield ("wait", f"P{bb}", s // NBUF)
+        if s == total - 1:
+            yield ("arrive", "ACC")
+        yield ("arrive", f"QE{s % NQS_H}")
+        yield ("arrive", f"DQF{bb}")           # dQ^T of step s into the buffer's dP^T columns
+        s2 = s + NBUF
+        if s2 < total:
+            yield from issue_u(s2)              # U^T of step s + 2 over P, which dV has read
+            yield ("wait", f"DQE{bb}", s // NBUF)  # dQ^T read out before the next dP^T
+            yield ("arrive", f"S{bb}")
+    yield ("arrive", "KVE0")
+
+
+def ew_half(n_i):
+    for s in range(n_i * SPT):
+        yield ("wait", f"S{s % NBUF}", s // NBUF)
+        yield ("wait", f"QF{s % NQS_H}", s // NQS_H)
+        yield ("arrive", f"P{s % NBUF}")
+    yield ("wait", "ACC", 0)
+
+
+def dq_half(n_i):
+    for s in range(n_i * SPT):
+        yield ("wait", f"DQF{s % NBUF}", s // NBUF)
+        yield ("arrive", f"DQE{s % NBUF}")
+
+
+def run_half(n_i, seed):
+    rng = random.Random(seed)
+    bars = Barriers()
+    roles = {"tma": tma_half(n_i), "mma": mma_half(n_i), "ew": ew_half(n_i), "dq": dq_half(n_i)}
+    pending = {name: next(gen, None) for name, gen in roles.items()}
+    while any(ev is not None for ev in pending.values()):
+        runnable = [n for n, ev in pending.items()
+                    if ev is not None and (ev[0] == "arrive" or bars.ready(ev[1], ev[2]))]
+        if not runnable:
+            raise AssertionError(f"deadlock at n_i = {n_i}: "
+                                 f"{ {n: e for n, e in pending.items() if e is not None} }")
+        name = rng.choice(runnable)
+        if pending[name][0] == "arrive":
+            bars.arrive(pending[name][1])
+        pending[name] = next(roles[name], None)
+
+
+@pytest.mark.parametrize("n_i", [1, 2, 3, 4, 7, 16])
+def test_protocol_d128(n_i):
+    for seed in range(40):
+        run_half(n_i, seed)
