@@ -5,8 +5,15 @@ the operator's hot path), inputs resident in HBM.  Timed with CUDA events on the
 launching stream, per step, with the L2 flushed (a 256 MiB write) between steps, after
 W warm-up steps.  Prints ONE JSON line (rank 0).
 
-  python bench.py [--gpus N] [--steps K] [--warmup W] [--config 10M|30M|100M|long|tiny]
-                  [--impl ours|reference] [--no-cpu-baseline]
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--config long|100M|30M|10M|tiny]
+                  [--also 100M,...|none] [--impl ours|reference] [--no-cpu-baseline]
+                  [--no-side]
+
+The headline line is the long-context workload (B=2, H=16, T=16384, d_h=128); the
+~100M-scale layer (B=8, H=12, T=2048, d_h=64) is measured in the same run as a
+sub-record (``sub_records``) with its own step time, roofline and tokens/s.  --no-side
+skips the side measurements (decode, Linear Relation, layer transforms, SDPA context),
+e.g. under a profiler.
 
 --impl reference times the fp64 CPU oracle (the reference arm of this operator: there
 is no other implementation) on the host cores over a bounded sample of the workload.
@@ -18,6 +25,7 @@ from __future__ import annotations
 
 import argparse
 import json
+import math
 import os
 import statistics
 import subprocess
@@ -114,10 +122,11 @@ class ClockSampler:
 
 
 def _profiled_traffic(w, kernel):
-    """DRAM bytes per launch of `kernel` from the committed ncu summary for this workload,
-    scaled to it, or None when there is none or the kernel source changed since."""
+    """DRAM bytes per launch of `kernel` on workload `w`, from the committed ncu record of
+    that kernel instantiation on that workload (profiles/<kernel>_<workload>_traffic.json),
+    or None when there is none or the kernel source changed since it was taken."""
     import hashlib
-    path = os.path.join(ROOT, "profiles", f"{kernel}_traffic.json")
+    path = os.path.join(ROOT, "profiles", f"{kernel}_{w.name}_traffic.json")
     try:
         with open(path) as f:
             rec = json.load(f)
@@ -125,8 +134,9 @@ def _profiled_traffic(w, kernel):
         with open(src, "rb") as f:
             if hashlib.sha256(f.read()).hexdigest() != rec["source_sha256"]:
                 return None
-        units = w.B * w.H * w.T * w.T  # traffic scales with the causal tile count
-        return rec["dram_bytes_per_launch"] * units / rec["units"]
+        if rec.get("head_dim") not in (None, w.d):
+            return None
+        return float(rec["dram_bytes_per_launch"])
     except (OSError, KeyError, ValueError):
         return None
 
@@ -159,31 +169,57 @@ def _max_over_ranks(dist, x: float, dev) -> float:
 # CPU oracle (baseline leg and --impl reference)
 # ------------------------------------------------------------------------------
 
-def _oracle_sample(w, n_heads):
-    """Inputs of the first n_heads (b, h) heads, fp64, [B', T, H', d] blocks."""
+ORACLE_BUDGET = 128 * 1024 * 1024 * 64  # heads x T^2 x d of one sample (~1 s on 16 cores)
+
+
+def _sample_plan(w, budget=ORACLE_BUDGET):
+    """A bounded sample of the workload for the fp64 oracle: (heads, T') with the first
+    `heads` (b, h) heads over their first T' rows.  The first T' rows of a causal head are
+    exactly the T'-row problem, so the sample is a smaller instance of the same
+    workload.  Whole sequences (T' = T) while at least one head fits the budget, whole
+    batches of heads where possible; long sequences take every head over a prefix."""
+    per_head = w.T * w.T * w.d
+    if per_head <= budget:
+        n = max(1, min(w.B * w.H, budget // per_head))
+        return (n if n < w.H else (n // w.H) * w.H), w.T
+    heads = w.B * w.H
+    t = w.T
+    while t > 128 and heads * t * t * w.d > budget:
+        t //= 2
+    return heads, t
+
+
+_SAMPLE_CACHE = {}
+
+
+def _oracle_sample(w, n_heads, t_rows):
+    """Inputs of the first n_heads (b, h) heads over rows [0, t_rows), fp64 [B', T', H', d]
+    (drawn once per sample shape)."""
+    key = (w, n_heads, t_rows)
+    if key not in _SAMPLE_CACHE:
+        _SAMPLE_CACHE.clear()
+        _SAMPLE_CACHE[key] = _draw_sample(w, n_heads, t_rows)
+    return _SAMPLE_CACHE[key]
+
+
+def _draw_sample(w, n_heads, t_rows):
     q, k, v, do = workloads.make_inputs(w)
     heads = [(b, h) for b in range(w.B) for h in range(w.H)][:n_heads]
     bs = sorted({b for b, _ in heads})
     hs = sorted({h for _, h in heads})
-    sl = (slice(bs[0], bs[-1] + 1), slice(None), slice(hs[0], hs[-1] + 1))
+    sl = (slice(bs[0], bs[-1] + 1), slice(0, t_rows), slice(hs[0], hs[-1] + 1))
     return [t[sl].double().numpy() for t in (q, k, v, do)], len(bs) * len(hs)
 
 
-def _sample_heads(w):
-    # a bounded sample: at most the cost of 128 heads of T=1024, d=64 (about 1 s of
-    # OpenMP oracle work on 16 cores), whole batches of heads where possible
-    per_head = w.T * w.T * w.d
-    budget = 128 * 1024 * 1024 * 64
-    n = max(1, min(w.B * w.H, budget // per_head))
-    return n if n < w.H else (n // w.H) * w.H
-
-
-def cpu_oracle_run(w, n_heads=None, min_seconds=0.0, max_reps=20):
-    """Time the fp64 oracle (forward + backward) on the first n_heads heads of the workload,
-    repeating the sample until min_seconds of CPU work have run."""
+def cpu_oracle_run(w, n_heads=None, t_rows=None, min_seconds=0.0, max_reps=20):
+    """Time the fp64 oracle (forward + backward) on a sample of the workload (the first
+    n_heads heads over their first t_rows rows), repeating the sample until min_seconds
+    of CPU work have run."""
     import oracle
-    n_heads = n_heads or _sample_heads(w)
-    (q, k, v, do), used = _oracle_sample(w, n_heads)
+    plan_heads, plan_rows = _sample_plan(w)
+    n_heads = n_heads or plan_heads
+    t_rows = t_rows or plan_rows
+    (q, k, v, do), used = _oracle_sample(w, n_heads, t_rows)
     threads = oracle.max_threads()
     reps, dt = 0, 0.0
     while reps < max_reps and (reps == 0 or dt < min_seconds):
@@ -192,26 +228,31 @@ def cpu_oracle_run(w, n_heads=None, min_seconds=0.0, max_reps=20):
         oracle.mhr_bwd(q, k, v, do, workloads.LAMBDA_INIT)
         dt += time.perf_counter() - t0
         reps += 1
-    flops = 7.0 * used * w.T * w.T * w.d * reps
-    return {"seconds": dt, "heads": used, "reps": reps, "flops": flops,
-            "tflops": flops / dt / 1e12, "tokens_per_s": reps * (used / w.H) * w.T / dt,
+    flops = 7.0 * used * t_rows * t_rows * w.d * reps
+    return {"seconds": dt, "heads": used, "rows": t_rows, "reps": reps, "flops": flops,
+            "tflops": flops / dt / 1e12, "tokens_per_s": reps * (used / w.H) * t_rows / dt,
             "cores": threads}
+
+
+def _sample_text(w, res):
+    rows = "" if res["rows"] == w.T else f" over their first {res['rows']} of {w.T} rows"
+    return f"{res['heads']} of {w.B * w.H} heads{rows}"
 
 
 def run_reference(args, w):
     dist, ws, rank, local = _dist()
     if rank != 0:
         return 0
-    n = _sample_heads(w)
+    n, rows = _sample_plan(w, ORACLE_BUDGET // 4)
     for _ in range(args.warmup):
-        cpu_oracle_run(w, n_heads=max(1, n // 4))
+        cpu_oracle_run(w, n_heads=n, t_rows=rows)
     times, res = [], None
     for _ in range(args.steps):
-        res = cpu_oracle_run(w, n_heads=max(1, n // 4))
+        res = cpu_oracle_run(w, n_heads=n, t_rows=rows)
         times.append(res["seconds"])
     tot_flops = res["flops"] * args.steps
     val = tot_flops / sum(times) / 1e12
-    sample = f"{res['heads']} of {w.B * w.H} heads per step (fwd+bwd, fp64, OpenMP over heads)"
+    sample = f"{_sample_text(w, res)} per step (fwd+bwd, fp64, OpenMP over heads)"
     line = {
         "impl": "reference", "metric": "FlashRelation fwd+bwd TFLOP/s (7*B*H*T^2*d causal)",
         "value": val, "unit": "TFLOP/s", "n_gpus": 0, "steps": args.steps, "warmup": args.warmup,
@@ -405,12 +446,11 @@ def linear_measure(binding, dev, steps=20, warmup=3):
             "gpu_launches_per_step": 3}
 
 
-def run_ours(args, w):
-    from paper_2608_20172_gb300 import binding
-    dist, ws, rank, local = _dist()
-    dev = torch.device("cuda", local)
-    torch.cuda.set_device(dev)
-    binding.load()
+def measure_workload(binding, w, dev, steps, warmup, family, peaks, dist=None, ws=1,
+                     sample_clocks=False, e2e=True):
+    """Time `steps` forward + backward steps of workload `w` (inputs resident in HBM, L2
+    flushed between steps) and, with `e2e`, the same steps through the public API from
+    pinned host buffers.  Returns the metrics of one JSON record."""
     lam, tau = workloads.LAMBDA_INIT, workloads.TAU_S
     q, k, v, do = workloads.make_inputs(w, seed=0)
     qd, kd, vd, dod = (t.to(dev) for t in (q, k, v, do))
@@ -422,7 +462,6 @@ def run_ours(args, w):
     status = torch.zeros(1, dtype=torch.int32, device=dev)
     flush = torch.empty(L2_FLUSH_BYTES, dtype=torch.uint8, device=dev)
     stream = torch.cuda.current_stream(dev)
-    family = args.kernel
 
     def step():
         binding.fwd(qd, kd, vd, lam, tau, kernel=family, out=y, logz=logz, dev_status=status,
@@ -430,36 +469,40 @@ def run_ours(args, w):
         binding.bwd(qd, kd, vd, y, dod, logz, lam, tau, kernel=family, workspace=wsb, dq=dq, dk=dk,
                     dv=dv, dlambda=dl, dev_status=status, stream=stream)
 
-    for _ in range(args.warmup):
+    for _ in range(warmup):
         step()
         flush.zero_()
     torch.cuda.synchronize(dev)
     if int(status.item()) != 0:
         raise SystemExit(f"device status {binding.status_string(int(status.item()))}")
 
-    n = args.steps
+    n = steps
     # per step: forward | backward row pass | backward tiles | backward finalisation
     ev = [[torch.cuda.Event(enable_timing=True) for _ in range(5)] for _ in range(n)]
     _barrier(dist, dev)
     torch.cuda.synchronize(dev)
-    with ClockSampler(dev.index) as clk:
+    clk = ClockSampler(dev.index) if sample_clocks else None
+    if clk is not None:
+        clk.__enter__()
         time.sleep(0.3)  # let the sampler start before the timed region
-        t_begin = time.time()
-        for i in range(n):
-            ev[i][0].record(stream)
-            binding.fwd(qd, kd, vd, lam, tau, kernel=family, out=y, logz=logz, dev_status=status,
-                        stream=stream)
-            ev[i][1].record(stream)
-            for j, stage in enumerate((binding.BWD_PREPARE, binding.BWD_TILES,
-                                       binding.BWD_FINALIZE)):
-                binding.bwd(qd, kd, vd, y, dod, logz, lam, tau, kernel=family, workspace=wsb,
-                            dq=dq, dk=dk, dv=dv, dlambda=dl, dev_status=status, stream=stream,
-                            stages=stage)
-                ev[i][2 + j].record(stream)
-            flush.zero_()
-        torch.cuda.synchronize(dev)
-        t_end = time.time()
+    t_begin = time.time()
+    for i in range(n):
+        ev[i][0].record(stream)
+        binding.fwd(qd, kd, vd, lam, tau, kernel=family, out=y, logz=logz, dev_status=status,
+                    stream=stream)
+        ev[i][1].record(stream)
+        for j, stage in enumerate((binding.BWD_PREPARE, binding.BWD_TILES,
+                                   binding.BWD_FINALIZE)):
+            binding.bwd(qd, kd, vd, y, dod, logz, lam, tau, kernel=family, workspace=wsb,
+                        dq=dq, dk=dk, dv=dv, dlambda=dl, dev_status=status, stream=stream,
+                        stages=stage)
+            ev[i][2 + j].record(stream)
+        flush.zero_()
+    torch.cuda.synchronize(dev)
+    t_end = time.time()
+    if clk is not None:
         time.sleep(0.1)
+        clk.__exit__(None, None, None)
     _barrier(dist, dev)
     t_fwd = [ev[i][0].elapsed_time(ev[i][1]) for i in range(n)]
     t_pre = [ev[i][1].elapsed_time(ev[i][2]) for i in range(n)]
@@ -477,74 +520,76 @@ def run_ours(args, w):
     if st != 0:
         raise SystemExit(f"device status {binding.status_string(st)}")
 
-    # End to end through the public API: every step copies its inputs from pinned host
-    # memory and its results (Y, dQ, dK, dV, dlambda) back.  Two device buffer sets: the
-    # inputs of step i + 1 go host->device (stream s_in) and the results of step i - 1
-    # device->host (stream s_out) while step i computes, so a step costs the largest of
-    # the three, not their sum.  The timed region starts drained and ends when the last
-    # results have landed.
-    hq, hk, hv, hdo = (t.pin_memory() for t in (q, k, v, do))
-    hy, hdq, hdk, hdv = (torch.empty_like(t).pin_memory() for t in (q, q, q, q))
-    hdl = torch.empty(1, dtype=torch.float32).pin_memory()
-    names = ("q", "k", "v", "do", "y", "dq", "dk", "dv", "dl")
-    sets = [dict(zip(names, (qd, kd, vd, dod, y, dq, dk, dv, dl)))]
-    sets.append({nm: torch.empty_like(t) for nm, t in sets[0].items()})
-    s_in, s_out = torch.cuda.Stream(dev), torch.cuda.Stream(dev)
-    total = n + args.warmup
-    ev_in, ev_cmp, ev_out = ([torch.cuda.Event() for _ in range(total)] for _ in range(3))
-    e2e_t0, e2e_t1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-    for i in range(total):
-        bs = sets[i % 2]
-        if i == args.warmup:
-            torch.cuda.synchronize(dev)
-            e2e_t0.record(s_in)
-        if i >= 2:
-            s_in.wait_event(ev_cmp[i - 2])  # set i % 2 no longer read by step i - 2
-        with torch.cuda.stream(s_in):
-            for src, nm in ((hq, "q"), (hk, "k"), (hv, "v"), (hdo, "do")):
-                bs[nm].copy_(src, non_blocking=True)
-        ev_in[i].record(s_in)
-        stream.wait_event(ev_in[i])
-        if i >= 2:
-            stream.wait_event(ev_out[i - 2])  # step i - 2's results have left set i % 2
-        binding.fwd(bs["q"], bs["k"], bs["v"], lam, tau, kernel=family, out=bs["y"], logz=logz,
-                    dev_status=status, stream=stream)
-        binding.bwd(bs["q"], bs["k"], bs["v"], bs["y"], bs["do"], logz, lam, tau, kernel=family,
-                    workspace=wsb, dq=bs["dq"], dk=bs["dk"], dv=bs["dv"], dlambda=bs["dl"],
-                    dev_status=status, stream=stream)
-        flush.zero_()
-        ev_cmp[i].record(stream)
-        s_out.wait_event(ev_cmp[i])
-        with torch.cuda.stream(s_out):
-            for nm, dst in (("y", hy), ("dq", hdq), ("dk", hdk), ("dv", hdv), ("dl", hdl)):
-                dst.copy_(bs[nm], non_blocking=True)
-        ev_out[i].record(s_out)
-    e2e_t1.record(s_out)
-    torch.cuda.synchronize(dev)
-    ms_e2e = _max_over_ranks(dist, e2e_t0.elapsed_time(e2e_t1) / n, dev)
-    h2d = sum(t.numel() * t.element_size() for t in (hq, hk, hv, hdo))
-    d2h = sum(t.numel() * t.element_size() for t in (hy, hdq, hdk, hdv, hdl))
+    rec = {}
+    if e2e:
+        # End to end through the public API: every step copies its inputs from pinned host
+        # memory and its results (Y, dQ, dK, dV, dlambda) back.  Two device buffer sets: the
+        # inputs of step i + 1 go host->device (stream s_in) and the results of step i - 1
+        # device->host (stream s_out) while step i computes, so a step costs the largest of
+        # the three, not their sum.  The timed region starts drained and ends when the last
+        # results have landed.
+        hq, hk, hv, hdo = (t.pin_memory() for t in (q, k, v, do))
+        hy, hdq, hdk, hdv = (torch.empty_like(t).pin_memory() for t in (q, q, q, q))
+        hdl = torch.empty(1, dtype=torch.float32).pin_memory()
+        names = ("q", "k", "v", "do", "y", "dq", "dk", "dv", "dl")
+        sets = [dict(zip(names, (qd, kd, vd, dod, y, dq, dk, dv, dl)))]
+        sets.append({nm: torch.empty_like(t) for nm, t in sets[0].items()})
+        s_in, s_out = torch.cuda.Stream(dev), torch.cuda.Stream(dev)
+        total = n + warmup
+        ev_in, ev_cmp, ev_out = ([torch.cuda.Event() for _ in range(total)] for _ in range(3))
+        e2e_t0 = torch.cuda.Event(enable_timing=True)
+        e2e_t1 = torch.cuda.Event(enable_timing=True)
+        for i in range(total):
+            bs = sets[i % 2]
+            if i == warmup:
+                torch.cuda.synchronize(dev)
+                e2e_t0.record(s_in)
+            if i >= 2:
+                s_in.wait_event(ev_cmp[i - 2])  # set i % 2 no longer read by step i - 2
+            with torch.cuda.stream(s_in):
+                for src, nm in ((hq, "q"), (hk, "k"), (hv, "v"), (hdo, "do")):
+                    bs[nm].copy_(src, non_blocking=True)
+            ev_in[i].record(s_in)
+            stream.wait_event(ev_in[i])
+            if i >= 2:
+                stream.wait_event(ev_out[i - 2])  # step i - 2's results have left set i % 2
+            binding.fwd(bs["q"], bs["k"], bs["v"], lam, tau, kernel=family, out=bs["y"],
+                        logz=logz, dev_status=status, stream=stream)
+            binding.bwd(bs["q"], bs["k"], bs["v"], bs["y"], bs["do"], logz, lam, tau,
+                        kernel=family, workspace=wsb, dq=bs["dq"], dk=bs["dk"], dv=bs["dv"],
+                        dlambda=bs["dl"], dev_status=status, stream=stream)
+            flush.zero_()
+            ev_cmp[i].record(stream)
+            s_out.wait_event(ev_cmp[i])
+            with torch.cuda.stream(s_out):
+                for nm, dst in (("y", hy), ("dq", hdq), ("dk", hdk), ("dv", hdv), ("dl", hdl)):
+                    dst.copy_(bs[nm], non_blocking=True)
+            ev_out[i].record(s_out)
+        e2e_t1.record(s_out)
+        torch.cuda.synchronize(dev)
+        ms_e2e = _max_over_ranks(dist, e2e_t0.elapsed_time(e2e_t1) / n, dev)
+        h2d = sum(t.numel() * t.element_size() for t in (hq, hk, hv, hdo))
+        d2h = sum(t.numel() * t.element_size() for t in (hy, hdq, hdk, hdv, hdl))
+        rec["e2e"] = {"value": ws * w.flops_fwd_bwd() / (ms_e2e * 1e-3) / 1e12,
+                      "unit": "TFLOP/s", "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
+                      "ms_per_step": ms_e2e,
+                      "overlap": "two buffer sets: step i+1's H2D and step i-1's D2H run on "
+                                 "their own streams during step i's compute (L2 flushed after "
+                                 "each step)"}
+        del sets
 
     flops = w.flops_fwd_bwd()
     tflops = ws * flops / (ms * 1e-3) / 1e12
-    peaks = _peaks()
     esz = 2 if w.dtype == "bf16" else 4
     bwd_flops = 5.0 * w.B * w.H * w.T * w.T * w.d  # causal bwd incl. the U recompute
     tiles_tflops = bwd_flops / (ms_tiles * 1e-3) / 1e12
     fwd_tflops = w.flops_fwd() / (ms_fwd * 1e-3) / 1e12
-    kname = "bwd_tc_kernel" if family != "simt" and w.dtype == "bf16" else "bwd_dkdv+dq (simt)"
-    traffic = _profiled_traffic(w, "bwd_tc_kernel") if kname == "bwd_tc_kernel" else None
-    clocks = clk.summary(t_begin, t_end) if rank == 0 else {}
-    line = {
-        "metric": "FlashRelation fwd+bwd TFLOP/s (7*B*H*T^2*d causal)",
-        "value": tflops, "unit": "TFLOP/s", "n_gpus": ws, "steps": n, "warmup": args.warmup,
-        "ms_per_step": ms, "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
-        "dtype": "bf16" if w.dtype == "bf16" else "f32", "data": "synthetic",
-        "config": {"workload": w.description, "B": w.B, "H": w.H, "T": w.T, "d_h": w.d,
-                   "lambda": workloads.LAMBDA_INIT, "tau_s": workloads.TAU_S,
-                   "kernel": family, "l2": "flushed between steps (256 MiB write)",
-                   "inputs": "Q,K,V,dO iid normal, seed 0 (workload recipe)",
-                   "parallelism": f"replicas x{ws}"},
+    tc = family != "simt" and w.dtype == "bf16"
+    dpad = 64 if w.d <= 64 else 128
+    kname = f"bwd_tc_kernel<{dpad}>" if tc else "bwd_dkdv+dq (simt)"
+    traffic = _profiled_traffic(w, "bwd_tc_kernel") if tc else None
+    rec.update({
+        "value": tflops, "unit": "TFLOP/s", "ms_per_step": ms,
         "tokens_per_s": ws * w.tokens / (ms * 1e-3),
         "pct_bf16_peak": 100.0 * tflops / (ws * peaks["bf16_tflops"]),
         "pct_bf16_peak_sustained": 100.0 * tflops / (ws * peaks["bf16_tflops_sustained"]),
@@ -561,17 +606,57 @@ def run_ours(args, w):
                      "algorithmic_flops_per_launch": bwd_flops,
                      "traffic": traffic,
                      "algorithmic_bytes_per_launch": 8.0 * w.B * w.T * w.H * w.d * esz,
-                     "fwd_kernel": {"achieved": fwd_tflops,
-                                    "frac": fwd_tflops / peaks["bf16_tflops"]}},
-        "e2e": {"value": ws * flops / (ms_e2e * 1e-3) / 1e12, "unit": "TFLOP/s",
-                "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h, "ms_per_step": ms_e2e,
-                "overlap": "two buffer sets: step i+1's H2D and step i-1's D2H run on their "
-                           "own streams during step i's compute (L2 flushed after each step)"},
+                     "fwd_kernel": {"kernel": f"fwd_tc_kernel<{dpad}>" if tc else "fwd (simt)",
+                                    "achieved": fwd_tflops,
+                                    "frac": fwd_tflops / peaks["bf16_tflops"]},
+                     "step": {"achieved": tflops / ws,
+                              "frac": tflops / ws / peaks["bf16_tflops"]}},
         "gpu_launches": n * (binding.launches_per_call(family, w.dtype, w.d, "fwd")
                              + binding.launches_per_call(family, w.dtype, w.d, "bwd")),
-        "clocks": clocks,
+        "config": {"workload": w.description, "B": w.B, "H": w.H, "T": w.T, "d_h": w.d,
+                   "lambda": workloads.LAMBDA_INIT, "tau_s": workloads.TAU_S,
+                   "kernel": family, "l2": "flushed between steps (256 MiB write)",
+                   "inputs": "Q,K,V,dO iid normal, seed 0 (workload recipe)",
+                   "parallelism": f"replicas x{ws}"},
+        "steps": n,
+    })
+    if clk is not None:
+        rec["clocks"] = clk.summary(t_begin, t_end)
+    return rec
+
+
+def run_ours(args, w):
+    from paper_2608_20172_gb300 import binding
+    dist, ws, rank, local = _dist()
+    dev = torch.device("cuda", local)
+    torch.cuda.set_device(dev)
+    binding.load()
+    peaks = _peaks()
+    family = args.kernel
+    head = measure_workload(binding, w, dev, args.steps, args.warmup, family, peaks, dist, ws,
+                            sample_clocks=(rank == 0))
+    line = {
+        "metric": "FlashRelation fwd+bwd TFLOP/s (7*B*H*T^2*d causal)",
+        "value": head["value"], "unit": "TFLOP/s", "n_gpus": ws, "steps": args.steps,
+        "warmup": args.warmup, "ms_per_step": head["ms_per_step"], "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None,
+        "dtype": "bf16" if w.dtype == "bf16" else "f32", "data": "synthetic",
     }
-    if rank == 0 and ws == 1:
+    line.update({k: v for k, v in head.items() if k not in line})
+    # further workloads of the same run, each with its own timed region (more steps on the
+    # short ones so that each region lasts tens of milliseconds)
+    subs = {}
+    for name in args.also:
+        sw = workloads.WORKLOADS[name]
+        if sw.name == w.name:
+            continue
+        steps = max(args.steps, int(math.ceil(0.1 / max(sw.flops_fwd_bwd() / 4e14, 1e-6))))
+        rec = measure_workload(binding, sw, dev, steps, args.warmup, family, peaks, dist, ws,
+                               sample_clocks=(rank == 0))
+        subs[name] = rec
+    if subs:
+        line["sub_records"] = subs
+    if rank == 0 and ws == 1 and not args.no_side:
         line["decode"] = decode_measure(binding, dev, peaks)
         line["linear"] = linear_measure(binding, dev)
         line["layer"] = layer_measure(binding, dev, peaks)
@@ -583,8 +668,8 @@ def run_ours(args, w):
         cb = cpu_oracle_run(w, min_seconds=10.0)
         line["cpu_baseline"] = {
             "value": cb["tflops"], "unit": "TFLOP/s", "cores": cb["cores"], "kind": "oracle",
-            "sample": f"{cb['heads']} of {w.B * w.H} heads x {cb['reps']}, fwd+bwd, fp64 C "
-                      f"oracle (OpenMP over heads), {cb['seconds']:.1f} s"}
+            "sample": f"{_sample_text(w, cb)} x {cb['reps']}, fwd+bwd, fp64 C oracle "
+                      f"(OpenMP over heads), {cb['seconds']:.1f} s"}
     if rank == 0:
         print(json.dumps(line), flush=True)
     if dist is not None:
@@ -595,13 +680,21 @@ def run_ours(args, w):
 def main(argv=None):
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
-    ap.add_argument("--steps", type=int, default=400)
+    ap.add_argument("--steps", type=int, default=100)
     ap.add_argument("--warmup", type=int, default=5)
-    ap.add_argument("--config", default="10M", choices=sorted(workloads.WORKLOADS))
+    ap.add_argument("--config", default="long", choices=sorted(workloads.WORKLOADS))
+    ap.add_argument("--also", default="100M",
+                    help="comma-separated further workloads measured as sub-records, or none")
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--kernel", default="auto", choices=["auto", "simt", "tcgen05"])
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-side", action="store_true",
+                    help="skip the decode, Linear Relation, layer-transform and SDPA legs")
     args = ap.parse_args(argv)
+    args.also = [] if args.also in ("", "none") else args.also.split(",")
+    for name in args.also:
+        if name not in workloads.WORKLOADS:
+            ap.error(f"--also: unknown workload {name}")
     args.warmup = max(args.warmup, 3)  # at least 3 untimed warm-up steps
     w = workloads.WORKLOADS[args.config]
     if args.impl == "reference":

@@ -272,10 +272,16 @@ relation_status relation_bwd_stages(const void* q, const void* k, const void* v,
  * The scratch is a fixed device array of RELATION_STATIC_SCRATCH_BYTES inside the library,
  * held on every GPU that loads the library until the process exits.  Shapes whose
  * relation_bwd_workspace_size() exceeds it are rejected with RELATION_ERR_WORKSPACE and
- * nothing is launched.  The first call on a device looks up the array's address on that
- * device (make it before any stream capture).  No call allocates memory.  Every call
- * shares the one array: calls that overlap on the GPU race on it and must be serialised
- * by the caller.  Arguments and results are otherwise those of relation_bwd_ex.
+ * nothing is launched.  The operands must be on the device current on the calling thread
+ * (that device's copy of the array is used); a q that is not device memory of that device
+ * is rejected with RELATION_ERR_INVALID_ARG and nothing is launched.  Each call looks up
+ * the array's address on the current device.  Under CUDA's lazy module loading, the first
+ * call on a device (or the library's first launch there) loads the module and so commits
+ * the RELATION_STATIC_SCRATCH_BYTES at that moment: a caller whose allocator owns the
+ * memory budget should make one call during set-up, before any stream capture (and again
+ * after a device reset).  No call allocates memory otherwise.  Every call shares the one
+ * array: calls that overlap on the GPU race on it and must be serialised by the caller.
+ * Arguments and results are otherwise those of relation_bwd_ex.
  */
 #define RELATION_STATIC_SCRATCH_BYTES (64u << 20)
 relation_status relation_bwd_static(const void* q, const void* k, const void* v, const void* o,

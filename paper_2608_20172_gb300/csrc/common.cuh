@@ -249,6 +249,36 @@ __host__ __device__ constexpr uint32_t idesc_bf16_f32(int M, int N, bool a_mn_ma
 }
 
 // ---------------------------------------------------------------------------
+// Work order of the tile kernels.  A unit is one 128-row tile of one head; unit w of the
+// launch order maps to (t, bh) with t = 0 the head's heaviest tile.  The B * H heads are
+// split into n_groups groups of equal size (the first BH % n_groups groups one head
+// larger) taken one after the other, the heaviest tiles of a group's heads first, so that
+// the rows the concurrently running units read and accumulate belong to few heads and
+// stay in L2.  head_groups (kernels.h) keeps every group large enough that its work per
+// resident CTA slot covers its heaviest unit; n_groups = 1 is plain heaviest-first order.
+// ---------------------------------------------------------------------------
+__device__ __forceinline__ void grouped_unit(int w, int n_t, int BH, int n_groups, int& t,
+                                             int& bh) {
+  const int q = BH / n_groups, r = BH % n_groups;  // r groups of q + 1 heads, then q heads
+  const int big = r * (q + 1) * n_t;
+  int base, gs, rem;
+  if (w < big) {
+    const int g = w / ((q + 1) * n_t);
+    base = g * (q + 1);
+    gs = q + 1;
+    rem = w - g * (q + 1) * n_t;
+  } else {
+    const int w2 = w - big;
+    const int g = w2 / (q * n_t);
+    base = r * (q + 1) + g * q;
+    gs = q;
+    rem = w2 - g * q * n_t;
+  }
+  t = rem / gs;
+  bh = base + rem % gs;
+}
+
+// ---------------------------------------------------------------------------
 // Math helpers
 // ---------------------------------------------------------------------------
 __device__ __forceinline__ float ex2_approx(float x) {

@@ -72,6 +72,16 @@ cudaError_t launch_dlambda(const Problem& p, const BwdWorkspace& ws, int n_main,
 }  // namespace bwd_common
 
 namespace tc {
+// Number of head groups of the tile kernels' work order (grouped_unit in common.cuh):
+// every group holds at least ceil(2.5 slots / (n_t + 1)) heads, so that one group's work
+// per resident CTA slot covers its heaviest unit (n_t tiles) with margin.  `slots` = CTAs
+// resident at once over the whole GPU.
+inline int head_groups(int n_t, int BH, int slots) {
+  long long g = (5LL * slots + 2LL * (n_t + 1) - 1) / (2LL * (n_t + 1));
+  if (g < 1) g = 1;
+  const long long n = BH / g;
+  return n < 1 ? 1 : (int)n;
+}
 bool supports(relation_dtype dt, int d);      // forward
 bool supports_bwd(relation_dtype dt, int d);  // backward
 cudaError_t launch_fwd(const Problem& p, cudaStream_t s);

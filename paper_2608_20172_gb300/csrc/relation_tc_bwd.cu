@@ -203,7 +203,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                   const __grid_constant__ CUtensorMap tmV, const __grid_constant__ CUtensorMap tmG,
                   const __grid_constant__ CUtensorMap tmDQ, const __grid_constant__ CUtensorMap tmDK,
                   const __grid_constant__ CUtensorMap tmDV, Problem p, BwdWorkspace ws, int n_t,
-                  int t_pad) {
+                  int t_pad, int n_groups) {
   using C = Cfg<D>;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>(
@@ -216,7 +216,8 @@ __global__ void __launch_bounds__(kThreads, 1)
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int BH = p.B * p.H;
-  const int n_work = n_t * BH;  // work units (key tile, head), most query tiles first
+  const int n_work = n_t * BH;  // work units (key tile, head), most query tiles first, heads
+                                // in groups (grouped_unit)
   // A unit: keys kt * 128 .. of head bh, query tiles kt .. n_t - 1.  Round r of the grid
   // takes units r G .. r G + G - 1 (G = gridDim.x), CTA c the unit r G + c in even rounds
   // and r G + G - 1 - c in odd ones: the units come heaviest first, so the zigzag evens
@@ -234,8 +235,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   };
   auto unit = [&](int w) {
     Unit u;
-    u.kt = w / BH;
-    u.bh = w % BH;
+    grouped_unit(w, n_t, BH, n_groups, u.kt, u.bh);
     u.b = u.bh / p.H;
     u.h = u.bh % p.H;
     u.k0 = u.kt * BK;
@@ -949,8 +949,15 @@ static cudaError_t bwd_t(const Problem& p, const BwdWorkspace& ws, unsigned stag
       note_failure("backward: TMA descriptor of the dQ accumulator");
       return cudaErrorInvalidValue;
     }
+    int dev = 0, nsm = 148;
+    if (cudaGetDevice(&dev) != cudaSuccess ||
+        cudaDeviceGetAttribute(&nsm, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess)
+      nsm = 148;
+    // d_h = 128 (one CTA per unit, dynamic scheduling): heads in groups, one CTA per SM;
+    // d_h = 64 (persistent, zigzag over a heaviest-first sequence): one group.
+    const int groups = D == 64 ? 1 : head_groups(n_t, p.B * p.H, nsm);
     bwd::bwd_tc_kernel<D><<<(unsigned)grid, bwd::kThreads, smem, s>>>(mq, mk, mv, mg, mdq, mdk,
-                                                                     mdv, p, ws, n_t, t_pad);
+                                                                     mdv, p, ws, n_t, t_pad, groups);
     if ((e = cudaGetLastError()) != cudaSuccess) { note_failure("backward: tile kernel launch"); return e; }
   }
   if (stages & 4) {

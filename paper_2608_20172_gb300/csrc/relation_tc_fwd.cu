@@ -3,7 +3,8 @@
 // One CTA owns a tile of BM = 128 query rows of one head and scans the key/value tiles
 // j0 = 0, 128, ... up to and including its diagonal tile (Sec. 5.1, App. A.3).  Two CTAs
 // share an SM (each allocates 256 TMEM columns), so the tensor core of one CTA overlaps
-// the elementwise work of the other.
+// the elementwise work of the other.  CTAs take the heaviest query tiles first, heads in
+// groups (grouped_unit), so that the K/V rows in use stay in L2.
 //
 // Warp roles (192 threads):
 //   warps 0-3  Exchange scan + epilogue: thread t owns query row q0 + t (TMEM lane t).
@@ -138,7 +139,7 @@ template <int D>
 __global__ void __launch_bounds__(kThreads, 2)
     fwd_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmK,
                   const __grid_constant__ CUtensorMap tmV, const __grid_constant__ CUtensorMap tmO,
-                  Problem p, int n_qt) {
+                  Problem p, int n_qt, int n_groups) {
   using C = FwdCfg<D>;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>(
@@ -150,8 +151,9 @@ __global__ void __launch_bounds__(kThreads, 2)
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int BH = p.B * p.H;
-  const int qt = n_qt - 1 - (int)(blockIdx.x / BH);  // heaviest query tiles first
-  const int bh = (int)(blockIdx.x % BH);
+  int tq, bh;  // heaviest query tiles first, heads in groups (common.cuh)
+  grouped_unit((int)blockIdx.x, n_qt, BH, n_groups, tq, bh);
+  const int qt = n_qt - 1 - tq;
   const int b = bh / p.H, h = bh % p.H;
   const int q0 = qt * BM;
   const int n_kv = qt + 1;
@@ -460,7 +462,12 @@ static cudaError_t fwd_t(const Problem& p, cudaStream_t s) {
   const int n_qt = (p.T + BM - 1) / BM;
   const long long grid = (long long)n_qt * p.B * p.H;
   if (grid > 0x7fffffffLL) return cudaErrorInvalidConfiguration;
-  fwd_tc_kernel<D><<<(unsigned)grid, kThreads, smem, s>>>(mq, mk, mv, mo, p, n_qt);
+  int dev = 0, nsm = 148;
+  if (cudaGetDevice(&dev) != cudaSuccess ||
+      cudaDeviceGetAttribute(&nsm, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess)
+    nsm = 148;
+  const int groups = head_groups(n_qt, p.B * p.H, 2 * nsm);  // two CTAs per SM
+  fwd_tc_kernel<D><<<(unsigned)grid, kThreads, smem, s>>>(mq, mk, mv, mo, p, n_qt, groups);
   if ((e = cudaGetLastError()) != cudaSuccess) note_failure("forward: kernel launch");
   return e;
 }

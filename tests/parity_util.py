@@ -123,3 +123,36 @@ def compare_heads(res, ref, dtype, bwd=True):
                 errs[(n, b, h)] = check(f"{n}[{b},{h}]", res[n][b, :, h].numpy(), r[n], dtype,
                                         "grad")
     return errs
+
+
+# Achieved errors of the full-size checks, printed at the end of the run by conftest's
+# terminal summary: (check, tensor) -> [normwise error, bound, elementwise relative error
+# over the entries with |ref| >= 1e-2 max|ref| (information only)].
+MARGINS = {}
+
+
+def elem_rel_err(got, ref) -> float:
+    """max |got - ref| / |ref| over the entries with |ref| >= 1e-2 max|ref|."""
+    got = np.asarray(got, dtype=np.float64)
+    ref = np.asarray(ref, dtype=np.float64)
+    if not ref.size:
+        return 0.0
+    big = np.abs(ref) >= 1e-2 * float(np.max(np.abs(ref)))
+    if not big.any():
+        return 0.0
+    return float(np.max(np.abs(got[big] - ref[big]) / np.abs(ref[big])))
+
+
+def record(check_name: str, tensor: str, err: float, bound: float, elem: float):
+    cur = MARGINS.get((check_name, tensor))
+    if cur is None or err > cur[0]:
+        MARGINS[(check_name, tensor)] = [err, bound, max(elem, cur[2] if cur else 0.0)]
+    else:
+        cur[2] = max(cur[2], elem)
+
+
+def check_recorded(check_name: str, tensor: str, got, ref, dtype: str, kind: str):
+    """check() plus a record of the achieved error for the end-of-run margin table."""
+    e = check(f"{check_name} {tensor}", got, ref, dtype, kind)
+    record(check_name, tensor, e, TOL[(dtype, kind)], elem_rel_err(got, ref))
+    return e

@@ -152,16 +152,64 @@ def run(units, seed):
         pending[name] = next(roles[name], None)
 
 
+def head_groups(n_t, BH, slots):
+    """Number of head groups of the kernels' work order (at least ceil(2.5 slots / (n_t + 1))
+    heads per group)."""
+    g = max(1, -(-5 * slots // (2 * (n_t + 1))))
+    return max(1, BH // g)
+
+
+def grouped_unit(w, n_t, BH, n_groups):
+    """(t, bh) of unit w: heads in n_groups equal groups (the first BH % n_groups one head
+    larger), heaviest tiles (t = 0) of a group first."""
+    q, r = divmod(BH, n_groups)
+    big = r * (q + 1) * n_t
+    if w < big:
+        g, rem = divmod(w, (q + 1) * n_t)
+        base, gs = g * (q + 1), q + 1
+    else:
+        g, rem = divmod(w - big, q * n_t)
+        base, gs = r * (q + 1) + g * q, q
+    return rem // gs, base + rem % gs
+
+
 def cta_units(n_t, BH, grid, c):
-    """Units (query tiles per key tile) of CTA c under the zigzag order of the kernel."""
+    """Units (query tiles per key tile) of CTA c under the zigzag order of the persistent
+    kernel (one head group)."""
     n_work, out, r = n_t * BH, [], 0
     while True:
         j = (grid - 1 - c) if (r & 1) else c
         w = r * grid + j
         if w >= n_work:
             return out
-        out.append(n_t - w // BH)
+        out.append(n_t - grouped_unit(w, n_t, BH, 1)[0])
         r += 1
+
+
+@pytest.mark.parametrize("n_t,BH,ng", [(128, 32, 10), (128, 32, 3), (16, 96, 4), (5, 7, 2),
+                                       (1, 3, 3), (4, 10, 3), (16, 96, 1)])
+def test_grouped_order_is_a_permutation(n_t, BH, ng):
+    """The grouped work order visits every (key tile, head) unit exactly once, within a group
+    the tiles come heaviest first, and the groups' sizes differ by at most one head."""
+    seen = [grouped_unit(w, n_t, BH, ng) for w in range(n_t * BH)]
+    assert sorted(seen) == sorted((t, bh) for t in range(n_t) for bh in range(BH))
+    sizes = [BH // ng + (1 if g < BH % ng else 0) for g in range(ng)]
+    w0, h0 = 0, 0
+    for gs in sizes:
+        chunk = seen[w0:w0 + gs * n_t]
+        assert {bh for _, bh in chunk} == set(range(h0, h0 + gs))
+        assert [t for t, _ in chunk] == sorted(t for t, _ in chunk)
+        w0, h0 = w0 + gs * n_t, h0 + gs
+    assert max(sizes) - min(sizes) <= 1 and w0 == n_t * BH
+
+
+def test_head_groups_cover_the_heaviest_unit():
+    for n_t, BH, slots in [(128, 32, 152), (128, 32, 304), (16, 96, 304), (8, 128, 304),
+                           (1, 5, 304)]:
+        ng = head_groups(n_t, BH, slots)
+        smallest = BH // ng
+        work_per_slot = smallest * n_t * (n_t + 1) / 2 / slots
+        assert ng == 1 or work_per_slot >= 1.25 * n_t
 
 
 @pytest.mark.parametrize("n_t,BH,grid", [(1, 400, 152), (2, 400, 152), (3, 320, 152),

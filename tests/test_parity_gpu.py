@@ -1,9 +1,10 @@
 """GPU parity: the CUDA path through the C ABI against the fp64 oracle.
 
 Small shapes span several tiles and a ragged tail and are compared element by element
-on every head.  The workloads' full sizes run in the benchmark's launch configuration
-and are compared on sampled heads (every element of those heads), and on the long
-sequence on sampled rows plus two exact restrictions the causal structure allows.
+on every head.  The 10M, 30M and 100M workloads run at full size in the benchmark's launch
+configuration and are compared on every head, element by element; the long sequence on
+sampled rows plus two exact restrictions the causal structure allows.  The achieved errors
+of the full-size checks are printed at the end of the run.
 """
 import numpy as np
 import pytest
@@ -123,21 +124,27 @@ def test_bhtd_layout():
 # --- full-size workloads in the benchmark's launch configuration --------------
 
 @pytest.mark.parametrize("name", ["10M", "30M", "100M"])
-def test_workload_full_size_sampled_heads(name):
+def test_workload_full_size_all_heads(name):
+    """The full workload in the benchmark's launch configuration, every head element by
+    element against the fp64 oracle (OpenMP over heads), dlambda over all heads."""
     w = workloads.WORKLOADS[name]
     q, k, v, do = workloads.make_inputs(w)
     res = pu.gpu_run(q, k, v, do, LAM)
-    heads = [(0, 0), (w.B - 1, w.H - 1), (w.B // 2, 1)]
-    ref = pu.oracle_heads(q, k, v, do, LAM, heads)
-    pu.compare_heads(res, ref, "bf16")
-    # every head: finite, logZ >= the Self logit's lower bound (logZ_i >= S_i > 0)
+    q64, k64, v64, g64 = (t.double().numpy() for t in (q, k, v, do))
+    ry, rlz = oracle.mhr_fwd(q64, k64, v64, LAM)
+    rdq, rdk, rdv, dl_all = oracle.mhr_bwd(q64, k64, v64, g64, LAM)
     for n in ("Y", "dQ", "dK", "dV", "logZ"):
         assert torch.isfinite(res[n]).all(), n
-    assert (res["logZ"] > 0).all()
-    # dlambda over all heads, from the oracle on all heads (multi-threaded)
-    _, _, _, dl_all = oracle.mhr_bwd(q.double().numpy(), k.double().numpy(), v.double().numpy(),
-                                     do.double().numpy(), LAM)
+    for b in range(w.B):
+        for h in range(w.H):
+            pu.check_recorded(name, "Y", res["Y"][b, :, h].numpy(), ry[b, :, h], "bf16", "out")
+            for n, r in (("dQ", rdq), ("dK", rdk), ("dV", rdv)):
+                pu.check_recorded(name, n, res[n][b, :, h].numpy(), r[b, :, h], "bf16", "grad")
+    e = pu.check_logz(f"{name} logZ", res["logZ"].numpy(), rlz, "bf16")
+    pu.record(name, "logZ(abs)", e, 2e-2, 0.0)
     pu.check_dlambda(res["dlambda"], dl_all, "bf16")
+    pu.record(name, "dlambda(rel)", abs(res["dlambda"] - dl_all) / max(abs(dl_all), 1e-3), 5e-2,
+              0.0)
 
 
 def test_long_context_full_size():
@@ -152,16 +159,17 @@ def test_long_context_full_size():
     for (b, h) in [(0, 0), (1, 15)]:
         qh, kh, vh = pu.head(q, b, h), pu.head(k, b, h), pu.head(v, b, h)
         y, lz = oracle.fwd_rows(qh, kh, vh, rows, LAM)
-        pu.check(f"Y rows [{b},{h}]", res["Y"][b, rows, h].numpy(), y, "bf16", "out")
-        pu.check_logz(f"logZ rows [{b},{h}]", res["logZ"][b, h, rows].numpy(), lz, "bf16")
+        pu.check_recorded("long rows", "Y", res["Y"][b, rows, h].numpy(), y, "bf16", "out")
+        e = pu.check_logz(f"logZ rows [{b},{h}]", res["logZ"][b, h, rows].numpy(), lz, "bf16")
+        pu.record("long rows", "logZ(abs)", e, 2e-2, 0.0)
     # backward, last 256 rows of one head: exact dQ rows and dK, dV keys >= T - 256
     b, h = 1, 7
     r0 = T - 256
     dq, dk, dv, _ = oracle.bwd_tail(pu.head(q, b, h), pu.head(k, b, h), pu.head(v, b, h),
                                     pu.head(do, b, h), LAM, r0)
-    pu.check("dQ tail", res["dQ"][b, r0:, h].numpy(), dq[r0:], "bf16", "grad")
-    pu.check("dK tail", res["dK"][b, r0:, h].numpy(), dk[r0:], "bf16", "grad")
-    pu.check("dV tail", res["dV"][b, r0:, h].numpy(), dv[r0:], "bf16", "grad")
+    pu.check_recorded("long tail", "dQ", res["dQ"][b, r0:, h].numpy(), dq[r0:], "bf16", "grad")
+    pu.check_recorded("long tail", "dK", res["dK"][b, r0:, h].numpy(), dk[r0:], "bf16", "grad")
+    pu.check_recorded("long tail", "dV", res["dV"][b, r0:, h].numpy(), dv[r0:], "bf16", "grad")
 
 
 def test_long_context_prefix_gradient():
@@ -177,9 +185,9 @@ def test_long_context_prefix_gradient():
     for (b, h) in [(0, 3), (1, 12)]:
         dq, dk, dv, _ = oracle.bwd(pu.head(q, b, h)[:Tp], pu.head(k, b, h)[:Tp],
                                    pu.head(v, b, h)[:Tp], pu.head(do, b, h)[:Tp], LAM)
-        pu.check(f"dQ prefix [{b},{h}]", res["dQ"][b, :Tp, h].numpy(), dq, "bf16", "grad")
-        pu.check(f"dK prefix [{b},{h}]", res["dK"][b, :Tp, h].numpy(), dk, "bf16", "grad")
-        pu.check(f"dV prefix [{b},{h}]", res["dV"][b, :Tp, h].numpy(), dv, "bf16", "grad")
+        pu.check_recorded("long prefix", "dQ", res["dQ"][b, :Tp, h].numpy(), dq, "bf16", "grad")
+        pu.check_recorded("long prefix", "dK", res["dK"][b, :Tp, h].numpy(), dk, "bf16", "grad")
+        pu.check_recorded("long prefix", "dV", res["dV"][b, :Tp, h].numpy(), dv, "bf16", "grad")
     for n in ("dQ", "dK", "dV"):
         assert torch.count_nonzero(res[n][:, Tp:]) == 0, n
     _, _, _, dl_all = oracle.mhr_bwd(q[:, :Tp].double().numpy(), k[:, :Tp].double().numpy(),

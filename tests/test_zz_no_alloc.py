@@ -56,3 +56,29 @@ def test_no_alloc_rejects_oversized_shapes():
     with pytest.raises(binding.RelationError) as e:
         binding.bwd_no_alloc(x, x, x, x, x, lz, 0.5, dq=x, dk=x, dv=x, dlambda=dl)
     assert e.value.code == binding.ERR_WORKSPACE
+
+
+def test_no_alloc_rejects_operands_off_the_current_device():
+    """The array used is the current device's copy, so operands elsewhere (here q in pinned
+    host memory, as a stand-in for another GPU's memory on a one-GPU machine) are rejected
+    before any launch, and the outputs are left untouched."""
+    import ctypes
+    w = workloads.custom(1, 2, 200, 64, "bf16")
+    dev = torch.device("cuda:0")
+    q, k, v, do = workloads.make_inputs(w, seed=31)
+    kd, vd, dod = (t.to(dev) for t in (k, v, do))
+    y, logz = binding.fwd(q.to(dev), kd, vd, workloads.LAMBDA_INIT)
+    q_host = q.pin_memory()
+    dq = torch.full_like(kd, 7.0)
+    dk, dv = torch.empty_like(kd), torch.empty_like(kd)
+    dl = torch.empty(1, device=dev, dtype=torch.float32)
+    lib = binding.load()
+    ptr = lambda t: ctypes.c_void_p(t.data_ptr())
+    rc = lib.relation_bwd_static(ptr(q_host), ptr(kd), ptr(vd), ptr(y), ptr(dod), ptr(logz),
+                                 ptr(dq), ptr(dk), ptr(dv), ptr(dl),
+                                 float(workloads.LAMBDA_INIT), 2.0, binding.shape_of(kd),
+                                 binding.BF16, binding.KERNELS["auto"], None,
+                                 ctypes.c_void_p(torch.cuda.current_stream().cuda_stream))
+    torch.cuda.synchronize()
+    assert rc == binding.ERR_INVALID_ARG
+    assert torch.all(dq == 7.0)
