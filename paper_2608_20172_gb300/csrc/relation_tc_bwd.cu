@@ -336,173 +336,172 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
   } else if (warp == W_MMA) {
     // ------------------------------------------------------ MMA issuer
-    if (lane == 0) {
-      constexpr uint32_t id_s = idesc_bf16_f32(128, C::QW, false, false);  // U^T, dP^T
-      constexpr uint32_t id_acc = idesc_bf16_f32(128, D, false, true);     // dV, dK
-      constexpr uint32_t id_dq = C::HALF ? idesc_bf16_f32(128, C::QW, true, true)  // dQ^T
-                                         : idesc_bf16_f32(128, D, true, true);     // dQ
-      bool ok = true;
-      bool acc_done = false;  // B_ACC of the current unit committed
-      // A unit's running offsets (steps, Q / dO stage loads) and its K / V tiles
-      struct Ctx {
-        int gs0, gq0;
-        uint32_t ks, vs;
-      };
-      auto ctx_of = [&](int ul_, int gs0_, int gq0_) {
-        const uint32_t k = sb + C::OFF_KV + (ul_ % C::NKV) * 2 * C::KVT;
-        return Ctx{gs0_, gq0_, k, k + C::KVT};
-      };
-      // U^T of step s into buffer (gs0 + s) % NBUF (waits for its Q / dO stage)
-      auto issue_u = [&](const Ctx& x, int s) -> bool {
-        const int g = x.gq0 + C::unit_of(s), st = g % C::NQS, bb = (x.gs0 + s) % C::NBUF;
-        const int hh = s % C::SPT;
-        if (C::HALF || hh == 0) {
-          if (!mbar_wait(bar(B_QF + st), (g / C::NQS) & 1, ab)) return false;
-          tc_fence_after();
-        }
-        const uint32_t rows = C::HALF ? 0u : (uint32_t)(hh * C::QW * 128);  // the step's rows
+    // Warp-uniform: every lane runs the loop and the waits, one elected lane issues.
+    constexpr uint32_t id_s = idesc_bf16_f32(128, C::QW, false, false);  // U^T, dP^T
+    constexpr uint32_t id_acc = idesc_bf16_f32(128, D, false, true);     // dV, dK
+    constexpr uint32_t id_dq = C::HALF ? idesc_bf16_f32(128, C::QW, true, true)  // dQ^T
+                                       : idesc_bf16_f32(128, D, true, true);     // dQ
+    bool ok = true;
+    bool acc_done = false;  // B_ACC of the current unit committed
+    // A unit's running offsets (steps, Q / dO stage loads) and its K / V tiles
+    struct Ctx {
+      int gs0, gq0;
+      uint32_t ks, vs;
+    };
+    auto ctx_of = [&](int ul_, int gs0_, int gq0_) {
+      const uint32_t k = sb + C::OFF_KV + (ul_ % C::NKV) * 2 * C::KVT;
+      return Ctx{gs0_, gq0_, k, k + C::KVT};
+    };
+    // U^T of step s into buffer (gs0 + s) % NBUF (waits for its Q / dO stage)
+    auto issue_u = [&](const Ctx& x, int s) -> bool {
+      const int g = x.gq0 + C::unit_of(s), st = g % C::NQS, bb = (x.gs0 + s) % C::NBUF;
+      const int hh = s % C::SPT;
+      if (C::HALF || hh == 0) {
+        if (!mbar_wait_warp(bar(B_QF + st), (g / C::NQS) & 1, ab)) return false;
+        tc_fence_after();
+      }
+      const uint32_t rows = C::HALF ? 0u : (uint32_t)(hh * C::QW * 128);  // the step's rows
 #pragma unroll
-        for (int kk = 0; kk < D / 16; ++kk) {
-          const uint32_t kof = (kk >> 2) * 16384 + (kk & 3) * 32;
-          const uint32_t qof = (kk >> 2) * C::KBQ + (kk & 3) * 32;
-          mma_ss(tmem + C::col_u(bb), smem_desc_sw128(x.ks + kof, 16, 1024),
+      for (int kk = 0; kk < D / 16; ++kk) {
+        const uint32_t kof = (kk >> 2) * 16384 + (kk & 3) * 32;
+        const uint32_t qof = (kk >> 2) * C::KBQ + (kk & 3) * 32;
+        mma_ss_w(tmem + C::col_u(bb), smem_desc_sw128(x.ks + kof, 16, 1024),
                  smem_desc_sw128(sb + C::OFF_Q + st * C::QSZ + rows + qof, 16, 1024), id_s,
                  kk > 0 ? 1u : 0u);
-        }
-        return true;
-      };
-      // dP^T of step s (after issue_u(s)), then the step's S barrier
-      auto issue_dp = [&](const Ctx& x, int s) {
-        const int st = (x.gq0 + C::unit_of(s)) % C::NQS, bb = (x.gs0 + s) % C::NBUF;
-        const int hh = s % C::SPT;
-        const uint32_t rows = C::HALF ? 0u : (uint32_t)(hh * C::QW * 128);
+      }
+      return true;
+    };
+    // dP^T of step s (after issue_u(s)), then the step's S barrier
+    auto issue_dp = [&](const Ctx& x, int s) {
+      const int st = (x.gq0 + C::unit_of(s)) % C::NQS, bb = (x.gs0 + s) % C::NBUF;
+      const int hh = s % C::SPT;
+      const uint32_t rows = C::HALF ? 0u : (uint32_t)(hh * C::QW * 128);
 #pragma unroll
-        for (int kk = 0; kk < D / 16; ++kk) {
-          const uint32_t kof = (kk >> 2) * 16384 + (kk & 3) * 32;
-          const uint32_t qof = (kk >> 2) * C::KBQ + (kk & 3) * 32;
-          mma_ss(tmem + C::col_g(bb), smem_desc_sw128(x.vs + kof, 16, 1024),
+      for (int kk = 0; kk < D / 16; ++kk) {
+        const uint32_t kof = (kk >> 2) * 16384 + (kk & 3) * 32;
+        const uint32_t qof = (kk >> 2) * C::KBQ + (kk & 3) * 32;
+        mma_ss_w(tmem + C::col_g(bb), smem_desc_sw128(x.vs + kof, 16, 1024),
                  smem_desc_sw128(sb + C::OFF_DO + st * C::QSZ + rows + qof, 16, 1024), id_s,
                  kk > 0 ? 1u : 0u);
+      }
+      mma_commit_w(bar(B_S + bb));
+    };
+    int ul = 0, gs0 = 0, gq0 = 0, gt0 = 0;
+    int pre = 0;  // steps of the current unit issued ahead by the previous unit
+    for (int w; ok && (w = unit_at(ul)) < n_work; ++ul) {
+      const Unit U = unit(w);
+      const int total = U.total;
+      acc_done = false;
+      const int kvb = ul % C::NKV;
+      const Ctx x = ctx_of(ul, gs0, gq0);
+      const uint32_t ks = x.ks;
+      if (pre == 0 && !(ok = mbar_wait_warp(bar(kv_full(kvb)), (ul / C::NKV) & 1, ab))) break;
+      // d_h = 64: U^T / dP^T of step sn may be issued once its buffer is free (step
+      // sn - NBUF done) and once the GEMM that releases the Q/dO stage it loads into has
+      // been issued: waiting for that stage's load earlier would deadlock.
+      int sn = pre, units_done = 0;
+      pre = 0;
+      while (ok && sn < total && sn < C::NBUF) {
+        ok = issue_u(x, sn);
+        if (ok) issue_dp(x, sn);
+        ++sn;
+      }
+      for (int s = 0; ok && s < total; ++s) {
+        const int t = s / C::SPT, hh = s % C::SPT, g = gs0 + s, bb = g % C::NBUF;
+        const int st = (gq0 + C::unit_of(s)) % C::NQS;
+        if (!(ok = mbar_wait_warp(bar(B_P + bb), (g / C::NBUF) & 1, ab))) break;
+        tc_fence_after();
+        // dV += P^T dO and dK += dS'^T Q with the A operands in TMEM: every 32-query chunk
+        // keeps its 16 packed columns of P (dS') at the start of its own U^T (dP^T)
+        // columns.  The first step of a unit starts the sums afresh; the epilogue has
+        // read the previous unit's sums before its warps finished this step (B_P).
+        const uint32_t pcol = C::col_u(bb), dcol = C::col_g(bb);
+        const uint32_t rows = C::HALF ? 0u : (uint32_t)(hh * C::QW * 128);
+#pragma unroll
+        for (int kk = 0; kk < C::QW / 16; ++kk) {
+          const uint32_t acol = (kk >> 1) * 32 + (kk & 1) * 8;
+          mma_ts_w(tmem + C::COL_DV, tmem + pcol + acol,
+                   smem_desc_sw128(sb + C::OFF_DO + st * C::QSZ + rows + kk * 2048, C::KBQ, 1024),
+                   id_acc, (s > 0 || kk > 0) ? 1u : 0u);
         }
-        mma_commit(bar(B_S + bb));
-      };
-      int ul = 0, gs0 = 0, gq0 = 0, gt0 = 0;
-      int pre = 0;  // steps of the current unit issued ahead by the previous unit
-      for (int w; ok && (w = unit_at(ul)) < n_work; ++ul) {
-        const Unit U = unit(w);
-        const int total = U.total;
-        acc_done = false;
-        const int kvb = ul % C::NKV;
-        const Ctx x = ctx_of(ul, gs0, gq0);
-        const uint32_t ks = x.ks;
-        if (pre == 0 && !(ok = mbar_wait(bar(kv_full(kvb)), (ul / C::NKV) & 1, ab))) break;
-        // d_h = 64: U^T / dP^T of step sn may be issued once its buffer is free (step
-        // sn - NBUF done) and once the GEMM that releases the Q/dO stage it loads into has
-        // been issued: waiting for that stage's load earlier would deadlock.
-        int sn = pre, units_done = 0;
-        pre = 0;
-        while (ok && sn < total && sn < C::NBUF) {
+#pragma unroll
+        for (int kk = 0; kk < C::QW / 16; ++kk) {
+          const uint32_t acol = (kk >> 1) * 32 + (kk & 1) * 8;
+          mma_ts_w(tmem + C::COL_DK, tmem + dcol + acol,
+                   smem_desc_sw128(sb + C::OFF_Q + st * C::QSZ + rows + kk * 2048, C::KBQ, 1024),
+                   id_acc, (s > 0 || kk > 0) ? 1u : 0u);
+        }
+        if (s == total - 1) {  // dK and dV are final: the epilogue need not wait for dQ
+          mma_commit_w(bar(B_ACC));
+          acc_done = true;
+          // d_h = 64: the next unit's first steps go ahead of this unit's last dQ (their
+          // buffers were read by the dV / dK just issued; its K / V came in beforehand)
+          const int wn = C::HALF ? n_work : unit_at(ul + 1);
+          if (wn < n_work) {
+            const Unit N = unit(wn);
+            if (!(ok = mbar_wait_warp(bar(kv_full((ul + 1) % C::NKV)), ((ul + 1) / C::NKV) & 1, ab)))
+              break;
+            const Ctx xn = ctx_of(ul + 1, gs0 + total, gq0 + U.n_units);
+            while (ok && pre < N.total && pre < C::NBUF) {
+              ok = issue_u(xn, pre);
+              if (ok) issue_dp(xn, pre);
+              ++pre;
+            }
+            if (!ok) break;
+          }
+        }
+        if (C::HALF) {
+          mma_commit_w(bar(B_QE + st));  // the step's Q / dO rows are no longer needed
+          // Buffer bb next holds step s + 2.  Issue order (executed in order): dQ^T of
+          // step s over dS' in the dP^T columns, which dK has read; U^T of step s + 2
+          // over P, which dV has read; dP^T of step s + 2 once dQ^T has been read out.
+          // dQ^T = K^T dS'^T (A = K tile, d-major; B = the step's dS', query-major)
+          const uint32_t dsb = sb + C::OFF_DS + (g & 1) * C::DSZ;
+#pragma unroll
+          for (int kk = 0; kk < BK / 16; ++kk)
+            mma_ss_w(tmem + C::col_g(bb), smem_desc_sw128(ks + kk * 2048, 16384, 1024),
+                     smem_desc_sw128(dsb + kk * 2048, 16384, 1024), id_dq, kk > 0 ? 1u : 0u);
+          mma_commit_w(bar(B_DQF + bb));
+          const int s2 = s + C::NBUF;
+          if (s2 < total && !(ok = issue_u(x, s2))) break;
+          if (s2 < total) {
+            if (!(ok = mbar_wait_warp(bar(B_DQE + bb), (g / C::NBUF) & 1, ab))) break;
+            tc_fence_after();
+            issue_dp(x, s2);
+          }
+          continue;
+        }
+        if (hh == C::SPT - 1) {
+          const int gt = gt0 + t;
+          if (gt > 0) {  // dQ of the previous query tile has been read out of TMEM
+            if (!(ok = mbar_wait_warp(bar(B_DQE), (gt - 1) & 1, ab))) break;
+            tc_fence_after();
+          }
+          // dQ_t = dS' K   (A = dS', queries x keys, M-major; B = K tile, N-major)
+          const uint32_t ds_base = sb + C::OFF_DS + (gt & 1) * C::DSZ;
+#pragma unroll
+          for (int kk = 0; kk < BK / 16; ++kk)
+            mma_ss_w(tmem + C::COL_DQ, smem_desc_sw128(ds_base + kk * 2048, 16384, 1024),
+                     smem_desc_sw128(ks + kk * 2048, 16384, 1024), id_dq,
+                     kk > 0 ? 1u : 0u);
+          mma_commit_w(bar(B_DQF));
+          mma_commit_w(bar(B_QE + st));
+          ++units_done;
+        }
+        while (ok && sn < total && sn <= s + C::NBUF &&
+               C::unit_of(sn) - C::NQS < units_done) {
           ok = issue_u(x, sn);
           if (ok) issue_dp(x, sn);
           ++sn;
         }
-        for (int s = 0; ok && s < total; ++s) {
-          const int t = s / C::SPT, hh = s % C::SPT, g = gs0 + s, bb = g % C::NBUF;
-          const int st = (gq0 + C::unit_of(s)) % C::NQS;
-          if (!(ok = mbar_wait(bar(B_P + bb), (g / C::NBUF) & 1, ab))) break;
-          tc_fence_after();
-          // dV += P^T dO and dK += dS'^T Q with the A operands in TMEM: every 32-query chunk
-          // keeps its 16 packed columns of P (dS') at the start of its own U^T (dP^T)
-          // columns.  The first step of a unit starts the sums afresh; the epilogue has
-          // read the previous unit's sums before its warps finished this step (B_P).
-          const uint32_t pcol = C::col_u(bb), dcol = C::col_g(bb);
-          const uint32_t rows = C::HALF ? 0u : (uint32_t)(hh * C::QW * 128);
-#pragma unroll
-          for (int kk = 0; kk < C::QW / 16; ++kk) {
-            const uint32_t acol = (kk >> 1) * 32 + (kk & 1) * 8;
-            mma_ts(tmem + C::COL_DV, tmem + pcol + acol,
-                   smem_desc_sw128(sb + C::OFF_DO + st * C::QSZ + rows + kk * 2048, C::KBQ, 1024),
-                   id_acc, (s > 0 || kk > 0) ? 1u : 0u);
-          }
-#pragma unroll
-          for (int kk = 0; kk < C::QW / 16; ++kk) {
-            const uint32_t acol = (kk >> 1) * 32 + (kk & 1) * 8;
-            mma_ts(tmem + C::COL_DK, tmem + dcol + acol,
-                   smem_desc_sw128(sb + C::OFF_Q + st * C::QSZ + rows + kk * 2048, C::KBQ, 1024),
-                   id_acc, (s > 0 || kk > 0) ? 1u : 0u);
-          }
-          if (s == total - 1) {  // dK and dV are final: the epilogue need not wait for dQ
-            mma_commit(bar(B_ACC));
-            acc_done = true;
-            // d_h = 64: the next unit's first steps go ahead of this unit's last dQ (their
-            // buffers were read by the dV / dK just issued; its K / V came in beforehand)
-            const int wn = C::HALF ? n_work : unit_at(ul + 1);
-            if (wn < n_work) {
-              const Unit N = unit(wn);
-              if (!(ok = mbar_wait(bar(kv_full((ul + 1) % C::NKV)), ((ul + 1) / C::NKV) & 1, ab)))
-                break;
-              const Ctx xn = ctx_of(ul + 1, gs0 + total, gq0 + U.n_units);
-              while (ok && pre < N.total && pre < C::NBUF) {
-                ok = issue_u(xn, pre);
-                if (ok) issue_dp(xn, pre);
-                ++pre;
-              }
-              if (!ok) break;
-            }
-          }
-          if (C::HALF) {
-            mma_commit(bar(B_QE + st));  // the step's Q / dO rows are no longer needed
-            // Buffer bb next holds step s + 2.  Issue order (executed in order): dQ^T of
-            // step s over dS' in the dP^T columns, which dK has read; U^T of step s + 2
-            // over P, which dV has read; dP^T of step s + 2 once dQ^T has been read out.
-            // dQ^T = K^T dS'^T (A = K tile, d-major; B = the step's dS', query-major)
-            const uint32_t dsb = sb + C::OFF_DS + (g & 1) * C::DSZ;
-#pragma unroll
-            for (int kk = 0; kk < BK / 16; ++kk)
-              mma_ss(tmem + C::col_g(bb), smem_desc_sw128(ks + kk * 2048, 16384, 1024),
-                     smem_desc_sw128(dsb + kk * 2048, 16384, 1024), id_dq, kk > 0 ? 1u : 0u);
-            mma_commit(bar(B_DQF + bb));
-            const int s2 = s + C::NBUF;
-            if (s2 < total && !(ok = issue_u(x, s2))) break;
-            if (s2 < total) {
-              if (!(ok = mbar_wait(bar(B_DQE + bb), (g / C::NBUF) & 1, ab))) break;
-              tc_fence_after();
-              issue_dp(x, s2);
-            }
-            continue;
-          }
-          if (hh == C::SPT - 1) {
-            const int gt = gt0 + t;
-            if (gt > 0) {  // dQ of the previous query tile has been read out of TMEM
-              if (!(ok = mbar_wait(bar(B_DQE), (gt - 1) & 1, ab))) break;
-              tc_fence_after();
-            }
-            // dQ_t = dS' K   (A = dS', queries x keys, M-major; B = K tile, N-major)
-            const uint32_t ds_base = sb + C::OFF_DS + (gt & 1) * C::DSZ;
-#pragma unroll
-            for (int kk = 0; kk < BK / 16; ++kk)
-              mma_ss(tmem + C::COL_DQ, smem_desc_sw128(ds_base + kk * 2048, 16384, 1024),
-                     smem_desc_sw128(ks + kk * 2048, 16384, 1024), id_dq,
-                     kk > 0 ? 1u : 0u);
-            mma_commit(bar(B_DQF));
-            mma_commit(bar(B_QE + st));
-            ++units_done;
-          }
-          while (ok && sn < total && sn <= s + C::NBUF &&
-                 C::unit_of(sn) - C::NQS < units_done) {
-            ok = issue_u(x, sn);
-            if (ok) issue_dp(x, sn);
-            ++sn;
-          }
-        }
-        if (!ok) break;
-        mma_commit(bar(B_KVE + kvb));  // every MMA of the unit (K / V buffer free) done
-        gs0 += total;
-        gq0 += U.n_units;
-        gt0 += U.n_i;
       }
-      if (!acc_done) mma_commit(bar(B_ACC));  // after an abort: whatever completed
+      if (!ok) break;
+      mma_commit_w(bar(B_KVE + kvb));  // every MMA of the unit (K / V buffer free) done
+      gs0 += total;
+      gq0 += U.n_units;
+      gt0 += U.n_i;
     }
+    if (!acc_done) mma_commit_w(bar(B_ACC));  // after an abort: whatever completed
     __syncwarp();
   } else if (warp >= W_DQ) {
     // ------------------------------------------------------ dQ -> fp32 accumulator

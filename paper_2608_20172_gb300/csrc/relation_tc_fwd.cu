@@ -221,52 +221,51 @@ __global__ void __launch_bounds__(kThreads, 2)
     }
   } else if (warp == 5) {
     // ------------------------------------------------------------------ MMA issuer
-    if (lane == 0) {
-      constexpr uint32_t idesc_qk = idesc_bf16_f32(BM, HN, false, false);
-      constexpr uint32_t idesc_pv = idesc_bf16_f32(BM, D, false, true);
-      const int total = 2 * n_kv;  // scan steps: two 64-key halves per K/V tile
-      // U of step s = Q K^T over keys [64 (s & 1), +64) of tile s / 2, into buffer s & 1
-      auto issue_u = [&](int s) -> bool {
-        const int j = s >> 1, hh = s & 1, st = j % C::STAGES;
-        if (hh == 0) {
-          if (!mbar_wait(bar(B_KF + st), (j / C::STAGES) & 1, ab)) return false;
-          tc_fence_after();
-        }
-#pragma unroll
-        for (int kk = 0; kk < D / 16; ++kk) {
-          const uint32_t koff = (kk >> 2) * (BN * 128) + (kk & 3) * 32;
-          const uint64_t a = smem_desc_sw128(sb + C::OFF_Q + koff, 16, 1024);
-          const uint64_t bd =
-              smem_desc_sw128(sb + C::OFF_K + st * C::TILE + hh * HN * 128 + koff, 16, 1024);
-          mma_ss(tmem + kSCol + hh * HN, a, bd, idesc_qk, kk > 0 ? 1u : 0u);
-        }
-        mma_commit(bar(B_S + hh));  // U ready (and every earlier z update done)
-        if (hh == 1) mma_commit(bar(B_KE + st));  // K stage free
-        return true;
-      };
-      bool ok = mbar_wait(bar(B_Q), 0, ab);
-      tc_fence_after();
-      if (ok) ok = issue_u(0);
-      if (ok && total > 1) ok = issue_u(1);
-      for (int s = 0; ok && s < total; ++s) {
-        const int j = s >> 1, hh = s & 1, st = j % C::STAGES;
-        if (hh == 0 && !(ok = mbar_wait(bar(B_VF + st), (j / C::STAGES) & 1, ab))) break;
-        if (!(ok = mbar_wait(bar(B_P + hh), (s >> 1) & 1, ab))) break;
+    // Warp-uniform: every lane runs the loop and the waits, one elected lane issues.
+    constexpr uint32_t idesc_qk = idesc_bf16_f32(BM, HN, false, false);
+    constexpr uint32_t idesc_pv = idesc_bf16_f32(BM, D, false, true);
+    const int total = 2 * n_kv;  // scan steps: two 64-key halves per K/V tile
+    // U of step s = Q K^T over keys [64 (s & 1), +64) of tile s / 2, into buffer s & 1
+    auto issue_u = [&](int s) -> bool {
+      const int j = s >> 1, hh = s & 1, st = j % C::STAGES;
+      if (hh == 0) {
+        if (!mbar_wait_warp(bar(B_KF + st), (j / C::STAGES) & 1, ab)) return false;
         tc_fence_after();
-        // z += P V over the step's 64 keys (A = P from TMEM; B = V rows, N = d contiguous)
-#pragma unroll
-        for (int kk = 0; kk < HN / 16; ++kk) {
-          const uint64_t bd = smem_desc_sw128(
-              sb + C::OFF_V + st * C::TILE + (hh * HN + kk * 16) * 128, BN * 128, 1024);
-          mma_ts(tmem + kOCol, tmem + kSCol + hh * HN + kk * 8, bd, idesc_pv,
-                 (s > 0 || kk > 0) ? 1u : 0u);
-        }
-        mma_commit(bar(B_OD));  // z update of step s done
-        if (hh == 1) mma_commit(bar(B_VE + st));  // V stage free
-        if (s + 2 < total && !(ok = issue_u(s + 2))) break;  // buffer hh: P read above
       }
-      mma_commit(bar(B_O));  // z final (or whatever completed before an abort)
+#pragma unroll
+      for (int kk = 0; kk < D / 16; ++kk) {
+        const uint32_t koff = (kk >> 2) * (BN * 128) + (kk & 3) * 32;
+        const uint64_t a = smem_desc_sw128(sb + C::OFF_Q + koff, 16, 1024);
+        const uint64_t bd =
+            smem_desc_sw128(sb + C::OFF_K + st * C::TILE + hh * HN * 128 + koff, 16, 1024);
+        mma_ss_w(tmem + kSCol + hh * HN, a, bd, idesc_qk, kk > 0 ? 1u : 0u);
+      }
+      mma_commit_w(bar(B_S + hh));  // U ready (and every earlier z update done)
+      if (hh == 1) mma_commit_w(bar(B_KE + st));  // K stage free
+      return true;
+    };
+    bool ok = mbar_wait_warp(bar(B_Q), 0, ab);
+    tc_fence_after();
+    if (ok) ok = issue_u(0);
+    if (ok && total > 1) ok = issue_u(1);
+    for (int s = 0; ok && s < total; ++s) {
+      const int j = s >> 1, hh = s & 1, st = j % C::STAGES;
+      if (hh == 0 && !(ok = mbar_wait_warp(bar(B_VF + st), (j / C::STAGES) & 1, ab))) break;
+      if (!(ok = mbar_wait_warp(bar(B_P + hh), (s >> 1) & 1, ab))) break;
+      tc_fence_after();
+      // z += P V over the step's 64 keys (A = P from TMEM; B = V rows, N = d contiguous)
+#pragma unroll
+      for (int kk = 0; kk < HN / 16; ++kk) {
+        const uint64_t bd = smem_desc_sw128(
+            sb + C::OFF_V + st * C::TILE + (hh * HN + kk * 16) * 128, BN * 128, 1024);
+        mma_ts_w(tmem + kOCol, tmem + kSCol + hh * HN + kk * 8, bd, idesc_pv,
+                 (s > 0 || kk > 0) ? 1u : 0u);
+      }
+      mma_commit_w(bar(B_OD));  // z update of step s done
+      if (hh == 1) mma_commit_w(bar(B_VE + st));  // V stage free
+      if (s + 2 < total && !(ok = issue_u(s + 2))) break;  // buffer hh: P read above
     }
+    mma_commit_w(bar(B_O));  // z final (or whatever completed before an abort)
     __syncwarp();
   } else {
     // ------------------------------------------------------------------ scan + epilogue
