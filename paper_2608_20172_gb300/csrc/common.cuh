@@ -60,6 +60,19 @@ __device__ __forceinline__ bool mbar_try_wait(uint32_t bar, uint32_t parity) {
   return ok != 0;
 }
 
+// Non-blocking check of the phase with parity `parity` of `bar`.
+__device__ __forceinline__ bool mbar_test_wait(uint32_t bar, uint32_t parity) {
+  uint32_t ok;
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "mbarrier.test_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
+      "selp.u32 %0, 1, 0, p;\n\t}"
+      : "=r"(ok)
+      : "r"(bar), "r"(parity)
+      : "memory");
+  return ok != 0;
+}
+
 // Abort protocol: one int in shared memory.  A thread whose wait expires sets it and
 // writes the status; every other bounded wait polls it and gives up as well, so each
 // role leaves its loop and the CTA reaches its teardown (TMEM release) in bounded time.
@@ -90,6 +103,18 @@ __device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity, const A
       }
     }
   }
+}
+
+// Wait for two phases at once (phase pa of bar a, phase pb of bar b): b is checked first
+// without blocking, so that its round trip overlaps the wait for a (b is usually complete
+// long before).  Same bound and abort behaviour as mbar_wait.
+__device__ __forceinline__ bool mbar_wait_both(uint32_t a, uint32_t pa, uint32_t b, uint32_t pb,
+                                               const Abort& ab) {
+  const bool db = mbar_test_wait(b, pb);
+  const bool da = mbar_try_wait(a, pa);
+  if (da && db) return true;
+  if (!db && !mbar_wait(b, pb, ab)) return false;
+  return da || mbar_wait(a, pa, ab);
 }
 
 // The bounded wait for a whole warp in warp-uniform code: true only when every lane saw

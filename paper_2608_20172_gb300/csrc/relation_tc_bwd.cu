@@ -609,12 +609,11 @@ __global__ void __launch_bounds__(kThreads, 1)
       for (int s = 0; s < U.total; ++s) {
         const int g = gs0 + s, bb = g % C::NBUF, i = s / C::SPT, hh = s % C::SPT;
         const int gu = gq0 + C::unit_of(s), st = gu % C::NQS;
-        ok = __all_sync(0xffffffffu, mbar_wait(bar(B_S + bb), (g / C::NBUF) & 1, ab));
+        // the step's U^T / dP^T, and the stage's per-query scalars (loaded long before)
+        ok = __all_sync(0xffffffffu, mbar_wait_both(bar(B_S + bb), (g / C::NBUF) & 1,
+                                                    bar(B_QF + st), (gu / C::NQS) & 1, ab));
         if (!ok) break;
         tc_fence_after();
-        // acquire the producer's per-query scalars of this stage (already complete)
-        ok = __all_sync(0xffffffffu, mbar_wait(bar(B_QF + st), (gu / C::NQS) & 1, ab));
-        if (!ok) break;
         const float* sts = reinterpret_cast<const float*>(smem + C::OFF_STAT + st * C::STB);
         const int cl = wg * 32;             // the chunk's first column within the step
         const int qt0 = hh * C::QW + cl;    // tile-local query index
