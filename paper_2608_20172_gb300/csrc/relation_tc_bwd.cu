@@ -24,8 +24,9 @@
 //        128-byte-swizzled shared memory, and the Exchange part of dlambda
 //   MMA  dV += P^T dO (P read from TMEM),  dK += dS'^T Q
 // Two TMEM buffers of U^T / dP^T: the MMAs of one buffer (dV, dK of the last step, U^T /
-// dP^T of the next) overlap the elementwise work on the other; both elementwise
-// warpgroups work on every step.  dQ goes to an fp32 accumulator through TMA reduce-add,
+// dP^T of the next) overlap the elementwise work on the other; every elementwise
+// warpgroup works on every step (d_h = 64: four warpgroups of 16 query columns, d_h = 128:
+// two of 32).  dQ goes to an fp32 accumulator through TMA reduce-add,
 // staged by warps 8-11:
 //   d_h = 64 : dQ_t = dS' K once per 128-query tile, in TMEM columns of its own.
 //   d_h = 128: dQ^T = K^T dS'^T once per step (d on TMEM lanes), written into the step's
@@ -52,9 +53,9 @@ namespace bwd {
 
 constexpr int BK = 128;        // keys per CTA
 constexpr int BT = 128;        // queries per TMA tile
-constexpr int kThreads = 448;  // warps 0-7 elementwise, 8-11 dQ, 12 TMA, 13 MMA
+// Warps: 4 NWG elementwise (NWG warpgroups, Cfg), then 4 dQ, 1 TMA, 1 MMA.
 constexpr int kTmemCols = 512;
-constexpr int W_DQ = 8, W_TMA = 12, W_MMA = 13;
+
 
 template <int D>
 struct Cfg {
@@ -89,6 +90,14 @@ struct Cfg {
   static constexpr int OFF_RED = OFF_STAT + NQS * STB;
   static constexpr int OFF_BAR = OFF_RED + 64;
   static constexpr int SMEM = OFF_BAR + 256 + 1024;
+  // Elementwise warpgroups: four at d_h = 64 (each takes 16 query columns of a step: more
+  // warps per SMSP hide the latency of the step's loads), two at d_h = 128 (32 columns
+  // each, in two halves of 16; the MMAs bound that path and a larger CTA spills).
+  static constexpr int NWG = D == 64 ? 4 : 2;
+  static constexpr int CW = QW / NWG;          // query columns per warpgroup and step
+  static constexpr int EW_THREADS = 128 * NWG;
+  static constexpr int W_DQ = 4 * NWG, W_TMA = W_DQ + 4, W_MMA = W_DQ + 5;
+  static constexpr int THREADS = 32 * (W_MMA + 1);
   static constexpr int COL_DK = NBUF * 2 * QW;  // 256
   static constexpr int COL_DV = COL_DK + D;     // 320 / 384
   static constexpr int COL_DQ = 384;            // d_h = 64 only
@@ -198,7 +207,7 @@ __device__ __forceinline__ void ew_chunk(const uint32_t (&U)[N], const uint32_t 
 }
 
 template <int D>
-__global__ void __launch_bounds__(kThreads, 1)
+__global__ void __launch_bounds__(Cfg<D>::THREADS, 1)
     bwd_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmK,
                   const __grid_constant__ CUtensorMap tmV, const __grid_constant__ CUtensorMap tmG,
                   const __grid_constant__ CUtensorMap tmDQ, const __grid_constant__ CUtensorMap tmDK,
@@ -256,23 +265,23 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
     for (int s = 0; s < C::NBUF; ++s) {
       mbar_init(bar(B_S + s), 1);
-      mbar_init(bar(B_P + s), 256);  // both elementwise warpgroups
+      mbar_init(bar(B_P + s), C::EW_THREADS);  // every elementwise warpgroup
       mbar_init(bar(B_DQF + s), 1);
       mbar_init(bar(B_DQE + s), 128);
     }
     mbar_init(bar(B_ACC), 1);
-    mbar_init(bar(B_STG), 256);
+    mbar_init(bar(B_STG), C::EW_THREADS);
     *abort_flag = 0;
     fence_mbar_init();
   }
-  if (warp == W_MMA) tmem_alloc(smem_u32(tmem_slot), kTmemCols);
+  if (warp == C::W_MMA) tmem_alloc(smem_u32(tmem_slot), kTmemCols);
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem = *tmem_slot;
   const Abort ab{abort_flag, p.dev_status};
 
-  if (warp == W_TMA) {
+  if (warp == C::W_TMA) {
     // ------------------------------------------------------ TMA + per-query scalars
     if (lane == 0) {
       tma_prefetch_desc(&tmQ);
@@ -334,7 +343,7 @@ __global__ void __launch_bounds__(kThreads, 1)
           drain_wait(bar(B_QF + g % C::NQS), (g / C::NQS) & 1);
       }
     }
-  } else if (warp == W_MMA) {
+  } else if (warp == C::W_MMA) {
     // ------------------------------------------------------ MMA issuer
     // Warp-uniform: every lane runs the loop and the waits, one elected lane issues.
     constexpr uint32_t id_s = idesc_bf16_f32(128, C::QW, false, false);  // U^T, dP^T
@@ -419,14 +428,16 @@ __global__ void __launch_bounds__(kThreads, 1)
         const uint32_t rows = C::HALF ? 0u : (uint32_t)(hh * C::QW * 128);
 #pragma unroll
         for (int kk = 0; kk < C::QW / 16; ++kk) {
-          const uint32_t acol = (kk >> 1) * 32 + (kk & 1) * 8;
+          constexpr int H = C::CW / 16;  // 16-query chunks per warpgroup
+          const uint32_t acol = (kk / H) * C::CW + (kk % H) * 8;
           mma_ts_w(tmem + C::COL_DV, tmem + pcol + acol,
                    smem_desc_sw128(sb + C::OFF_DO + st * C::QSZ + rows + kk * 2048, C::KBQ, 1024),
                    id_acc, (s > 0 || kk > 0) ? 1u : 0u);
         }
 #pragma unroll
         for (int kk = 0; kk < C::QW / 16; ++kk) {
-          const uint32_t acol = (kk >> 1) * 32 + (kk & 1) * 8;
+          constexpr int H = C::CW / 16;
+          const uint32_t acol = (kk / H) * C::CW + (kk % H) * 8;
           mma_ts_w(tmem + C::COL_DK, tmem + dcol + acol,
                    smem_desc_sw128(sb + C::OFF_Q + st * C::QSZ + rows + kk * 2048, C::KBQ, 1024),
                    id_acc, (s > 0 || kk > 0) ? 1u : 0u);
@@ -503,7 +514,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
     if (!acc_done) mma_commit_w(bar(B_ACC));  // after an abort: whatever completed
     __syncwarp();
-  } else if (warp >= W_DQ) {
+  } else if (warp >= C::W_DQ) {
     // ------------------------------------------------------ dQ -> fp32 accumulator
     const int quad = warp & 3;
     const uint32_t trow = tmem + ((uint32_t)(quad * 32) << 16);
@@ -615,18 +626,21 @@ __global__ void __launch_bounds__(kThreads, 1)
         if (!ok) break;
         tc_fence_after();
         const float* sts = reinterpret_cast<const float*>(smem + C::OFF_STAT + st * C::STB);
-        const int cl = wg * 32;             // the chunk's first column within the step
+        constexpr int CW = C::CW, H = CW / 16;
+        const int cl = wg * CW;             // the warpgroup's columns within the step
         const int qt0 = hh * C::QW + cl;    // tile-local query index
-        // Two halves of 16 queries: the second half's TMEM load is in flight while the
-        // first is computed.  P (dS') of queries cl + 16 h .. go packed to columns
-        // cl + 8 h .. of the U^T (dP^T) columns, which the first half has already read.
+        // Chunks of 16 queries (the next chunk's TMEM load in flight while one is
+        // computed).  P (dS') of queries cl + 16 h .. go packed to columns cl + 8 h .. of
+        // the U^T (dP^T) columns, which the first chunk has already read.
         uint32_t U0[16], G0[16], U1[16], G1[16];
         tmem_ld16(trow + C::col_u(bb) + cl, U0);
         tmem_ld16(trow + C::col_g(bb) + cl, G0);
         tmem_ld_wait();
-        tmem_ld16(trow + C::col_u(bb) + cl + 16, U1);
-        tmem_ld16(trow + C::col_g(bb) + cl + 16, G1);
-        uint32_t pk[16], dk[16];
+        if (H > 1) {
+          tmem_ld16(trow + C::col_u(bb) + cl + 16, U1);
+          tmem_ld16(trow + C::col_g(bb) + cl + 16, G1);
+        }
+        uint32_t pk[CW / 2], dk[CW / 2];
         const float* stc = sts + (C::HALF ? cl : qt0);
         {
           uint32_t (&p0)[8] = *reinterpret_cast<uint32_t(*)[8]>(pk);
@@ -638,10 +652,10 @@ __global__ void __launch_bounds__(kThreads, 1)
           tmem_st8(trow + C::col_u(bb) + cl, p0);  // P   (A operand of dV += P^T dO)
           tmem_st8(trow + C::col_g(bb) + cl, d0);  // dS' (A operand of dK += dS'^T Q)
         }
-        tmem_ld_wait();
-        {
-          uint32_t (&p1)[8] = *reinterpret_cast<uint32_t(*)[8]>(pk + 8);
-          uint32_t (&d1)[8] = *reinterpret_cast<uint32_t(*)[8]>(dk + 8);
+        if (H > 1) {
+          tmem_ld_wait();
+          uint32_t (&p1)[8] = *reinterpret_cast<uint32_t(*)[8]>(pk + 8 * (H - 1));
+          uint32_t (&d1)[8] = *reinterpret_cast<uint32_t(*)[8]>(dk + 8 * (H - 1));
           if (i == 0)
             ew_chunk<true, C::SW, 16>(U1, G1, stc + 16, qt0 + 16, t, kc, self2, p1, d1, dl2);
           else
@@ -651,21 +665,21 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
         if (s == 0 && ul > 0) {
           // the previous unit's dK / dV staging, in the dS' buffer written next, has been
-          // read by the stores of all eight warps
+          // read by the stores of warpgroups 0 and 1 (every elementwise warp arrives)
           if (lane == 0) tma_store_wait_read_all();
           __syncwarp();
           mbar_arrive(bar(B_STG));
           ok = __all_sync(0xffffffffu, mbar_wait(bar(B_STG), (ul - 1) & 1, ab));
           if (!ok) break;
         }
-        // dS' row t (key), 32 queries, into the 128-byte-swizzled query-major layout the
-        // dQ product reads: 64-query blocks of 128 key rows
+        // dS' row t (key), the warpgroup's queries, into the 128-byte-swizzled query-major
+        // layout the dQ product reads: 64-query blocks of 128 key rows
         uint8_t* ds_row = C::HALF ? smem + C::OFF_DS + (g & 1) * C::DSZ + t * 128
                                   : smem + C::OFF_DS + ((gt0 + i) & 1) * C::DSZ +
                                         (qt0 >> 6) * 16384 + t * 128;
         const int cb = (qt0 & 63) >> 3;
 #pragma unroll
-        for (int qd = 0; qd < 4; ++qd)
+        for (int qd = 0; qd < CW / 8; ++qd)
           *reinterpret_cast<uint4*>(ds_row + (((cb + qd) ^ (t & 7)) << 4)) =
               make_uint4(dk[4 * qd], dk[4 * qd + 1], dk[4 * qd + 2], dk[4 * qd + 3]);
         tmem_st_wait();
@@ -677,48 +691,51 @@ __global__ void __launch_bounds__(kThreads, 1)
       // -------------------------------------------------- dK (warpgroup 0) / dV (1)
       // The sums over the unit's queries, Self entry included (diagonal of P and dS'):
       //   dK_j = (sum_i dS'_ij q_i) / (2 sqrt d),   dV_j = sum_i P_ij dO_i
-      if (!(ok = __all_sync(0xffffffffu, mbar_wait(bar(B_ACC), ul & 1, ab)))) break;
-      tc_fence_after();
-      const uint32_t col = wg == 0 ? C::COL_DK : C::COL_DV;
-      const float sc = wg == 0 ? 0.5f * isd : 1.0f;
-      // Staged as 32 rows x D per warp (128-byte swizzle) and written by TMA stores that
-      // clip rows past T and padding columns.  d_h = 64: in the dS' buffer the next unit
-      // writes first (its last reader, the dQ of the tile before last, precedes B_ACC);
-      // d_h = 128 (one unit per CTA): in the Q (dK) and dO (dV) stages, which no MMA
-      // reads any more.
-      const uint32_t stg_off =
-          (C::HALF ? (wg == 0 ? C::OFF_Q : C::OFF_DO)
-                   : C::OFF_DS + ((gt0 + U.n_i) & 1) * C::DSZ + wg * (4 * 32 * D * 2)) +
-          wq * (32 * D * 2);
-      uint8_t* stg = smem + stg_off + lane * 128;
-#pragma unroll
-      for (int c0 = 0; c0 < D; c0 += 32) {
-        uint32_t a[32];
-        tmem_ld32(trow + col + c0, a);
-        tmem_ld_wait();
-        const int kb = c0 >> 6;  // 64-column block
-#pragma unroll
-        for (int c8 = 0; c8 < 32; c8 += 8) {
-          uint32_t o4[4];
-#pragma unroll
-          for (int e = 0; e < 4; ++e)
-            o4[e] = pack_bf16x2(__uint_as_float(a[c8 + 2 * e]) * sc,
-                                __uint_as_float(a[c8 + 2 * e + 1]) * sc);
-          const int chunk = ((c0 & 63) + c8) >> 3;  // 16-byte chunk within the 128-byte row
-          *reinterpret_cast<uint4*>(stg + kb * (32 * 128) + ((chunk ^ (lane & 7)) << 4)) =
-              make_uint4(o4[0], o4[1], o4[2], o4[3]);
+      // (warpgroups 2 and 3 go on to the next unit)
+      if (wg < 2) {
+        if (!(ok = __all_sync(0xffffffffu, mbar_wait(bar(B_ACC), ul & 1, ab)))) break;
+        tc_fence_after();
+        const uint32_t col = wg == 0 ? C::COL_DK : C::COL_DV;
+        const float sc = wg == 0 ? 0.5f * isd : 1.0f;
+        // Staged as 32 rows x D per warp (128-byte swizzle) and written by TMA stores that
+        // clip rows past T and padding columns.  d_h = 64: in the dS' buffer the next unit
+        // writes first (its last reader, the dQ of the tile before last, precedes B_ACC);
+        // d_h = 128 (one unit per CTA): in the Q (dK) and dO (dV) stages, which no MMA
+        // reads any more.
+        const uint32_t stg_off =
+            (C::HALF ? (wg == 0 ? C::OFF_Q : C::OFF_DO)
+                     : C::OFF_DS + ((gt0 + U.n_i) & 1) * C::DSZ + wg * (4 * 32 * D * 2)) +
+            wq * (32 * D * 2);
+        uint8_t* stg = smem + stg_off + lane * 128;
+  #pragma unroll
+        for (int c0 = 0; c0 < D; c0 += 32) {
+          uint32_t a[32];
+          tmem_ld32(trow + col + c0, a);
+          tmem_ld_wait();
+          const int kb = c0 >> 6;  // 64-column block
+  #pragma unroll
+          for (int c8 = 0; c8 < 32; c8 += 8) {
+            uint32_t o4[4];
+  #pragma unroll
+            for (int e = 0; e < 4; ++e)
+              o4[e] = pack_bf16x2(__uint_as_float(a[c8 + 2 * e]) * sc,
+                                  __uint_as_float(a[c8 + 2 * e + 1]) * sc);
+            const int chunk = ((c0 & 63) + c8) >> 3;  // 16-byte chunk within the 128-byte row
+            *reinterpret_cast<uint4*>(stg + kb * (32 * 128) + ((chunk ^ (lane & 7)) << 4)) =
+                make_uint4(o4[0], o4[1], o4[2], o4[3]);
+          }
         }
+        fence_async_smem();
+        __syncwarp();
+        if (lane == 0) {
+          const CUtensorMap* tm = wg == 0 ? &tmDK : &tmDV;
+  #pragma unroll
+          for (int kb = 0; kb < C::KB; ++kb)
+            tma_store_4d(tm, sb + stg_off + kb * (32 * 128), kb * 64, U.k0 + wq * 32, U.h, U.b);
+          tma_store_commit();  // its reads are awaited before the staging is written again
+        }
+        __syncwarp();
       }
-      fence_async_smem();
-      __syncwarp();
-      if (lane == 0) {
-        const CUtensorMap* tm = wg == 0 ? &tmDK : &tmDV;
-#pragma unroll
-        for (int kb = 0; kb < C::KB; ++kb)
-          tma_store_4d(tm, sb + stg_off + kb * (32 * 128), kb * 64, U.k0 + wq * 32, U.h, U.b);
-        tma_store_commit();  // its reads are awaited before the staging is written again
-      }
-      __syncwarp();
       gs0 += U.total;
       gq0 += U.n_units;
       gt0 += U.n_i;
@@ -735,10 +752,10 @@ __global__ void __launch_bounds__(kThreads, 1)
   if (threadIdx.x == 0) {
     float s = 0.f;
 #pragma unroll
-    for (int w = 0; w < 8; ++w) s += red[w];
+    for (int w = 0; w < C::EW_THREADS / 32; ++w) s += red[w];
     ws.dlam_part[ws.n_pre_blocks + blockIdx.x] = s;
   }
-  if (warp == W_MMA) {
+  if (warp == C::W_MMA) {
     tc_fence_after();
     tmem_dealloc(tmem, kTmemCols);
   }
@@ -954,7 +971,7 @@ static cudaError_t bwd_t(const Problem& p, const BwdWorkspace& ws, unsigned stag
     // d_h = 128 (one CTA per unit, dynamic scheduling): heads in groups, one CTA per SM;
     // d_h = 64 (persistent, zigzag over a heaviest-first sequence): one group.
     const int groups = D == 64 ? 1 : head_groups(n_t, p.B * p.H, nsm);
-    bwd::bwd_tc_kernel<D><<<(unsigned)grid, bwd::kThreads, smem, s>>>(mq, mk, mv, mg, mdq, mdk,
+    bwd::bwd_tc_kernel<D><<<(unsigned)grid, bwd::Cfg<D>::THREADS, smem, s>>>(mq, mk, mv, mg, mdq, mdk,
                                                                      mdv, p, ws, n_t, t_pad, groups);
     if ((e = cudaGetLastError()) != cudaSuccess) { note_failure("backward: tile kernel launch"); return e; }
   }
