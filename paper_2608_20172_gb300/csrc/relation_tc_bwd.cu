@@ -27,7 +27,7 @@
 // dP^T of the next) overlap the elementwise work on the other; every elementwise
 // warpgroup works on every step (d_h = 64: four warpgroups of 16 query columns, d_h = 128:
 // two of 32).  dQ goes to an fp32 accumulator through TMA reduce-add,
-// staged by warps 8-11:
+// staged by the four dQ warps (after the elementwise warps):
 //   d_h = 64 : dQ_t = dS' K once per 128-query tile, in TMEM columns of its own.
 //   d_h = 128: dQ^T = K^T dS'^T once per step (d on TMEM lanes), written into the step's
 //              dP^T columns after dK has read dS' (TMEM is full otherwise); the next U^T

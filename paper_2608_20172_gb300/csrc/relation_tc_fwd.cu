@@ -15,7 +15,8 @@
 // (U of step s + 2, z += P V of step s) overlap the elementwise work of the next.  Step s:
 //   MMA   U = Q K^T over 64 keys                 -> TMEM columns [64 b, 64 b + 64), b = s & 1
 //   scan  E = SiLU(U / sqrt(d)) for keys < row (Self excluded); running maximum m (kept
-//         as an upper bound of max E, rescaling z only when it grows by > 2^8), row sum
+//         as an upper bound of max E, max(U, 0) / sqrt(d), rescaling z only when it grows
+//         by > 2^8), row sum
 //         l += sum exp(E - m); P = exp(E - m) as bf16 written back into the buffer's
 //         first 32 columns (two per 32-bit column); the diagonal tile also yields
 //         S_i = sigmoid(U_ii / (sqrt(d) tau_S)).
@@ -68,8 +69,6 @@ __device__ __forceinline__ void drain_wait(uint32_t bar, uint32_t parity) {
     if (globaltimer_ns() - t0 > 20ull * 1000ull * 1000ull) return;  // 20 ms
   }
 }
-
-__device__ __forceinline__ float silu_acc(float x) { return x / (1.0f + __expf(-x)); }
 
 __device__ __forceinline__ float fmax3(float a, float b, float c) {
   float d;
@@ -294,18 +293,13 @@ __global__ void __launch_bounds__(kThreads, 2)
       // Pass 1: maximum of the raw evidence over the row's history (on the diagonal tile
       // only the keys before the row, c < tl; every key of an earlier tile), and U_ii.
       const float umax = diag ? row_max<true>(U, tl, u_self) : row_max<false>(U, tl, u_self);
-      // Upper bound of max E: SiLU is increasing on [0, inf) and negative on (-inf, 0).
-      float mt;
-      if (umax == -INFINITY) {
-        mt = -INFINITY;
-      } else if (umax >= 0.f) {
-        mt = silu_acc(umax * isd) * kLog2e;
-      } else {
-        mt = 0.f;
-      }
+      // Upper bound of max E: SiLU(u) = u sigma(u) <= max(u, 0), and the bound exceeds
+      // SiLU(u) by u sigma(-u) <= 0.28, so P = 2^(E log2 e - m) stays in (0.75, 1] at the
+      // row's largest entry; no transcendental on this path.
+      const float mt = umax == -INFINITY ? -INFINITY : fmaxf(umax, 0.f) * (isd * kLog2e);
       const float mn = fmaxf(m, mt);
       const bool grow = mn > m + kRescaleLog2;  // false while both are -inf
-      const float scale = grow ? exp2f(m - mn) : 1.0f;
+      const float scale = grow ? ex2_approx(m - mn) : 1.0f;
       if (grow) m = mn;
       l *= scale;
       if (s > 0 && __any_sync(0xffffffffu, grow)) {
