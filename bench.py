@@ -134,7 +134,7 @@ def _profiled_traffic(w, kernel):
         with open(src, "rb") as f:
             if hashlib.sha256(f.read()).hexdigest() != rec["source_sha256"]:
                 return None
-        if rec.get("head_dim") not in (None, w.d):
+        if [rec.get(k) for k in ("B", "H", "T", "d_h")] != [w.B, w.H, w.T, w.d]:
             return None
         return float(rec["dram_bytes_per_launch"])
     except (OSError, KeyError, ValueError):
@@ -690,6 +690,10 @@ def main(argv=None):
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-side", action="store_true",
                     help="skip the decode, Linear Relation, layer-transform and SDPA legs")
+    ap.add_argument("--batch", type=int, default=None,
+                    help="override the workload's batch (a slice for profiler captures)")
+    ap.add_argument("--heads", type=int, default=None,
+                    help="override the workload's head count (a slice for profiler captures)")
     args = ap.parse_args(argv)
     args.also = [] if args.also in ("", "none") else args.also.split(",")
     for name in args.also:
@@ -697,6 +701,10 @@ def main(argv=None):
             ap.error(f"--also: unknown workload {name}")
     args.warmup = max(args.warmup, 3)  # at least 3 untimed warm-up steps
     w = workloads.WORKLOADS[args.config]
+    if args.batch or args.heads:
+        import dataclasses
+        B, H = args.batch or w.B, args.heads or w.H
+        w = dataclasses.replace(w, B=B, H=H, description=f"{w.description}, slice B={B} H={H}")
     if args.impl == "reference":
         return run_reference(args, w)
     return run_ours(args, w)
