@@ -403,14 +403,40 @@ def sdpa_context(w, dev, steps=20, warmup=3):
 
 
 LINEAR_CFG = {"B": 8, "H": 12, "T": 2048, "d_h": 64}  # the 100M layer geometry, bf16
+LINEAR_SWEEP_TOKENS = 32768  # B * T of each point of the long-context sweep (H = 12, d_h = 64)
 FP32_FMA_TFLOPS = 152 * 128 * 2 * 2.07e9 / 1e12  # 152 SMs x 128 FFMA lanes x 2 flops x 2.07 GHz
 
 
-def linear_measure(binding, dev, steps=20, warmup=3):
-    """Linear Relation forward and backward on the 100M geometry (bf16, column splits).
-    Arithmetic per token and head: forward 5 d^2 (decay, read, write); backward 16 d^2
-    (checkpoint pass 3, chunk recompute 3, reverse step 10).  ALU roofline against the
-    fp32 FMA peak of the SMs."""
+def _linear_chunked_flops(B, H, T, d):
+    """Tensor-core work of the chunked forward per call: per 128-token block and 64-column
+    split, S = Qm Km^T (2 128 128 d), E = Qs C_0 (2 128 64 d), E += tril(S) I~ (2 128 64 128)
+    and the state C += KL^T I~ (2 128 64 128; d_h = 64 pads the channels to 128)."""
+    nb, splits = -(-T // 128), max(1, d // 64)
+    per = 2 * 128 * 128 * d + 2 * 128 * 64 * d + 2 * 128 * 64 * 128 + 2 * 128 * 64 * 128
+    return float(B * H * nb * splits * per)
+
+
+def _time_calls(call, dev, steps, warmup):
+    stream = torch.cuda.current_stream(dev)
+    for _ in range(warmup):
+        call()
+    ev = [torch.cuda.Event(enable_timing=True) for _ in range(steps + 1)]
+    torch.cuda.synchronize(dev)
+    ev[0].record(stream)
+    for i in range(steps):
+        call()
+        ev[i + 1].record(stream)
+    torch.cuda.synchronize(dev)
+    return statistics.mean(ev[i].elapsed_time(ev[i + 1]) for i in range(steps))
+
+
+def linear_measure(binding, dev, peaks, steps=20, warmup=3):
+    """Linear Relation on the 100M geometry (bf16): the chunked tensor-core forward, the
+    recurrent CUDA-core forward and backward.  Recurrent arithmetic per token and head:
+    forward 5 d^2 (decay, read, write), backward 16 d^2; ALU roofline against the fp32 FMA
+    peak of the SMs.  Chunked forward: tensor-core work as counted by _linear_chunked_flops,
+    against the measured bf16 peak.  Then the long-context sweep of the chunked forward,
+    T = 1k .. 32k at B T = 32768 tokens."""
     c = LINEAR_CFG
     w = workloads.custom(c["B"], c["H"], c["T"], c["d_h"], "bf16")
     p1, p2, v, alpha, dy = (t.to(dev) for t in workloads.make_linear_inputs(w, seed=0))
@@ -420,30 +446,49 @@ def linear_measure(binding, dev, steps=20, warmup=3):
     need = int(binding.load().relation_linear_bwd_workspace_size(binding.shape_of(p1),
                                                                   binding.BF16))
     wsb = torch.empty(need, dtype=torch.uint8, device=dev)
-    fwd = lambda: binding.linear_fwd(p1, p2, v, alpha, out=out, dev_status=status, stream=stream)
+    fwd = lambda fam: (lambda: binding.linear_fwd(p1, p2, v, alpha, kernel=fam, out=out,
+                                                  dev_status=status, stream=stream))
     bwd = lambda: binding.linear_bwd(p1, p2, v, alpha, dy, workspace=wsb, dev_status=status,
                                      stream=stream)
-    for _ in range(warmup):
-        fwd(); bwd()
-    ev = [[torch.cuda.Event(enable_timing=True) for _ in range(3)] for _ in range(steps)]
-    torch.cuda.synchronize(dev)
-    for e in ev:
-        e[0].record(stream); fwd(); e[1].record(stream); bwd(); e[2].record(stream)
-    torch.cuda.synchronize(dev)
+    ms_tc = _time_calls(fwd("tcgen05"), dev, steps, warmup)
+    ms_f = _time_calls(fwd("simt"), dev, steps, warmup)
+    ms_b = _time_calls(bwd, dev, steps, warmup)
     if int(status.item()) != 0:
         raise SystemExit(f"linear device status {binding.status_string(int(status.item()))}")
-    ms_f = statistics.mean(e[0].elapsed_time(e[1]) for e in ev)
-    ms_b = statistics.mean(e[1].elapsed_time(e[2]) for e in ev)
     tok_h = w.B * w.T * w.H
     fl_f, fl_b = 5.0 * tok_h * w.d * w.d, 16.0 * tok_h * w.d * w.d
     ach = fl_f / (ms_f * 1e-3) / 1e12
+    tc_fl = _linear_chunked_flops(w.B, w.H, w.T, w.d)
+    tc_ach = tc_fl / (ms_tc * 1e-3) / 1e12
+    sweep = []
+    for T in (1024, 2048, 4096, 8192, 16384, 32768):
+        B = max(1, LINEAR_SWEEP_TOKENS // T)
+        ws_ = workloads.custom(B, 12, T, 64, "bf16")
+        a = [t.to(dev) for t in workloads.make_linear_inputs(ws_, seed=1)[:4]]
+        o = torch.empty_like(a[0])
+        ms = _time_calls(lambda: binding.linear_fwd(*a, kernel="tcgen05", out=o, dev_status=status,
+                                                    stream=stream), dev, 5, 2)
+        fl = _linear_chunked_flops(B, 12, T, 64)
+        sweep.append({"B": B, "T": T, "ms_fwd": ms, "tokens_per_s": B * T / (ms * 1e-3),
+                      "tensor_tflops": fl / (ms * 1e-3) / 1e12,
+                      "tensor_frac": fl / (ms * 1e-3) / 1e12 / peaks["bf16_tflops"]})
+        del a, o
+    if int(status.item()) != 0:
+        raise SystemExit(f"linear device status {binding.status_string(int(status.item()))}")
     return {"config": {**c, "dtype": "bf16", "alpha": "KDA-style draw (workloads)"},
-            "ms_fwd": ms_f, "ms_bwd": ms_b, "tokens_per_s": w.B * w.T / ((ms_f + ms_b) * 1e-3),
-            "roofline": {"bound": "alu", "kernel": "linear fwd_kernel", "achieved": ach,
+            "ms_fwd_chunked": ms_tc, "ms_fwd": ms_f, "ms_bwd": ms_b,
+            "tokens_per_s": w.B * w.T / ((ms_tc + ms_b) * 1e-3),
+            "roofline": {"bound": "alu", "kernel": "linear fwd_kernel (recurrent)", "achieved": ach,
                          "peak": FP32_FMA_TFLOPS, "unit": "TFLOP/s (fp32 FMA)",
                          "frac": ach / FP32_FMA_TFLOPS,
                          "bwd_achieved": fl_b / (ms_b * 1e-3) / 1e12},
-            "gpu_launches_per_step": 3}
+            "roofline_chunked": {"bound": "tensor", "kernel": "lin_tc_fwd_kernel<64>",
+                                 "achieved": tc_ach, "peak": peaks["bf16_tflops"],
+                                 "unit": "TFLOP/s", "frac": tc_ach / peaks["bf16_tflops"],
+                                 "algorithmic_flops_per_launch": tc_fl},
+            "long_context_sweep": {"kernel": "chunked forward", "H": 12, "d_h": 64,
+                                   "tokens_per_point": LINEAR_SWEEP_TOKENS, "points": sweep},
+            "gpu_launches_per_step": {"fwd_chunked": 1, "fwd": 1, "bwd": 2}}
 
 
 def measure_workload(binding, w, dev, steps, warmup, family, peaks, dist=None, ws=1,
@@ -658,7 +703,7 @@ def run_ours(args, w):
         line["sub_records"] = subs
     if rank == 0 and ws == 1 and not args.no_side:
         line["decode"] = decode_measure(binding, dev, peaks)
-        line["linear"] = linear_measure(binding, dev)
+        line["linear"] = linear_measure(binding, dev, peaks)
         line["layer"] = layer_measure(binding, dev, peaks)
         try:
             line["context_sdpa"] = sdpa_context(w, dev)

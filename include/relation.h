@@ -134,6 +134,30 @@ relation_status relation_linear_fwd(const void* p1, const void* p2, const void* 
                                    relation_dtype dt, int* dev_status, relation_stream_t stream);
 
 /*
+ * relation_linear_fwd with a choice of kernel family (relation_linear_fwd uses AUTO):
+ *   RELATION_KERNEL_SIMT    the token-sequential recurrence on CUDA cores (every dtype and
+ *                           width above; the state and all products in fp32).
+ *   RELATION_KERNEL_TCGEN05 the chunked form on the tensor cores: blocks of 128 tokens, the
+ *                           within-block pairs and the state's read and update as tcgen05
+ *                           products with bf16 operands and fp32 accumulation, the fp32 state
+ *                           in tensor memory.  bf16 with d_h 64 or 128 only, element strides
+ *                           multiples of 8 (else RELATION_ERR_UNSUPPORTED or
+ *                           RELATION_ERR_ALIGNMENT, nothing launched).  The retention ratios
+ *                           a_t / a_j inside a block are split at its midpoint, so a factor
+ *                           covers at most 64 tokens of decay: a channel whose retention
+ *                           product over 64 consecutive tokens of one block falls below 2^-120
+ *                           has its factor clamped, the result is then not exact, and
+ *                           RELATION_ERR_UNSUPPORTED is written to *dev_status (non-null) once
+ *                           the call completes.
+ *   RELATION_KERNEL_AUTO    the chunked kernel where it applies, else the recurrence.
+ */
+relation_status relation_linear_fwd_ex(const void* p1, const void* p2, const void* v,
+                                      const float* alpha, void* y, float tau_s,
+                                      relation_shape shp, relation_dtype dt,
+                                      relation_kernel kernel, int* dev_status,
+                                      relation_stream_t stream);
+
+/*
  * Linear Relation backward: the reverse-mode derivative of the recurrence above (the paper
  * writes out the forward only), given dy = dL/dY:
  *   dp1, dp2, dv : [B][T][H][d_h] in dt, with the inputs' strides (overwritten);

@@ -31,6 +31,7 @@ EXPORTED = ("relation_fwd", "relation_fwd_ex", "relation_bwd", "relation_bwd_ex"
             "relation_selftest_wait_timeout", "relation_launch_count", "relation_last_cuda_error",
             "relation_bwd_stages", "relation_bwd_static", "relation_fwd_flow",
             "relation_decode", "relation_decode_workspace_size", "relation_linear_fwd",
+            "relation_linear_fwd_ex",
             "relation_linear_bwd", "relation_linear_bwd_workspace_size", "relation_layer_prep",
             "relation_layer_grad", "relation_layer_grad_workspace_size")
 
@@ -79,6 +80,7 @@ def load(path: str | None = None):
                                         ctypes.c_size_t, ip, vp]
         lib.relation_decode_workspace_size.argtypes = [Shape, i]
         lib.relation_linear_fwd.argtypes = [vp, vp, vp, vp, vp, f, Shape, i, ip, vp]
+        lib.relation_linear_fwd_ex.argtypes = [vp, vp, vp, vp, vp, f, Shape, i, i, ip, vp]
         lib.relation_linear_bwd.argtypes = [vp, vp, vp, vp, vp, vp, vp, vp, vp, f, Shape, i, vp,
                                             ctypes.c_size_t, ip, vp]
         lib.relation_linear_bwd_workspace_size.argtypes = [Shape, i]
@@ -200,20 +202,23 @@ def fwd_flow(q, k, v, lam: float, tau_s: float = 2.0, *, kernel: str = "auto", o
     return out, logz, self_flow
 
 
-def linear_fwd(p1, p2, v, alpha, tau_s: float = 2.0, *, out=None, dev_status=None, stream=None):
+def linear_fwd(p1, p2, v, alpha, tau_s: float = 2.0, *, kernel: str = "auto", out=None,
+               dev_status=None, stream=None):
     """Linear Relation forward.  p1, p2, v [B, T, H, d] (fp32 or bf16), alpha [B, T, H, d]
-    fp32 with p1's strides.  Returns Y."""
+    fp32 with p1's strides.  ``kernel``: "simt" (the recurrence), "tcgen05" (the chunked
+    tensor-core form) or "auto".  Returns Y."""
     _same_layout(p1, p2, v)
     if alpha.dtype != torch.float32 or tuple(alpha.shape) != tuple(p1.shape) or \
             tuple(alpha.stride()) != tuple(p1.stride()):
         raise ValueError("alpha must be fp32 with p1's shape and strides")
     out = torch.empty_like(p1) if out is None else out
     _same_layout(p1, out)
-    rc = load().relation_linear_fwd(_ptr(p1), _ptr(p2), _ptr(v), _ptr(alpha), _ptr(out),
-                                    float(tau_s), shape_of(p1), _dtype_code(p1),
-                                    _ptr(dev_status), ctypes.c_void_p(_stream(stream)))
+    rc = load().relation_linear_fwd_ex(_ptr(p1), _ptr(p2), _ptr(v), _ptr(alpha), _ptr(out),
+                                       float(tau_s), shape_of(p1), _dtype_code(p1),
+                                       KERNELS[kernel], _ptr(dev_status),
+                                       ctypes.c_void_p(_stream(stream)))
     if rc != OK:
-        raise RelationError(rc, "relation_linear_fwd")
+        raise RelationError(rc, "relation_linear_fwd_ex")
     return out
 
 

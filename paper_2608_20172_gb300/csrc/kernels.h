@@ -126,6 +126,10 @@ struct LinearProblem {
 };
 bool linear_supports(relation_dtype dt, int d);
 cudaError_t launch_linear_fwd(const LinearProblem& p, cudaStream_t s);
+// Chunked tensor-core forward (relation_linear_tc.cu): bf16, d_h 64 or 128, element
+// strides multiples of 8.
+bool linear_tc_supports(const LinearProblem& p);
+cudaError_t launch_linear_tc_fwd(const LinearProblem& p, cudaStream_t s);
 size_t linear_bwd_workspace_bytes(int B, int H, int T, int d);
 cudaError_t launch_linear_bwd(const LinearProblem& p, cudaStream_t s);
 

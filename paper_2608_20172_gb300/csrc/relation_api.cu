@@ -122,7 +122,19 @@ relation_status relation_fwd(const void* q, const void* k, const void* v, void* 
 relation_status relation_linear_fwd(const void* p1, const void* p2, const void* v,
                                    const float* alpha, void* y, float tau_s, relation_shape shp,
                                    relation_dtype dt, int* dev_status, relation_stream_t stream) {
+  return relation_linear_fwd_ex(p1, p2, v, alpha, y, tau_s, shp, dt, RELATION_KERNEL_AUTO,
+                                dev_status, stream);
+}
+
+relation_status relation_linear_fwd_ex(const void* p1, const void* p2, const void* v,
+                                      const float* alpha, void* y, float tau_s,
+                                      relation_shape shp, relation_dtype dt,
+                                      relation_kernel kernel, int* dev_status,
+                                      relation_stream_t stream) {
   relation_status st;
+  if (kernel != RELATION_KERNEL_AUTO && kernel != RELATION_KERNEL_SIMT &&
+      kernel != RELATION_KERNEL_TCGEN05)
+    return RELATION_ERR_INVALID_ARG;
   if (dt != RELATION_F32 && dt != RELATION_BF16) return RELATION_ERR_INVALID_ARG;
   if (shp.B < 1 || shp.T < 1 || shp.H < 1 || shp.d_h < 1) return RELATION_ERR_INVALID_ARG;
   if (shp.sB < 1 || shp.sT < 1 || shp.sH < 1) return RELATION_ERR_INVALID_ARG;
@@ -138,7 +150,13 @@ relation_status relation_linear_fwd(const void* p1, const void* p2, const void* 
   p.p1 = p1; p.p2 = p2; p.v = v; p.alpha = alpha; p.y = y; p.dev_status = dev_status;
   p.tau_s = tau_s; p.B = shp.B; p.T = shp.T; p.H = shp.H; p.d = shp.d_h;
   p.sB = shp.sB; p.sT = shp.sT; p.sH = shp.sH; p.dtype = dt;
-  return from_cuda(rel::launch_linear_fwd(p, reinterpret_cast<cudaStream_t>(stream)));
+  const bool tc = rel::linear_tc_supports(p);
+  if (kernel == RELATION_KERNEL_TCGEN05 && !tc)
+    return (dt == RELATION_BF16 && (shp.d_h == 64 || shp.d_h == 128)) ? RELATION_ERR_ALIGNMENT
+                                                                     : RELATION_ERR_UNSUPPORTED;
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  if (tc && kernel != RELATION_KERNEL_SIMT) return from_cuda(rel::launch_linear_tc_fwd(p, s));
+  return from_cuda(rel::launch_linear_fwd(p, s));
 }
 
 size_t relation_linear_bwd_workspace_size(relation_shape shp, relation_dtype dt) {

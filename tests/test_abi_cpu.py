@@ -224,6 +224,29 @@ def test_linear_rejects_bad_arguments(lib, case, expect):
     assert rc == expect
 
 
+@pytest.mark.parametrize("case,expect", [
+    ("tcgen05 fp32", binding.ERR_UNSUPPORTED),
+    ("tcgen05 d = 32", binding.ERR_UNSUPPORTED),
+    ("tcgen05 stride not a multiple of 8", binding.ERR_ALIGNMENT),
+    ("unknown family", binding.ERR_INVALID_ARG),
+])
+def test_linear_fwd_ex_family_rules(lib, case, expect):
+    """The chunked tensor-core family serves bf16 with d_h 64 or 128 and element strides
+    that are multiples of 8; other requests for it are refused with nothing launched."""
+    p = [ctypes.c_void_p(0x10000 * (i + 1)) for i in range(5)]
+    shape, dt, fam = _shape(d=64), binding.BF16, binding.KERNELS["tcgen05"]
+    if case == "tcgen05 fp32":
+        dt = binding.F32
+    elif case == "tcgen05 d = 32":
+        shape = _shape(d=32)
+    elif case == "tcgen05 stride not a multiple of 8":
+        shape = _shape(d=64, sH=68, sT=2 * 68, sB=8 * 2 * 68)
+    elif case == "unknown family":
+        fam = 7
+    rc = lib.relation_linear_fwd_ex(p[0], p[1], p[2], p[3], p[4], 2.0, shape, dt, fam, None, None)
+    assert rc == expect
+
+
 def test_linear_bwd_workspace_rules(lib):
     shape = _shape(B=2, T=20, H=3, d=64)
     need = lib.relation_linear_bwd_workspace_size(shape, binding.BF16)

@@ -76,3 +76,66 @@ def test_linear_bhtd_layout():
     y0 = binding.linear_fwd(*(t.to(dev) for t in (p1, p2, v, alpha)))
     y1 = binding.linear_fwd(*(bhtd(t) for t in (p1, p2, v, alpha)))
     assert torch.equal(y0.cpu(), y1.cpu())
+
+
+# --- the chunked tensor-core forward ------------------------------------------
+
+@pytest.mark.parametrize("d", [64, 128])
+@pytest.mark.parametrize("T", [1, 2, 127, 128, 129, 300, 513])
+def test_linear_forward_chunked_every_head(d, T):
+    """The chunked tcgen05 forward (blocks of 128 tokens: T spans whole blocks, ragged
+    tails and a single token) against the fp64 recurrence on every head."""
+    w = workloads.custom(2, 3, T, d, "bf16")
+    p1, p2, v, alpha, _ = workloads.make_linear_inputs(w, seed=500 + T + d)
+    dev = torch.device("cuda:0")
+    status = torch.zeros(1, dtype=torch.int32, device=dev)
+    y = binding.linear_fwd(p1.to(dev), p2.to(dev), v.to(dev), alpha.to(dev), kernel="tcgen05",
+                           dev_status=status)
+    torch.cuda.synchronize()
+    assert int(status.item()) == 0
+    y = y.float().cpu().numpy()
+    for b in range(w.B):
+        for h in range(w.H):
+            ref, _ = oracle.linear_fwd(_heads(p1, b, h), _heads(p2, b, h), _heads(v, b, h),
+                                       _heads(alpha, b, h))
+            pu.check(f"chunked linear Y ({b},{h}) T={T}", y[b, :, h], ref, "bf16", "out")
+
+
+@pytest.mark.parametrize("d", [64, 128])
+def test_linear_forward_chunked_long_sequence(d):
+    """A long sequence (64 blocks of 128 tokens: the state carried through them) on every
+    head, and the chunked and recurrent kernels against each other."""
+    w = workloads.custom(1, 2, 8192, d, "bf16")
+    p1, p2, v, alpha, _ = workloads.make_linear_inputs(w, seed=77 + d)
+    dev = torch.device("cuda:0")
+    args = [t.to(dev) for t in (p1, p2, v, alpha)]
+    status = torch.zeros(1, dtype=torch.int32, device=dev)
+    y_tc = binding.linear_fwd(*args, kernel="tcgen05", dev_status=status)
+    y_rec = binding.linear_fwd(*args, kernel="simt", dev_status=status)
+    torch.cuda.synchronize()
+    assert int(status.item()) == 0
+    y_tc, y_rec = y_tc.float().cpu().numpy(), y_rec.float().cpu().numpy()
+    for h in range(w.H):
+        ref, _ = oracle.linear_fwd(_heads(p1, 0, h), _heads(p2, 0, h), _heads(v, 0, h),
+                                   _heads(alpha, 0, h))
+        e = pu.check_recorded("linear 8192", f"Y d={d}", y_tc[0, :, h], ref, "bf16", "out")
+        pu.check(f"recurrent linear Y h={h}", y_rec[0, :, h], ref, "bf16", "out")
+
+
+def test_linear_chunked_reports_decay_beyond_its_range():
+    """Retention so small that a 64-token product falls below 2^-120: the chunked kernel
+    clamps its ratio factors and says so through dev_status (the output stays finite); the
+    recurrent kernel has no such limit."""
+    w = workloads.custom(1, 2, 256, 64, "bf16")
+    p1, p2, v, alpha, _ = workloads.make_linear_inputs(w, seed=3)
+    alpha = torch.full_like(alpha, 1e-3)
+    dev = torch.device("cuda:0")
+    args = [t.to(dev) for t in (p1, p2, v, alpha)]
+    st_tc = torch.zeros(1, dtype=torch.int32, device=dev)
+    st_rec = torch.zeros(1, dtype=torch.int32, device=dev)
+    y = binding.linear_fwd(*args, kernel="tcgen05", dev_status=st_tc)
+    binding.linear_fwd(*args, kernel="simt", dev_status=st_rec)
+    torch.cuda.synchronize()
+    assert int(st_tc.item()) == binding.ERR_UNSUPPORTED
+    assert int(st_rec.item()) == 0
+    assert torch.isfinite(y.float()).all()
