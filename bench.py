@@ -466,13 +466,16 @@ def linear_measure(binding, dev, peaks, steps=20, warmup=3):
         ws_ = workloads.custom(B, 12, T, 64, "bf16")
         a = [t.to(dev) for t in workloads.make_linear_inputs(ws_, seed=1)[:4]]
         o = torch.empty_like(a[0])
-        ms = _time_calls(lambda: binding.linear_fwd(*a, kernel="tcgen05", out=o, dev_status=status,
-                                                    stream=stream), dev, 5, 2)
+        wsl = torch.empty(max(binding.linear_fwd_workspace_size(a[0]), 16), dtype=torch.uint8,
+                          device=dev)
+        ms = _time_calls(lambda: binding.linear_fwd_ws(*a, workspace=wsl, out=o,
+                                                       dev_status=status, stream=stream),
+                         dev, 5, 2)
         fl = _linear_chunked_flops(B, 12, T, 64)
         sweep.append({"B": B, "T": T, "ms_fwd": ms, "tokens_per_s": B * T / (ms * 1e-3),
                       "tensor_tflops": fl / (ms * 1e-3) / 1e12,
                       "tensor_frac": fl / (ms * 1e-3) / 1e12 / peaks["bf16_tflops"]})
-        del a, o
+        del a, o, wsl
     if int(status.item()) != 0:
         raise SystemExit(f"linear device status {binding.status_string(int(status.item()))}")
     return {"config": {**c, "dtype": "bf16", "alpha": "KDA-style draw (workloads)"},
@@ -486,7 +489,9 @@ def linear_measure(binding, dev, peaks, steps=20, warmup=3):
                                  "achieved": tc_ach, "peak": peaks["bf16_tflops"],
                                  "unit": "TFLOP/s", "frac": tc_ach / peaks["bf16_tflops"],
                                  "algorithmic_flops_per_launch": tc_fl},
-            "long_context_sweep": {"kernel": "chunked forward", "H": 12, "d_h": 64,
+            "long_context_sweep": {"kernel": "chunked forward with a workspace (chunk-parallel "
+                                             "below one (head, column) pair per SM)",
+                                   "H": 12, "d_h": 64,
                                    "tokens_per_point": LINEAR_SWEEP_TOKENS, "points": sweep},
             "gpu_launches_per_step": {"fwd_chunked": 1, "fwd": 1, "bwd": 2}}
 

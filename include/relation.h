@@ -158,6 +158,31 @@ relation_status relation_linear_fwd_ex(const void* p1, const void* p2, const voi
                                       relation_stream_t stream);
 
 /*
+ * relation_linear_fwd with a caller workspace, for long sequences.  The chunked kernel walks
+ * a head's 128-token blocks in order, one CTA per (head, 64 information columns), so a call
+ * with fewer such pairs than the GPU has SMs leaves SMs idle.  With a workspace the blocks
+ * run in parallel instead: every block's state contribution (its decayed sum of k' I~^T and
+ * its decay, fp32), then a scan of the state over the blocks, then every block's output from
+ * the state it starts from (stored in bf16 between the passes; three launches).
+ *   workspace : device scratch of relation_linear_fwd_workspace_size(shp, dt) bytes
+ *               (B H (d_h / 64) ceil(T / 128) d_h rows of 64 fp32 + 64 bf16 + 1 fp32),
+ *               16-byte aligned, or RELATION_ERR_WORKSPACE / RELATION_ERR_ALIGNMENT with
+ *               nothing launched.
+ * The chunk-parallel form runs when B H (d_h / 64) is below half the device's SM count, the
+ * sequential chunked kernel otherwise (same results up to rounding).  Requests the chunked
+ * kernel does not serve (workspace size 0: fp32, d_h other than 64 and 128, strides not
+ * multiples of 8) go to relation_linear_fwd_ex(..., RELATION_KERNEL_AUTO, ...) and ignore the
+ * workspace.  Other arguments, results and the decay-range report are those of
+ * relation_linear_fwd_ex with RELATION_KERNEL_TCGEN05.
+ */
+size_t relation_linear_fwd_workspace_size(relation_shape shp, relation_dtype dt);
+relation_status relation_linear_fwd_ws(const void* p1, const void* p2, const void* v,
+                                      const float* alpha, void* y, float tau_s,
+                                      relation_shape shp, relation_dtype dt, void* workspace,
+                                      size_t ws_bytes, int* dev_status,
+                                      relation_stream_t stream);
+
+/*
  * Linear Relation backward: the reverse-mode derivative of the recurrence above (the paper
  * writes out the forward only), given dy = dL/dY:
  *   dp1, dp2, dv : [B][T][H][d_h] in dt, with the inputs' strides (overwritten);

@@ -31,7 +31,8 @@ EXPORTED = ("relation_fwd", "relation_fwd_ex", "relation_bwd", "relation_bwd_ex"
             "relation_selftest_wait_timeout", "relation_launch_count", "relation_last_cuda_error",
             "relation_bwd_stages", "relation_bwd_static", "relation_fwd_flow",
             "relation_decode", "relation_decode_workspace_size", "relation_linear_fwd",
-            "relation_linear_fwd_ex",
+            "relation_linear_fwd_ex", "relation_linear_fwd_ws",
+            "relation_linear_fwd_workspace_size",
             "relation_linear_bwd", "relation_linear_bwd_workspace_size", "relation_layer_prep",
             "relation_layer_grad", "relation_layer_grad_workspace_size")
 
@@ -81,6 +82,9 @@ def load(path: str | None = None):
         lib.relation_decode_workspace_size.argtypes = [Shape, i]
         lib.relation_linear_fwd.argtypes = [vp, vp, vp, vp, vp, f, Shape, i, ip, vp]
         lib.relation_linear_fwd_ex.argtypes = [vp, vp, vp, vp, vp, f, Shape, i, i, ip, vp]
+        lib.relation_linear_fwd_ws.argtypes = [vp, vp, vp, vp, vp, f, Shape, i, vp, sz, ip, vp]
+        lib.relation_linear_fwd_workspace_size.argtypes = [Shape, i]
+        lib.relation_linear_fwd_workspace_size.restype = sz
         lib.relation_linear_bwd.argtypes = [vp, vp, vp, vp, vp, vp, vp, vp, vp, f, Shape, i, vp,
                                             ctypes.c_size_t, ip, vp]
         lib.relation_linear_bwd_workspace_size.argtypes = [Shape, i]
@@ -219,6 +223,33 @@ def linear_fwd(p1, p2, v, alpha, tau_s: float = 2.0, *, kernel: str = "auto", ou
                                        ctypes.c_void_p(_stream(stream)))
     if rc != OK:
         raise RelationError(rc, "relation_linear_fwd_ex")
+    return out
+
+
+def linear_fwd_workspace_size(p1) -> int:
+    return int(load().relation_linear_fwd_workspace_size(shape_of(p1), _dtype_code(p1)))
+
+
+def linear_fwd_ws(p1, p2, v, alpha, tau_s: float = 2.0, *, workspace=None, out=None,
+                  dev_status=None, stream=None):
+    """Linear Relation forward through relation_linear_fwd_ws (the chunk-parallel form for
+    long sequences with few heads).  ``workspace``: a uint8 CUDA tensor of at least
+    linear_fwd_workspace_size(p1) bytes (allocated here when None).  Returns Y."""
+    _same_layout(p1, p2, v)
+    if alpha.dtype != torch.float32 or tuple(alpha.shape) != tuple(p1.shape) or \
+            tuple(alpha.stride()) != tuple(p1.stride()):
+        raise ValueError("alpha must be fp32 with p1's shape and strides")
+    out = torch.empty_like(p1) if out is None else out
+    _same_layout(p1, out)
+    need = linear_fwd_workspace_size(p1)
+    if workspace is None:
+        workspace = torch.empty(max(need, 16), dtype=torch.uint8, device=p1.device)
+    rc = load().relation_linear_fwd_ws(_ptr(p1), _ptr(p2), _ptr(v), _ptr(alpha), _ptr(out),
+                                       float(tau_s), shape_of(p1), _dtype_code(p1),
+                                       _ptr(workspace), workspace.numel(), _ptr(dev_status),
+                                       ctypes.c_void_p(_stream(stream)))
+    if rc != OK:
+        raise RelationError(rc, "relation_linear_fwd_ws")
     return out
 
 

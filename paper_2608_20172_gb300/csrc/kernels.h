@@ -128,8 +128,13 @@ bool linear_supports(relation_dtype dt, int d);
 cudaError_t launch_linear_fwd(const LinearProblem& p, cudaStream_t s);
 // Chunked tensor-core forward (relation_linear_tc.cu): bf16, d_h 64 or 128, element
 // strides multiples of 8.
+// workspace == nullptr: one CTA per (head, 64 columns) walks the blocks in order;
+// otherwise the chunk-parallel form (every block's state contribution in parallel, a scan
+// of the state over the blocks, every block's output in parallel) in that workspace of
+// linear_tc_workspace_bytes(p) bytes.
 bool linear_tc_supports(const LinearProblem& p);
-cudaError_t launch_linear_tc_fwd(const LinearProblem& p, cudaStream_t s);
+size_t linear_tc_workspace_bytes(const LinearProblem& p);
+cudaError_t launch_linear_tc_fwd(const LinearProblem& p, void* workspace, cudaStream_t s);
 size_t linear_bwd_workspace_bytes(int B, int H, int T, int d);
 cudaError_t launch_linear_bwd(const LinearProblem& p, cudaStream_t s);
 

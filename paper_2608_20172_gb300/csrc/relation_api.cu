@@ -155,8 +155,50 @@ relation_status relation_linear_fwd_ex(const void* p1, const void* p2, const voi
     return (dt == RELATION_BF16 && (shp.d_h == 64 || shp.d_h == 128)) ? RELATION_ERR_ALIGNMENT
                                                                      : RELATION_ERR_UNSUPPORTED;
   cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
-  if (tc && kernel != RELATION_KERNEL_SIMT) return from_cuda(rel::launch_linear_tc_fwd(p, s));
+  if (tc && kernel != RELATION_KERNEL_SIMT)
+    return from_cuda(rel::launch_linear_tc_fwd(p, nullptr, s));
   return from_cuda(rel::launch_linear_fwd(p, s));
+}
+
+size_t relation_linear_fwd_workspace_size(relation_shape shp, relation_dtype dt) {
+  if (dt != RELATION_BF16 || shp.B < 1 || shp.T < 1 || shp.H < 1) return 0;
+  rel::LinearProblem p{};
+  p.B = shp.B; p.T = shp.T; p.H = shp.H; p.d = shp.d_h;
+  p.sB = shp.sB; p.sT = shp.sT; p.sH = shp.sH; p.dtype = dt;
+  return rel::linear_tc_workspace_bytes(p);
+}
+
+relation_status relation_linear_fwd_ws(const void* p1, const void* p2, const void* v,
+                                      const float* alpha, void* y, float tau_s,
+                                      relation_shape shp, relation_dtype dt, void* workspace,
+                                      size_t ws_bytes, int* dev_status,
+                                      relation_stream_t stream) {
+  const size_t need = relation_linear_fwd_workspace_size(shp, dt);
+  if (need == 0)  // no chunked kernel for this request: the regular entry point decides
+    return relation_linear_fwd_ex(p1, p2, v, alpha, y, tau_s, shp, dt, RELATION_KERNEL_AUTO,
+                                  dev_status, stream);
+  if (!workspace || ws_bytes < need) return RELATION_ERR_WORKSPACE;
+  if (!aligned16(workspace)) return RELATION_ERR_ALIGNMENT;
+  int dev = 0, nsm = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess ||
+      cudaDeviceGetAttribute(&nsm, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess)
+    return RELATION_ERR_CUDA;
+  const long long ctas = (long long)shp.B * shp.H * (shp.d_h / 64);
+  // enough (head, column) pairs for the sequential walk (measured on GB300: 96 pairs on 152
+  // SMs still favour it, 0.14 against 0.19 ms; 12 pairs at T = 32768 take 1.9 ms against 0.38)
+  if (2 * ctas >= nsm)
+    return relation_linear_fwd_ex(p1, p2, v, alpha, y, tau_s, shp, dt, RELATION_KERNEL_TCGEN05,
+                                  dev_status, stream);
+  relation_status st;
+  if ((st = check_ptrs({p1, p2, v, alpha, y})) != RELATION_OK) return st;
+  if (!isfinite(tau_s) || !(tau_s > 0.0f)) return RELATION_ERR_INVALID_ARG;
+  if (dev_status && (reinterpret_cast<uintptr_t>(dev_status) & 3u)) return RELATION_ERR_ALIGNMENT;
+  if ((long long)ctas * ((shp.T + 127) / 128) > 0x7fffffffLL) return RELATION_ERR_UNSUPPORTED;
+  rel::LinearProblem p{};
+  p.p1 = p1; p.p2 = p2; p.v = v; p.alpha = alpha; p.y = y; p.dev_status = dev_status;
+  p.tau_s = tau_s; p.B = shp.B; p.T = shp.T; p.H = shp.H; p.d = shp.d_h;
+  p.sB = shp.sB; p.sT = shp.sT; p.sH = shp.sH; p.dtype = dt;
+  return from_cuda(rel::launch_linear_tc_fwd(p, workspace, reinterpret_cast<cudaStream_t>(stream)));
 }
 
 size_t relation_linear_bwd_workspace_size(relation_shape shp, relation_dtype dt) {

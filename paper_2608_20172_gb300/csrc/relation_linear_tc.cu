@@ -69,6 +69,21 @@ struct Cfg {
 };
 static_assert(Cfg<64>::SMEM <= 232448 && Cfg<128>::SMEM <= 232448, "shared memory");
 
+// Modes of the kernel: SEQ walks all blocks of a (head, split) in order with the state in
+// TMEM; the chunk-parallel pair takes one block per CTA: DELTA writes the block's state
+// contribution sum_j KL_j I~_j^T and decay a_L (fp32) to the workspace, OUT reads the
+// state the block starts from (bf16, produced by scan_kernel) and writes the block's Y.
+enum : int { MODE_SEQ = 0, MODE_DELTA = 1, MODE_OUT = 2 };
+
+// Workspace of the chunk-parallel forward, per (head, split, block): dC [D][64] fp32, the
+// decay g [D] fp32, and the entering state C0 [D][64] bf16.
+struct LinCp {
+  float* dC;
+  float* g;
+  __nv_bfloat16* c0;
+  int nb;
+};
+
 // B_LOAD, B_FREE, B_EPI: one per input stage (stage s at + s)
 enum : int { B_LOAD = 0, B_FREE = 2, B_EPI = 4, B_OPS = 6, B_C0, B_S, B_A, B_E, B_STATE, NBAR };
 
@@ -77,6 +92,15 @@ __device__ __forceinline__ void drain_wait(uint32_t bar, uint32_t parity) {
   while (!mbar_try_wait(bar, parity)) {
     if (globaltimer_ns() - t0 > 20ull * 1000ull * 1000ull) return;
   }
+}
+// 2-D tiled load into shared memory, completing on `bar` (transaction bytes).
+__device__ __forceinline__ void tma_load_2d(uint32_t dst, const CUtensorMap* m, uint32_t bar,
+                                            int c0, int c1) {
+  asm volatile(
+      "cp.async.bulk.tensor.2d.shared::cluster.global.mbarrier::complete_tx::bytes"
+      " [%0], [%1, {%3, %4}], [%2];" ::"r"(dst),
+      "l"(reinterpret_cast<uint64_t>(m)), "r"(bar), "r"(c0), "r"(c1)
+      : "memory");
 }
 __device__ __forceinline__ void ew_sync() {  // the 128 elementwise threads
   asm volatile("bar.sync 1, 128;" ::: "memory");
@@ -94,13 +118,14 @@ __device__ __forceinline__ void st_bf(uint8_t* base, uint32_t off, float x) {
   *reinterpret_cast<__nv_bfloat16*>(base + off) = __float2bfloat16_rn(x);
 }
 
-template <int D>
+template <int D, int MODE>
 __global__ void __launch_bounds__(kThreads, 1)
     lin_tc_fwd_kernel(const __grid_constant__ CUtensorMap tmP1,
                       const __grid_constant__ CUtensorMap tmP2,
                       const __grid_constant__ CUtensorMap tmV,
                       const __grid_constant__ CUtensorMap tmA,
-                      const __grid_constant__ CUtensorMap tmY, LinearProblem p) {
+                      const __grid_constant__ CUtensorMap tmY,
+                      const __grid_constant__ CUtensorMap tmC0, LinearProblem p, LinCp cp) {
   using C = Cfg<D>;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>(
@@ -110,7 +135,9 @@ __global__ void __launch_bounds__(kThreads, 1)
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(smem + C::OFF_BAR + 96);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(smem + C::OFF_BAR + 104);
   int* clamped = reinterpret_cast<int*>(smem + C::OFF_BAR + 108);
-  float* sq = reinterpret_cast<float*>(smem + C::OFF_C0);        // [128] S_t / |p1_t|
+  // per-token / per-channel scalars: in the C0 tile's space, or (OUT, where C0 is loaded
+  // with the inputs) in KL's, which that mode does not use
+  float* sq = reinterpret_cast<float*>(smem + (MODE == MODE_OUT ? C::OFF_KL : C::OFF_C0));
   float* sk = sq + LT;                                             // [128] S_t / |p2_t|
   float* half_sum = sk + LT;                                       // [2][128] (d_h = 64)
   float* lmid_s = half_sum + 2 * LT;                               // [128] L_m per channel
@@ -118,10 +145,14 @@ __global__ void __launch_bounds__(kThreads, 1)
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   constexpr int NSPLIT = D / NC;
-  const int split = (int)(blockIdx.x % NSPLIT);
-  const int bh = (int)(blockIdx.x / NSPLIT);
-  const int b = bh / p.H, h = bh % p.H;
   const int nb = (p.T + LT - 1) / LT;
+  // SEQ: one CTA per (head, split) over blocks [0, nb); DELTA / OUT: one block per CTA
+  const int cta_blk = MODE == MODE_SEQ ? 0 : (int)(blockIdx.x % nb);
+  const int bhs = MODE == MODE_SEQ ? (int)blockIdx.x : (int)(blockIdx.x / nb);
+  const int split = bhs % NSPLIT;
+  const int bh = bhs / NSPLIT;
+  const int b = bh / p.H, h = bh % p.H;
+  const int blk_first = cta_blk, blk_end = MODE == MODE_SEQ ? nb : cta_blk + 1;
 
   if (threadIdx.x == 0) {
     for (int i = 0; i < NBAR; ++i)  // arrivals of the 128 elementwise threads, or one
@@ -131,7 +162,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     *clamped = 0;
     fence_mbar_init();
   }
-  if (D == 64) {  // KL's channels 64..127 stay zero (the state product runs at M = 128)
+  if (D == 64 && MODE != MODE_OUT) {  // KL's channels 64..127 stay zero (M = 128 product)
     for (int i = threadIdx.x; i < LT * 64 * 2 / 16; i += kThreads)
       *reinterpret_cast<uint4*>(smem + C::OFF_KL + LT * 128 + i * 16) = make_uint4(0, 0, 0, 0);
     fence_async_smem();
@@ -151,8 +182,9 @@ __global__ void __launch_bounds__(kThreads, 1)
       tma_prefetch_desc(&tmV);
       tma_prefetch_desc(&tmA);
       int issued = 0;
-      for (int blk = 0; blk < nb; ++blk) {
-        const int st = blk % C::STAGES, use = blk / C::STAGES;
+      for (int blk = blk_first; blk < blk_end; ++blk) {
+        const int it = blk - blk_first;
+        const int st = it % C::STAGES, use = it / C::STAGES;
         // the stage's previous block: its MMAs and its output staging are done
         if (use > 0 && (!mbar_wait(bar(B_FREE + st), (use - 1) & 1, ab) ||
                         !mbar_wait(bar(B_EPI + st), (use - 1) & 1, ab)))
@@ -160,7 +192,9 @@ __global__ void __launch_bounds__(kThreads, 1)
         const int t0 = blk * LT;
         const uint32_t sg = sb + st * C::STAGE;
         const uint32_t lb = bar(B_LOAD + st);
-        mbar_arrive_expect_tx(lb, C::LOAD_BYTES);
+        mbar_arrive_expect_tx(lb, C::LOAD_BYTES + (MODE == MODE_OUT ? C::C0T : 0));
+        if (MODE == MODE_OUT)  // the state the block starts from, in the MN-major B layout
+          tma_load_2d(sb + C::OFF_C0, &tmC0, lb, 0, (bhs * nb + blk) * D);
         for (int kb = 0; kb < C::KB; ++kb) {
           tma_load_4d(sg + C::OFF_P1 + kb * LT * 128, &tmP1, lb, kb * 64, t0, h, b);
           tma_load_4d(sg + C::OFF_P2 + kb * LT * 128, &tmP2, lb, kb * 64, t0, h, b);
@@ -168,11 +202,11 @@ __global__ void __launch_bounds__(kThreads, 1)
         tma_load_4d(sg + C::OFF_V, &tmV, lb, split * NC, t0, h, b);
         for (int k = 0; k < D / 32; ++k)
           tma_load_4d(sg + C::OFF_A + k * LT * 128, &tmA, lb, k * 32, t0, h, b);
-        issued = blk + 1;
+        issued = it + 1;
       }
       if (ab.raised())  // copies in flight land before the CTA releases its shared memory
-        for (int blk = issued - C::STAGES > 0 ? issued - C::STAGES : 0; blk < issued; ++blk)
-          drain_wait(bar(B_LOAD + blk % C::STAGES), (blk / C::STAGES) & 1);
+        for (int it = issued - C::STAGES > 0 ? issued - C::STAGES : 0; it < issued; ++it)
+          drain_wait(bar(B_LOAD + it % C::STAGES), (it / C::STAGES) & 1);
     }
   } else if (warp == 5) {
     // ------------------------------------------------------------------ MMA issuer
@@ -180,41 +214,47 @@ __global__ void __launch_bounds__(kThreads, 1)
     constexpr uint32_t id_e = idesc_bf16_f32(128, NC, false, true);
     constexpr uint32_t id_c = idesc_bf16_f32(128, NC, true, true);
     bool ok = true;
-    for (int blk = 0; ok && blk < nb; ++blk) {
-      const uint32_t ph = blk & 1;
-      const int st = blk % C::STAGES;
+    for (int blk = blk_first; ok && blk < blk_end; ++blk) {
+      const int it = blk - blk_first;
+      const uint32_t ph = it & 1;
+      const int st = it % C::STAGES;
       const uint32_t sg = sb + st * C::STAGE;
       if (!(ok = mbar_wait_warp(bar(B_OPS), ph, ab))) break;
       tc_fence_after();
+      if (MODE != MODE_DELTA) {
 #pragma unroll
-      for (int kk = 0; kk < D / 16; ++kk) {  // S = Qm Km^T
-        const uint32_t koff = (kk >> 2) * (LT * 128) + (kk & 3) * 32;
-        mma_ss_w(tmem + COL_S, smem_desc_sw128(sg + C::OFF_P1 + koff, 16, 1024),
-                 smem_desc_sw128(sg + C::OFF_P2 + koff, 16, 1024), id_s, kk > 0 ? 1u : 0u);
+        for (int kk = 0; kk < D / 16; ++kk) {  // S = Qm Km^T
+          const uint32_t koff = (kk >> 2) * (LT * 128) + (kk & 3) * 32;
+          mma_ss_w(tmem + COL_S, smem_desc_sw128(sg + C::OFF_P1 + koff, 16, 1024),
+                   smem_desc_sw128(sg + C::OFF_P2 + koff, 16, 1024), id_s, kk > 0 ? 1u : 0u);
+        }
+        mma_commit_w(bar(B_S));
+        if (!(ok = mbar_wait_warp(bar(B_C0), ph, ab))) break;
+        tc_fence_after();
+#pragma unroll
+        for (int kk = 0; kk < D / 16; ++kk) {  // E = Qs C_0
+          const uint32_t koff = (kk >> 2) * (LT * 128) + (kk & 3) * 32;
+          mma_ss_w(tmem + COL_E, smem_desc_sw128(sb + C::OFF_QS + koff, 16, 1024),
+                   smem_desc_sw128(sb + C::OFF_C0 + kk * 16 * 128, D * 128, 1024), id_e,
+                   kk > 0 ? 1u : 0u);
+        }
+        if (!(ok = mbar_wait_warp(bar(B_A), ph, ab))) break;
+        tc_fence_after();
+#pragma unroll
+        for (int kk = 0; kk < LT / 16; ++kk)  // E += tril(S, -1) I~   (A from TMEM)
+          mma_ts_w(tmem + COL_E, tmem + COL_S + kk * 8,
+                   smem_desc_sw128(sg + C::OFF_V + kk * 16 * 128, LT * 128, 1024), id_e, 1u);
+        mma_commit_w(bar(B_E));
       }
-      mma_commit_w(bar(B_S));
-      if (!(ok = mbar_wait_warp(bar(B_C0), ph, ab))) break;
-      tc_fence_after();
+      if (MODE != MODE_OUT) {
+        // SEQ: C += KL^T I~ (C decayed by the threads); DELTA: the block's own sum
 #pragma unroll
-      for (int kk = 0; kk < D / 16; ++kk) {  // E = Qs C_0
-        const uint32_t koff = (kk >> 2) * (LT * 128) + (kk & 3) * 32;
-        mma_ss_w(tmem + COL_E, smem_desc_sw128(sb + C::OFF_QS + koff, 16, 1024),
-                 smem_desc_sw128(sb + C::OFF_C0 + kk * 16 * 128, D * 128, 1024), id_e,
-                 kk > 0 ? 1u : 0u);
+        for (int kk = 0; kk < LT / 16; ++kk)
+          mma_ss_w(tmem + COL_C, smem_desc_sw128(sb + C::OFF_KL + kk * 16 * 128, LT * 128, 1024),
+                   smem_desc_sw128(sg + C::OFF_V + kk * 16 * 128, LT * 128, 1024), id_c,
+                   ((MODE == MODE_SEQ && blk > 0) || kk > 0) ? 1u : 0u);
+        mma_commit_w(bar(B_STATE));
       }
-      if (!(ok = mbar_wait_warp(bar(B_A), ph, ab))) break;
-      tc_fence_after();
-#pragma unroll
-      for (int kk = 0; kk < LT / 16; ++kk)  // E += tril(S, -1) I~   (A from TMEM)
-        mma_ts_w(tmem + COL_E, tmem + COL_S + kk * 8,
-                 smem_desc_sw128(sg + C::OFF_V + kk * 16 * 128, LT * 128, 1024), id_e, 1u);
-      mma_commit_w(bar(B_E));
-#pragma unroll
-      for (int kk = 0; kk < LT / 16; ++kk)  // C += KL^T I~   (C decayed by the threads)
-        mma_ss_w(tmem + COL_C, smem_desc_sw128(sb + C::OFF_KL + kk * 16 * 128, LT * 128, 1024),
-                 smem_desc_sw128(sg + C::OFF_V + kk * 16 * 128, LT * 128, 1024), id_c,
-                 (blk > 0 || kk > 0) ? 1u : 0u);
-      mma_commit_w(bar(B_STATE));
       mma_commit_w(bar(B_FREE + st));
     }
     __syncwarp();
@@ -236,15 +276,16 @@ __global__ void __launch_bounds__(kThreads, 1)
     };
     float l_end = 0.f;  // this channel's L at the block's last token (phase C, c < D)
     bool ok = true, my_clamp = false;
-    for (int blk = 0; ok && blk < nb; ++blk) {
-      const uint32_t ph = blk & 1;
+    for (int blk = blk_first; ok && blk < blk_end; ++blk) {
+      const int it = blk - blk_first;
+      const uint32_t ph = it & 1;
       const int t0 = blk * LT;
-      const int st = blk % C::STAGES;
+      const int st = it % C::STAGES;
       uint8_t* const sg = smem + st * C::STAGE;
       p1s = sg + C::OFF_P1;
       p2s = sg + C::OFF_P2;
       al = reinterpret_cast<float*>(sg + C::OFF_A);
-      ok = __all_sync(0xffffffffu, mbar_wait(bar(B_LOAD + st), (blk / C::STAGES) & 1, ab));
+      ok = __all_sync(0xffffffffu, mbar_wait(bar(B_LOAD + st), (it / C::STAGES) & 1, ab));
       if (!ok) break;
       // ---- phase A: Ask Self of token t (rows past T give zero operands)
       {
@@ -309,7 +350,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       ew_sync();
       // Qs, KL and the state are single buffers: the last block's state product (the last
       // reader of KL; Qs's reader precedes B_E) must be done before they are written
-      if (blk > 0) {
+      if (MODE == MODE_SEQ && blk > 0) {
         ok = __all_sync(0xffffffffu, mbar_wait(bar(B_STATE), (blk - 1) & 1, ab));
         if (!ok) break;
         tc_fence_after();
@@ -352,25 +393,57 @@ __global__ void __launch_bounds__(kThreads, 1)
                 my_clamp = true;
               }
               const float xv = u ? x.y : x.x, yv = u ? y.y : y.x;
-              r[u][0] = xv * s1 * ex2_approx(dm);        // Qm
-              r[u][1] = yv * s2 * ex2_approx(-dm);       // Km
-              r[u][2] = xv * s1 * ex2_approx(L);         // Qs (factor <= 1)
-              r[u][3] = yv * s2 * ex2_approx(Ev[ch] - L);  // KL (factor <= 1)
+              if (MODE != MODE_DELTA) {
+                r[u][0] = xv * s1 * ex2_approx(dm);      // Qm
+                r[u][1] = yv * s2 * ex2_approx(-dm);     // Km
+                r[u][2] = xv * s1 * ex2_approx(L);       // Qs (factor <= 1)
+              }
+              if (MODE != MODE_OUT) r[u][3] = yv * s2 * ex2_approx(Ev[ch] - L);  // KL (<= 1)
             }
-            qm[e] = pack_bf16x2(r[0][0], r[1][0]);
-            km[e] = pack_bf16x2(r[0][1], r[1][1]);
-            qs[e] = pack_bf16x2(r[0][2], r[1][2]);
-            kl[e] = pack_bf16x2(r[0][3], r[1][3]);
+            if (MODE != MODE_DELTA) {
+              qm[e] = pack_bf16x2(r[0][0], r[1][0]);
+              km[e] = pack_bf16x2(r[0][1], r[1][1]);
+              qs[e] = pack_bf16x2(r[0][2], r[1][2]);
+            }
+            if (MODE != MODE_OUT) kl[e] = pack_bf16x2(r[0][3], r[1][3]);
           }
-          *reinterpret_cast<uint4*>(p1s + off) = make_uint4(qm[0], qm[1], qm[2], qm[3]);
-          *reinterpret_cast<uint4*>(p2s + off) = make_uint4(km[0], km[1], km[2], km[3]);
-          *reinterpret_cast<uint4*>(smem + C::OFF_QS + off) = make_uint4(qs[0], qs[1], qs[2], qs[3]);
-          *reinterpret_cast<uint4*>(smem + C::OFF_KL + off) = make_uint4(kl[0], kl[1], kl[2], kl[3]);
+          if (MODE != MODE_DELTA) {
+            *reinterpret_cast<uint4*>(p1s + off) = make_uint4(qm[0], qm[1], qm[2], qm[3]);
+            *reinterpret_cast<uint4*>(p2s + off) = make_uint4(km[0], km[1], km[2], km[3]);
+            *reinterpret_cast<uint4*>(smem + C::OFF_QS + off) =
+                make_uint4(qs[0], qs[1], qs[2], qs[3]);
+          }
+          if (MODE != MODE_OUT)
+            *reinterpret_cast<uint4*>(smem + C::OFF_KL + off) =
+                make_uint4(kl[0], kl[1], kl[2], kl[3]);
         }
       }
       fence_async_smem();
       ew_sync();
       mbar_arrive(bar(B_OPS));
+      if (MODE == MODE_DELTA) {
+        // the block's state contribution and decay, to the workspace
+        ok = __all_sync(0xffffffffu, mbar_wait(bar(B_STATE), 0, ab));
+        if (!ok) break;
+        tc_fence_after();
+        if (t < D) {
+          uint32_t z[64];
+          tmem_ld32(trow + COL_C, z);
+          tmem_ld32(trow + COL_C + 32, z + 32);
+          tmem_ld_wait();
+          const long long row = (long long)(bhs * nb + blk) * D + t;
+          float4* dst = reinterpret_cast<float4*>(cp.dC + row * 64);
+#pragma unroll
+          for (int k = 0; k < 16; ++k)
+            dst[k] = make_float4(__uint_as_float(z[4 * k]), __uint_as_float(z[4 * k + 1]),
+                                 __uint_as_float(z[4 * k + 2]), __uint_as_float(z[4 * k + 3]));
+          cp.g[row] = ex2_approx(l_end);
+        }
+        continue;
+      }
+      if (MODE == MODE_OUT) {
+        mbar_arrive(bar(B_C0));  // C0 came with the block's inputs
+      } else {
       // ---- phase C: the state after the last block (complete, waited above), its bf16
       // copy, then decayed by a_L
       if (t < D) {
@@ -406,6 +479,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       fence_async_smem();
       tc_fence_before();
       mbar_arrive(bar(B_C0));
+      }
       // ---- phase D: S masked to the strictly earlier tokens, packed to bf16 in place
       ok = __all_sync(0xffffffffu, mbar_wait(bar(B_S), ph, ab));
       if (!ok) break;
@@ -497,25 +571,144 @@ static bool make_tmap_alpha(CUtensorMap* m, const LinearProblem& p) {
             CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
+// Sequential scan of the state over the blocks of one (head, split), for the chunk-parallel
+// forward: C_0(0) = 0, C_0(b + 1) = Diag(g_b) C_0(b) + dC_b, each C_0(b) written in bf16
+// (row-major [D][64] per block, the OUT pass's B operand after a swizzled TMA load).  A CTA
+// takes 8 channels x 64 columns, two per thread (a warp = one channel's 64 columns,
+// coalesced); the loads of the next 8 blocks are in flight while 8 are combined.
 template <int D>
-static cudaError_t fwd_t(const LinearProblem& lp, cudaStream_t s) {
+__global__ void __launch_bounds__(256) scan_kernel(LinCp cp) {
+  constexpr int CPB = 8, P = 8;
+  const int cg = (int)(blockIdx.x % (D / CPB));
+  const int bhs = (int)(blockIdx.x / (D / CPB));
+  const int c = cg * CPB + (int)(threadIdx.x >> 5);
+  const int n = (int)(threadIdx.x & 31) * 2;
+  const int nb = cp.nb;
+  const long long base = (long long)bhs * nb * D + c;  // row of block blk: base + blk D
+  auto load = [&](int b0, float2 (&dv)[P], float (&gv)[P]) {
+#pragma unroll
+    for (int u = 0; u < P; ++u) {
+      const int blk = b0 + u;
+      if (blk < nb) {
+        const long long row = base + (long long)blk * D;
+        dv[u] = *reinterpret_cast<const float2*>(cp.dC + row * 64 + n);
+        gv[u] = cp.g[row];
+      } else {
+        dv[u] = make_float2(0.f, 0.f);
+        gv[u] = 1.f;
+      }
+    }
+  };
+  float2 st = make_float2(0.f, 0.f), cur[P];
+  float gc[P];
+  load(0, cur, gc);
+  for (int b0 = 0; b0 < nb; b0 += P) {
+    float2 nxt[P];
+    float gn[P];
+    load(b0 + P, nxt, gn);
+#pragma unroll
+    for (int u = 0; u < P; ++u) {
+      const int blk = b0 + u;
+      if (blk < nb) {
+        const long long row = base + (long long)blk * D;
+        *reinterpret_cast<__nv_bfloat162*>(cp.c0 + row * 64 + n) = __floats2bfloat162_rn(st.x, st.y);
+        st = make_float2(fmaf(gc[u], st.x, cur[u].x), fmaf(gc[u], st.y, cur[u].y));
+      }
+    }
+#pragma unroll
+    for (int u = 0; u < P; ++u) {
+      cur[u] = nxt[u];
+      gc[u] = gn[u];
+    }
+  }
+}
+
+// 2-D map over the bf16 C0 rows of the workspace: [rows][64], boxes of D rows, 128-byte
+// swizzle (the MN-major B layout of the E = Qs C_0 product).
+static bool make_tmap_c0(CUtensorMap* m, void* base, long long rows, int d) {
+  static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
+  if (!fn) {
+    void* ptr = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &ptr, 12000, cudaEnableDefault,
+                                         &q) != cudaSuccess ||
+        q != cudaDriverEntryPointSuccess)
+      return false;
+    fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(ptr);
+  }
+  cuuint64_t dims[2] = {64, (cuuint64_t)rows};
+  cuuint64_t strides[1] = {128};
+  cuuint32_t box[2] = {64, (cuuint32_t)d};
+  cuuint32_t estr[2] = {1, 1};
+  return fn(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, base, dims, strides, box, estr,
+            CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+            CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+static size_t align256(size_t x) { return (x + 255) & ~(size_t)255; }
+
+// Workspace layout of the chunk-parallel forward: dC, g, C0 (see LinCp).
+static size_t cp_bytes(long long rows, LinCp* out, void* base) {
+  const size_t b_dc = align256((size_t)rows * 64 * 4), b_g = align256((size_t)rows * 4);
+  const size_t b_c0 = align256((size_t)rows * 64 * 2);
+  if (out) {
+    uint8_t* q = static_cast<uint8_t*>(base);
+    out->dC = reinterpret_cast<float*>(q);
+    out->g = reinterpret_cast<float*>(q + b_dc);
+    out->c0 = reinterpret_cast<__nv_bfloat16*>(q + b_dc + b_g);
+  }
+  return b_dc + b_g + b_c0;
+}
+
+template <int D>
+static cudaError_t fwd_t(const LinearProblem& lp, void* workspace, cudaStream_t s) {
   const int smem = Cfg<D>::SMEM;
-  cudaError_t e =
-      cudaFuncSetAttribute(lin_tc_fwd_kernel<D>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
-  if (e != cudaSuccess) { note_failure("linear chunked forward: shared memory attribute"); return e; }
+  const bool cp_path = workspace != nullptr;
+  cudaError_t e;
+  for (auto fn : {lin_tc_fwd_kernel<D, MODE_SEQ>, lin_tc_fwd_kernel<D, MODE_DELTA>,
+                  lin_tc_fwd_kernel<D, MODE_OUT>})
+    if ((e = cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, smem)) !=
+        cudaSuccess) {
+      note_failure("linear chunked forward: shared memory attribute");
+      return e;
+    }
   Problem p{};  // the bf16 tensor-map helper's view of the shapes
   p.B = lp.B; p.T = lp.T; p.H = lp.H; p.d = lp.d;
   p.sB = lp.sB; p.sT = lp.sT; p.sH = lp.sH;
-  CUtensorMap m1, m2, mv, ma, my;
+  const int nb = (lp.T + LT - 1) / LT;
+  const long long heads = (long long)lp.B * lp.H * (D / NC);
+  LinCp cp{};
+  cp.nb = nb;
+  CUtensorMap m1, m2, mv, ma, my, mc;
   if (!tc::make_tmap_bf16(&m1, lp.p1, p, LT) || !tc::make_tmap_bf16(&m2, lp.p2, p, LT) ||
       !tc::make_tmap_bf16(&mv, lp.v, p, LT) || !tc::make_tmap_bf16(&my, lp.y, p, 32) ||
       !make_tmap_alpha(&ma, lp)) {
     note_failure("linear chunked forward: TMA descriptors");
     return cudaErrorInvalidValue;
   }
-  const long long grid = (long long)lp.B * lp.H * (D / NC);
-  if (grid > 0x7fffffffLL) return cudaErrorInvalidConfiguration;
-  lin_tc_fwd_kernel<D><<<(unsigned)grid, kThreads, smem, s>>>(m1, m2, mv, ma, my, lp);
+  mc = m1;  // unused by the sequential mode
+  if (cp_path) {
+    cp_bytes(heads * nb * D, &cp, workspace);
+    if (!make_tmap_c0(&mc, cp.c0, heads * nb * D, D)) {
+      note_failure("linear chunked forward: TMA descriptor of the workspace");
+      return cudaErrorInvalidValue;
+    }
+  }
+  if (!cp_path) {
+    if (heads > 0x7fffffffLL) return cudaErrorInvalidConfiguration;
+    lin_tc_fwd_kernel<D, MODE_SEQ><<<(unsigned)heads, kThreads, smem, s>>>(m1, m2, mv, ma, my, mc,
+                                                                          lp, cp);
+  } else {
+    const long long grid = heads * nb;
+    if (grid > 0x7fffffffLL) return cudaErrorInvalidConfiguration;
+    lin_tc_fwd_kernel<D, MODE_DELTA><<<(unsigned)grid, kThreads, smem, s>>>(m1, m2, mv, ma, my, mc,
+                                                                           lp, cp);
+    if ((e = cudaGetLastError()) != cudaSuccess) { note_failure("linear chunked forward: launch"); return e; }
+    scan_kernel<D><<<(unsigned)(heads * (D / 8)), 256, 0, s>>>(cp);
+    if ((e = cudaGetLastError()) != cudaSuccess) { note_failure("linear chunked forward: launch"); return e; }
+    lin_tc_fwd_kernel<D, MODE_OUT><<<(unsigned)grid, kThreads, smem, s>>>(m1, m2, mv, ma, my, mc,
+                                                                         lp, cp);
+  }
   if ((e = cudaGetLastError()) != cudaSuccess) note_failure("linear chunked forward: launch");
   return e;
 }
@@ -527,9 +720,16 @@ bool linear_tc_supports(const LinearProblem& p) {
          p.sT % 8 == 0 && p.sH % 8 == 0;
 }
 
-cudaError_t launch_linear_tc_fwd(const LinearProblem& p, cudaStream_t s) {
+size_t linear_tc_workspace_bytes(const LinearProblem& p) {
+  if (!linear_tc_supports(p)) return 0;
+  const long long heads = (long long)p.B * p.H * (p.d / lintc::NC);
+  const long long nb = (p.T + lintc::LT - 1) / lintc::LT;
+  return lintc::cp_bytes(heads * nb * p.d, nullptr, nullptr);
+}
+
+cudaError_t launch_linear_tc_fwd(const LinearProblem& p, void* workspace, cudaStream_t s) {
   if (!linear_tc_supports(p)) return cudaErrorInvalidValue;
-  return p.d == 64 ? lintc::fwd_t<64>(p, s) : lintc::fwd_t<128>(p, s);
+  return p.d == 64 ? lintc::fwd_t<64>(p, workspace, s) : lintc::fwd_t<128>(p, workspace, s);
 }
 
 }  // namespace rel

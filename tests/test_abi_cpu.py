@@ -247,6 +247,26 @@ def test_linear_fwd_ex_family_rules(lib, case, expect):
     assert rc == expect
 
 
+def test_linear_fwd_ws_workspace_rules(lib):
+    """The chunk-parallel forward's workspace: B H (d/64) ceil(T/128) d rows of 64 fp32 dC,
+    one fp32 decay and 64 bf16 of entering state, each array padded to 256 bytes; fp32 and
+    other widths need none; a short or misaligned workspace is refused before any launch."""
+    shape = _shape(B=1, T=300, H=2, d=64)
+    rows = 1 * 2 * 1 * 3 * 64
+    pad = lambda x: (x + 255) // 256 * 256
+    need = lib.relation_linear_fwd_workspace_size(shape, binding.BF16)
+    assert need == pad(rows * 64 * 4) + pad(rows * 4) + pad(rows * 64 * 2)
+    assert lib.relation_linear_fwd_workspace_size(shape, binding.F32) == 0
+    assert lib.relation_linear_fwd_workspace_size(_shape(d=32), binding.BF16) == 0
+    p = [ctypes.c_void_p(0x10000 * (i + 1)) for i in range(5)]
+    rc = lib.relation_linear_fwd_ws(*p, 2.0, shape, binding.BF16, ctypes.c_void_p(0x100000),
+                                    need - 1, None, None)
+    assert rc == binding.ERR_WORKSPACE
+    rc = lib.relation_linear_fwd_ws(*p, 2.0, shape, binding.BF16, ctypes.c_void_p(0x100008),
+                                    need, None, None)
+    assert rc == binding.ERR_ALIGNMENT
+
+
 def test_linear_bwd_workspace_rules(lib):
     shape = _shape(B=2, T=20, H=3, d=64)
     need = lib.relation_linear_bwd_workspace_size(shape, binding.BF16)

@@ -139,3 +139,41 @@ def test_linear_chunked_reports_decay_beyond_its_range():
     assert int(st_tc.item()) == binding.ERR_UNSUPPORTED
     assert int(st_rec.item()) == 0
     assert torch.isfinite(y.float()).all()
+
+
+@pytest.mark.parametrize("d", [64, 128])
+@pytest.mark.parametrize("T", [1, 129, 1000, 4097])
+def test_linear_forward_chunk_parallel(d, T):
+    """The chunk-parallel form (few heads: every block's state contribution, the scan over
+    blocks, every block's output in parallel) against the fp64 recurrence on every head, and
+    against the sequential chunked kernel."""
+    w = workloads.custom(1, 2, T, d, "bf16")
+    p1, p2, v, alpha, _ = workloads.make_linear_inputs(w, seed=900 + T + d)
+    dev = torch.device("cuda:0")
+    args = [t.to(dev) for t in (p1, p2, v, alpha)]
+    status = torch.zeros(1, dtype=torch.int32, device=dev)
+    assert binding.linear_fwd_workspace_size(args[0]) > 0
+    y = binding.linear_fwd_ws(*args, dev_status=status)
+    y_seq = binding.linear_fwd(*args, kernel="tcgen05", dev_status=status)
+    torch.cuda.synchronize()
+    assert int(status.item()) == 0
+    y, y_seq = y.float().cpu().numpy(), y_seq.float().cpu().numpy()
+    for h in range(w.H):
+        ref, _ = oracle.linear_fwd(_heads(p1, 0, h), _heads(p2, 0, h), _heads(v, 0, h),
+                                   _heads(alpha, 0, h))
+        pu.check_recorded("linear chunk-parallel", f"Y d={d}", y[0, :, h], ref, "bf16", "out")
+        pu.check(f"chunk-parallel vs sequential h={h}", y[0, :, h], y_seq[0, :, h], "bf16", "out")
+
+
+def test_linear_forward_ws_many_heads_uses_the_sequential_walk():
+    """With at least half as many (head, column) pairs as SMs the workspace entry point takes
+    the sequential chunked kernel: its output equals relation_linear_fwd_ex(TCGEN05) bit for
+    bit."""
+    w = workloads.custom(4, 40, 300, 64, "bf16")
+    p1, p2, v, alpha, _ = workloads.make_linear_inputs(w, seed=4)
+    dev = torch.device("cuda:0")
+    args = [t.to(dev) for t in (p1, p2, v, alpha)]
+    y = binding.linear_fwd_ws(*args)
+    y_seq = binding.linear_fwd(*args, kernel="tcgen05")
+    torch.cuda.synchronize()
+    assert torch.equal(y, y_seq)
