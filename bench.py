@@ -416,6 +416,18 @@ def _linear_chunked_flops(B, H, T, d):
     return float(B * H * nb * splits * per)
 
 
+def _linear_chunked_bwd_flops(B, H, T, d):
+    """Tensor-core work of the chunked backward per call (d_h = 64), as executed: per
+    128-token block, the two state passes' block products (KL^T I~ and Qs^T dY, 2 128 64 128
+    each with the channels padded to 128), then S = Qm Km^T and dA = G I~^T (2 128 128 64
+    each), X = G C_0^T, Y = I~ dC^T and dI~ = KL dC (2 128 64 64 each), dI~ += A^T G,
+    X += dA Km and Y += dA^T Qm (2 128 64 128 each)."""
+    nb = -(-T // 128)
+    per = 2 * (2 * 128 * 64 * 128) + 2 * (2 * 128 * 128 * d) + 3 * (2 * 128 * 64 * d) + \
+        3 * (2 * 128 * 64 * 128)
+    return float(B * H * nb * per)
+
+
 def _time_calls(call, dev, steps, warmup):
     stream = torch.cuda.current_stream(dev)
     for _ in range(warmup):
@@ -431,11 +443,12 @@ def _time_calls(call, dev, steps, warmup):
 
 
 def linear_measure(binding, dev, peaks, steps=20, warmup=3):
-    """Linear Relation on the 100M geometry (bf16): the chunked tensor-core forward, the
-    recurrent CUDA-core forward and backward.  Recurrent arithmetic per token and head:
+    """Linear Relation on the 100M geometry (bf16): the chunked tensor-core forward and
+    backward, the recurrent CUDA-core forward and backward.  Recurrent arithmetic per token and head:
     forward 5 d^2 (decay, read, write), backward 16 d^2; ALU roofline against the fp32 FMA
     peak of the SMs.  Chunked forward: tensor-core work as counted by _linear_chunked_flops,
-    against the measured bf16 peak.  Then the long-context sweep of the chunked forward,
+    against the measured bf16 peak; chunked backward likewise (_linear_chunked_bwd_flops).
+    Then the long-context sweep of the chunked forward,
     T = 1k .. 32k at B T = 32768 tokens."""
     c = LINEAR_CFG
     w = workloads.custom(c["B"], c["H"], c["T"], c["d_h"], "bf16")
@@ -443,16 +456,17 @@ def linear_measure(binding, dev, peaks, steps=20, warmup=3):
     out = torch.empty_like(p1)
     status = torch.zeros(1, dtype=torch.int32, device=dev)
     stream = torch.cuda.current_stream(dev)
-    need = int(binding.load().relation_linear_bwd_workspace_size(binding.shape_of(p1),
-                                                                  binding.BF16))
+    need = max(binding.linear_bwd_workspace_size(p1, "simt"),
+               binding.linear_bwd_workspace_size(p1, "tcgen05"))
     wsb = torch.empty(need, dtype=torch.uint8, device=dev)
     fwd = lambda fam: (lambda: binding.linear_fwd(p1, p2, v, alpha, kernel=fam, out=out,
                                                   dev_status=status, stream=stream))
-    bwd = lambda: binding.linear_bwd(p1, p2, v, alpha, dy, workspace=wsb, dev_status=status,
-                                     stream=stream)
+    bwd = lambda fam: (lambda: binding.linear_bwd(p1, p2, v, alpha, dy, kernel=fam, workspace=wsb,
+                                                  dev_status=status, stream=stream))
     ms_tc = _time_calls(fwd("tcgen05"), dev, steps, warmup)
     ms_f = _time_calls(fwd("simt"), dev, steps, warmup)
-    ms_b = _time_calls(bwd, dev, steps, warmup)
+    ms_btc = _time_calls(bwd("tcgen05"), dev, steps, warmup)
+    ms_b = _time_calls(bwd("simt"), dev, steps, warmup)
     if int(status.item()) != 0:
         raise SystemExit(f"linear device status {binding.status_string(int(status.item()))}")
     tok_h = w.B * w.T * w.H
@@ -460,6 +474,8 @@ def linear_measure(binding, dev, peaks, steps=20, warmup=3):
     ach = fl_f / (ms_f * 1e-3) / 1e12
     tc_fl = _linear_chunked_flops(w.B, w.H, w.T, w.d)
     tc_ach = tc_fl / (ms_tc * 1e-3) / 1e12
+    tcb_fl = _linear_chunked_bwd_flops(w.B, w.H, w.T, w.d)
+    tcb_ach = tcb_fl / (ms_btc * 1e-3) / 1e12
     sweep = []
     for T in (1024, 2048, 4096, 8192, 16384, 32768):
         B = max(1, LINEAR_SWEEP_TOKENS // T)
@@ -479,8 +495,8 @@ def linear_measure(binding, dev, peaks, steps=20, warmup=3):
     if int(status.item()) != 0:
         raise SystemExit(f"linear device status {binding.status_string(int(status.item()))}")
     return {"config": {**c, "dtype": "bf16", "alpha": "KDA-style draw (workloads)"},
-            "ms_fwd_chunked": ms_tc, "ms_fwd": ms_f, "ms_bwd": ms_b,
-            "tokens_per_s": w.B * w.T / ((ms_tc + ms_b) * 1e-3),
+            "ms_fwd_chunked": ms_tc, "ms_bwd_chunked": ms_btc, "ms_fwd": ms_f, "ms_bwd": ms_b,
+            "tokens_per_s": w.B * w.T / ((ms_tc + ms_btc) * 1e-3),
             "roofline": {"bound": "alu", "kernel": "linear fwd_kernel (recurrent)", "achieved": ach,
                          "peak": FP32_FMA_TFLOPS, "unit": "TFLOP/s (fp32 FMA)",
                          "frac": ach / FP32_FMA_TFLOPS,
@@ -489,11 +505,16 @@ def linear_measure(binding, dev, peaks, steps=20, warmup=3):
                                  "achieved": tc_ach, "peak": peaks["bf16_tflops"],
                                  "unit": "TFLOP/s", "frac": tc_ach / peaks["bf16_tflops"],
                                  "algorithmic_flops_per_launch": tc_fl},
+            "roofline_chunked_bwd": {"bound": "tensor",
+                                     "kernel": "chunked backward (five launches)",
+                                     "achieved": tcb_ach, "peak": peaks["bf16_tflops"],
+                                     "unit": "TFLOP/s", "frac": tcb_ach / peaks["bf16_tflops"],
+                                     "flops_per_call": tcb_fl},
             "long_context_sweep": {"kernel": "chunked forward with a workspace (chunk-parallel "
                                              "below one (head, column) pair per SM)",
                                    "H": 12, "d_h": 64,
                                    "tokens_per_point": LINEAR_SWEEP_TOKENS, "points": sweep},
-            "gpu_launches_per_step": {"fwd_chunked": 1, "fwd": 1, "bwd": 2}}
+            "gpu_launches_per_step": {"fwd_chunked": 1, "bwd_chunked": 5, "fwd": 1, "bwd": 2}}
 
 
 def measure_workload(binding, w, dev, steps, warmup, family, peaks, dist=None, ws=1,

@@ -165,7 +165,8 @@ relation_status relation_linear_fwd_ex(const void* p1, const void* p2, const voi
  * its decay, fp32), then a scan of the state over the blocks, then every block's output from
  * the state it starts from (stored in bf16 between the passes; three launches).
  *   workspace : device scratch of relation_linear_fwd_workspace_size(shp, dt) bytes
- *               (B H (d_h / 64) ceil(T / 128) d_h rows of 64 fp32 + 64 bf16 + 1 fp32),
+ *               (B H (d_h / 64) ceil(T / 128) d_h rows of 64 + 1 fp32, and
+ *               B H (d_h / 64) (ceil(T / 128) + 1) d_h rows of 64 bf16),
  *               16-byte aligned, or RELATION_ERR_WORKSPACE / RELATION_ERR_ALIGNMENT with
  *               nothing launched.
  * The chunk-parallel form runs when B H (d_h / 64) is below half the device's SM count, the
@@ -187,10 +188,11 @@ relation_status relation_linear_fwd_ws(const void* p1, const void* p2, const voi
  * writes out the forward only), given dy = dL/dY:
  *   dp1, dp2, dv : [B][T][H][d_h] in dt, with the inputs' strides (overwritten);
  *   dalpha       : [B][T][H][d_h] fp32 with alpha's strides (overwritten);
- *   workspace    : device scratch of relation_linear_bwd_workspace_size(shp, dt) bytes
- *                  (state checkpoints every 8 tokens plus fp32 partial row sums of the
- *                  state's column splits, [B][H][splits][T][3][d_h]).
- * Same dtypes and widths as relation_linear_fwd; asynchronous on `stream`.
+ *   workspace    : device scratch of relation_linear_bwd_workspace_size(shp, dt) bytes,
+ *                  the size relation_linear_bwd_ex_workspace_size gives for
+ *                  RELATION_KERNEL_AUTO (16-byte aligned).
+ * Same dtypes and widths as relation_linear_fwd; asynchronous on `stream`.  Equals
+ * relation_linear_bwd_ex(..., RELATION_KERNEL_AUTO, ...).
  */
 size_t relation_linear_bwd_workspace_size(relation_shape shp, relation_dtype dt);
 relation_status relation_linear_bwd(const void* p1, const void* p2, const void* v,
@@ -198,6 +200,38 @@ relation_status relation_linear_bwd(const void* p1, const void* p2, const void* 
                                    void* dv, float* dalpha, float tau_s, relation_shape shp,
                                    relation_dtype dt, void* workspace, size_t ws_bytes,
                                    int* dev_status, relation_stream_t stream);
+
+/*
+ * relation_linear_bwd with the kernel family chosen (relation_kernel, as for the forward):
+ *   RELATION_KERNEL_SIMT    reverse mode through the token recurrence on CUDA cores (every
+ *                           dtype and width of relation_linear_fwd).  Workspace: state
+ *                           checkpoints every 8 tokens plus fp32 partial row sums of the
+ *                           state's column splits, B H (ceil(T / 8) d_h^2 + (d_h / 32) T 3 d_h)
+ *                           fp32.
+ *   RELATION_KERNEL_TCGEN05 reverse mode through the 128-token blocks of the chunked
+ *                           forward, every block in parallel: the states entering every block
+ *                           (a forward state pass), the state's adjoint leaving every block
+ *                           (dC(b - 1) = Diag(a_L(b)) dC(b) + Qs_b^T dY_b, a reverse pass),
+ *                           then per block the gradients as tcgen05 products with bf16
+ *                           operands and fp32 accumulation (five launches).  bf16 with d_h = 64,
+ *                           element strides multiples of 8 (else RELATION_ERR_UNSUPPORTED or
+ *                           RELATION_ERR_ALIGNMENT, nothing launched).  Workspace, in
+ *                           256-byte-aligned parts, with n = ceil(T / 128): B H n 64 rows of 64
+ *                           fp32, B H n 64 fp32, B H (n + 1) 64 rows of 64 bf16 (the states,
+ *                           the final one last) and B H n 64 rows of 64 bf16 (the adjoints).
+ *                           The decay-range clamp and its report are the chunked forward's.
+ *   RELATION_KERNEL_AUTO    the chunked kernel where it applies, else the recurrence.
+ * workspace is 16-byte aligned and holds relation_linear_bwd_ex_workspace_size(shp, dt,
+ * kernel) bytes (0: the family does not serve the request), else RELATION_ERR_WORKSPACE /
+ * RELATION_ERR_ALIGNMENT with nothing launched.  Other arguments as relation_linear_bwd.
+ */
+size_t relation_linear_bwd_ex_workspace_size(relation_shape shp, relation_dtype dt,
+                                             relation_kernel kernel);
+relation_status relation_linear_bwd_ex(const void* p1, const void* p2, const void* v,
+                                      const float* alpha, const void* dy, void* dp1, void* dp2,
+                                      void* dv, float* dalpha, float tau_s, relation_shape shp,
+                                      relation_dtype dt, relation_kernel kernel, void* workspace,
+                                      size_t ws_bytes, int* dev_status, relation_stream_t stream);
 
 /*
  * Decoding: the forward row of one new token per sequence, against a key/value cache.

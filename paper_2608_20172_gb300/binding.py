@@ -33,7 +33,8 @@ EXPORTED = ("relation_fwd", "relation_fwd_ex", "relation_bwd", "relation_bwd_ex"
             "relation_decode", "relation_decode_workspace_size", "relation_linear_fwd",
             "relation_linear_fwd_ex", "relation_linear_fwd_ws",
             "relation_linear_fwd_workspace_size",
-            "relation_linear_bwd", "relation_linear_bwd_workspace_size", "relation_layer_prep",
+            "relation_linear_bwd", "relation_linear_bwd_workspace_size",
+            "relation_linear_bwd_ex", "relation_linear_bwd_ex_workspace_size", "relation_layer_prep",
             "relation_layer_grad", "relation_layer_grad_workspace_size")
 
 
@@ -88,6 +89,10 @@ def load(path: str | None = None):
         lib.relation_linear_bwd.argtypes = [vp, vp, vp, vp, vp, vp, vp, vp, vp, f, Shape, i, vp,
                                             ctypes.c_size_t, ip, vp]
         lib.relation_linear_bwd_workspace_size.argtypes = [Shape, i]
+        lib.relation_linear_bwd_ex.argtypes = [vp, vp, vp, vp, vp, vp, vp, vp, vp, f, Shape, i, i,
+                                               vp, sz, ip, vp]
+        lib.relation_linear_bwd_ex_workspace_size.argtypes = [Shape, i, i]
+        lib.relation_linear_bwd_ex_workspace_size.restype = sz
         lib.relation_layer_prep.argtypes = [vp, vp, vp, vp, i, f, vp, vp, vp, Shape, i, vp]
         lib.relation_layer_grad.argtypes = [vp, vp, vp, vp, vp, i, f, vp, vp, vp, vp, Shape, i,
                                             vp, sz, vp]
@@ -253,25 +258,35 @@ def linear_fwd_ws(p1, p2, v, alpha, tau_s: float = 2.0, *, workspace=None, out=N
     return out
 
 
-def linear_bwd(p1, p2, v, alpha, dy, tau_s: float = 2.0, *, workspace=None, dev_status=None,
-               stream=None):
-    """Linear Relation backward.  Returns (dp1, dp2, dv, dalpha) with dalpha fp32."""
+def linear_bwd_workspace_size(p1, kernel: str = "auto") -> int:
+    """Bytes of device scratch linear_bwd needs for tensors shaped like p1 (0: the kernel
+    family does not serve this request)."""
+    return int(load().relation_linear_bwd_ex_workspace_size(shape_of(p1), _dtype_code(p1),
+                                                            KERNELS[kernel]))
+
+
+def linear_bwd(p1, p2, v, alpha, dy, tau_s: float = 2.0, *, kernel: str = "auto",
+               workspace=None, dev_status=None, stream=None):
+    """Linear Relation backward.  Returns (dp1, dp2, dv, dalpha) with dalpha fp32.
+    ``kernel``: "auto", "simt" (reverse mode through the token recurrence) or "tcgen05"
+    (through the 128-token blocks of the chunked forward; bf16, d_h 64)."""
     _same_layout(p1, p2, v, dy)
     if alpha.dtype != torch.float32 or tuple(alpha.shape) != tuple(p1.shape) or \
             tuple(alpha.stride()) != tuple(p1.stride()):
         raise ValueError("alpha must be fp32 with p1's shape and strides")
     dp1, dp2, dv = torch.empty_like(p1), torch.empty_like(p1), torch.empty_like(p1)
     dalpha = torch.empty_like(alpha)
-    need = int(load().relation_linear_bwd_workspace_size(shape_of(p1), _dtype_code(p1)))
+    need = linear_bwd_workspace_size(p1, kernel)
     if workspace is None:
         workspace = torch.empty(max(need, 16), device=p1.device, dtype=torch.uint8)
-    rc = load().relation_linear_bwd(_ptr(p1), _ptr(p2), _ptr(v), _ptr(alpha), _ptr(dy),
-                                    _ptr(dp1), _ptr(dp2), _ptr(dv), _ptr(dalpha), float(tau_s),
-                                    shape_of(p1), _dtype_code(p1), _ptr(workspace),
-                                    workspace.numel() * workspace.element_size(),
-                                    _ptr(dev_status), ctypes.c_void_p(_stream(stream)))
+    rc = load().relation_linear_bwd_ex(_ptr(p1), _ptr(p2), _ptr(v), _ptr(alpha), _ptr(dy),
+                                       _ptr(dp1), _ptr(dp2), _ptr(dv), _ptr(dalpha),
+                                       float(tau_s), shape_of(p1), _dtype_code(p1),
+                                       KERNELS[kernel], _ptr(workspace),
+                                       workspace.numel() * workspace.element_size(),
+                                       _ptr(dev_status), ctypes.c_void_p(_stream(stream)))
     if rc != OK:
-        raise RelationError(rc, "relation_linear_bwd")
+        raise RelationError(rc, "relation_linear_bwd_ex")
     return dp1, dp2, dv, dalpha
 
 

@@ -135,6 +135,12 @@ cudaError_t launch_linear_fwd(const LinearProblem& p, cudaStream_t s);
 bool linear_tc_supports(const LinearProblem& p);
 size_t linear_tc_workspace_bytes(const LinearProblem& p);
 cudaError_t launch_linear_tc_fwd(const LinearProblem& p, void* workspace, cudaStream_t s);
+// Chunked tensor-core backward (relation_linear_tc_bwd.cu): bf16, d_h 64, element strides
+// multiples of 8; p.workspace holds linear_tc_bwd_workspace_bytes(p) bytes (the forward's
+// block states and the state's adjoints, bf16).
+bool linear_tc_bwd_supports(const LinearProblem& p);
+size_t linear_tc_bwd_workspace_bytes(const LinearProblem& p);
+cudaError_t launch_linear_tc_bwd(const LinearProblem& p, cudaStream_t s);
 size_t linear_bwd_workspace_bytes(int B, int H, int T, int d);
 cudaError_t launch_linear_bwd(const LinearProblem& p, cudaStream_t s);
 

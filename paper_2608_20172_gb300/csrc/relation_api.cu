@@ -201,10 +201,57 @@ relation_status relation_linear_fwd_ws(const void* p1, const void* p2, const voi
   return from_cuda(rel::launch_linear_tc_fwd(p, workspace, reinterpret_cast<cudaStream_t>(stream)));
 }
 
+namespace {
+
+// The kernel family a backward request runs on (SIMT or TCGEN05), or -1 when the request
+// is not served: the arguments' shapes and dtypes only, no pointers.
+int linear_bwd_family(const relation_shape& shp, relation_dtype dt, relation_kernel kernel,
+                      relation_status* why) {
+  *why = RELATION_OK;
+  if (kernel != RELATION_KERNEL_AUTO && kernel != RELATION_KERNEL_SIMT &&
+      kernel != RELATION_KERNEL_TCGEN05) { *why = RELATION_ERR_INVALID_ARG; return -1; }
+  if (dt != RELATION_F32 && dt != RELATION_BF16) { *why = RELATION_ERR_INVALID_ARG; return -1; }
+  if (shp.B < 1 || shp.T < 1 || shp.H < 1 || shp.d_h < 1) { *why = RELATION_ERR_INVALID_ARG; return -1; }
+  if (shp.sB < 1 || shp.sT < 1 || shp.sH < 1) { *why = RELATION_ERR_INVALID_ARG; return -1; }
+  if (!rel::linear_supports(dt, shp.d_h)) { *why = RELATION_ERR_UNSUPPORTED; return -1; }
+  // grid: up to 8 column splits per head
+  if ((long long)shp.B * shp.H * 8 > 0x7fffffffLL) { *why = RELATION_ERR_UNSUPPORTED; return -1; }
+  // 4-element vector loads of every token row (alpha is fp32 with the same strides)
+  if (shp.sB % 4 || shp.sT % 4 || shp.sH % 4) { *why = RELATION_ERR_ALIGNMENT; return -1; }
+  rel::LinearProblem p{};
+  p.B = shp.B; p.T = shp.T; p.H = shp.H; p.d = shp.d_h;
+  p.sB = shp.sB; p.sT = shp.sT; p.sH = shp.sH; p.dtype = dt;
+  const bool tc = rel::linear_tc_bwd_supports(p) &&
+                  (long long)shp.B * shp.H * ((shp.T + 127) / 128) <= 0x7fffffffLL;
+  if (kernel == RELATION_KERNEL_TCGEN05 && !tc) {
+    *why = (dt == RELATION_BF16 && shp.d_h == 64 && (shp.sB % 8 || shp.sT % 8 || shp.sH % 8))
+               ? RELATION_ERR_ALIGNMENT : RELATION_ERR_UNSUPPORTED;
+    return -1;
+  }
+  return (tc && kernel != RELATION_KERNEL_SIMT) ? (int)RELATION_KERNEL_TCGEN05
+                                                : (int)RELATION_KERNEL_SIMT;
+}
+
+size_t linear_bwd_bytes(const relation_shape& shp, relation_dtype dt, int family) {
+  if (family == (int)RELATION_KERNEL_SIMT)
+    return rel::linear_bwd_workspace_bytes(shp.B, shp.H, shp.T, shp.d_h);
+  rel::LinearProblem p{};
+  p.B = shp.B; p.T = shp.T; p.H = shp.H; p.d = shp.d_h;
+  p.sB = shp.sB; p.sT = shp.sT; p.sH = shp.sH; p.dtype = dt;
+  return rel::linear_tc_bwd_workspace_bytes(p);
+}
+
+}  // namespace
+
+size_t relation_linear_bwd_ex_workspace_size(relation_shape shp, relation_dtype dt,
+                                             relation_kernel kernel) {
+  relation_status why;
+  const int fam = linear_bwd_family(shp, dt, kernel, &why);
+  return fam < 0 ? 0 : linear_bwd_bytes(shp, dt, fam);
+}
+
 size_t relation_linear_bwd_workspace_size(relation_shape shp, relation_dtype dt) {
-  if (dt != RELATION_F32 && dt != RELATION_BF16) return 0;
-  if (shp.B < 1 || shp.T < 1 || shp.H < 1 || !rel::linear_supports(dt, shp.d_h)) return 0;
-  return rel::linear_bwd_workspace_bytes(shp.B, shp.H, shp.T, shp.d_h);
+  return relation_linear_bwd_ex_workspace_size(shp, dt, RELATION_KERNEL_AUTO);
 }
 
 relation_status relation_linear_bwd(const void* p1, const void* p2, const void* v,
@@ -212,28 +259,34 @@ relation_status relation_linear_bwd(const void* p1, const void* p2, const void* 
                                    void* dv, float* dalpha, float tau_s, relation_shape shp,
                                    relation_dtype dt, void* workspace, size_t ws_bytes,
                                    int* dev_status, relation_stream_t stream) {
+  return relation_linear_bwd_ex(p1, p2, v, alpha, dy, dp1, dp2, dv, dalpha, tau_s, shp, dt,
+                                RELATION_KERNEL_AUTO, workspace, ws_bytes, dev_status, stream);
+}
+
+relation_status relation_linear_bwd_ex(const void* p1, const void* p2, const void* v,
+                                      const float* alpha, const void* dy, void* dp1, void* dp2,
+                                      void* dv, float* dalpha, float tau_s, relation_shape shp,
+                                      relation_dtype dt, relation_kernel kernel, void* workspace,
+                                      size_t ws_bytes, int* dev_status,
+                                      relation_stream_t stream) {
   relation_status st;
-  if (dt != RELATION_F32 && dt != RELATION_BF16) return RELATION_ERR_INVALID_ARG;
-  if (shp.B < 1 || shp.T < 1 || shp.H < 1 || shp.d_h < 1) return RELATION_ERR_INVALID_ARG;
-  if (shp.sB < 1 || shp.sT < 1 || shp.sH < 1) return RELATION_ERR_INVALID_ARG;
-  if (!rel::linear_supports(dt, shp.d_h)) return RELATION_ERR_UNSUPPORTED;
-  // grid: up to 8 column splits per head
-  if ((long long)shp.B * shp.H * 8 > 0x7fffffffLL) return RELATION_ERR_UNSUPPORTED;
-  // 4-element vector loads of every token row (alpha is fp32 with the same strides)
-  if (shp.sB % 4 || shp.sT % 4 || shp.sH % 4) return RELATION_ERR_ALIGNMENT;
+  const int fam = linear_bwd_family(shp, dt, kernel, &st);
+  if (fam < 0) return st;
   if (!isfinite(tau_s) || !(tau_s > 0.0f)) return RELATION_ERR_INVALID_ARG;
   if ((st = check_ptrs({p1, p2, v, alpha, dy, dp1, dp2, dv, dalpha, workspace})) != RELATION_OK)
     return st;
   if (dev_status && (reinterpret_cast<uintptr_t>(dev_status) & 3u)) return RELATION_ERR_ALIGNMENT;
-  if (ws_bytes < rel::linear_bwd_workspace_bytes(shp.B, shp.H, shp.T, shp.d_h))
-    return RELATION_ERR_WORKSPACE;
+  if (ws_bytes < linear_bwd_bytes(shp, dt, fam)) return RELATION_ERR_WORKSPACE;
+  if (!aligned16(workspace)) return RELATION_ERR_ALIGNMENT;
   rel::LinearProblem p{};
   p.p1 = p1; p.p2 = p2; p.v = v; p.alpha = alpha; p.dy = dy;
   p.dp1 = dp1; p.dp2 = dp2; p.dv = dv; p.dalpha = dalpha; p.workspace = workspace;
   p.dev_status = dev_status; p.tau_s = tau_s;
   p.B = shp.B; p.T = shp.T; p.H = shp.H; p.d = shp.d_h;
   p.sB = shp.sB; p.sT = shp.sT; p.sH = shp.sH; p.dtype = dt;
-  return from_cuda(rel::launch_linear_bwd(p, reinterpret_cast<cudaStream_t>(stream)));
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  if (fam == (int)RELATION_KERNEL_TCGEN05) return from_cuda(rel::launch_linear_tc_bwd(p, s));
+  return from_cuda(rel::launch_linear_bwd(p, s));
 }
 
 namespace {

@@ -26,23 +26,10 @@
 #include <cudaTypedefs.h>
 #include <math.h>
 
-#include "common.cuh"
-#include "kernels.h"
+#include "relation_linear_tc.cuh"
 
 namespace rel {
-namespace tc {
-bool make_tmap_bf16(CUtensorMap* m, const void* base, const Problem& p, int rows);
-}
-
 namespace lintc {
-
-constexpr int LT = 128;          // tokens per block
-constexpr int NC = 64;           // information columns per CTA
-constexpr int kThreads = 192;    // warps 0-3 elementwise, 4 TMA, 5 MMA
-constexpr int kTmemCols = 256;   // S 128 | E 64 | C 64
-constexpr int COL_S = 0, COL_E = 128, COL_C = 192;
-constexpr float kClampLog2 = 120.0f;
-
 template <int D>
 struct Cfg {
   static constexpr int KB = D / 64;          // 64-channel (128-byte) blocks of a p tile
@@ -69,55 +56,6 @@ struct Cfg {
 };
 static_assert(Cfg<64>::SMEM <= 232448 && Cfg<128>::SMEM <= 232448, "shared memory");
 
-// Modes of the kernel: SEQ walks all blocks of a (head, split) in order with the state in
-// TMEM; the chunk-parallel pair takes one block per CTA: DELTA writes the block's state
-// contribution sum_j KL_j I~_j^T and decay a_L (fp32) to the workspace, OUT reads the
-// state the block starts from (bf16, produced by scan_kernel) and writes the block's Y.
-enum : int { MODE_SEQ = 0, MODE_DELTA = 1, MODE_OUT = 2 };
-
-// Workspace of the chunk-parallel forward, per (head, split, block): dC [D][64] fp32, the
-// decay g [D] fp32, and the entering state C0 [D][64] bf16.
-struct LinCp {
-  float* dC;
-  float* g;
-  __nv_bfloat16* c0;
-  int nb;
-};
-
-// B_LOAD, B_FREE, B_EPI: one per input stage (stage s at + s)
-enum : int { B_LOAD = 0, B_FREE = 2, B_EPI = 4, B_OPS = 6, B_C0, B_S, B_A, B_E, B_STATE, NBAR };
-
-__device__ __forceinline__ void drain_wait(uint32_t bar, uint32_t parity) {
-  const unsigned long long t0 = globaltimer_ns();
-  while (!mbar_try_wait(bar, parity)) {
-    if (globaltimer_ns() - t0 > 20ull * 1000ull * 1000ull) return;
-  }
-}
-// 2-D tiled load into shared memory, completing on `bar` (transaction bytes).
-__device__ __forceinline__ void tma_load_2d(uint32_t dst, const CUtensorMap* m, uint32_t bar,
-                                            int c0, int c1) {
-  asm volatile(
-      "cp.async.bulk.tensor.2d.shared::cluster.global.mbarrier::complete_tx::bytes"
-      " [%0], [%1, {%3, %4}], [%2];" ::"r"(dst),
-      "l"(reinterpret_cast<uint64_t>(m)), "r"(bar), "r"(c0), "r"(c1)
-      : "memory");
-}
-__device__ __forceinline__ void ew_sync() {  // the 128 elementwise threads
-  asm volatile("bar.sync 1, 128;" ::: "memory");
-}
-// byte offset of element (row r, column c) in a tile of 128-byte-swizzled rows of 64
-// bf16 columns, blocks of `rows` rows per 64 columns
-__device__ __forceinline__ uint32_t swz(int r, int c, int rows) {
-  return (uint32_t)((c >> 6) * rows * 128 + r * 128 + ((((c & 63) >> 3) ^ (r & 7)) << 4) +
-                    (c & 7) * 2);
-}
-__device__ __forceinline__ float ld_bf(const uint8_t* base, uint32_t off) {
-  return __bfloat162float(*reinterpret_cast<const __nv_bfloat16*>(base + off));
-}
-__device__ __forceinline__ void st_bf(uint8_t* base, uint32_t off, float x) {
-  *reinterpret_cast<__nv_bfloat16*>(base + off) = __float2bfloat16_rn(x);
-}
-
 template <int D, int MODE>
 __global__ void __launch_bounds__(kThreads, 1)
     lin_tc_fwd_kernel(const __grid_constant__ CUtensorMap tmP1,
@@ -127,6 +65,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                       const __grid_constant__ CUtensorMap tmY,
                       const __grid_constant__ CUtensorMap tmC0, LinearProblem p, LinCp cp) {
   using C = Cfg<D>;
+  constexpr bool kDelta = MODE == MODE_DELTA || MODE == MODE_BDELTA;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>(
       (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
@@ -194,7 +133,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         const uint32_t lb = bar(B_LOAD + st);
         mbar_arrive_expect_tx(lb, C::LOAD_BYTES + (MODE == MODE_OUT ? C::C0T : 0));
         if (MODE == MODE_OUT)  // the state the block starts from, in the MN-major B layout
-          tma_load_2d(sb + C::OFF_C0, &tmC0, lb, 0, (bhs * nb + blk) * D);
+          tma_load_2d(sb + C::OFF_C0, &tmC0, lb, 0, (bhs * (nb + 1) + blk) * D);
         for (int kb = 0; kb < C::KB; ++kb) {
           tma_load_4d(sg + C::OFF_P1 + kb * LT * 128, &tmP1, lb, kb * 64, t0, h, b);
           tma_load_4d(sg + C::OFF_P2 + kb * LT * 128, &tmP2, lb, kb * 64, t0, h, b);
@@ -221,7 +160,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       const uint32_t sg = sb + st * C::STAGE;
       if (!(ok = mbar_wait_warp(bar(B_OPS), ph, ab))) break;
       tc_fence_after();
-      if (MODE != MODE_DELTA) {
+      if (!kDelta) {
 #pragma unroll
         for (int kk = 0; kk < D / 16; ++kk) {  // S = Qm Km^T
           const uint32_t koff = (kk >> 2) * (LT * 128) + (kk & 3) * 32;
@@ -247,7 +186,8 @@ __global__ void __launch_bounds__(kThreads, 1)
         mma_commit_w(bar(B_E));
       }
       if (MODE != MODE_OUT) {
-        // SEQ: C += KL^T I~ (C decayed by the threads); DELTA: the block's own sum
+        // SEQ: C += KL^T I~ (C decayed by the threads); DELTA: the block's own sum;
+        // BDELTA: Qs^T dY
 #pragma unroll
         for (int kk = 0; kk < LT / 16; ++kk)
           mma_ss_w(tmem + COL_C, smem_desc_sw128(sb + C::OFF_KL + kk * 16 * 128, LT * 128, 1024),
@@ -393,21 +333,24 @@ __global__ void __launch_bounds__(kThreads, 1)
                 my_clamp = true;
               }
               const float xv = u ? x.y : x.x, yv = u ? y.y : y.x;
-              if (MODE != MODE_DELTA) {
+              if (!kDelta) {
                 r[u][0] = xv * s1 * ex2_approx(dm);      // Qm
                 r[u][1] = yv * s2 * ex2_approx(-dm);     // Km
                 r[u][2] = xv * s1 * ex2_approx(L);       // Qs (factor <= 1)
               }
-              if (MODE != MODE_OUT) r[u][3] = yv * s2 * ex2_approx(Ev[ch] - L);  // KL (<= 1)
+              if (MODE == MODE_BDELTA)
+                r[u][3] = xv * s1 * ex2_approx(L);         // Qs, in KL's place
+              else if (MODE != MODE_OUT)
+                r[u][3] = yv * s2 * ex2_approx(Ev[ch] - L);  // KL (factor <= 1)
             }
-            if (MODE != MODE_DELTA) {
+            if (!kDelta) {
               qm[e] = pack_bf16x2(r[0][0], r[1][0]);
               km[e] = pack_bf16x2(r[0][1], r[1][1]);
               qs[e] = pack_bf16x2(r[0][2], r[1][2]);
             }
             if (MODE != MODE_OUT) kl[e] = pack_bf16x2(r[0][3], r[1][3]);
           }
-          if (MODE != MODE_DELTA) {
+          if (!kDelta) {
             *reinterpret_cast<uint4*>(p1s + off) = make_uint4(qm[0], qm[1], qm[2], qm[3]);
             *reinterpret_cast<uint4*>(p2s + off) = make_uint4(km[0], km[1], km[2], km[3]);
             *reinterpret_cast<uint4*>(smem + C::OFF_QS + off) =
@@ -421,8 +364,8 @@ __global__ void __launch_bounds__(kThreads, 1)
       fence_async_smem();
       ew_sync();
       mbar_arrive(bar(B_OPS));
-      if (MODE == MODE_DELTA) {
-        // the block's state contribution and decay, to the workspace
+      if (kDelta) {
+        // the block's state (adjoint) contribution and decay, to the workspace
         ok = __all_sync(0xffffffffu, mbar_wait(bar(B_STATE), 0, ab));
         if (!ok) break;
         tc_fence_after();
@@ -550,34 +493,16 @@ __global__ void __launch_bounds__(kThreads, 1)
   }
 }
 
-// 4-D map over the [B][T][H][d] fp32 retention: boxes of 32 channels x 128 tokens, no swizzle.
-static bool make_tmap_alpha(CUtensorMap* m, const LinearProblem& p) {
-  static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
-  if (!fn) {
-    void* ptr = nullptr;
-    cudaDriverEntryPointQueryResult q;
-    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &ptr, 12000, cudaEnableDefault,
-                                         &q) != cudaSuccess ||
-        q != cudaDriverEntryPointSuccess)
-      return false;
-    fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(ptr);
-  }
-  cuuint64_t dims[4] = {(cuuint64_t)p.d, (cuuint64_t)p.T, (cuuint64_t)p.H, (cuuint64_t)p.B};
-  cuuint64_t strides[3] = {(cuuint64_t)p.sT * 4, (cuuint64_t)p.sH * 4, (cuuint64_t)p.sB * 4};
-  cuuint32_t box[4] = {32, (cuuint32_t)LT, 1, 1};
-  cuuint32_t estr[4] = {1, 1, 1, 1};
-  return fn(m, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 4, const_cast<float*>(p.alpha), dims, strides, box,
-            estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_NONE,
-            CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
-}
-
 // Sequential scan of the state over the blocks of one (head, split), for the chunk-parallel
 // forward: C_0(0) = 0, C_0(b + 1) = Diag(g_b) C_0(b) + dC_b, each C_0(b) written in bf16
 // (row-major [D][64] per block, the OUT pass's B operand after a swizzled TMA load).  A CTA
 // takes 8 channels x 64 columns, two per thread (a warp = one channel's 64 columns,
 // coalesced); the loads of the next 8 blocks are in flight while 8 are combined.
-template <int D>
-__global__ void __launch_bounds__(256) scan_kernel(LinCp cp) {
+//   REV (the backward): from the last block down, the state's adjoint leaving block b,
+//   dC(nb - 1) = 0, dC(b - 1) = Diag(g_b) dC(b) + dQ_b (dQ_b = Qs_b^T dY_b in dC's place),
+//   written to out_rows (bf16 [nb][D][64] per (head, split)).  Forward: nb + 1 states.
+template <int D, bool REV>
+__global__ void __launch_bounds__(256) scan_kernel(LinCp cp, __nv_bfloat16* out_rows) {
   constexpr int CPB = 8, P = 8;
   const int cg = (int)(blockIdx.x % (D / CPB));
   const int bhs = (int)(blockIdx.x / (D / CPB));
@@ -585,11 +510,13 @@ __global__ void __launch_bounds__(256) scan_kernel(LinCp cp) {
   const int n = (int)(threadIdx.x & 31) * 2;
   const int nb = cp.nb;
   const long long base = (long long)bhs * nb * D + c;  // row of block blk: base + blk D
+  // output rows: forward nb + 1 states per (head, split), backward nb adjoints
+  const long long obase = (long long)bhs * (REV ? nb : nb + 1) * D + c;
   auto load = [&](int b0, float2 (&dv)[P], float (&gv)[P]) {
 #pragma unroll
     for (int u = 0; u < P; ++u) {
-      const int blk = b0 + u;
-      if (blk < nb) {
+      const int blk = REV ? nb - 1 - (b0 + u) : b0 + u;
+      if (blk >= 0 && blk < nb) {
         const long long row = base + (long long)blk * D;
         dv[u] = *reinterpret_cast<const float2*>(cp.dC + row * 64 + n);
         gv[u] = cp.g[row];
@@ -608,10 +535,12 @@ __global__ void __launch_bounds__(256) scan_kernel(LinCp cp) {
     load(b0 + P, nxt, gn);
 #pragma unroll
     for (int u = 0; u < P; ++u) {
-      const int blk = b0 + u;
-      if (blk < nb) {
-        const long long row = base + (long long)blk * D;
-        *reinterpret_cast<__nv_bfloat162*>(cp.c0 + row * 64 + n) = __floats2bfloat162_rn(st.x, st.y);
+      const int i = b0 + u;
+      if (i < nb) {
+        const int blk = REV ? nb - 1 - i : i;
+        const long long orow = obase + (long long)blk * D;
+        *reinterpret_cast<__nv_bfloat162*>(out_rows + orow * 64 + n) =
+            __floats2bfloat162_rn(st.x, st.y);
         st = make_float2(fmaf(gc[u], st.x, cur[u].x), fmaf(gc[u], st.y, cur[u].y));
       }
     }
@@ -621,36 +550,17 @@ __global__ void __launch_bounds__(256) scan_kernel(LinCp cp) {
       gc[u] = gn[u];
     }
   }
+  if (!REV)  // the final state, after the last block
+    *reinterpret_cast<__nv_bfloat162*>(out_rows + (obase + (long long)nb * D) * 64 + n) =
+        __floats2bfloat162_rn(st.x, st.y);
 }
 
-// 2-D map over the bf16 C0 rows of the workspace: [rows][64], boxes of D rows, 128-byte
-// swizzle (the MN-major B layout of the E = Qs C_0 product).
-static bool make_tmap_c0(CUtensorMap* m, void* base, long long rows, int d) {
-  static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
-  if (!fn) {
-    void* ptr = nullptr;
-    cudaDriverEntryPointQueryResult q;
-    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &ptr, 12000, cudaEnableDefault,
-                                         &q) != cudaSuccess ||
-        q != cudaDriverEntryPointSuccess)
-      return false;
-    fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(ptr);
-  }
-  cuuint64_t dims[2] = {64, (cuuint64_t)rows};
-  cuuint64_t strides[1] = {128};
-  cuuint32_t box[2] = {64, (cuuint32_t)d};
-  cuuint32_t estr[2] = {1, 1};
-  return fn(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, base, dims, strides, box, estr,
-            CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
-            CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
-}
-
-static size_t align256(size_t x) { return (x + 255) & ~(size_t)255; }
-
-// Workspace layout of the chunk-parallel forward: dC, g, C0 (see LinCp).
-static size_t cp_bytes(long long rows, LinCp* out, void* base) {
+// Workspace layout of the chunk-parallel forward: dC and g per (head, split, block), C0 per
+// (head, split) and block plus the final state (see LinCp).
+static size_t cp_bytes(long long heads, long long nb, int d, LinCp* out, void* base) {
+  const long long rows = heads * nb * d, rows_c0 = heads * (nb + 1) * d;
   const size_t b_dc = align256((size_t)rows * 64 * 4), b_g = align256((size_t)rows * 4);
-  const size_t b_c0 = align256((size_t)rows * 64 * 2);
+  const size_t b_c0 = align256((size_t)rows_c0 * 64 * 2);
   if (out) {
     uint8_t* q = static_cast<uint8_t*>(base);
     out->dC = reinterpret_cast<float*>(q);
@@ -688,8 +598,8 @@ static cudaError_t fwd_t(const LinearProblem& lp, void* workspace, cudaStream_t 
   }
   mc = m1;  // unused by the sequential mode
   if (cp_path) {
-    cp_bytes(heads * nb * D, &cp, workspace);
-    if (!make_tmap_c0(&mc, cp.c0, heads * nb * D, D)) {
+    cp_bytes(heads, nb, D, &cp, workspace);
+    if (!make_tmap_c0(&mc, cp.c0, heads * (nb + 1) * D, D)) {
       note_failure("linear chunked forward: TMA descriptor of the workspace");
       return cudaErrorInvalidValue;
     }
@@ -704,7 +614,7 @@ static cudaError_t fwd_t(const LinearProblem& lp, void* workspace, cudaStream_t 
     lin_tc_fwd_kernel<D, MODE_DELTA><<<(unsigned)grid, kThreads, smem, s>>>(m1, m2, mv, ma, my, mc,
                                                                            lp, cp);
     if ((e = cudaGetLastError()) != cudaSuccess) { note_failure("linear chunked forward: launch"); return e; }
-    scan_kernel<D><<<(unsigned)(heads * (D / 8)), 256, 0, s>>>(cp);
+    scan_kernel<D, false><<<(unsigned)(heads * (D / 8)), 256, 0, s>>>(cp, cp.c0);
     if ((e = cudaGetLastError()) != cudaSuccess) { note_failure("linear chunked forward: launch"); return e; }
     lin_tc_fwd_kernel<D, MODE_OUT><<<(unsigned)grid, kThreads, smem, s>>>(m1, m2, mv, ma, my, mc,
                                                                          lp, cp);
@@ -712,6 +622,60 @@ static cudaError_t fwd_t(const LinearProblem& lp, void* workspace, cudaStream_t 
   if ((e = cudaGetLastError()) != cudaSuccess) note_failure("linear chunked forward: launch");
   return e;
 }
+
+// The state passes the chunked backward needs (relation_linear_tc_bwd.cu), in the
+// workspace laid out by bwd_bytes: the forward's states entering every block and the final
+// one (cp.c0), then the state's adjoint leaving every block (dcb, bf16 [heads][nb][D][64]).
+// Four launches: forward DELTA, forward scan, BDELTA (Qs^T dY per block), reverse scan.
+size_t bwd_bytes(long long heads, long long nb, int d, LinCp* cp, __nv_bfloat16** dcb,
+                 void* base) {
+  const size_t f = cp_bytes(heads, nb, d, cp, base);
+  if (dcb) *dcb = reinterpret_cast<__nv_bfloat16*>(static_cast<uint8_t*>(base) + f);
+  return f + align256((size_t)(heads * nb * d) * 64 * 2);
+}
+
+template <int D>
+cudaError_t states_t(const LinearProblem& lp, const void* dy, void* workspace, cudaStream_t s) {
+  const int smem = Cfg<D>::SMEM;
+  cudaError_t e;
+  for (auto fn : {lin_tc_fwd_kernel<D, MODE_DELTA>, lin_tc_fwd_kernel<D, MODE_BDELTA>})
+    if ((e = cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, smem)) !=
+        cudaSuccess) {
+      note_failure("linear chunked backward: shared memory attribute");
+      return e;
+    }
+  Problem p{};
+  p.B = lp.B; p.T = lp.T; p.H = lp.H; p.d = lp.d;
+  p.sB = lp.sB; p.sT = lp.sT; p.sH = lp.sH;
+  const int nb = (lp.T + LT - 1) / LT;
+  const long long heads = (long long)lp.B * lp.H * (D / NC);
+  LinCp cp{};
+  cp.nb = nb;
+  __nv_bfloat16* dcb = nullptr;
+  bwd_bytes(heads, nb, D, &cp, &dcb, workspace);
+  CUtensorMap m1, m2, mv, mg, ma;
+  if (!tc::make_tmap_bf16(&m1, lp.p1, p, LT) || !tc::make_tmap_bf16(&m2, lp.p2, p, LT) ||
+      !tc::make_tmap_bf16(&mv, lp.v, p, LT) || !tc::make_tmap_bf16(&mg, dy, p, LT) ||
+      !make_tmap_alpha(&ma, lp)) {
+    note_failure("linear chunked backward: TMA descriptors");
+    return cudaErrorInvalidValue;
+  }
+  const long long grid = heads * nb;
+  if (grid > 0x7fffffffLL) return cudaErrorInvalidConfiguration;
+  // (the Y map is unused in these modes; m1 stands in)
+  lin_tc_fwd_kernel<D, MODE_DELTA><<<(unsigned)grid, kThreads, smem, s>>>(m1, m2, mv, ma, m1, m1,
+                                                                         lp, cp);
+  if ((e = cudaGetLastError()) != cudaSuccess) { note_failure("linear chunked backward: launch"); return e; }
+  scan_kernel<D, false><<<(unsigned)(heads * (D / 8)), 256, 0, s>>>(cp, cp.c0);
+  if ((e = cudaGetLastError()) != cudaSuccess) { note_failure("linear chunked backward: launch"); return e; }
+  lin_tc_fwd_kernel<D, MODE_BDELTA><<<(unsigned)grid, kThreads, smem, s>>>(m1, m2, mg, ma, m1, m1,
+                                                                          lp, cp);
+  if ((e = cudaGetLastError()) != cudaSuccess) { note_failure("linear chunked backward: launch"); return e; }
+  scan_kernel<D, true><<<(unsigned)(heads * (D / 8)), 256, 0, s>>>(cp, dcb);
+  if ((e = cudaGetLastError()) != cudaSuccess) note_failure("linear chunked backward: launch");
+  return e;
+}
+template cudaError_t states_t<64>(const LinearProblem&, const void*, void*, cudaStream_t);
 
 }  // namespace lintc
 
@@ -724,7 +688,7 @@ size_t linear_tc_workspace_bytes(const LinearProblem& p) {
   if (!linear_tc_supports(p)) return 0;
   const long long heads = (long long)p.B * p.H * (p.d / lintc::NC);
   const long long nb = (p.T + lintc::LT - 1) / lintc::LT;
-  return lintc::cp_bytes(heads * nb * p.d, nullptr, nullptr);
+  return lintc::cp_bytes(heads, nb, p.d, nullptr, nullptr);
 }
 
 cudaError_t launch_linear_tc_fwd(const LinearProblem& p, void* workspace, cudaStream_t s) {

@@ -248,14 +248,15 @@ def test_linear_fwd_ex_family_rules(lib, case, expect):
 
 
 def test_linear_fwd_ws_workspace_rules(lib):
-    """The chunk-parallel forward's workspace: B H (d/64) ceil(T/128) d rows of 64 fp32 dC,
-    one fp32 decay and 64 bf16 of entering state, each array padded to 256 bytes; fp32 and
+    """The chunk-parallel forward's workspace: B H (d/64) ceil(T/128) d rows of 64 fp32 dC and
+    one fp32 decay, B H (d/64) (ceil(T/128) + 1) d rows of 64 bf16 states, each array padded
+    to 256 bytes; fp32 and
     other widths need none; a short or misaligned workspace is refused before any launch."""
     shape = _shape(B=1, T=300, H=2, d=64)
-    rows = 1 * 2 * 1 * 3 * 64
+    rows, rows_c0 = 1 * 2 * 1 * 3 * 64, 1 * 2 * 1 * 4 * 64  # C0: every block's and the final
     pad = lambda x: (x + 255) // 256 * 256
     need = lib.relation_linear_fwd_workspace_size(shape, binding.BF16)
-    assert need == pad(rows * 64 * 4) + pad(rows * 4) + pad(rows * 64 * 2)
+    assert need == pad(rows * 64 * 4) + pad(rows * 4) + pad(rows_c0 * 64 * 2)
     assert lib.relation_linear_fwd_workspace_size(shape, binding.F32) == 0
     assert lib.relation_linear_fwd_workspace_size(_shape(d=32), binding.BF16) == 0
     p = [ctypes.c_void_p(0x10000 * (i + 1)) for i in range(5)]
@@ -269,14 +270,45 @@ def test_linear_fwd_ws_workspace_rules(lib):
 
 def test_linear_bwd_workspace_rules(lib):
     shape = _shape(B=2, T=20, H=3, d=64)
-    need = lib.relation_linear_bwd_workspace_size(shape, binding.BF16)
+    simt = lib.relation_linear_bwd_ex_workspace_size(shape, binding.BF16, binding.KERNELS["simt"])
     # checkpoints every 8 tokens (3 of 64 x 64) plus the column splits' partial row sums
-    assert need == (2 * 3 * 3 * 64 * 64 + 2 * 3 * 2 * 20 * 3 * 64) * 4
+    assert simt == (2 * 3 * 3 * 64 * 64 + 2 * 3 * 2 * 20 * 3 * 64) * 4
+    # the chunked family, one 128-token block per head (6 heads): fp32 rows of 64 and the
+    # decays, the states entering the block and the final one, the adjoints (bf16)
+    tc = lib.relation_linear_bwd_ex_workspace_size(shape, binding.BF16, binding.KERNELS["tcgen05"])
+    assert tc == 6 * 64 * 64 * 4 + 6 * 64 * 4 + 6 * 2 * 64 * 64 * 2 + 6 * 64 * 64 * 2
+    need = lib.relation_linear_bwd_workspace_size(shape, binding.BF16)
+    assert need == tc  # AUTO takes the chunked kernel for bf16 at d_h = 64
+    assert lib.relation_linear_bwd_ex_workspace_size(shape, binding.F32,
+                                                     binding.KERNELS["tcgen05"]) == 0
+    assert lib.relation_linear_bwd_workspace_size(shape, binding.F32) == simt
+    d128 = _shape(B=2, T=20, H=3, d=128)
+    assert lib.relation_linear_bwd_ex_workspace_size(d128, binding.BF16,
+                                                     binding.KERNELS["tcgen05"]) == 0
+    assert lib.relation_linear_bwd_workspace_size(d128, binding.BF16) == \
+        lib.relation_linear_bwd_ex_workspace_size(d128, binding.BF16, binding.KERNELS["simt"])
     assert lib.relation_linear_bwd_workspace_size(_shape(d=48), binding.BF16) == 0
     p = [ctypes.c_void_p(0x10000 * (i + 1)) for i in range(9)]
     rc = lib.relation_linear_bwd(*p, 2.0, shape, binding.BF16, ctypes.c_void_p(0x100000), need - 1,
                                  None, None)
     assert rc == binding.ERR_WORKSPACE
+    rc = lib.relation_linear_bwd_ex(*p, 2.0, shape, binding.BF16, binding.KERNELS["simt"],
+                                    ctypes.c_void_p(0x100000), simt - 1, None, None)
+    assert rc == binding.ERR_WORKSPACE
+    rc = lib.relation_linear_bwd_ex(*p, 2.0, shape, binding.BF16, binding.KERNELS["tcgen05"],
+                                    ctypes.c_void_p(0x100008), tc, None, None)
+    assert rc == binding.ERR_ALIGNMENT
+    rc = lib.relation_linear_bwd_ex(*p, 2.0, shape, binding.F32, binding.KERNELS["tcgen05"],
+                                    ctypes.c_void_p(0x100000), 1 << 30, None, None)
+    assert rc == binding.ERR_UNSUPPORTED
+    odd = _shape(B=2, T=20, H=3, d=64)
+    odd.sB, odd.sT, odd.sH = 20 * 3 * 68, 3 * 68, 68
+    rc = lib.relation_linear_bwd_ex(*p, 2.0, odd, binding.BF16, binding.KERNELS["tcgen05"],
+                                    ctypes.c_void_p(0x100000), 1 << 30, None, None)
+    assert rc == binding.ERR_ALIGNMENT
+    rc = lib.relation_linear_bwd_ex(*p, 2.0, shape, binding.BF16, 7, ctypes.c_void_p(0x100000),
+                                    1 << 30, None, None)
+    assert rc == binding.ERR_INVALID_ARG
 
 
 @pytest.mark.parametrize("case,expect", [

@@ -51,7 +51,8 @@ def test_linear_backward(dtype, d, T):
     p1, p2, v, alpha, dy = workloads.make_linear_inputs(w, seed=100 + T + d)
     dev = torch.device("cuda:0")
     status = torch.zeros(1, dtype=torch.int32, device=dev)
-    g = binding.linear_bwd(*(t.to(dev) for t in (p1, p2, v, alpha, dy)), dev_status=status)
+    g = binding.linear_bwd(*(t.to(dev) for t in (p1, p2, v, alpha, dy)), kernel="simt",
+                           dev_status=status)
     torch.cuda.synchronize()
     assert int(status.item()) == 0
     g = [t.float().cpu().numpy() for t in g]
@@ -177,3 +178,81 @@ def test_linear_forward_ws_many_heads_uses_the_sequential_walk():
     y_seq = binding.linear_fwd(*args, kernel="tcgen05")
     torch.cuda.synchronize()
     assert torch.equal(y, y_seq)
+
+
+# --- the chunked tensor-core backward -----------------------------------------
+
+def _check_grads(tag, g, p1, p2, v, alpha, dy, heads):
+    g = [t.float().cpu().numpy() for t in g]
+    for b, h in heads:
+        ref = oracle.linear_bwd(_heads(p1, b, h), _heads(p2, b, h), _heads(v, b, h),
+                                _heads(alpha, b, h), _heads(dy, b, h))
+        for name, got, r in zip(("dp1", "dp2", "dv", "dalpha"), g, ref):
+            pu.check_recorded(tag, name, got[b, :, h], r, "bf16", "grad")
+
+
+@pytest.mark.parametrize("T", [1, 2, 64, 127, 128, 129, 300, 513])
+def test_linear_backward_chunked_every_head(T):
+    """The chunked tcgen05 backward (the states entering and the adjoints leaving every
+    128-token block, then every block's gradients in parallel) against the fp64 reverse
+    mode of the recurrence on every head: whole blocks, ragged tails, a single token."""
+    w = workloads.custom(2, 3, T, 64, "bf16")
+    p1, p2, v, alpha, dy = workloads.make_linear_inputs(w, seed=700 + T)
+    dev = torch.device("cuda:0")
+    status = torch.zeros(1, dtype=torch.int32, device=dev)
+    g = binding.linear_bwd(*(t.to(dev) for t in (p1, p2, v, alpha, dy)), kernel="tcgen05",
+                           dev_status=status)
+    torch.cuda.synchronize()
+    assert int(status.item()) == 0
+    _check_grads("linear chunked bwd", g, p1, p2, v, alpha, dy,
+                 [(b, h) for b in range(w.B) for h in range(w.H)])
+
+
+def test_linear_backward_chunked_long_sequence():
+    """32 blocks of 128 tokens (the states and adjoints carried through all of them) on every
+    head, against the oracle and against the recurrent backward."""
+    w = workloads.custom(1, 2, 4096, 64, "bf16")
+    p1, p2, v, alpha, dy = workloads.make_linear_inputs(w, seed=91)
+    dev = torch.device("cuda:0")
+    args = [t.to(dev) for t in (p1, p2, v, alpha, dy)]
+    status = torch.zeros(1, dtype=torch.int32, device=dev)
+    g_tc = binding.linear_bwd(*args, kernel="tcgen05", dev_status=status)
+    g_rec = binding.linear_bwd(*args, kernel="simt", dev_status=status)
+    torch.cuda.synchronize()
+    assert int(status.item()) == 0
+    _check_grads("linear chunked bwd 4096", g_tc, p1, p2, v, alpha, dy, [(0, 0), (0, 1)])
+    for name, a, r in zip(("dp1", "dp2", "dv", "dalpha"), g_tc, g_rec):
+        pu.check(f"chunked vs recurrent {name}", a.float().cpu().numpy(),
+                 r.float().cpu().numpy(), "bf16", "grad")
+
+
+def test_linear_backward_auto_takes_the_chunked_kernel():
+    """AUTO serves bf16 at d_h = 64 with the chunked kernel: bit-identical results to
+    TCGEN05, in a workspace of the chunked family's size."""
+    w = workloads.custom(2, 4, 300, 64, "bf16")
+    p1, p2, v, alpha, dy = workloads.make_linear_inputs(w, seed=5)
+    dev = torch.device("cuda:0")
+    args = [t.to(dev) for t in (p1, p2, v, alpha, dy)]
+    assert binding.linear_bwd_workspace_size(args[0]) == \
+        binding.linear_bwd_workspace_size(args[0], "tcgen05") > 0
+    g_auto = binding.linear_bwd(*args)
+    g_tc = binding.linear_bwd(*args, kernel="tcgen05")
+    torch.cuda.synchronize()
+    for a, b in zip(g_auto, g_tc):
+        assert torch.equal(a, b)
+
+
+def test_linear_backward_chunked_reports_decay_beyond_its_range():
+    """Retention whose 64-token product falls below 2^-120: the chunked backward clamps like
+    the chunked forward, reports RELATION_ERR_UNSUPPORTED and keeps every output finite."""
+    w = workloads.custom(1, 2, 256, 64, "bf16")
+    p1, p2, v, alpha, dy = workloads.make_linear_inputs(w, seed=3)
+    alpha = torch.full_like(alpha, 1e-3)
+    dev = torch.device("cuda:0")
+    status = torch.zeros(1, dtype=torch.int32, device=dev)
+    g = binding.linear_bwd(*(t.to(dev) for t in (p1, p2, v, alpha, dy)), kernel="tcgen05",
+                           dev_status=status)
+    torch.cuda.synchronize()
+    assert int(status.item()) == binding.ERR_UNSUPPORTED
+    for t in g:
+        assert torch.isfinite(t.float()).all()
