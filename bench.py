@@ -360,6 +360,64 @@ def layer_measure(binding, dev, peaks, steps=10, warmup=3):
             "gpu_launches_per_call": {"prep": 1, "grad": 2}}
 
 
+# The paper's layer geometries (App. B model configurations: heads x width, context and
+# per-GPU micro-batch of the Relation runs): 10M 8 x 48 at T = 1024, 30M 8 x 64 at 2048,
+# 100M 8 x 80 at 4096.
+PAPER_LAYERS = {"10M": (32, 8, 1024, 48), "30M": (16, 8, 2048, 64), "100M": (4, 8, 4096, 80)}
+
+
+def paper_layers_measure(binding, dev, peaks, steps=10, warmup=3):
+    """One Relation layer's token mixing at each paper geometry, fwd + bwd through the
+    public API: the layer transforms (RoPE of P1, P2 and the Givens mixing of I), the
+    operator forward and backward, and the transforms' gradient, on synthetic bf16 inputs
+    (P1, P2, I, dY ~ N(0, 1), Givens angles ~ U(-1, 1), lambda = 0.5).  Operator work as
+    7 B H T^2 d_h (the real width; d_h = 48 and 80 run on zero-padded 64- and 128-wide
+    tiles)."""
+    out = {}
+    stream = torch.cuda.current_stream(dev)
+    lam, tau = workloads.LAMBDA_INIT, workloads.TAU_S
+    for name, (B, H, T, d) in PAPER_LAYERS.items():
+        g = torch.Generator(device="cpu").manual_seed(0)
+        p1, p2, info, dy = (torch.randn((B, T, H, d), generator=g).to(torch.bfloat16).to(dev)
+                            for _ in range(4))
+        theta = (torch.rand(H // 2, generator=g) * 2.0 - 1.0).float().to(dev)
+        qkv = tuple(torch.empty_like(p1) for _ in range(3))
+        y = torch.empty_like(p1)
+        logz = torch.empty((B, H, T), device=dev, dtype=torch.float32)
+        dq, dk, dv = torch.empty_like(p1), torch.empty_like(p1), torch.empty_like(p1)
+        dl = torch.empty(1, device=dev, dtype=torch.float32)
+        wsb = torch.empty(binding.workspace_size(p1), device=dev, dtype=torch.uint8)
+        wsg = torch.empty(max(binding.layer_grad_workspace_size(p1), 16), device=dev,
+                          dtype=torch.uint8)
+        status = torch.zeros(1, dtype=torch.int32, device=dev)
+        q, k, v = qkv
+        calls = {
+            "prep": lambda: binding.layer_prep(p1, p2, info, theta, 0, out=qkv, stream=stream),
+            "fwd": lambda: binding.fwd(q, k, v, lam, tau, out=y, logz=logz, dev_status=status,
+                                       stream=stream),
+            "bwd": lambda: binding.bwd(q, k, v, y, dy, logz, lam, tau, workspace=wsb, dq=dq,
+                                       dk=dk, dv=dv, dlambda=dl, dev_status=status,
+                                       stream=stream),
+            "grad": lambda: binding.layer_grad(dq, dk, dv, info, theta, 0, workspace=wsg,
+                                               stream=stream),
+        }
+        ms = {k2: _time_calls(c, dev, steps, warmup) for k2, c in calls.items()}
+        if int(status.item()) != 0:
+            raise SystemExit(f"paper layer {name}: device status "
+                             f"{binding.status_string(int(status.item()))}")
+        tot = sum(ms.values())
+        fl = 7.0 * B * H * T * T * d
+        out[name] = {"B": B, "H": H, "T": T, "d_h": d, "ms": ms, "ms_step": tot,
+                     "tokens_per_s": B * T / (tot * 1e-3),
+                     "operator_tflops": fl / ((ms["fwd"] + ms["bwd"]) * 1e-3) / 1e12,
+                     "operator_frac": fl / ((ms["fwd"] + ms["bwd"]) * 1e-3) / 1e12 /
+                     peaks["bf16_tflops"]}
+        del p1, p2, info, dy, qkv, y, dq, dk, dv, wsb, wsg
+    return {"layers": out, "dtype": "bf16", "data": "synthetic",
+            "note": "one layer's token mixing; the paper's Table of scale-matched runs reports "
+                    "whole-model training tok/s on another GPU (context only)"}
+
+
 def sdpa_context(w, dev, steps=20, warmup=3):
     """Context only, not this library: PyTorch's causal scaled-dot-product attention
     (softmax attention, the paper's comparison operator) forward + backward on the same
@@ -731,6 +789,7 @@ def run_ours(args, w):
         line["decode"] = decode_measure(binding, dev, peaks)
         line["linear"] = linear_measure(binding, dev, peaks)
         line["layer"] = layer_measure(binding, dev, peaks)
+        line["paper_layers"] = paper_layers_measure(binding, dev, peaks)
         try:
             line["context_sdpa"] = sdpa_context(w, dev)
         except Exception as exc:  # context only: never at the expense of the line
