@@ -257,6 +257,48 @@ relation_status relation_decode(const void* q, const void* k_cache, const void* 
                                 int* dev_status, relation_stream_t stream);
 
 /*
+ * Context parallelism (sequence sharding) of the forward.  The Exchange summary of a query
+ * row over a set of history keys is (m, l, z): l = sum_j exp(E_ij - m) and
+ * z = sum_j exp(E_ij - m) I~_j over those keys, for any log-scale m (here an upper bound of
+ * their max E); summaries over disjoint key sets merge associatively (App. A.3, the online
+ * update of the scan), and the epilogue of App. A.3.3-A.3.5 needs only the merged summary,
+ * the row's own q_i, k_i (Self) and v_i, and its position i.  A sequence split into shards
+ * of consecutive tokens is thus computed shard by shard:
+ *   relation_fwd_state(causal = 1) over the shard's own tokens, then for every earlier
+ *   shard relation_fwd_state(causal = 0) of the shard's queries against that shard's keys
+ *   and relation_state_merge into the first, then relation_state_finish with pos0 = the
+ *   shard's first position -- Y and logZ equal relation_fwd over the whole sequence up to
+ *   rounding.
+ * Summary layout (dense, fp32, caller-owned): m, l [B][H][T_q], z [B][H][T_q][d_h].
+ *
+ * relation_fwd_state: the summary of every row of q ([B][T_q][H][d_h], strides of shp_q)
+ *   over the keys of k, v ([B][T_k][H][d_h], strides of shp_kv; B, H, d_h as shp_q):
+ *   causal = 1: k, v are the queries' own tokens (T_k = T_q), row i takes keys j < i (Self
+ *   excluded; row 0's summary is empty: m = -inf, l = 0, z = 0); causal = 0: every one of
+ *   the T_k keys precedes every query.  bf16 with d_h a multiple of 8 up to 128 (the
+ *   tensor-core forward's tiles; otherwise RELATION_ERR_UNSUPPORTED).
+ * relation_state_merge: (m, l, z) <- merge of (m, l, z) and (m2, l2, z2), rows of
+ *   shp.B, shp.H, shp.T (strides ignored), d_h <= 128 a multiple of 4.
+ * relation_state_finish: Y (o, [B][T][H][d_h] with q's strides, dt) and logZ ([B][H][T]
+ *   fp32) of the rows of q, k, v from their summaries; row r sits at one-based position
+ *   pos0 + r + 1 of the sequence (the ln i of the count term); self_flow (optional) gets
+ *   F_ii.  bf16 or fp32, d_h <= 128 a multiple of 4.
+ * All three are asynchronous on `stream`; nothing is launched on an argument error.
+ */
+relation_status relation_fwd_state(const void* q, const void* k, const void* v, float* m,
+                                   float* l, float* z, relation_shape shp_q,
+                                   relation_shape shp_kv, int causal, relation_dtype dt,
+                                   int* dev_status, relation_stream_t stream);
+relation_status relation_state_merge(float* m, float* l, float* z, const float* m2,
+                                     const float* l2, const float* z2, relation_shape shp,
+                                     relation_stream_t stream);
+relation_status relation_state_finish(const void* q, const void* k, const void* v,
+                                      const float* m, const float* l, const float* z, void* o,
+                                      float* logz, float* self_flow, float lambda, float tau_s,
+                                      long long pos0, relation_shape shp, relation_dtype dt,
+                                      relation_stream_t stream);
+
+/*
  * The paper layer's transforms around the operator (Sec. 3.1-3.2, Eq. (givens-rotation),
  * App. A.2.2, App. B.3), producing the operator's inputs from the projected states:
  *   q = RoPE(p1), k = RoPE(p2): full-head rotary embedding, channel pairs (2c, 2c+1)

@@ -30,7 +30,8 @@ EXPORTED = ("relation_fwd", "relation_fwd_ex", "relation_bwd", "relation_bwd_ex"
             "relation_bwd_workspace_size", "relation_status_string", "relation_version",
             "relation_selftest_wait_timeout", "relation_launch_count", "relation_last_cuda_error",
             "relation_bwd_stages", "relation_bwd_static", "relation_fwd_flow",
-            "relation_decode", "relation_decode_workspace_size", "relation_linear_fwd",
+            "relation_decode", "relation_decode_workspace_size", "relation_fwd_state",
+            "relation_state_merge", "relation_state_finish", "relation_linear_fwd",
             "relation_linear_fwd_ex", "relation_linear_fwd_ws",
             "relation_linear_fwd_workspace_size",
             "relation_linear_bwd", "relation_linear_bwd_workspace_size",
@@ -81,6 +82,10 @@ def load(path: str | None = None):
         lib.relation_decode.argtypes = [vp, vp, vp, vp, vp, vp, f, f, Shape, ll, ll, i, vp,
                                         ctypes.c_size_t, ip, vp]
         lib.relation_decode_workspace_size.argtypes = [Shape, i]
+        lib.relation_fwd_state.argtypes = [vp, vp, vp, vp, vp, vp, Shape, Shape, i, i, ip, vp]
+        lib.relation_state_merge.argtypes = [vp, vp, vp, vp, vp, vp, Shape, vp]
+        lib.relation_state_finish.argtypes = [vp, vp, vp, vp, vp, vp, vp, vp, vp, f, f, ll, Shape,
+                                              i, vp]
         lib.relation_linear_fwd.argtypes = [vp, vp, vp, vp, vp, f, Shape, i, ip, vp]
         lib.relation_linear_fwd_ex.argtypes = [vp, vp, vp, vp, vp, f, Shape, i, i, ip, vp]
         lib.relation_linear_fwd_ws.argtypes = [vp, vp, vp, vp, vp, f, Shape, i, vp, sz, ip, vp]
@@ -229,6 +234,59 @@ def linear_fwd(p1, p2, v, alpha, tau_s: float = 2.0, *, kernel: str = "auto", ou
     if rc != OK:
         raise RelationError(rc, "relation_linear_fwd_ex")
     return out
+
+
+def fwd_state(q, k, v, causal: bool, *, out=None, dev_status=None, stream=None):
+    """Exchange summary of every row of q ([B, Tq, H, d]) over the keys of k, v ([B, Tk, H,
+    d]): causal = the queries' own tokens (keys before each row), else every key precedes
+    every query.  Returns (m, l, z): m, l [B, H, Tq] and z [B, H, Tq, d], fp32."""
+    _same_layout(k, v)
+    if causal:
+        _same_layout(q, k, v)
+    B, Tq, H, d = q.shape
+    if out is None:
+        out = (torch.empty((B, H, Tq), dtype=torch.float32, device=q.device),
+               torch.empty((B, H, Tq), dtype=torch.float32, device=q.device),
+               torch.empty((B, H, Tq, d), dtype=torch.float32, device=q.device))
+    m, l, z = out
+    rc = load().relation_fwd_state(_ptr(q), _ptr(k), _ptr(v), _ptr(m), _ptr(l), _ptr(z),
+                                   shape_of(q), shape_of(k), int(bool(causal)), _dtype_code(q),
+                                   _ptr(dev_status), ctypes.c_void_p(_stream(stream)))
+    if rc != OK:
+        raise RelationError(rc, "relation_fwd_state")
+    return m, l, z
+
+
+def state_merge(state, other, *, stream=None):
+    """Merge the summary ``other`` into ``state`` (both (m, l, z) as fwd_state returns them,
+    same rows) in place; returns ``state``."""
+    m, l, z = state
+    m2, l2, z2 = other
+    B, H, T, d = z.shape
+    rc = load().relation_state_merge(_ptr(m), _ptr(l), _ptr(z), _ptr(m2), _ptr(l2), _ptr(z2),
+                                     Shape(B, T, H, d, T * H * d, H * d, d),
+                                     ctypes.c_void_p(_stream(stream)))
+    if rc != OK:
+        raise RelationError(rc, "relation_state_merge")
+    return state
+
+
+def state_finish(q, k, v, state, lam: float, tau_s: float = 2.0, pos0: int = 0, *, out=None,
+                 logz=None, self_flow=None, stream=None):
+    """Y and logZ of the rows of q, k, v from their merged summary ``state``; row r is at
+    zero-based position pos0 + r of the sequence.  Returns (Y, logZ)."""
+    _same_layout(q, k, v)
+    m, l, z = state
+    B, T, H, d = q.shape
+    out = torch.empty_like(q) if out is None else out
+    logz = torch.empty((B, H, T), dtype=torch.float32, device=q.device) if logz is None else logz
+    rc = load().relation_state_finish(_ptr(q), _ptr(k), _ptr(v), _ptr(m), _ptr(l), _ptr(z),
+                                      _ptr(out), _ptr(logz), _ptr(self_flow), float(lam),
+                                      float(tau_s), int(pos0), shape_of(q), _dtype_code(q),
+                                      ctypes.c_void_p(_stream(stream)))
+    if rc != OK:
+        raise RelationError(rc, "relation_state_finish")
+    return out, logz
 
 
 def linear_fwd_workspace_size(p1) -> int:

@@ -34,6 +34,27 @@ struct Problem {
   relation_dtype dtype;
 };
 
+// The Exchange summary of a forward over part of the keys (context parallelism): per query
+// row the log-scale m (natural log), the sum l = sum_j exp(E_ij - m) and the unnormalised
+// z = sum_j exp(E_ij - m) v_j over the keys visited; Self is never part of it.
+struct StateArgs {
+  int causal;                    // 1: keys = the queries' own tokens (j < i); 0: all keys
+  int Tk;                        // keys (causal: = T)
+  long long k_sB, k_sT, k_sH;    // element strides of k and v (causal: the queries')
+  float* m;                      // [B][H][T]
+  float* l;                      // [B][H][T]
+  float* z;                      // [B][H][T][d] (d real columns)
+};
+
+// Context parallelism (relation_cp.cu): merge (m2, l2, z2) into (m, l, z) over `rows` rows
+// of d <= 128 columns; the epilogue of p's rows from their summaries, the first row at
+// zero-based position pos0 of the sequence (reads p.q, p.k, p.v; writes p.out, p.logz and,
+// if set, p.fself).
+cudaError_t launch_state_merge(float* m, float* l, float* z, const float* m2, const float* l2,
+                               const float* z2, long long rows, int d, cudaStream_t s);
+cudaError_t launch_state_finish(const Problem& p, const float* m, const float* l, const float* z,
+                                long long pos0, cudaStream_t s);
+
 // Backward workspace carved out of the caller's buffer (all fp32, 256-byte aligned).
 struct BwdWorkspace {
   float* dq_acc;     // [B][H][T_pad][d_pad] 2 sqrt(d) dL/dP1 in fp32, T_pad = T rounded up to
@@ -85,6 +106,10 @@ inline int head_groups(int n_t, int BH, int slots) {
 bool supports(relation_dtype dt, int d);      // forward
 bool supports_bwd(relation_dtype dt, int d);  // backward
 cudaError_t launch_fwd(const Problem& p, cudaStream_t s);
+// The forward's scan without its epilogue: the Exchange summary of every query row over
+// the keys of st (causal: the queries' own earlier tokens; else every key of k, v), written
+// to st.m, st.l, st.z (relation_tc_fwd.cu).
+cudaError_t launch_fwd_state(const Problem& p, const StateArgs& st, cudaStream_t s);
 // Backward stages (bit 1: row pass, 2: tile kernel, 4: finalisation).
 cudaError_t launch_bwd(const Problem& p, const BwdWorkspace& ws, unsigned stages, cudaStream_t s);
 int bwd_launches();  // launches made by launch_bwd with every stage

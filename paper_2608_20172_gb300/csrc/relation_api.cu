@@ -119,6 +119,62 @@ relation_status relation_fwd(const void* q, const void* k, const void* v, void* 
                          dev_status, stream);
 }
 
+relation_status relation_fwd_state(const void* q, const void* k, const void* v, float* m,
+                                   float* l, float* z, relation_shape shp_q,
+                                   relation_shape shp_kv, int causal, relation_dtype dt,
+                                   int* dev_status, relation_stream_t stream) {
+  relation_status st;
+  if ((st = check_shape(shp_q, dt)) != RELATION_OK) return st;
+  if ((st = check_shape(shp_kv, dt)) != RELATION_OK) return st;
+  if (causal != 0 && causal != 1) return RELATION_ERR_INVALID_ARG;
+  if (shp_kv.B != shp_q.B || shp_kv.H != shp_q.H || shp_kv.d_h != shp_q.d_h)
+    return RELATION_ERR_INVALID_ARG;
+  if (causal && shp_kv.T != shp_q.T) return RELATION_ERR_INVALID_ARG;
+  if (!rel::tc::supports(dt, shp_q.d_h)) return RELATION_ERR_UNSUPPORTED;  // bf16 tiles
+  if ((long long)((shp_q.T + 127) / 128) * shp_q.B * shp_q.H > 0x7fffffffLL)
+    return RELATION_ERR_UNSUPPORTED;
+  if ((st = check_ptrs({q, k, v, m, l, z})) != RELATION_OK) return st;
+  if (dev_status && (reinterpret_cast<uintptr_t>(dev_status) & 3u)) return RELATION_ERR_ALIGNMENT;
+  Problem p = make_problem(shp_q, dt, 0.0f, 1.0f, dev_status);
+  p.q = q; p.k = k; p.v = v;
+  rel::StateArgs sa{};
+  sa.causal = causal;
+  sa.Tk = shp_kv.T;
+  sa.k_sB = shp_kv.sB; sa.k_sT = shp_kv.sT; sa.k_sH = shp_kv.sH;
+  sa.m = m; sa.l = l; sa.z = z;
+  return from_cuda(rel::tc::launch_fwd_state(p, sa, reinterpret_cast<cudaStream_t>(stream)));
+}
+
+relation_status relation_state_merge(float* m, float* l, float* z, const float* m2,
+                                     const float* l2, const float* z2, relation_shape shp,
+                                     relation_stream_t stream) {
+  if (shp.B < 1 || shp.T < 1 || shp.H < 1) return RELATION_ERR_INVALID_ARG;
+  if (shp.d_h < 4 || shp.d_h > 128 || shp.d_h % 4) return RELATION_ERR_UNSUPPORTED;
+  relation_status st;
+  if ((st = check_ptrs({m, l, z, m2, l2, z2})) != RELATION_OK) return st;
+  const long long rows = (long long)shp.B * shp.H * shp.T;
+  return from_cuda(rel::launch_state_merge(m, l, z, m2, l2, z2, rows, shp.d_h,
+                                           reinterpret_cast<cudaStream_t>(stream)));
+}
+
+relation_status relation_state_finish(const void* q, const void* k, const void* v,
+                                      const float* m, const float* l, const float* z, void* o,
+                                      float* logz, float* self_flow, float lambda, float tau_s,
+                                      long long pos0, relation_shape shp, relation_dtype dt,
+                                      relation_stream_t stream) {
+  relation_status st;
+  if ((st = check_shape(shp, dt)) != RELATION_OK) return st;
+  if ((st = check_scalars(lambda, tau_s)) != RELATION_OK) return st;
+  if (pos0 < 0) return RELATION_ERR_INVALID_ARG;
+  if (shp.d_h < 4 || shp.d_h > 128 || shp.d_h % 4) return RELATION_ERR_UNSUPPORTED;
+  if ((st = check_ptrs({q, k, v, m, l, z, o, logz})) != RELATION_OK) return st;
+  if (self_flow && (st = check_ptrs({self_flow})) != RELATION_OK) return st;
+  Problem p = make_problem(shp, dt, lambda, tau_s, nullptr);
+  p.q = q; p.k = k; p.v = v; p.out = o; p.logz = logz; p.fself = self_flow;
+  return from_cuda(rel::launch_state_finish(p, m, l, z, pos0,
+                                            reinterpret_cast<cudaStream_t>(stream)));
+}
+
 relation_status relation_linear_fwd(const void* p1, const void* p2, const void* v,
                                    const float* alpha, void* y, float tau_s, relation_shape shp,
                                    relation_dtype dt, int* dev_status, relation_stream_t stream) {

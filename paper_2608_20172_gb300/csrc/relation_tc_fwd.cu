@@ -155,11 +155,14 @@ __device__ __forceinline__ float2 scan_p(const uint32_t (&U)[N], int t, int kc0,
   return sum;
 }
 
-template <int D>
+// MODE 0: the forward (epilogue: Y, logZ, F_ii).  MODE 1: the Exchange summary only
+// (st.m, st.l, st.z), over the queries' own earlier tokens (st.causal) or over every key
+// of k, v (st.Tk of them, all preceding the queries; the ragged last tile masked).
+template <int D, int MODE>
 __global__ void __launch_bounds__(FwdCfg<D>::THREADS, 2)
     fwd_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmK,
                   const __grid_constant__ CUtensorMap tmV, const __grid_constant__ CUtensorMap tmO,
-                  Problem p, int n_qt, int n_groups) {
+                  Problem p, int n_qt, int n_groups, StateArgs sa) {
   using C = FwdCfg<D>;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>(
@@ -176,7 +179,8 @@ __global__ void __launch_bounds__(FwdCfg<D>::THREADS, 2)
   const int qt = n_qt - 1 - tq;
   const int b = bh / p.H, h = bh % p.H;
   const int q0 = qt * BM;
-  const int n_kv = qt + 1;
+  const bool causal = MODE == 0 || sa.causal;
+  const int n_kv = causal ? qt + 1 : (sa.Tk + BN - 1) / BN;
 
   if (threadIdx.x == 0) {
     mbar_init(bar(B_Q), 1);
@@ -321,8 +325,10 @@ __global__ void __launch_bounds__(FwdCfg<D>::THREADS, 2)
       const int j = s >> 1, hh = s & 1;
       if (ok) ok = __all_sync(0xffffffffu, mbar_wait(bar(B_S + hh), (s >> 1) & 1, ab));
       const uint32_t ucol = trow + kSCol + hh * HN + wg * C::CW;
-      const bool diag = (j == qt);
-      const int tl = t - hh * HN;  // this row's index relative to the step's first key
+      // causal: the diagonal tile masks the keys at and after the row (tl, relative to the
+      // step's first key); otherwise keys at and past Tk (a ragged last tile) are masked
+      const int tl = causal ? t - hh * HN : sa.Tk - j * BN - hh * HN;
+      const bool diag = causal ? (j == qt) : (tl < HN);
       uint32_t U[C::CW];
       float umax = -INFINITY;
       if (ok) {
@@ -401,7 +407,29 @@ __global__ void __launch_bounds__(FwdCfg<D>::THREADS, 2)
       }
     }
     tc_fence_after();
-    if (ok) {
+    if (MODE == 1 && ok) {
+      // the Exchange summary of row r: m in natural-log units, l, and z (real columns).
+      // The TMEM loads are warp-collective: every lane loads, rows past T store nothing.
+      const bool live = r < p.T;
+      const long long row = (long long)bh * p.T + r;
+      if (live) {
+        sa.m[row] = m == -INFINITY ? -INFINITY : m * kLn2;
+        sa.l[row] = l;
+      }
+      float* zr = sa.z + row * p.d;
+#pragma unroll
+      for (int c0 = 0; c0 < D; c0 += 32) {
+        uint32_t z[32];
+        tmem_ld32(trow + kOCol + c0, z);
+        tmem_ld_wait();
+#pragma unroll
+        for (int c = 0; c < 32; c += 4)
+          if (live && c0 + c < p.d)
+            *reinterpret_cast<float4*>(zr + c0 + c) =
+                make_float4(__uint_as_float(z[c]), __uint_as_float(z[c + 1]),
+                            __uint_as_float(z[c + 2]), __uint_as_float(z[c + 3]));
+      }
+    } else if (ok) {
       float g = 0.f, inv_l = 0.f, fself = 1.0f;  // F_ii = 1 - g: the Self flow
       float lz;
       const float S = 1.0f / (1.0f + __expf(-(u_self * isd) / p.tau_s));
@@ -510,17 +538,23 @@ bool supports(relation_dtype dt, int d) {
   return dt == RELATION_BF16 && d >= 8 && d <= 128 && d % 8 == 0;
 }
 
-template <int D>
-static cudaError_t fwd_t(const Problem& p, cudaStream_t s) {
+template <int D, int MODE>
+static cudaError_t fwd_t(const Problem& p, const StateArgs& sa, cudaStream_t s) {
   // A runtime call first: it makes the primary context current on this thread, which the
   // driver's tensor-map encoder needs.
   const int smem = FwdCfg<D>::SMEM;
-  cudaError_t e =
-      cudaFuncSetAttribute(fwd_tc_kernel<D>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+  cudaError_t e = cudaFuncSetAttribute(fwd_tc_kernel<D, MODE>,
+                                       cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
   if (e != cudaSuccess) { note_failure("forward: shared memory attribute"); return e; }
+  Problem pk = p;  // the keys' view: their own strides, and count (the state over other keys)
+  if (MODE == 1) {
+    pk.T = sa.causal ? p.T : sa.Tk;
+    pk.sB = sa.k_sB; pk.sT = sa.k_sT; pk.sH = sa.k_sH;
+  }
   CUtensorMap mq, mk, mv, mo;
-  if (!make_tmap_bf16(&mq, p.q, p, BM) || !make_tmap_bf16(&mk, p.k, p, BN) ||
-      !make_tmap_bf16(&mv, p.v, p, BN) || !make_tmap_bf16(&mo, p.out, p, 32)) {
+  if (!make_tmap_bf16(&mq, p.q, p, BM) || !make_tmap_bf16(&mk, p.k, pk, BN) ||
+      !make_tmap_bf16(&mv, p.v, pk, BN) ||
+      !make_tmap_bf16(&mo, MODE == 0 ? p.out : p.q, p, 32)) {  // (no output tile in MODE 1)
     note_failure("forward: TMA descriptor of Q/K/V/Y");
     return cudaErrorInvalidValue;
   }
@@ -532,15 +566,23 @@ static cudaError_t fwd_t(const Problem& p, cudaStream_t s) {
       cudaDeviceGetAttribute(&nsm, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess)
     nsm = 148;
   const int groups = head_groups(n_qt, p.B * p.H, 2 * nsm);  // two CTAs per SM
-  fwd_tc_kernel<D><<<(unsigned)grid, FwdCfg<D>::THREADS, smem, s>>>(mq, mk, mv, mo, p, n_qt,
-                                                                   groups);
+  fwd_tc_kernel<D, MODE><<<(unsigned)grid, FwdCfg<D>::THREADS, smem, s>>>(mq, mk, mv, mo, p,
+                                                                         n_qt, groups, sa);
   if ((e = cudaGetLastError()) != cudaSuccess) note_failure("forward: kernel launch");
   return e;
 }
 
 cudaError_t launch_fwd(const Problem& p, cudaStream_t s) {
   if (!supports(p.dtype, p.d)) return cudaErrorInvalidValue;
-  return p.d <= 64 ? fwd_t<64>(p, s) : fwd_t<128>(p, s);
+  StateArgs none{};
+  none.causal = 1;
+  return p.d <= 64 ? fwd_t<64, 0>(p, none, s) : fwd_t<128, 0>(p, none, s);
+}
+
+cudaError_t launch_fwd_state(const Problem& p, const StateArgs& sa, cudaStream_t s) {
+  if (!supports(p.dtype, p.d) || !sa.m || !sa.l || !sa.z || (!sa.causal && sa.Tk < 1))
+    return cudaErrorInvalidValue;
+  return p.d <= 64 ? fwd_t<64, 1>(p, sa, s) : fwd_t<128, 1>(p, sa, s);
 }
 
 }  // namespace tc

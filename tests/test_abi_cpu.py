@@ -336,3 +336,29 @@ def test_decode_rejects_bad_arguments(lib, case, expect):
     rc = lib.relation_decode(p[0], p[1], p[2], p[3], p[4], p[5], lam, 2.0, cache, qsB, qsH,
                              binding.BF16, ctypes.c_void_p(0x100000), ws, None, None)
     assert rc == expect
+
+
+def test_context_parallel_entry_points_reject_bad_arguments(lib):
+    """The context-parallel calls check their arguments on the host and launch nothing."""
+    q = _shape(B=2, T=100, H=3, d=64)
+    kv = _shape(B=2, T=40, H=3, d=64)
+    p = [ctypes.c_void_p(0x10000 * (i + 1)) for i in range(6)]
+    st = lambda *a: lib.relation_fwd_state(*p, *a, None, None)
+    assert st(q, kv, 0, binding.F32) == binding.ERR_UNSUPPORTED  # tensor-core tiles: bf16
+    assert st(q, kv, 2, binding.BF16) == binding.ERR_INVALID_ARG
+    assert st(q, kv, 1, binding.BF16) == binding.ERR_INVALID_ARG  # causal: T_k = T_q
+    assert st(q, _shape(B=2, T=40, H=4, d=64), 0, binding.BF16) == binding.ERR_INVALID_ARG
+    assert st(_shape(B=2, T=100, H=3, d=136), _shape(B=2, T=40, H=3, d=136), 0,
+              binding.BF16) == binding.ERR_UNSUPPORTED
+    assert lib.relation_fwd_state(*p[:3], None, *p[4:], q, kv, 0, binding.BF16, None,
+                                  None) == binding.ERR_INVALID_ARG
+    assert lib.relation_fwd_state(*p[:3], ctypes.c_void_p(0x10004), *p[4:], q, kv, 0,
+                                  binding.BF16, None, None) == binding.ERR_ALIGNMENT
+    assert lib.relation_state_merge(*p, _shape(d=132), None) == binding.ERR_UNSUPPORTED
+    assert lib.relation_state_merge(*p, _shape(T=0), None) == binding.ERR_INVALID_ARG
+    f = [ctypes.c_void_p(0x10000 * (i + 1)) for i in range(8)]
+    fin = lambda pos0, shp=q, lam=0.5: lib.relation_state_finish(*f, None, lam, 2.0, pos0, shp,
+                                                                 binding.BF16, None)
+    assert fin(-1) == binding.ERR_INVALID_ARG
+    assert fin(0, lam=float("nan")) == binding.ERR_INVALID_ARG
+    assert fin(0, shp=_shape(d=136)) == binding.ERR_UNSUPPORTED
