@@ -418,6 +418,50 @@ def paper_layers_measure(binding, dev, peaks, steps=10, warmup=3):
                     "whole-model training tok/s on another GPU (context only)"}
 
 
+def cp_measure(binding, w, dev, peaks, shards=4, steps=5, warmup=2):
+    """The forward of workload w computed as `shards` sequence shards on one GPU (each
+    shard's own causal summary, its summaries over every earlier shard's keys merged in,
+    then the epilogue at its positions), against the single-call forward: the cost of the
+    context-parallel form (the same causal pairs, plus the summaries' fp32 traffic)."""
+    q, k, v, _ = workloads.make_inputs(w, seed=0)
+    qd, kd, vd = (t.to(dev) for t in (q, k, v))
+    lam, tau = workloads.LAMBDA_INIT, workloads.TAU_S
+    stream = torch.cuda.current_stream(dev)
+    T = w.T
+    bounds = [T * s // shards for s in range(shards + 1)]
+    parts = [tuple(t[:, bounds[s]:bounds[s + 1]].contiguous() for t in (qd, kd, vd))
+             for s in range(shards)]
+    states = [binding.fwd_state(*parts[s], causal=True, stream=stream) for s in range(shards)]
+    other = [tuple(torch.empty_like(x) for x in st) for st in states]
+    outs = [(torch.empty_like(parts[s][0]),
+             torch.empty((w.B, w.H, bounds[s + 1] - bounds[s]), device=dev, dtype=torch.float32))
+            for s in range(shards)]
+    y_one = torch.empty_like(qd)
+    lz_one = torch.empty((w.B, w.H, T), device=dev, dtype=torch.float32)
+
+    def sharded():
+        for s in range(shards):
+            binding.fwd_state(*parts[s], causal=True, out=states[s], stream=stream)
+            for e in range(s):
+                binding.fwd_state(parts[s][0], parts[e][1], parts[e][2], causal=False,
+                                  out=other[s], stream=stream)
+                binding.state_merge(states[s], other[s], stream=stream)
+            binding.state_finish(*parts[s], states[s], lam, tau, pos0=bounds[s],
+                                 out=outs[s][0], logz=outs[s][1], stream=stream)
+
+    ms_cp = _time_calls(sharded, dev, steps, warmup)
+    ms_one = _time_calls(lambda: binding.fwd(qd, kd, vd, lam, tau, out=y_one, logz=lz_one,
+                                             stream=stream), dev, steps, warmup)
+    err = max(float((outs[s][0].float() - y_one[:, bounds[s]:bounds[s + 1]].float()).abs().max())
+              for s in range(shards))
+    fl = w.flops_fwd()
+    return {"workload": w.name, "shards": shards, "bounds": bounds, "ms_sharded": ms_cp,
+            "ms_one_call": ms_one, "overhead": ms_cp / ms_one,
+            "sharded_tflops": fl / (ms_cp * 1e-3) / 1e12,
+            "max_abs_diff_vs_one_call": err,
+            "gpu_launches": sum(2 + 2 * s for s in range(shards))}
+
+
 def sdpa_context(w, dev, steps=20, warmup=3):
     """Context only, not this library: PyTorch's causal scaled-dot-product attention
     (softmax attention, the paper's comparison operator) forward + backward on the same
@@ -790,6 +834,7 @@ def run_ours(args, w):
         line["linear"] = linear_measure(binding, dev, peaks)
         line["layer"] = layer_measure(binding, dev, peaks)
         line["paper_layers"] = paper_layers_measure(binding, dev, peaks)
+        line["context_parallel"] = cp_measure(binding, w, dev, peaks)
         try:
             line["context_sdpa"] = sdpa_context(w, dev)
         except Exception as exc:  # context only: never at the expense of the line

@@ -6,12 +6,10 @@
 // the elementwise work of the other.  CTAs take the heaviest query tiles first, heads in
 // groups (grouped_unit), so that the K/V rows in use stay in L2.
 //
-// Warp roles (128 NWG + 64 threads):
-//   warps 0 .. 4 NWG - 1  Exchange scan + epilogue: thread t of warpgroup g owns query row
-//              q0 + t (TMEM lane t) and the g-th of NWG column slices of every step (and
-//              of z); the warpgroups of a row agree on its maximum through shared memory.
-//   warp  4 NWG      TMA producer: Q tile once, then K and V tiles through a ring of stages.
-//   warp  4 NWG + 1  TMEM allocator and MMA issuer (one elected thread).
+// Warp roles (192 threads):
+//   warps 0-3  Exchange scan + epilogue: thread t owns query row q0 + t (TMEM lane t).
+//   warp  4    TMA producer: Q tile once, then K and V tiles through a ring of stages.
+//   warp  5    TMEM allocator and MMA issuer (one elected thread).
 // Per key tile j:
 // The scan advances 64 keys per step through two TMEM buffers, so the MMAs of one step
 // (U of step s + 2, z += P V of step s) overlap the elementwise work of the next.  Step s:
@@ -45,14 +43,12 @@ constexpr int kTmemCols = 256; // two U/P buffers of 64 columns + z accumulator 
 constexpr int kSCol = 0;       // buffer b at kSCol + 64 b
 constexpr int kOCol = 128;
 constexpr float kRescaleLog2 = 8.0f;  // rescale z only when the max grows by > 2^8
+constexpr float kStaleLog2 = 32.0f;   // a step's P may reach 2^32 at the previous scale
 
 template <int D>
 struct FwdCfg {
-  static constexpr int NWG = 1;  // scan warpgroups (column slices of a step)
-  static constexpr int CW = HN / NWG;          // keys of a step per warpgroup
-  static constexpr int ZW = D / NWG;           // z / Y columns per warpgroup
-  static constexpr int W_TMA = 4 * NWG, W_MMA = 4 * NWG + 1;
-  static constexpr int THREADS = 128 * NWG + 64;
+  static constexpr int W_TMA = 4, W_MMA = 5;
+  static constexpr int THREADS = 192;
   static constexpr int KB = D / 64;            // 64-column (128-byte) swizzle blocks along d
   static constexpr int TILE = BN * D * 2;      // bytes of one K, V (or Q) tile
   static constexpr int STAGES = D == 64 ? 2 : 1;
@@ -60,16 +56,9 @@ struct FwdCfg {
   static constexpr int OFF_K = OFF_Q + TILE;
   static constexpr int OFF_V = OFF_K + STAGES * TILE;
   static constexpr int OFF_BAR = OFF_V + STAGES * TILE;
-  // row exchange between the warpgroups: partial maxima [2 steps][NWG][128], U_ii [128],
-  // partial row sums [NWG][128] (fp32), ok flags [2][NWG][4] (int)
-  static constexpr int OFF_X = OFF_BAR + 256;
-  static constexpr int SMEM = OFF_X + (2 * NWG + 1 + NWG) * BM * 4 + 2 * NWG * 4 * 4 + 1024;
+  static constexpr int SMEM = OFF_BAR + 256 + 1024;  // barriers + 1024-byte alignment slack
   static_assert(SMEM <= 232448 / 2, "two CTAs per SM");
 };
-// the cross-warpgroup exchange of a row (the NWG warps that share TMEM lanes 32 (w & 3) ..)
-__device__ __forceinline__ void row_sync(int warp, int nwg) {
-  asm volatile("bar.sync %0, %1;" ::"r"(1 + (warp & 3)), "r"(32 * nwg) : "memory");
-}
 
 // mbarrier slots
 enum : int {
@@ -90,50 +79,49 @@ __device__ __forceinline__ float fmax3(float a, float b, float c) {
   return d;
 }
 
-// Maximum of the raw evidence U over the row's history, for N keys whose first is key c0
-// of the step; on the diagonal tile only the keys before the row's own (t, relative to the
-// step) count, and U at key t (the Self evidence U_ii) is returned in u_self.
-template <bool DIAG, int N>
-__device__ __forceinline__ float row_max(const uint32_t (&U)[N], int t, int c0, float& u_self) {
-  static_assert(N % 8 == 4 || N % 8 == 0, "four running maxima over key pairs");
+// Maximum of the raw evidence U over the row's history in one step; on the diagonal tile
+// only the keys before the row's own (t, relative to the step's first key) count, and U at
+// key t (the Self evidence U_ii) is returned in u_self.
+template <bool DIAG>
+__device__ __forceinline__ float row_max(const uint32_t (&U)[HN], int t, float& u_self) {
   if (!DIAG) {
     float m0 = __uint_as_float(U[0]), m1 = __uint_as_float(U[1]);
     float m2 = __uint_as_float(U[2]), m3 = __uint_as_float(U[3]);
 #pragma unroll
-    for (int c = 4; c + 8 <= N; c += 8) {
+    for (int c = 4; c + 8 <= HN; c += 8) {
       m0 = fmax3(m0, __uint_as_float(U[c]), __uint_as_float(U[c + 1]));
       m1 = fmax3(m1, __uint_as_float(U[c + 2]), __uint_as_float(U[c + 3]));
       m2 = fmax3(m2, __uint_as_float(U[c + 4]), __uint_as_float(U[c + 5]));
       m3 = fmax3(m3, __uint_as_float(U[c + 6]), __uint_as_float(U[c + 7]));
     }
-    if (N % 8 == 0) {  // the last four keys
-      m0 = fmax3(m0, __uint_as_float(U[N - 4]), __uint_as_float(U[N - 3]));
-      m1 = fmax3(m1, __uint_as_float(U[N - 2]), __uint_as_float(U[N - 1]));
-    }
+    // the last four keys (the loop covers keys 4 .. HN - 5)
+    m0 = fmax3(m0, __uint_as_float(U[HN - 4]), __uint_as_float(U[HN - 3]));
+    m1 = fmax3(m1, __uint_as_float(U[HN - 2]), __uint_as_float(U[HN - 1]));
     return fmaxf(fmax3(m0, m1, m2), m3);
   }
   float m = -INFINITY;
 #pragma unroll
-  for (int c = 0; c < N; ++c) {
+  for (int c = 0; c < HN; ++c) {
     const float x = __uint_as_float(U[c]);
-    m = c0 + c < t ? fmaxf(m, x) : m;
-    u_self = c0 + c == t ? x : u_self;
+    m = c < t ? fmaxf(m, x) : m;
+    u_self = c == t ? x : u_self;
   }
   return m;
 }
 
-// P = 2^(U c2k (1 + tanh(U ch)) - m) for N keys of a step, the first of them key c0 of the
-// step (0 off the history on the diagonal tile), written to TMEM columns pcol.. as bf16
-// pairs; returns the row sum as two halves.
-template <bool DIAG, int N>
-__device__ __forceinline__ float2 scan_p(const uint32_t (&U)[N], int t, int kc0, uint32_t pcol,
-                                         float ch, float c2k, float negm) {
-  static_assert(N % 32 == 0, "32 keys per TMEM store");
+// P = 2^(U c2k (1 + tanh(U ch)) - m) for the 64 keys of a step (0 off the history on the
+// diagonal tile), written to TMEM columns pcol.. as bf16 pairs; returns the row sum as two
+// halves, and on the way the maximum of the raw evidence over the row's history in the
+// step (umax) and, on the diagonal tile, U_ii (u_self).
+template <bool DIAG>
+__device__ __forceinline__ float2 scan_p(const uint32_t (&U)[HN], int t, uint32_t pcol, float ch,
+                                         float c2k, float negm, float& umax, float& u_self) {
   const float2 ch2 = make_float2(ch, ch), c2k2 = make_float2(c2k, c2k);
   const float2 nm2 = make_float2(negm, negm);
   float2 sum = make_float2(0.f, 0.f);
+  float mx0 = -INFINITY, mx1 = -INFINITY;
 #pragma unroll
-  for (int c0 = 0; c0 < N; c0 += 32) {
+  for (int c0 = 0; c0 < HN; c0 += 32) {
     uint32_t pk[16];
 #pragma unroll
     for (int c = 0; c < 32; c += 2) {
@@ -144,14 +132,20 @@ __device__ __forceinline__ float2 scan_p(const uint32_t (&U)[N], int t, int kc0,
       const float2 e = __ffma2_rn(x, w, nm2);
       float2 pv = make_float2(ex2_approx(e.x), ex2_approx(e.y));
       if (DIAG) {
-        pv.x = (kc0 + c0 + c < t) ? pv.x : 0.f;
-        pv.y = (kc0 + c0 + c + 1 < t) ? pv.y : 0.f;
+        const bool in0 = c0 + c < t, in1 = c0 + c + 1 < t;
+        pv.x = in0 ? pv.x : 0.f;
+        pv.y = in1 ? pv.y : 0.f;
+        mx0 = fmax3(mx0, in0 ? x.x : -INFINITY, in1 ? x.y : -INFINITY);
+        u_self = c0 + c == t ? x.x : (c0 + c + 1 == t ? x.y : u_self);
+      } else {
+        (c & 2 ? mx1 : mx0) = fmax3(c & 2 ? mx1 : mx0, x.x, x.y);
       }
       sum = __fadd2_rn(sum, pv);
       pk[c >> 1] = pack_bf16x2(pv.x, pv.y);
     }
     tmem_st16(pcol + (c0 >> 1), pk);
   }
+  umax = fmaxf(mx0, mx1);
   return sum;
 }
 
@@ -192,7 +186,7 @@ __global__ void __launch_bounds__(FwdCfg<D>::THREADS, 2)
     }
     for (int bb = 0; bb < 2; ++bb) {
       mbar_init(bar(B_S + bb), 1);
-      mbar_init(bar(B_P + bb), 128 * C::NWG);
+      mbar_init(bar(B_P + bb), 128);
     }
     mbar_init(bar(B_O), 1);
     mbar_init(bar(B_OD), 1);
@@ -277,14 +271,13 @@ __global__ void __launch_bounds__(FwdCfg<D>::THREADS, 2)
       if (hh == 0 && !(ok = mbar_wait_warp(bar(B_VF + st), (j / C::STAGES) & 1, ab))) break;
       if (!(ok = mbar_wait_warp(bar(B_P + hh), (s >> 1) & 1, ab))) break;
       tc_fence_after();
-      // z += P V over the step's 64 keys (A = P from TMEM: warpgroup g's keys as bf16
-      // pairs at the start of its own U columns; B = V rows, N = d contiguous)
+      // z += P V over the step's 64 keys (A = P from TMEM as bf16 pairs in the first 32
+      // columns of the step's buffer; B = V rows, N = d contiguous)
 #pragma unroll
       for (int kk = 0; kk < HN / 16; ++kk) {
         const uint64_t bd = smem_desc_sw128(
             sb + C::OFF_V + st * C::TILE + (hh * HN + kk * 16) * 128, BN * 128, 1024);
-        const int pc = (16 * kk / C::CW) * C::CW + (16 * kk % C::CW) / 2;
-        mma_ts_w(tmem + kOCol, tmem + kSCol + hh * HN + pc, bd, idesc_pv,
+        mma_ts_w(tmem + kOCol, tmem + kSCol + hh * HN + kk * 8, bd, idesc_pv,
                  (s > 0 || kk > 0) ? 1u : 0u);
       }
       mma_commit_w(bar(B_OD));  // z update of step s done
@@ -295,117 +288,88 @@ __global__ void __launch_bounds__(FwdCfg<D>::THREADS, 2)
     __syncwarp();
   } else {
     // ------------------------------------------------------------------ scan + epilogue
-    const int t = threadIdx.x & 127;  // row q0 + t, TMEM lane t
-    const int wg = threadIdx.x >> 7;    // this warpgroup's slice: keys [wg CW, +CW) of a step
+    const int t = threadIdx.x;  // 0..127: row q0 + t, TMEM lane t
     const int r = q0 + t;
-    const uint32_t trow = tmem + ((uint32_t)((warp & 3) * 32) << 16);
-    float* const xmax = reinterpret_cast<float*>(smem + C::OFF_X);  // [2][NWG][128]
-    float* const xself = xmax + 2 * C::NWG * BM;                       // [128] U_ii
-    float* const xsum = xself + BM;                                    // [NWG][128]
-    int* const xok = reinterpret_cast<int*>(xsum + C::NWG * BM);       // [2][NWG][4] per warp
-    // Row exchange between the slices of a row: every warp takes the same sequence of
-    // exchanges (one per step, one at the end), whatever happened to its waits, and each
-    // exchange also combines the warps' ok flags, so that all slices leave together.
-    auto exchange_ok = [&](int buf, bool mine) -> bool {
-      if (lane == 0) xok[(buf * C::NWG + wg) * 4 + (warp & 3)] = mine ? 1 : 0;
-      row_sync(warp, C::NWG);
-      bool all = true;
-#pragma unroll
-      for (int g = 0; g < C::NWG; ++g) all = all && xok[(buf * C::NWG + g) * 4 + (warp & 3)] != 0;
-      return all;
-    };
+    const uint32_t trow = tmem + ((uint32_t)(warp * 32) << 16);
     const float isd = p.inv_sqrt_d;
     const float ch = 0.5f * isd;            // h = U * ch = u / 2
     const float c2k = ch * kLog2e;          // E log2(e) = U * c2k * (1 + tanh(h))
-    float m = -INFINITY;                    // running bound of max E, log2 units
-    float l = 0.f;                          // this slice's share of the row sum
+    const float bk = isd * kLog2e;          // bound of E log2 e: max(U, 0) bk (see below)
+    // The row's scale m (log2 units): P = 2^(E log2 e - m), l = sum P, z = sum P v, all
+    // at the same m.  m is set from the first step's bound of max E, SiLU(u) = u sigma(u)
+    // <= max(u, 0) (which exceeds max SiLU by u sigma(-u) <= 0.28, no transcendental), and
+    // afterwards every step runs at the scale of the steps before it: its own maximum is
+    // taken on the way (not before), and a bound that grew by more than 2^8 raises m once
+    // the step's z update has landed (m_next, applied at the next step).  A bound that
+    // jumps by more than 2^kStaleLog2 redoes the step at the new scale, so P stays below
+    // 2^(kStaleLog2 + 0.28).
+    float m = -INFINITY, m_next = -INFINITY;
+    float l = 0.f;
     float u_self = 0.f;
     bool ok = true;
+    // z (and l) from scale m to mn where `go`, once the z update of step s_done has landed
+    auto rescale = [&](bool go, float mn, int s_done) -> bool {
+      if (!__any_sync(0xffffffffu, go)) return true;
+      const float sc = go ? ex2_approx(m - mn) : 1.0f;
+      if (s_done >= 0) {
+        if (!__all_sync(0xffffffffu, mbar_wait(bar(B_OD), s_done & 1, ab))) return false;
+        tc_fence_after();
+#pragma unroll
+        for (int c0 = 0; c0 < D; c0 += 32) {
+          uint32_t z[32];
+          tmem_ld32(trow + kOCol + c0, z);
+          tmem_ld_wait();
+#pragma unroll
+          for (int c = 0; c < 32; ++c) z[c] = __float_as_uint(__uint_as_float(z[c]) * sc);
+          tmem_st16(trow + kOCol + c0, z);
+          tmem_st16(trow + kOCol + c0 + 16, z + 16);
+        }
+      }
+      l *= sc;
+      if (go) m = mn;
+      return true;
+    };
     for (int s = 0; s < 2 * n_kv; ++s) {
       const int j = s >> 1, hh = s & 1;
-      if (ok) ok = __all_sync(0xffffffffu, mbar_wait(bar(B_S + hh), (s >> 1) & 1, ab));
-      const uint32_t ucol = trow + kSCol + hh * HN + wg * C::CW;
+      // the larger scale decided at step s - 1, after that step's z update
+      if (!(ok = rescale(m_next > m, m_next, s - 1))) break;
+      ok = __all_sync(0xffffffffu, mbar_wait(bar(B_S + hh), (s >> 1) & 1, ab));  // warp-uniform
+      if (!ok) break;
+      tc_fence_after();
+      const uint32_t ucol = trow + kSCol + hh * HN;
+      uint32_t U[HN];
+      tmem_ld32(ucol, U);
+      tmem_ld32(ucol + 32, U + 32);
+      tmem_ld_wait();
       // causal: the diagonal tile masks the keys at and after the row (tl, relative to the
       // step's first key); otherwise keys at and past Tk (a ragged last tile) are masked
       const int tl = causal ? t - hh * HN : sa.Tk - j * BN - hh * HN;
       const bool diag = causal ? (j == qt) : (tl < HN);
-      uint32_t U[C::CW];
-      float umax = -INFINITY;
-      if (ok) {
-        tc_fence_after();
-#pragma unroll
-        for (int c = 0; c < C::CW; c += 32) tmem_ld32(ucol + c, U + c);
-        tmem_ld_wait();
-        // Pass 1: maximum of the raw evidence over the row's history (on the diagonal
-        // tile only the keys before the row, tl; every key of an earlier tile), and U_ii
-        umax = diag ? row_max<true>(U, tl, wg * C::CW, u_self)
-                    : row_max<false>(U, tl, wg * C::CW, u_self);
+      // a row that has seen no key yet (z = 0, l = 0) takes this step's bound first
+      if (__any_sync(0xffffffffu, m == -INFINITY)) {
+        const float um = diag ? row_max<true>(U, tl, u_self) : row_max<false>(U, tl, u_self);
+        if (m == -INFINITY && um != -INFINITY) m = fmaxf(um, 0.f) * bk;
       }
-      if (C::NWG > 1) {  // the slices' maxima (two buffers: a slice may write the next
-                         // step's while another still reads this one's)
-        float* xm = xmax + (s & 1) * C::NWG * BM;
-        xm[wg * BM + t] = umax;
-        ok = exchange_ok(s & 1, ok);
-        if (ok) {
-#pragma unroll
-          for (int g = 0; g < C::NWG; ++g) umax = fmaxf(umax, xm[g * BM + t]);
-        }
+      float umax;
+      float2 rs = diag ? scan_p<true>(U, tl, ucol, ch, c2k, m == -INFINITY ? 0.f : -m, umax, u_self)
+                       : scan_p<false>(U, tl, ucol, ch, c2k, m == -INFINITY ? 0.f : -m, umax, u_self);
+      const float mt = umax == -INFINITY ? -INFINITY : fmaxf(umax, 0.f) * bk;
+      const bool jump = mt > m + kStaleLog2;  // false while both are -inf
+      if (__any_sync(0xffffffffu, jump)) {
+        // rare: redo the step at the new scale (z rescaled after step s - 1's update)
+        if (!(ok = rescale(jump, fmaxf(mt, m_next), s - 1))) break;
+        rs = diag ? scan_p<true>(U, tl, ucol, ch, c2k, -m, umax, u_self)
+                  : scan_p<false>(U, tl, ucol, ch, c2k, -m, umax, u_self);
       }
-      if (!ok) break;
-      // Upper bound of max E: SiLU(u) = u sigma(u) <= max(u, 0), and the bound exceeds
-      // SiLU(u) by u sigma(-u) <= 0.28, so P = 2^(E log2 e - m) stays in (0.75, 1] at the
-      // row's largest entry; no transcendental on this path.  Every slice takes the same
-      // decision from the same numbers.
-      const float mt = umax == -INFINITY ? -INFINITY : fmaxf(umax, 0.f) * (isd * kLog2e);
-      const float mn = fmaxf(m, mt);
-      const bool grow = mn > m + kRescaleLog2;  // false while both are -inf
-      const float scale = grow ? ex2_approx(m - mn) : 1.0f;
-      if (grow) m = mn;
-      l *= scale;
-      if (s > 0 && __any_sync(0xffffffffu, grow)) {
-        // rescale this slice's z columns once the z update of step s-1 has landed (the
-        // one of step s waits for this step's P); a failed wait ends the scan at the
-        // next exchange
-        ok = __all_sync(0xffffffffu, mbar_wait(bar(B_OD), (s - 1) & 1, ab));
-        if (!ok) continue;
-        tc_fence_after();
-#pragma unroll
-        for (int c0 = 0; c0 < C::ZW; c0 += 32) {
-          uint32_t z[32];
-          tmem_ld32(trow + kOCol + wg * C::ZW + c0, z);
-          tmem_ld_wait();
-#pragma unroll
-          for (int c = 0; c < 32; ++c) z[c] = __float_as_uint(__uint_as_float(z[c]) * scale);
-          tmem_st16(trow + kOCol + wg * C::ZW + c0, z);
-          tmem_st16(trow + kOCol + wg * C::ZW + c0 + 16, z + 16);
-        }
-      }
-      // Pass 2: P = 2^(E log2 e - m) on the history, 0 elsewhere; written back as bf16 at
-      // the start of this slice's own U columns (read into registers above).
-      const float negm = (m == -INFINITY) ? 0.f : -m;
-      const float2 rs = diag ? scan_p<true>(U, tl, wg * C::CW, ucol, ch, c2k, negm)
-                             : scan_p<false>(U, tl, wg * C::CW, ucol, ch, c2k, negm);
+      if (mt > m + kRescaleLog2) m_next = fmaxf(m_next, mt);
       l += rs.x + rs.y;
       tmem_st_wait();
       tc_fence_before();
       mbar_arrive(bar(B_P + hh));
     }
     // ---------------------------------------------------------------- epilogue
+    // (a scale still pending at the end needs nothing: m, l and z agree)
     if (ok) ok = __all_sync(0xffffffffu, mbar_wait(bar(B_O), 0, ab));
-    if (C::NWG > 1) {
-      // the row's sum and U_ii from every slice (U_ii: the slice that holds key t of the
-      // diagonal tile's step)
-      xsum[wg * BM + t] = l;
-      const int own = t - (t < HN ? 0 : HN);
-      if (own >= wg * C::CW && own < (wg + 1) * C::CW) xself[t] = u_self;
-      ok = exchange_ok(0, ok);
-      if (ok) {
-        l = 0.f;
-#pragma unroll
-        for (int g = 0; g < C::NWG; ++g) l += xsum[g * BM + t];
-        u_self = xself[t];
-      }
-    }
     tc_fence_after();
     if (MODE == 1 && ok) {
       // the Exchange summary of row r: m in natural-log units, l, and z (real columns).
@@ -444,13 +408,12 @@ __global__ void __launch_bounds__(FwdCfg<D>::THREADS, 2)
         lz = S;  // empty history (row 1)
       }
       // v_i from the diagonal tile's V rows, still in shared memory (row t of the stage,
-      // 128-byte swizzle); Y (this slice's columns) staged in the Q tile's space (free:
-      // every MMA has completed) and written by TMA, 32 rows per row-warp, once every
-      // slice has staged its columns (rows >= T are clipped).
+      // 128-byte swizzle); Y staged in the Q tile's space (free: every MMA has completed)
+      // and written by one TMA store of 32 rows per warp (rows >= T are clipped).
       const uint8_t* vrow = smem + C::OFF_V + (qt % C::STAGES) * C::TILE + t * 128;
-      uint8_t* ystage = smem + C::OFF_Q + (warp & 3) * (32 * D * 2) + lane * 128;
+      uint8_t* ystage = smem + C::OFF_Q + warp * (32 * D * 2) + lane * 128;
 #pragma unroll
-      for (int c0 = wg * C::ZW; c0 < (wg + 1) * C::ZW; c0 += 32) {
+      for (int c0 = 0; c0 < D; c0 += 32) {
         uint32_t z[32];
         tmem_ld32(trow + kOCol + c0, z);
         tmem_ld_wait();
@@ -474,17 +437,16 @@ __global__ void __launch_bounds__(FwdCfg<D>::THREADS, 2)
         }
       }
       fence_async_smem();
-      if (C::NWG > 1) row_sync(warp, C::NWG);  // every slice agreed on ok above
-      else __syncwarp();
-      if (wg == 0 && lane == 0) {
+      __syncwarp();
+      if (lane == 0) {
         for (int kb = 0; kb < C::KB; ++kb)
-          tma_store_4d(&tmO, sb + C::OFF_Q + (warp & 3) * (32 * D * 2) + kb * (32 * 128),
-                       kb * 64, q0 + (warp & 3) * 32, h, b);
+          tma_store_4d(&tmO, sb + C::OFF_Q + warp * (32 * D * 2) + kb * (32 * 128), kb * 64,
+                       q0 + warp * 32, h, b);
         tma_store_commit();
         tma_store_wait_read_all();  // the staging buffer must outlive the store's reads
       }
       __syncwarp();
-      if (wg == 0 && r < p.T) {
+      if (r < p.T) {
         p.logz[(long long)bh * p.T + r] = lz;
         if (p.fself) p.fself[(long long)bh * p.T + r] = fself;
       }
