@@ -331,11 +331,14 @@ __global__ void __launch_bounds__(FwdCfg<D>::THREADS, 2)
     };
     for (int s = 0; s < 2 * n_kv; ++s) {
       const int j = s >> 1, hh = s & 1;
-      // the larger scale decided at step s - 1, after that step's z update
-      if (!(ok = rescale(m_next > m, m_next, s - 1))) break;
       ok = __all_sync(0xffffffffu, mbar_wait(bar(B_S + hh), (s >> 1) & 1, ab));  // warp-uniform
       if (!ok) break;
       tc_fence_after();
+      // the larger scale decided at step s - 1, after that step's z update.  Only here:
+      // U of step s was issued after the z update of step s - 2, so the z-update barrier
+      // has completed at least s - 1 phases and its parity wait for phase s - 1 is exact
+      // (before the wait above it could still be two phases short and pass at once).
+      if (!(ok = rescale(m_next > m, m_next, s - 1))) break;
       const uint32_t ucol = trow + kSCol + hh * HN;
       uint32_t U[HN];
       tmem_ld32(ucol, U);

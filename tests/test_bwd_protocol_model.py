@@ -28,10 +28,16 @@ class Barriers:
         self.done[name] = self.completed(name) + 1
 
     def ready(self, name, k):
-        """A wait for completion k (0-based), as mbarrier parity k & 1 sees it."""
+        """A wait for completion k (0-based), as mbarrier parity k & 1 sees it: exact only
+        while the barrier has completed k or k + 1 phases.  Two phases ahead the parity
+        test would never pass; one phase short (k - 1 completed) it passes at once, as if
+        phase k had completed."""
         c = self.completed(name)
         if c >= k + 2:
             raise Ambiguous(f"{name}: waiting for phase {k}, already {c} completed")
+        if c <= k - 1:
+            raise Ambiguous(f"{name}: waiting for phase {k} with only {c} completed: the "
+                            "parity test passes early")
         return c >= k + 1
 
 

@@ -2,13 +2,13 @@
 TMA (Q once, K and V through a ring of stages), MMA (U of step s + 2 after the z update of
 step s, 64-key steps on two TMEM buffers) and the scan warps (with the data-dependent
 wait for the previous z update before a rescale), run under random interleavings for
-both stage counts.  Checks for deadlock and for parity waits on a barrier already two
-phases ahead.  CPU only; the model mirrors the kernel's code, it does not run it."""
+both stage counts.  Checks for deadlock and for parity waits on a barrier two phases
+ahead or one phase short of the awaited completion.  CPU only; the model mirrors the kernel's code, it does not run it."""
 import random
 
 import pytest
 
-from tests.test_bwd_protocol_model import Barriers
+from tests.test_bwd_protocol_model import Ambiguous, Barriers
 
 
 def tma(n_kv, stages):
@@ -53,20 +53,29 @@ def mma(n_kv, stages):
     yield ("arrive", "O")
 
 
-def scan(n_kv, rescale_rng):
+def scan(n_kv, rescale_rng, rescale_first=False):
+    """The scan warps' waits: U of step s, then (data-dependent) the z update of step
+    s - 1 before a rescale: the scale raised at step s - 1, applied at step s, and the
+    rarer redo of a step whose bound jumped.  rescale_first puts the first of them
+    before the wait for U (an order the kernel must not use)."""
     for s in range(2 * n_kv):
+        pending = s > 0 and rescale_rng.random() < 0.3
+        if rescale_first and pending:
+            yield ("wait", "OD", s - 1)
         yield ("wait", f"S{s & 1}", s >> 1)
-        if s > 0 and rescale_rng.random() < 0.3:  # the running bound grew: rescale z
+        if pending and not rescale_first:
+            yield ("wait", "OD", s - 1)
+        if s > 0 and rescale_rng.random() < 0.1:  # the step's bound jumped: redo it
             yield ("wait", "OD", s - 1)
         yield ("arrive", f"P{s & 1}")
     yield ("wait", "O", 0)
 
 
-def run(n_kv, stages, seed):
+def run(n_kv, stages, seed, rescale_first=False):
     rng = random.Random(seed)
     bars = Barriers()
     roles = {"tma": tma(n_kv, stages), "mma": mma(n_kv, stages),
-             "scan": scan(n_kv, random.Random(seed + 1000))}
+             "scan": scan(n_kv, random.Random(seed + 1000), rescale_first)}
     pending = {name: next(gen, None) for name, gen in roles.items()}
     while any(ev is not None for ev in pending.values()):
         runnable = [n for n, ev in pending.items()
@@ -85,3 +94,16 @@ def run(n_kv, stages, seed):
 def test_forward_protocol(n_kv, stages):
     for seed in range(40):
         run(n_kv, stages, seed)
+
+
+def test_rescale_wait_before_the_step_is_caught():
+    """Waiting for the z update of step s - 1 before U of step s can meet the barrier one
+    phase short, where its parity test passes at once (z rescaled under an update still in
+    flight): the model flags that order."""
+    caught = 0
+    for seed in range(200):
+        try:
+            run(16, 2, seed, rescale_first=True)
+        except Ambiguous:
+            caught += 1
+    assert caught > 0

@@ -317,3 +317,25 @@ def test_persistent_backward_many_units(B, H, T, d):
     _, _, _, dl_all = oracle.mhr_bwd(q.double().numpy(), k.double().numpy(), v.double().numpy(),
                                      do.double().numpy(), LAM)
     pu.check_dlambda(res["dlambda"], dl_all, "bf16")
+
+
+@pytest.mark.parametrize("d", [64, 128])
+def test_forward_maximum_growing_through_the_sequence(d):
+    """Keys scaled up along the sequence (by 1 + 6 j / T), so the rows' maximum grows by
+    more than 2^8 many times after their first step: the scale is raised a step late,
+    after the z update in flight has landed.  Every row of every head against the oracle
+    (a rescale racing the update shows up as a few rows with z off by a large factor)."""
+    T = 2048
+    w = workloads.custom(1, 2, T, d, "bf16")
+    q, k, v, _ = workloads.make_inputs(w, seed=31 + d)
+    ramp = (1.0 + 6.0 * torch.arange(T, dtype=torch.float32) / T)[None, :, None, None]
+    k = (k.float() * ramp).to(torch.bfloat16)
+    lam, tau = workloads.LAMBDA_INIT, workloads.TAU_S
+    res = pu.gpu_run(q, k, v, None, lam, tau, kernel="tcgen05", bwd=False)
+    ref = pu.oracle_heads(q, k, v, None, lam, [(0, 0), (0, 1)], tau, bwd=False)
+    for (b, h), r in ref.items():
+        pu.check_recorded("growing maximum", f"Y d={d}", res["Y"][b, :, h].numpy(), r["Y"],
+                          "bf16", "out")
+        pu.check_logz(f"logZ[{b},{h}]", res["logZ"][b, h].numpy(), r["logZ"], "bf16")
+        # a wrong z shows up as rows far off even when the normwise error stays small
+        assert np.max(np.abs(res["Y"][b, :, h].numpy() - r["Y"])) < 0.25
