@@ -211,8 +211,8 @@ __global__ void __launch_bounds__(kThreads, 1)
     uint8_t* p1s = smem + C::OFF_P1;
     uint8_t* p2s = smem + C::OFF_P2;
     float* al = reinterpret_cast<float*>(smem + C::OFF_A);
-    auto al_at = [&](int tok, int ch) -> float& {  // [D / 32][128][32] fp32
-      return al[(ch >> 5) * (LT * 32) + tok * 32 + (ch & 31)];
+    auto al_at = [&](int tok, int ch) -> float& {  // [D / 32][128][32] fp32, 128-byte swizzle
+      return al[al_swz(tok, ch)];
     };
     float l_end = 0.f;  // this channel's L at the block's last token (phase C, c < D)
     bool ok = true, my_clamp = false;
@@ -305,9 +305,8 @@ __global__ void __launch_bounds__(kThreads, 1)
           const uint32_t off = (k >> 3) * LT * 128 + tok * 128 + (((k & 7) ^ (tok & 7)) << 4);
           const uint4 a4 = *reinterpret_cast<const uint4*>(p1s + off);
           const uint4 b4 = *reinterpret_cast<const uint4*>(p2s + off);
-          const float* lrow = &al_at(tok, 8 * k);
-          const float4 L0 = *reinterpret_cast<const float4*>(lrow);
-          const float4 L1 = *reinterpret_cast<const float4*>(lrow + 4);
+          const float4 L0 = *reinterpret_cast<const float4*>(&al_at(tok, 8 * k));
+          const float4 L1 = *reinterpret_cast<const float4*>(&al_at(tok, 8 * k + 4));
           const float4 M0 = *reinterpret_cast<const float4*>(lmid_s + 8 * k);
           const float4 M1 = *reinterpret_cast<const float4*>(lmid_s + 8 * k + 4);
           const float4 E0 = *reinterpret_cast<const float4*>(lend_s + 8 * k);
@@ -592,7 +591,7 @@ static cudaError_t fwd_t(const LinearProblem& lp, void* workspace, cudaStream_t 
   CUtensorMap m1, m2, mv, ma, my, mc;
   if (!tc::make_tmap_bf16(&m1, lp.p1, p, LT) || !tc::make_tmap_bf16(&m2, lp.p2, p, LT) ||
       !tc::make_tmap_bf16(&mv, lp.v, p, LT) || !tc::make_tmap_bf16(&my, lp.y, p, 32) ||
-      !make_tmap_alpha(&ma, lp)) {
+      !make_tmap_alpha(&ma, lp, true)) {
     note_failure("linear chunked forward: TMA descriptors");
     return cudaErrorInvalidValue;
   }
@@ -656,7 +655,7 @@ cudaError_t states_t(const LinearProblem& lp, const void* dy, void* workspace, c
   CUtensorMap m1, m2, mv, mg, ma;
   if (!tc::make_tmap_bf16(&m1, lp.p1, p, LT) || !tc::make_tmap_bf16(&m2, lp.p2, p, LT) ||
       !tc::make_tmap_bf16(&mv, lp.v, p, LT) || !tc::make_tmap_bf16(&mg, dy, p, LT) ||
-      !make_tmap_alpha(&ma, lp)) {
+      !make_tmap_alpha(&ma, lp, true)) {
     note_failure("linear chunked backward: TMA descriptors");
     return cudaErrorInvalidValue;
   }

@@ -68,6 +68,11 @@ __device__ __forceinline__ uint32_t swz(int r, int c, int rows) {
   return (uint32_t)((c >> 6) * rows * 128 + r * 128 + ((((c & 63) >> 3) ^ (r & 7)) << 4) +
                     (c & 7) * 2);
 }
+// element (token, channel) of [d / 32][128][32] fp32 tiles written by the swizzled
+// retention map: the 16-byte groups of a token's 128-byte row permuted by (token & 7)
+__device__ __forceinline__ int al_swz(int tok, int ch) {
+  return (ch >> 5) * (LT * 32) + tok * 32 + ((((ch & 31) >> 2) ^ (tok & 7)) << 2) + (ch & 3);
+}
 __device__ __forceinline__ float ld_bf(const uint8_t* base, uint32_t off) {
   return __bfloat162float(*reinterpret_cast<const __nv_bfloat16*>(base + off));
 }
@@ -76,8 +81,10 @@ __device__ __forceinline__ void st_bf(uint8_t* base, uint32_t off, float x) {
 }
 
 
-// 4-D map over the [B][T][H][d] fp32 retention: boxes of 32 channels x 128 tokens, no swizzle.
-inline bool make_tmap_alpha(CUtensorMap* m, const LinearProblem& p) {
+// 4-D map over the [B][T][H][d] fp32 retention: boxes of 32 channels x 128 tokens, no
+// swizzle, or (swz) with the 128-byte swizzle, so that a thread per token reading its row
+// and a thread per channel reading a column both spread over the banks (al_swz).
+inline bool make_tmap_alpha(CUtensorMap* m, const LinearProblem& p, bool swz = false) {
   static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
   if (!fn) {
     void* ptr = nullptr;
@@ -93,7 +100,8 @@ inline bool make_tmap_alpha(CUtensorMap* m, const LinearProblem& p) {
   cuuint32_t box[4] = {32, (cuuint32_t)LT, 1, 1};
   cuuint32_t estr[4] = {1, 1, 1, 1};
   return fn(m, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 4, const_cast<float*>(p.alpha), dims, strides, box,
-            estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_NONE,
+            estr, CU_TENSOR_MAP_INTERLEAVE_NONE,
+            swz ? CU_TENSOR_MAP_SWIZZLE_128B : CU_TENSOR_MAP_SWIZZLE_NONE,
             CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 

@@ -219,8 +219,8 @@ __global__ void __launch_bounds__(kThreads, 1)
     uint8_t* const p1s = smem + OFF_P1;
     uint8_t* const p2s = smem + OFF_P2;
     float* const al = reinterpret_cast<float*>(smem + OFF_AL);
-    auto al_at = [&](int tok, int ch) -> float& {  // [2][128][32] fp32
-      return al[(ch >> 5) * (LT * 32) + tok * 32 + (ch & 31)];
+    auto al_at = [&](int tok, int ch) -> float& {  // [2][128][32] fp32, 128-byte swizzle
+      return al[al_swz(tok, ch)];
     };
     float* const gl = reinterpret_cast<float*>(smem + OFF_GL);  // dL [t][GS]
     float* const ts = reinterpret_cast<float*>(smem + OFF_TS);  // Km Ys [t][GS]
@@ -287,7 +287,8 @@ __global__ void __launch_bounds__(kThreads, 1)
         const uint8_t* rd = smem + OFF_DC + c * 128;
         uint8_t* rp = smem + OFF_DCP + c * 128;
 #pragma unroll
-        for (int k = 0; k < 8; ++k) {
+        for (int k0 = 0; k0 < 8; ++k0) {
+          const int k = (k0 + c) & 7;  // rows 128 bytes apart: rotate the 16-byte groups
           const uint4 a4 = *reinterpret_cast<const uint4*>(r0 + 16 * k);
           const uint4 d4 = *reinterpret_cast<const uint4*>(rd + 16 * k);
           const uint32_t aw[4] = {a4.x, a4.y, a4.z, a4.w}, dw[4] = {d4.x, d4.y, d4.z, d4.w};
@@ -312,9 +313,8 @@ __global__ void __launch_bounds__(kThreads, 1)
           const uint32_t off = t * 128 + ((k ^ (t & 7)) << 4);
           const uint4 a4 = *reinterpret_cast<const uint4*>(p1s + off);
           const uint4 b4 = *reinterpret_cast<const uint4*>(p2s + off);
-          const float* lrow = &al_at(t, 8 * k);
-          const float4 L0 = *reinterpret_cast<const float4*>(lrow);
-          const float4 L1 = *reinterpret_cast<const float4*>(lrow + 4);
+          const float4 L0 = *reinterpret_cast<const float4*>(&al_at(t, 8 * k));
+          const float4 L1 = *reinterpret_cast<const float4*>(&al_at(t, 8 * k + 4));
           const float Lv[8] = {L0.x, L0.y, L0.z, L0.w, L1.x, L1.y, L1.z, L1.w};
           const uint32_t aw[4] = {a4.x, a4.y, a4.z, a4.w}, bw[4] = {b4.x, b4.y, b4.z, b4.w};
           uint32_t qm[4], km[4], kl[4];
@@ -405,9 +405,8 @@ __global__ void __launch_bounds__(kThreads, 1)
             const uint4 a4 = *reinterpret_cast<const uint4*>(p1s + off);
             const uint4 b4 = *reinterpret_cast<const uint4*>(p2s + off);
             const uint4 g4 = *reinterpret_cast<const uint4*>(gs + off);
-            const float* lrow = &al_at(t, 8 * kc);
-            const float4 L0 = *reinterpret_cast<const float4*>(lrow);
-            const float4 L1 = *reinterpret_cast<const float4*>(lrow + 4);
+            const float4 L0 = *reinterpret_cast<const float4*>(&al_at(t, 8 * kc));
+            const float4 L1 = *reinterpret_cast<const float4*>(&al_at(t, 8 * kc + 4));
             const float Lv[8] = {L0.x, L0.y, L0.z, L0.w, L1.x, L1.y, L1.z, L1.w};
             const uint32_t aw[4] = {a4.x, a4.y, a4.z, a4.w}, bw[4] = {b4.x, b4.y, b4.z, b4.w},
                            gw[4] = {g4.x, g4.y, g4.z, g4.w};
@@ -461,9 +460,8 @@ __global__ void __launch_bounds__(kThreads, 1)
             const uint32_t off = t * 128 + ((kc ^ (t & 7)) << 4);
             const uint4 a4 = *reinterpret_cast<const uint4*>(p1s + off);
             const uint4 b4 = *reinterpret_cast<const uint4*>(p2s + off);
-            const float* lrow = &al_at(t, 8 * kc);
-            const float4 L0 = *reinterpret_cast<const float4*>(lrow);
-            const float4 L1 = *reinterpret_cast<const float4*>(lrow + 4);
+            const float4 L0 = *reinterpret_cast<const float4*>(&al_at(t, 8 * kc));
+            const float4 L1 = *reinterpret_cast<const float4*>(&al_at(t, 8 * kc + 4));
             const float Lv[8] = {L0.x, L0.y, L0.z, L0.w, L1.x, L1.y, L1.z, L1.w};
             const uint32_t aw[4] = {a4.x, a4.y, a4.z, a4.w}, bw[4] = {b4.x, b4.y, b4.z, b4.w};
             uint32_t o1[4], o2[4];
@@ -508,7 +506,8 @@ __global__ void __launch_bounds__(kThreads, 1)
         const uint8_t* rc0 = smem + OFF_C0 + c * 128;
         const uint8_t* rdp = smem + OFF_DCP + c * 128;
 #pragma unroll
-        for (int k = 0; k < 8; ++k) {  // same swizzle in both tiles: a plain row dot
+        for (int k0 = 0; k0 < 8; ++k0) {  // same swizzle in both tiles: a plain row dot
+          const int k = (k0 + c) & 7;     // rows 128 bytes apart: rotate the 16-byte groups
           const uint4 a4 = *reinterpret_cast<const uint4*>(rc0 + 16 * k);
           const uint4 d4 = *reinterpret_cast<const uint4*>(rdp + 16 * k);
           const uint32_t aw[4] = {a4.x, a4.y, a4.z, a4.w}, dw[4] = {d4.x, d4.y, d4.z, d4.w};
@@ -520,9 +519,19 @@ __global__ void __launch_bounds__(kThreads, 1)
           }
         }
         float glh = 0.f, tsh = 0.f;
-        for (int i = 0; i < 64; ++i) {
-          glh += gl[(half * 64 + i) * GS + c];
-          tsh += ts[(half * 64 + i) * GS + c];
+#pragma unroll
+        for (int i0 = 0; i0 < 64; i0 += 16) {  // 16 independent loads in flight
+          float g16[16], t16[16];
+#pragma unroll
+          for (int u = 0; u < 16; ++u) {
+            g16[u] = gl[(half * 64 + i0 + u) * GS + c];
+            t16[u] = ts[(half * 64 + i0 + u) * GS + c];
+          }
+#pragma unroll
+          for (int u = 0; u < 16; ++u) {
+            glh += g16[u];
+            tsh += t16[u];
+          }
         }
         half_sum[half * 128 + c] = glh;
         half_sum[half * 128 + 64 + c] = tsh;
@@ -532,12 +541,19 @@ __global__ void __launch_bounds__(kThreads, 1)
                     (half == 0 ? half_sum[128 + c] : 0.f);
         const float* arow = p.alpha + (long long)b * p.sB + (long long)h * p.sH + c;
         float* drow = p.dalpha + (long long)b * p.sB + (long long)h * p.sH + c;
-        for (int i = 63; i >= 0; --i) {
-          const int tok = half * 64 + i;
-          run += gl[tok * GS + c];
-          if (t0 + tok < p.T) {
-            const long long o = (long long)(t0 + tok) * p.sT;
-            drow[o] = run / __ldg(arow + o);
+        for (int i0 = 48; i0 >= 0; i0 -= 16) {  // 16 tokens: loads first, then the suffix
+          float a16[16], g16[16];
+#pragma unroll
+          for (int u = 0; u < 16; ++u) {
+            const int tok = half * 64 + i0 + u;
+            a16[u] = t0 + tok < p.T ? __ldg(arow + (long long)(t0 + tok) * p.sT) : 1.f;
+            g16[u] = gl[tok * GS + c];
+          }
+#pragma unroll
+          for (int u = 15; u >= 0; --u) {
+            const int tok = half * 64 + i0 + u;
+            run += g16[u];
+            if (t0 + tok < p.T) drow[(long long)(t0 + tok) * p.sT] = run / a16[u];
           }
         }
       }
@@ -595,7 +611,7 @@ cudaError_t launch_linear_tc_bwd(const LinearProblem& p, cudaStream_t s) {
   CUtensorMap m1, m2, mv, mg, ma, mc0, mdc, o1, o2, ov;
   if (!tc::make_tmap_bf16(&m1, p.p1, q, LT) || !tc::make_tmap_bf16(&m2, p.p2, q, LT) ||
       !tc::make_tmap_bf16(&mv, p.v, q, LT) || !tc::make_tmap_bf16(&mg, p.dy, q, LT) ||
-      !make_tmap_alpha(&ma, p) || !make_tmap_c0(&mc0, cp.c0, heads * (nb + 1) * 64, 64) ||
+      !make_tmap_alpha(&ma, p, true) || !make_tmap_c0(&mc0, cp.c0, heads * (nb + 1) * 64, 64) ||
       !make_tmap_c0(&mdc, dcb, heads * nb * 64, 64) || !tc::make_tmap_bf16(&o1, p.dp1, q, 32) ||
       !tc::make_tmap_bf16(&o2, p.dp2, q, 32) || !tc::make_tmap_bf16(&ov, p.dv, q, 32)) {
     note_failure("linear chunked backward: TMA descriptors");
