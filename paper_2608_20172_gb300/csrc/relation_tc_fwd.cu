@@ -39,25 +39,36 @@ namespace tc {
 constexpr int BM = 128;        // query rows per CTA
 constexpr int BN = 128;        // keys per K/V tile (TMA granularity)
 constexpr int HN = 64;         // keys per scan step: two steps per K/V tile
-constexpr int kTmemCols = 256; // two U/P buffers of 64 columns + z accumulator (<= 128)
-constexpr int kSCol = 0;       // buffer b at kSCol + 64 b
-constexpr int kOCol = 128;
+constexpr int kSCol = 0;       // U/P buffer b at kSCol + 64 b
 constexpr float kRescaleLog2 = 8.0f;  // rescale z only when the max grows by > 2^8
 constexpr float kStaleLog2 = 32.0f;   // a step's P may reach 2^32 at the previous scale
 
+// d_h = 64 (QUAD): four CTAs per SM, so that each SM sub-partition runs four scan warps:
+//   TMEM 128 columns (one U/P buffer of 64 + z 64), K and V in 64-key halves through two
+//   stages each (50 KB of shared memory), the scan in 32-key halves (85 registers).
+// d_h = 128: two CTAs per SM: TMEM 256 columns (two U/P buffers + z 128), whole 128-key
+//   K/V tiles through one stage.
 template <int D>
 struct FwdCfg {
+  static constexpr bool QUAD = D == 64;
+  static constexpr int CTAS = QUAD ? 4 : 2;      // CTAs per SM
+  static constexpr int TMEM_COLS = QUAD ? 128 : 256;
+  static constexpr int NBUF = QUAD ? 1 : 2;      // U/P buffers
+  static constexpr int OCOL = NBUF * HN;         // z accumulator
   static constexpr int W_TMA = 4, W_MMA = 5;
   static constexpr int THREADS = 192;
-  static constexpr int KB = D / 64;            // 64-column (128-byte) swizzle blocks along d
-  static constexpr int TILE = BN * D * 2;      // bytes of one K, V (or Q) tile
-  static constexpr int STAGES = D == 64 ? 2 : 1;
+  static constexpr int KB = D / 64;              // 64-column (128-byte) swizzle blocks along d
+  static constexpr int TILE = BN * D * 2;        // bytes of the Q tile
+  static constexpr int KVR = QUAD ? HN : BN;     // K / V rows per load
+  static constexpr int KVT = KVR * D * 2;        // bytes of one K or V load
+  static constexpr int STAGES = QUAD ? 2 : 1;
   static constexpr int OFF_Q = 0;
   static constexpr int OFF_K = OFF_Q + TILE;
-  static constexpr int OFF_V = OFF_K + STAGES * TILE;
-  static constexpr int OFF_BAR = OFF_V + STAGES * TILE;
+  static constexpr int OFF_V = OFF_K + STAGES * KVT;
+  static constexpr int OFF_BAR = OFF_V + STAGES * KVT;
   static constexpr int SMEM = OFF_BAR + 256 + 1024;  // barriers + 1024-byte alignment slack
-  static_assert(SMEM <= 232448 / 2, "two CTAs per SM");
+  static_assert(CTAS * (SMEM + 1024) <= 233472, "CTAs per SM");
+  static_assert(OCOL + D <= TMEM_COLS, "TMEM");
 };
 
 // mbarrier slots
@@ -149,11 +160,74 @@ __device__ __forceinline__ float2 scan_p(const uint32_t (&U)[HN], int t, uint32_
   return sum;
 }
 
+// The four-CTA layout's scan works on 32 keys at a time (registers): the maximum of the
+// raw evidence over the history among them (keys before t, relative to their first key,
+// on a masked step), and U at key t in u_self.
+template <bool DIAG>
+__device__ __forceinline__ float row_max32(const uint32_t (&U)[32], int t, float& u_self) {
+  if (!DIAG) {
+    float m0 = __uint_as_float(U[0]), m1 = __uint_as_float(U[1]);
+    float m2 = __uint_as_float(U[2]), m3 = __uint_as_float(U[3]);
+#pragma unroll
+    for (int c = 4; c + 8 <= 32; c += 8) {
+      m0 = fmax3(m0, __uint_as_float(U[c]), __uint_as_float(U[c + 1]));
+      m1 = fmax3(m1, __uint_as_float(U[c + 2]), __uint_as_float(U[c + 3]));
+      m2 = fmax3(m2, __uint_as_float(U[c + 4]), __uint_as_float(U[c + 5]));
+      m3 = fmax3(m3, __uint_as_float(U[c + 6]), __uint_as_float(U[c + 7]));
+    }
+    m0 = fmax3(m0, __uint_as_float(U[28]), __uint_as_float(U[29]));
+    m1 = fmax3(m1, __uint_as_float(U[30]), __uint_as_float(U[31]));
+    return fmaxf(fmax3(m0, m1, m2), m3);
+  }
+  float m = -INFINITY;
+#pragma unroll
+  for (int c = 0; c < 32; ++c) {
+    const float x = __uint_as_float(U[c]);
+    m = c < t ? fmaxf(m, x) : m;
+    u_self = c == t ? x : u_self;
+  }
+  return m;
+}
+
+// P of 32 keys as 16 bf16 pairs (not stored), their row sum, and on the way the maximum
+// of their raw evidence over the history and U_ii (as scan_p).
+template <bool DIAG>
+__device__ __forceinline__ float2 scan_p32(const uint32_t (&U)[32], int t, float ch, float c2k,
+                                           float negm, float& umax, float& u_self,
+                                           uint32_t (&pk)[16]) {
+  const float2 ch2 = make_float2(ch, ch), c2k2 = make_float2(c2k, c2k);
+  const float2 nm2 = make_float2(negm, negm);
+  float2 sum = make_float2(0.f, 0.f);
+  float mx0 = -INFINITY, mx1 = -INFINITY;
+#pragma unroll
+  for (int c = 0; c < 32; c += 2) {
+    const float2 x = make_float2(__uint_as_float(U[c]), __uint_as_float(U[c + 1]));
+    const float2 h = __fmul2_rn(x, ch2);
+    const float2 th = make_float2(tanh_approx(h.x), tanh_approx(h.y));
+    const float2 w = __ffma2_rn(th, c2k2, c2k2);
+    const float2 e = __ffma2_rn(x, w, nm2);
+    float2 pv = make_float2(ex2_approx(e.x), ex2_approx(e.y));
+    if (DIAG) {
+      const bool in0 = c < t, in1 = c + 1 < t;
+      pv.x = in0 ? pv.x : 0.f;
+      pv.y = in1 ? pv.y : 0.f;
+      mx0 = fmax3(mx0, in0 ? x.x : -INFINITY, in1 ? x.y : -INFINITY);
+      u_self = c == t ? x.x : (c + 1 == t ? x.y : u_self);
+    } else {
+      (c & 2 ? mx1 : mx0) = fmax3(c & 2 ? mx1 : mx0, x.x, x.y);
+    }
+    sum = __fadd2_rn(sum, pv);
+    pk[c >> 1] = pack_bf16x2(pv.x, pv.y);
+  }
+  umax = fmaxf(mx0, mx1);
+  return sum;
+}
+
 // MODE 0: the forward (epilogue: Y, logZ, F_ii).  MODE 1: the Exchange summary only
 // (st.m, st.l, st.z), over the queries' own earlier tokens (st.causal) or over every key
 // of k, v (st.Tk of them, all preceding the queries; the ragged last tile masked).
 template <int D, int MODE>
-__global__ void __launch_bounds__(FwdCfg<D>::THREADS, 2)
+__global__ void __launch_bounds__(FwdCfg<D>::THREADS, FwdCfg<D>::CTAS)
     fwd_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmK,
                   const __grid_constant__ CUtensorMap tmV, const __grid_constant__ CUtensorMap tmO,
                   Problem p, int n_qt, int n_groups, StateArgs sa) {
@@ -193,7 +267,7 @@ __global__ void __launch_bounds__(FwdCfg<D>::THREADS, 2)
     *abort_flag = 0;
     fence_mbar_init();
   }
-  if (warp == C::W_MMA) tmem_alloc(smem_u32(tmem_slot), kTmemCols);
+  if (warp == C::W_MMA) tmem_alloc(smem_u32(tmem_slot), C::TMEM_COLS);
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
@@ -209,22 +283,26 @@ __global__ void __launch_bounds__(FwdCfg<D>::THREADS, 2)
       mbar_arrive_expect_tx(bar(B_Q), C::TILE);
       for (int kb = 0; kb < C::KB; ++kb)
         tma_load_4d(sb + C::OFF_Q + kb * BM * 128, &tmQ, bar(B_Q), kb * 64, q0, h, b);
+      // K and V through the stage ring, one load unit (QUAD: a 64-key half, one scan step;
+      // else a 128-key tile, two steps) at a time
+      constexpr int SPL = C::QUAD ? 1 : 2;  // scan steps per load unit
+      const int n_ld = 2 * n_kv / SPL;
       int issued = 0;
-      for (int j = 0; j < n_kv; ++j) {
+      for (int j = 0; j < n_ld; ++j) {
         const int s = j % C::STAGES, u = j / C::STAGES;
         if (u > 0 && !mbar_wait(bar(B_KE + s), (u - 1) & 1, ab)) break;
-        mbar_arrive_expect_tx(bar(B_KF + s), C::TILE);
+        mbar_arrive_expect_tx(bar(B_KF + s), C::KVT);
         for (int kb = 0; kb < C::KB; ++kb)
-          tma_load_4d(sb + C::OFF_K + s * C::TILE + kb * BN * 128, &tmK, bar(B_KF + s), kb * 64,
-                      j * BN, h, b);
+          tma_load_4d(sb + C::OFF_K + s * C::KVT + kb * C::KVR * 128, &tmK, bar(B_KF + s),
+                      kb * 64, j * C::KVR, h, b);
         if (u > 0 && !mbar_wait(bar(B_VE + s), (u - 1) & 1, ab)) {
-          issued = j + 1;  // K of tile j is in flight, V is not
+          issued = j + 1;  // K of unit j is in flight, V is not
           break;
         }
-        mbar_arrive_expect_tx(bar(B_VF + s), C::TILE);
+        mbar_arrive_expect_tx(bar(B_VF + s), C::KVT);
         for (int kb = 0; kb < C::KB; ++kb)
-          tma_load_4d(sb + C::OFF_V + s * C::TILE + kb * BN * 128, &tmV, bar(B_VF + s), kb * 64,
-                      j * BN, h, b);
+          tma_load_4d(sb + C::OFF_V + s * C::KVT + kb * C::KVR * 128, &tmV, bar(B_VF + s),
+                      kb * 64, j * C::KVR, h, b);
         issued = j + 1;
       }
       if (ab.raised()) {
@@ -242,10 +320,11 @@ __global__ void __launch_bounds__(FwdCfg<D>::THREADS, 2)
     // Warp-uniform: every lane runs the loop and the waits, one elected lane issues.
     constexpr uint32_t idesc_qk = idesc_bf16_f32(BM, HN, false, false);
     constexpr uint32_t idesc_pv = idesc_bf16_f32(BM, D, false, true);
-    const int total = 2 * n_kv;  // scan steps: two 64-key halves per K/V tile
-    // U of step s = Q K^T over keys [64 (s & 1), +64) of tile s / 2, into buffer s & 1
+    const int total = 2 * n_kv;  // scan steps of 64 keys
+    constexpr int SPL = C::QUAD ? 1 : 2;  // scan steps per K/V load unit
+    // U of step s = Q K^T over keys [64 s, +64) into buffer s % NBUF
     auto issue_u = [&](int s) -> bool {
-      const int j = s >> 1, hh = s & 1, st = j % C::STAGES;
+      const int j = s / SPL, hh = s % SPL, st = j % C::STAGES, bf = s % C::NBUF;
       if (hh == 0) {
         if (!mbar_wait_warp(bar(B_KF + st), (j / C::STAGES) & 1, ab)) return false;
         tc_fence_after();
@@ -253,36 +332,38 @@ __global__ void __launch_bounds__(FwdCfg<D>::THREADS, 2)
 #pragma unroll
       for (int kk = 0; kk < D / 16; ++kk) {
         const uint32_t koff = (kk >> 2) * (BN * 128) + (kk & 3) * 32;
+        const uint32_t kkoff = (kk >> 2) * (C::KVR * 128) + (kk & 3) * 32;
         const uint64_t a = smem_desc_sw128(sb + C::OFF_Q + koff, 16, 1024);
         const uint64_t bd =
-            smem_desc_sw128(sb + C::OFF_K + st * C::TILE + hh * HN * 128 + koff, 16, 1024);
-        mma_ss_w(tmem + kSCol + hh * HN, a, bd, idesc_qk, kk > 0 ? 1u : 0u);
+            smem_desc_sw128(sb + C::OFF_K + st * C::KVT + hh * HN * 128 + kkoff, 16, 1024);
+        mma_ss_w(tmem + kSCol + bf * HN, a, bd, idesc_qk, kk > 0 ? 1u : 0u);
       }
-      mma_commit_w(bar(B_S + hh));  // U ready (and every earlier z update done)
-      if (hh == 1) mma_commit_w(bar(B_KE + st));  // K stage free
+      mma_commit_w(bar(B_S + bf));  // U ready (and every earlier z update done)
+      if (hh == SPL - 1) mma_commit_w(bar(B_KE + st));  // K stage free
       return true;
     };
     bool ok = mbar_wait_warp(bar(B_Q), 0, ab);
     tc_fence_after();
     if (ok) ok = issue_u(0);
-    if (ok && total > 1) ok = issue_u(1);
+    if (ok && total > 1 && C::NBUF == 2) ok = issue_u(1);
     for (int s = 0; ok && s < total; ++s) {
-      const int j = s >> 1, hh = s & 1, st = j % C::STAGES;
+      const int j = s / SPL, hh = s % SPL, st = j % C::STAGES, bf = s % C::NBUF;
       if (hh == 0 && !(ok = mbar_wait_warp(bar(B_VF + st), (j / C::STAGES) & 1, ab))) break;
-      if (!(ok = mbar_wait_warp(bar(B_P + hh), (s >> 1) & 1, ab))) break;
+      if (!(ok = mbar_wait_warp(bar(B_P + bf), (s / C::NBUF) & 1, ab))) break;
       tc_fence_after();
       // z += P V over the step's 64 keys (A = P from TMEM as bf16 pairs in the first 32
       // columns of the step's buffer; B = V rows, N = d contiguous)
 #pragma unroll
       for (int kk = 0; kk < HN / 16; ++kk) {
         const uint64_t bd = smem_desc_sw128(
-            sb + C::OFF_V + st * C::TILE + (hh * HN + kk * 16) * 128, BN * 128, 1024);
-        mma_ts_w(tmem + kOCol, tmem + kSCol + hh * HN + kk * 8, bd, idesc_pv,
+            sb + C::OFF_V + st * C::KVT + (hh * HN + kk * 16) * 128, C::KVR * 128, 1024);
+        mma_ts_w(tmem + C::OCOL, tmem + kSCol + bf * HN + kk * 8, bd, idesc_pv,
                  (s > 0 || kk > 0) ? 1u : 0u);
       }
       mma_commit_w(bar(B_OD));  // z update of step s done
-      if (hh == 1) mma_commit_w(bar(B_VE + st));  // V stage free
-      if (s + 2 < total && !(ok = issue_u(s + 2))) break;  // buffer hh: P read above
+      if (hh == SPL - 1) mma_commit_w(bar(B_VE + st));  // V stage free
+      // the next U into the buffer whose P was read above (tcgen05 MMAs run in order)
+      if (s + C::NBUF < total && !(ok = issue_u(s + C::NBUF))) break;
     }
     mma_commit_w(bar(B_O));  // z final (or whatever completed before an abort)
     __syncwarp();
@@ -307,22 +388,24 @@ __global__ void __launch_bounds__(FwdCfg<D>::THREADS, 2)
     float l = 0.f;
     float u_self = 0.f;
     bool ok = true;
-    // z (and l) from scale m to mn where `go`, once the z update of step s_done has landed
-    auto rescale = [&](bool go, float mn, int s_done) -> bool {
-      if (!__any_sync(0xffffffffu, go)) return true;
+    // z (and l) from scale m to mn where `go`, once the z update of step s_done has landed;
+    // *scp gets the lane's factor (1 where not `go`)
+    auto rescale = [&](bool go, float mn, int s_done, float* scp) -> bool {
       const float sc = go ? ex2_approx(m - mn) : 1.0f;
+      if (scp) *scp = sc;
+      if (!__any_sync(0xffffffffu, go)) return true;
       if (s_done >= 0) {
         if (!__all_sync(0xffffffffu, mbar_wait(bar(B_OD), s_done & 1, ab))) return false;
         tc_fence_after();
 #pragma unroll
         for (int c0 = 0; c0 < D; c0 += 32) {
           uint32_t z[32];
-          tmem_ld32(trow + kOCol + c0, z);
+          tmem_ld32(trow + C::OCOL + c0, z);
           tmem_ld_wait();
 #pragma unroll
           for (int c = 0; c < 32; ++c) z[c] = __float_as_uint(__uint_as_float(z[c]) * sc);
-          tmem_st16(trow + kOCol + c0, z);
-          tmem_st16(trow + kOCol + c0 + 16, z + 16);
+          tmem_st16(trow + C::OCOL + c0, z);
+          tmem_st16(trow + C::OCOL + c0 + 16, z + 16);
         }
       }
       l *= sc;
@@ -330,45 +413,97 @@ __global__ void __launch_bounds__(FwdCfg<D>::THREADS, 2)
       return true;
     };
     for (int s = 0; s < 2 * n_kv; ++s) {
-      const int j = s >> 1, hh = s & 1;
-      ok = __all_sync(0xffffffffu, mbar_wait(bar(B_S + hh), (s >> 1) & 1, ab));  // warp-uniform
+      const int j = s >> 1, hh = s & 1, bf = s % C::NBUF;
+      ok = __all_sync(0xffffffffu, mbar_wait(bar(B_S + bf), (s / C::NBUF) & 1, ab));
       if (!ok) break;
       tc_fence_after();
       // the larger scale decided at step s - 1, after that step's z update.  Only here:
-      // U of step s was issued after the z update of step s - 2, so the z-update barrier
-      // has completed at least s - 1 phases and its parity wait for phase s - 1 is exact
-      // (before the wait above it could still be two phases short and pass at once).
-      if (!(ok = rescale(m_next > m, m_next, s - 1))) break;
-      const uint32_t ucol = trow + kSCol + hh * HN;
-      uint32_t U[HN];
-      tmem_ld32(ucol, U);
-      tmem_ld32(ucol + 32, U + 32);
-      tmem_ld_wait();
+      // U of step s was issued after the z update of step s - 2 (of step s - 1 with one
+      // buffer), so the z-update barrier has completed at least s - 1 phases and its
+      // parity wait for phase s - 1 is exact (before the wait above it could still be two
+      // phases short and pass at once).
+      if (!(ok = rescale(m_next > m, m_next, s - 1, nullptr))) break;
+      const uint32_t ucol = trow + kSCol + bf * HN;
       // causal: the diagonal tile masks the keys at and after the row (tl, relative to the
       // step's first key); otherwise keys at and past Tk (a ragged last tile) are masked
       const int tl = causal ? t - hh * HN : sa.Tk - j * BN - hh * HN;
       const bool diag = causal ? (j == qt) : (tl < HN);
-      // a row that has seen no key yet (z = 0, l = 0) takes this step's bound first
-      if (__any_sync(0xffffffffu, m == -INFINITY)) {
-        const float um = diag ? row_max<true>(U, tl, u_self) : row_max<false>(U, tl, u_self);
-        if (m == -INFINITY && um != -INFINITY) m = fmaxf(um, 0.f) * bk;
-      }
       float umax;
-      float2 rs = diag ? scan_p<true>(U, tl, ucol, ch, c2k, m == -INFINITY ? 0.f : -m, umax, u_self)
-                       : scan_p<false>(U, tl, ucol, ch, c2k, m == -INFINITY ? 0.f : -m, umax, u_self);
-      const float mt = umax == -INFINITY ? -INFINITY : fmaxf(umax, 0.f) * bk;
-      const bool jump = mt > m + kStaleLog2;  // false while both are -inf
-      if (__any_sync(0xffffffffu, jump)) {
-        // rare: redo the step at the new scale (z rescaled after step s - 1's update)
-        if (!(ok = rescale(jump, fmaxf(mt, m_next), s - 1))) break;
-        rs = diag ? scan_p<true>(U, tl, ucol, ch, c2k, -m, umax, u_self)
-                  : scan_p<false>(U, tl, ucol, ch, c2k, -m, umax, u_self);
+      float2 rs;
+      if constexpr (C::QUAD) {
+        // two halves of 32 keys; P of each written back into the first 16 columns of its
+        // own U columns once the half's bound is known (a jump of the second half also
+        // rescales the first half's P, already in TMEM)
+        rs = make_float2(0.f, 0.f);
+        umax = -INFINITY;
+#pragma unroll
+        for (int hb = 0; hb < 2; ++hb) {
+          uint32_t U[32];
+          tmem_ld32(ucol + hb * 32, U);
+          tmem_ld_wait();
+          const int th = tl - hb * 32;        // the row's index relative to the half
+          const bool dg = diag && th < 32;    // some key of the half masked
+          if (__any_sync(0xffffffffu, m == -INFINITY)) {
+            const float um = dg ? row_max32<true>(U, th, u_self) : row_max32<false>(U, th, u_self);
+            if (m == -INFINITY && um != -INFINITY) m = fmaxf(um, 0.f) * bk;
+          }
+          uint32_t pk[16];
+          float mx;
+          float2 r = dg ? scan_p32<true>(U, th, ch, c2k, m == -INFINITY ? 0.f : -m, mx, u_self, pk)
+                        : scan_p32<false>(U, th, ch, c2k, m == -INFINITY ? 0.f : -m, mx, u_self, pk);
+          const float mt = mx == -INFINITY ? -INFINITY : fmaxf(mx, 0.f) * bk;
+          const bool jump = mt > m + kStaleLog2;
+          if (__any_sync(0xffffffffu, jump)) {
+            float sc;
+            if (!(ok = rescale(jump, fmaxf(mt, m_next), s - 1, &sc))) break;
+            rs = make_float2(rs.x * sc, rs.y * sc);  // the first half, at the old scale
+            if (hb == 1) {
+              uint32_t pa[16];
+              tmem_st_wait();
+              tmem_ld16(ucol, pa);
+              tmem_ld_wait();
+#pragma unroll
+              for (int c = 0; c < 16; ++c) {
+                const float2 v2 = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&pa[c]));
+                pa[c] = pack_bf16x2(v2.x * sc, v2.y * sc);
+              }
+              tmem_st16(ucol, pa);
+            }
+            r = dg ? scan_p32<true>(U, th, ch, c2k, -m, mx, u_self, pk)
+                   : scan_p32<false>(U, th, ch, c2k, -m, mx, u_self, pk);
+          }
+          tmem_st16(ucol + hb * 16, pk);
+          rs = __fadd2_rn(rs, r);
+          umax = fmaxf(umax, mx);
+        }
+        if (!ok) break;
+      } else {
+        uint32_t U[HN];
+        tmem_ld32(ucol, U);
+        tmem_ld32(ucol + 32, U + 32);
+        tmem_ld_wait();
+        // a row that has seen no key yet (z = 0, l = 0) takes this step's bound first
+        if (__any_sync(0xffffffffu, m == -INFINITY)) {
+          const float um = diag ? row_max<true>(U, tl, u_self) : row_max<false>(U, tl, u_self);
+          if (m == -INFINITY && um != -INFINITY) m = fmaxf(um, 0.f) * bk;
+        }
+        rs = diag ? scan_p<true>(U, tl, ucol, ch, c2k, m == -INFINITY ? 0.f : -m, umax, u_self)
+                  : scan_p<false>(U, tl, ucol, ch, c2k, m == -INFINITY ? 0.f : -m, umax, u_self);
+        const float mt = umax == -INFINITY ? -INFINITY : fmaxf(umax, 0.f) * bk;
+        const bool jump = mt > m + kStaleLog2;  // false while both are -inf
+        if (__any_sync(0xffffffffu, jump)) {
+          // rare: redo the step at the new scale (z rescaled after step s - 1's update)
+          if (!(ok = rescale(jump, fmaxf(mt, m_next), s - 1, nullptr))) break;
+          rs = diag ? scan_p<true>(U, tl, ucol, ch, c2k, -m, umax, u_self)
+                    : scan_p<false>(U, tl, ucol, ch, c2k, -m, umax, u_self);
+        }
       }
+      const float mt = umax == -INFINITY ? -INFINITY : fmaxf(umax, 0.f) * bk;
       if (mt > m + kRescaleLog2) m_next = fmaxf(m_next, mt);
       l += rs.x + rs.y;
       tmem_st_wait();
       tc_fence_before();
-      mbar_arrive(bar(B_P + hh));
+      mbar_arrive(bar(B_P + bf));
     }
     // ---------------------------------------------------------------- epilogue
     // (a scale still pending at the end needs nothing: m, l and z agree)
@@ -387,7 +522,7 @@ __global__ void __launch_bounds__(FwdCfg<D>::THREADS, 2)
 #pragma unroll
       for (int c0 = 0; c0 < D; c0 += 32) {
         uint32_t z[32];
-        tmem_ld32(trow + kOCol + c0, z);
+        tmem_ld32(trow + C::OCOL + c0, z);
         tmem_ld_wait();
 #pragma unroll
         for (int c = 0; c < 32; c += 4)
@@ -413,18 +548,21 @@ __global__ void __launch_bounds__(FwdCfg<D>::THREADS, 2)
       // v_i from the diagonal tile's V rows, still in shared memory (row t of the stage,
       // 128-byte swizzle); Y staged in the Q tile's space (free: every MMA has completed)
       // and written by one TMA store of 32 rows per warp (rows >= T are clipped).
-      const uint8_t* vrow = smem + C::OFF_V + (qt % C::STAGES) * C::TILE + t * 128;
+      // (QUAD: the last two 64-key halves, stages 0 and 1, rows t & 63 of the half t / 64)
+      const uint8_t* vrow = C::QUAD
+          ? smem + C::OFF_V + (t >> 6) * C::KVT + (t & 63) * 128
+          : smem + C::OFF_V + (qt % C::STAGES) * C::KVT + t * 128;
       uint8_t* ystage = smem + C::OFF_Q + warp * (32 * D * 2) + lane * 128;
 #pragma unroll
       for (int c0 = 0; c0 < D; c0 += 32) {
         uint32_t z[32];
-        tmem_ld32(trow + kOCol + c0, z);
+        tmem_ld32(trow + C::OCOL + c0, z);
         tmem_ld_wait();
         const int kb = c0 >> 6;  // 64-column block of the tile
 #pragma unroll
         for (int c8 = 0; c8 < 32; c8 += 8) {
           const int chunk = ((c0 & 63) + c8) >> 3;  // 16-byte chunk within the 128-byte row
-          const uint4 vv = *reinterpret_cast<const uint4*>(vrow + kb * BN * 128 +
+          const uint4 vv = *reinterpret_cast<const uint4*>(vrow + kb * C::KVR * 128 +
                                                            ((chunk ^ (t & 7)) << 4));
           const uint32_t vw[4] = {vv.x, vv.y, vv.z, vv.w};
           uint32_t yw[4];
@@ -460,7 +598,7 @@ __global__ void __launch_bounds__(FwdCfg<D>::THREADS, 2)
   __syncthreads();
   if (warp == C::W_MMA) {
     tc_fence_after();
-    tmem_dealloc(tmem, kTmemCols);
+    tmem_dealloc(tmem, C::TMEM_COLS);
   }
 }
 
@@ -517,8 +655,8 @@ static cudaError_t fwd_t(const Problem& p, const StateArgs& sa, cudaStream_t s) 
     pk.sB = sa.k_sB; pk.sT = sa.k_sT; pk.sH = sa.k_sH;
   }
   CUtensorMap mq, mk, mv, mo;
-  if (!make_tmap_bf16(&mq, p.q, p, BM) || !make_tmap_bf16(&mk, p.k, pk, BN) ||
-      !make_tmap_bf16(&mv, p.v, pk, BN) ||
+  if (!make_tmap_bf16(&mq, p.q, p, BM) || !make_tmap_bf16(&mk, p.k, pk, FwdCfg<D>::KVR) ||
+      !make_tmap_bf16(&mv, p.v, pk, FwdCfg<D>::KVR) ||
       !make_tmap_bf16(&mo, MODE == 0 ? p.out : p.q, p, 32)) {  // (no output tile in MODE 1)
     note_failure("forward: TMA descriptor of Q/K/V/Y");
     return cudaErrorInvalidValue;
@@ -530,7 +668,7 @@ static cudaError_t fwd_t(const Problem& p, const StateArgs& sa, cudaStream_t s) 
   if (cudaGetDevice(&dev) != cudaSuccess ||
       cudaDeviceGetAttribute(&nsm, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess)
     nsm = 148;
-  const int groups = head_groups(n_qt, p.B * p.H, 2 * nsm);  // two CTAs per SM
+  const int groups = head_groups(n_qt, p.B * p.H, FwdCfg<D>::CTAS * nsm);
   fwd_tc_kernel<D, MODE><<<(unsigned)grid, FwdCfg<D>::THREADS, smem, s>>>(mq, mk, mv, mo, p,
                                                                          n_qt, groups, sa);
   if ((e = cudaGetLastError()) != cudaSuccess) note_failure("forward: kernel launch");
