@@ -45,21 +45,27 @@ constexpr float kStaleLog2 = 32.0f;   // a step's P may reach 2^32 at the previo
 
 // d_h = 64 (QUAD): four CTAs per SM, so that each SM sub-partition runs four scan warps:
 //   TMEM 128 columns (one U/P buffer of 64 + z 64), K and V in 64-key halves through two
-//   stages each (50 KB of shared memory), the scan in 32-key halves (85 registers).
-// d_h = 128: two CTAs per SM: TMEM 256 columns (two U/P buffers + z 128), whole 128-key
-//   K/V tiles through one stage.
+//   stages each (50 KB of shared memory), steps of 64 keys.
+// d_h = 128: two CTAs per SM, two U/P buffers of 64-key steps (so that the MMAs of one step
+//   overlap the scan of the next) + z 128 = 256 TMEM columns, 128-key K/V tiles through one
+//   stage.  (WIDE, steps of a whole 128-key tile in one buffer of 128 columns so that
+//   U = Q K^T runs at N = 128, measured slower on the long workload, 2.40 against 1.98 ms:
+//   each step then waits for its own 1024 cycles of MMAs, which two CTAs do not cover.)
+// With one U/P buffer the scan takes a step in chunks of 32 keys (registers).
 template <int D>
 struct FwdCfg {
   static constexpr bool QUAD = D == 64;
+  static constexpr bool WIDE = false;
+  static constexpr int SK = WIDE ? 128 : HN;     // keys per scan step
   static constexpr int CTAS = QUAD ? 4 : 2;      // CTAs per SM
   static constexpr int TMEM_COLS = QUAD ? 128 : 256;
-  static constexpr int NBUF = QUAD ? 1 : 2;      // U/P buffers
-  static constexpr int OCOL = NBUF * HN;         // z accumulator
+  static constexpr int NBUF = (QUAD || WIDE) ? 1 : 2;  // U/P buffers
+  static constexpr int OCOL = NBUF * SK;         // z accumulator
   static constexpr int W_TMA = 4, W_MMA = 5;
   static constexpr int THREADS = 192;
   static constexpr int KB = D / 64;              // 64-column (128-byte) swizzle blocks along d
   static constexpr int TILE = BN * D * 2;        // bytes of the Q tile
-  static constexpr int KVR = QUAD ? HN : BN;     // K / V rows per load
+  static constexpr int KVR = QUAD ? HN : BN;     // K / V rows per load (SK or 2 SK)
   static constexpr int KVT = KVR * D * 2;        // bytes of one K or V load
   static constexpr int STAGES = QUAD ? 2 : 1;
   static constexpr int OFF_Q = 0;
@@ -285,8 +291,7 @@ __global__ void __launch_bounds__(FwdCfg<D>::THREADS, FwdCfg<D>::CTAS)
         tma_load_4d(sb + C::OFF_Q + kb * BM * 128, &tmQ, bar(B_Q), kb * 64, q0, h, b);
       // K and V through the stage ring, one load unit (QUAD: a 64-key half, one scan step;
       // else a 128-key tile, two steps) at a time
-      constexpr int SPL = C::QUAD ? 1 : 2;  // scan steps per load unit
-      const int n_ld = 2 * n_kv / SPL;
+      const int n_ld = n_kv * (BN / C::KVR);
       int issued = 0;
       for (int j = 0; j < n_ld; ++j) {
         const int s = j % C::STAGES, u = j / C::STAGES;
@@ -318,11 +323,11 @@ __global__ void __launch_bounds__(FwdCfg<D>::THREADS, FwdCfg<D>::CTAS)
   } else if (warp == C::W_MMA) {
     // ------------------------------------------------------------------ MMA issuer
     // Warp-uniform: every lane runs the loop and the waits, one elected lane issues.
-    constexpr uint32_t idesc_qk = idesc_bf16_f32(BM, HN, false, false);
+    constexpr uint32_t idesc_qk = idesc_bf16_f32(BM, C::SK, false, false);
     constexpr uint32_t idesc_pv = idesc_bf16_f32(BM, D, false, true);
-    const int total = 2 * n_kv;  // scan steps of 64 keys
-    constexpr int SPL = C::QUAD ? 1 : 2;  // scan steps per K/V load unit
-    // U of step s = Q K^T over keys [64 s, +64) into buffer s % NBUF
+    const int total = n_kv * (BN / C::SK);  // scan steps of SK keys
+    constexpr int SPL = C::KVR / C::SK;     // scan steps per K/V load unit
+    // U of step s = Q K^T over keys [SK s, +SK) into buffer s % NBUF
     auto issue_u = [&](int s) -> bool {
       const int j = s / SPL, hh = s % SPL, st = j % C::STAGES, bf = s % C::NBUF;
       if (hh == 0) {
@@ -335,8 +340,8 @@ __global__ void __launch_bounds__(FwdCfg<D>::THREADS, FwdCfg<D>::CTAS)
         const uint32_t kkoff = (kk >> 2) * (C::KVR * 128) + (kk & 3) * 32;
         const uint64_t a = smem_desc_sw128(sb + C::OFF_Q + koff, 16, 1024);
         const uint64_t bd =
-            smem_desc_sw128(sb + C::OFF_K + st * C::KVT + hh * HN * 128 + kkoff, 16, 1024);
-        mma_ss_w(tmem + kSCol + bf * HN, a, bd, idesc_qk, kk > 0 ? 1u : 0u);
+            smem_desc_sw128(sb + C::OFF_K + st * C::KVT + hh * C::SK * 128 + kkoff, 16, 1024);
+        mma_ss_w(tmem + kSCol + bf * C::SK, a, bd, idesc_qk, kk > 0 ? 1u : 0u);
       }
       mma_commit_w(bar(B_S + bf));  // U ready (and every earlier z update done)
       if (hh == SPL - 1) mma_commit_w(bar(B_KE + st));  // K stage free
@@ -351,13 +356,13 @@ __global__ void __launch_bounds__(FwdCfg<D>::THREADS, FwdCfg<D>::CTAS)
       if (hh == 0 && !(ok = mbar_wait_warp(bar(B_VF + st), (j / C::STAGES) & 1, ab))) break;
       if (!(ok = mbar_wait_warp(bar(B_P + bf), (s / C::NBUF) & 1, ab))) break;
       tc_fence_after();
-      // z += P V over the step's 64 keys (A = P from TMEM as bf16 pairs in the first 32
-      // columns of the step's buffer; B = V rows, N = d contiguous)
+      // z += P V over the step's SK keys (A = P from TMEM as bf16 pairs in the first
+      // SK / 2 columns of the step's buffer; B = V rows, N = d contiguous)
 #pragma unroll
-      for (int kk = 0; kk < HN / 16; ++kk) {
+      for (int kk = 0; kk < C::SK / 16; ++kk) {
         const uint64_t bd = smem_desc_sw128(
-            sb + C::OFF_V + st * C::KVT + (hh * HN + kk * 16) * 128, C::KVR * 128, 1024);
-        mma_ts_w(tmem + C::OCOL, tmem + kSCol + bf * HN + kk * 8, bd, idesc_pv,
+            sb + C::OFF_V + st * C::KVT + (hh * C::SK + kk * 16) * 128, C::KVR * 128, 1024);
+        mma_ts_w(tmem + C::OCOL, tmem + kSCol + bf * C::SK + kk * 8, bd, idesc_pv,
                  (s > 0 || kk > 0) ? 1u : 0u);
       }
       mma_commit_w(bar(B_OD));  // z update of step s done
@@ -412,8 +417,9 @@ __global__ void __launch_bounds__(FwdCfg<D>::THREADS, FwdCfg<D>::CTAS)
       if (go) m = mn;
       return true;
     };
-    for (int s = 0; s < 2 * n_kv; ++s) {
-      const int j = s >> 1, hh = s & 1, bf = s % C::NBUF;
+    constexpr int SPT = BN / C::SK;  // scan steps per 128-key tile
+    for (int s = 0; s < n_kv * SPT; ++s) {
+      const int j = s / SPT, hh = s % SPT, bf = s % C::NBUF;
       ok = __all_sync(0xffffffffu, mbar_wait(bar(B_S + bf), (s / C::NBUF) & 1, ab));
       if (!ok) break;
       tc_fence_after();
@@ -423,21 +429,21 @@ __global__ void __launch_bounds__(FwdCfg<D>::THREADS, FwdCfg<D>::CTAS)
       // parity wait for phase s - 1 is exact (before the wait above it could still be two
       // phases short and pass at once).
       if (!(ok = rescale(m_next > m, m_next, s - 1, nullptr))) break;
-      const uint32_t ucol = trow + kSCol + bf * HN;
+      const uint32_t ucol = trow + kSCol + bf * C::SK;
       // causal: the diagonal tile masks the keys at and after the row (tl, relative to the
       // step's first key); otherwise keys at and past Tk (a ragged last tile) are masked
-      const int tl = causal ? t - hh * HN : sa.Tk - j * BN - hh * HN;
-      const bool diag = causal ? (j == qt) : (tl < HN);
+      const int tl = causal ? t - hh * C::SK : sa.Tk - j * BN - hh * C::SK;
+      const bool diag = causal ? (j == qt) : (tl < C::SK);
       float umax;
       float2 rs;
-      if constexpr (C::QUAD) {
-        // two halves of 32 keys; P of each written back into the first 16 columns of its
-        // own U columns once the half's bound is known (a jump of the second half also
-        // rescales the first half's P, already in TMEM)
+      if constexpr (C::NBUF == 1) {
+        // chunks of 32 keys; P of chunk hb written as 16 bf16 pairs to columns 16 hb ..
+        // (never ahead of the U columns still to be read) once the chunk's bound is known
+        // (a jump in a later chunk also rescales the earlier chunks' P, already in TMEM)
         rs = make_float2(0.f, 0.f);
         umax = -INFINITY;
 #pragma unroll
-        for (int hb = 0; hb < 2; ++hb) {
+        for (int hb = 0; hb < C::SK / 32; ++hb) {
           uint32_t U[32];
           tmem_ld32(ucol + hb * 32, U);
           tmem_ld_wait();
@@ -456,18 +462,18 @@ __global__ void __launch_bounds__(FwdCfg<D>::THREADS, FwdCfg<D>::CTAS)
           if (__any_sync(0xffffffffu, jump)) {
             float sc;
             if (!(ok = rescale(jump, fmaxf(mt, m_next), s - 1, &sc))) break;
-            rs = make_float2(rs.x * sc, rs.y * sc);  // the first half, at the old scale
-            if (hb == 1) {
+            rs = make_float2(rs.x * sc, rs.y * sc);  // the earlier chunks, at the old scale
+            if (hb > 0) tmem_st_wait();
+            for (int pc = 0; pc < hb; ++pc) {
               uint32_t pa[16];
-              tmem_st_wait();
-              tmem_ld16(ucol, pa);
+              tmem_ld16(ucol + pc * 16, pa);
               tmem_ld_wait();
 #pragma unroll
               for (int c = 0; c < 16; ++c) {
                 const float2 v2 = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&pa[c]));
                 pa[c] = pack_bf16x2(v2.x * sc, v2.y * sc);
               }
-              tmem_st16(ucol, pa);
+              tmem_st16(ucol + pc * 16, pa);
             }
             r = dg ? scan_p32<true>(U, th, ch, c2k, -m, mx, u_self, pk)
                    : scan_p32<false>(U, th, ch, c2k, -m, mx, u_self, pk);
@@ -478,6 +484,7 @@ __global__ void __launch_bounds__(FwdCfg<D>::THREADS, FwdCfg<D>::CTAS)
         }
         if (!ok) break;
       } else {
+        static_assert(C::SK == HN, "two buffers of 64-key steps");
         uint32_t U[HN];
         tmem_ld32(ucol, U);
         tmem_ld32(ucol + 32, U + 32);
