@@ -162,6 +162,13 @@ def _same_layout(ref: torch.Tensor, *others: torch.Tensor):
             raise ValueError("all tensors must live on the same CUDA device")
 
 
+def _like(t: torch.Tensor) -> torch.Tensor:
+    """An output with t's shape, dtype, device and strides.  The C ABI writes an output
+    with its input's element strides, which torch.empty_like does not keep for a view that
+    is not dense (e.g. a slice of a padded tensor)."""
+    return torch.empty_strided(t.size(), t.stride(), dtype=t.dtype, device=t.device)
+
+
 def _stream(stream) -> int:
     if stream is None:
         return torch.cuda.current_stream().cuda_stream
@@ -182,7 +189,7 @@ def fwd(q, k, v, lam: float, tau_s: float = 2.0, *, kernel: str = "auto", out=No
     _same_layout(q, k, v)
     B, T, H, _ = q.shape
     if out is None:
-        out = torch.empty_like(q)
+        out = _like(q)
     _same_layout(q, out)
     if logz is None:
         logz = torch.empty((B, H, T), device=q.device, dtype=torch.float32)
@@ -201,7 +208,7 @@ def fwd_flow(q, k, v, lam: float, tau_s: float = 2.0, *, kernel: str = "auto", o
     _same_layout(q, k, v)
     B, T, H, _ = q.shape
     if out is None:
-        out = torch.empty_like(q)
+        out = _like(q)
     _same_layout(q, out)
     if logz is None:
         logz = torch.empty((B, H, T), device=q.device, dtype=torch.float32)
@@ -225,7 +232,7 @@ def linear_fwd(p1, p2, v, alpha, tau_s: float = 2.0, *, kernel: str = "auto", ou
     if alpha.dtype != torch.float32 or tuple(alpha.shape) != tuple(p1.shape) or \
             tuple(alpha.stride()) != tuple(p1.stride()):
         raise ValueError("alpha must be fp32 with p1's shape and strides")
-    out = torch.empty_like(p1) if out is None else out
+    out = _like(p1) if out is None else out
     _same_layout(p1, out)
     rc = load().relation_linear_fwd_ex(_ptr(p1), _ptr(p2), _ptr(v), _ptr(alpha), _ptr(out),
                                        float(tau_s), shape_of(p1), _dtype_code(p1),
@@ -234,6 +241,16 @@ def linear_fwd(p1, p2, v, alpha, tau_s: float = 2.0, *, kernel: str = "auto", ou
     if rc != OK:
         raise RelationError(rc, "relation_linear_fwd_ex")
     return out
+
+
+def _check_summary(state, B, H, T, d, device):
+    """(m, l, z): dense fp32 [B, H, T], [B, H, T], [B, H, T, d] on `device`."""
+    m, l, z = state
+    for t, shp in ((m, (B, H, T)), (l, (B, H, T)), (z, (B, H, T, d))):
+        if tuple(t.shape) != shp or t.dtype != torch.float32 or not t.is_contiguous() or \
+                t.device != device:
+            raise ValueError("an Exchange summary is dense fp32 (m, l [B, H, T], z [B, H, T, d]) "
+                             "on the operands' device")
 
 
 def fwd_state(q, k, v, causal: bool, *, out=None, dev_status=None, stream=None):
@@ -249,6 +266,7 @@ def fwd_state(q, k, v, causal: bool, *, out=None, dev_status=None, stream=None):
                torch.empty((B, H, Tq), dtype=torch.float32, device=q.device),
                torch.empty((B, H, Tq, d), dtype=torch.float32, device=q.device))
     m, l, z = out
+    _check_summary(out, B, H, Tq, d, q.device)
     rc = load().relation_fwd_state(_ptr(q), _ptr(k), _ptr(v), _ptr(m), _ptr(l), _ptr(z),
                                    shape_of(q), shape_of(k), int(bool(causal)), _dtype_code(q),
                                    _ptr(dev_status), ctypes.c_void_p(_stream(stream)))
@@ -263,6 +281,8 @@ def state_merge(state, other, *, stream=None):
     m, l, z = state
     m2, l2, z2 = other
     B, H, T, d = z.shape
+    _check_summary(state, B, H, T, d, z.device)
+    _check_summary(other, B, H, T, d, z.device)
     rc = load().relation_state_merge(_ptr(m), _ptr(l), _ptr(z), _ptr(m2), _ptr(l2), _ptr(z2),
                                      Shape(B, T, H, d, T * H * d, H * d, d),
                                      ctypes.c_void_p(_stream(stream)))
@@ -278,8 +298,12 @@ def state_finish(q, k, v, state, lam: float, tau_s: float = 2.0, pos0: int = 0, 
     _same_layout(q, k, v)
     m, l, z = state
     B, T, H, d = q.shape
-    out = torch.empty_like(q) if out is None else out
+    out = _like(q) if out is None else out
+    _same_layout(q, out)
     logz = torch.empty((B, H, T), dtype=torch.float32, device=q.device) if logz is None else logz
+    _check_summary(state, B, H, T, d, q.device)
+    if tuple(logz.shape) != (B, H, T) or logz.dtype != torch.float32 or not logz.is_contiguous():
+        raise ValueError("logz must be a dense fp32 [B, H, T] tensor")
     rc = load().relation_state_finish(_ptr(q), _ptr(k), _ptr(v), _ptr(m), _ptr(l), _ptr(z),
                                       _ptr(out), _ptr(logz), _ptr(self_flow), float(lam),
                                       float(tau_s), int(pos0), shape_of(q), _dtype_code(q),
@@ -302,7 +326,7 @@ def linear_fwd_ws(p1, p2, v, alpha, tau_s: float = 2.0, *, workspace=None, out=N
     if alpha.dtype != torch.float32 or tuple(alpha.shape) != tuple(p1.shape) or \
             tuple(alpha.stride()) != tuple(p1.stride()):
         raise ValueError("alpha must be fp32 with p1's shape and strides")
-    out = torch.empty_like(p1) if out is None else out
+    out = _like(p1) if out is None else out
     _same_layout(p1, out)
     need = linear_fwd_workspace_size(p1)
     if workspace is None:
@@ -332,8 +356,8 @@ def linear_bwd(p1, p2, v, alpha, dy, tau_s: float = 2.0, *, kernel: str = "auto"
     if alpha.dtype != torch.float32 or tuple(alpha.shape) != tuple(p1.shape) or \
             tuple(alpha.stride()) != tuple(p1.stride()):
         raise ValueError("alpha must be fp32 with p1's shape and strides")
-    dp1, dp2, dv = torch.empty_like(p1), torch.empty_like(p1), torch.empty_like(p1)
-    dalpha = torch.empty_like(alpha)
+    dp1, dp2, dv = _like(p1), _like(p1), _like(p1)
+    dalpha = _like(alpha)
     need = linear_bwd_workspace_size(p1, kernel)
     if workspace is None:
         workspace = torch.empty(max(need, 16), device=p1.device, dtype=torch.uint8)
@@ -362,8 +386,8 @@ def layer_prep(p1, p2, info, theta, pairing: int = 0, rope_base: float = 1.0e4, 
     RoPE(p2), Givens(info)) for [B, T, H, d] inputs of one layout, theta fp32 [H/2]."""
     _same_layout(p1, p2, info)
     theta, pairing, rope_base = _layer_args(theta, pairing, rope_base, p1)
-    q, k, v = out if out is not None else (torch.empty_like(p1), torch.empty_like(p1),
-                                           torch.empty_like(p1))
+    q, k, v = out if out is not None else (_like(p1), _like(p1),
+                                           _like(p1))
     _same_layout(p1, q, k, v)
     rc = load().relation_layer_prep(_ptr(p1), _ptr(p2), _ptr(info), _ptr(theta), pairing,
                                     rope_base, _ptr(q), _ptr(k), _ptr(v), shape_of(p1),
@@ -383,8 +407,8 @@ def layer_grad(dq, dk, dv, info, theta, pairing: int = 0, rope_base: float = 1.0
     """Gradient of layer_prep: returns (dp1, dp2, dinfo, dtheta)."""
     _same_layout(dq, dk, dv, info)
     theta, pairing, rope_base = _layer_args(theta, pairing, rope_base, dq)
-    dp1, dp2, dinfo = torch.empty_like(dq), torch.empty_like(dq), torch.empty_like(dq)
-    dtheta = torch.empty_like(theta)
+    dp1, dp2, dinfo = _like(dq), _like(dq), _like(dq)
+    dtheta = _like(theta)
     need = layer_grad_workspace_size(dq)
     if workspace is None:
         workspace = torch.empty(max(need, 16), device=dq.device, dtype=torch.uint8)
@@ -414,7 +438,7 @@ def decode(q, k_cache, v_cache, lengths, lam: float, tau_s: float = 2.0, *, out=
         raise ValueError("q must be [B, H, d] with d contiguous, of the cache's dtype")
     if lengths.dtype != torch.int32 or lengths.numel() != B or not lengths.is_contiguous():
         raise ValueError("lengths must be a contiguous int32 tensor of B entries")
-    out = torch.empty_like(q) if out is None else out
+    out = _like(q) if out is None else out
     if tuple(out.stride()) != tuple(q.stride()):
         raise ValueError("out must have q's layout")
     if logz is None:
@@ -441,9 +465,9 @@ def bwd(q, k, v, o, dout, logz, lam: float, tau_s: float = 2.0, *, kernel: str =
     """Backward.  Returns (dQ, dK, dV, dlambda) with dlambda a 1-element fp32 device tensor.
     ``stages`` selects a subset of the three backward stages (see relation_bwd_stages)."""
     _same_layout(q, k, v, o, dout)
-    dq = torch.empty_like(q) if dq is None else dq
-    dk = torch.empty_like(q) if dk is None else dk
-    dv = torch.empty_like(q) if dv is None else dv
+    dq = _like(q) if dq is None else dq
+    dk = _like(q) if dk is None else dk
+    dv = _like(q) if dv is None else dv
     _same_layout(q, dq, dk, dv)
     if dlambda is None:
         dlambda = torch.empty(1, device=q.device, dtype=torch.float32)
@@ -506,6 +530,6 @@ class RelationFunction(torch.autograd.Function):
     def backward(ctx, dy):
         q, k, v, y, logz = ctx.saved_tensors
         if dy.stride() != q.stride() or dy.dtype != q.dtype:
-            dy = torch.empty_like(q).copy_(dy)
+            dy = _like(q).copy_(dy)
         dq, dk, dv, dl = bwd(q, k, v, y, dy, logz, ctx.lam, ctx.tau_s, kernel=ctx.kernel)
         return dq, dk, dv, dl.reshape(()).to(torch.float32), None, None

@@ -120,3 +120,27 @@ def test_state_against_the_oracle_rows():
         ry, rlz = oracle.fwd(pu.head(q, 0, h), pu.head(k, 0, h), pu.head(v, 0, h), lam, tau)
         pu.check(f"rows 100.. h={h}", y[0, :, h].float().cpu().numpy(), ry[100:], "bf16", "out")
         pu.check_logz(f"logZ h={h}", lz[0, h].cpu().numpy(), rlz[100:], "bf16")
+
+
+def test_sharded_forward_on_bhtd_storage():
+    """Shards of [B, H, T, d] storage (permuted views: every stride differs from the dense
+    layout) give the dense layout's results."""
+    w = workloads.custom(2, 2, 300, 64, "bf16")
+    q, k, v, _ = workloads.make_inputs(w, seed=5)
+    lam, tau = workloads.LAMBDA_INIT, workloads.TAU_S
+    dev = torch.device("cuda:0")
+
+    def bhtd(t):
+        return t.permute(0, 2, 1, 3).contiguous().to(dev).permute(0, 2, 1, 3)
+
+    def shards(qq, kk, vv):
+        a, b = 0, 130
+        st = binding.fwd_state(qq[:, b:], kk[:, b:], vv[:, b:], causal=True)
+        binding.state_merge(st, binding.fwd_state(qq[:, b:], kk[:, a:b], vv[:, a:b], causal=False))
+        return binding.state_finish(qq[:, b:], kk[:, b:], vv[:, b:], st, lam, tau, pos0=b)
+
+    y0, l0 = shards(*(t.to(dev) for t in (q, k, v)))
+    y1, l1 = shards(*(bhtd(t) for t in (q, k, v)))
+    torch.cuda.synchronize()
+    assert torch.equal(y0.contiguous(), y1.contiguous())
+    assert torch.equal(l0, l1)

@@ -256,3 +256,35 @@ def test_linear_backward_chunked_reports_decay_beyond_its_range():
     assert int(status.item()) == binding.ERR_UNSUPPORTED
     for t in g:
         assert torch.isfinite(t.float()).all()
+
+
+def test_linear_backward_chunked_bhtd_layout_and_stride_fallback():
+    """The chunked backward on [B, H, T, d] storage (a permuted view) gives the results of
+    the [B, T, H, d] layout bit for bit; a row stride that is a multiple of 4 but not of 8
+    elements leaves the chunked kernel's reach, and AUTO then runs the recurrence (still
+    against the oracle)."""
+    w = workloads.custom(2, 3, 200, 64, "bf16")
+    p1, p2, v, alpha, dy = workloads.make_linear_inputs(w, seed=12)
+    dev = torch.device("cuda:0")
+
+    def bhtd(t):
+        return t.permute(0, 2, 1, 3).contiguous().to(dev).permute(0, 2, 1, 3)
+
+    g0 = binding.linear_bwd(*(t.to(dev) for t in (p1, p2, v, alpha, dy)), kernel="tcgen05")
+    g1 = binding.linear_bwd(*(bhtd(t) for t in (p1, p2, v, alpha, dy)), kernel="tcgen05")
+    torch.cuda.synchronize()
+    for a, b in zip(g0, g1):
+        assert torch.equal(a.contiguous(), b.contiguous())
+
+    def padded(t):  # d padded to 68: element strides (T H 68, H 68, 68), multiples of 4 only
+        pad = torch.zeros(t.shape[:-1] + (68,), dtype=t.dtype)
+        pad[..., :64] = t
+        return pad.to(dev)[..., :64]
+
+    args = [padded(t) for t in (p1, p2, v, alpha, dy)]
+    assert binding.linear_bwd_workspace_size(args[0], "tcgen05") == 0
+    status = torch.zeros(1, dtype=torch.int32, device=dev)
+    g = binding.linear_bwd(*args, dev_status=status)
+    torch.cuda.synchronize()
+    assert int(status.item()) == 0
+    _check_grads("linear bwd strided", g, p1, p2, v, alpha, dy, [(0, 0), (1, 2)])
