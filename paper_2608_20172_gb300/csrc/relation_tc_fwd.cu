@@ -56,10 +56,10 @@ template <int D>
 struct FwdCfg {
   static constexpr bool QUAD = D == 64;
   static constexpr bool WIDE = false;
-  static constexpr int SK = WIDE ? 128 : HN;     // keys per scan step
+  static constexpr int SK = WIDE ? 128 : (QUAD ? 32 : HN);  // keys per scan step
   static constexpr int CTAS = QUAD ? 4 : 2;      // CTAs per SM
   static constexpr int TMEM_COLS = QUAD ? 128 : 256;
-  static constexpr int NBUF = (QUAD || WIDE) ? 1 : 2;  // U/P buffers
+  static constexpr int NBUF = WIDE ? 1 : 2;      // U/P buffers
   static constexpr int OCOL = NBUF * SK;         // z accumulator
   static constexpr int W_TMA = 4, W_MMA = 5;
   static constexpr int THREADS = 192;
@@ -436,7 +436,7 @@ __global__ void __launch_bounds__(FwdCfg<D>::THREADS, FwdCfg<D>::CTAS)
       const bool diag = causal ? (j == qt) : (tl < C::SK);
       float umax;
       float2 rs;
-      if constexpr (C::NBUF == 1) {
+      if constexpr (C::NBUF == 1 || C::SK != HN) {
         // chunks of 32 keys; P of chunk hb written as 16 bf16 pairs to columns 16 hb ..
         // (never ahead of the U columns still to be read) once the chunk's bound is known
         // (a jump in a later chunk also rescales the earlier chunks' P, already in TMEM)
@@ -484,7 +484,7 @@ __global__ void __launch_bounds__(FwdCfg<D>::THREADS, FwdCfg<D>::CTAS)
         }
         if (!ok) break;
       } else {
-        static_assert(C::SK == HN, "two buffers of 64-key steps");
+        static_assert(C::SK == HN, "64-key steps in registers");
         uint32_t U[HN];
         tmem_ld32(ucol, U);
         tmem_ld32(ucol + 32, U + 32);
