@@ -1,26 +1,26 @@
 // relation_tc_fwd.cu -- tcgen05 / TMA / TMEM forward of FlashRelation (bf16, d_h 64 or 128).
 //
 // One CTA owns a tile of BM = 128 query rows of one head and scans the key/value tiles
-// j0 = 0, 128, ... up to and including its diagonal tile (Sec. 5.1, App. A.3).  Two CTAs
-// share an SM (each allocates 256 TMEM columns), so the tensor core of one CTA overlaps
-// the elementwise work of the other.  CTAs take the heaviest query tiles first, heads in
-// groups (grouped_unit), so that the K/V rows in use stay in L2.
+// j0 = 0, 128, ... up to and including its diagonal tile (Sec. 5.1, App. A.3).  Several
+// CTAs share an SM (d_h = 128: two of 256 TMEM columns; d_h = 64: four of 128), so the
+// tensor core of one CTA overlaps the elementwise work of the others.  CTAs take the
+// heaviest query tiles first, heads in groups (grouped_unit), so that the K/V rows in use
+// stay in L2.
 //
 // Warp roles (192 threads):
 //   warps 0-3  Exchange scan + epilogue: thread t owns query row q0 + t (TMEM lane t).
-//   warp  4    TMA producer: Q tile once, then K and V tiles through a ring of stages.
+//   warp  4    TMA producer: Q tile once, then K and V through a ring of stages.
 //   warp  5    TMEM allocator and MMA issuer (one elected thread).
-// Per key tile j:
-// The scan advances 64 keys per step through two TMEM buffers, so the MMAs of one step
-// (U of step s + 2, z += P V of step s) overlap the elementwise work of the next.  Step s:
-//   MMA   U = Q K^T over 64 keys                 -> TMEM columns [64 b, 64 b + 64), b = s & 1
-//   scan  E = SiLU(U / sqrt(d)) for keys < row (Self excluded); running maximum m (kept
-//         as an upper bound of max E, max(U, 0) / sqrt(d), rescaling z only when it grows
-//         by > 2^8), row sum
-//         l += sum exp(E - m); P = exp(E - m) as bf16 written back into the buffer's
-//         first 32 columns (two per 32-bit column); the diagonal tile also yields
+// The scan advances SK keys per step (64 at d_h = 128, 32 at d_h = 64) through two TMEM
+// buffers, so the MMAs of one step (U of step s + 2, z += P V of step s) overlap the
+// elementwise work of the next.  Step s:
+//   MMA   U = Q K^T over SK keys                -> TMEM columns [SK b, SK b + SK), b = s & 1
+//   scan  E = SiLU(U / sqrt(d)) for keys < row (Self excluded); P = exp(E - m) at the row's
+//         scale m (an upper bound of max E, max(U, 0) / sqrt(d), raised a step late when
+//         it grew by > 2^8), row sum l += sum P; P as bf16 written back into the buffer's
+//         first SK / 2 columns (two per 32-bit column); the diagonal tile also yields
 //         S_i = sigmoid(U_ii / (sqrt(d) tau_S)).
-//   MMA   z += P V  (A operand P read from TMEM)  -> TMEM columns [128, 128 + d)
+//   MMA   z += P V  (A operand P read from TMEM)  -> TMEM columns [2 SK, 2 SK + d)
 // Epilogue (App. A.3.3-A.3.5): L^E = m + log l, A = L^E - lambda log i,
 //   g = sigmoid(A - S), Y = (1 - g) v_i + g z / l, logZ = logaddexp(S, A); row 1 has an
 //   empty history: g = 0, Y = v_1, logZ = S_1 (App. A.1.8).
@@ -44,8 +44,8 @@ constexpr float kRescaleLog2 = 8.0f;  // rescale z only when the max grows by > 
 constexpr float kStaleLog2 = 32.0f;   // a step's P may reach 2^32 at the previous scale
 
 // d_h = 64 (QUAD): four CTAs per SM, so that each SM sub-partition runs four scan warps:
-//   TMEM 128 columns (one U/P buffer of 64 + z 64), K and V in 64-key halves through two
-//   stages each (50 KB of shared memory), steps of 64 keys.
+//   TMEM 128 columns (two U/P buffers of 32-key steps + z 64), K and V in 64-key halves
+//   through two stages each (50 KB of shared memory).
 // d_h = 128: two CTAs per SM, two U/P buffers of 64-key steps (so that the MMAs of one step
 //   overlap the scan of the next) + z 128 = 256 TMEM columns, 128-key K/V tiles through one
 //   stage.  (WIDE, steps of a whole 128-key tile in one buffer of 128 columns so that
@@ -56,10 +56,14 @@ template <int D>
 struct FwdCfg {
   static constexpr bool QUAD = D == 64;
   static constexpr bool WIDE = false;
-  static constexpr int SK = WIDE ? 128 : (QUAD ? 32 : HN);  // keys per scan step
+  // DEEP: four buffers of 32-key steps (U three steps ahead) in the same 256 columns;
+  // measured slower at d_h = 128 (long forward 1.97 -> 2.35 ms: U = Q K^T at N = 32 reads
+  // the Q tile from shared memory twice as often per key)
+  static constexpr bool DEEP = false;
+  static constexpr int SK = WIDE ? 128 : ((QUAD || DEEP) ? 32 : HN);  // keys per scan step
   static constexpr int CTAS = QUAD ? 4 : 2;      // CTAs per SM
   static constexpr int TMEM_COLS = QUAD ? 128 : 256;
-  static constexpr int NBUF = WIDE ? 1 : 2;      // U/P buffers
+  static constexpr int NBUF = WIDE ? 1 : (DEEP ? 4 : 2);  // U/P buffers
   static constexpr int OCOL = NBUF * SK;         // z accumulator
   static constexpr int W_TMA = 4, W_MMA = 5;
   static constexpr int THREADS = 192;
@@ -79,7 +83,11 @@ struct FwdCfg {
 
 // mbarrier slots
 enum : int {
-  B_Q = 0, B_KF = 1, B_KE = 3, B_VF = 5, B_VE = 7, B_S = 9, B_P = 11, B_O = 13, B_OD = 14
+  // per stage (2): B_KF .. B_VE; per U/P buffer (up to 4): B_S, B_P and B_OD (the z update
+  // of a step of that buffer done, so that a wait for step s - 1's update is exact for any
+  // number of buffers: U of step s implies the buffer's previous update)
+  B_Q = 0, B_KF = 1, B_KE = 3, B_VF = 5, B_VE = 7, B_S = 9, B_P = 13, B_OD = 17, B_O = 21,
+  NBAR_FWD = 22
 };
 
 // Bounded wait used while draining at teardown: never raises, just gives up.
@@ -243,8 +251,9 @@ __global__ void __launch_bounds__(FwdCfg<D>::THREADS, FwdCfg<D>::CTAS)
       (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
   const uint32_t sb = smem_u32(smem);
   auto bar = [&](int i) -> uint32_t { return sb + C::OFF_BAR + 8u * (uint32_t)i; };
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(smem + C::OFF_BAR + 128);
-  volatile int* abort_flag = reinterpret_cast<volatile int*>(smem + C::OFF_BAR + 136);
+  static_assert(NBAR_FWD * 8 <= 192, "barrier slots");
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(smem + C::OFF_BAR + 192);
+  volatile int* abort_flag = reinterpret_cast<volatile int*>(smem + C::OFF_BAR + 200);
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int BH = p.B * p.H;
@@ -264,12 +273,12 @@ __global__ void __launch_bounds__(FwdCfg<D>::THREADS, FwdCfg<D>::CTAS)
       mbar_init(bar(B_VF + s), 1);
       mbar_init(bar(B_VE + s), 1);
     }
-    for (int bb = 0; bb < 2; ++bb) {
+    for (int bb = 0; bb < C::NBUF; ++bb) {
       mbar_init(bar(B_S + bb), 1);
       mbar_init(bar(B_P + bb), 128);
+      mbar_init(bar(B_OD + bb), 1);
     }
     mbar_init(bar(B_O), 1);
-    mbar_init(bar(B_OD), 1);
     *abort_flag = 0;
     fence_mbar_init();
   }
@@ -349,8 +358,7 @@ __global__ void __launch_bounds__(FwdCfg<D>::THREADS, FwdCfg<D>::CTAS)
     };
     bool ok = mbar_wait_warp(bar(B_Q), 0, ab);
     tc_fence_after();
-    if (ok) ok = issue_u(0);
-    if (ok && total > 1 && C::NBUF == 2) ok = issue_u(1);
+    for (int s0 = 0; ok && s0 < C::NBUF && s0 < total; ++s0) ok = issue_u(s0);
     for (int s = 0; ok && s < total; ++s) {
       const int j = s / SPL, hh = s % SPL, st = j % C::STAGES, bf = s % C::NBUF;
       if (hh == 0 && !(ok = mbar_wait_warp(bar(B_VF + st), (j / C::STAGES) & 1, ab))) break;
@@ -365,7 +373,7 @@ __global__ void __launch_bounds__(FwdCfg<D>::THREADS, FwdCfg<D>::CTAS)
         mma_ts_w(tmem + C::OCOL, tmem + kSCol + bf * C::SK + kk * 8, bd, idesc_pv,
                  (s > 0 || kk > 0) ? 1u : 0u);
       }
-      mma_commit_w(bar(B_OD));  // z update of step s done
+      mma_commit_w(bar(B_OD + bf));  // z update of step s done
       if (hh == SPL - 1) mma_commit_w(bar(B_VE + st));  // V stage free
       // the next U into the buffer whose P was read above (tcgen05 MMAs run in order)
       if (s + C::NBUF < total && !(ok = issue_u(s + C::NBUF))) break;
@@ -400,7 +408,9 @@ __global__ void __launch_bounds__(FwdCfg<D>::THREADS, FwdCfg<D>::CTAS)
       if (scp) *scp = sc;
       if (!__any_sync(0xffffffffu, go)) return true;
       if (s_done >= 0) {
-        if (!__all_sync(0xffffffffu, mbar_wait(bar(B_OD), s_done & 1, ab))) return false;
+        if (!__all_sync(0xffffffffu, mbar_wait(bar(B_OD + s_done % C::NBUF),
+                                                (s_done / C::NBUF) & 1, ab)))
+          return false;
         tc_fence_after();
 #pragma unroll
         for (int c0 = 0; c0 < D; c0 += 32) {

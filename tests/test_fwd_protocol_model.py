@@ -11,11 +11,13 @@ import pytest
 from tests.test_bwd_protocol_model import Ambiguous, Barriers
 
 
-# Layouts of the kernel (FwdCfg): U/P buffers, 64-key scan steps per K/V load unit, stages.
+# Layouts of the kernel (FwdCfg): U/P buffers, scan steps per K/V load unit, stages, scan
+# steps per 128-key tile.
 LAYOUTS = {
-    "two buffers, one stage (d_h = 128)": (2, 2, 1),
-    "two buffers, two stages": (2, 2, 2),
-    "one buffer, 64-key units, two stages (d_h = 64, four CTAs per SM)": (1, 1, 2),
+    "two buffers of 64 keys, one stage (d_h = 128)": (2, 2, 1, 2),
+    "two buffers of 32 keys, 64-key units, two stages (d_h = 64)": (2, 2, 2, 4),
+    "one buffer of 64 keys, two stages": (1, 1, 2, 2),
+    "four buffers of 32 keys, one stage": (4, 4, 1, 4),
 }
 
 
@@ -31,7 +33,7 @@ def tma(n_ld, stages):
         yield ("arrive", f"VF{s}")
 
 
-def mma(total, spl, nbuf, stages):
+def mma(total, spl, nbuf, stages, shared_od=False):
     def issue_u(s):
         j, hh = s // spl, s % spl
         st, bf = j % stages, s % nbuf
@@ -42,16 +44,15 @@ def mma(total, spl, nbuf, stages):
             yield ("arrive", f"KE{st}")
 
     yield ("wait", "Q", 0)
-    yield from issue_u(0)
-    if total > 1 and nbuf == 2:
-        yield from issue_u(1)
+    for s0 in range(min(nbuf, total)):  # every buffer's first step ahead
+        yield from issue_u(s0)
     for s in range(total):
         j, hh = s // spl, s % spl
         st, bf = j % stages, s % nbuf
         if hh == 0:
             yield ("wait", f"VF{st}", j // stages)
         yield ("wait", f"P{bf}", s // nbuf)
-        yield ("arrive", "OD")
+        yield ("arrive", "OD" if shared_od else f"OD{bf}")
         if hh == spl - 1:
             yield ("arrive", f"VE{st}")
         if s + nbuf < total:
@@ -59,32 +60,35 @@ def mma(total, spl, nbuf, stages):
     yield ("arrive", "O")
 
 
-def scan(total, nbuf, rescale_rng, rescale_first=False):
+def scan(total, nbuf, rescale_rng, rescale_first=False, shared_od=False):
     """The scan warps' waits: U of step s, then (data-dependent) the z update of step
     s - 1 before a rescale: the scale raised at step s - 1, applied at step s, and the
     rarer redo of a step whose bound jumped.  rescale_first puts the first of them
     before the wait for U (an order the kernel must not use)."""
+    def od(k):  # the z update of step k: that step's buffer's barrier (or one shared)
+        return ("wait", "OD", k) if shared_od else ("wait", f"OD{k % nbuf}", k // nbuf)
+
     for s in range(total):
         bf = s % nbuf
         pending = s > 0 and rescale_rng.random() < 0.3
         if rescale_first and pending:
-            yield ("wait", "OD", s - 1)
+            yield od(s - 1)
         yield ("wait", f"S{bf}", s // nbuf)
         if pending and not rescale_first:
-            yield ("wait", "OD", s - 1)
+            yield od(s - 1)
         if s > 0 and rescale_rng.random() < 0.1:  # the step's bound jumped: redo it
-            yield ("wait", "OD", s - 1)
+            yield od(s - 1)
         yield ("arrive", f"P{bf}")
     yield ("wait", "O", 0)
 
 
-def run(n_kv, layout, seed, rescale_first=False):
-    nbuf, spl, stages = LAYOUTS[layout]
-    total = 2 * n_kv
+def run(n_kv, layout, seed, rescale_first=False, shared_od=False):
+    nbuf, spl, stages, spt = LAYOUTS[layout]
+    total = spt * n_kv
     rng = random.Random(seed)
     bars = Barriers()
-    roles = {"tma": tma(total // spl, stages), "mma": mma(total, spl, nbuf, stages),
-             "scan": scan(total, nbuf, random.Random(seed + 1000), rescale_first)}
+    roles = {"tma": tma(total // spl, stages), "mma": mma(total, spl, nbuf, stages, shared_od),
+             "scan": scan(total, nbuf, random.Random(seed + 1000), rescale_first, shared_od)}
     pending = {name: next(gen, None) for name, gen in roles.items()}
     while any(ev is not None for ev in pending.values()):
         runnable = [n for n, ev in pending.items()
@@ -106,13 +110,19 @@ def test_forward_protocol(n_kv, layout):
 
 
 def test_rescale_wait_before_the_step_is_caught():
-    """Waiting for the z update of step s - 1 before U of step s can meet the barrier one
-    phase short, where its parity test passes at once (z rescaled under an update still in
-    flight): the model flags that order."""
+    """With one z-update barrier shared by the buffers, waiting for the update of step
+    s - 1 before U of step s can meet the barrier one phase short, where its parity test
+    passes at once (z rescaled under an update still in flight): the model flags that
+    order.  With a barrier per buffer (the kernel), U of step s - 1 already implies the
+    buffer's previous update, so the wait is exact in either order."""
+    layout = "two buffers of 64 keys, one stage (d_h = 128)"
     caught = 0
     for seed in range(200):
         try:
-            run(16, "two buffers, one stage (d_h = 128)", seed, rescale_first=True)
+            run(16, layout, seed, rescale_first=True, shared_od=True)
         except Ambiguous:
             caught += 1
     assert caught > 0
+    for lay in LAYOUTS:
+        for seed in range(40):
+            run(16, lay, seed, rescale_first=True)
