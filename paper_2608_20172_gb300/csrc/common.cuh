@@ -225,6 +225,18 @@ __device__ __forceinline__ void mma_ts_w(uint32_t d_tmem, uint32_t a_tmem, uint6
       "r"(a_tmem), "l"(b_desc), "r"(idesc), "r"(accumulate)
       : "memory");
 }
+// Copy of a 128-row x 32-byte slice of a shared-memory matrix (the descriptor's layout,
+// e.g. one K step of a 128-byte-swizzled K-major tile) into TMEM lanes 0-127, 8 columns:
+// the A-operand layout of tcgen05.mma with A in TMEM.  Issued from warp-uniform code by one
+// elected lane, in order with the MMAs of the same thread.
+__device__ __forceinline__ void tmem_cp_w(uint32_t taddr, uint64_t s_desc) {
+  asm volatile(
+      "{\n\t.reg .pred e;\n\t"
+      "elect.sync _|e, 0xffffffff;\n\t"
+      "@e tcgen05.cp.cta_group::1.128x256b [%0], %1;\n\t}" ::"r"(taddr),
+      "l"(s_desc)
+      : "memory");
+}
 __device__ __forceinline__ void mma_commit_w(uint32_t bar) {
   asm volatile(
       "{\n\t.reg .pred e;\n\t"

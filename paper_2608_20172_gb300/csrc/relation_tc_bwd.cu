@@ -101,6 +101,11 @@ struct Cfg {
   static constexpr int COL_DK = NBUF * 2 * QW;  // 256
   static constexpr int COL_DV = COL_DK + D;     // 320 / 384
   static constexpr int COL_DQ = 384;            // d_h = 64 only
+  // d_h = 64: the unit's K and V tiles also in TMEM (A operands of U^T = K Q^T and
+  // dP^T = V dO^T, which then read only Q / dO from shared memory: an SS MMA at N = 64
+  // reads 6 KB of operands in 48 cycles of shared-memory bandwidth against 32 of math)
+  static constexpr int COL_KT = 448, COL_VT = 480;
+  static_assert(HALF || COL_VT + D / 2 <= 512, "TMEM");
   __host__ __device__ static constexpr int col_u(int b) { return b * 2 * QW; }
   __host__ __device__ static constexpr int col_g(int b) { return b * 2 * QW + QW; }
   // Q / dO stage unit of a step: the step itself (d_h = 128) or its query tile
@@ -374,9 +379,12 @@ __global__ void __launch_bounds__(Cfg<D>::THREADS, 1)
       for (int kk = 0; kk < D / 16; ++kk) {
         const uint32_t kof = (kk >> 2) * 16384 + (kk & 3) * 32;
         const uint32_t qof = (kk >> 2) * C::KBQ + (kk & 3) * 32;
-        mma_ss_w(tmem + C::col_u(bb), smem_desc_sw128(x.ks + kof, 16, 1024),
-                 smem_desc_sw128(sb + C::OFF_Q + st * C::QSZ + rows + qof, 16, 1024), id_s,
-                 kk > 0 ? 1u : 0u);
+        const uint64_t bq = smem_desc_sw128(sb + C::OFF_Q + st * C::QSZ + rows + qof, 16, 1024);
+        if (C::HALF)
+          mma_ss_w(tmem + C::col_u(bb), smem_desc_sw128(x.ks + kof, 16, 1024), bq, id_s,
+                   kk > 0 ? 1u : 0u);
+        else
+          mma_ts_w(tmem + C::col_u(bb), tmem + C::COL_KT + kk * 8, bq, id_s, kk > 0 ? 1u : 0u);
       }
       return true;
     };
@@ -389,11 +397,25 @@ __global__ void __launch_bounds__(Cfg<D>::THREADS, 1)
       for (int kk = 0; kk < D / 16; ++kk) {
         const uint32_t kof = (kk >> 2) * 16384 + (kk & 3) * 32;
         const uint32_t qof = (kk >> 2) * C::KBQ + (kk & 3) * 32;
-        mma_ss_w(tmem + C::col_g(bb), smem_desc_sw128(x.vs + kof, 16, 1024),
-                 smem_desc_sw128(sb + C::OFF_DO + st * C::QSZ + rows + qof, 16, 1024), id_s,
-                 kk > 0 ? 1u : 0u);
+        const uint64_t bg = smem_desc_sw128(sb + C::OFF_DO + st * C::QSZ + rows + qof, 16, 1024);
+        if (C::HALF)
+          mma_ss_w(tmem + C::col_g(bb), smem_desc_sw128(x.vs + kof, 16, 1024), bg, id_s,
+                   kk > 0 ? 1u : 0u);
+        else
+          mma_ts_w(tmem + C::col_g(bb), tmem + C::COL_VT + kk * 8, bg, id_s, kk > 0 ? 1u : 0u);
       }
       mma_commit_w(bar(B_S + bb));
+    };
+    // d_h = 64: the unit's K and V tiles into TMEM (in order after every earlier MMA, so the
+    // previous unit's products have read the old ones)
+    auto load_kv_tmem = [&](const Ctx& x) {
+      if (!C::HALF) {
+#pragma unroll
+        for (int kk = 0; kk < D / 16; ++kk) {
+          tmem_cp_w(tmem + C::COL_KT + kk * 8, smem_desc_sw128(x.ks + kk * 32, 16, 1024));
+          tmem_cp_w(tmem + C::COL_VT + kk * 8, smem_desc_sw128(x.vs + kk * 32, 16, 1024));
+        }
+      }
     };
     int ul = 0, gs0 = 0, gq0 = 0, gt0 = 0;
     int pre = 0;  // steps of the current unit issued ahead by the previous unit
@@ -404,7 +426,11 @@ __global__ void __launch_bounds__(Cfg<D>::THREADS, 1)
       const int kvb = ul % C::NKV;
       const Ctx x = ctx_of(ul, gs0, gq0);
       const uint32_t ks = x.ks;
-      if (pre == 0 && !(ok = mbar_wait_warp(bar(kv_full(kvb)), (ul / C::NKV) & 1, ab))) break;
+      if (pre == 0) {
+        if (!(ok = mbar_wait_warp(bar(kv_full(kvb)), (ul / C::NKV) & 1, ab))) break;
+        tc_fence_after();
+        load_kv_tmem(x);
+      }
       // d_h = 64: U^T / dP^T of step sn may be issued once its buffer is free (step
       // sn - NBUF done) and once the GEMM that releases the Q/dO stage it loads into has
       // been issued: waiting for that stage's load earlier would deadlock.
@@ -453,6 +479,8 @@ __global__ void __launch_bounds__(Cfg<D>::THREADS, 1)
             if (!(ok = mbar_wait_warp(bar(kv_full((ul + 1) % C::NKV)), ((ul + 1) / C::NKV) & 1, ab)))
               break;
             const Ctx xn = ctx_of(ul + 1, gs0 + total, gq0 + U.n_units);
+            tc_fence_after();
+            load_kv_tmem(xn);
             while (ok && pre < N.total && pre < C::NBUF) {
               ok = issue_u(xn, pre);
               if (ok) issue_dp(xn, pre);
