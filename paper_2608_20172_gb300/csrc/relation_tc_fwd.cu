@@ -38,8 +38,8 @@ namespace tc {
 
 constexpr int BM = 128;        // query rows per CTA
 constexpr int BN = 128;        // keys per K/V tile (TMA granularity)
-constexpr int HN = 64;         // keys per scan step: two steps per K/V tile
-constexpr int kSCol = 0;       // U/P buffer b at kSCol + 64 b
+constexpr int HN = 64;         // half a K/V tile: the register scan's step, the d_h = 64 load
+constexpr int kSCol = 0;       // U/P buffer b at kSCol + SK b
 constexpr float kRescaleLog2 = 8.0f;  // rescale z only when the max grows by > 2^8
 constexpr float kStaleLog2 = 32.0f;   // a step's P may reach 2^32 at the previous scale
 

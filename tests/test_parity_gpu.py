@@ -207,6 +207,34 @@ def test_deterministic_repeat():
     pu.check("dQ repeat", a["dQ"].numpy(), b["dQ"].numpy(), "bf16", "grad")
 
 
+@pytest.mark.parametrize("d,T", [(64, 700), (128, 333), (48, 257)])
+def test_staged_backward_and_workspace_reuse(d, T):
+    """The backward run stage by stage (row pass, tiles, finalisation) into outputs filled
+    with NaN equals the one-call backward (every real element written), and a second call
+    on the same workspace repeats dK, dV and dlambda bit for bit."""
+    w = workloads.custom(2, 3, T, d, "bf16")
+    q, k, v, do = workloads.make_inputs(w, seed=71 + d)
+    dev = torch.device("cuda:0")
+    qd, kd, vd, dod = (t.to(dev) for t in (q, k, v, do))
+    y, lz = binding.fwd(qd, kd, vd, LAM, kernel="tcgen05")
+    ws = torch.empty(binding.workspace_size(qd), device=dev, dtype=torch.uint8)
+    one = [t.clone() for t in binding.bwd(qd, kd, vd, y, dod, lz, LAM, kernel="tcgen05",
+                                          workspace=ws)]
+    outs = [torch.full_like(qd, float("nan")) for _ in range(3)]
+    dl = torch.full((1,), float("nan"), device=dev)
+    for st in (binding.BWD_PREPARE, binding.BWD_TILES, binding.BWD_FINALIZE):
+        binding.bwd(qd, kd, vd, y, dod, lz, LAM, kernel="tcgen05", workspace=ws, dq=outs[0],
+                    dk=outs[1], dv=outs[2], dlambda=dl, stages=st)
+    again = binding.bwd(qd, kd, vd, y, dod, lz, LAM, kernel="tcgen05", workspace=ws)
+    torch.cuda.synchronize()
+    for got in ((*outs, dl), again):
+        assert torch.equal(got[1], one[1]) and torch.equal(got[2], one[2])
+        assert torch.equal(got[3], one[3])
+        assert not torch.isnan(got[0]).any()
+        pu.check("dQ staged", got[0].float().cpu().numpy(), one[0].float().cpu().numpy(),
+                 "bf16", "grad")
+
+
 def test_large_lambda_keeps_self():
     """lambda >> 0 suppresses Exchange (-lambda log i): Y = V on rows i >= 2 up to bf16."""
     w = workloads.custom(1, 2, 300, 64, "bf16")
