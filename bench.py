@@ -211,21 +211,21 @@ def _draw_sample(w, n_heads, t_rows):
     return [t[sl].double().numpy() for t in (q, k, v, do)], len(bs) * len(hs)
 
 
-def cpu_oracle_run(w, n_heads=None, t_rows=None, min_seconds=0.0, max_reps=20):
+def cpu_oracle_run(w, n_heads=None, t_rows=None, min_seconds=0.0, max_reps=20, nthreads=0):
     """Time the fp64 oracle (forward + backward) on a sample of the workload (the first
     n_heads heads over their first t_rows rows), repeating the sample until min_seconds
-    of CPU work have run."""
+    of CPU work have run; nthreads = 0: every OpenMP thread."""
     import oracle
     plan_heads, plan_rows = _sample_plan(w)
     n_heads = n_heads or plan_heads
     t_rows = t_rows or plan_rows
     (q, k, v, do), used = _oracle_sample(w, n_heads, t_rows)
-    threads = oracle.max_threads()
+    threads = nthreads or oracle.max_threads()
     reps, dt = 0, 0.0
     while reps < max_reps and (reps == 0 or dt < min_seconds):
         t0 = time.perf_counter()
-        oracle.mhr_fwd(q, k, v, workloads.LAMBDA_INIT)
-        oracle.mhr_bwd(q, k, v, do, workloads.LAMBDA_INIT)
+        oracle.mhr_fwd(q, k, v, workloads.LAMBDA_INIT, nthreads=nthreads)
+        oracle.mhr_bwd(q, k, v, do, workloads.LAMBDA_INIT, nthreads=nthreads)
         dt += time.perf_counter() - t0
         reps += 1
     flops = 7.0 * used * t_rows * t_rows * w.d * reps
@@ -841,10 +841,16 @@ def run_ours(args, w):
             line["context_sdpa"] = {"not_measured": f"{type(exc).__name__}: {exc}"[:200]}
     if rank == 0 and not args.no_cpu_baseline and ws == 1:
         cb = cpu_oracle_run(w, min_seconds=10.0)
+        # the same oracle on one thread, over a sample one head wide per thread of the above
+        c1 = cpu_oracle_run(w, n_heads=max(1, cb["heads"] // max(1, cb["cores"])),
+                            t_rows=cb["rows"], min_seconds=3.0, nthreads=1)
         line["cpu_baseline"] = {
             "value": cb["tflops"], "unit": "TFLOP/s", "cores": cb["cores"], "kind": "oracle",
             "sample": f"{_sample_text(w, cb)} x {cb['reps']}, fwd+bwd, fp64 C oracle "
-                      f"(OpenMP over heads), {cb['seconds']:.1f} s"}
+                      f"(OpenMP over heads), {cb['seconds']:.1f} s",
+            "single_thread": {"value": c1["tflops"], "unit": "TFLOP/s", "cores": 1,
+                              "sample": f"{_sample_text(w, c1)} x {c1['reps']}, "
+                                        f"{c1['seconds']:.1f} s"}}
     if rank == 0:
         print(json.dumps(line), flush=True)
     if dist is not None:
