@@ -89,3 +89,14 @@ def test_sdpa_context_runs_on_cpu():
     r = bench.sdpa_context(w, torch.device("cpu"), steps=2, warmup=1)
     assert r["ms_per_step"] > 0 and r["tflops"] > 0
     assert "context only" in r["note"]
+
+
+def test_oracle_timing_on_one_thread():
+    """The single-thread leg of the CPU baseline: the oracle with nthreads = 1 over a
+    sample one head wide, reported with cores = 1."""
+    from paper_2608_20172_gb300 import workloads
+    w = workloads.WORKLOADS["tiny"]
+    one = bench.cpu_oracle_run(w, n_heads=1, t_rows=64, nthreads=1)
+    assert one["cores"] == 1 and one["heads"] == 1 and one["rows"] == 64
+    assert one["tflops"] > 0 and one["reps"] >= 1
+    assert bench._sample_text(w, one) == "1 of 2 heads over their first 64 of 128 rows"
