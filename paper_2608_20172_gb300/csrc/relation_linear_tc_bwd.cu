@@ -77,7 +77,20 @@ __device__ __forceinline__ void qm_km(float x, float y, float s1, float s2, floa
   km = __bfloat162float(__float2bfloat16_rn(y * s2 * ex2_approx(-dm)));
 }
 
-enum : int { B_LOAD = 0, B_OPS, B_S, B_A, B_DA, B_DAS, B_MM, B_RELOAD, NBAR };
+// Retention below this takes dalpha from the state and its adjoint at the token (phase F).
+constexpr float kSmallAlpha = 1.0f / 1024.0f;
+
+// The small-retention fix-up's tiles (dY, p1, p2 loaded again), over the epilogue's dL and
+// Km Ys arrays once phase F has read them
+constexpr int OFF_FIX_G = OFF_KL, OFF_FIX_P1 = OFF_KL + T16, OFF_FIX_P2 = OFF_KL + 2 * T16;
+static_assert(OFF_FIX_P2 + T16 <= OFF_C0 && OFF_KL % 1024 == 0, "fix-up tiles");
+
+enum : int { B_LOAD = 0, B_OPS, B_S, B_A, B_DA, B_DAS, B_MM, B_RELOAD, B_FIX, NBAR };
+
+// Some lane of the warp has a token flagged in its 64-bit mask.
+__device__ __forceinline__ bool small_any_warp(unsigned long long m) {
+  return __any_sync(0xffffffffu, m != 0ull);
+}
 
 __global__ void __launch_bounds__(kThreads, 1)
     lin_tc_bwd_kernel(const __grid_constant__ CUtensorMap tmP1,
@@ -98,6 +111,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(smem + OFF_BAR + 96);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(smem + OFF_BAR + 104);
   int* clamped = reinterpret_cast<int*>(smem + OFF_BAR + 108);
+  volatile int* fix_any = reinterpret_cast<volatile int*>(smem + OFF_BAR + 112);
   float* sc = reinterpret_cast<float*>(smem + OFF_SC);
   float* sq = sc;                 // S_t / |p1_t|
   float* sk = sc + LT;            // S_t / |p2_t|
@@ -120,6 +134,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       mbar_init(bar(i), (i == B_OPS || i == B_A || i == B_DAS) ? 128 : 1);
     *abort_flag = 0;
     *clamped = 0;
+    *fix_any = 0;
     fence_mbar_init();
   }
   if (warp == 5) tmem_alloc(smem_u32(tmem_slot), kTmemCols);
@@ -541,6 +556,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                     (half == 0 ? half_sum[128 + c] : 0.f);
         const float* arow = p.alpha + (long long)b * p.sB + (long long)h * p.sH + c;
         float* drow = p.dalpha + (long long)b * p.sB + (long long)h * p.sH + c;
+        unsigned long long small = 0ull;  // tokens of the half with alpha < kSmallAlpha
         for (int i0 = 48; i0 >= 0; i0 -= 16) {  // 16 tokens: loads first, then the suffix
           float a16[16], g16[16];
 #pragma unroll
@@ -554,6 +570,116 @@ __global__ void __launch_bounds__(kThreads, 1)
             const int tok = half * 64 + i0 + u;
             run += g16[u];
             if (t0 + tok < p.T) drow[(long long)(t0 + tok) * p.sT] = run / a16[u];
+            if (a16[u] < kSmallAlpha) small |= 1ull << (i0 + u);
+          }
+        }
+        // A small alpha_u (below 2^-10) leaves the suffix sum above a small remainder of
+        // terms that cancel, whose fp32 rounding the division magnifies.  There dalpha comes
+        // from the state entering u and the adjoint of Diag(alpha_u) C_{u-1}, channel c (row
+        // c), at the midpoint scale:
+        //   P_u = 2^{L_m} C_0 + sum_{j < u} Km_j I~_j,   Q_u = 2^{L_end - L_m} dC + sum_{t >= u} Qm_t dY_t,
+        //   dalpha_u = <P_u, Q_u> / alpha_u,
+        // where every term of P_u (u in the first half) or of Q_u (the second) carries the
+        // factor alpha_u, so nothing large cancels.  A block with such tokens loads dY, p1
+        // and p2 again (their tiles now hold the outputs) over the dL arrays, which every
+        // elementwise warp has read by then; one warp per (u, c), Km and Qm in fp32.
+        const bool warp_small = small_any_warp(small);  // every lane takes part in the vote
+        if (lane == 0 && warp_small) *fix_any = 1;
+        ew_sync();
+        if (*fix_any) {
+          if (threadIdx.x == 0) {
+            fence_async_smem();  // the dL arrays' generic accesses precede the copies
+            mbar_arrive_expect_tx(bar(B_FIX), 3 * T16);
+            tma_load_4d(sb + OFF_FIX_G, &tmG, bar(B_FIX), 0, t0, h, b);
+            tma_load_4d(sb + OFF_FIX_P1, &tmP1, bar(B_FIX), 0, t0, h, b);
+            tma_load_4d(sb + OFF_FIX_P2, &tmP2, bar(B_FIX), 0, t0, h, b);
+          }
+          if (!(ok = __all_sync(0xffffffffu, mbar_wait(bar(B_FIX), 0, ab)))) break;
+          const uint8_t* vt = smem + OFF_V;
+          const uint8_t* gt = smem + OFF_FIX_G;
+          const uint8_t* p1t = smem + OFF_FIX_P1;
+          const uint8_t* p2t = smem + OFF_FIX_P2;
+          const uint8_t* c0t = smem + OFF_C0;
+          const uint8_t* dct = smem + OFF_DCP;
+          const int t_live = min(LT, p.T - t0);
+          bool unused_clamp = false;
+          // lanes: token group g4 (tokens = g4 mod 4) and the 8 columns from nc (16-byte
+          // group lane & 7 of a 128-byte swizzled row)
+          const int g4 = lane >> 3;
+          auto row16 = [&](const uint8_t* tile, int r) {
+            return *reinterpret_cast<const uint4*>(
+                tile + r * 128 + ((((uint32_t)lane & 7) ^ ((uint32_t)r & 7)) << 4));
+          };
+          auto elem = [&](const uint8_t* tile, int r, int col) {
+            return __bfloat162float(*reinterpret_cast<const __nv_bfloat16*>(
+                tile + r * 128 + ((((uint32_t)col >> 3) ^ ((uint32_t)r & 7)) << 4) + (col & 7) * 2));
+          };
+          for (int i = 0; i < 64 && warp_small; ++i) {
+            unsigned fl = __ballot_sync(0xffffffffu, ((small >> i) & 1ull) != 0ull);
+            while (fl) {
+              const int src = __ffs(fl) - 1;
+              fl &= fl - 1;
+              const int cc = (warp & 1) * 32 + src;  // that lane's channel
+              const int u = half * 64 + i;
+              const float lmc = lmid_s[cc];
+              // Km of the tokens before u and Qm of those from u on, channel cc: lane l
+              // holds tokens l + 32 k
+              float kmr[4], qmr[4];
+#pragma unroll
+              for (int k = 0; k < 4; ++k) {
+                const int tok = lane + 32 * k;
+                const float dm = dm_of(al_at(tok, cc), lmc, tok >= 64, unused_clamp);
+                const float x2 = tok < u ? elem(p2t, tok, cc) : 0.f;
+                const float x1 = (tok >= u && tok < t_live) ? elem(p1t, tok, cc) : 0.f;
+                kmr[k] = x2 * sk[tok] * ex2_approx(-dm);
+                qmr[k] = x1 * sq[tok] * ex2_approx(dm);
+              }
+              float P[8], Q[8];
+#pragma unroll
+              for (int e = 0; e < 8; ++e) P[e] = Q[e] = 0.f;
+#pragma unroll 4
+              for (int j0 = 0; j0 < LT; j0 += 4) {  // tokens j0 + g4
+                const int j = j0 + g4, kq = j0 >> 5;
+                const float ksel = kq == 0 ? kmr[0] : kq == 1 ? kmr[1] : kq == 2 ? kmr[2] : kmr[3];
+                const float qsel = kq == 0 ? qmr[0] : kq == 1 ? qmr[1] : kq == 2 ? qmr[2] : qmr[3];
+                const float km = __shfl_sync(0xffffffffu, ksel, (j0 & 31) + g4);
+                const float qm = __shfl_sync(0xffffffffu, qsel, (j0 & 31) + g4);
+                const uint4 v4 = row16(vt, j), d4 = row16(gt, j);
+                const uint32_t vw[4] = {v4.x, v4.y, v4.z, v4.w}, dw[4] = {d4.x, d4.y, d4.z, d4.w};
+#pragma unroll
+                for (int e = 0; e < 4; ++e) {
+                  const float2 fv = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&vw[e]));
+                  const float2 fd = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&dw[e]));
+                  P[2 * e] = fmaf(km, fv.x, P[2 * e]);
+                  P[2 * e + 1] = fmaf(km, fv.y, P[2 * e + 1]);
+                  Q[2 * e] = fmaf(qm, fd.x, Q[2 * e]);
+                  Q[2 * e + 1] = fmaf(qm, fd.y, Q[2 * e + 1]);
+                }
+              }
+              // the four token groups' sums, the block-boundary rows, and <P_u, Q_u>
+              const uint4 c4 = row16(c0t, cc), e4 = row16(dct, cc);
+              const uint32_t cw[4] = {c4.x, c4.y, c4.z, c4.w}, ew[4] = {e4.x, e4.y, e4.z, e4.w};
+              float pq = 0.f;
+#pragma unroll
+              for (int e = 0; e < 4; ++e) {
+                const float2 cf = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&cw[e]));
+                const float2 ef = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&ew[e]));
+#pragma unroll
+                for (int h2 = 0; h2 < 2; ++h2) {
+                  float pe = P[2 * e + h2], qe = Q[2 * e + h2];
+                  pe += __shfl_xor_sync(0xffffffffu, pe, 8);
+                  pe += __shfl_xor_sync(0xffffffffu, pe, 16);
+                  qe += __shfl_xor_sync(0xffffffffu, qe, 8);
+                  qe += __shfl_xor_sync(0xffffffffu, qe, 16);
+                  pq = fmaf(pe + (h2 ? cf.y : cf.x), qe + (h2 ? ef.y : ef.x), pq);
+                }
+              }
+              pq += __shfl_xor_sync(0xffffffffu, pq, 1);
+              pq += __shfl_xor_sync(0xffffffffu, pq, 2);
+              pq += __shfl_xor_sync(0xffffffffu, pq, 4);
+              if (lane == src)
+                drow[(long long)(t0 + u) * p.sT] = pq / __ldg(arow + (long long)(t0 + u) * p.sT);
+            }
           }
         }
       }
@@ -563,6 +689,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   }
 
   if (warp == 5) drain_wait(bar(B_MM), 0);  // no product in flight past the teardown
+  if (threadIdx.x == 0 && *fix_any) drain_wait(bar(B_FIX), 0);  // nor the fix-up's copies
   tc_fence_before();
   __syncthreads();
   if (threadIdx.x == 0 && *clamped && p.dev_status && !*abort_flag)

@@ -288,3 +288,28 @@ def test_linear_backward_chunked_bhtd_layout_and_stride_fallback():
     torch.cuda.synchronize()
     assert int(status.item()) == 0
     _check_grads("linear bwd strided", g, p1, p2, v, alpha, dy, [(0, 0), (1, 2)])
+
+
+def test_linear_chunked_at_the_longest_sweep_point():
+    """The long-context sweep's last point as the benchmark runs it (B = 1, H = 12,
+    T = 32768, d_h = 64, 256 blocks of 128 tokens): the chunk-parallel forward (workspace
+    entry point), the sequential chunked forward and the chunked backward, each against the
+    fp64 oracle on three heads over the whole sequence."""
+    w = workloads.custom(1, 12, 32768, 64, "bf16")
+    p1, p2, v, alpha, dy = workloads.make_linear_inputs(w, seed=1)
+    dev = torch.device("cuda:0")
+    args = [t.to(dev) for t in (p1, p2, v, alpha)]
+    status = torch.zeros(1, dtype=torch.int32, device=dev)
+    y_ws = binding.linear_fwd_ws(*args, dev_status=status)
+    y_seq = binding.linear_fwd(*args, kernel="tcgen05", dev_status=status)
+    g = binding.linear_bwd(*args, dy.to(dev), kernel="tcgen05", dev_status=status)
+    torch.cuda.synchronize()
+    assert int(status.item()) == 0
+    y_ws, y_seq = y_ws.float().cpu().numpy(), y_seq.float().cpu().numpy()
+    heads = [(0, 0), (0, 5), (0, 11)]
+    for b, h in heads:
+        ref, _ = oracle.linear_fwd(_heads(p1, b, h), _heads(p2, b, h), _heads(v, b, h),
+                                   _heads(alpha, b, h))
+        pu.check_recorded("linear 32768", "Y chunk-parallel", y_ws[b, :, h], ref, "bf16", "out")
+        pu.check_recorded("linear 32768", "Y sequential", y_seq[b, :, h], ref, "bf16", "out")
+    _check_grads("linear 32768 bwd", g, p1, p2, v, alpha, dy, heads)
