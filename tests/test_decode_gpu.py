@@ -68,3 +68,32 @@ def test_decode_bad_length_reported():
     binding.decode(q, k, k, lens, LAM, dev_status=status)
     torch.cuda.synchronize()
     assert int(status.item()) == binding.ERR_INVALID_ARG
+
+
+def test_decode_at_the_benchmark_cache_size():
+    """The benchmark's decode geometry (B = 32 sequences, H = 16, a T = 8192 cache, d_h = 128,
+    2.1 GB of bf16 K and V): full-length sequences as the benchmark runs them and a few
+    ragged ones, the new token's Y and logZ on sampled (b, h) against the oracle's row."""
+    B, H, T, d = 32, 16, 8192, 128
+    g = torch.Generator().manual_seed(11)
+    kc = torch.randn((B, T, H, d), generator=g).to(torch.bfloat16)
+    vc = torch.randn((B, T, H, d), generator=g).to(torch.bfloat16)
+    qn = torch.randn((B, H, d), generator=g).to(torch.bfloat16)
+    lengths = [T] * B
+    lengths[1], lengths[2], lengths[3] = 1, 4097, T - 1
+    dev = torch.device("cuda:0")
+    lens = torch.tensor(lengths, dtype=torch.int32, device=dev)
+    status = torch.zeros(1, dtype=torch.int32, device=dev)
+    y, lz = binding.decode(qn.to(dev), kc.to(dev), vc.to(dev), lens, LAM, dev_status=status)
+    torch.cuda.synchronize()
+    assert int(status.item()) == 0
+    y, lz = y.float().cpu().numpy(), lz.cpu().numpy()
+    for b in (0, 1, 2, 3, 31):
+        n = lengths[b]
+        for h in (0, 9, 15):
+            qs = np.zeros((n, d))
+            qs[n - 1] = qn[b, h].double().numpy()
+            yr, lr = oracle.fwd_rows(qs, kc[b, :n, h].double().numpy(),
+                                     vc[b, :n, h].double().numpy(), [n - 1], LAM)
+            pu.check_recorded("decode 8192", "Y", y[b, h][None], yr, "bf16", "out")
+            pu.check_logz(f"logZ decode b{b} h{h}", lz[b, h][None], lr, "bf16")

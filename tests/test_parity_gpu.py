@@ -174,6 +174,27 @@ def test_long_context_full_size():
     pu.check_recorded("long head", "dV", res["dV"][b, :, h].numpy(), dv, "bf16", "grad")
 
 
+@pytest.mark.parametrize("B,H,T,d", [(32, 8, 1024, 48), (4, 8, 4096, 80)])
+def test_paper_layer_geometries_full_size(B, H, T, d):
+    """The paper's layer geometries the benchmark times with head widths that run on
+    zero-padded tiles (d_h = 48 on 64-wide, 80 on 128-wide), at full size: every row of two
+    heads (forward) and one whole head's gradients, against the oracle."""
+    w = workloads.custom(B, H, T, d, "bf16")
+    q, k, v, do = workloads.make_inputs(w, seed=d)
+    res = pu.gpu_run(q, k, v, do, LAM)
+    rows = list(range(T))
+    for (b, h) in [(0, 0), (B - 1, H - 1)]:
+        y, lz = oracle.fwd_rows(pu.head(q, b, h), pu.head(k, b, h), pu.head(v, b, h), rows, LAM)
+        pu.check_recorded(f"paper layer d={d}", "Y", res["Y"][b, :, h].numpy(), y, "bf16", "out")
+        pu.check_logz(f"logZ [{b},{h}] d={d}", res["logZ"][b, h].numpy(), lz, "bf16")
+    b, h = B // 2, H // 2
+    dq, dk, dv, _ = oracle.bwd_tail(pu.head(q, b, h), pu.head(k, b, h), pu.head(v, b, h),
+                                    pu.head(do, b, h), LAM, 0)
+    pu.check_recorded(f"paper layer d={d}", "dQ", res["dQ"][b, :, h].numpy(), dq, "bf16", "grad")
+    pu.check_recorded(f"paper layer d={d}", "dK", res["dK"][b, :, h].numpy(), dk, "bf16", "grad")
+    pu.check_recorded(f"paper layer d={d}", "dV", res["dV"][b, :, h].numpy(), dv, "bf16", "grad")
+
+
 def test_long_context_prefix_gradient():
     """dO = 0 on rows >= T' makes every gradient equal to that of the T'-prefix problem
     (rows i >= T' then carry dR_i. = 0): the full-size launch is checked exactly on the
